@@ -1,0 +1,265 @@
+"""CPU oracle for the LittleBit linear forward (arXiv 2506.13771).
+
+TEST INFRASTRUCTURE ONLY.  This package is the independent fp64 reference the
+CUDA path is checked against.  Only ``tests/``, ``__graft_entry__.smoke()`` and
+the ``cpu_baseline`` / ``--impl reference`` leg of ``bench.py`` may import it;
+the product package never does, and this package never imports the product.
+
+The arithmetic lives in ``lb_oracle.c`` (plain C, fp64, one function per
+definition of the paper: Eq. 2 packing, Eq. 4-6 dense weight, Prop. 1 factored
+forward, App. E bit accounting).  This module only builds it with gcc and
+marshals numpy arrays through ctypes.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "lb_oracle.c")
+_HDR = os.path.join(_HERE, "lb_oracle.h")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD, "liblboracle.so")
+
+_lib = None
+_lock = threading.Lock()
+
+
+def build(force: bool = False) -> str:
+    """Compile lb_oracle.c into _build/liblboracle.so with gcc (+OpenMP)."""
+    os.makedirs(_BUILD, exist_ok=True)
+    newest_src = max(os.path.getmtime(_SRC), os.path.getmtime(_HDR))
+    if (not force and os.path.exists(_LIB_PATH)
+            and os.path.getmtime(_LIB_PATH) >= newest_src):
+        return _LIB_PATH
+    tmp = _LIB_PATH + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-std=c11", "-O2", "-fPIC", "-shared", "-fopenmp",
+           "-ffp-contract=off", "-Wall", "-Wextra", "-o", tmp, _SRC, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+class Path(ctypes.Structure):
+    _fields_ = [("r", ctypes.c_int32),
+                ("v_words", ctypes.c_void_p),
+                ("u_words", ctypes.c_void_p),
+                ("g", ctypes.c_void_p),
+                ("l", ctypes.c_void_p),
+                ("h", ctypes.c_void_p)]
+
+
+class Linear(ctypes.Structure):
+    _fields_ = [("d_in", ctypes.c_int32),
+                ("d_out", ctypes.c_int32),
+                ("n_paths", ctypes.c_int32),
+                ("path", Path * 2)]
+
+
+def _bind(lib):
+    d, i64, u16, vp = ctypes.c_double, ctypes.c_int64, ctypes.c_uint16, ctypes.c_void_p
+    lib.lbo_half_to_double.argtypes = [u16]
+    lib.lbo_half_to_double.restype = d
+    lib.lbo_bf16_to_double.argtypes = [u16]
+    lib.lbo_bf16_to_double.restype = d
+    for name in ("lbo_pack_u", "lbo_pack_v"):
+        getattr(lib, name).argtypes = [vp, i64, i64, vp]
+        getattr(lib, name).restype = ctypes.c_int
+    for name in ("lbo_unpack_u", "lbo_unpack_v"):
+        getattr(lib, name).argtypes = [vp, i64, i64, vp]
+        getattr(lib, name).restype = None
+    lib.lbo_forward_dense.argtypes = [ctypes.POINTER(Linear), vp, i64, vp]
+    lib.lbo_forward_dense.restype = ctypes.c_int
+    lib.lbo_forward_factored.argtypes = [ctypes.POINTER(Linear), vp, i64, vp]
+    lib.lbo_forward_factored.restype = ctypes.c_int
+    lib.lbo_apply_factored.argtypes = [ctypes.POINTER(Linear), vp, i64, vp, vp]
+    lib.lbo_apply_factored.restype = ctypes.c_int
+    lib.lbo_stack_forward.argtypes = [ctypes.POINTER(Linear), ctypes.c_int32, vp, vp, vp]
+    lib.lbo_stack_forward.restype = ctypes.c_int
+    lib.lbo_bpw.argtypes = [i64, i64, i64, ctypes.c_int32]
+    lib.lbo_bpw.restype = d
+    lib.lbo_rank_for_bpw.argtypes = [d, i64, i64, ctypes.c_int32]
+    lib.lbo_rank_for_bpw.restype = d
+    lib.lbo_flops.argtypes = [i64, i64, i64, i64, ctypes.c_int32]
+    lib.lbo_flops.restype = d
+    lib.lbo_set_threads.argtypes = [ctypes.c_int32]
+    lib.lbo_set_threads.restype = None
+    lib.lbo_get_threads.argtypes = []
+    lib.lbo_get_threads.restype = ctypes.c_int32
+    return lib
+
+
+def _ptr(a: np.ndarray) -> int:
+    return a.ctypes.data
+
+
+def _c(a, dtype) -> np.ndarray:
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+class _Holder:
+    """Keeps the numpy buffers referenced by a ctypes Linear alive."""
+
+    def __init__(self, layer: dict):
+        self.keep = []
+        self.c = Linear()
+        self.c.d_in = int(layer["d_in"])
+        self.c.d_out = int(layer["d_out"])
+        paths = layer["paths"]
+        self.c.n_paths = len(paths)
+        for p, P in enumerate(paths):
+            arrs = {
+                "v_words": _c(P["v_words"], np.uint32),
+                "u_words": _c(P["u_words"], np.uint32),
+                "g": _c(P["g"], np.uint16),
+                "l": _c(P["l"], np.uint16),
+                "h": _c(P["h"], np.uint16),
+            }
+            self.keep.append(arrs)
+            cp = self.c.path[p]
+            cp.r = int(P["r"])
+            for k, a in arrs.items():
+                setattr(cp, k, _ptr(a))
+
+
+class Oracle:
+    """The oracle functions bound to one compiled copy of lb_oracle.c."""
+
+    def __init__(self, lib_path: str | None = None):
+        self.lib = _bind(ctypes.CDLL(lib_path or build()))
+
+    # ------------------------------------------------------------ formats
+    def half_to_double(self, bits: int) -> float:
+        """IEEE binary16 bit pattern -> value (from the format definition)."""
+        return self.lib.lbo_half_to_double(int(bits))
+
+    def bf16_to_double(self, bits: int) -> float:
+        """bfloat16 bit pattern -> value (from the format definition)."""
+        return self.lib.lbo_bf16_to_double(int(bits))
+
+    # ------------------------------------------------------------ packing (Eq. 2)
+    def pack_u(self, signs: np.ndarray) -> np.ndarray:
+        """U_sign [d_out][r] (+-1 int8) -> words [d_out][ceil(r/32)]."""
+        s = _c(signs, np.int8)
+        rows, cols = s.shape
+        out = np.zeros((rows, (cols + 31) // 32), dtype=np.uint32)
+        if self.lib.lbo_pack_u(_ptr(s), rows, cols, _ptr(out)) != 0:
+            raise ValueError("signs must be +1 or -1")
+        return out
+
+    def pack_v(self, signs: np.ndarray) -> np.ndarray:
+        """V_sign [d_in][r] (+-1 int8) -> words [ceil(d_in/32)][r]."""
+        s = _c(signs, np.int8)
+        rows, cols = s.shape
+        out = np.zeros(((rows + 31) // 32, cols), dtype=np.uint32)
+        if self.lib.lbo_pack_v(_ptr(s), rows, cols, _ptr(out)) != 0:
+            raise ValueError("signs must be +1 or -1")
+        return out
+
+    def unpack_u(self, words: np.ndarray, rows: int, cols: int) -> np.ndarray:
+        w = _c(words, np.uint32)
+        out = np.zeros((rows, cols), dtype=np.int8)
+        self.lib.lbo_unpack_u(_ptr(w), rows, cols, _ptr(out))
+        return out
+
+    def unpack_v(self, words: np.ndarray, rows: int, cols: int) -> np.ndarray:
+        w = _c(words, np.uint32)
+        out = np.zeros((rows, cols), dtype=np.int8)
+        self.lib.lbo_unpack_v(_ptr(w), rows, cols, _ptr(out))
+        return out
+
+    # ------------------------------------------------------------ forward
+    def forward_dense(self, layer: dict, x_bf16: np.ndarray) -> np.ndarray:
+        """Eq. 4-6 then Y = X W^T, fp64.  x_bf16: uint16 bit patterns [T][d_in]."""
+        hold = _Holder(layer)
+        x = _c(x_bf16, np.uint16)
+        y = np.zeros((x.shape[0], layer["d_out"]), dtype=np.float64)
+        if self.lib.lbo_forward_dense(ctypes.byref(hold.c), _ptr(x), x.shape[0], _ptr(y)):
+            raise MemoryError("oracle dense forward failed")
+        return y
+
+    def forward_factored(self, layer: dict, x_bf16: np.ndarray) -> np.ndarray:
+        """Prop. 1 per path, paths summed (Eq. 6), fp64."""
+        hold = _Holder(layer)
+        x = _c(x_bf16, np.uint16)
+        y = np.zeros((x.shape[0], layer["d_out"]), dtype=np.float64)
+        if self.lib.lbo_forward_factored(ctypes.byref(hold.c), _ptr(x), x.shape[0], _ptr(y)):
+            raise MemoryError("oracle factored forward failed")
+        return y
+
+    def apply_factored(self, layer: dict, x: np.ndarray, want_t: bool = False):
+        """Prop. 1 on an fp64 input [T][d_in]; optionally also the stage-1 t_p."""
+        hold = _Holder(layer)
+        X = _c(x, np.float64)
+        T = X.shape[0]
+        y = np.zeros((T, layer["d_out"]), dtype=np.float64)
+        rs = [int(P["r"]) for P in layer["paths"]]
+        t = np.zeros(T * sum(rs), dtype=np.float64) if want_t else None
+        if self.lib.lbo_apply_factored(ctypes.byref(hold.c), _ptr(X), T, _ptr(y),
+                                       _ptr(t) if want_t else None):
+            raise MemoryError("oracle factored forward failed")
+        if not want_t:
+            return y
+        ts, off = [], 0
+        for r in rs:
+            ts.append(t[off:off + T * r].reshape(T, r))
+            off += T * r
+        return y, ts
+
+    def stack_forward(self, layers: list, x0_bf16: np.ndarray, want_kv: bool = True):
+        """Decode chain of n_layers x (q,k,v,o,gate,up,down); returns (out, kv)."""
+        assert len(layers) % 7 == 0
+        n_layers = len(layers) // 7
+        holders = [_Holder(L) for L in layers]
+        arr = (Linear * len(layers))(*[h.c for h in holders])
+        x0 = _c(x0_bf16, np.uint16)
+        out = np.zeros(layers[0]["d_in"], dtype=np.float64)
+        kv = np.zeros((n_layers, 2, layers[1]["d_out"]), dtype=np.float64) if want_kv else None
+        if self.lib.lbo_stack_forward(arr, n_layers, _ptr(x0), _ptr(out),
+                                      _ptr(kv) if want_kv else None):
+            raise MemoryError("oracle stack forward failed")
+        return out, kv
+
+    # ------------------------------------------------------------ accounting (App. E, I.1)
+    def bpw(self, d_out: int, d_in: int, r: int, n_paths: int = 2) -> float:
+        return self.lib.lbo_bpw(d_out, d_in, r, n_paths)
+
+    def rank_for_bpw(self, b: float, d_out: int, d_in: int, n_paths: int = 2) -> float:
+        return self.lib.lbo_rank_for_bpw(b, d_out, d_in, n_paths)
+
+    def flops(self, T: int, d_out: int, d_in: int, r: int, n_paths: int = 2) -> float:
+        return self.lib.lbo_flops(T, d_out, d_in, r, n_paths)
+
+    def set_threads(self, n: int) -> None:
+        self.lib.lbo_set_threads(int(n))
+
+    def get_threads(self) -> int:
+        return int(self.lib.lbo_get_threads())
+
+
+def default() -> Oracle:
+    """The oracle built from the committed lb_oracle.c (built on first use)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            _lib = Oracle()
+        return _lib
+
+
+def _forward(name):
+    def f(*args, **kwargs):
+        return getattr(default(), name)(*args, **kwargs)
+    f.__name__ = name
+    f.__doc__ = getattr(Oracle, name).__doc__
+    return f
+
+
+for _name in ("half_to_double", "bf16_to_double", "pack_u", "pack_v", "unpack_u", "unpack_v",
+              "forward_dense", "forward_factored", "apply_factored", "stack_forward",
+              "bpw", "rank_for_bpw", "flops", "set_threads", "get_threads"):
+    globals()[_name] = _forward(_name)
+del _name

@@ -1,0 +1,407 @@
+"""Pins of the CPU oracle against facts that do not come from the oracle itself.
+
+Each pin takes an ``oracle.Oracle`` and raises AssertionError on a mismatch.
+They are collected by test_oracle_pins.py, and re-run against deliberately
+broken copies of the oracle by test_oracle_mutations.py to show that a
+plausible mistake (dropped term, wrong sign, wrong index, transposed operand)
+fails at least one of them.
+
+Sources of truth used here, none of which is the oracle:
+  * numpy's own float16 / float32 decoders (exhaustive over all 2^16 patterns)
+  * numpy.packbits (an independent bit packer)
+  * closed forms of Prop. 1 / Eq. 4 for special parameter choices (rank 1,
+    all-equal signs, Sylvester-Hadamard factors with unit scales)
+  * a hand-expanded quadruple sum over every sign pattern of a tiny layer
+  * the worked examples of App. E and App. I.1 (tests/golden/)
+  * algebraic invariants: path-swap symmetry of Eq. 6, h_res = 0 reducing to
+    one path, scale invariance of the rms-normalised decode chain
+"""
+from __future__ import annotations
+
+import os
+
+import numpy as np
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+
+# ------------------------------------------------------------------ helpers
+
+
+def np_half(bits) -> np.ndarray:
+    return np.asarray(bits, dtype=np.uint16).view(np.float16).astype(np.float64)
+
+
+def np_bf16(bits) -> np.ndarray:
+    u = np.asarray(bits, dtype=np.uint16).astype(np.uint32) << 16
+    with np.errstate(invalid="ignore"):
+        return u.view(np.float32).astype(np.float64)
+
+
+def half_bits(v) -> np.ndarray:
+    return np.asarray(v, dtype=np.float64).astype(np.float16).view(np.uint16)
+
+
+def bf16_bits_exact(v) -> np.ndarray:
+    """bf16 bits of values that are exactly representable (checked)."""
+    f = np.asarray(v, dtype=np.float32)
+    u = f.view(np.uint32)
+    assert np.all((u & 0xFFFF) == 0), "value not exactly representable in bf16"
+    return (u >> 16).astype(np.uint16)
+
+
+def rel(a, b) -> float:
+    a = np.asarray(a, dtype=np.float64)
+    b = np.asarray(b, dtype=np.float64)
+    den = np.linalg.norm(b)
+    return float(np.linalg.norm(a - b) / (den if den > 0 else 1.0))
+
+
+def layer_from_signs(orc, d_in, d_out, paths):
+    """paths: list of dicts with u_signs, v_signs, g, l, h (fp16 bits)."""
+    out = []
+    for P in paths:
+        out.append({"r": P["u_signs"].shape[1],
+                    "u_words": orc.pack_u(P["u_signs"]),
+                    "v_words": orc.pack_v(P["v_signs"]),
+                    "g": P["g"], "l": P["l"], "h": P["h"]})
+    return {"d_in": d_in, "d_out": d_out, "paths": out}
+
+
+def rand_path(rng, d_in, d_out, r, c=0.3):
+    return {"u_signs": (1 - 2 * rng.integers(0, 2, (d_out, r))).astype(np.int8),
+            "v_signs": (1 - 2 * rng.integers(0, 2, (d_in, r))).astype(np.int8),
+            "g": half_bits(np.abs(rng.standard_normal(d_in)) * c + 0.05),
+            "l": half_bits(np.abs(rng.standard_normal(r)) * c + 0.05),
+            "h": half_bits(np.abs(rng.standard_normal(d_out)) * c + 0.05)}
+
+
+def rand_x(rng, T, d_in):
+    f = rng.standard_normal((T, d_in)).astype(np.float32)
+    u = f.view(np.uint32).astype(np.uint64)
+    return ((u + 0x7FFF + ((u >> 16) & 1)) >> 16).astype(np.uint16)
+
+
+def sylvester(n: int) -> np.ndarray:
+    H = np.ones((1, 1), dtype=np.int8)
+    while H.shape[0] < n:
+        H = np.block([[H, H], [H, -H]]).astype(np.int8)
+    return H
+
+
+def fwht(v: np.ndarray) -> np.ndarray:
+    """Textbook in-place fast Walsh-Hadamard transform (Sylvester order)."""
+    a = np.array(v, dtype=np.float64)
+    h = 1
+    n = a.shape[-1]
+    while h < n:
+        for i in range(0, n, 2 * h):
+            x = a[..., i:i + h].copy()
+            y = a[..., i + h:i + 2 * h].copy()
+            a[..., i:i + h] = x + y
+            a[..., i + h:i + 2 * h] = x - y
+        h *= 2
+    return a
+
+
+# ------------------------------------------------------------------ pins: formats
+
+
+def pin_fp16_exhaustive(orc):
+    bits = np.arange(65536, dtype=np.uint32)
+    ref = np_half(bits.astype(np.uint16))
+    got = np.array([orc.half_to_double(int(b)) for b in bits])
+    nan = np.isnan(ref)
+    assert np.array_equal(np.isnan(got), nan)
+    assert np.array_equal(got[~nan], ref[~nan])
+
+
+def pin_bf16_exhaustive(orc):
+    bits = np.arange(65536, dtype=np.uint32)
+    ref = np_bf16(bits.astype(np.uint16))
+    got = np.array([orc.bf16_to_double(int(b)) for b in bits])
+    nan = np.isnan(ref)
+    assert np.array_equal(np.isnan(got), nan)
+    assert np.array_equal(got[~nan], ref[~nan])
+
+
+# ------------------------------------------------------------------ pins: packing (Eq. 2)
+
+
+def pin_pack_structured(orc):
+    ones = np.ones((3, 64), np.int8)
+    assert np.all(orc.pack_u(ones) == 0)
+    assert np.all(orc.pack_u(-ones) == 0xFFFFFFFF)
+    alt = np.tile(np.array([1, -1], np.int8), (3, 32))
+    assert np.all(orc.pack_u(alt) == 0xAAAAAAAA)
+    # rank 16: half a word, padding bits zero
+    assert np.all(orc.pack_u(-np.ones((5, 16), np.int8)) == 0x0000FFFF)
+    # V packs along rows
+    assert np.all(orc.pack_v(-np.ones((64, 3), np.int8)) == 0xFFFFFFFF)
+    assert np.all(orc.pack_v(np.tile(np.array([[1], [-1]], np.int8), (32, 3))) == 0xAAAAAAAA)
+    assert np.all(orc.pack_v(-np.ones((40, 2), np.int8))[1] == 0x000000FF)
+    # a lone -1 at element (o, j) sets exactly bit j%32 of word j//32 in row o
+    s = np.ones((4, 70), np.int8)
+    s[2, 37] = -1
+    w = orc.pack_u(s)
+    exp = np.zeros_like(w)
+    exp[2, 1] = 1 << 5
+    assert np.array_equal(w, exp)
+    try:
+        orc.pack_u(np.zeros((2, 8), np.int8))
+    except ValueError:
+        pass
+    else:
+        raise AssertionError("pack accepted a 0 sign")
+
+
+def _np_pack_rows(signs: np.ndarray) -> np.ndarray:
+    """Independent packer: numpy.packbits, little bit order, bytes -> uint32 LE."""
+    rows, cols = signs.shape
+    nw = (cols + 31) // 32
+    bits = np.zeros((rows, nw * 32), np.uint8)
+    bits[:, :cols] = (signs == -1)
+    by = np.packbits(bits, axis=1, bitorder="little")
+    return by.reshape(rows, nw, 4).astype(np.uint32) @ np.array([1, 1 << 8, 1 << 16, 1 << 24],
+                                                                 dtype=np.uint32)
+
+
+def pin_pack_vs_numpy(orc):
+    rng = np.random.default_rng(7)
+    for rows, cols in [(5, 1), (7, 31), (3, 32), (9, 33), (17, 100), (64, 192)]:
+        s = (1 - 2 * rng.integers(0, 2, (rows, cols))).astype(np.int8)
+        wu = orc.pack_u(s)
+        assert np.array_equal(wu, _np_pack_rows(s))
+        wv = orc.pack_v(s)
+        assert np.array_equal(wv, _np_pack_rows(s.T).T)
+        assert np.array_equal(orc.unpack_u(wu, rows, cols), s)
+        assert np.array_equal(orc.unpack_v(wv, rows, cols), s)
+
+
+# ------------------------------------------------------------------ pins: forward
+
+
+def pin_dense_equals_factored(orc):
+    """Prop. 1 is an identity: factored (Prop. 1) == dense (Eq. 4-6)."""
+    rng = np.random.default_rng(11)
+    for (d_in, d_out, rs, T) in [(40, 24, (3, 5), 3), (70, 33, (33, 1), 2), (64, 64, (16, 16), 4),
+                                 (96, 17, (40,), 1)]:
+        L = layer_from_signs(orc, d_in, d_out, [rand_path(rng, d_in, d_out, r) for r in rs])
+        x = rand_x(rng, T, d_in)
+        yd = orc.forward_dense(L, x)
+        yf = orc.forward_factored(L, x)
+        assert rel(yf, yd) <= 1e-12, rel(yf, yd)
+
+
+def pin_rank1_closed_form(orc):
+    """r = 1: W = h u l v^T g, so Y[t][o] = h_o u_o l * sum_i v_i g_i X[t][i]."""
+    rng = np.random.default_rng(12)
+    d_in, d_out, T = 77, 45, 3
+    P = rand_path(rng, d_in, d_out, 1)
+    L = layer_from_signs(orc, d_in, d_out, [P])
+    x = rand_x(rng, T, d_in)
+    X = np_bf16(x)
+    u = P["u_signs"][:, 0].astype(np.float64)
+    v = P["v_signs"][:, 0].astype(np.float64)
+    s = X @ (v * np_half(P["g"]))
+    ref = np.outer(s, np_half(P["h"]) * u * np_half(P["l"])[0])
+    for y in (orc.forward_factored(L, x), orc.forward_dense(L, x)):
+        assert rel(y, ref) <= 1e-14, rel(y, ref)
+
+
+def pin_all_equal_signs(orc):
+    """All +1 signs: Y[t][o] = h_o (sum_j l_j)(sum_i g_i X[t][i]); U all -1 negates it;
+    U and V both all -1 leaves it unchanged."""
+    rng = np.random.default_rng(13)
+    d_in, d_out, r, T = 50, 20, 9, 2
+    x = rand_x(rng, T, d_in)
+    X = np_bf16(x)
+    for su, sv, sign in [(1, 1, 1.0), (-1, 1, -1.0), (-1, -1, 1.0), (1, -1, -1.0)]:
+        P = rand_path(rng, d_in, d_out, r)
+        P["u_signs"] = np.full((d_out, r), su, np.int8)
+        P["v_signs"] = np.full((d_in, r), sv, np.int8)
+        L = layer_from_signs(orc, d_in, d_out, [P])
+        ref = sign * np.outer(X @ np_half(P["g"]), np_half(P["h"])) * np_half(P["l"]).sum()
+        y = orc.forward_factored(L, x)
+        assert rel(y, ref) <= 1e-14, rel(y, ref)
+
+
+def pin_hadamard_identity(orc):
+    """Unit scales and U = V = H (Sylvester, r = d = 512): W = H H^T = d I, so
+    Y = 512 X exactly.  With r < d, W x = H_r H_r^T x = FWHT(mask_r(FWHT(x)))."""
+    d = 512
+    H = sylvester(d)
+    one = np.full(d, 0x3C00, np.uint16)  # fp16 1.0
+    P = {"u_signs": H, "v_signs": H, "g": one, "l": one, "h": one}
+    L = layer_from_signs(orc, d, d, [P])
+    rng = np.random.default_rng(14)
+    x = rand_x(rng, 3, d)
+    y = orc.forward_factored(L, x)
+    assert np.array_equal(y, 512.0 * np_bf16(x))
+    d, r = 256, 200
+    H = sylvester(d)
+    P = {"u_signs": H[:, :r].copy(), "v_signs": H[:, :r].copy(),
+         "g": np.full(d, 0x3C00, np.uint16), "l": np.full(r, 0x3C00, np.uint16),
+         "h": np.full(d, 0x3C00, np.uint16)}
+    L = layer_from_signs(orc, d, d, [P])
+    x = rand_x(rng, 2, d)
+    c = fwht(np_bf16(x))
+    c[:, r:] = 0.0
+    ref = fwht(c)
+    assert np.array_equal(orc.forward_factored(L, x), ref)
+    assert np.array_equal(orc.forward_dense(L, x), ref)
+
+
+def pin_brute_force(orc):
+    """Every sign pattern of a 2 -> 3 layer of rank 2: the oracle agrees with a
+    hand-expanded sum_j sum_i h_o U[o][j] l_j V[i][j] g_i X[t][i]."""
+    rng = np.random.default_rng(15)
+    d_in, d_out, r, T = 2, 3, 2, 2
+    P = rand_path(rng, d_in, d_out, r)
+    x = rand_x(rng, T, d_in)
+    X = np_bf16(x)
+    g, l, h = np_half(P["g"]), np_half(P["l"]), np_half(P["h"])
+    nbits = d_out * r + d_in * r
+    for pattern in range(1 << nbits):
+        bits = [(pattern >> k) & 1 for k in range(nbits)]
+        U = np.array([1 - 2 * b for b in bits[:d_out * r]], np.int8).reshape(d_out, r)
+        V = np.array([1 - 2 * b for b in bits[d_out * r:]], np.int8).reshape(d_in, r)
+        Q = dict(P, u_signs=U, v_signs=V)
+        L = layer_from_signs(orc, d_in, d_out, [Q])
+        ref = np.zeros((T, d_out))
+        for t in range(T):
+            for o in range(d_out):
+                acc = 0.0
+                for j in range(r):
+                    for i in range(d_in):
+                        acc += h[o] * U[o, j] * l[j] * V[i, j] * g[i] * X[t, i]
+                ref[t, o] = acc
+        yf = orc.forward_factored(L, x)
+        yd = orc.forward_dense(L, x)
+        assert rel(yf, ref) <= 1e-14 and rel(yd, ref) <= 1e-14, pattern
+
+
+def pin_residual_paths(orc):
+    """Eq. 6: swapping the primary and residual paths leaves Y unchanged; a
+    residual path with h_res = 0 reduces Y to the primary path alone."""
+    rng = np.random.default_rng(16)
+    d_in, d_out, T = 48, 40, 3
+    A = rand_path(rng, d_in, d_out, 7)
+    B = rand_path(rng, d_in, d_out, 12)
+    x = rand_x(rng, T, d_in)
+    y_ab = orc.forward_factored(layer_from_signs(orc, d_in, d_out, [A, B]), x)
+    y_ba = orc.forward_factored(layer_from_signs(orc, d_in, d_out, [B, A]), x)
+    assert rel(y_ab, y_ba) <= 1e-15
+    y_a = orc.forward_factored(layer_from_signs(orc, d_in, d_out, [A]), x)
+    y_b = orc.forward_factored(layer_from_signs(orc, d_in, d_out, [B]), x)
+    assert rel(y_ab, y_a + y_b) <= 1e-15
+    assert rel(y_a, y_b) > 0.1
+    Z = dict(B, h=np.zeros(d_out, np.uint16))
+    y_a0 = orc.forward_factored(layer_from_signs(orc, d_in, d_out, [A, Z]), x)
+    assert np.array_equal(y_a0, y_a)
+
+
+def pin_padding_ignored(orc):
+    """Bits beyond r (U words) and beyond d_in (V words) carry no signs."""
+    rng = np.random.default_rng(17)
+    d_in, d_out, r, T = 40, 24, 16, 2
+    P = rand_path(rng, d_in, d_out, r)
+    L = layer_from_signs(orc, d_in, d_out, [P])
+    x = rand_x(rng, T, d_in)
+    y = orc.forward_factored(L, x)
+    Lp = {"d_in": d_in, "d_out": d_out, "paths": [dict(L["paths"][0])]}
+    Lp["paths"][0]["u_words"] = L["paths"][0]["u_words"] | np.uint32(0xFFFF0000)
+    vw = L["paths"][0]["v_words"].copy()
+    vw[-1] |= np.uint32(0xFFFFFF00)
+    Lp["paths"][0]["v_words"] = vw
+    assert np.array_equal(orc.forward_factored(Lp, x), y)
+    assert np.array_equal(orc.forward_dense(Lp, x), orc.forward_dense(L, x))
+
+
+# ------------------------------------------------------------------ pins: accounting
+
+
+def _golden_rows(name):
+    rows = []
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            line = line.strip()
+            if line and not line.startswith("#"):
+                rows.append(line.split())
+    return rows
+
+
+def pin_bpw_worked_examples(orc):
+    for d_out, d_in, b, r, b_at_r in _golden_rows("bpw_worked_examples.txt"):
+        d_out, d_in, b, r = int(d_out), int(d_in), float(b), int(r)
+        r_real = orc.rank_for_bpw(b, d_out, d_in, 2)
+        assert round(r_real) == r, (r_real, r)
+        assert abs(orc.bpw(d_out, d_in, round(r_real), 2) - b) < 0.01
+        if b_at_r != "-":
+            # the paper prints b cut to 4 decimals (0.54987 -> "0.5498")
+            assert 0.0 <= orc.bpw(d_out, d_in, r, 2) - float(b_at_r) < 1e-4
+    # the rank solve inverts the accounting exactly, and one path halves the
+    # sign and scale bits (App. E note on dropping Residual Compensation)
+    for (d_out, d_in, r) in [(512, 512, 16), (8192, 28672, 320), (1024, 8192, 32)]:
+        assert abs(orc.rank_for_bpw(orc.bpw(d_out, d_in, r, 2), d_out, d_in, 2) - r) < 1e-9
+        assert abs(orc.bpw(d_out, d_in, r, 1) * 2 - orc.bpw(d_out, d_in, r, 2)) < 1e-15
+
+
+def pin_theoretical_cost(orc):
+    for T, d_out, d_in, r, mflops in _golden_rows("theoretical_cost.txt"):
+        f = orc.flops(int(T), int(d_out), int(d_in), int(r), 1)
+        assert abs(f / 1e6 - float(mflops)) < 0.05, f
+
+
+# ------------------------------------------------------------------ pins: decode chain
+
+
+def small_stack(rng, n_layers=2, d=64, dkv=32, dff=96, rq=8, rkv=4, rm=12):
+    from paper_2506_13771_gb300 import inputs
+    shapes = inputs.stack_shapes(d, dkv, dff, rq, rkv, rm)
+    layers = []
+    for _ in range(n_layers):
+        for (di, do, r) in shapes:
+            layers.append(inputs.make_linear(rng, di, do, r, 2, 0.3))
+    x0 = inputs.bf16_normal(rng, (d,))
+    return layers, x0
+
+
+def _rho(v):
+    return v / np.sqrt(np.mean(v * v))
+
+
+def pin_stack_chain(orc):
+    """The chain re-built here from single-linear oracle calls and numpy rms."""
+    rng = np.random.default_rng(18)
+    layers, x0 = small_stack(rng)
+    out, kv = orc.stack_forward(layers, x0)
+    a = np_bf16(x0)
+    for l in range(len(layers) // 7):
+        Q, K, V, O, G, Up, D = layers[7 * l:7 * l + 7]
+        an = _rho(a)[None, :]
+        q = orc.apply_factored(Q, an)[0]
+        k = orc.apply_factored(K, an)[0]
+        v = orc.apply_factored(V, an)[0]
+        assert rel(kv[l, 0], k) <= 1e-12 and rel(kv[l, 1], v) <= 1e-12
+        o = orc.apply_factored(O, _rho(q)[None, :])[0]
+        on = _rho(o)[None, :]
+        m = orc.apply_factored(G, on)[0] * orc.apply_factored(Up, on)[0]
+        a = orc.apply_factored(D, _rho(m)[None, :])[0]
+    assert rel(out, a) <= 1e-12, rel(out, a)
+
+
+def pin_stack_scale_invariance(orc):
+    """rho is scale free, so the chain of 2*x0 equals the chain of x0 exactly."""
+    rng = np.random.default_rng(19)
+    layers, x0 = small_stack(rng)
+    out1, kv1 = orc.stack_forward(layers, x0)
+    x2 = bf16_bits_exact(2.0 * np_bf16(x0).astype(np.float32))
+    out2, kv2 = orc.stack_forward(layers, x2)
+    assert np.array_equal(out1, out2) and np.array_equal(kv1, kv2)
+
+
+ALL_PINS = [pin_fp16_exhaustive, pin_bf16_exhaustive, pin_pack_structured, pin_pack_vs_numpy,
+            pin_dense_equals_factored, pin_rank1_closed_form, pin_all_equal_signs,
+            pin_hadamard_identity, pin_brute_force, pin_residual_paths, pin_padding_ignored,
+            pin_bpw_worked_examples, pin_theoretical_cost, pin_stack_chain,
+            pin_stack_scale_invariance]

@@ -1,0 +1,61 @@
+"""Plant plausible mistakes in a copy of the oracle (on the CPU) and check that
+the pins catch every one: a dropped term, a wrong sign, a wrong index, a wrong
+exponent bias, a reversed bit order, a dropped path, a wrong chain step."""
+import os
+import subprocess
+
+import pytest
+
+import oracle
+from tests import oracle_pins
+
+SRC = os.path.join(os.path.dirname(oracle.__file__), "lb_oracle.c")
+
+# (name, text in lb_oracle.c, replacement)
+MUTATIONS = [
+    ("u_sign_polarity", "return ((word >> (j % 32)) & 1u) ? -1 : 1;",
+     "return ((word >> (j % 32)) & 1u) ? 1 : -1;"),
+    ("v_bit_index", "return ((word >> (i % 32)) & 1u) ? -1 : 1;",
+     "return ((word >> (j % 32)) & 1u) ? -1 : 1;"),
+    ("v_word_index", "uint32_t word = words[(i / 32) * r + j];",
+     "uint32_t word = words[(i / 32) * r + (r - 1 - j)];"),
+    ("factored_drops_g", "a[tt * din + i] = X[tt * din + i] * lbo_half_to_double(P->g[i]);",
+     "a[tt * din + i] = X[tt * din + i];"),
+    ("factored_drops_l", "t[tj] *= lbo_half_to_double(P->l[tj % r]);", "t[tj] *= 1.0;"),
+    ("factored_h_index", "y[to] += s * lbo_half_to_double(P->h[o]);",
+     "y[to] += s * lbo_half_to_double(P->h[tt]);"),
+    ("factored_one_path", "    int64_t t_off = 0;\n    for (int p = 0; p < L->n_paths; p++) {",
+     "    int64_t t_off = 0;\n    for (int p = 0; p < 1; p++) {"),
+    ("dense_drops_g", "W[o * din + i] += ho * s * gi;", "W[o * din + i] += ho * s;"),
+    ("half_bias", "v = ldexp((double)(1024 + f), e - 25);", "v = ldexp((double)(1024 + f), e - 24);"),
+    ("half_subnormal", "v = ldexp((double)f, -24);", "v = ldexp((double)f, -25);"),
+    ("bf16_bias", "v = ldexp((double)(128 + f), e - 134);", "v = ldexp((double)(128 + f), e - 133);"),
+    ("pack_bit_order", "word |= (uint32_t)1 << k;\n                else if (v != 1)\n                    return -1;\n            }\n            out[o * nw + w] = word;",
+     "word |= (uint32_t)1 << (31 - k);\n                else if (v != 1)\n                    return -1;\n            }\n            out[o * nw + w] = word;"),
+    ("rms_not_mean", "double inv = 1.0 / sqrt(ss / (double)n);", "double inv = 1.0 / sqrt(ss);"),
+    ("chain_gate_plus_up", "gt[i] *= up[i];", "gt[i] += up[i];"),
+    ("chain_o_from_a", "rms_normalize(q, d, an);", "rms_normalize(a, d, an);"),
+    ("bpw_drops_latent_scale", "+ 16.0 * (double)(d_out + d_in + r);", "+ 16.0 * (double)(d_out + d_in);"),
+    ("rank_solve_one_path", "(n_paths * s + n_paths * 16.0);", "(s + n_paths * 16.0);"),
+    ("flops_factor", "return (double)n_paths * 2.0 * (double)T", "return (double)n_paths * 1.0 * (double)T"),
+]
+
+
+@pytest.mark.parametrize("name,old,new", MUTATIONS, ids=[m[0] for m in MUTATIONS])
+def test_pins_catch_planted_mistake(tmp_path, name, old, new):
+    src = open(SRC).read()
+    assert src.count(old) == 1, f"mutation anchor for {name} not unique"
+    mutated = tmp_path / "lb_oracle.c"
+    mutated.write_text(src.replace(old, new))
+    (tmp_path / "lb_oracle.h").write_text(open(SRC[:-1] + "h").read())
+    so = tmp_path / f"liblboracle_{name}.so"
+    subprocess.run(["gcc", "-std=c11", "-O2", "-fPIC", "-shared", "-fopenmp", "-ffp-contract=off",
+                    "-o", str(so), str(mutated), "-lm"], check=True)
+    bad = oracle.Oracle(str(so))
+    caught = []
+    for pin in oracle_pins.ALL_PINS:
+        try:
+            pin(bad)
+        except (AssertionError, ValueError, MemoryError):
+            caught.append(pin.__name__)
+    assert caught, f"no pin caught the planted mistake {name}"
