@@ -78,7 +78,8 @@ def _bind(lib):
     lib.lbo_forward_factored.restype = ctypes.c_int
     lib.lbo_apply_factored.argtypes = [ctypes.POINTER(Linear), vp, i64, vp, vp]
     lib.lbo_apply_factored.restype = ctypes.c_int
-    lib.lbo_stack_forward.argtypes = [ctypes.POINTER(Linear), ctypes.c_int32, vp, vp, vp]
+    lib.lbo_stack_forward.argtypes = [ctypes.POINTER(Linear), ctypes.c_int32, ctypes.c_int32,
+                                      vp, vp, vp, vp]
     lib.lbo_stack_forward.restype = ctypes.c_int
     lib.lbo_bpw.argtypes = [i64, i64, i64, ctypes.c_int32]
     lib.lbo_bpw.restype = d
@@ -210,19 +211,24 @@ class Oracle:
             off += T * r
         return y, ts
 
-    def stack_forward(self, layers: list, x0_bf16: np.ndarray, want_kv: bool = True):
-        """Decode chain of n_layers x (q,k,v,o,gate,up,down); returns (out, kv)."""
+    def stack_forward(self, layers: list, x0_bf16: np.ndarray, head_dim: int = 128,
+                      want_q: bool = True, want_kv: bool = True):
+        """Decode step at position 0 through n_layers x (q,k,v,o,gate,up,down);
+        returns (out [d], q [n_layers][d] or None, kv [n_layers][2][d_kv] or None)."""
         assert len(layers) % 7 == 0
         n_layers = len(layers) // 7
         holders = [_Holder(L) for L in layers]
         arr = (Linear * len(layers))(*[h.c for h in holders])
         x0 = _c(x0_bf16, np.uint16)
-        out = np.zeros(layers[0]["d_in"], dtype=np.float64)
+        d = layers[0]["d_in"]
+        out = np.zeros(d, dtype=np.float64)
+        q = np.zeros((n_layers, d), dtype=np.float64) if want_q else None
         kv = np.zeros((n_layers, 2, layers[1]["d_out"]), dtype=np.float64) if want_kv else None
-        if self.lib.lbo_stack_forward(arr, n_layers, _ptr(x0), _ptr(out),
+        if self.lib.lbo_stack_forward(arr, n_layers, int(head_dim), _ptr(x0), _ptr(out),
+                                      _ptr(q) if want_q else None,
                                       _ptr(kv) if want_kv else None):
             raise MemoryError("oracle stack forward failed")
-        return out, kv
+        return out, q, kv
 
     # ------------------------------------------------------------ accounting (App. E, I.1)
     def bpw(self, d_out: int, d_in: int, r: int, n_paths: int = 2) -> float:

@@ -266,7 +266,7 @@ int lbo_forward_factored(const lbo_linear *L, const uint16_t *x, int64_t T, doub
 /* Decode chain of the 70B-shaped stack                                     */
 /* ------------------------------------------------------------------------ */
 
-/* rho(v) = v / sqrt(mean(v^2)), written into dst. */
+/* rho(v) = v / sqrt(mean(v^2)) (RMS normalisation with unit weight, eps 0). */
 static void rms_normalize(const double *v, int64_t n, double *dst)
 {
     double ss = 0.0;
@@ -277,60 +277,80 @@ static void rms_normalize(const double *v, int64_t n, double *dst)
         dst[i] = v[i] * inv;
 }
 
-int lbo_stack_forward(const lbo_linear *lin, int32_t n_layers, const uint16_t *x0,
-                      double *out, double *kv_out)
+/* silu(x) = x * sigmoid(x) = x / (1 + e^-x). */
+static double silu(double x) { return x / (1.0 + exp(-x)); }
+
+int lbo_stack_forward(const lbo_linear *lin, int32_t n_layers, int32_t head_dim,
+                      const uint16_t *x0, double *out, double *q_out, double *kv_out)
 {
-    int64_t d = lin[0].d_in;      /* d_model: input of q */
-    int64_t dkv = lin[1].d_out;   /* k width */
-    int64_t dff = lin[4].d_out;   /* gate width */
-    int64_t nmax = dff > d ? dff : d;
+    int64_t d = lin[0].d_in;      /* d_model */
+    int64_t dkv = lin[1].d_out;   /* n_kv_heads * head_dim */
+    int64_t dff = lin[4].d_out;   /* MLP width */
+    int64_t group = d / dkv;      /* query heads per kv head */
     double *a = decode_bf16_array(x0, d);
-    double *an = (double *)malloc((size_t)nmax * sizeof(double));
+    double *n = (double *)malloc((size_t)d * sizeof(double));
     double *q = (double *)malloc((size_t)d * sizeof(double));
-    double *o = (double *)malloc((size_t)d * sizeof(double));
     double *k = (double *)malloc((size_t)dkv * sizeof(double));
     double *v = (double *)malloc((size_t)dkv * sizeof(double));
+    double *attn = (double *)malloc((size_t)d * sizeof(double));
+    double *o = (double *)malloc((size_t)d * sizeof(double));
     double *gt = (double *)malloc((size_t)dff * sizeof(double));
     double *up = (double *)malloc((size_t)dff * sizeof(double));
+    double *dn = (double *)malloc((size_t)d * sizeof(double));
     int rc = -1;
-    if (!a || !an || !q || !o || !k || !v || !gt || !up)
+    if (!a || !n || !q || !k || !v || !attn || !o || !gt || !up || !dn)
         goto done;
     for (int32_t layer = 0; layer < n_layers; layer++) {
         const lbo_linear *Lq = &lin[7 * layer + 0], *Lk = &lin[7 * layer + 1],
                          *Lv = &lin[7 * layer + 2], *Lo = &lin[7 * layer + 3],
                          *Lg = &lin[7 * layer + 4], *Lu = &lin[7 * layer + 5],
                          *Ld = &lin[7 * layer + 6];
-        rms_normalize(a, d, an);
-        if (lbo_apply_factored(Lq, an, 1, q, NULL) || lbo_apply_factored(Lk, an, 1, k, NULL) ||
-            lbo_apply_factored(Lv, an, 1, v, NULL))
+        /* attention block: n = rho(a); q, k, v projections */
+        rms_normalize(a, d, n);
+        if (lbo_apply_factored(Lq, n, 1, q, NULL) || lbo_apply_factored(Lk, n, 1, k, NULL) ||
+            lbo_apply_factored(Lv, n, 1, v, NULL))
             goto done;
+        if (q_out)
+            memcpy(q_out + (int64_t)layer * d, q, (size_t)d * sizeof(double));
         if (kv_out) {
             memcpy(kv_out + (2 * (int64_t)layer + 0) * dkv, k, (size_t)dkv * sizeof(double));
             memcpy(kv_out + (2 * (int64_t)layer + 1) * dkv, v, (size_t)dkv * sizeof(double));
         }
-        rms_normalize(q, d, an);
-        if (lbo_apply_factored(Lo, an, 1, o, NULL))
+        /* attention over a one-position context: the softmax of a single
+         * score is 1, so query head hq reads the value of its kv head
+         * hq / group unchanged */
+        for (int64_t j = 0; j < d; j++) {
+            int64_t hq = j / head_dim, c = j % head_dim;
+            attn[j] = v[(hq / group) * head_dim + c];
+        }
+        if (lbo_apply_factored(Lo, attn, 1, o, NULL))
             goto done;
-        rms_normalize(o, d, an);
-        if (lbo_apply_factored(Lg, an, 1, gt, NULL) || lbo_apply_factored(Lu, an, 1, up, NULL))
+        for (int64_t i = 0; i < d; i++)
+            a[i] += o[i];                       /* h = a + o */
+        /* MLP block: n = rho(h); m = silu(gate(n)) * up(n); a = h + down(m) */
+        rms_normalize(a, d, n);
+        if (lbo_apply_factored(Lg, n, 1, gt, NULL) || lbo_apply_factored(Lu, n, 1, up, NULL))
             goto done;
         for (int64_t i = 0; i < dff; i++)
-            gt[i] *= up[i];
-        rms_normalize(gt, dff, an);
-        if (lbo_apply_factored(Ld, an, 1, a, NULL))
+            gt[i] = silu(gt[i]) * up[i];
+        if (lbo_apply_factored(Ld, gt, 1, dn, NULL))
             goto done;
+        for (int64_t i = 0; i < d; i++)
+            a[i] += dn[i];
     }
     memcpy(out, a, (size_t)d * sizeof(double));
     rc = 0;
 done:
     free(a);
-    free(an);
+    free(n);
     free(q);
-    free(o);
     free(k);
     free(v);
+    free(attn);
+    free(o);
     free(gt);
     free(up);
+    free(dn);
     return rc;
 }
 

@@ -76,14 +76,21 @@ int lbo_forward_factored(const lbo_linear *L, const uint16_t *x, int64_t T, doub
 int lbo_apply_factored(const lbo_linear *L, const double *x, int64_t T, double *y,
                        double *t_out);
 
-/* The 70B-shaped decode chain: n_layers x (q, k, v, o, gate, up, down), seven
- * linears per layer in that order.  With rho(v) = v / sqrt(mean(v^2)):
- *   q = Q(rho(a)); k = K(rho(a)); v = V(rho(a)); o = O(rho(q));
- *   m = G(rho(o)) . Up(rho(o));  a_next = Down(rho(m)).
- * x0: bf16 [d_model]; out: the final a, [d_model]; kv_out: [n_layers][2][d_kv]
- * (k then v of each layer), may be NULL.  Returns 0 or -1. */
-int lbo_stack_forward(const lbo_linear *lin, int32_t n_layers, const uint16_t *x0,
-                      double *out, double *kv_out);
+/* One decode step of a Llama-shaped decoder stack at sequence position 0,
+ * n_layers x (q, k, v, o, gate, up, down), seven linears per layer in that
+ * order, only the linears being LittleBit (the paper's end-to-end setting
+ * keeps attention and norms in FP16, App. I.3).  With rho(v) = v /
+ * sqrt(mean(v^2)) and a = x0:
+ *   n = rho(a); q = Q(n); k = K(n); v = V(n)
+ *   attn = v broadcast over the query heads of each kv head (attention over a
+ *          one-position context: the softmax of one score is 1)
+ *   h = a + O(attn)
+ *   n = rho(h); m = silu(Gate(n)) * Up(n); a = h + Down(m)
+ * head_dim: width of one attention head (d_model and d_kv are multiples).
+ * x0: bf16 [d_model]; out: the final a, [d_model]; q_out: [n_layers][d_model]
+ * and kv_out: [n_layers][2][d_kv] (k then v), each may be NULL.  Returns 0/-1. */
+int lbo_stack_forward(const lbo_linear *lin, int32_t n_layers, int32_t head_dim,
+                      const uint16_t *x0, double *out, double *q_out, double *kv_out);
 
 /* App. E bits per weight: total parameter bits / (d_out * d_in), where each
  * path stores r*(d_out+d_in) sign bits and 16*(d_out+d_in+r) scale bits. */

@@ -144,7 +144,7 @@ def config4(shape: str = "4096x4096_r64", T: int = 2048):
 
 STACK_70B = {
     "d_model": 8192, "d_kv": 1024, "d_ff": 28672, "n_layers": 80,
-    "r_qo": 192, "r_kv": 32, "r_mlp": 320,
+    "r_qo": 192, "r_kv": 32, "r_mlp": 320, "head_dim": 128,
 }
 
 
@@ -155,20 +155,29 @@ def stack_shapes(d_model, d_kv, d_ff, r_qo, r_kv, r_mlp):
             (d_ff, d_model, r_mlp)]
 
 
+def unit_gain_scale(d_in: int, r: int, n_paths: int = 2) -> float:
+    """Scale c of |N(0,1)|*c for h, g and l such that a linear maps an input of
+    rms 1 to an output of rms about 1 (each output is a sum of n_paths*r*d_in
+    sign-weighted products of three scales: rms ~ c^3 sqrt(n_paths r d_in))."""
+    return float((n_paths * r * d_in) ** (-1.0 / 6.0))
+
+
 def make_stack(n_layers: int = 80, d_model: int = 8192, d_kv: int = 1024, d_ff: int = 28672,
-               r_qo: int = 192, r_kv: int = 32, r_mlp: int = 320, scale: float = 0.02,
+               r_qo: int = 192, r_kv: int = 32, r_mlp: int = 320, head_dim: int = 128,
                config_id: int = 5):
     """Llama2-70B-shaped decode stack: n_layers x (q,k,v,o,gate,up,down), two
-    paths each, random sign words.  Returns (list of 7*n_layers linears, x0)."""
+    paths each, random sign words, unit-gain scales.
+    Returns (list of 7*n_layers linears, x0 bf16 bits [d_model])."""
     rng = rng_for(config_id)
     shapes = stack_shapes(d_model, d_kv, d_ff, r_qo, r_kv, r_mlp)
     layers = []
     for _ in range(n_layers):
         for (di, do, r) in shapes:
-            layers.append(make_linear(rng, di, do, r, 2, scale))
+            layers.append(make_linear(rng, di, do, r, 2, unit_gain_scale(di, r, 2)))
     x0 = bf16_normal(rng, (d_model,))
     return layers, x0
 
 
 def config5(n_layers: int = 80):
-    return make_stack(n_layers=n_layers, **{k: v for k, v in STACK_70B.items() if k != "n_layers"})
+    kw = {k: v for k, v in STACK_70B.items() if k not in ("n_layers", "head_dim")}
+    return make_stack(n_layers=n_layers, **kw)

@@ -14,7 +14,9 @@ Sources of truth used here, none of which is the oracle:
   * a hand-expanded quadruple sum over every sign pattern of a tiny layer
   * the worked examples of App. E and App. I.1 (tests/golden/)
   * algebraic invariants: path-swap symmetry of Eq. 6, h_res = 0 reducing to
-    one path, scale invariance of the rms-normalised decode chain
+    one path
+  * for the decoder chain: textbook softmax attention over the one cached
+    position, and closed forms with branches switched off or made the identity
 """
 from __future__ import annotations
 
@@ -355,13 +357,13 @@ def pin_theoretical_cost(orc):
 # ------------------------------------------------------------------ pins: decode chain
 
 
-def small_stack(rng, n_layers=2, d=64, dkv=32, dff=96, rq=8, rkv=4, rm=12):
+def small_stack(rng, n_layers=3, d=64, dkv=16, dff=96, rq=8, rkv=4, rm=12):
     from paper_2506_13771_gb300 import inputs
     shapes = inputs.stack_shapes(d, dkv, dff, rq, rkv, rm)
     layers = []
     for _ in range(n_layers):
         for (di, do, r) in shapes:
-            layers.append(inputs.make_linear(rng, di, do, r, 2, 0.3))
+            layers.append(inputs.make_linear(rng, di, do, r, 2, inputs.unit_gain_scale(di, r)))
     x0 = inputs.bf16_normal(rng, (d,))
     return layers, x0
 
@@ -370,38 +372,92 @@ def _rho(v):
     return v / np.sqrt(np.mean(v * v))
 
 
+def _attention(q, k_cache, v_cache, head_dim):
+    """Textbook grouped-query attention of one query over a cached sequence:
+    per query head, softmax(q_h . k_{g,s} / sqrt(head_dim)) over positions s,
+    then the weighted sum of v_{g,s}; g = the kv head the query head shares."""
+    n_q = q.shape[0] // head_dim
+    n_kv = k_cache.shape[1] // head_dim
+    out = np.zeros_like(q)
+    for hq in range(n_q):
+        g = hq // (n_q // n_kv)
+        qh = q[hq * head_dim:(hq + 1) * head_dim]
+        ks = k_cache[:, g * head_dim:(g + 1) * head_dim]
+        vs = v_cache[:, g * head_dim:(g + 1) * head_dim]
+        s = ks @ qh / np.sqrt(head_dim)
+        w = np.exp(s - s.max())
+        w /= w.sum()
+        out[hq * head_dim:(hq + 1) * head_dim] = w @ vs
+    return out
+
+
 def pin_stack_chain(orc):
-    """The chain re-built here from single-linear oracle calls and numpy rms."""
+    """The decoder chain re-built from single-linear oracle calls, numpy RMS
+    normalisation, SiLU and textbook attention over the one cached position."""
     rng = np.random.default_rng(18)
+    hd = 8
     layers, x0 = small_stack(rng)
-    out, kv = orc.stack_forward(layers, x0)
+    out, qs, kv = orc.stack_forward(layers, x0, head_dim=hd)
     a = np_bf16(x0)
     for l in range(len(layers) // 7):
         Q, K, V, O, G, Up, D = layers[7 * l:7 * l + 7]
-        an = _rho(a)[None, :]
-        q = orc.apply_factored(Q, an)[0]
-        k = orc.apply_factored(K, an)[0]
-        v = orc.apply_factored(V, an)[0]
-        assert rel(kv[l, 0], k) <= 1e-12 and rel(kv[l, 1], v) <= 1e-12
-        o = orc.apply_factored(O, _rho(q)[None, :])[0]
-        on = _rho(o)[None, :]
-        m = orc.apply_factored(G, on)[0] * orc.apply_factored(Up, on)[0]
-        a = orc.apply_factored(D, _rho(m)[None, :])[0]
+        n = _rho(a)[None, :]
+        q = orc.apply_factored(Q, n)[0]
+        k = orc.apply_factored(K, n)[0]
+        v = orc.apply_factored(V, n)[0]
+        assert rel(qs[l], q) <= 1e-12 and rel(kv[l, 0], k) <= 1e-12 and rel(kv[l, 1], v) <= 1e-12
+        attn = _attention(q, k[None, :], v[None, :], hd)
+        h = a + orc.apply_factored(O, attn[None, :])[0]
+        n = _rho(h)[None, :]
+        gt = orc.apply_factored(G, n)[0]
+        m = gt / (1.0 + np.exp(-gt)) * orc.apply_factored(Up, n)[0]
+        a = h + orc.apply_factored(D, m[None, :])[0]
     assert rel(out, a) <= 1e-12, rel(out, a)
 
 
-def pin_stack_scale_invariance(orc):
-    """rho is scale free, so the chain of 2*x0 equals the chain of x0 exactly."""
+def pin_stack_zero_branches(orc):
+    """With h = 0 in every O and Down path no branch reaches the residual
+    stream: the output is x0 exactly, while q, k, v are still produced."""
     rng = np.random.default_rng(19)
     layers, x0 = small_stack(rng)
-    out1, kv1 = orc.stack_forward(layers, x0)
-    x2 = bf16_bits_exact(2.0 * np_bf16(x0).astype(np.float32))
-    out2, kv2 = orc.stack_forward(layers, x2)
-    assert np.array_equal(out1, out2) and np.array_equal(kv1, kv2)
+    for l in range(len(layers) // 7):
+        for idx in (3, 6):
+            for P in layers[7 * l + idx]["paths"]:
+                P["h"] = np.zeros_like(P["h"])
+    out, qs, kv = orc.stack_forward(layers, x0, head_dim=8)
+    assert np.array_equal(out, np_bf16(x0))
+    n = _rho(np_bf16(x0))[None, :]
+    for l in range(len(layers) // 7):
+        assert rel(qs[l], orc.apply_factored(layers[7 * l], n)[0]) <= 1e-12
+        assert rel(kv[l, 1], orc.apply_factored(layers[7 * l + 2], n)[0]) <= 1e-12
+
+
+def pin_stack_attention_closed_form(orc):
+    """Down switched off (h = 0) and O = the unit-scale Sylvester-Hadamard
+    linear (W = d I): every layer adds exactly d * broadcast(v) to the stream."""
+    rng = np.random.default_rng(20)
+    d, dkv, hd = 64, 16, 8
+    layers, x0 = small_stack(rng, d=d, dkv=dkv)
+    H = sylvester(d)
+    one = np.full(d, 0x3C00, np.uint16)
+    for l in range(len(layers) // 7):
+        layers[7 * l + 3] = layer_from_signs(orc, d, d, [{"u_signs": H, "v_signs": H,
+                                                           "g": one, "l": one, "h": one}])
+        for P in layers[7 * l + 6]["paths"]:
+            P["h"] = np.zeros_like(P["h"])
+    out, _, kv = orc.stack_forward(layers, x0, head_dim=hd)
+    a = np_bf16(x0)
+    for l in range(len(layers) // 7):
+        v = orc.apply_factored(layers[7 * l + 2], _rho(a)[None, :])[0]
+        assert rel(kv[l, 1], v) <= 1e-12
+        bcast = np.concatenate([v[(hq // (d // dkv)) * hd:(hq // (d // dkv) + 1) * hd]
+                                for hq in range(d // hd)])
+        a = a + d * bcast
+    assert rel(out, a) <= 1e-13, rel(out, a)
 
 
 ALL_PINS = [pin_fp16_exhaustive, pin_bf16_exhaustive, pin_pack_structured, pin_pack_vs_numpy,
             pin_dense_equals_factored, pin_rank1_closed_form, pin_all_equal_signs,
             pin_hadamard_identity, pin_brute_force, pin_residual_paths, pin_padding_ignored,
             pin_bpw_worked_examples, pin_theoretical_cost, pin_stack_chain,
-            pin_stack_scale_invariance]
+            pin_stack_zero_branches, pin_stack_attention_closed_form]

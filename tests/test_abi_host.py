@@ -1,0 +1,143 @@
+"""Host-side checks of the C ABI (no GPU needed): the library builds, loads and
+exports every entry point include/littlebit.h declares, and argument
+validation answers with status codes before any CUDA call is made."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2506_13771_gb300 import build as lb_build
+from paper_2506_13771_gb300 import littlebit as lb
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include",
+                      "littlebit.h")
+
+
+@pytest.fixture(scope="module")
+def L():
+    lb_build.build()
+    return lb.lib()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(littlebit_\w+)\s*\(", text)))
+
+
+def test_exports_every_declared_symbol(L):
+    names = declared_functions()
+    assert len(names) >= 8
+    for n in names:
+        assert hasattr(L, n), f"{n} declared in littlebit.h but not exported"
+    assert sorted(lb.EXPORTED) == names
+
+
+def test_status_strings(L):
+    for code, name in [(lb.LB_OK, "LB_OK"), (lb.LB_ERR_INVALID_ARG, "LB_ERR_INVALID_ARG"),
+                       (lb.LB_ERR_UNSUPPORTED, "LB_ERR_UNSUPPORTED"), (lb.LB_ERR_CUDA, "LB_ERR_CUDA"),
+                       (lb.LB_ERR_TIMEOUT, "LB_ERR_TIMEOUT"), (lb.LB_ERR_WORKSPACE, "LB_ERR_WORKSPACE")]:
+        assert lb.status_string(code) == name
+    assert lb.status_string(99) == "LB_ERR_UNKNOWN"
+
+
+FAKE = 0x10000000  # a 16-byte aligned address; never dereferenced on these paths
+
+
+def fake_linear(d_in=4096, d_out=4096, rs=(64, 64)):
+    c = lb.lb_linear()
+    c.d_in, c.d_out, c.n_paths = d_in, d_out, len(rs)
+    for p, r in enumerate(rs):
+        c.path[p].r = r
+        for k, f in enumerate(["v_bits", "u_bits", "g", "l", "h"]):
+            setattr(c.path[p], f, FAKE + 0x100000 * (5 * p + k))
+    return c
+
+
+def fwd(L, c, T=1, x=FAKE, y=FAKE, dtype=0, ws=FAKE, ws_bytes=1 << 30):
+    return L.littlebit_linear_forward(ctypes.byref(c) if c is not None else None, x, T, y, dtype,
+                                      ws, ws_bytes, None)
+
+
+def test_workspace_sizes(L):
+    c = fake_linear()
+    n1 = L.littlebit_workspace_size(ctypes.byref(c), 1)
+    n8 = L.littlebit_workspace_size(ctypes.byref(c), 8)
+    assert n1 >= 256 + 4 * 128 and n8 >= 256 + 4 * 8 * 128
+    assert n1 % 256 == 0 and n8 % 256 == 0
+    assert L.littlebit_workspace_size(None, 1) == 0
+    bad = fake_linear(rs=(0, 64))
+    assert L.littlebit_workspace_size(ctypes.byref(bad), 1) == 0
+
+
+def test_forward_argument_validation(L):
+    assert fwd(L, None) == lb.LB_ERR_INVALID_ARG
+    c = fake_linear()
+    assert fwd(L, c, T=-1) == lb.LB_ERR_INVALID_ARG
+    assert fwd(L, c, dtype=7) == lb.LB_ERR_INVALID_ARG
+    assert fwd(L, c, x=0) == lb.LB_ERR_INVALID_ARG
+    assert fwd(L, c, y=FAKE + 4) == lb.LB_ERR_INVALID_ARG          # misaligned output
+    assert fwd(L, c, ws=0) == lb.LB_ERR_WORKSPACE
+    assert fwd(L, c, ws=FAKE + 16) == lb.LB_ERR_WORKSPACE           # ws must be 256-aligned
+    assert fwd(L, c, ws_bytes=64) == lb.LB_ERR_WORKSPACE
+    assert fwd(L, c, T=0) == lb.LB_OK                               # no-op
+    c3 = fake_linear()
+    c3.n_paths = 3
+    assert fwd(L, c3) == lb.LB_ERR_INVALID_ARG
+    cz = fake_linear(d_in=0)
+    assert fwd(L, cz) == lb.LB_ERR_INVALID_ARG
+    cmis = fake_linear()
+    cmis.path[1].g = FAKE + 2
+    assert fwd(L, cmis) == lb.LB_ERR_INVALID_ARG
+    cnull = fake_linear()
+    cnull.path[0].u_bits = None
+    assert fwd(L, cnull) == lb.LB_ERR_INVALID_ARG
+    assert fwd(L, fake_linear(d_in=40)) == lb.LB_ERR_UNSUPPORTED    # d_in % 32
+    assert fwd(L, fake_linear(rs=(2000, 64))) == lb.LB_ERR_UNSUPPORTED
+
+
+def fake_stack(n_layers=2, d=256, dkv=64, dff=512, rq=16, rk=8, rm=24):
+    shapes = [(d, d, rq), (d, dkv, rk), (d, dkv, rk), (d, d, rq), (d, dff, rm), (d, dff, rm),
+              (dff, d, rm)]
+    arr = (lb.lb_linear * (7 * n_layers))()
+    for l in range(n_layers):
+        for i, (di, do, r) in enumerate(shapes):
+            arr[7 * l + i] = fake_linear(di, do, (r, r))
+    return arr
+
+
+def test_stack_argument_validation(L):
+    arr = fake_stack()
+    n = L.littlebit_stack_workspace_size(arr, 2)
+    assert n > 256 and n % 256 == 0
+    st = L.littlebit_stack_forward
+    assert st(arr, 0, FAKE, FAKE, None, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    assert st(arr, 2, 0, FAKE, None, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    assert st(arr, 2, FAKE, FAKE, FAKE + 8, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    assert st(arr, 2, FAKE, FAKE, None, FAKE, n - 256, None) == lb.LB_ERR_WORKSPACE
+    broken = fake_stack()
+    broken[3] = fake_linear(256, 128, (16, 16))                      # o must be d -> d
+    assert L.littlebit_stack_workspace_size(broken, 2) == 0
+    assert st(broken, 2, FAKE, FAKE, None, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    uneven = fake_stack()
+    uneven[7] = fake_linear(256, 256, (32, 16))                      # layer 1 q differs
+    assert st(uneven, 2, FAKE, FAKE, None, FAKE, n, None) == lb.LB_ERR_UNSUPPORTED
+
+
+def test_pack_argument_validation(L):
+    p = L.littlebit_pack
+    assert p(None, 4, 4, lb.LB_PACK_U, FAKE, 4, None, None) == lb.LB_ERR_INVALID_ARG
+    assert p(FAKE, 0, 4, lb.LB_PACK_U, FAKE, 4, None, None) == lb.LB_ERR_INVALID_ARG
+    assert p(FAKE, 4, 4, 5, FAKE, 4, None, None) == lb.LB_ERR_INVALID_ARG
+    assert p(FAKE, 4, 40, lb.LB_PACK_U, FAKE, 7, None, None) == lb.LB_ERR_INVALID_ARG  # needs 8
+    assert p(FAKE, 40, 4, lb.LB_PACK_V, FAKE, 7, None, None) == lb.LB_ERR_INVALID_ARG  # needs 8
+    assert p(FAKE + 1, 4, 4, lb.LB_PACK_U, FAKE, 4, None, None) == lb.LB_ERR_INVALID_ARG
+    assert L.littlebit_poll_error(None, None) == lb.LB_ERR_WORKSPACE
+    assert L.littlebit_selftest_wait_timeout(FAKE + 16, None) == lb.LB_ERR_WORKSPACE
+
+
+def test_product_path_has_no_cpu_fallback(tmp_path):
+    """The binding refuses to run without the compiled library."""
+    with pytest.raises(OSError):
+        lb.lib(str(tmp_path / "liblittlebit.so"))

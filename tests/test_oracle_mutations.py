@@ -33,8 +33,13 @@ MUTATIONS = [
     ("pack_bit_order", "word |= (uint32_t)1 << k;\n                else if (v != 1)\n                    return -1;\n            }\n            out[o * nw + w] = word;",
      "word |= (uint32_t)1 << (31 - k);\n                else if (v != 1)\n                    return -1;\n            }\n            out[o * nw + w] = word;"),
     ("rms_not_mean", "double inv = 1.0 / sqrt(ss / (double)n);", "double inv = 1.0 / sqrt(ss);"),
-    ("chain_gate_plus_up", "gt[i] *= up[i];", "gt[i] += up[i];"),
-    ("chain_o_from_a", "rms_normalize(q, d, an);", "rms_normalize(a, d, an);"),
+    ("chain_no_silu", "gt[i] = silu(gt[i]) * up[i];", "gt[i] = gt[i] * up[i];"),
+    ("chain_gqa_index", "attn[j] = v[(hq / group) * head_dim + c];",
+     "attn[j] = v[(hq % (dkv / head_dim)) * head_dim + c];"),
+    ("chain_no_attn_residual", "a[i] += o[i];                       /* h = a + o */",
+     "a[i] = o[i];"),
+    ("chain_no_mlp_residual", "a[i] += dn[i];", "a[i] = dn[i];"),
+    ("chain_silu_sign", "return x / (1.0 + exp(-x));", "return x / (1.0 + exp(x));"),
     ("bpw_drops_latent_scale", "+ 16.0 * (double)(d_out + d_in + r);", "+ 16.0 * (double)(d_out + d_in);"),
     ("rank_solve_one_path", "(n_paths * s + n_paths * 16.0);", "(s + n_paths * 16.0);"),
     ("flops_factor", "return (double)n_paths * 2.0 * (double)T", "return (double)n_paths * 1.0 * (double)T"),
