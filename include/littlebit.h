@@ -1,0 +1,177 @@
+/*
+ * littlebit.h -- C ABI of the GB300 (sm_103a) LittleBit linear forward.
+ *
+ * LittleBit (arXiv 2506.13771) stores a d_out x d_in weight as one or two
+ * factored, binarised paths (Sec. 3.1, Eq. 1-4; Residual Compensation,
+ * Sec. 3.3, Eq. 5-6):
+ *
+ *     W_p  = diag(h_p) U_p,sign diag(l_p) V_p,sign^T diag(g_p)      (Eq. 4, 5)
+ *     W    = W_pri + W_res                                          (Eq. 6)
+ *
+ * with U_sign in {-1,+1}^{d_out x r}, V_sign in {-1,+1}^{d_in x r} (Eq. 2) and
+ * FP16 scales h in R^{d_out}, g in R^{d_in}, l in R^r (Eq. 3).  The forward
+ * Y = X W^T is computed as Prop. 1 prescribes, per path,
+ *
+ *     Y += ((((X . g) V_sign) . l) U_sign^T) . h
+ *
+ * i.e. a +-1 reduction over d_in (stage 1, rank-r output t), a latent scale,
+ * a +-1 reduction over r (stage 2) and a row scale.
+ *
+ * Conventions shared by every entry point
+ *   - Sign bits: bit = 1 means -1, bit = 0 means +1 (sign(0) = +1).  Bits are
+ *     packed LSB first, 32 per uint32, along the reduction dimension:
+ *       U words  [d_out][ceil(r/32)]    bit k of word (o, w) = U_sign[o][32w+k]
+ *       V words  [ceil(d_in/32)][r]     bit k of word (w, j) = V_sign[32w+k][j]
+ *     Padding bits (beyond r, beyond d_in) are ignored on input.
+ *   - Scales h, g, l are IEEE binary16 bit patterns; activations X are
+ *     bfloat16 bit patterns, row-major [T][d_in]; Y is row-major [T][d_out].
+ *   - All pointers passed to forward calls are DEVICE pointers on the current
+ *     CUDA device and must be 16-byte aligned; the library checks alignment
+ *     and nullness, not that the memory is on the device.
+ *   - The caller owns every buffer.  The library allocates no device memory;
+ *     scratch space is the caller's workspace ("ws"), sized by the
+ *     *_workspace_size functions, 256-byte aligned, and zero-filled once
+ *     before its first use (its first word is the sticky error word below;
+ *     the calls themselves re-initialise everything else they use).
+ *   - Everything is enqueued on the given stream (NULL = legacy default
+ *     stream); no call synchronises except littlebit_poll_error.  Calls are
+ *     safe from several host threads if they use distinct workspaces.
+ *   - Arithmetic: products and sums in fp32 (the paper's kernel uses FP16,
+ *     App. I.2; fp32 accumulation is this library's choice); outputs are
+ *     bf16 (round to nearest even) or fp32.
+ *   - Errors are returned as lb_status; launch failures map to LB_ERR_CUDA.
+ *     Asynchronous device faults surface on a later CUDA call.  A grid-wide
+ *     wait that exceeds its time limit (about one second) makes the kernel
+ *     record LB_ERR_TIMEOUT in the workspace's sticky error word and return;
+ *     while that word is set, kernels using the workspace return at once
+ *     without writing outputs; littlebit_poll_error reads and clears it.
+ */
+#ifndef LITTLEBIT_H
+#define LITTLEBIT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* A CUDA stream (cudaStream_t).  NULL selects the legacy default stream. */
+typedef struct CUstream_st *lb_stream_t;
+
+typedef enum {
+    LB_OK = 0,
+    LB_ERR_INVALID_ARG = 1,  /* null/misaligned pointer, bad size or layout */
+    LB_ERR_UNSUPPORTED = 2,  /* valid but outside what the kernels handle */
+    LB_ERR_CUDA = 3,         /* a CUDA runtime call or launch failed */
+    LB_ERR_TIMEOUT = 4,      /* a device-side grid wait ran out (see poll) */
+    LB_ERR_WORKSPACE = 5,    /* ws is NULL, misaligned or too small */
+    LB_ERR_PLAN = 6          /* stack workspace not prepared for these linears */
+} lb_status;
+
+typedef enum { LB_OUT_BF16 = 0, LB_OUT_FP32 = 1 } lb_out_dtype;
+
+typedef enum {
+    LB_PACK_U = 0,  /* pack a [rows][cols] matrix along cols -> [rows][ceil(cols/32)] */
+    LB_PACK_V = 1   /* pack a [rows][cols] matrix along rows -> [ceil(rows/32)][cols] */
+} lb_pack_layout;
+
+/* One path of Eq. 4 / Eq. 5.  All pointers are device memory. */
+typedef struct {
+    int32_t r;                /* latent rank, 1 <= r <= 1024 */
+    const uint32_t *v_bits;   /* V_sign, [ceil(d_in/32)][r] words */
+    const uint32_t *u_bits;   /* U_sign, [d_out][ceil(r/32)] words */
+    const uint16_t *g;        /* column scale, fp16 [d_in] */
+    const uint16_t *l;        /* latent scale, fp16 [r] */
+    const uint16_t *h;        /* row scale,    fp16 [d_out] */
+} lb_path;
+
+/* One LittleBit linear: n_paths = 2 (primary + residual, Eq. 6) or 1 (the
+ * paper's variant without Residual Compensation, App. E note). */
+typedef struct {
+    int32_t d_in, d_out, n_paths;
+    lb_path path[2];
+} lb_linear;
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char *littlebit_status_string(lb_status s);
+
+/* Eq. 2 binarisation of already-signed factors: packs a row-major int8
+ * [rows][cols] matrix of +1/-1 (DEVICE memory) into sign words (DEVICE) in
+ * the given layout; out_words must be at least the layout's word count.
+ * Padding bits are written 0.  An element other than +1/-1 makes the kernel
+ * set *bad (a DEVICE int32, may be NULL) to 1; the words are then undefined.
+ * *bad is not cleared by the call.  rows, cols >= 1. */
+lb_status littlebit_pack(const int8_t *signs, int64_t rows, int64_t cols, int32_t layout,
+                         uint32_t *out, int64_t out_words, int32_t *bad, lb_stream_t stream);
+
+/* Workspace bytes littlebit_linear_forward needs for this layer and T tokens
+ * (0 if the arguments are invalid). */
+size_t littlebit_workspace_size(const lb_linear *L, int64_t T);
+
+/* Y = X W^T for one LittleBit linear (Prop. 1 per path, paths summed by
+ * Eq. 6).  L is a HOST struct holding device pointers.  x: bf16 [T][d_in];
+ * y: [T][d_out] in y_dtype.  T = 0 is a no-op.  Requires d_in % 32 == 0 and
+ * 1 <= r <= 1024 for every path (else LB_ERR_UNSUPPORTED). */
+lb_status littlebit_linear_forward(const lb_linear *L, const uint16_t *x, int64_t T, void *y,
+                                   int32_t y_dtype, void *ws, size_t ws_bytes,
+                                   lb_stream_t stream);
+
+/* Workspace bytes littlebit_stack_prepare / littlebit_stack_forward need
+ * (0 if the arguments are invalid). */
+size_t littlebit_stack_workspace_size(const lb_linear *lin, int32_t n_layers, int32_t head_dim);
+
+/* Prepares a stack workspace for the linears lin[0 .. 7*n_layers): validates
+ * them (same rules as littlebit_stack_forward), writes their device
+ * descriptor table into ws, zeroes its counters and accumulators and records
+ * a fingerprint of (lin, n_layers, head_dim).  Enqueued on the stream.  Call
+ * it once per workspace, again whenever the linears change, and after any
+ * error a stack launch recorded in the workspace. */
+lb_status littlebit_stack_prepare(const lb_linear *lin, int32_t n_layers, int32_t head_dim,
+                                  void *ws, size_t ws_bytes, lb_stream_t stream);
+
+/* One decode step, at sequence position 0, of n_layers Llama-shaped decoder
+ * blocks whose seven linears are LittleBit linears, lin[7*l + {0..6}] =
+ * q, k, v, o, gate, up, down of layer l.  The paper's end-to-end setting
+ * (App. I.3) replaces only nn.Linear; the rest of the block is computed here
+ * in fp32 with unit RMSNorm weights.  With rho(v) = v / sqrt(mean(v^2)) and
+ * a = x0, each layer computes
+ *     n = rho(a);  q = Q(n);  k = K(n);  v = V(n)
+ *     attn = v broadcast over the query heads of each kv head (attention over
+ *            a one-position context: the softmax of a single score is 1)
+ *     h = a + O(attn)
+ *     n = rho(h);  m = silu(Gate(n)) * Up(n);  a = h + Down(m)
+ * Shapes: q, o d->d; k, v d->d_kv; gate, up d->d_ff; down d_ff->d, with
+ * d = n_heads * head_dim, d_kv = n_kv_heads * head_dim and n_heads a multiple
+ * of n_kv_heads (else LB_ERR_INVALID_ARG); every layer has the same shapes
+ * and ranks, d and d_ff are multiples of 32 (else LB_ERR_UNSUPPORTED).
+ * lin is a HOST array of 7*n_layers structs holding device pointers.
+ * x0: bf16 [d]; out: fp32 [d], the last a; q_out: fp32 [n_layers][d] or NULL;
+ * kv_out: fp32 [n_layers][2][d_kv] (k then v) or NULL.  ws must have been
+ * prepared for the same lin array by littlebit_stack_prepare: the launch
+ * compares fingerprints on the device and, on a mismatch, records
+ * LB_ERR_PLAN in the sticky error word and writes nothing.  Runs as ONE
+ * persistent kernel with one CTA per SM (LB_ERR_UNSUPPORTED if the GPU
+ * cannot hold that grid) and leaves the workspace ready for the next call;
+ * its 4 grid-wide exchanges per layer use the bounded wait described above.
+ * Calls that share a workspace must not overlap in time. */
+lb_status littlebit_stack_forward(const lb_linear *lin, int32_t n_layers, int32_t head_dim,
+                                  const uint16_t *x0, float *out, float *q_out, float *kv_out,
+                                  void *ws, size_t ws_bytes, lb_stream_t stream);
+
+/* Synchronises the stream, reads the workspace's sticky error word, clears
+ * it, and returns LB_OK or the recorded error (LB_ERR_TIMEOUT, LB_ERR_PLAN). */
+lb_status littlebit_poll_error(void *ws, lb_stream_t stream);
+
+/* Diagnostic for the bounded grid-wide wait used by the persistent kernels:
+ * launches one CTA that waits on an arrival which never comes.  The wait
+ * gives up after its limit (about one second), records LB_ERR_TIMEOUT in the
+ * workspace's sticky error word and the kernel returns; read it with
+ * littlebit_poll_error.  ws: a zero-filled workspace of at least 256 bytes. */
+lb_status littlebit_selftest_wait_timeout(void *ws, lb_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* LITTLEBIT_H */

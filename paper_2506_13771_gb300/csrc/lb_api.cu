@@ -1,0 +1,255 @@
+// lb_api.cu -- the extern "C" entry points of liblittlebit.so: argument
+// validation, workspace layout and dispatch to the kernels.  See
+// include/littlebit.h for the contract of every function.
+#include <cstdint>
+#include <cstring>
+
+#include "lb_common.cuh"
+#include "lb_kernels.h"
+
+namespace {
+
+using lb::kWsHeader;
+
+constexpr int kMaxDevices = 64;
+int g_num_sms[kMaxDevices];  // per-device SM count cache (0 = unknown)
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+lb_status from_cuda(cudaError_t e) {
+    if (e == cudaSuccess) return LB_OK;
+    if (e == cudaErrorCooperativeLaunchTooLarge) {
+        cudaGetLastError();
+        return LB_ERR_UNSUPPORTED;
+    }
+    return LB_ERR_CUDA;
+}
+
+lb_status num_sms(int *out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return LB_ERR_CUDA;
+    if (dev >= 0 && dev < kMaxDevices && g_num_sms[dev] > 0) {
+        *out = g_num_sms[dev];
+        return LB_OK;
+    }
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+        return LB_ERR_CUDA;
+    if (dev >= 0 && dev < kMaxDevices) g_num_sms[dev] = n;
+    *out = n;
+    return LB_OK;
+}
+
+// Shape and pointer checks of one linear.  Returns LB_OK, LB_ERR_INVALID_ARG
+// or LB_ERR_UNSUPPORTED.
+lb_status check_linear(const lb_linear *L) {
+    if (!L) return LB_ERR_INVALID_ARG;
+    if (L->d_in <= 0 || L->d_out <= 0) return LB_ERR_INVALID_ARG;
+    if (L->n_paths != 1 && L->n_paths != 2) return LB_ERR_INVALID_ARG;
+    for (int p = 0; p < L->n_paths; ++p) {
+        const lb_path &P = L->path[p];
+        if (P.r <= 0) return LB_ERR_INVALID_ARG;
+        if (!P.v_bits || !P.u_bits || !P.g || !P.l || !P.h) return LB_ERR_INVALID_ARG;
+        if (!aligned16(P.v_bits) || !aligned16(P.u_bits) || !aligned16(P.g) || !aligned16(P.l) ||
+            !aligned16(P.h))
+            return LB_ERR_INVALID_ARG;
+        if (P.r > lb::kMaxRank) return LB_ERR_UNSUPPORTED;
+    }
+    if (L->d_in % 32 != 0) return LB_ERR_UNSUPPORTED;
+    return LB_OK;
+}
+
+bool same_shape(const lb_linear &a, const lb_linear &b) {
+    if (a.d_in != b.d_in || a.d_out != b.d_out || a.n_paths != b.n_paths) return false;
+    for (int p = 0; p < a.n_paths; ++p)
+        if (a.path[p].r != b.path[p].r) return false;
+    return true;
+}
+
+// Shape checks of the seven-linear-per-layer chain.
+lb_status check_stack(const lb_linear *lin, int32_t n_layers, int32_t head_dim,
+                      lb::StackShape *shape) {
+    if (!lin || n_layers <= 0 || head_dim <= 0) return LB_ERR_INVALID_ARG;
+    for (int i = 0; i < 7 * n_layers; ++i) {
+        lb_status st = check_linear(&lin[i]);
+        if (st != LB_OK) return st;
+    }
+    const int d = lin[0].d_in, dkv = lin[1].d_out, dff = lin[4].d_out;
+    // q: d->d, k, v: d->dkv, o: d->d, gate, up: d->dff, down: dff->d
+    const bool chain = lin[0].d_out == d && lin[1].d_in == d && lin[2].d_in == d &&
+                       lin[2].d_out == dkv && lin[3].d_in == d && lin[3].d_out == d &&
+                       lin[4].d_in == d && lin[5].d_in == d && lin[5].d_out == dff &&
+                       lin[6].d_in == dff && lin[6].d_out == d;
+    if (!chain) return LB_ERR_INVALID_ARG;
+    for (int i = 7; i < 7 * n_layers; ++i)
+        if (!same_shape(lin[i], lin[i - 7])) return LB_ERR_UNSUPPORTED;
+    // attention heads: d = n_heads * head_dim, dkv = n_kv_heads * head_dim,
+    // n_heads a multiple of n_kv_heads (grouped-query attention)
+    if (d % head_dim != 0 || dkv % head_dim != 0 || (d / head_dim) % (dkv / head_dim) != 0)
+        return LB_ERR_INVALID_ARG;
+    if (d % 32 != 0 || dff % 32 != 0) return LB_ERR_UNSUPPORTED;
+    shape->head_dim = head_dim;
+    shape->n_layers = n_layers;
+    shape->d = d;
+    shape->dkv = dkv;
+    shape->dff = dff;
+    return LB_OK;
+}
+
+// FNV-1a over the host description of a stack: shapes, ranks and pointers.
+unsigned long long stack_fingerprint(const lb_linear *lin, int32_t n_layers, int32_t head_dim) {
+    unsigned long long h = 1469598103934665603ull;
+    auto mix = [&h](unsigned long long v) {
+        for (int b = 0; b < 8; ++b) {
+            h ^= (v >> (8 * b)) & 0xffu;
+            h *= 1099511628211ull;
+        }
+    };
+    mix((unsigned long long)n_layers);
+    mix((unsigned long long)head_dim);
+    for (int i = 0; i < 7 * n_layers; ++i) {
+        const lb_linear &L = lin[i];
+        mix((unsigned long long)L.d_in);
+        mix((unsigned long long)L.d_out);
+        mix((unsigned long long)L.n_paths);
+        for (int p = 0; p < L.n_paths; ++p) {
+            mix((unsigned long long)L.path[p].r);
+            mix(reinterpret_cast<uintptr_t>(L.path[p].v_bits));
+            mix(reinterpret_cast<uintptr_t>(L.path[p].u_bits));
+            mix(reinterpret_cast<uintptr_t>(L.path[p].g));
+            mix(reinterpret_cast<uintptr_t>(L.path[p].l));
+            mix(reinterpret_cast<uintptr_t>(L.path[p].h));
+        }
+    }
+    return h | 1ull;  // never 0, the value of a zero-filled workspace
+}
+
+// One token goes through the single-launch persistent kernel.
+bool use_decode(const lb_linear &, int64_t T) { return T == 1; }
+
+}  // namespace
+
+extern "C" {
+
+const char *littlebit_status_string(lb_status s) {
+    switch (s) {
+        case LB_OK: return "LB_OK";
+        case LB_ERR_INVALID_ARG: return "LB_ERR_INVALID_ARG";
+        case LB_ERR_UNSUPPORTED: return "LB_ERR_UNSUPPORTED";
+        case LB_ERR_CUDA: return "LB_ERR_CUDA";
+        case LB_ERR_TIMEOUT: return "LB_ERR_TIMEOUT";
+        case LB_ERR_WORKSPACE: return "LB_ERR_WORKSPACE";
+        case LB_ERR_PLAN: return "LB_ERR_PLAN";
+    }
+    return "LB_ERR_UNKNOWN";
+}
+
+lb_status littlebit_pack(const int8_t *signs, int64_t rows, int64_t cols, int32_t layout,
+                         uint32_t *out, int64_t out_words, int32_t *bad, lb_stream_t stream) {
+    if (!signs || !out || rows <= 0 || cols <= 0) return LB_ERR_INVALID_ARG;
+    if (layout != LB_PACK_U && layout != LB_PACK_V) return LB_ERR_INVALID_ARG;
+    const int64_t need = layout == LB_PACK_U ? rows * ((cols + 31) / 32) : ((rows + 31) / 32) * cols;
+    if (out_words < need) return LB_ERR_INVALID_ARG;
+    if (!aligned16(signs) || !aligned16(out)) return LB_ERR_INVALID_ARG;
+    return from_cuda(lb::launch_pack(signs, rows, cols, layout, out, bad, (cudaStream_t)stream));
+}
+
+size_t littlebit_workspace_size(const lb_linear *L, int64_t T) {
+    if (check_linear(L) != LB_OK || T < 0) return 0;
+    size_t floats = lb::generic_ws_floats(*L, T);
+    // the decode path falls back to the two-launch path when its grid cannot
+    // be co-resident, so size for both
+    if (use_decode(*L, T) && lb::decode_ws_floats(*L) > floats) floats = lb::decode_ws_floats(*L);
+    return kWsHeader + ((floats * sizeof(float) + 255) & ~(size_t)255);
+}
+
+lb_status littlebit_linear_forward(const lb_linear *L, const uint16_t *x, int64_t T, void *y,
+                                   int32_t y_dtype, void *ws, size_t ws_bytes,
+                                   lb_stream_t stream) {
+    lb_status st = check_linear(L);
+    if (st != LB_OK) return st;
+    if (T < 0 || (y_dtype != LB_OUT_BF16 && y_dtype != LB_OUT_FP32)) return LB_ERR_INVALID_ARG;
+    if (T == 0) return LB_OK;
+    if (T > INT32_MAX / 8) return LB_ERR_UNSUPPORTED;
+    if (!x || !y || !aligned16(x) || !aligned16(y)) return LB_ERR_INVALID_ARG;
+    if (!ws || ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) ||
+        ws_bytes < littlebit_workspace_size(L, T))
+        return LB_ERR_WORKSPACE;
+    int sms = 0;
+    if ((st = num_sms(&sms)) != LB_OK) return st;
+    cudaStream_t s = (cudaStream_t)stream;
+    unsigned *words = static_cast<unsigned *>(ws);
+    float *data = reinterpret_cast<float *>(static_cast<char *>(ws) + kWsHeader);
+    const int fp32 = y_dtype == LB_OUT_FP32;
+    if (use_decode(*L, T)) {
+        cudaError_t e = lb::launch_decode(*L, x, y, fp32, words, data, sms, s);
+        if (e != cudaErrorCooperativeLaunchTooLarge) return from_cuda(e);
+        cudaGetLastError();  // grid cannot be co-resident here: take the two-launch path
+    }
+    return from_cuda(lb::launch_generic(*L, x, T, y, fp32, data, sms, s));
+}
+
+size_t littlebit_stack_workspace_size(const lb_linear *lin, int32_t n_layers, int32_t head_dim) {
+    lb::StackShape shape;
+    if (check_stack(lin, n_layers, head_dim, &shape) != LB_OK) return 0;
+    return kWsHeader + lb::stack_ws_bytes_after_header(lin, n_layers);
+}
+
+lb_status littlebit_stack_prepare(const lb_linear *lin, int32_t n_layers, int32_t head_dim,
+                                  void *ws, size_t ws_bytes, lb_stream_t stream) {
+    lb::StackShape shape;
+    lb_status st = check_stack(lin, n_layers, head_dim, &shape);
+    if (st != LB_OK) return st;
+    if (!ws || ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) ||
+        ws_bytes < littlebit_stack_workspace_size(lin, n_layers, head_dim))
+        return LB_ERR_WORKSPACE;
+    return from_cuda(lb::launch_stack_prepare(lin, n_layers,
+                                              stack_fingerprint(lin, n_layers, head_dim),
+                                              static_cast<unsigned *>(ws),
+                                              static_cast<char *>(ws) + kWsHeader,
+                                              (cudaStream_t)stream));
+}
+
+lb_status littlebit_stack_forward(const lb_linear *lin, int32_t n_layers, int32_t head_dim,
+                                  const uint16_t *x0, float *out, float *q_out, float *kv_out,
+                                  void *ws, size_t ws_bytes, lb_stream_t stream) {
+    lb::StackShape shape;
+    lb_status st = check_stack(lin, n_layers, head_dim, &shape);
+    if (st != LB_OK) return st;
+    if (!x0 || !out || !aligned16(x0) || !aligned16(out) || (q_out && !aligned16(q_out)) ||
+        (kv_out && !aligned16(kv_out)))
+        return LB_ERR_INVALID_ARG;
+    if (!ws || ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) ||
+        ws_bytes < littlebit_stack_workspace_size(lin, n_layers, head_dim))
+        return LB_ERR_WORKSPACE;
+    int sms = 0;
+    if ((st = num_sms(&sms)) != LB_OK) return st;
+    return from_cuda(lb::launch_stack(lin, n_layers, shape,
+                                      stack_fingerprint(lin, n_layers, head_dim), x0, out, q_out,
+                                      kv_out, static_cast<unsigned *>(ws),
+                                      static_cast<char *>(ws) + kWsHeader, sms,
+                                      (cudaStream_t)stream));
+}
+
+lb_status littlebit_poll_error(void *ws, lb_stream_t stream) {
+    if (!ws) return LB_ERR_WORKSPACE;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return LB_ERR_CUDA;
+    unsigned err = 0;
+    if (cudaMemcpy(&err, ws, sizeof(unsigned), cudaMemcpyDeviceToHost) != cudaSuccess)
+        return LB_ERR_CUDA;
+    if (err != 0u) {
+        const unsigned zero = 0;
+        if (cudaMemcpy(ws, &zero, sizeof(unsigned), cudaMemcpyHostToDevice) != cudaSuccess)
+            return LB_ERR_CUDA;
+        return (lb_status)err;
+    }
+    return LB_OK;
+}
+
+lb_status littlebit_selftest_wait_timeout(void *ws, lb_stream_t stream) {
+    if (!ws || ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0)) return LB_ERR_WORKSPACE;
+    return from_cuda(lb::launch_wait_timeout(static_cast<unsigned *>(ws), (cudaStream_t)stream));
+}
+
+}  // extern "C"

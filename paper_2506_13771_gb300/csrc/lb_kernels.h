@@ -1,0 +1,48 @@
+// lb_kernels.h -- host-side launchers of the LittleBit kernels (internal).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "littlebit.h"
+
+namespace lb {
+
+struct LinDesc;
+
+// Two-launch CUDA-core path for any T (lb_generic.cu).  t_acc: workspace
+// floats, generic_ws_floats() of them.
+size_t generic_ws_floats(const lb_linear &L, int64_t T);
+cudaError_t launch_generic(const lb_linear &L, const uint16_t *x, int64_t T, void *y, int y_fp32,
+                           float *t_acc, int num_sms, cudaStream_t s);
+
+// Single-launch persistent decode of one linear, T = 1 (lb_persistent.cu).
+size_t decode_ws_floats(const lb_linear &L);
+// Returns cudaErrorCooperativeLaunchTooLarge when the grid cannot be co-resident.
+cudaError_t launch_decode(const lb_linear &L, const uint16_t *x, void *y, int y_fp32,
+                          unsigned *ws_words, float *acc, int num_sms, cudaStream_t s);
+
+// Persistent decode of the seven-linear-per-layer stack (lb_persistent.cu).
+struct StackShape {
+    int n_layers, d, dkv, dff, head_dim;
+};
+size_t stack_ws_bytes_after_header(const lb_linear *lin, int n_layers);
+// Writes the device descriptor table, zeroes counters and accumulators, and
+// stores the plan fingerprint.
+cudaError_t launch_stack_prepare(const lb_linear *lin, int n_layers, unsigned long long plan,
+                                 unsigned *ws_words, char *ws_after_header, cudaStream_t s);
+// One persistent launch; leaves counters and accumulators zeroed.
+cudaError_t launch_stack(const lb_linear *lin, int n_layers, const StackShape &shape,
+                         unsigned long long plan, const uint16_t *x0, float *out, float *q_out,
+                         float *kv_out, unsigned *ws_words, char *ws_after_header, int num_sms,
+                         cudaStream_t s);
+
+// Bounded-wait diagnostic (lb_persistent.cu).
+cudaError_t launch_wait_timeout(unsigned *ws_words, cudaStream_t s);
+
+// Sign packing (lb_pack.cu).
+cudaError_t launch_pack(const int8_t *signs, int64_t rows, int64_t cols, int layout,
+                        uint32_t *out, int32_t *bad, cudaStream_t s);
+
+}  // namespace lb

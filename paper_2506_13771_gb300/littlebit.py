@@ -1,0 +1,269 @@
+"""Python binding of liblittlebit.so (include/littlebit.h).
+
+Argument marshalling only: torch owns device memory and streams, every step
+of the LittleBit forward runs in the library's CUDA kernels.  There is no
+CPU fallback: if the library is missing or fails to load, ``lib()`` raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import numpy as np
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_build", "liblittlebit.so")
+
+(LB_OK, LB_ERR_INVALID_ARG, LB_ERR_UNSUPPORTED, LB_ERR_CUDA, LB_ERR_TIMEOUT, LB_ERR_WORKSPACE,
+ LB_ERR_PLAN) = range(7)
+LB_OUT_BF16, LB_OUT_FP32 = 0, 1
+LB_PACK_U, LB_PACK_V = 0, 1
+
+EXPORTED = ["littlebit_status_string", "littlebit_pack", "littlebit_workspace_size",
+            "littlebit_linear_forward", "littlebit_stack_workspace_size",
+            "littlebit_stack_prepare", "littlebit_stack_forward", "littlebit_poll_error",
+            "littlebit_selftest_wait_timeout"]
+
+
+class LittleBitError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        super().__init__(f"{what}: {status_string(status)}")
+
+
+class lb_path(ctypes.Structure):
+    _fields_ = [("r", ctypes.c_int32),
+                ("v_bits", ctypes.c_void_p),
+                ("u_bits", ctypes.c_void_p),
+                ("g", ctypes.c_void_p),
+                ("l", ctypes.c_void_p),
+                ("h", ctypes.c_void_p)]
+
+
+class lb_linear(ctypes.Structure):
+    _fields_ = [("d_in", ctypes.c_int32),
+                ("d_out", ctypes.c_int32),
+                ("n_paths", ctypes.c_int32),
+                ("path", lb_path * 2)]
+
+
+_lib = None
+_lock = threading.Lock()
+
+
+def lib(path: str | None = None):
+    """Load liblittlebit.so (raises OSError if it is not built)."""
+    global _lib
+    with _lock:
+        if _lib is not None and path is None:
+            return _lib
+        p = path or LIB_PATH
+        if not os.path.exists(p):
+            raise OSError(f"{p} is missing: build it with paper_2506_13771_gb300.build.build()")
+        L = ctypes.CDLL(p)
+        vp, i64, i32, sz = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_size_t
+        L.littlebit_status_string.argtypes = [ctypes.c_int]
+        L.littlebit_status_string.restype = ctypes.c_char_p
+        L.littlebit_pack.argtypes = [vp, i64, i64, i32, vp, i64, vp, vp]
+        L.littlebit_pack.restype = ctypes.c_int
+        L.littlebit_workspace_size.argtypes = [ctypes.POINTER(lb_linear), i64]
+        L.littlebit_workspace_size.restype = sz
+        L.littlebit_linear_forward.argtypes = [ctypes.POINTER(lb_linear), vp, i64, vp, i32, vp,
+                                               sz, vp]
+        L.littlebit_linear_forward.restype = ctypes.c_int
+        L.littlebit_stack_workspace_size.argtypes = [ctypes.POINTER(lb_linear), i32, i32]
+        L.littlebit_stack_workspace_size.restype = sz
+        L.littlebit_stack_prepare.argtypes = [ctypes.POINTER(lb_linear), i32, i32, vp, sz, vp]
+        L.littlebit_stack_prepare.restype = ctypes.c_int
+        L.littlebit_stack_forward.argtypes = [ctypes.POINTER(lb_linear), i32, i32, vp, vp, vp, vp,
+                                              vp, sz, vp]
+        L.littlebit_stack_forward.restype = ctypes.c_int
+        L.littlebit_poll_error.argtypes = [vp, vp]
+        L.littlebit_poll_error.restype = ctypes.c_int
+        L.littlebit_selftest_wait_timeout.argtypes = [vp, vp]
+        L.littlebit_selftest_wait_timeout.restype = ctypes.c_int
+        if path is None:
+            _lib = L
+        return L
+
+
+def status_string(status: int) -> str:
+    return lib().littlebit_status_string(int(status)).decode()
+
+
+def _check(status: int, what: str) -> None:
+    if status != LB_OK:
+        raise LittleBitError(status, what)
+
+
+def _stream(stream) -> int | None:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream)
+
+
+# ------------------------------------------------------------------ tensors
+
+
+def to_device_bits(a: np.ndarray, device) -> torch.Tensor:
+    """Copy a numpy bit-pattern array (uint16 / uint32) to the device unchanged."""
+    a = np.ascontiguousarray(a)
+    if a.dtype == np.uint32:
+        return torch.from_numpy(a.view(np.int32)).to(device)
+    if a.dtype == np.uint16:
+        return torch.from_numpy(a.view(np.int16)).to(device)
+    raise TypeError(f"unsupported bit array dtype {a.dtype}")
+
+
+def bf16_tensor(x_bits: np.ndarray, device) -> torch.Tensor:
+    """bf16 bit patterns (uint16) -> torch.bfloat16 tensor on device."""
+    return to_device_bits(x_bits, device).view(torch.bfloat16)
+
+
+class DeviceLinear:
+    """One LittleBit linear resident on the device, and its lb_linear struct.
+
+    Built from a layer dict of ``inputs.make_linear``: packed words are copied
+    as they are; explicit +-1 signs are packed on the device by littlebit_pack.
+    """
+
+    def __init__(self, layer: dict, device="cuda", stream=None):
+        self.d_in = int(layer["d_in"])
+        self.d_out = int(layer["d_out"])
+        self.paths = []
+        self.c = lb_linear()
+        self.c.d_in = self.d_in
+        self.c.d_out = self.d_out
+        self.c.n_paths = len(layer["paths"])
+        for p, P in enumerate(layer["paths"]):
+            r = int(P["r"])
+            if "v_words" in P:
+                v = to_device_bits(P["v_words"], device)
+                u = to_device_bits(P["u_words"], device)
+            else:
+                v = pack(torch.from_numpy(P["v_signs"]).to(device), LB_PACK_V, stream=stream)
+                u = pack(torch.from_numpy(P["u_signs"]).to(device), LB_PACK_U, stream=stream)
+            t = {"v_bits": v, "u_bits": u, "g": to_device_bits(P["g"], device),
+                 "l": to_device_bits(P["l"], device), "h": to_device_bits(P["h"], device)}
+            self.paths.append(t)
+            cp = self.c.path[p]
+            cp.r = r
+            for k, ten in t.items():
+                setattr(cp, k, ten.data_ptr())
+
+    @property
+    def nbytes(self) -> int:
+        return sum(t.numel() * t.element_size() for P in self.paths for t in P.values())
+
+
+# ------------------------------------------------------------------ entry points
+
+
+def pack(signs: torch.Tensor, layout: int, out: torch.Tensor | None = None,
+         bad: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """Eq. 2 packing of a device int8 [rows][cols] +-1 matrix -> int32 words
+    (uint32 bit patterns) in the U or V layout."""
+    assert signs.dtype == torch.int8 and signs.dim() == 2 and signs.is_contiguous()
+    rows, cols = signs.shape
+    shape = (rows, (cols + 31) // 32) if layout == LB_PACK_U else ((rows + 31) // 32, cols)
+    if out is None:
+        out = torch.empty(shape, dtype=torch.int32, device=signs.device)
+    _check(lib().littlebit_pack(signs.data_ptr(), rows, cols, layout, out.data_ptr(), out.numel(),
+                                bad.data_ptr() if bad is not None else None, _stream(stream)),
+           "littlebit_pack")
+    return out
+
+
+def workspace_size(L: DeviceLinear, T: int) -> int:
+    return int(lib().littlebit_workspace_size(ctypes.byref(L.c), int(T)))
+
+
+def new_workspace(nbytes: int, device="cuda") -> torch.Tensor:
+    """A zero-filled workspace (uint8), as the ABI requires before first use."""
+    return torch.zeros(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+
+
+def linear_forward(L: DeviceLinear, x: torch.Tensor, out_dtype=torch.bfloat16,
+                   y: torch.Tensor | None = None, ws: torch.Tensor | None = None,
+                   stream=None) -> torch.Tensor:
+    """Y = X W^T (Prop. 1 per path, Eq. 6 sum) for x bf16 [T][d_in] on device."""
+    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.shape[1] == L.d_in
+    x = x.contiguous()
+    T = x.shape[0]
+    if y is None:
+        y = torch.empty((T, L.d_out), dtype=out_dtype, device=x.device)
+    y_dtype = LB_OUT_FP32 if y.dtype == torch.float32 else LB_OUT_BF16
+    if ws is None:
+        ws = new_workspace(workspace_size(L, T), x.device)
+    _check(lib().littlebit_linear_forward(ctypes.byref(L.c), x.data_ptr(), T, y.data_ptr(),
+                                          y_dtype, ws.data_ptr(), ws.numel(), _stream(stream)),
+           "littlebit_linear_forward")
+    return y
+
+
+class DeviceStack:
+    """n_layers x (q, k, v, o, gate, up, down) LittleBit linears on the device."""
+
+    def __init__(self, layers: list, head_dim: int = 128, device="cuda"):
+        assert len(layers) % 7 == 0
+        self.n_layers = len(layers) // 7
+        self.head_dim = int(head_dim)
+        self.linears = [DeviceLinear(L, device) for L in layers]
+        self.carray = (lb_linear * len(self.linears))(*[L.c for L in self.linears])
+        self.d_model = self.linears[0].d_in
+        self.d_kv = self.linears[1].d_out
+
+    @property
+    def nbytes(self) -> int:
+        return sum(L.nbytes for L in self.linears)
+
+    def workspace_size(self) -> int:
+        return int(lib().littlebit_stack_workspace_size(self.carray, self.n_layers, self.head_dim))
+
+    def prepare(self, ws: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+        """Prepare (and return) a workspace for this stack."""
+        if ws is None:
+            ws = new_workspace(self.workspace_size(), self.linears[0].paths[0]["g"].device)
+        _check(lib().littlebit_stack_prepare(self.carray, self.n_layers, self.head_dim,
+                                             ws.data_ptr(), ws.numel(), _stream(stream)),
+               "littlebit_stack_prepare")
+        return ws
+
+
+def stack_forward(S: DeviceStack, x0: torch.Tensor, out: torch.Tensor | None = None,
+                  q_out: torch.Tensor | None = None, kv_out: torch.Tensor | None = None,
+                  want_q: bool = True, want_kv: bool = True, ws: torch.Tensor | None = None,
+                  stream=None):
+    """One decode step through the stack; returns (out fp32 [d_model],
+    q fp32 [n_layers][d_model] or None, kv fp32 [n_layers][2][d_kv] or None).
+    ws: a workspace prepared by ``S.prepare()`` (one is made if None)."""
+    assert x0.dtype == torch.bfloat16 and x0.numel() == S.d_model
+    dev = x0.device
+    if out is None:
+        out = torch.empty(S.d_model, dtype=torch.float32, device=dev)
+    if q_out is None and want_q:
+        q_out = torch.empty((S.n_layers, S.d_model), dtype=torch.float32, device=dev)
+    if kv_out is None and want_kv:
+        kv_out = torch.empty((S.n_layers, 2, S.d_kv), dtype=torch.float32, device=dev)
+    if ws is None:
+        ws = S.prepare(stream=stream)
+    _check(lib().littlebit_stack_forward(S.carray, S.n_layers, S.head_dim, x0.data_ptr(),
+                                         out.data_ptr(),
+                                         q_out.data_ptr() if q_out is not None else None,
+                                         kv_out.data_ptr() if kv_out is not None else None,
+                                         ws.data_ptr(), ws.numel(), _stream(stream)),
+           "littlebit_stack_forward")
+    return out, q_out, kv_out
+
+
+def poll_error(ws: torch.Tensor, stream=None) -> int:
+    """Synchronise and return (and clear) the workspace's sticky error status."""
+    return int(lib().littlebit_poll_error(ws.data_ptr(), _stream(stream)))
+
+
+def selftest_wait_timeout(ws: torch.Tensor, stream=None) -> None:
+    """Launch the bounded-wait diagnostic (records LB_ERR_TIMEOUT in ws)."""
+    _check(lib().littlebit_selftest_wait_timeout(ws.data_ptr(), _stream(stream)),
+           "littlebit_selftest_wait_timeout")

@@ -37,7 +37,8 @@ def test_exports_every_declared_symbol(L):
 def test_status_strings(L):
     for code, name in [(lb.LB_OK, "LB_OK"), (lb.LB_ERR_INVALID_ARG, "LB_ERR_INVALID_ARG"),
                        (lb.LB_ERR_UNSUPPORTED, "LB_ERR_UNSUPPORTED"), (lb.LB_ERR_CUDA, "LB_ERR_CUDA"),
-                       (lb.LB_ERR_TIMEOUT, "LB_ERR_TIMEOUT"), (lb.LB_ERR_WORKSPACE, "LB_ERR_WORKSPACE")]:
+                       (lb.LB_ERR_TIMEOUT, "LB_ERR_TIMEOUT"), (lb.LB_ERR_WORKSPACE, "LB_ERR_WORKSPACE"),
+                       (lb.LB_ERR_PLAN, "LB_ERR_PLAN")]:
         assert lb.status_string(code) == name
     assert lb.status_string(99) == "LB_ERR_UNKNOWN"
 
@@ -109,20 +110,34 @@ def fake_stack(n_layers=2, d=256, dkv=64, dff=512, rq=16, rk=8, rm=24):
 
 def test_stack_argument_validation(L):
     arr = fake_stack()
-    n = L.littlebit_stack_workspace_size(arr, 2)
+    hd = 32
+    n = L.littlebit_stack_workspace_size(arr, 2, hd)
     assert n > 256 and n % 256 == 0
     st = L.littlebit_stack_forward
-    assert st(arr, 0, FAKE, FAKE, None, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
-    assert st(arr, 2, 0, FAKE, None, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
-    assert st(arr, 2, FAKE, FAKE, FAKE + 8, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
-    assert st(arr, 2, FAKE, FAKE, None, FAKE, n - 256, None) == lb.LB_ERR_WORKSPACE
+    ok = dict(x0=FAKE, out=FAKE, q=None, kv=None, ws=FAKE, nb=n)
+
+    def call(a=arr, layers=2, head_dim=hd, **kw):
+        v = dict(ok, **kw)
+        return st(a, layers, head_dim, v["x0"], v["out"], v["q"], v["kv"], v["ws"], v["nb"], None)
+
+    assert call(layers=0) == lb.LB_ERR_INVALID_ARG
+    assert call(head_dim=0) == lb.LB_ERR_INVALID_ARG
+    assert call(head_dim=48) == lb.LB_ERR_INVALID_ARG               # 256 % 48 != 0
+    assert call(x0=0) == lb.LB_ERR_INVALID_ARG
+    assert call(kv=FAKE + 8) == lb.LB_ERR_INVALID_ARG
+    assert call(q=FAKE + 4) == lb.LB_ERR_INVALID_ARG
+    assert call(nb=n - 256) == lb.LB_ERR_WORKSPACE
     broken = fake_stack()
     broken[3] = fake_linear(256, 128, (16, 16))                      # o must be d -> d
-    assert L.littlebit_stack_workspace_size(broken, 2) == 0
-    assert st(broken, 2, FAKE, FAKE, None, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    assert L.littlebit_stack_workspace_size(broken, 2, hd) == 0
+    assert call(a=broken) == lb.LB_ERR_INVALID_ARG
     uneven = fake_stack()
     uneven[7] = fake_linear(256, 256, (32, 16))                      # layer 1 q differs
-    assert st(uneven, 2, FAKE, FAKE, None, FAKE, n, None) == lb.LB_ERR_UNSUPPORTED
+    assert call(a=uneven) == lb.LB_ERR_UNSUPPORTED
+    prep = L.littlebit_stack_prepare
+    assert prep(arr, 2, 0, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    assert prep(arr, 2, hd, FAKE, n - 256, None) == lb.LB_ERR_WORKSPACE
+    assert prep(uneven, 2, hd, FAKE, n, None) == lb.LB_ERR_UNSUPPORTED
 
 
 def test_pack_argument_validation(L):

@@ -1,0 +1,271 @@
+"""CUDA path vs the fp64 CPU oracle, through the C ABI (needs a GB300).
+
+Bars: sign packing bit-exact; float outputs within relative L2 2e-3 of the
+oracle (bf16 inputs, fp32 accumulation), the tolerance the workload states.
+fp32 outputs are also held to 1e-4: fp32 sums of n sign-weighted terms of
+unit-scale data carry a relative error of order 2^-24 * sqrt(n) (about 1e-5
+for the largest reduction here, n = 28672), so 1e-4 leaves a 10x margin;
+bf16 outputs carry the bf16 rounding itself (relative RMS about 1.2e-3).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2506_13771_gb300 import build as lb_build
+from paper_2506_13771_gb300 import inputs
+from paper_2506_13771_gb300 import littlebit as lb
+
+pytestmark = pytest.mark.gpu
+
+TOL = 2e-3
+TOL_FP32 = 1e-4
+DEV = "cuda"
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    lb_build.build()
+    lb.lib()
+
+
+def rel(a, b) -> float:
+    a = np.asarray(a, np.float64)
+    b = np.asarray(b, np.float64)
+    return float(np.linalg.norm(a - b) / np.linalg.norm(b))
+
+
+def oracle_layer(layer: dict) -> dict:
+    """The oracle's view of a layer: explicit signs packed by the ORACLE packer."""
+    paths = []
+    for P in layer["paths"]:
+        if "v_words" in P:
+            paths.append(P)
+        else:
+            paths.append(dict(r=P["r"], v_words=oracle.pack_v(P["v_signs"]),
+                              u_words=oracle.pack_u(P["u_signs"]), g=P["g"], l=P["l"], h=P["h"]))
+    return {"d_in": layer["d_in"], "d_out": layer["d_out"], "paths": paths}
+
+
+def gpu_forward(D: lb.DeviceLinear, x_bits: np.ndarray, out_dtype) -> np.ndarray:
+    x = lb.bf16_tensor(x_bits, DEV)
+    y = torch.full((x.shape[0], D.d_out), float("nan"), dtype=out_dtype, device=DEV)
+    lb.linear_forward(D, x, y=y)
+    torch.cuda.synchronize()
+    return y.float().cpu().numpy().astype(np.float64)
+
+
+def check(y_gpu, y_ref, out_dtype):
+    assert np.all(np.isfinite(y_gpu)), "unwritten (NaN sentinel) or non-finite outputs"
+    e = rel(y_gpu, y_ref)
+    assert e <= TOL, e
+    if out_dtype == torch.float32:
+        assert e <= TOL_FP32, e
+    return e
+
+
+# ------------------------------------------------------------------ packing (Eq. 2)
+
+
+@pytest.mark.parametrize("rows,cols", [(1, 1), (5, 16), (33, 70), (64, 192), (100, 33),
+                                       (512, 512), (4096, 64)])
+def test_pack_bit_exact(rows, cols):
+    rng = np.random.default_rng(rows * 1000 + cols)
+    s = inputs.random_signs(rng, rows, cols)
+    d = torch.from_numpy(s).to(DEV)
+    wu = lb.pack(d, lb.LB_PACK_U).cpu().numpy().view(np.uint32)
+    wv = lb.pack(d, lb.LB_PACK_V).cpu().numpy().view(np.uint32)
+    assert np.array_equal(wu, oracle.pack_u(s))
+    assert np.array_equal(wv, oracle.pack_v(s))
+
+
+def test_pack_flags_invalid_sign():
+    s = np.ones((8, 40), np.int8)
+    s[3, 17] = 0
+    bad = torch.zeros(1, dtype=torch.int32, device=DEV)
+    lb.pack(torch.from_numpy(s).to(DEV), lb.LB_PACK_U, bad=bad)
+    assert int(bad.item()) == 1
+    ok = torch.zeros(1, dtype=torch.int32, device=DEV)
+    lb.pack(torch.from_numpy(np.ones((8, 40), np.int8)).to(DEV), lb.LB_PACK_V, bad=ok)
+    assert int(ok.item()) == 0
+
+
+# ------------------------------------------------------------------ single linears
+
+
+@pytest.mark.parametrize("out_dtype", [torch.float32, torch.bfloat16])
+def test_config1_512_r16_T4(out_dtype):
+    L, x = inputs.config1()
+    D = lb.DeviceLinear(L, DEV)
+    y = gpu_forward(D, x, out_dtype)
+    OL = oracle_layer(L)
+    check(y, oracle.forward_factored(OL, x), out_dtype)
+    check(y, oracle.forward_dense(OL, x), out_dtype)
+
+
+@pytest.mark.parametrize("T", [1, 8])
+@pytest.mark.parametrize("out_dtype", [torch.float32, torch.bfloat16])
+def test_config2_4096_r64(T, out_dtype):
+    L, x = inputs.config2(T)
+    D = lb.DeviceLinear(L, DEV)
+    check(gpu_forward(D, x, out_dtype), oracle.forward_factored(L, x), out_dtype)
+
+
+@pytest.mark.parametrize("r", [128, 512])
+@pytest.mark.parametrize("T", [1, 16, 64])
+def test_config3_ffn_triple(r, T):
+    lins, x, x_down = inputs.config3(r, T)
+    for name in ("gate", "up", "down"):
+        L = lins[name]
+        xin = x_down if name == "down" else x
+        D = lb.DeviceLinear(L, DEV)
+        check(gpu_forward(D, xin, torch.float32), oracle.forward_factored(L, xin), torch.float32)
+    D = lb.DeviceLinear(lins["down"], DEV)
+    check(gpu_forward(D, x_down, torch.bfloat16), oracle.forward_factored(lins["down"], x_down),
+          torch.bfloat16)
+
+
+@pytest.mark.parametrize("shape", list(inputs.PREFILL_SHAPES))
+@pytest.mark.parametrize("T", [2048, 8192])
+def test_config4_prefill_sampled_tokens(shape, T):
+    """Full-size prefill on the GPU; the oracle recomputes sampled tokens."""
+    L, x = inputs.config4(shape, T)
+    D = lb.DeviceLinear(L, DEV)
+    y = gpu_forward(D, x, torch.bfloat16)
+    assert np.all(np.isfinite(y))
+    rng = np.random.default_rng(T)
+    rows = np.unique(np.concatenate([[0, T - 1], rng.choice(T, 14, replace=False)]))
+    check(y[rows], oracle.forward_factored(L, x[rows]), torch.bfloat16)
+
+
+STRESS = [
+    # d_in, d_out, ranks, T
+    (32, 17, (1,), 1), (32, 1000, (16, 33), 2), (4128, 17, (96, 1), 3), (4128, 1000, (33, 96), 7),
+    (64, 64, (96,), 8), (4128, 1000, (16,), 9), (1024, 300, (33, 16), 65), (4128, 40, (1, 1), 1),
+    (96, 2048, (1000, 24), 1), (8192, 8, (64, 64), 1),
+]
+
+
+@pytest.mark.parametrize("d_in,d_out,rs,T", STRESS)
+def test_stress_shapes(d_in, d_out, rs, T):
+    rng = inputs.rng_for(100, salt=d_in + d_out + T)
+    L = inputs.make_linear(rng, d_in, d_out, list(rs), len(rs), 0.1)
+    x = inputs.bf16_normal(rng, (T, d_in))
+    D = lb.DeviceLinear(L, DEV)
+    check(gpu_forward(D, x, torch.float32), oracle.forward_factored(L, x), torch.float32)
+
+
+@pytest.mark.parametrize("T", [1, 4])
+def test_padding_bits_are_ignored(T):
+    """U words with every padding bit set (r = 33, 16) give the same output."""
+    rng = inputs.rng_for(101, salt=T)
+    L = inputs.make_linear(rng, 256, 96, [33, 16], 2, 0.1)
+    x = inputs.bf16_normal(rng, (T, 256))
+    y_ref = oracle.forward_factored(L, x)
+    for P, pad in zip(L["paths"], (0xFFFFFFFE, 0xFFFF0000)):
+        P["u_words"] = P["u_words"].copy()
+        P["u_words"][:, -1] |= np.uint32(pad)
+    D = lb.DeviceLinear(L, DEV)
+    check(gpu_forward(D, x, torch.float32), y_ref, torch.float32)
+
+
+# ------------------------------------------------------------------ stack
+
+
+def run_stack(layers, x0, head_dim):
+    S = lb.DeviceStack(layers, head_dim, DEV)
+    x = lb.bf16_tensor(x0, DEV)
+    out = torch.full((S.d_model,), float("nan"), device=DEV)
+    q = torch.full((S.n_layers, S.d_model), float("nan"), device=DEV)
+    kv = torch.full((S.n_layers, 2, S.d_kv), float("nan"), device=DEV)
+    ws = S.prepare()
+    lb.stack_forward(S, x, out=out, q_out=q, kv_out=kv, ws=ws)
+    assert lb.poll_error(ws) == lb.LB_OK
+    return (out.cpu().numpy().astype(np.float64), q.cpu().numpy().astype(np.float64),
+            kv.cpu().numpy().astype(np.float64))
+
+
+def check_stack(got, ref):
+    out, q, kv = got
+    r_out, r_q, r_kv = ref
+    for g, r in ((out, r_out), (q, r_q), (kv, r_kv)):
+        assert np.all(np.isfinite(g))
+    assert rel(out, r_out) <= TOL_FP32, rel(out, r_out)
+    for l in range(q.shape[0]):
+        assert rel(q[l], r_q[l]) <= TOL_FP32, (l, rel(q[l], r_q[l]))
+        assert rel(kv[l, 0], r_kv[l, 0]) <= TOL_FP32, (l, "k")
+        assert rel(kv[l, 1], r_kv[l, 1]) <= TOL_FP32, (l, "v")
+
+
+def test_stack_small():
+    layers, x0 = inputs.make_stack(n_layers=3, d_model=1024, d_kv=256, d_ff=2048, r_qo=48,
+                                   r_kv=16, r_mlp=64, head_dim=64, config_id=102)
+    check_stack(run_stack(layers, x0, 64), oracle.stack_forward(layers, x0, head_dim=64))
+
+
+def test_stack_ragged_slices():
+    """d_model / 32 and d_ff / 32 not multiples of the CTA count; one path."""
+    layers, x0 = inputs.make_stack(n_layers=2, d_model=640, d_kv=160, d_ff=1696, r_qo=40,
+                                   r_kv=8, r_mlp=56, head_dim=32, config_id=103)
+    for L in layers:
+        L["paths"] = L["paths"][:1]
+    check_stack(run_stack(layers, x0, 32), oracle.stack_forward(layers, x0, head_dim=32))
+
+
+def test_stack_workspace_reuse_and_plan_check():
+    """Back-to-back launches on one prepared workspace agree (the launch leaves
+    it clean); a workspace prepared for other linears is refused on the
+    device with LB_ERR_PLAN and no output is written."""
+    layers, x0 = inputs.make_stack(n_layers=2, d_model=512, d_kv=128, d_ff=1024, r_qo=32,
+                                   r_kv=8, r_mlp=48, head_dim=64, config_id=104)
+    S = lb.DeviceStack(layers, 64, DEV)
+    x = lb.bf16_tensor(x0, DEV)
+    ws = S.prepare()
+    outs = []
+    for _ in range(3):
+        out, _, _ = lb.stack_forward(S, x, ws=ws)
+        outs.append(out.cpu().numpy().astype(np.float64))
+    assert lb.poll_error(ws) == lb.LB_OK
+    ref = oracle.stack_forward(layers, x0, head_dim=64)[0]
+    for o in outs:
+        assert rel(o, ref) <= TOL_FP32
+    other_layers, _ = inputs.make_stack(n_layers=2, d_model=512, d_kv=128, d_ff=1024, r_qo=32,
+                                        r_kv=8, r_mlp=48, head_dim=64, config_id=105)
+    S2 = lb.DeviceStack(other_layers, 64, DEV)
+    out2 = torch.full((512,), float("nan"), device=DEV)
+    lb.stack_forward(S2, x, out=out2, want_q=False, want_kv=False, ws=ws)
+    assert lb.poll_error(ws) == lb.LB_ERR_PLAN
+    assert torch.isnan(out2).all()
+    S2.prepare(ws)
+    lb.stack_forward(S2, x, out=out2, want_q=False, want_kv=False, ws=ws)
+    assert lb.poll_error(ws) == lb.LB_OK
+    assert rel(out2.cpu().numpy(), oracle.stack_forward(other_layers, x0, head_dim=64)[0]) <= TOL_FP32
+
+
+def test_stack_70b_full():
+    """The full 80-layer Llama2-70B-shaped stack, every output checked."""
+    layers, x0 = inputs.config5()
+    check_stack(run_stack(layers, x0, 128), oracle.stack_forward(layers, x0, head_dim=128))
+
+
+# ------------------------------------------------------------------ bounded waits
+
+
+def test_grid_wait_times_out_and_is_sticky():
+    """A wait nobody releases gives up after its limit with LB_ERR_TIMEOUT; until
+    polled, kernels on that workspace return without writing; after the poll
+    the workspace works again."""
+    L, x = inputs.config2(1)
+    D = lb.DeviceLinear(L, DEV)
+    ws = lb.new_workspace(lb.workspace_size(D, 1), DEV)
+    lb.selftest_wait_timeout(ws)
+    xin = lb.bf16_tensor(x, DEV)
+    y = torch.full((1, D.d_out), float("nan"), dtype=torch.float32, device=DEV)
+    lb.linear_forward(D, xin, y=y, ws=ws)
+    assert lb.poll_error(ws) == lb.LB_ERR_TIMEOUT
+    assert torch.isnan(y).all(), "a kernel wrote outputs while the error word was set"
+    assert lb.poll_error(ws) == lb.LB_OK
+    lb.linear_forward(D, xin, y=y, ws=ws)
+    torch.cuda.synchronize()
+    check(y.cpu().numpy().astype(np.float64), oracle.forward_factored(L, x), torch.float32)
