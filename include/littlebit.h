@@ -66,7 +66,8 @@ typedef enum {
     LB_ERR_CUDA = 3,         /* a CUDA runtime call or launch failed */
     LB_ERR_TIMEOUT = 4,      /* a device-side grid wait ran out (see poll) */
     LB_ERR_WORKSPACE = 5,    /* ws is NULL, misaligned or too small */
-    LB_ERR_PLAN = 6          /* stack workspace not prepared for these linears */
+    LB_ERR_PLAN = 6,         /* stack workspace not prepared for these linears */
+    LB_ERR_RANGE = 7         /* a stack intermediate left the exchange's range */
 } lb_status;
 
 typedef enum { LB_OUT_BF16 = 0, LB_OUT_FP32 = 1 } lb_out_dtype;

@@ -140,6 +140,7 @@ const char *littlebit_status_string(lb_status s) {
         case LB_ERR_TIMEOUT: return "LB_ERR_TIMEOUT";
         case LB_ERR_WORKSPACE: return "LB_ERR_WORKSPACE";
         case LB_ERR_PLAN: return "LB_ERR_PLAN";
+        case LB_ERR_RANGE: return "LB_ERR_RANGE";
     }
     return "LB_ERR_UNKNOWN";
 }
@@ -224,6 +225,7 @@ lb_status littlebit_stack_forward(const lb_linear *lin, int32_t n_layers, int32_
         return LB_ERR_WORKSPACE;
     int sms = 0;
     if ((st = num_sms(&sms)) != LB_OK) return st;
+    if (!lb::stack_supported(lin, shape, sms)) return LB_ERR_UNSUPPORTED;
     return from_cuda(lb::launch_stack(lin, n_layers, shape,
                                       stack_fingerprint(lin, n_layers, head_dim), x0, out, q_out,
                                       kv_out, static_cast<unsigned *>(ws),

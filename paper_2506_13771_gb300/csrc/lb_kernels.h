@@ -32,6 +32,10 @@ size_t stack_ws_bytes_after_header(const lb_linear *lin, int n_layers);
 // stores the plan fingerprint.
 cudaError_t launch_stack_prepare(const lb_linear *lin, int n_layers, unsigned long long plan,
                                  unsigned *ws_words, char *ws_after_header, cudaStream_t s);
+// Whether the one-launch stack kernel handles these shapes on this GPU
+// (ranks multiples of 8, head_dim multiple of 32, d_kv multiple of 8, the
+// shared-memory plan fits).
+bool stack_supported(const lb_linear *lin, const StackShape &shape, int num_sms);
 // One persistent launch; leaves counters and accumulators zeroed.
 cudaError_t launch_stack(const lb_linear *lin, int n_layers, const StackShape &shape,
                          unsigned long long plan, const uint16_t *x0, float *out, float *q_out,

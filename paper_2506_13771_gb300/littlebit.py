@@ -17,7 +17,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "_build", "liblittlebit.so")
 
 (LB_OK, LB_ERR_INVALID_ARG, LB_ERR_UNSUPPORTED, LB_ERR_CUDA, LB_ERR_TIMEOUT, LB_ERR_WORKSPACE,
- LB_ERR_PLAN) = range(7)
+ LB_ERR_PLAN, LB_ERR_RANGE) = range(8)
 LB_OUT_BF16, LB_OUT_FP32 = 0, 1
 LB_PACK_U, LB_PACK_V = 0, 1
 

@@ -38,7 +38,7 @@ def test_status_strings(L):
     for code, name in [(lb.LB_OK, "LB_OK"), (lb.LB_ERR_INVALID_ARG, "LB_ERR_INVALID_ARG"),
                        (lb.LB_ERR_UNSUPPORTED, "LB_ERR_UNSUPPORTED"), (lb.LB_ERR_CUDA, "LB_ERR_CUDA"),
                        (lb.LB_ERR_TIMEOUT, "LB_ERR_TIMEOUT"), (lb.LB_ERR_WORKSPACE, "LB_ERR_WORKSPACE"),
-                       (lb.LB_ERR_PLAN, "LB_ERR_PLAN")]:
+                       (lb.LB_ERR_PLAN, "LB_ERR_PLAN"), (lb.LB_ERR_RANGE, "LB_ERR_RANGE")]:
         assert lb.status_string(code) == name
     assert lb.status_string(99) == "LB_ERR_UNKNOWN"
 
