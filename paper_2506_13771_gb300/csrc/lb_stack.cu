@@ -40,7 +40,8 @@ namespace lb {
 namespace {
 
 constexpr int kST = 512;        // threads per CTA
-constexpr int kSW = kST / 32;   // warps per CTA
+constexpr int kCW = 15;         // compute warps; warp 15 issues the bulk copies
+constexpr int kCT = kCW * 32;   // compute threads
 constexpr float kFix = 16777216.f;            // 2^24
 constexpr float kFixInv = 1.f / 16777216.f;
 
@@ -177,70 +178,137 @@ __device__ __forceinline__ void split_word(uint32_t word, uint32_t copy, uint32_
     hi = ((word >> 2) & 0x3C3C3C3Cu) | copy;
 }
 
-// Fill n_tab nibble tables at byte offset tb: table n holds, for e = 0..15,
-// sum_{k<4} (bit k of e ? -v : +v)[4n + k] with v_i = src[i] * scale[i] * mul
-// (scale: fp16, may be null), twice (entries e and 16 + e).  Tables past the
-// n_vals values are zero, so sign bits beyond them contribute nothing.
-__device__ void build_tables(int tb, int n_tab, const float *src, const uint16_t *scale, float mul,
-                             int n_vals) {
-    float *T = sm_f(tb);
-    for (int idx = threadIdx.x; idx < n_tab * 16; idx += blockDim.x) {
-        const int n = idx >> 4, e = idx & 15;
-        float v = 0.f;
-        if (4 * n < n_vals) {
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const int i = 4 * n + k;
-                float x = src[i] * mul;
-                if (scale) x *= half_bits_to_float(scale[i]);
-                v += ((e >> k) & 1) ? -x : x;
-            }
-        }
-        T[n * 32 + e] = v;
-        T[n * 32 + 16 + e] = v;
-    }
-}
+// Compute helpers.  Job arrays have a compile-time size NJ (the jobs a step
+// could have with two paths per linear) and are indexed with compile-time
+// indices only, so they stay in registers; a job that does not exist (a
+// linear with one path) has no rows / columns / tables.  All buffers are
+// byte offsets into g_smem.
 
-// One stage-2 job: rows [0, nrows) of one path, U words and h in shared memory.
-struct UJob {
-    int U, h;     // byte offsets: U words [nrows][R], h fp16 [nrows]
-    int R, nrows;
-    int tb;       // byte offset of the z tables (R * 1024 bytes)
-    float *ys;    // output rows (accumulated with atomicAdd)
+// Nibble tables of one value vector: table n (n < n_tab), entry e = 0..15 is
+// sum_{k<4} (bit k of e ? -v : +v)[4n + k] with v_i = src[i] * mul * scale[i]
+// (scale: fp16 offset, or -1 for none), stored twice (entries e and 16 + e,
+// one copy per half-warp).  Tables at or past n_vals / 4 are zero, so sign
+// bits beyond the data (padding) add nothing.
+struct TJ {
+    int tb;      // byte offset of table 0 (256-aligned)
+    int n_tab;   // tables to fill (0: job absent)
+    int n_vals;  // values available
+    int src;     // byte offset of the fp32 values
+    int scale;   // byte offset of the fp16 scales, or -1
+    float mul;
 };
 
-// ys[row] += h[row] * sum_j U_sign[row][j] z[j]; a warp takes 32 rows x one
-// word at a time, so all its lanes read the same 8 tables.
-__device__ void u_stage(const UJob *jobs, int njobs) {
+// One thread per (table, 16-byte quarter): 8 consecutive threads write one
+// table's 128 bytes, so the float4 stores of a warp are bank-conflict free.
+template <int NJ>
+__device__ __forceinline__ void build_tables(const TJ (&J)[NJ]) {
+    int cum[NJ + 1];
+    cum[0] = 0;
+#pragma unroll
+    for (int j = 0; j < NJ; ++j) cum[j + 1] = cum[j] + 8 * J[j].n_tab;
+    for (int idx = threadIdx.x; idx < cum[NJ]; idx += kCT) {
+        int tb = J[0].tb, n_vals = J[0].n_vals, src = J[0].src, scale = J[0].scale, t = idx;
+        float mul = J[0].mul;
+#pragma unroll
+        for (int j = 1; j < NJ; ++j)
+            if (idx >= cum[j]) {
+                tb = J[j].tb;
+                n_vals = J[j].n_vals;
+                src = J[j].src;
+                scale = J[j].scale;
+                mul = J[j].mul;
+                t = idx - cum[j];
+            }
+        const int n = t >> 3, q = t & 7;
+        float z[4] = {0.f, 0.f, 0.f, 0.f};
+        if (4 * n < n_vals) {
+            const float4 v = *reinterpret_cast<const float4 *>(g_smem + src + 16 * n);
+            z[0] = v.x * mul;
+            z[1] = v.y * mul;
+            z[2] = v.z * mul;
+            z[3] = v.w * mul;
+            if (scale >= 0) {
+                const uint2 hb = *reinterpret_cast<const uint2 *>(g_smem + scale + 8 * n);
+                z[0] *= half_bits_to_float((uint16_t)(hb.x & 0xffffu));
+                z[1] *= half_bits_to_float((uint16_t)(hb.x >> 16));
+                z[2] *= half_bits_to_float((uint16_t)(hb.y & 0xffffu));
+                z[3] *= half_bits_to_float((uint16_t)(hb.y >> 16));
+            }
+        }
+        // entries 4(q&3) .. 4(q&3)+3: high bits (e3 e2) = q & 3, low bits run 0..3
+        const int hb2 = q & 3;
+        const float s2 = (hb2 & 1) ? -z[2] : z[2];
+        const float s3 = (hb2 & 2) ? -z[3] : z[3];
+        const float qv = s2 + s3;
+        const float4 r = make_float4(z[0] + z[1] + qv, z[1] - z[0] + qv, z[0] - z[1] + qv,
+                                     -z[0] - z[1] + qv);
+        *reinterpret_cast<float4 *>(g_smem + tb + n * 128 + q * 16) = r;
+    }
+}
+
+// Stage 2 job: ys[row] += h[row] * sum_j U_sign[row][j] z[j] for rows
+// [0, nrows) of one path; U words [nrows][R] and h at U / h; z tables at tb.
+struct UJ {
+    int U, h, R, nrows, tb, ys;
+};
+
+// A task is 32 rows x a run of words of one job; its lanes (rows) read the
+// same 8 tables per word, so lookups are bank-conflict free.  Runs are split
+// when the jobs have fewer 32-row blocks than twice the compute warps.
+template <int NJ>
+__device__ __forceinline__ void u_stage(const UJ (&J)[NJ]) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
-    int total = 0;
-    for (int j = 0; j < njobs; ++j) total += ((jobs[j].nrows + 31) >> 5) * jobs[j].R;
-    for (int task = warp; task < total; task += kSW) {
-        int jb = 0, t = task;
-        while (t >= ((jobs[jb].nrows + 31) >> 5) * jobs[jb].R) {
-            t -= ((jobs[jb].nrows + 31) >> 5) * jobs[jb].R;
-            ++jb;
-        }
-        const UJob &J = jobs[jb];
-        const int rb = t / J.R, w = t - rb * J.R;
+    int blocks = 0;
+#pragma unroll
+    for (int j = 0; j < NJ; ++j) blocks += (J[j].nrows + 31) >> 5;
+    const int split = blocks >= 2 * kCW ? 1 : (2 * kCW + blocks - 1) / max(blocks, 1);
+    int cum[NJ + 1], nch[NJ], wc[NJ];
+    cum[0] = 0;
+#pragma unroll
+    for (int j = 0; j < NJ; ++j) {
+        const int n0 = min(split, J[j].R);
+        wc[j] = (J[j].R + n0 - 1) / n0;
+        nch[j] = (J[j].R + wc[j] - 1) / wc[j];
+        cum[j + 1] = cum[j] + ((J[j].nrows + 31) >> 5) * nch[j];
+    }
+    for (int task = warp; task < cum[NJ]; task += kCW) {
+        int U = J[0].U, h = J[0].h, R = J[0].R, nrows = J[0].nrows, tb = J[0].tb, ys = J[0].ys;
+        int t = task, nc = nch[0], w_c = wc[0];
+#pragma unroll
+        for (int j = 1; j < NJ; ++j)
+            if (task >= cum[j]) {
+                U = J[j].U;
+                h = J[j].h;
+                R = J[j].R;
+                nrows = J[j].nrows;
+                tb = J[j].tb;
+                ys = J[j].ys;
+                t = task - cum[j];
+                nc = nch[j];
+                w_c = wc[j];
+            }
+        const int rb = t / nc, w0 = (t - rb * nc) * w_c;
+        const int w1 = min(w0 + w_c, R);
         const int row = 32 * rb + lane;
-        if (row < J.nrows) {
-            const uint32_t word = sm_u32(J.U)[row * J.R + w];
-            uint32_t lo, hi;
-            split_word(word, copy, lo, hi);
-            const float acc = lut8(lo, hi, (uint32_t)(J.tb + w * 1024));
-            atomicAdd(J.ys + row, acc * half_bits_to_float(sm_u16(J.h)[row]));
+        if (row < nrows) {
+            const uint32_t *Uw = sm_u32(U) + row * R;
+            float acc = 0.f;
+            for (int w = w0; w < w1; ++w) {
+                uint32_t lo, hi;
+                split_word(Uw[w], copy, lo, hi);
+                acc += lut8(lo, hi, (uint32_t)(tb + w * 1024));
+            }
+            atomicAdd(sm_f(ys) + row, acc * half_bits_to_float(sm_u16(h)[row]));
         }
     }
 }
 
-// One stage-1 job: all r columns of one path over the CTA's nw input words.
-struct VJob {
-    int V;        // byte offset of V words [nw][r]
-    int r, nw;
-    int tb;       // byte offset of the input tables (nw * 1024 bytes)
-    unsigned long long *dst;  // exchange words of this path's t
+// Stage 1 job: all r columns of one path over the CTA's nw input words; V
+// words [nw][r] at V, input tables at tb; the partial t goes to dst.
+struct VJ {
+    int V, r, nw, tb;
+    unsigned long long *dst;
 };
 
 __device__ __forceinline__ void red_fix(unsigned long long *p, float v, float limit,
@@ -254,60 +322,109 @@ __device__ __forceinline__ void red_fix(unsigned long long *p, float v, float li
 }
 
 // t[j] partial over the slice, added to the exchange words (one contribution
-// per CTA per element, also when the slice is empty).
-__device__ void v_stage(const VJob *jobs, int njobs, float limit, unsigned *err) {
+// per CTA per element, also when the slice is empty).  A task is 32 columns
+// x all slice words of one job.
+template <int NJ>
+__device__ __forceinline__ void v_stage(const VJ (&J)[NJ], float limit, unsigned *err) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
-    int total = 0;
-    for (int j = 0; j < njobs; ++j) total += (jobs[j].r + 31) >> 5;
-    for (int task = warp; task < total; task += kSW) {
-        int jb = 0, t = task;
-        while (t >= ((jobs[jb].r + 31) >> 5)) {
-            t -= (jobs[jb].r + 31) >> 5;
-            ++jb;
-        }
-        const VJob &J = jobs[jb];
-        const int col = 32 * t + lane;
-        if (col < J.r) {
-            float acc = 0.f;
-            const uint32_t *V = sm_u32(J.V);
-            for (int w = 0; w < J.nw; ++w) {
-                uint32_t lo, hi;
-                split_word(V[w * J.r + col], copy, lo, hi);
-                acc += lut8(lo, hi, (uint32_t)(J.tb + w * 1024));
+    int cum[NJ + 1];
+    cum[0] = 0;
+#pragma unroll
+    for (int j = 0; j < NJ; ++j) cum[j + 1] = cum[j] + ((J[j].r + 31) >> 5);
+    for (int task = warp; task < cum[NJ]; task += kCW) {
+        int V = J[0].V, r = J[0].r, nw = J[0].nw, tb = J[0].tb, t = task;
+        unsigned long long *dst = J[0].dst;
+#pragma unroll
+        for (int j = 1; j < NJ; ++j)
+            if (task >= cum[j]) {
+                V = J[j].V;
+                r = J[j].r;
+                nw = J[j].nw;
+                tb = J[j].tb;
+                dst = J[j].dst;
+                t = task - cum[j];
             }
-            red_fix(J.dst + col, acc, limit, err);
+        const int col = 32 * t + lane;
+        if (col < r) {
+            float acc = 0.f;
+            const uint32_t *Vw = sm_u32(V) + col;
+            for (int w = 0; w < nw; ++w) {
+                uint32_t lo, hi;
+                split_word(Vw[w * r], copy, lo, hi);
+                acc += lut8(lo, hi, (uint32_t)(tb + w * 1024));
+            }
+            red_fix(dst + col, acc, limit, err);
         }
     }
 }
 
-__device__ __forceinline__ float block_sum_sq(const float *v, int n) {
+// Barrier over the compute warps only (named barrier 1).
+__device__ __forceinline__ void csync() { asm volatile("bar.sync 1, %0;" ::"n"(kCT) : "memory"); }
+
+// AND of pred over the compute threads, returned to each of them.
+__device__ __forceinline__ int csync_and(int pred) {
+    int r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\tsetp.ne.s32 p, %1, 0;\n\tbar.red.and.pred q, 1, %2, p;\n\t"
+        "selp.s32 %0, 1, 0, q;\n\t}"
+        : "=r"(r)
+        : "r"(pred), "n"(kCT)
+        : "memory");
+    return r;
+}
+
+// Sum of v over the compute threads, returned to each of them.
+__device__ float csum(float v) {
+    __shared__ float s_part[kCW];
+    __shared__ float s_total;
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) s_part[warp] = v;
+    csync();
+    if (warp == 0) {
+        float t = lane < kCW ? s_part[lane] : 0.f;
+        for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+        if (lane == 0) s_total = t;
+    }
+    csync();
+    const float total = s_total;
+    csync();
+    return total;
+}
+
+__device__ __forceinline__ float sum_sq(const float *v, int n) {
     float s = 0.f;
-    for (int i = threadIdx.x; i < n; i += blockDim.x) s += v[i] * v[i];
-    return block_sum(s);
+    for (int i = threadIdx.x; i < n; i += kCT) s += v[i] * v[i];
+    return csum(s);
 }
 
 __device__ __forceinline__ void zero_f(float *p, int n) {
-    for (int i = threadIdx.x; i < n; i += blockDim.x) p[i] = 0.f;
+    for (int i = threadIdx.x; i < n; i += kCT) p[i] = 0.f;
 }
 
 // Zero this CTA's stripe of an exchange region whose readers are all done.
 __device__ __forceinline__ void zero_stripe(unsigned long long *region, int len) {
     const int a = (int)((long long)blockIdx.x * len / gridDim.x);
     const int b = (int)((long long)(blockIdx.x + 1) * len / gridDim.x);
-    for (int i = a + threadIdx.x; i < b; i += blockDim.x) region[i] = 0ull;
+    for (int i = a + threadIdx.x; i < b; i += kCT) region[i] = 0ull;
 }
 
 __device__ __forceinline__ bool sticky(const unsigned *ws_words) {
     return ld_relaxed_gpu(ws_words + kErrWord) != 0u;
 }
 
+__device__ __forceinline__ void record(unsigned *ws_words, lb_status st) {
+    atomicCAS(ws_words + kErrWord, 0u, static_cast<unsigned>(st));
+}
+
 // Wait until each of region[0..n) counts n_ctas contributions and decode the
-// sums into out[0..n).  Bounded; returns false (to every thread) on failure.
-__device__ bool poll_decode(const unsigned long long *region, int n, unsigned n_ctas, float *out,
-                            unsigned *ws_words) {
+// sums into out[0..n).  Bounded; returns false (to every compute thread) on
+// failure.
+__device__ __noinline__ bool poll_decode(const unsigned long long *region, int n, unsigned n_ctas,
+                                         float *out, unsigned *ws_words) {
     int ok = 1;
-    for (int i = 2 * threadIdx.x; i < n && ok; i += 2 * blockDim.x) {
+    for (int i = 2 * threadIdx.x; i < n && ok; i += 2 * kCT) {
         unsigned long long t0 = 0;
         for (int spin = 0;; ++spin) {
             unsigned long long a, b;
@@ -326,14 +443,30 @@ __device__ bool poll_decode(const unsigned long long *region, int n, unsigned n_
                 const unsigned long long now = globaltimer_ns();
                 if (t0 == 0) t0 = now;
                 if (now - t0 > kWaitLimitNs) {
-                    atomicCAS(ws_words + kErrWord, 0u, static_cast<unsigned>(LB_ERR_TIMEOUT));
+                    record(ws_words, LB_ERR_TIMEOUT);
                     ok = 0;
                     break;
                 }
             }
         }
     }
-    return __syncthreads_and(ok) != 0;
+    return csync_and(ok) != 0;
+}
+
+// Bounded wait on an mbarrier phase by every compute thread.
+__device__ bool wait_full(unsigned long long *bar, unsigned parity, unsigned *ws_words) {
+    int ok = 1;
+    if (!mbar_try_wait(bar, parity)) {
+        const unsigned long long t0 = globaltimer_ns();
+        while (!mbar_try_wait(bar, parity)) {
+            if (globaltimer_ns() - t0 > kWaitLimitNs) {
+                record(ws_words, LB_ERR_TIMEOUT);
+                ok = 0;
+                break;
+            }
+        }
+    }
+    return csync_and(ok) != 0;
 }
 
 __device__ __forceinline__ float silu(float x) { return x / (1.f + __expf(-x)); }
@@ -344,10 +477,13 @@ struct Part {
     int dw0, nd, fw0, nf, k0, nkv;
 };
 
+// The bulk-copy producer (lane 0 of warp 15).  Phase X of layer l has its
+// own buffer; the copies for X(l+1) are issued once the compute warps have
+// released X(l) (empty barrier), and land on the full barrier of X.
 struct Loader {
     const Params *P;
     Part s;
-    unsigned long long *bar;  // 4 mbarriers: phases A, B, C, D
+    unsigned long long *full;
 
     __device__ void copy(int dst, const void *src, unsigned bytes, unsigned long long *b) const {
         if (bytes == 0) return;
@@ -373,7 +509,7 @@ struct Loader {
     // phase A of layer l (0 <= l <= n_layers): down of layer l-1 on R_c rows,
     // stage 1 of q, k, v of layer l on R_c (absent for l = n_layers).
     __device__ void issue_A(int l) const {
-        unsigned long long *b = bar + 0;
+        unsigned long long *b = full + 0;
         const Offsets &o = P->o;
         if (l > 0) {
             const LinDesc &D = P->lin[7 * (l - 1) + LD];
@@ -392,7 +528,7 @@ struct Loader {
         mbar_arrive(b);
     }
     __device__ void issue_B(int l) const {
-        unsigned long long *b = bar + 1;
+        unsigned long long *b = full + 1;
         const Offsets &o = P->o;
         const LinDesc &Q = P->lin[7 * l + LQ], &K = P->lin[7 * l + LK], &V = P->lin[7 * l + LV],
                       &O = P->lin[7 * l + LO];
@@ -421,7 +557,7 @@ struct Loader {
         mbar_arrive(b);
     }
     __device__ void issue_C(int l) const {
-        unsigned long long *b = bar + 2;
+        unsigned long long *b = full + 2;
         const Offsets &o = P->o;
         const LinDesc &O = P->lin[7 * l + LO], &G = P->lin[7 * l + LG], &U = P->lin[7 * l + LU];
         for (int p = 0; p < O.n_paths; ++p) {
@@ -433,7 +569,7 @@ struct Loader {
         mbar_arrive(b);
     }
     __device__ void issue_D(int l) const {
-        unsigned long long *b = bar + 3;
+        unsigned long long *b = full + 3;
         const Offsets &o = P->o;
         const LinDesc &G = P->lin[7 * l + LG], &U = P->lin[7 * l + LU], &D = P->lin[7 * l + LD];
         for (int p = 0; p < G.n_paths; ++p) {
@@ -447,49 +583,65 @@ struct Loader {
         for (int p = 0; p < D.n_paths; ++p) vslice(o.d_Vd[p], o.d_gd[p], D, p, s.fw0, s.nf, b);
         mbar_arrive(b);
     }
+    __device__ void issue(int buf, int l) const {
+        if (buf == 0) issue_A(l);
+        else if (buf == 1) issue_B(l);
+        else if (buf == 2) issue_C(l);
+        else issue_D(l);
+    }
 };
 
-// Bounded wait for a phase buffer.  On failure records LB_ERR_TIMEOUT.
-__device__ bool wait_buffer(unsigned long long *bar, unsigned parity, unsigned *ws_words) {
-    __shared__ int s_ok;
-    if (threadIdx.x == 0) {
-        int ok = 1;
-        if (!mbar_try_wait(bar, parity)) {
-            const unsigned long long t0 = globaltimer_ns();
-            while (!mbar_try_wait(bar, parity)) {
-                if (globaltimer_ns() - t0 > kWaitLimitNs) {
-                    atomicCAS(ws_words + kErrWord, 0u, static_cast<unsigned>(LB_ERR_TIMEOUT));
-                    ok = 0;
-                    break;
+// Producer loop: issue every phase buffer of every layer in consumption
+// order, each after the compute warps released its previous use.  Waits are
+// bounded and stop at the first recorded error; before returning, the
+// producer waits (bounded) for all copies it issued to land, so none arrives
+// after the CTA is gone.
+__device__ void producer(const Loader &ld, unsigned long long *empty, unsigned *ws_words) {
+    const int L = ld.P->n_layers;
+    int last_use[4] = {0, 0, 0, 0};
+    for (int b = 0; b < 4; ++b) ld.issue(b, 0);
+    bool ok = true;
+    for (int l = 1; l <= L && ok; ++l) {
+        for (int b = 0; b < 4 && ok; ++b) {
+            if (b > 0 && l == L) break;  // the final phase needs only buffer A
+            const unsigned parity = (unsigned)((l - 1) & 1);
+            unsigned long long t0 = 0;
+            for (int spin = 0; !mbar_try_wait(empty + b, parity); ++spin) {
+                if ((spin & 63) == 63) {
+                    if (sticky(ws_words)) {
+                        ok = false;
+                        break;
+                    }
+                    const unsigned long long now = globaltimer_ns();
+                    if (t0 == 0) t0 = now;
+                    if (now - t0 > kWaitLimitNs) {
+                        record(ws_words, LB_ERR_TIMEOUT);
+                        ok = false;
+                        break;
+                    }
                 }
             }
+            if (!ok) break;
+            fence_proxy_async();
+            ld.issue(b, l);
+            last_use[b] = l;
         }
-        s_ok = ok;
     }
-    __syncthreads();
-    return s_ok != 0;
-}
-
-// Error exit: wait (bounded) for the bulk copies still in flight into this
-// CTA's buffers, so none lands after the CTA is gone.
-__device__ void drain(unsigned long long *bar, const int *pending_parity) {
-    if (threadIdx.x != 0) return;
+    // drain: the last issued use of each buffer has parity last_use & 1
     for (int b = 0; b < 4; ++b) {
-        if (pending_parity[b] < 0) continue;
         const unsigned long long t0 = globaltimer_ns();
-        while (!mbar_try_wait(bar + b, (unsigned)pending_parity[b]))
+        while (!mbar_try_wait(ld.full + b, (unsigned)(last_use[b] & 1)))
             if (globaltimer_ns() - t0 > kWaitLimitNs) break;
     }
 }
 
 __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params P) {
-    __shared__ __align__(8) unsigned long long bars[4];
+    __shared__ __align__(8) unsigned long long full[4], empty[4];
     __shared__ int s_last;
     unsigned *err = P.ws_words + kErrWord;
     if (sticky(P.ws_words)) return;
     if (*reinterpret_cast<const volatile unsigned long long *>(P.ws_words + kPlanWord) != P.plan) {
-        if (blockIdx.x == 0 && threadIdx.x == 0)
-            atomicCAS(err, 0u, static_cast<unsigned>(LB_ERR_PLAN));
+        if (blockIdx.x == 0 && threadIdx.x == 0) record(P.ws_words, LB_ERR_PLAN);
         return;
     }
     const int N = gridDim.x, c = blockIdx.x;
@@ -505,313 +657,303 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         s.k0 = 8 * u0;
         s.nkv = 8 * (u1 - u0);
     }
-    const int rows_d = 32 * s.nd, rows_f = 32 * s.nf;
-    const Offsets &o = P.o;
-    Loader ld{&P, s, bars};
-    // parity of the load outstanding in each buffer (-1: none)
-    int pending[4] = {-1, -1, -1, -1};
-
     if (threadIdx.x == 0) {
-        for (int b = 0; b < 4; ++b) mbar_init(bars + b, 1);
+        for (int b = 0; b < 4; ++b) {
+            mbar_init(full + b, 1);
+            mbar_init(empty + b, 1);
+        }
         fence_barrier_init();
     }
     __syncthreads();
-    if (threadIdx.x == 0) {
-        ld.issue_A(0);
-        ld.issue_B(0);
-        ld.issue_C(0);
-        ld.issue_D(0);
+    if (threadIdx.x >= kCT) {
+        if (threadIdx.x == kCT) producer(Loader{&P, s, full}, empty, P.ws_words);
+        return;
     }
-    for (int b = 0; b < 4; ++b) pending[b] = 0;
 
+    // ------------------------------------------------------------ compute warps
+    const int nd = s.nd, nf = s.nf, nkv = s.nkv;
+    const int rows_d = 32 * nd, rows_f = 32 * nf;
+    const Offsets &o = P.o;
     float *res = sm_f(o.res), *xs = sm_f(o.xs), *ys = sm_f(o.ys), *yq = sm_f(o.yq);
     float *tz = sm_f(o.tz);
-    for (int i = threadIdx.x; i < rows_d; i += blockDim.x)
+    for (int i = threadIdx.x; i < rows_d; i += kCT)
         res[i] = bf16_bits_to_float(P.x0[32 * s.dw0 + i]);
-
-    UJob uj[6];
-    VJob vj[6];
-    const int rq[2] = {P.r[LQ][0], P.r[LQ][1]};
-#define FAIL_EXIT()            \
-    do {                       \
-        drain(bars, pending);  \
-        return;                \
-    } while (0)
+    int nr[7];
+#pragma unroll
+    for (int k = 0; k < 7; ++k) nr[k] = P.r[k][0] + (P.np[k] > 1 ? P.r[k][1] : 0);
+    const int ssA = nr[LQ] + nr[LK] + nr[LV], ssC = nr[LG] + nr[LU];
+    const bool lead = threadIdx.x == 0;
+    // rank and presence of path p of linear k
+    auto rk = [&](int k, int p) { return p < P.np[k] ? P.r[k][p] : 0; };
+    auto release = [&](int b) {
+        csync();
+        if (lead) mbar_arrive(empty + b);
+    };
+    // stage 2 of down (both paths) on R_c into ys, from t in tz
+    auto down_rows = [&]() {
+        TJ T[2];
+        UJ U[2];
+        int tb = o.tables, off = 0;
+#pragma unroll
+        for (int p = 0; p < 2; ++p) {
+            const int r = rk(LD, p), R = r ? wordsR(r) : 1;
+            T[p] = TJ{tb, r ? 8 * R : 0, r, o.tz + 4 * off, o.a_ld[p], 1.f};
+            U[p] = UJ{o.a_Ud[p], o.a_hd[p], R, r ? rows_d : 0, tb, o.ys};
+            tb += r ? R * 1024 : 0;
+            off += r;
+        }
+        zero_f(ys, rows_d);
+        build_tables(T);
+        csync();
+        u_stage(U);
+        csync();
+    };
+#define FAIL_EXIT() return
 
     for (int l = 0; l < P.n_layers; ++l) {
-        const LinDesc *Ly = P.lin + 7 * l;
         unsigned long long *xA = P.xacc + (size_t)l * P.acc_layer + P.offA;
         unsigned long long *xB = P.xacc + (size_t)l * P.acc_layer + P.offB;
         unsigned long long *xC = P.xacc + (size_t)l * P.acc_layer + P.offC;
         unsigned long long *xD = P.xacc + (size_t)l * P.acc_layer + P.offD;
-        int nrq = 0, nrk = 0, nrv = 0;
-        for (int p = 0; p < P.np[LQ]; ++p) nrq += P.r[LQ][p];
-        for (int p = 0; p < P.np[LK]; ++p) nrk += P.r[LK][p];
-        for (int p = 0; p < P.np[LV]; ++p) nrv += P.r[LV][p];
-        int nro = 0, nrg = 0, nru = 0, nrd = 0;
-        for (int p = 0; p < P.np[LO]; ++p) nro += P.r[LO][p];
-        for (int p = 0; p < P.np[LG]; ++p) nrg += P.r[LG][p];
-        for (int p = 0; p < P.np[LU]; ++p) nru += P.r[LU][p];
-        for (int p = 0; p < P.np[LD]; ++p) nrd += P.r[LD][p];
-        const int ssA = nrq + nrk + nrv, ssC = nrg + nru;
+        const unsigned par = (unsigned)(l & 1);
 
         // ================= phase A: a = h + Down_{l-1}(m) on R_c; stage 1 of q, k, v
         if (l > 0) {
-            unsigned long long *xDp = P.xacc + (size_t)(l - 1) * P.acc_layer + P.offD;
-            if (!poll_decode(xDp, nrd, n_ctas, tz, P.ws_words)) FAIL_EXIT();
-            zero_stripe(P.xacc + (size_t)(l - 1) * P.acc_layer + P.offC, P.lenC);
+            if (!poll_decode(xD - P.acc_layer, nr[LD], n_ctas, tz, P.ws_words)) FAIL_EXIT();
+            zero_stripe(xC - P.acc_layer, P.lenC);
         }
-        if (!wait_buffer(bars + 0, (unsigned)(l & 1), P.ws_words)) FAIL_EXIT();
-        pending[0] = -1;
+        if (!wait_full(full + 0, par, P.ws_words)) FAIL_EXIT();
         if (l > 0) {
-            const LinDesc &Dn = P.lin[7 * (l - 1) + LD];
-            int tb = o.tables, off = 0, nj = 0;
-            for (int p = 0; p < Dn.n_paths; ++p) {
-                const int R = wordsR(Dn.r[p]);
-                build_tables(tb, 8 * R, tz + off, sm_u16(o.a_ld[p]), 1.f, Dn.r[p]);
-                uj[nj++] = UJob{o.a_Ud[p], o.a_hd[p], R, rows_d, tb, ys};
-                tb += R * 1024;
-                off += Dn.r[p];
-            }
-            zero_f(ys, rows_d);
-            __syncthreads();
-            u_stage(uj, nj);
-            __syncthreads();
-            for (int i = threadIdx.x; i < rows_d; i += blockDim.x) res[i] += ys[i];
+            down_rows();
+            for (int i = threadIdx.x; i < rows_d; i += kCT) res[i] += ys[i];
+            csync();
         }
-        __syncthreads();
         {
-            const float ss = block_sum_sq(res, rows_d);
-            if (threadIdx.x == 0) red_fix(xA + ssA, ss, P.fix_limit, err);
-            int tb = o.tables, nj = 0;
+            const float ss = sum_sq(res, rows_d);
+            if (lead) red_fix(xA + ssA, ss, P.fix_limit, err);
+            TJ T[6];
+            VJ V[6];
+            int tb = o.tables;
             unsigned long long *dst = xA;
-            for (int k = 0; k < 3; ++k) {
-                const LinDesc &L = Ly[k];
-                for (int p = 0; p < L.n_paths; ++p) {
-                    build_tables(tb, 8 * s.nd, res, sm_u16(o.a_g[k][p]), 1.f, rows_d);
-                    vj[nj++] = VJob{o.a_V[k][p], L.r[p], s.nd, tb, dst};
-                    tb += s.nd * 1024;
-                    dst += L.r[p];
+#pragma unroll
+            for (int k = 0; k < 3; ++k)
+#pragma unroll
+                for (int p = 0; p < 2; ++p) {
+                    const int r = rk(k, p);
+                    T[2 * k + p] = TJ{tb, r ? 8 * nd : 0, rows_d, o.res, o.a_g[k][p], 1.f};
+                    V[2 * k + p] = VJ{o.a_V[k][p], r, nd, tb, dst};
+                    tb += r ? nd * 1024 : 0;
+                    dst += r;
                 }
-            }
-            __syncthreads();
-            v_stage(vj, nj, P.fix_limit, err);
+            build_tables(T);
+            csync();
+            v_stage(V, P.fix_limit, err);
         }
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            fence_proxy_async();
-            ld.issue_A(l + 1);
-        }
-        pending[0] = (l + 1) & 1;
+        release(0);
 
         // ================= phase B: v rows for attention, stage 1 of o; then q, k, v out
         if (!poll_decode(xA, ssA + 1, n_ctas, tz, P.ws_words)) FAIL_EXIT();
-        if (l > 0) zero_stripe(P.xacc + (size_t)(l - 1) * P.acc_layer + P.offD, P.lenD);
-        if (!wait_buffer(bars + 1, (unsigned)(l & 1), P.ws_words)) FAIL_EXIT();
-        pending[1] = -1;
+        if (l > 0) zero_stripe(xD - P.acc_layer, P.lenD);
+        if (!wait_full(full + 1, par, P.ws_words)) FAIL_EXIT();
         {
             const float inv = rsqrtf(tz[ssA] / (float)P.d);
-            const LinDesc &V = Ly[LV], &O = Ly[LO];
-            float *attn = xs;
-            int tb = o.tables, nj = 0;
-            for (int p = 0, off = nrq + nrk; p < V.n_paths; off += V.r[p], ++p) {
-                const int R = wordsR(V.r[p]);
-                build_tables(tb, 8 * R, tz + off, sm_u16(o.b_lv[p]), inv, V.r[p]);
-                uj[nj++] = UJob{o.b_Uat[p], o.b_hat[p], R, rows_d, tb, attn};
-                tb += R * 1024;
-            }
-            const int tb_after_v = tb;
-            zero_f(attn, rows_d);
-            __syncthreads();
-            u_stage(uj, nj);
-            __syncthreads();
-            nj = 0;
-            unsigned long long *dst = xB;
-            for (int p = 0; p < O.n_paths; ++p) {
-                build_tables(tb, 8 * s.nd, attn, sm_u16(o.b_go[p]), 1.f, rows_d);
-                vj[nj++] = VJob{o.b_Vo[p], O.r[p], s.nd, tb, dst};
-                tb += s.nd * 1024;
-                dst += O.r[p];
-            }
-            __syncthreads();
-            v_stage(vj, nj, P.fix_limit, err);
-            // ---- off the critical path: q on R_c, k and v on K_c
-            const LinDesc &Q = Ly[LQ], &K = Ly[LK];
-            float *yk = ys, *yv = ys + s.nkv;
-            nj = 0;
-            int tb2 = tb;
-            for (int p = 0, off = 0; p < Q.n_paths; off += Q.r[p], ++p) {
-                const int R = wordsR(Q.r[p]);
-                build_tables(tb2, 8 * R, tz + off, sm_u16(o.b_lq[p]), inv, Q.r[p]);
-                uj[nj++] = UJob{o.b_Uq[p], o.b_hq[p], R, rows_d, tb2, yq};
-                tb2 += R * 1024;
-            }
-            for (int p = 0, off = nrq; p < K.n_paths; off += K.r[p], ++p) {
-                const int R = wordsR(K.r[p]);
-                build_tables(tb2, 8 * R, tz + off, sm_u16(o.b_lk[p]), inv, K.r[p]);
-                uj[nj++] = UJob{o.b_Uk[p], o.b_hk[p], R, s.nkv, tb2, yk};
-                tb2 += R * 1024;
-            }
-            // v on K_c reuses v's tables built above
-            for (int p = 0, tbv = o.tables; p < V.n_paths; ++p) {
-                const int R = wordsR(V.r[p]);
-                uj[nj++] = UJob{o.b_Uvk[p], o.b_hvk[p], R, s.nkv, tbv, yv};
-                tbv += R * 1024;
-            }
-            (void)tb_after_v;
-            zero_f(yq, rows_d);
-            zero_f(ys, 2 * s.nkv);
-            __syncthreads();
-            u_stage(uj, nj);
-            __syncthreads();
-            if (P.q_out)
-                for (int i = threadIdx.x; i < rows_d; i += blockDim.x)
-                    P.q_out[(size_t)l * P.d + 32 * s.dw0 + i] = yq[i];
-            if (P.kv_out)
-                for (int i = threadIdx.x; i < s.nkv; i += blockDim.x) {
-                    P.kv_out[((size_t)l * 2 + 0) * P.dkv + s.k0 + i] = yk[i];
-                    P.kv_out[((size_t)l * 2 + 1) * P.dkv + s.k0 + i] = yv[i];
+            int tb = o.tables;
+            const int tb_v = tb;
+            {
+                TJ T[2];
+                UJ U[2];
+#pragma unroll
+                for (int p = 0, off = nr[LQ] + nr[LK]; p < 2; ++p) {
+                    const int r = rk(LV, p), R = r ? wordsR(r) : 1;
+                    T[p] = TJ{tb, r ? 8 * R : 0, r, o.tz + 4 * off, o.b_lv[p], inv};
+                    U[p] = UJ{o.b_Uat[p], o.b_hat[p], R, r ? rows_d : 0, tb, o.xs};
+                    tb += r ? R * 1024 : 0;
+                    off += r;
                 }
+                zero_f(xs, rows_d);
+                build_tables(T);
+                csync();
+                u_stage(U);
+                csync();
+            }
+            {
+                TJ T[2];
+                VJ V[2];
+                unsigned long long *dst = xB;
+#pragma unroll
+                for (int p = 0; p < 2; ++p) {
+                    const int r = rk(LO, p);
+                    T[p] = TJ{tb, r ? 8 * nd : 0, rows_d, o.xs, o.b_go[p], 1.f};
+                    V[p] = VJ{o.b_Vo[p], r, nd, tb, dst};
+                    tb += r ? nd * 1024 : 0;
+                    dst += r;
+                }
+                build_tables(T);
+                csync();
+                v_stage(V, P.fix_limit, err);
+            }
+            // ---- off the critical path: q on R_c, k and v on K_c
+            {
+                TJ T[4];
+                UJ U[6];
+                int tbv = tb_v;
+#pragma unroll
+                for (int p = 0, off = 0; p < 2; ++p) {
+                    const int r = rk(LQ, p), R = r ? wordsR(r) : 1;
+                    T[p] = TJ{tb, r ? 8 * R : 0, r, o.tz + 4 * off, o.b_lq[p], inv};
+                    U[p] = UJ{o.b_Uq[p], o.b_hq[p], R, r ? rows_d : 0, tb, o.yq};
+                    tb += r ? R * 1024 : 0;
+                    off += r;
+                }
+#pragma unroll
+                for (int p = 0, off = nr[LQ]; p < 2; ++p) {
+                    const int r = rk(LK, p), R = r ? wordsR(r) : 1;
+                    T[2 + p] = TJ{tb, r ? 8 * R : 0, r, o.tz + 4 * off, o.b_lk[p], inv};
+                    U[2 + p] = UJ{o.b_Uk[p], o.b_hk[p], R, r ? nkv : 0, tb, o.ys};
+                    tb += r ? R * 1024 : 0;
+                    off += r;
+                }
+#pragma unroll
+                for (int p = 0; p < 2; ++p) {  // v on K_c reuses v's tables
+                    const int r = rk(LV, p), R = r ? wordsR(r) : 1;
+                    U[4 + p] = UJ{o.b_Uvk[p], o.b_hvk[p], R, r ? nkv : 0, tbv, o.ys + 4 * nkv};
+                    tbv += r ? R * 1024 : 0;
+                }
+                zero_f(yq, rows_d);
+                zero_f(ys, 2 * nkv);
+                build_tables(T);
+                csync();
+                u_stage(U);
+                csync();
+                if (P.q_out)
+                    for (int i = threadIdx.x; i < rows_d; i += kCT)
+                        P.q_out[(size_t)l * P.d + 32 * s.dw0 + i] = yq[i];
+                if (P.kv_out)
+                    for (int i = threadIdx.x; i < nkv; i += kCT) {
+                        P.kv_out[((size_t)l * 2 + 0) * P.dkv + s.k0 + i] = ys[i];
+                        P.kv_out[((size_t)l * 2 + 1) * P.dkv + s.k0 + i] = ys[nkv + i];
+                    }
+            }
         }
-        __syncthreads();
-        if (threadIdx.x == 0 && l + 1 < P.n_layers) {
-            fence_proxy_async();
-            ld.issue_B(l + 1);
-        }
-        pending[1] = l + 1 < P.n_layers ? ((l + 1) & 1) : -1;
+        release(1);
 
         // ================= phase C: h = a + O(attn) on R_c; stage 1 of gate, up
-        if (!poll_decode(xB, nro, n_ctas, tz, P.ws_words)) FAIL_EXIT();
+        if (!poll_decode(xB, nr[LO], n_ctas, tz, P.ws_words)) FAIL_EXIT();
         zero_stripe(xA, P.lenA);
-        if (!wait_buffer(bars + 2, (unsigned)(l & 1), P.ws_words)) FAIL_EXIT();
-        pending[2] = -1;
+        if (!wait_full(full + 2, par, P.ws_words)) FAIL_EXIT();
         {
-            const LinDesc &O = Ly[LO], &G = Ly[LG], &U = Ly[LU];
-            int tb = o.tables, nj = 0;
-            for (int p = 0, off = 0; p < O.n_paths; off += O.r[p], ++p) {
-                const int R = wordsR(O.r[p]);
-                build_tables(tb, 8 * R, tz + off, sm_u16(o.c_lo[p]), 1.f, O.r[p]);
-                uj[nj++] = UJob{o.c_Uo[p], o.c_ho[p], R, rows_d, tb, ys};
-                tb += R * 1024;
+            {
+                TJ T[2];
+                UJ U[2];
+                int tb = o.tables;
+#pragma unroll
+                for (int p = 0, off = 0; p < 2; ++p) {
+                    const int r = rk(LO, p), R = r ? wordsR(r) : 1;
+                    T[p] = TJ{tb, r ? 8 * R : 0, r, o.tz + 4 * off, o.c_lo[p], 1.f};
+                    U[p] = UJ{o.c_Uo[p], o.c_ho[p], R, r ? rows_d : 0, tb, o.ys};
+                    tb += r ? R * 1024 : 0;
+                    off += r;
+                }
+                zero_f(ys, rows_d);
+                build_tables(T);
+                csync();
+                u_stage(U);
+                csync();
             }
-            zero_f(ys, rows_d);
-            __syncthreads();
-            u_stage(uj, nj);
-            __syncthreads();
-            for (int i = threadIdx.x; i < rows_d; i += blockDim.x) res[i] += ys[i];
-            __syncthreads();
-            const float ss = block_sum_sq(res, rows_d);
-            if (threadIdx.x == 0) red_fix(xC + ssC, ss, P.fix_limit, err);
-            tb = o.tables;
-            nj = 0;
+            for (int i = threadIdx.x; i < rows_d; i += kCT) res[i] += ys[i];
+            csync();
+            const float ss = sum_sq(res, rows_d);
+            if (lead) red_fix(xC + ssC, ss, P.fix_limit, err);
+            TJ T[4];
+            VJ V[4];
+            int tb = o.tables;
             unsigned long long *dst = xC;
-            for (int p = 0; p < G.n_paths; ++p) {
-                build_tables(tb, 8 * s.nd, res, sm_u16(o.c_gg[p]), 1.f, rows_d);
-                vj[nj++] = VJob{o.c_Vg[p], G.r[p], s.nd, tb, dst};
-                tb += s.nd * 1024;
-                dst += G.r[p];
-            }
-            for (int p = 0; p < U.n_paths; ++p) {
-                build_tables(tb, 8 * s.nd, res, sm_u16(o.c_gu[p]), 1.f, rows_d);
-                vj[nj++] = VJob{o.c_Vu[p], U.r[p], s.nd, tb, dst};
-                tb += s.nd * 1024;
-                dst += U.r[p];
-            }
-            __syncthreads();
-            v_stage(vj, nj, P.fix_limit, err);
+#pragma unroll
+            for (int k = 0; k < 2; ++k)
+#pragma unroll
+                for (int p = 0; p < 2; ++p) {
+                    const int r = rk(LG + k, p);
+                    const int g = k ? o.c_gu[p] : o.c_gg[p], Vw = k ? o.c_Vu[p] : o.c_Vg[p];
+                    T[2 * k + p] = TJ{tb, r ? 8 * nd : 0, rows_d, o.res, g, 1.f};
+                    V[2 * k + p] = VJ{Vw, r, nd, tb, dst};
+                    tb += r ? nd * 1024 : 0;
+                    dst += r;
+                }
+            build_tables(T);
+            csync();
+            v_stage(V, P.fix_limit, err);
         }
-        __syncthreads();
-        if (threadIdx.x == 0 && l + 1 < P.n_layers) {
-            fence_proxy_async();
-            ld.issue_C(l + 1);
-        }
-        pending[2] = l + 1 < P.n_layers ? ((l + 1) & 1) : -1;
+        release(2);
 
         // ================= phase D: m = silu(gate) * up on F_c; stage 1 of down
         if (!poll_decode(xC, ssC + 1, n_ctas, tz, P.ws_words)) FAIL_EXIT();
         zero_stripe(xB, P.lenB);
-        if (!wait_buffer(bars + 3, (unsigned)(l & 1), P.ws_words)) FAIL_EXIT();
-        pending[3] = -1;
+        if (!wait_full(full + 3, par, P.ws_words)) FAIL_EXIT();
         {
             const float inv = rsqrtf(tz[ssC] / (float)P.d);
-            const LinDesc &G = Ly[LG], &U = Ly[LU], &D = Ly[LD];
-            float *yg = ys, *yu = ys + rows_f;
-            int tb = o.tables, nj = 0;
-            for (int p = 0, off = 0; p < G.n_paths; off += G.r[p], ++p) {
-                const int R = wordsR(G.r[p]);
-                build_tables(tb, 8 * R, tz + off, sm_u16(o.d_lg[p]), inv, G.r[p]);
-                uj[nj++] = UJob{o.d_Ug[p], o.d_hg[p], R, rows_f, tb, yg};
-                tb += R * 1024;
+            {
+                TJ T[4];
+                UJ U[4];
+                int tb = o.tables;
+#pragma unroll
+                for (int k = 0; k < 2; ++k)
+#pragma unroll
+                    for (int p = 0; p < 2; ++p) {
+                        const int r = rk(LG + k, p), R = r ? wordsR(r) : 1;
+                        const int off = (k ? nr[LG] : 0) + (p ? rk(LG + k, 0) : 0);
+                        const int lo16 = k ? o.d_lu[p] : o.d_lg[p];
+                        const int Uw = k ? o.d_Uu[p] : o.d_Ug[p], h = k ? o.d_hu[p] : o.d_hg[p];
+                        T[2 * k + p] = TJ{tb, r ? 8 * R : 0, r, o.tz + 4 * off, lo16, inv};
+                        U[2 * k + p] = UJ{Uw, h, R, r ? rows_f : 0, tb, o.ys + (k ? 4 * rows_f : 0)};
+                        tb += r ? R * 1024 : 0;
+                    }
+                zero_f(ys, 2 * rows_f);
+                build_tables(T);
+                csync();
+                u_stage(U);
+                csync();
             }
-            for (int p = 0, off = nrg; p < U.n_paths; off += U.r[p], ++p) {
-                const int R = wordsR(U.r[p]);
-                build_tables(tb, 8 * R, tz + off, sm_u16(o.d_lu[p]), inv, U.r[p]);
-                uj[nj++] = UJob{o.d_Uu[p], o.d_hu[p], R, rows_f, tb, yu};
-                tb += R * 1024;
-            }
-            zero_f(ys, 2 * rows_f);
-            __syncthreads();
-            u_stage(uj, nj);
-            __syncthreads();
-            for (int i = threadIdx.x; i < rows_f; i += blockDim.x) xs[i] = silu(yg[i]) * yu[i];
-            __syncthreads();
-            tb = o.tables;
-            nj = 0;
+            for (int i = threadIdx.x; i < rows_f; i += kCT) xs[i] = silu(ys[i]) * ys[rows_f + i];
+            csync();
+            TJ T[2];
+            VJ V[2];
+            int tb = o.tables;
             unsigned long long *dst = xD;
-            for (int p = 0; p < D.n_paths; ++p) {
-                build_tables(tb, 8 * s.nf, xs, sm_u16(o.d_gd[p]), 1.f, rows_f);
-                vj[nj++] = VJob{o.d_Vd[p], D.r[p], s.nf, tb, dst};
-                tb += s.nf * 1024;
-                dst += D.r[p];
+#pragma unroll
+            for (int p = 0; p < 2; ++p) {
+                const int r = rk(LD, p);
+                T[p] = TJ{tb, r ? 8 * nf : 0, rows_f, o.xs, o.d_gd[p], 1.f};
+                V[p] = VJ{o.d_Vd[p], r, nf, tb, dst};
+                tb += r ? nf * 1024 : 0;
+                dst += r;
             }
-            __syncthreads();
-            v_stage(vj, nj, P.fix_limit, err);
+            build_tables(T);
+            csync();
+            v_stage(V, P.fix_limit, err);
         }
-        __syncthreads();
-        if (threadIdx.x == 0 && l + 1 < P.n_layers) {
-            fence_proxy_async();
-            ld.issue_D(l + 1);
-        }
-        pending[3] = l + 1 < P.n_layers ? ((l + 1) & 1) : -1;
-        (void)rq;
+        release(3);
     }
 
     // ================= final: out = h + Down_{L-1}(m) on R_c
     {
         const int l = P.n_layers;
         unsigned long long *xDl = P.xacc + (size_t)(l - 1) * P.acc_layer + P.offD;
-        const LinDesc &Dn = P.lin[7 * (l - 1) + LD];
-        int nrd = 0;
-        for (int p = 0; p < Dn.n_paths; ++p) nrd += Dn.r[p];
-        if (!poll_decode(xDl, nrd, n_ctas, tz, P.ws_words)) FAIL_EXIT();
+        if (!poll_decode(xDl, nr[LD], n_ctas, tz, P.ws_words)) FAIL_EXIT();
         zero_stripe(P.xacc + (size_t)(l - 1) * P.acc_layer + P.offC, P.lenC);
-        if (!wait_buffer(bars + 0, (unsigned)(l & 1), P.ws_words)) FAIL_EXIT();
-        pending[0] = -1;
-        int tb = o.tables, off = 0, nj = 0;
-        for (int p = 0; p < Dn.n_paths; ++p) {
-            const int R = wordsR(Dn.r[p]);
-            build_tables(tb, 8 * R, tz + off, sm_u16(o.a_ld[p]), 1.f, Dn.r[p]);
-            uj[nj++] = UJob{o.a_Ud[p], o.a_hd[p], R, rows_d, tb, ys};
-            tb += R * 1024;
-            off += Dn.r[p];
-        }
-        zero_f(ys, rows_d);
-        __syncthreads();
-        u_stage(uj, nj);
-        __syncthreads();
-        for (int i = threadIdx.x; i < rows_d; i += blockDim.x)
-            P.out[32 * s.dw0 + i] = res[i] + ys[i];
+        if (!wait_full(full + 0, (unsigned)(l & 1), P.ws_words)) FAIL_EXIT();
+        down_rows();
+        for (int i = threadIdx.x; i < rows_d; i += kCT) P.out[32 * s.dw0 + i] = res[i] + ys[i];
         // The last CTA to finish has seen every other CTA's reads of the final
         // region: it clears that region and the counters for the next launch.
-        if (threadIdx.x == 0) {
+        if (lead) {
             __threadfence();
             s_last = atomicAdd(P.ws_words + kDoneWord, 1u) == n_ctas - 1;
         }
-        __syncthreads();
+        csync();
         if (s_last) {
             __threadfence();
-            for (int i = threadIdx.x; i < P.lenD; i += blockDim.x) xDl[i] = 0ull;
-            if (threadIdx.x == 0) P.ws_words[kDoneWord] = 0u;
+            for (int i = threadIdx.x; i < P.lenD; i += kCT) xDl[i] = 0ull;
+            if (lead) P.ws_words[kDoneWord] = 0u;
         }
     }
 #undef FAIL_EXIT
