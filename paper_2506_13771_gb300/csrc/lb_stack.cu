@@ -127,7 +127,7 @@ struct Offsets {
     int c_Uo[2], c_ho[2], c_lo[2], c_Vg[2], c_Vu[2], c_gg[2], c_gu[2];
     // phase D: stage 2 of gate, up, stage 1 of down
     int d_Ug[2], d_Uu[2], d_hg[2], d_hu[2], d_lg[2], d_lu[2], d_Vd[2], d_gd[2];
-    int tables, tz, res, xs, ys, yq;  // work areas
+    int tables, tz, res, xs, ys, yq, tsave;  // work areas
 };
 
 struct Params {
@@ -253,8 +253,10 @@ struct UJ {
 };
 
 // A task is 32 rows x a run of words of one job; its lanes (rows) read the
-// same 8 tables per word, so lookups are bank-conflict free.  Runs are split
-// when the jobs have fewer 32-row blocks than twice the compute warps.
+// same 8 tables per word, so lookups are bank-conflict free.  When the jobs
+// have fewer 32-row blocks than twice the compute warps, each row's words are
+// split into a power-of-two number of runs (shifts only: this runs on the
+// critical path of every phase).
 template <int NJ>
 __device__ __forceinline__ void u_stage(const UJ (&J)[NJ]) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -262,19 +264,21 @@ __device__ __forceinline__ void u_stage(const UJ (&J)[NJ]) {
     int blocks = 0;
 #pragma unroll
     for (int j = 0; j < NJ; ++j) blocks += (J[j].nrows + 31) >> 5;
-    const int split = blocks >= 2 * kCW ? 1 : (2 * kCW + blocks - 1) / max(blocks, 1);
-    int cum[NJ + 1], nch[NJ], wc[NJ];
+    int slog = 0;
+#pragma unroll
+    for (int k = 0; k < 5; ++k) slog += (blocks << slog) < 2 * kCW ? 1 : 0;
+    int cum[NJ + 1], nlog[NJ], wc[NJ];
     cum[0] = 0;
 #pragma unroll
     for (int j = 0; j < NJ; ++j) {
-        const int n0 = min(split, J[j].R);
-        wc[j] = (J[j].R + n0 - 1) / n0;
-        nch[j] = (J[j].R + wc[j] - 1) / wc[j];
-        cum[j + 1] = cum[j] + ((J[j].nrows + 31) >> 5) * nch[j];
+        const int R = J[j].R;
+        nlog[j] = min(slog, 31 - __clz(max(R, 1)));
+        wc[j] = (R + (1 << nlog[j]) - 1) >> nlog[j];
+        cum[j + 1] = cum[j] + (((J[j].nrows + 31) >> 5) << nlog[j]);
     }
     for (int task = warp; task < cum[NJ]; task += kCW) {
         int U = J[0].U, h = J[0].h, R = J[0].R, nrows = J[0].nrows, tb = J[0].tb, ys = J[0].ys;
-        int t = task, nc = nch[0], w_c = wc[0];
+        int t = task, nl = nlog[0], w_c = wc[0];
 #pragma unroll
         for (int j = 1; j < NJ; ++j)
             if (task >= cum[j]) {
@@ -285,10 +289,10 @@ __device__ __forceinline__ void u_stage(const UJ (&J)[NJ]) {
                 tb = J[j].tb;
                 ys = J[j].ys;
                 t = task - cum[j];
-                nc = nch[j];
+                nl = nlog[j];
                 w_c = wc[j];
             }
-        const int rb = t / nc, w0 = (t - rb * nc) * w_c;
+        const int rb = t >> nl, w0 = (t & ((1 << nl) - 1)) * w_c;
         const int w1 = min(w0 + w_c, R);
         const int row = 32 * rb + lane;
         if (row < nrows) {
@@ -374,23 +378,17 @@ __device__ __forceinline__ int csync_and(int pred) {
     return r;
 }
 
-// Sum of v over the compute threads, returned to each of them.
+// Sum of v over the compute threads, returned to each of them (one barrier:
+// the partials are read back before any later barrier lets them be rewritten).
 __device__ float csum(float v) {
     __shared__ float s_part[kCW];
-    __shared__ float s_total;
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    if (lane == 0) s_part[warp] = v;
+    if ((threadIdx.x & 31) == 0) s_part[threadIdx.x >> 5] = v;
     csync();
-    if (warp == 0) {
-        float t = lane < kCW ? s_part[lane] : 0.f;
-        for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
-        if (lane == 0) s_total = t;
-    }
-    csync();
-    const float total = s_total;
-    csync();
-    return total;
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < kCW; ++w) t += s_part[w];
+    return t;
 }
 
 __device__ __forceinline__ float sum_sq(const float *v, int n) {
@@ -792,31 +790,37 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
                 csync();
                 v_stage(V, P.fix_limit, err);
             }
-            // ---- off the critical path: q on R_c, k and v on K_c
+            // ---- off the critical path, while exchange B is in flight:
+            //      k and v on K_c, and path 0 of q on R_c (path 1 of q runs
+            //      after exchange C is sent, from the saved t and rms)
             {
-                TJ T[4];
-                UJ U[6];
+                const int rq1 = rk(LQ, 1);
+                if (rq1) {
+                    float *sv = sm_f(o.tsave);
+                    for (int i = threadIdx.x; i < rq1; i += kCT) sv[i] = tz[rk(LQ, 0) + i];
+                    if (lead) sv[rq1] = inv;
+                }
+                TJ T[3];
+                UJ U[5];
                 int tbv = tb_v;
-#pragma unroll
-                for (int p = 0, off = 0; p < 2; ++p) {
-                    const int r = rk(LQ, p), R = r ? wordsR(r) : 1;
-                    T[p] = TJ{tb, r ? 8 * R : 0, r, o.tz + 4 * off, o.b_lq[p], inv};
-                    U[p] = UJ{o.b_Uq[p], o.b_hq[p], R, r ? rows_d : 0, tb, o.yq};
-                    tb += r ? R * 1024 : 0;
-                    off += r;
+                {
+                    const int r = rk(LQ, 0), R = wordsR(r);
+                    T[0] = TJ{tb, 8 * R, r, o.tz, o.b_lq[0], inv};
+                    U[0] = UJ{o.b_Uq[0], o.b_hq[0], R, rows_d, tb, o.yq};
+                    tb += R * 1024;
                 }
 #pragma unroll
                 for (int p = 0, off = nr[LQ]; p < 2; ++p) {
                     const int r = rk(LK, p), R = r ? wordsR(r) : 1;
-                    T[2 + p] = TJ{tb, r ? 8 * R : 0, r, o.tz + 4 * off, o.b_lk[p], inv};
-                    U[2 + p] = UJ{o.b_Uk[p], o.b_hk[p], R, r ? nkv : 0, tb, o.ys};
+                    T[1 + p] = TJ{tb, r ? 8 * R : 0, r, o.tz + 4 * off, o.b_lk[p], inv};
+                    U[1 + p] = UJ{o.b_Uk[p], o.b_hk[p], R, r ? nkv : 0, tb, o.ys};
                     tb += r ? R * 1024 : 0;
                     off += r;
                 }
 #pragma unroll
                 for (int p = 0; p < 2; ++p) {  // v on K_c reuses v's tables
                     const int r = rk(LV, p), R = r ? wordsR(r) : 1;
-                    U[4 + p] = UJ{o.b_Uvk[p], o.b_hvk[p], R, r ? nkv : 0, tbv, o.ys + 4 * nkv};
+                    U[3 + p] = UJ{o.b_Uvk[p], o.b_hvk[p], R, r ? nkv : 0, tbv, o.ys + 4 * nkv};
                     tbv += r ? R * 1024 : 0;
                 }
                 zero_f(yq, rows_d);
@@ -825,17 +829,16 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
                 csync();
                 u_stage(U);
                 csync();
-                if (P.q_out)
-                    for (int i = threadIdx.x; i < rows_d; i += kCT)
-                        P.q_out[(size_t)l * P.d + 32 * s.dw0 + i] = yq[i];
                 if (P.kv_out)
                     for (int i = threadIdx.x; i < nkv; i += kCT) {
                         P.kv_out[((size_t)l * 2 + 0) * P.dkv + s.k0 + i] = ys[i];
                         P.kv_out[((size_t)l * 2 + 1) * P.dkv + s.k0 + i] = ys[nkv + i];
                     }
+                if (!rq1 && P.q_out)
+                    for (int i = threadIdx.x; i < rows_d; i += kCT)
+                        P.q_out[(size_t)l * P.d + 32 * s.dw0 + i] = yq[i];
             }
         }
-        release(1);
 
         // ================= phase C: h = a + O(attn) on R_c; stage 1 of gate, up
         if (!poll_decode(xB, nr[LO], n_ctas, tz, P.ws_words)) FAIL_EXIT();
@@ -883,6 +886,21 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
             csync();
             v_stage(V, P.fix_limit, err);
         }
+        // ---- off the critical path, while exchange C is in flight: path 1 of q
+        if (rk(LQ, 1)) {
+            csync();
+            const int r = rk(LQ, 1), R = wordsR(r);
+            TJ T[1] = {TJ{o.tables, 8 * R, r, o.tsave, o.b_lq[1], sm_f(o.tsave)[r]}};
+            UJ U[1] = {UJ{o.b_Uq[1], o.b_hq[1], R, rows_d, o.tables, o.yq}};
+            build_tables(T);
+            csync();
+            u_stage(U);
+            csync();
+            if (P.q_out)
+                for (int i = threadIdx.x; i < rows_d; i += kCT)
+                    P.q_out[(size_t)l * P.d + 32 * s.dw0 + i] = yq[i];
+        }
+        release(1);
         release(2);
 
         // ================= phase D: m = silu(gate) * up on F_c; stage 1 of down
@@ -1110,6 +1128,7 @@ SmemPlan smem_plan(const lb_linear *lin, const StackShape &sh, int N) {
     o.xs = take(4 * 32 * std::max(nd, nf));
     o.ys = take(4 * std::max(32 * nd, std::max(2 * nkv, 2 * 32 * nf)));
     o.yq = take(4 * 32 * nd);
+    o.tsave = take(4 * (lin[LQ].path[lin[LQ].n_paths - 1].r + 4));
     S.bytes = up(at, 128);
     return S;
 }
