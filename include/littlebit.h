@@ -160,6 +160,30 @@ lb_status littlebit_stack_forward(const lb_linear *lin, int32_t n_layers, int32_
                                   const uint16_t *x0, float *out, float *q_out, float *kv_out,
                                   void *ws, size_t ws_bytes, lb_stream_t stream);
 
+/* The forward of littlebit_linear_forward for callers that cannot allocate
+ * device memory.  The paper has no counterpart: this exists for hosts such as
+ * serving loops and plugins whose device memory is owned by someone else or
+ * whose hot path may not call cudaMalloc (it can synchronise the whole device
+ * and take unbounded time), so they cannot provide a workspace.
+ *
+ * Same arguments and results as littlebit_linear_forward minus the
+ * workspace; it runs the two-launch CUDA-core path (any T).  Its scratch is
+ * a 256 KiB array compiled into the library, held by every GPU that loads
+ * the library until the process exits, and shared by all calls: it allocates
+ * nothing and calls no allocating routine.
+ *   - Limit: T * (sum of the paths' ranks) <= 65536 fp32 values; a larger
+ *     request returns LB_ERR_WORKSPACE without launching anything.
+ *   - The first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress, with that device current); make that first call
+ *     before any stream capture.  Later calls reuse the address.
+ *   - Each call clears the part of the array it uses before adding into it,
+ *     but the array keeps the last call's contents afterwards.  Calls whose
+ *     kernels overlap on the GPU (different streams, or different host
+ *     threads, without ordering between them) race on the shared array:
+ *     order them, e.g. issue them on one stream. */
+lb_status littlebit_linear_forward_noalloc(const lb_linear *L, const uint16_t *x, int64_t T,
+                                           void *y, int32_t y_dtype, lb_stream_t stream);
+
 /* Synchronises the stream, reads the workspace's sticky error word, clears
  * it, and returns LB_OK or the recorded error (LB_ERR_TIMEOUT, LB_ERR_PLAN). */
 lb_status littlebit_poll_error(void *ws, lb_stream_t stream);

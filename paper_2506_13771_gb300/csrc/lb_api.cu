@@ -129,6 +129,8 @@ bool use_decode(const lb_linear &, int64_t T) { return T == 1; }
 
 }  // namespace
 
+lb_status lb::validate_linear(const lb_linear *L) { return check_linear(L); }
+
 extern "C" {
 
 const char *littlebit_status_string(lb_status s) {

@@ -11,6 +11,9 @@ namespace lb {
 
 struct LinDesc;
 
+// Shape and pointer checks of one linear, as littlebit_linear_forward does them.
+lb_status validate_linear(const lb_linear *L);
+
 // Two-launch CUDA-core path for any T (lb_generic.cu).  t_acc: workspace
 // floats, generic_ws_floats() of them.
 size_t generic_ws_floats(const lb_linear &L, int64_t T);

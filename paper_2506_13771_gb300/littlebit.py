@@ -24,7 +24,7 @@ LB_PACK_U, LB_PACK_V = 0, 1
 EXPORTED = ["littlebit_status_string", "littlebit_pack", "littlebit_workspace_size",
             "littlebit_linear_forward", "littlebit_stack_workspace_size",
             "littlebit_stack_prepare", "littlebit_stack_forward", "littlebit_poll_error",
-            "littlebit_selftest_wait_timeout"]
+            "littlebit_selftest_wait_timeout", "littlebit_linear_forward_noalloc"]
 
 
 class LittleBitError(RuntimeError):
@@ -84,6 +84,9 @@ def lib(path: str | None = None):
         L.littlebit_poll_error.restype = ctypes.c_int
         L.littlebit_selftest_wait_timeout.argtypes = [vp, vp]
         L.littlebit_selftest_wait_timeout.restype = ctypes.c_int
+        L.littlebit_linear_forward_noalloc.argtypes = [ctypes.POINTER(lb_linear), vp, i64, vp,
+                                                       i32, vp]
+        L.littlebit_linear_forward_noalloc.restype = ctypes.c_int
         if path is None:
             _lib = L
         return L
@@ -267,3 +270,19 @@ def selftest_wait_timeout(ws: torch.Tensor, stream=None) -> None:
     """Launch the bounded-wait diagnostic (records LB_ERR_TIMEOUT in ws)."""
     _check(lib().littlebit_selftest_wait_timeout(ws.data_ptr(), _stream(stream)),
            "littlebit_selftest_wait_timeout")
+
+
+def linear_forward_noalloc(L: DeviceLinear, x: torch.Tensor, out_dtype=torch.bfloat16,
+                           y: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """Y = X W^T without a workspace: the library's built-in scratch is used
+    (for callers that cannot allocate device memory; see littlebit.h)."""
+    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.shape[1] == L.d_in
+    x = x.contiguous()
+    T = x.shape[0]
+    if y is None:
+        y = torch.empty((T, L.d_out), dtype=out_dtype, device=x.device)
+    y_dtype = LB_OUT_FP32 if y.dtype == torch.float32 else LB_OUT_BF16
+    _check(lib().littlebit_linear_forward_noalloc(ctypes.byref(L.c), x.data_ptr(), T, y.data_ptr(),
+                                                  y_dtype, _stream(stream)),
+           "littlebit_linear_forward_noalloc")
+    return y
