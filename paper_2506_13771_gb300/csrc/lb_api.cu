@@ -127,6 +127,13 @@ unsigned long long stack_fingerprint(const lb_linear *lin, int32_t n_layers, int
 // One token goes through the single-launch persistent kernel.
 bool use_decode(const lb_linear &, int64_t T) { return T == 1; }
 
+// From this many tokens on, the layer is a dense contraction worth the
+// tensor cores (tcgen05, 128-token tiles).
+constexpr int64_t kPrefillMinTokens = 32;
+bool use_prefill(const lb_linear &L, int64_t T) {
+    return T >= kPrefillMinTokens && lb::prefill_supported(L, T);
+}
+
 }  // namespace
 
 lb_status lb::validate_linear(const lb_linear *L) { return check_linear(L); }
@@ -163,7 +170,9 @@ size_t littlebit_workspace_size(const lb_linear *L, int64_t T) {
     // the decode path falls back to the two-launch path when its grid cannot
     // be co-resident, so size for both
     if (use_decode(*L, T) && lb::decode_ws_floats(*L) > floats) floats = lb::decode_ws_floats(*L);
-    return kWsHeader + ((floats * sizeof(float) + 255) & ~(size_t)255);
+    size_t bytes = (floats * sizeof(float) + 255) & ~(size_t)255;
+    if (use_prefill(*L, T) && lb::prefill_ws_bytes(*L, T) > bytes) bytes = lb::prefill_ws_bytes(*L, T);
+    return kWsHeader + bytes;
 }
 
 lb_status littlebit_linear_forward(const lb_linear *L, const uint16_t *x, int64_t T, void *y,
@@ -189,6 +198,7 @@ lb_status littlebit_linear_forward(const lb_linear *L, const uint16_t *x, int64_
         if (e != cudaErrorCooperativeLaunchTooLarge) return from_cuda(e);
         cudaGetLastError();  // grid cannot be co-resident here: take the two-launch path
     }
+    if (use_prefill(*L, T)) return from_cuda(lb::launch_prefill(*L, x, T, y, fp32, words, data, s));
     return from_cuda(lb::launch_generic(*L, x, T, y, fp32, data, sms, s));
 }
 

@@ -45,6 +45,13 @@ cudaError_t launch_stack(const lb_linear *lin, int n_layers, const StackShape &s
                          float *kv_out, unsigned *ws_words, char *ws_after_header, int num_sms,
                          cudaStream_t s);
 
+// Many-token path on the tensor cores (lb_prefill.cu): stage 1 writes z
+// (fp16 [T][sum r]) into z_ws, stage 2 reads it.
+bool prefill_supported(const lb_linear &L, int64_t T);
+size_t prefill_ws_bytes(const lb_linear &L, int64_t T);
+cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, void *y, int y_fp32,
+                           unsigned *ws_words, void *z_ws, cudaStream_t s);
+
 // Bounded-wait diagnostic (lb_persistent.cu).
 cudaError_t launch_wait_timeout(unsigned *ws_words, cudaStream_t s);
 

@@ -1,0 +1,490 @@
+// lb_prefill.cu -- many-token LittleBit forward on the 5th-generation tensor
+// cores (tcgen05, fp16 operands, fp32 accumulators in TMEM).
+//
+// Prop. 1 (LittleBit, arXiv 2506.13771) as two dense contractions:
+//   stage 1   z = fp16( l . (X diag(g) V_sign) )     [T x N1],  N1 = sum_p r_p
+//   stage 2   Y = z [diag(h_p) U_p,sign]_p^T          [T x d_out]  (Eq. 6 sum
+//             over the paths is the K dimension of this GEMM)
+// The sign factors never exist in memory as numbers: each CTA unpacks the
+// +-1 bits of its K-slice into shared memory as +-g (stage 1) or +-h (stage
+// 2) fp16 values, in the tensor cores' 128-byte-swizzled K-major layout.  X
+// arrives by TMA (bf16) and is converted to fp16 in shared memory (exact for
+// |x| < 65504); z goes to the workspace as fp16 and comes back by TMA.
+//
+// One CTA = 4 warps computes a 128 x BN tile (BN <= 256 fp32 TMEM columns).
+// K runs in 64-element stages through a 4-deep shared-memory ring: the TMA
+// of stage k+2 and the unpacking of stage k overlap the MMAs of stage k-1.
+// Thread 0 issues the TMA copies and the MMAs (tcgen05.mma, one thread per
+// CTA); tcgen05.commit releases a stage.  Every wait is bounded (about one
+// second); on a timeout the CTA records LB_ERR_TIMEOUT, waits for its own
+// copies and MMAs in flight, frees its TMEM and returns.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
+#include "lb_common.cuh"
+#include "lb_kernels.h"
+
+namespace lb {
+
+namespace {
+
+constexpr int BM = 128;       // tokens per tile (MMA M)
+constexpr int BN = 256;       // columns per tile (MMA N)
+constexpr int BK = 64;        // K per stage: 64 fp16 = one 128-byte swizzle row
+constexpr int STAGES = 4;
+constexpr int kThreads = 128;
+constexpr int A_BYTES = BM * BK * 2;   // 16 KB
+constexpr int B_BYTES = BN * BK * 2;   // 32 KB
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024;  // + alignment slack
+
+extern __shared__ __align__(1024) unsigned char p_smem[];
+
+// ---------------------------------------------------------------- PTX helpers
+
+__device__ __forceinline__ uint32_t su32(const void *p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ void mb_init(uint64_t *b, unsigned n) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(b)), "r"(n) : "memory");
+}
+__device__ __forceinline__ void mb_expect_tx(uint64_t *b, unsigned bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(b)),
+                 "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ bool mb_try(uint64_t *b, unsigned parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(su32(b)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Bounded wait (every calling thread); false after the limit.
+__device__ bool mb_wait(uint64_t *b, unsigned parity) {
+    if (mb_try(b, parity)) return true;
+    const unsigned long long t0 = globaltimer_ns();
+    while (!mb_try(b, parity))
+        if (globaltimer_ns() - t0 > kWaitLimitNs) return false;
+    return true;
+}
+
+__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, int x, int y,
+                                            uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];" ::"r"(su32(dst)),
+        "l"(map), "r"(x), "r"(y), "r"(su32(bar))
+        : "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row groups
+// 1024 bytes apart (stride byte offset), descriptor version 1.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFF) >> 4);      // start address
+    d |= (uint64_t)1 << 16;                        // leading byte offset (unused when swizzled)
+    d |= (uint64_t)(1024 >> 4) << 32;              // stride byte offset
+    d |= (uint64_t)1 << 46;                        // version
+    d |= (uint64_t)2 << 61;                        // 128-byte swizzle
+    return d;
+}
+
+// Instruction descriptor, kind::f16: D f32, A f16, B f16, both K-major, M x N.
+__host__ __device__ constexpr uint32_t instr_desc(int M, int N) {
+    return (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_f16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                        uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint64_t *bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+            su32(bar))
+        : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// 32 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+        "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
+          "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+          "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
+          "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// Byte offset of the 16-byte chunk c (0..7) of row n in a K-major tile with
+// 128-byte rows, 128-byte swizzle (chunk index XOR row mod 8).
+__device__ __forceinline__ int sw128(int n, int c) {
+    return (n >> 3) * 1024 + (n & 7) * 128 + ((c ^ (n & 7)) << 4);
+}
+
+// 8 fp16 values: scale[k] with its sign flipped where bit k of bits is set.
+__device__ __forceinline__ uint4 signed8(uint32_t bits, uint4 mag) {
+    // bit 2i -> bit 15 of word i, bit 2i+1 -> bit 31 of word i
+    uint4 r;
+    r.x = mag.x ^ (((bits << 15) & 0x8000u) | ((bits << 30) & 0x80000000u));
+    r.y = mag.y ^ (((bits << 13) & 0x8000u) | ((bits << 28) & 0x80000000u));
+    r.z = mag.z ^ (((bits << 11) & 0x8000u) | ((bits << 26) & 0x80000000u));
+    r.w = mag.w ^ (((bits << 9) & 0x8000u) | ((bits << 24) & 0x80000000u));
+    return r;
+}
+
+struct PrefillParams {
+    LinDesc L;
+    int T, N1, d_out;
+    int bn1;           // stage-1 tile width: N1 if N1 <= 256, else 256
+    int off1;          // column offset of path 1 in the N1 concatenation (= r_0)
+    uint16_t *z;       // stage 1 output / stage 2 input, fp16 [T][N1]
+    void *y;           // stage 2 output [T][d_out]
+    int y_fp32;
+    unsigned *ws_words;
+};
+
+// Fill B stage with the +-scale values of K-chunk kc for columns [n0, n0+BN).
+template <bool STAGE1>
+__device__ __forceinline__ void unpack_b(const PrefillParams &P, unsigned char *Bs, int kc,
+                                         int n0, int bn) {
+    // each item = one 16-byte chunk (8 K values) of one B row
+    for (int item = threadIdx.x; item < bn * 8; item += kThreads) {
+        const int n = item >> 3, c = item & 7;
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (STAGE1) {
+            const int col = n0 + n;
+            if (col < P.N1) {
+                const int p = col >= P.off1 ? 1 : 0, j = col - (p ? P.off1 : 0);
+                const int r = P.L.r[p];
+                // inputs 64kc + 8c .. +7 live in word 2kc + (c >> 2), bits 8(c&3)..
+                const uint32_t word = __ldg(P.L.v[p] + (size_t)(2 * kc + (c >> 2)) * r + j);
+                const uint32_t bits = (word >> (8 * (c & 3))) & 0xffu;
+                const uint4 mag =
+                    __ldg(reinterpret_cast<const uint4 *>(P.L.g[p] + 64 * kc + 8 * c));
+                v = signed8(bits, mag);
+            }
+        } else {
+            const int o = n0 + n;
+            if (o < P.d_out) {
+                const int k0 = 64 * kc;
+                const int p = k0 >= P.off1 ? 1 : 0, j0 = k0 - (p ? P.off1 : 0);
+                const int R = (P.L.r[p] + 31) >> 5;
+                const uint32_t word = __ldg(P.L.u[p] + (size_t)o * R + (j0 >> 5) + (c >> 2));
+                const uint32_t bits = (word >> (8 * (c & 3))) & 0xffu;
+                const uint32_t hb = __ldg(P.L.h[p] + o);
+                const uint32_t hh = hb | (hb << 16);
+                v = signed8(bits, make_uint4(hh, hh, hh, hh));
+            }
+        }
+        *reinterpret_cast<uint4 *>(Bs + sw128(n, c)) = v;
+    }
+}
+
+// In-place bf16 -> fp16 of the A stage (layout-preserving, elementwise).
+__device__ __forceinline__ void convert_a(unsigned char *As) {
+    for (int i = threadIdx.x; i < A_BYTES / 16; i += kThreads) {
+        uint4 *p = reinterpret_cast<uint4 *>(As) + i;
+        uint4 u = *p;
+        uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float lo = __uint_as_float(w[k] << 16), hi = __uint_as_float(w[k] & 0xffff0000u);
+            const __half2 h = __floats2half2_rn(lo, hi);
+            w[k] = *reinterpret_cast<const uint32_t *>(&h);
+        }
+        *p = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+
+template <bool STAGE1>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_prefill(const __grid_constant__ CUtensorMap amap, const __grid_constant__ PrefillParams P) {
+    __shared__ __align__(8) uint64_t full[STAGES], done[STAGES];
+    __shared__ uint32_t s_tmem;
+    __shared__ int s_fail;
+    unsigned char *smem = reinterpret_cast<unsigned char *>(
+        (reinterpret_cast<uintptr_t>(p_smem) + 1023) & ~(uintptr_t)1023);
+    const int m0 = blockIdx.x * BM, n0 = blockIdx.y * BN;
+    const int K = STAGE1 ? P.L.d_in : P.N1;
+    const int KC = K / BK;
+    const int warp = threadIdx.x >> 5;
+    const bool t0 = threadIdx.x == 0;
+    const int bn = STAGE1 ? P.bn1 : BN;
+    if (ld_relaxed_gpu(P.ws_words + kErrWord) != 0u) return;
+
+    if (t0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mb_init(full + s, 1);
+            mb_init(done + s, 1);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        s_fail = 0;
+    }
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         su32(&s_tmem)),
+                     "r"(BN)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = s_tmem;
+    const uint32_t idesc = instr_desc(BM, bn);
+
+    auto A_of = [&](int s) { return smem + s * STAGE_BYTES; };
+    auto B_of = [&](int s) { return smem + s * STAGE_BYTES + A_BYTES; };
+    int loads_issued = 0, mmas_issued = 0;  // K-chunks loaded / multiplied (thread 0)
+    auto issue_load = [&](int kc) {
+        const int s = kc % STAGES;
+        mb_expect_tx(full + s, A_BYTES);
+        tma_load_2d(A_of(s), &amap, kc * BK, m0, full + s);
+    };
+    if (t0) {
+        for (int kc = 0; kc < 2 && kc < KC; ++kc) issue_load(kc);
+        loads_issued = KC < 2 ? KC : 2;
+    }
+
+    bool ok = true;
+    for (int kc = 0; kc < KC && ok; ++kc) {
+        const int s = kc % STAGES;
+        // refill two stages ahead once the MMAs that last read that stage finished
+        if (t0 && kc + 2 < KC) {
+            const int kr = kc + 2;
+            if (kr >= STAGES && !mb_wait(done + (kr % STAGES), (unsigned)(((kr / STAGES) - 1) & 1)))
+                s_fail = 1;
+            else {
+                issue_load(kr);
+                ++loads_issued;
+            }
+        }
+        __syncthreads();
+        if (s_fail) {
+            ok = false;
+            break;
+        }
+        unpack_b<STAGE1>(P, B_of(s), kc, n0, bn);
+        if (!mb_wait(full + s, (unsigned)((kc / STAGES) & 1))) s_fail = 1;
+        __syncthreads();
+        if (s_fail) {
+            ok = false;
+            break;
+        }
+        if (STAGE1) convert_a(A_of(s));
+        fence_proxy_async_smem();
+        __syncthreads();
+        if (t0) {
+            tc_fence_after();
+            const uint32_t a0 = su32(A_of(s)), b0 = su32(B_of(s));
+#pragma unroll
+            for (int k = 0; k < BK / 16; ++k)
+                mma_f16(tmem, smem_desc(a0 + 32 * k), smem_desc(b0 + 32 * k), idesc,
+                        (kc > 0 || k > 0) ? 1u : 0u);
+            mma_commit(done + s);
+            ++mmas_issued;
+        }
+    }
+    // wait for the last MMA (the accumulator is complete when its commit lands)
+    if (ok && KC > 0) {
+        const int kl = KC - 1;
+        if (!mb_wait(done + (kl % STAGES), (unsigned)((kl / STAGES) & 1))) ok = false;
+    }
+    if (!ok) {
+        if (t0) {
+            atomicCAS(P.ws_words + kErrWord, 0u, static_cast<unsigned>(LB_ERR_TIMEOUT));
+            // let every issued copy and MMA land before the CTA goes away: for
+            // each stage wait for the phase of its last issued use
+            for (int kc = loads_issued - STAGES; kc < loads_issued; ++kc)
+                if (kc >= 0) mb_wait(full + kc % STAGES, (unsigned)((kc / STAGES) & 1));
+            for (int kc = mmas_issued - STAGES; kc < mmas_issued; ++kc)
+                if (kc >= 0) mb_wait(done + kc % STAGES, (unsigned)((kc / STAGES) & 1));
+        }
+        __syncthreads();
+    } else {
+        tc_fence_after();
+        // epilogue: warp w reads TMEM lanes 32w..32w+31 = tile rows
+        const int row = m0 + 32 * warp + (threadIdx.x & 31);
+        const uint32_t lane_base = tmem + ((uint32_t)(32 * warp) << 16);
+        for (int cb = 0; cb < bn; cb += 32) {
+            float v[32];
+            tmem_ld32(lane_base + cb, v);
+            if (row >= P.T) continue;
+            if (STAGE1) {
+                // z = l . t as fp16
+                uint32_t packed[16];
+#pragma unroll
+                for (int i = 0; i < 32; i += 2) {
+                    float a = 0.f, b = 0.f;
+                    const int c0 = n0 + cb + i;
+                    if (c0 < P.N1) {
+                        const int p = c0 >= P.off1 ? 1 : 0;
+                        const int j = c0 - (p ? P.off1 : 0);
+                        a = v[i] * half_bits_to_float(__ldg(P.L.l[p] + j));
+                        b = v[i + 1] * half_bits_to_float(__ldg(P.L.l[p] + j + 1));
+                    }
+                    const __half2 h = __floats2half2_rn(a, b);
+                    packed[i >> 1] = *reinterpret_cast<const uint32_t *>(&h);
+                }
+                if (n0 + cb < P.N1) {
+                    uint4 *dst = reinterpret_cast<uint4 *>(P.z + (size_t)row * P.N1 + n0 + cb);
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        dst[q] = make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2],
+                                            packed[4 * q + 3]);
+                }
+            } else {
+                const int o0 = n0 + cb;
+                if (P.y_fp32) {
+                    float *dst = static_cast<float *>(P.y) + (size_t)row * P.d_out + o0;
+                    if (o0 + 32 <= P.d_out && (P.d_out & 3) == 0) {
+#pragma unroll
+                        for (int q = 0; q < 8; ++q)
+                            reinterpret_cast<float4 *>(dst)[q] =
+                                make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                    } else {
+                        for (int i = 0; i < 32 && o0 + i < P.d_out; ++i) dst[i] = v[i];
+                    }
+                } else {
+                    uint16_t *dst = static_cast<uint16_t *>(P.y) + (size_t)row * P.d_out + o0;
+                    if (o0 + 32 <= P.d_out && (P.d_out & 7) == 0) {
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            uint32_t w[4];
+#pragma unroll
+                            for (int e = 0; e < 4; ++e)
+                                w[e] = (uint32_t)float_to_bf16_bits(v[8 * q + 2 * e]) |
+                                       ((uint32_t)float_to_bf16_bits(v[8 * q + 2 * e + 1]) << 16);
+                            reinterpret_cast<uint4 *>(dst)[q] = make_uint4(w[0], w[1], w[2], w[3]);
+                        }
+                    } else {
+                        for (int i = 0; i < 32 && o0 + i < P.d_out; ++i)
+                            dst[i] = float_to_bf16_bits(v[i]);
+                    }
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                     "r"(BN)
+                     : "memory");
+}
+
+// ---------------------------------------------------------------- host side
+
+PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+std::once_flag g_encode_once;
+
+bool encoder() {
+    std::call_once(g_encode_once, [] {
+        void *fn = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            g_encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    });
+    return g_encode != nullptr;
+}
+
+// 2-D map over a row-major [rows][cols] 16-bit matrix, box BK x BM, 128B swizzle,
+// out-of-range rows read as zero.
+bool make_map(CUtensorMap *m, const void *base, CUtensorMapDataType dt, int64_t rows,
+              int64_t cols) {
+    const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    const cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+    const cuuint32_t box[2] = {BK, BM};
+    const cuuint32_t estr[2] = {1, 1};
+    return g_encode(m, dt, 2, const_cast<void *>(base), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+bool prefill_supported(const lb_linear &L, int64_t T) {
+    if (T < 1 || T > (1LL << 30)) return false;
+    if (L.d_in % BK != 0) return false;
+    for (int p = 0; p < L.n_paths; ++p)
+        if (L.path[p].r % BK != 0) return false;
+    return encoder();
+}
+
+size_t prefill_ws_bytes(const lb_linear &L, int64_t T) {
+    size_t n1 = 0;
+    for (int p = 0; p < L.n_paths; ++p) n1 += (size_t)L.path[p].r;
+    return ((size_t)T * n1 * 2 + 255) & ~(size_t)255;
+}
+
+cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, void *y, int y_fp32,
+                           unsigned *ws_words, void *z_ws, cudaStream_t s) {
+    if (!encoder()) return cudaErrorNotSupported;
+    PrefillParams P{};
+    P.L = make_desc(L);
+    P.T = (int)T;
+    P.N1 = 0;
+    for (int p = 0; p < L.n_paths; ++p) P.N1 += L.path[p].r;
+    P.off1 = L.path[0].r;
+    P.bn1 = P.N1 <= BN ? P.N1 : BN;
+    P.d_out = L.d_out;
+    P.z = static_cast<uint16_t *>(z_ws);
+    P.y = y;
+    P.y_fp32 = y_fp32;
+    P.ws_words = ws_words;
+    CUtensorMap xmap, zmap;
+    if (!make_map(&xmap, x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, T, L.d_in) ||
+        !make_map(&zmap, z_ws, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, T, P.N1))
+        return cudaErrorInvalidValue;
+    cudaError_t e;
+    e = cudaFuncSetAttribute(k_prefill<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             SMEM_BYTES);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_prefill<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 SMEM_BYTES);
+    if (e != cudaSuccess) return e;
+    const dim3 g1((unsigned)((T + BM - 1) / BM), (unsigned)((P.N1 + P.bn1 - 1) / P.bn1));
+    k_prefill<true><<<g1, kThreads, SMEM_BYTES, s>>>(xmap, P);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const dim3 g2((unsigned)((T + BM - 1) / BM), (unsigned)((L.d_out + BN - 1) / BN));
+    k_prefill<false><<<g2, kThreads, SMEM_BYTES, s>>>(zmap, P);
+    return cudaGetLastError();
+}
+
+}  // namespace lb
