@@ -7,7 +7,10 @@
 //             over the paths is the K dimension of this GEMM)
 // The sign factors never exist in memory as numbers: each CTA unpacks the
 // +-1 bits of its K-slice into shared memory as +-g (stage 1) or +-h (stage
-// 2) fp16 values, in the tensor cores' 128-byte-swizzled K-major layout.  X
+// 2) fp16 values, in the tensor cores' 128-byte-swizzled K-major layout.
+// The bits come from shared memory too: stage 1 bulk-copies each K-stage's
+// two V word rows (and its 64 g values) on the stage's mbarrier beside the
+// TMA of X; stage 2 bulk-copies the tile's U rows and h once per CTA.  X
 // arrives by TMA (bf16) and is converted to fp16 in shared memory (exact for
 // |x| < 65504); z goes to the workspace as fp16 and comes back by TMA.
 //
@@ -37,8 +40,21 @@ constexpr int STAGES = 4;
 constexpr int kThreads = 128;
 constexpr int A_BYTES = BM * BK * 2;   // 16 KB
 constexpr int B_BYTES = BN * BK * 2;   // 32 KB
-constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024;  // + alignment slack
+// stage 1: per stage, the two V word rows of the stage's 64 inputs for the
+// tile's columns (2 x BN words) and the 64 g values of each path
+constexpr int SRC_BYTES = 2 * BN * 4 + 2 * 64 * 2;
+constexpr int MAX_R = 512;  // ranks up to this take the tensor-core path
+// stage 2: once per CTA, the tile's U rows (BN x R words per path) and h
+constexpr int SLAB_U_BYTES = BN * (MAX_R / 32) * 4;
+constexpr int SLAB_BYTES = 2 * SLAB_U_BYTES + 2 * BN * 2;
+// Layout: the A|B stage ring (1024-byte aligned stages, as the 128-byte
+// swizzle requires), then stage 1's ring of sign words or stage 2's slab.
+constexpr int RING_BYTES = STAGES * (A_BYTES + B_BYTES);
+template <bool STAGE1>
+__host__ __device__ constexpr int smem_bytes() {
+    return RING_BYTES + (STAGE1 ? STAGES * SRC_BYTES : SLAB_BYTES) + 1024;
+}
+static_assert(smem_bytes<true>() <= 232448 && smem_bytes<false>() <= 232448, "shared memory");
 
 extern __shared__ __align__(1024) unsigned char p_smem[];
 
@@ -175,10 +191,15 @@ struct PrefillParams {
     unsigned *ws_words;
 };
 
-// Fill B stage with the +-scale values of K-chunk kc for columns [n0, n0+BN).
+// Fill B stage with the +-scale values of K-chunk kc for columns [n0, n0+bn),
+// from sign words and scales already in shared memory (src: stage 1's
+// per-stage words and g; slab: stage 2's U rows and h).
 template <bool STAGE1>
-__device__ __forceinline__ void unpack_b(const PrefillParams &P, unsigned char *Bs, int kc,
-                                         int n0, int bn) {
+__device__ __forceinline__ void unpack_b(const PrefillParams &P, unsigned char *Bs,
+                                         const unsigned char *src, const unsigned char *slab,
+                                         int kc, int n0, int bn) {
+    const uint32_t *words = reinterpret_cast<const uint32_t *>(src);
+    const uint16_t *gs = reinterpret_cast<const uint16_t *>(src + 2 * BN * 4);
     // each item = one 16-byte chunk (8 K values) of one B row
     for (int item = threadIdx.x; item < bn * 8; item += kThreads) {
         const int n = item >> 3, c = item & 7;
@@ -186,13 +207,11 @@ __device__ __forceinline__ void unpack_b(const PrefillParams &P, unsigned char *
         if (STAGE1) {
             const int col = n0 + n;
             if (col < P.N1) {
-                const int p = col >= P.off1 ? 1 : 0, j = col - (p ? P.off1 : 0);
-                const int r = P.L.r[p];
-                // inputs 64kc + 8c .. +7 live in word 2kc + (c >> 2), bits 8(c&3)..
-                const uint32_t word = __ldg(P.L.v[p] + (size_t)(2 * kc + (c >> 2)) * r + j);
+                const int p = col >= P.off1 ? 1 : 0;
+                // inputs 64kc + 8c .. +7: word row (c >> 2), bits 8(c&3) ..
+                const uint32_t word = words[(c >> 2) * BN + n];
                 const uint32_t bits = (word >> (8 * (c & 3))) & 0xffu;
-                const uint4 mag =
-                    __ldg(reinterpret_cast<const uint4 *>(P.L.g[p] + 64 * kc + 8 * c));
+                const uint4 mag = *reinterpret_cast<const uint4 *>(gs + p * 64 + 8 * c);
                 v = signed8(bits, mag);
             }
         } else {
@@ -200,16 +219,34 @@ __device__ __forceinline__ void unpack_b(const PrefillParams &P, unsigned char *
             if (o < P.d_out) {
                 const int k0 = 64 * kc;
                 const int p = k0 >= P.off1 ? 1 : 0, j0 = k0 - (p ? P.off1 : 0);
-                const int R = (P.L.r[p] + 31) >> 5;
-                const uint32_t word = __ldg(P.L.u[p] + (size_t)o * R + (j0 >> 5) + (c >> 2));
+                const int R = ((p ? P.L.r[1] : P.L.r[0]) + 31) >> 5;
+                const uint32_t *U = reinterpret_cast<const uint32_t *>(slab + p * SLAB_U_BYTES);
+                const uint16_t *h =
+                    reinterpret_cast<const uint16_t *>(slab + 2 * SLAB_U_BYTES) + p * BN;
+                const uint32_t word = U[n * R + (j0 >> 5) + (c >> 2)];
                 const uint32_t bits = (word >> (8 * (c & 3))) & 0xffu;
-                const uint32_t hb = __ldg(P.L.h[p] + o);
+                const uint32_t hb = h[n];
                 const uint32_t hh = hb | (hb << 16);
                 v = signed8(bits, make_uint4(hh, hh, hh, hh));
             }
         }
         *reinterpret_cast<uint4 *>(Bs + sw128(n, c)) = v;
     }
+}
+
+__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, unsigned bytes,
+                                         uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::
+            "r"(su32(dst)),
+        "l"(src), "r"(bytes), "r"(su32(bar))
+        : "memory");
+}
+
+__device__ __forceinline__ void mb_expect_only(uint64_t *b, unsigned bytes) {
+    asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(su32(b)),
+                 "r"(bytes)
+                 : "memory");
 }
 
 // In-place bf16 -> fp16 of the A stage (layout-preserving, elementwise).
@@ -234,8 +271,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     __shared__ __align__(8) uint64_t full[STAGES], done[STAGES];
     __shared__ uint32_t s_tmem;
     __shared__ int s_fail;
+    __shared__ __align__(8) uint64_t slab_bar;
     unsigned char *smem = reinterpret_cast<unsigned char *>(
         (reinterpret_cast<uintptr_t>(p_smem) + 1023) & ~(uintptr_t)1023);
+    constexpr int SB = A_BYTES + B_BYTES;
+    unsigned char *slab = smem + RING_BYTES;
     const int m0 = blockIdx.x * BM, n0 = blockIdx.y * BN;
     const int K = STAGE1 ? P.L.d_in : P.N1;
     const int KC = K / BK;
@@ -249,6 +289,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             mb_init(full + s, 1);
             mb_init(done + s, 1);
         }
+        mb_init(&slab_bar, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         s_fail = 0;
     }
@@ -265,20 +306,58 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem = s_tmem;
     const uint32_t idesc = instr_desc(BM, bn);
 
-    auto A_of = [&](int s) { return smem + s * STAGE_BYTES; };
-    auto B_of = [&](int s) { return smem + s * STAGE_BYTES + A_BYTES; };
+    auto A_of = [&](int s) { return smem + s * SB; };
+    auto B_of = [&](int s) { return smem + s * SB + A_BYTES; };
+    auto S_of = [&](int s) { return smem + RING_BYTES + s * SRC_BYTES; };
     int loads_issued = 0, mmas_issued = 0;  // K-chunks loaded / multiplied (thread 0)
+    // The x / z tile of K-chunk kc by TMA; in stage 1 also the chunk's two V
+    // word rows for the tile's columns and the chunk's g values, by bulk copy.
     auto issue_load = [&](int kc) {
         const int s = kc % STAGES;
-        mb_expect_tx(full + s, A_BYTES);
-        tma_load_2d(A_of(s), &amap, kc * BK, m0, full + s);
+        uint64_t *b = full + s;
+        if (STAGE1) {
+            unsigned char *src = S_of(s);
+            for (int p = 0; p < P.L.n_paths; ++p) {
+                const int c0 = p ? P.off1 : 0, c1 = p ? P.N1 : P.off1;
+                const int lo = max(n0, c0), hi = min(n0 + bn, c1);
+                if (lo >= hi) continue;
+                const int r = p ? P.L.r[1] : P.L.r[0];
+                const uint32_t *V = p ? P.L.v[1] : P.L.v[0];
+                for (int wr = 0; wr < 2; ++wr) {
+                    const unsigned bytes = (unsigned)(hi - lo) * 4;
+                    mb_expect_only(b, bytes);
+                    bulk_g2s(src + wr * BN * 4 + (lo - n0) * 4,
+                             V + (size_t)(2 * kc + wr) * r + (lo - c0), bytes, b);
+                }
+                mb_expect_only(b, 128);
+                bulk_g2s(src + 2 * BN * 4 + p * 128, (p ? P.L.g[1] : P.L.g[0]) + 64 * kc, 128, b);
+            }
+        }
+        mb_expect_tx(b, A_BYTES);
+        tma_load_2d(A_of(s), &amap, kc * BK, m0, b);
     };
     if (t0) {
+        if (!STAGE1) {
+            // the tile's U rows and h of every path, once
+            const int nrows = min(BN, P.d_out - n0);
+            for (int p = 0; p < P.L.n_paths; ++p) {
+                const int R = ((p ? P.L.r[1] : P.L.r[0]) + 31) >> 5;
+                mb_expect_only(&slab_bar, (unsigned)(nrows * R * 4 + nrows * 2));
+                bulk_g2s(slab + p * SLAB_U_BYTES, (p ? P.L.u[1] : P.L.u[0]) + (size_t)n0 * R,
+                         (unsigned)(nrows * R * 4), &slab_bar);
+                bulk_g2s(slab + 2 * SLAB_U_BYTES + p * BN * 2, (p ? P.L.h[1] : P.L.h[0]) + n0,
+                         (unsigned)(nrows * 2), &slab_bar);
+            }
+            asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(&slab_bar))
+                         : "memory");
+        }
         for (int kc = 0; kc < 2 && kc < KC; ++kc) issue_load(kc);
         loads_issued = KC < 2 ? KC : 2;
     }
+    bool slab_ok = true;
+    if (!STAGE1) slab_ok = mb_wait(&slab_bar, 0);
 
-    bool ok = true;
+    bool ok = __syncthreads_and(slab_ok) != 0;
     for (int kc = 0; kc < KC && ok; ++kc) {
         const int s = kc % STAGES;
         // refill two stages ahead once the MMAs that last read that stage finished
@@ -296,9 +375,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             ok = false;
             break;
         }
-        unpack_b<STAGE1>(P, B_of(s), kc, n0, bn);
         if (!mb_wait(full + s, (unsigned)((kc / STAGES) & 1))) s_fail = 1;
         __syncthreads();
+        if (s_fail) {
+            ok = false;
+            break;
+        }
+        unpack_b<STAGE1>(P, B_of(s), S_of(s), slab, kc, n0, bn);
         if (s_fail) {
             ok = false;
             break;
@@ -331,6 +414,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 if (kc >= 0) mb_wait(full + kc % STAGES, (unsigned)((kc / STAGES) & 1));
             for (int kc = mmas_issued - STAGES; kc < mmas_issued; ++kc)
                 if (kc >= 0) mb_wait(done + kc % STAGES, (unsigned)((kc / STAGES) & 1));
+            if (!STAGE1) mb_wait(&slab_bar, 0);
         }
         __syncthreads();
     } else {
@@ -352,8 +436,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                     if (c0 < P.N1) {
                         const int p = c0 >= P.off1 ? 1 : 0;
                         const int j = c0 - (p ? P.off1 : 0);
-                        a = v[i] * half_bits_to_float(__ldg(P.L.l[p] + j));
-                        b = v[i + 1] * half_bits_to_float(__ldg(P.L.l[p] + j + 1));
+                        const uint16_t *lp = p ? P.L.l[1] : P.L.l[0];
+                        a = v[i] * half_bits_to_float(__ldg(lp + j));
+                        b = v[i + 1] * half_bits_to_float(__ldg(lp + j + 1));
                     }
                     const __half2 h = __floats2half2_rn(a, b);
                     packed[i >> 1] = *reinterpret_cast<const uint32_t *>(&h);
@@ -375,7 +460,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                             reinterpret_cast<float4 *>(dst)[q] =
                                 make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
                     } else {
-                        for (int i = 0; i < 32 && o0 + i < P.d_out; ++i) dst[i] = v[i];
+#pragma unroll
+                        for (int i = 0; i < 32; ++i)
+                            if (o0 + i < P.d_out) dst[i] = v[i];
                     }
                 } else {
                     uint16_t *dst = static_cast<uint16_t *>(P.y) + (size_t)row * P.d_out + o0;
@@ -390,8 +477,9 @@ __global__ void __launch_bounds__(kThreads, 1)
                             reinterpret_cast<uint4 *>(dst)[q] = make_uint4(w[0], w[1], w[2], w[3]);
                         }
                     } else {
-                        for (int i = 0; i < 32 && o0 + i < P.d_out; ++i)
-                            dst[i] = float_to_bf16_bits(v[i]);
+#pragma unroll
+                        for (int i = 0; i < 32; ++i)
+                            if (o0 + i < P.d_out) dst[i] = float_to_bf16_bits(v[i]);
                     }
                 }
             }
@@ -440,9 +528,9 @@ bool make_map(CUtensorMap *m, const void *base, CUtensorMapDataType dt, int64_t 
 
 bool prefill_supported(const lb_linear &L, int64_t T) {
     if (T < 1 || T > (1LL << 30)) return false;
-    if (L.d_in % BK != 0) return false;
+    if (L.d_in % BK != 0 || L.d_out % 8 != 0) return false;
     for (int p = 0; p < L.n_paths; ++p)
-        if (L.path[p].r % BK != 0) return false;
+        if (L.path[p].r % BK != 0 || L.path[p].r > MAX_R) return false;
     return encoder();
 }
 
@@ -473,17 +561,17 @@ cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, voi
         return cudaErrorInvalidValue;
     cudaError_t e;
     e = cudaFuncSetAttribute(k_prefill<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             SMEM_BYTES);
+                             smem_bytes<true>());
     if (e == cudaSuccess)
         e = cudaFuncSetAttribute(k_prefill<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 SMEM_BYTES);
+                                 smem_bytes<false>());
     if (e != cudaSuccess) return e;
     const dim3 g1((unsigned)((T + BM - 1) / BM), (unsigned)((P.N1 + P.bn1 - 1) / P.bn1));
-    k_prefill<true><<<g1, kThreads, SMEM_BYTES, s>>>(xmap, P);
+    k_prefill<true><<<g1, kThreads, smem_bytes<true>(), s>>>(xmap, P);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const dim3 g2((unsigned)((T + BM - 1) / BM), (unsigned)((L.d_out + BN - 1) / BN));
-    k_prefill<false><<<g2, kThreads, SMEM_BYTES, s>>>(zmap, P);
+    k_prefill<false><<<g2, kThreads, smem_bytes<false>(), s>>>(zmap, P);
     return cudaGetLastError();
 }
 

@@ -147,6 +147,8 @@ STRESS = [
     (32, 17, (1,), 1), (32, 1000, (16, 33), 2), (4128, 17, (96, 1), 3), (4128, 1000, (33, 96), 7),
     (64, 64, (96,), 8), (4128, 1000, (16,), 9), (1024, 300, (33, 16), 65), (4128, 40, (1, 1), 1),
     (96, 2048, (1000, 24), 1), (8192, 8, (64, 64), 1),
+    # T >= 32 but d_out % 8 != 0 or r > 512: the CUDA-core path
+    (512, 2100, (192,), 300), (256, 512, (576,), 40),
 ]
 
 
@@ -161,9 +163,10 @@ def test_stress_shapes(d_in, d_out, rs, T):
 
 
 PREFILL = [
-    # d_in, d_out, ranks, T   (the tensor-core path: T >= 32, ranks multiples of 64)
+    # d_in, d_out, ranks, T   (the tensor-core path: T >= 32, ranks multiples of 64
+    # up to 512, d_out a multiple of 8)
     (64, 256, (64,), 128), (128, 512, (64, 64), 256), (4096, 4096, (64, 64), 200),
-    (256, 1000, (128, 64), 77), (512, 2100, (192,), 300), (1024, 768, (512, 512), 130),
+    (256, 1000, (128, 64), 77), (512, 2104, (192,), 300), (1024, 768, (512, 512), 130),
     (4096, 11008, (128, 128), 64), (64, 8, (64, 64), 33),
 ]
 
