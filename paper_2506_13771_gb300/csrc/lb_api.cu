@@ -96,8 +96,10 @@ lb_status check_stack(const lb_linear *lin, int32_t n_layers, int32_t head_dim,
     return LB_OK;
 }
 
-// FNV-1a over the host description of a stack: shapes, ranks and pointers.
-unsigned long long stack_fingerprint(const lb_linear *lin, int32_t n_layers, int32_t head_dim) {
+// FNV-1a over the host description of a stack (shapes, ranks and pointers)
+// and the SM count the per-CTA programs were built for.
+unsigned long long stack_fingerprint(const lb_linear *lin, int32_t n_layers, int32_t head_dim,
+                                     int sms) {
     unsigned long long h = 1469598103934665603ull;
     auto mix = [&h](unsigned long long v) {
         for (int b = 0; b < 8; ++b) {
@@ -107,6 +109,7 @@ unsigned long long stack_fingerprint(const lb_linear *lin, int32_t n_layers, int
     };
     mix((unsigned long long)n_layers);
     mix((unsigned long long)head_dim);
+    mix((unsigned long long)sms);
     for (int i = 0; i < 7 * n_layers; ++i) {
         const lb_linear &L = lin[i];
         mix((unsigned long long)L.d_in);
@@ -216,11 +219,12 @@ lb_status littlebit_stack_prepare(const lb_linear *lin, int32_t n_layers, int32_
     if (!ws || ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) ||
         ws_bytes < littlebit_stack_workspace_size(lin, n_layers, head_dim))
         return LB_ERR_WORKSPACE;
-    return from_cuda(lb::launch_stack_prepare(lin, n_layers,
-                                              stack_fingerprint(lin, n_layers, head_dim),
-                                              static_cast<unsigned *>(ws),
-                                              static_cast<char *>(ws) + kWsHeader,
-                                              (cudaStream_t)stream));
+    int sms = 0;
+    if ((st = num_sms(&sms)) != LB_OK) return st;
+    const cudaError_t e = lb::launch_stack_prepare(
+        lin, n_layers, shape, sms, stack_fingerprint(lin, n_layers, head_dim, sms),
+        static_cast<unsigned *>(ws), static_cast<char *>(ws) + kWsHeader, (cudaStream_t)stream);
+    return e == cudaErrorNotSupported ? LB_ERR_UNSUPPORTED : from_cuda(e);
 }
 
 lb_status littlebit_stack_forward(const lb_linear *lin, int32_t n_layers, int32_t head_dim,
@@ -239,7 +243,8 @@ lb_status littlebit_stack_forward(const lb_linear *lin, int32_t n_layers, int32_
     if ((st = num_sms(&sms)) != LB_OK) return st;
     if (!lb::stack_supported(lin, shape, sms)) return LB_ERR_UNSUPPORTED;
     return from_cuda(lb::launch_stack(lin, n_layers, shape,
-                                      stack_fingerprint(lin, n_layers, head_dim), x0, out, q_out,
+                                      stack_fingerprint(lin, n_layers, head_dim, sms), x0, out,
+                                      q_out,
                                       kv_out, static_cast<unsigned *>(ws),
                                       static_cast<char *>(ws) + kWsHeader, sms,
                                       (cudaStream_t)stream));

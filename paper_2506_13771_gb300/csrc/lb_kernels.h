@@ -26,15 +26,17 @@ size_t decode_ws_floats(const lb_linear &L);
 cudaError_t launch_decode(const lb_linear &L, const uint16_t *x, void *y, int y_fp32,
                           unsigned *ws_words, float *acc, int num_sms, cudaStream_t s);
 
-// Persistent decode of the seven-linear-per-layer stack (lb_persistent.cu).
+// Persistent decode of the seven-linear-per-layer stack (lb_stack.cu).
 struct StackShape {
     int n_layers, d, dkv, dff, head_dim;
 };
 size_t stack_ws_bytes_after_header(const lb_linear *lin, int n_layers);
-// Writes the device descriptor table, zeroes counters and accumulators, and
-// stores the plan fingerprint.
-cudaError_t launch_stack_prepare(const lb_linear *lin, int n_layers, unsigned long long plan,
-                                 unsigned *ws_words, char *ws_after_header, cudaStream_t s);
+// Writes the device descriptor table and the per-CTA programs for num_sms
+// CTAs, zeroes counters and accumulators, and stores the plan fingerprint.
+// cudaErrorNotSupported when the shapes or the programs do not fit.
+cudaError_t launch_stack_prepare(const lb_linear *lin, int n_layers, const StackShape &shape,
+                                 int num_sms, unsigned long long plan, unsigned *ws_words,
+                                 char *ws_after_header, cudaStream_t s);
 // Whether the one-launch stack kernel handles these shapes on this GPU
 // (ranks multiples of 8, head_dim multiple of 32, d_kv multiple of 8, the
 // shared-memory plan fits).

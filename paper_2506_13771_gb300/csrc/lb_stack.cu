@@ -6,7 +6,7 @@
 // d_in (stage 1, rank-r result t) followed by a +-1 reduction over r (stage
 // 2), per path, paths summed (Eq. 6).  CTA c owns
 //   R_c : a slice of d rows, whole 32-row words    (q, o, down outputs; the
-//         residual stream a/h; stage-1 inputs of q, k, v, o, gate, up)
+//         residual stream; stage-1 inputs of q, k, v, o, gate, up)
 //   F_c : a slice of d_ff rows, whole 32-row words (gate, up outputs; m;
 //         stage-1 input of down)
 //   K_c : a slice of d_kv rows, multiples of 8     (k, v outputs)
@@ -21,6 +21,12 @@
 //  * +-1 sums use 4-bit lookup tables in shared memory: 16 signed sums of 4
 //    values, stored twice so the two half-warps use disjoint banks; a 32-bit
 //    sign word costs 8 table lookups (PRMT forms the address, LDS reads it);
+//  * the compute warps run a per-CTA program built on the host by
+//    littlebit_stack_prepare: for every step, table jobs and warp-balanced
+//    work units (32 rows x a run of words, or 32 columns x the slice) with
+//    their shared-memory offsets.  The shapes are those of every layer, so
+//    the program is the same for all of them; the device code is a handful
+//    of generic loops, small enough to stay in the instruction cache;
 //  * the all-reduce of t accumulates fixed-point values in 64-bit words whose
 //    low 8 bits count contributions: each CTA adds (round(v * 2^24) << 8) + 1
 //    with one red.add per element and readers poll the words they need until
@@ -31,6 +37,8 @@
 // Every wait is bounded (about one second); on a timeout the CTA records
 // LB_ERR_TIMEOUT, waits for its own bulk copies to land, and returns.
 #include <algorithm>
+#include <cstring>
+#include <vector>
 
 #include "lb_common.cuh"
 #include "lb_kernels.h"
@@ -127,11 +135,47 @@ struct Offsets {
     int c_Uo[2], c_ho[2], c_lo[2], c_Vg[2], c_Vu[2], c_gg[2], c_gu[2];
     // phase D: stage 2 of gate, up, stage 1 of down
     int d_Ug[2], d_Uu[2], d_hg[2], d_hu[2], d_lg[2], d_lu[2], d_Vd[2], d_gd[2];
-    int tables, tz, res, xs, ys, yq, tsave;  // work areas
+    // work areas: stage-2 and stage-1 tables, decoded exchange, residual
+    // stream (two buffers: phase A reads 0 and writes 1, phase C the reverse),
+    // stage-2 outputs (added into, zeroed by their consumer), saved t of q's
+    // second path, the sum-of-squares accumulator, the program
+    int t2, t1, tz, res0, res1, y, xa, yq, yk, yv, yg, yu, tsave, ssacc, prog;
 };
+
+// Steps of the per-CTA program (one per table build or unit loop).
+enum StepId {
+    A_T2, A_S2, A_T1, A_S1,
+    B_T2V, B_S2V, B_T1, B_S1, B_T2QK, B_S2QKV,
+    C_T2, C_S2, C_T1, C_S1, C_T2Q1, C_S2Q1,
+    D_T2, D_S2, D_T1, D_S1,
+    N_STEPS
+};
+
+// One program record (8 ints).  Meaning by step kind:
+//   table unit  : tb, n_tab, n_vals, mode, s0, s1, s2, scale   (up to 32
+//                 tables of one job, from its table t0 on; the offsets and
+//                 n_vals are those of table t0)
+//   stage-2 unit: U, R, nw, tb, h, out, nrows, -
+//   stage-1 unit: V, r, nw, tb, dst, ncols, -, -
+struct Item {
+    int f[8];
+};
+// Table-job modes: source kind in bits 0-1, flags above.
+enum { TAB_PLAIN = 0, TAB_RES = 1, TAB_SILU = 2, TAB_WRITER = 4, TAB_MUL = 8 };
+
+// Warp w runs units [first + wo[w], first + wo[w + 1]) of its step.
+struct Step {
+    int first;
+    int wo[kCW + 1];
+};
+constexpr int kStepBytes = (int)((N_STEPS * sizeof(Step) + 15) / 16 * 16);
+constexpr int kProgBytes = 16384;  // per CTA, in the workspace and in shared memory
+constexpr int kMaxItems = (kProgBytes - kStepBytes) / (int)sizeof(Item);
+constexpr int kMaxCtas = 255;      // the 8-bit contribution count of the exchange
 
 struct Params {
     const LinDesc *lin;  // 7 * n_layers descriptors in the workspace
+    const int *prog;     // kProgBytes per CTA in the workspace
     int n_layers, d, dkv, dff, hd;
     int np[7], r[7][2];  // paths and ranks of q, k, v, o, gate, up, down
     const uint16_t *x0;
@@ -172,194 +216,151 @@ __device__ __forceinline__ float lut8(uint32_t lo, uint32_t hi, uint32_t base) {
     return ((a0 + a1) + (a2 + a3)) + ((a4 + a5) + (a6 + a7));
 }
 
-__device__ __forceinline__ void split_word(uint32_t word, uint32_t copy, uint32_t &lo,
-                                           uint32_t &hi) {
-    lo = ((word << 2) & 0x3C3C3C3Cu) | copy;
-    hi = ((word >> 2) & 0x3C3C3C3Cu) | copy;
+__device__ __forceinline__ float lut_word(uint32_t word, uint32_t copy, uint32_t base) {
+    const uint32_t lo = ((word << 2) & 0x3C3C3C3Cu) | copy;
+    const uint32_t hi = ((word >> 2) & 0x3C3C3C3Cu) | copy;
+    return lut8(lo, hi, base);
 }
 
-// Compute helpers.  Job arrays have a compile-time size NJ (the jobs a step
-// could have with two paths per linear) and are indexed with compile-time
-// indices only, so they stay in registers; a job that does not exist (a
-// linear with one path) has no rows / columns / tables.  All buffers are
-// byte offsets into g_smem.
+__device__ __forceinline__ float silu(float x) { return x / (1.f + __expf(-x)); }
 
-// Nibble tables of one value vector: table n (n < n_tab), entry e = 0..15 is
-// sum_{k<4} (bit k of e ? -v : +v)[4n + k] with v_i = src[i] * mul * scale[i]
-// (scale: fp16 offset, or -1 for none), stored twice (entries e and 16 + e,
-// one copy per half-warp).  Tables at or past n_vals / 4 are zero, so sign
-// bits beyond the data (padding) add nothing.
-struct TJ {
-    int tb;      // byte offset of table 0 (256-aligned)
-    int n_tab;   // tables to fill (0: job absent)
-    int n_vals;  // values available
-    int src;     // byte offset of the fp32 values
-    int scale;   // byte offset of the fp16 scales, or -1
-    float mul;
-};
+__device__ __forceinline__ float4 ld_f4(int off) {
+    return *reinterpret_cast<const float4 *>(g_smem + off);
+}
 
-// One thread per (table, 16-byte quarter): 8 consecutive threads write one
-// table's 128 bytes, so the float4 stores of a warp are bank-conflict free.
-template <int NJ>
-__device__ __forceinline__ void build_tables(const TJ (&J)[NJ]) {
-    int cum[NJ + 1];
-    cum[0] = 0;
-#pragma unroll
-    for (int j = 0; j < NJ; ++j) cum[j + 1] = cum[j] + 8 * J[j].n_tab;
-    for (int idx = threadIdx.x; idx < cum[NJ]; idx += kCT) {
-        int tb = J[0].tb, n_vals = J[0].n_vals, src = J[0].src, scale = J[0].scale, t = idx;
-        float mul = J[0].mul;
-#pragma unroll
-        for (int j = 1; j < NJ; ++j)
-            if (idx >= cum[j]) {
-                tb = J[j].tb;
-                n_vals = J[j].n_vals;
-                src = J[j].src;
-                scale = J[j].scale;
-                mul = J[j].mul;
-                t = idx - cum[j];
+// The program lives in shared memory at byte offset prog; step and unit
+// records are read with shared-memory loads (the step functions take byte
+// offsets, not generic pointers, so the compiler knows the state space).
+__device__ __forceinline__ const Step &step_at(int prog, int s) {
+    return *reinterpret_cast<const Step *>(g_smem + prog + s * (int)sizeof(Step));
+}
+__device__ __forceinline__ void item_at(int prog, int u, int4 &a, int4 &b) {
+    const unsigned char *p = g_smem + prog + kStepBytes + u * (int)sizeof(Item);
+    a = *reinterpret_cast<const int4 *>(p);
+    b = *reinterpret_cast<const int4 *>(p + 16);
+}
+
+// Table units: lane n builds table n of the unit.  Table n holds, for
+// e = 0..15, sum_{k<4} (bit k of e ? -v : +v) of v_i = x_i * scale_i
+// (* inv with TAB_MUL), i = 4n + k, where x_i is
+//   TAB_PLAIN: s0[i]    TAB_RES: s0[i] + s1[i]    TAB_SILU: silu(s0[i]) * s1[i]
+// (values at or past n_vals are 0, so padding bits add nothing).  It is
+// stored twice (entries e and 16 + e, one copy per half-warp).  A TAB_WRITER
+// unit also stores x into s2 and adds sum x^2 into the float at ss_off.
+// Each lane writes its table's eight 16-byte chunks starting at chunk
+// (lane & 7): the eight lanes of a quarter-warp hit distinct banks.
+__device__ __noinline__ void run_tables(int prog, int s, float inv, int ss_off) {
+    const Step &st = step_at(prog, s);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int u1 = st.first + st.wo[warp + 1];
+    for (int u = st.first + st.wo[warp]; u < u1; ++u) {
+        int4 a, b;
+        item_at(prog, u, a, b);
+        const int n_vals = a.z - 4 * lane, mode = a.w;
+        float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+        float ss = 0.f;
+        if (lane < a.y && n_vals > 0) {
+            x = ld_f4(b.x + 16 * lane);
+            if ((mode & 3) == TAB_RES) {
+                const float4 y = ld_f4(b.y + 16 * lane);
+                x = make_float4(x.x + y.x, x.y + y.y, x.z + y.z, x.w + y.w);
+            } else if ((mode & 3) == TAB_SILU) {
+                const float4 y = ld_f4(b.y + 16 * lane);
+                x = make_float4(silu(x.x) * y.x, silu(x.y) * y.y, silu(x.z) * y.z,
+                                silu(x.w) * y.w);
             }
-        const int n = t >> 3, q = t & 7;
-        float z[4] = {0.f, 0.f, 0.f, 0.f};
-        if (4 * n < n_vals) {
-            const float4 v = *reinterpret_cast<const float4 *>(g_smem + src + 16 * n);
-            z[0] = v.x * mul;
-            z[1] = v.y * mul;
-            z[2] = v.z * mul;
-            z[3] = v.w * mul;
-            if (scale >= 0) {
-                const uint2 hb = *reinterpret_cast<const uint2 *>(g_smem + scale + 8 * n);
-                z[0] *= half_bits_to_float((uint16_t)(hb.x & 0xffffu));
-                z[1] *= half_bits_to_float((uint16_t)(hb.x >> 16));
-                z[2] *= half_bits_to_float((uint16_t)(hb.y & 0xffffu));
-                z[3] *= half_bits_to_float((uint16_t)(hb.y >> 16));
+            if (mode & TAB_WRITER) {
+                *reinterpret_cast<float4 *>(g_smem + b.z + 16 * lane) = x;
+                ss = x.x * x.x + x.y * x.y + x.z * x.z + x.w * x.w;
+            }
+            const uint2 hb = *reinterpret_cast<const uint2 *>(g_smem + b.w + 8 * lane);
+            const float m = (mode & TAB_MUL) ? inv : 1.f;
+            x.x *= half_bits_to_float((uint16_t)(hb.x & 0xffffu)) * m;
+            x.y *= half_bits_to_float((uint16_t)(hb.x >> 16)) * m;
+            x.z *= half_bits_to_float((uint16_t)(hb.y & 0xffffu)) * m;
+            x.w *= half_bits_to_float((uint16_t)(hb.y >> 16)) * m;
+        }
+        if (lane < a.y) {
+            unsigned char *T = g_smem + a.x + lane * 128;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                const int q = (k + lane) & 7;
+                // chunk q: entries 4(q&3) .. +3; high bits (e3 e2) = q & 3
+                const float qv = ((q & 1) ? -x.z : x.z) + ((q & 2) ? -x.w : x.w);
+                *reinterpret_cast<float4 *>(T + 16 * q) = make_float4(
+                    x.x + x.y + qv, x.y - x.x + qv, x.x - x.y + qv, -x.x - x.y + qv);
             }
         }
-        // entries 4(q&3) .. 4(q&3)+3: high bits (e3 e2) = q & 3, low bits run 0..3
-        const int hb2 = q & 3;
-        const float s2 = (hb2 & 1) ? -z[2] : z[2];
-        const float s3 = (hb2 & 2) ? -z[3] : z[3];
-        const float qv = s2 + s3;
-        const float4 r = make_float4(z[0] + z[1] + qv, z[1] - z[0] + qv, z[0] - z[1] + qv,
-                                     -z[0] - z[1] + qv);
-        *reinterpret_cast<float4 *>(g_smem + tb + n * 128 + q * 16) = r;
+        if (mode & TAB_WRITER) {
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+            if (lane == 0) atomicAdd(sm_f(ss_off), ss);
+        }
     }
 }
 
-// Stage 2 job: ys[row] += h[row] * sum_j U_sign[row][j] z[j] for rows
-// [0, nrows) of one path; U words [nrows][R] and h at U / h; z tables at tb.
-struct UJ {
-    int U, h, R, nrows, tb, ys;
-};
-
-// A task is 32 rows x a run of words of one job; its lanes (rows) read the
-// same 8 tables per word, so lookups are bank-conflict free.  When the jobs
-// have fewer 32-row blocks than twice the compute warps, each row's words are
-// split into a power-of-two number of runs (shifts only: this runs on the
-// critical path of every phase).
-template <int NJ>
-__device__ __forceinline__ void u_stage(const UJ (&J)[NJ]) {
+// Stage-2 units: out[row] += h[row] * sum over the unit's words of the
+// +-1 products of U's row with the tabled t (lane = row).
+__device__ __noinline__ void run_s2(int prog, int s) {
+    const Step &st = step_at(prog, s);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
-    int blocks = 0;
-#pragma unroll
-    for (int j = 0; j < NJ; ++j) blocks += (J[j].nrows + 31) >> 5;
-    int slog = 0;
-#pragma unroll
-    for (int k = 0; k < 5; ++k) slog += (blocks << slog) < 2 * kCW ? 1 : 0;
-    int cum[NJ + 1], nlog[NJ], wc[NJ];
-    cum[0] = 0;
-#pragma unroll
-    for (int j = 0; j < NJ; ++j) {
-        const int R = J[j].R;
-        nlog[j] = min(slog, 31 - __clz(max(R, 1)));
-        wc[j] = (R + (1 << nlog[j]) - 1) >> nlog[j];
-        cum[j + 1] = cum[j] + (((J[j].nrows + 31) >> 5) << nlog[j]);
-    }
-    for (int task = warp; task < cum[NJ]; task += kCW) {
-        int U = J[0].U, h = J[0].h, R = J[0].R, nrows = J[0].nrows, tb = J[0].tb, ys = J[0].ys;
-        int t = task, nl = nlog[0], w_c = wc[0];
-#pragma unroll
-        for (int j = 1; j < NJ; ++j)
-            if (task >= cum[j]) {
-                U = J[j].U;
-                h = J[j].h;
-                R = J[j].R;
-                nrows = J[j].nrows;
-                tb = J[j].tb;
-                ys = J[j].ys;
-                t = task - cum[j];
-                nl = nlog[j];
-                w_c = wc[j];
-            }
-        const int rb = t >> nl, w0 = (t & ((1 << nl) - 1)) * w_c;
-        const int w1 = min(w0 + w_c, R);
-        const int row = 32 * rb + lane;
-        if (row < nrows) {
-            const uint32_t *Uw = sm_u32(U) + row * R;
-            float acc = 0.f;
-            for (int w = w0; w < w1; ++w) {
-                uint32_t lo, hi;
-                split_word(Uw[w], copy, lo, hi);
-                acc += lut8(lo, hi, (uint32_t)(tb + w * 1024));
-            }
-            atomicAdd(sm_f(ys) + row, acc * half_bits_to_float(sm_u16(h)[row]));
+    const int u1 = st.first + st.wo[warp + 1];
+    for (int u = st.first + st.wo[warp]; u < u1; ++u) {
+        int4 a, b;
+        item_at(prog, u, a, b);
+        const int R = a.y, nw = a.z, nrows = b.z;
+        const uint32_t tb = (uint32_t)a.w;
+        const int row = min(lane, nrows - 1);
+        const uint32_t *Uw = sm_u32(a.x) + row * R;
+        float acc0 = 0.f, acc1 = 0.f;
+        int w = 0;
+        for (; w + 2 <= nw; w += 2) {
+            const uint32_t w0 = Uw[w], w1 = Uw[w + 1];
+            acc0 += lut_word(w0, copy, tb + w * 1024);
+            acc1 += lut_word(w1, copy, tb + (w + 1) * 1024);
         }
+        if (w < nw) acc0 += lut_word(Uw[w], copy, tb + w * 1024);
+        if (lane < nrows)
+            atomicAdd(sm_f(b.y) + lane, (acc0 + acc1) * half_bits_to_float(sm_u16(b.x)[lane]));
     }
 }
 
-// Stage 1 job: all r columns of one path over the CTA's nw input words; V
-// words [nw][r] at V, input tables at tb; the partial t goes to dst.
-struct VJ {
-    int V, r, nw, tb;
-    unsigned long long *dst;
-};
-
-__device__ __forceinline__ void red_fix(unsigned long long *p, float v, float limit,
-                                        unsigned *err) {
+// One contribution to an exchange word: (round(v * 2^24) << 8) + 1.
+__device__ __forceinline__ unsigned long long enc_fix(float v, float limit, unsigned *err) {
     if (!(fabsf(v) < limit)) {
         atomicCAS(err, 0u, static_cast<unsigned>(LB_ERR_RANGE));
         v = 0.f;
     }
     const long long f = __float2ll_rn(v * kFix);
-    red_add_u64(p, (static_cast<unsigned long long>(f) << 8) + 1ull);
+    return (static_cast<unsigned long long>(f) << 8) + 1ull;
 }
 
-// t[j] partial over the slice, added to the exchange words (one contribution
-// per CTA per element, also when the slice is empty).  A task is 32 columns
-// x all slice words of one job.
-template <int NJ>
-__device__ __forceinline__ void v_stage(const VJ (&J)[NJ], float limit, unsigned *err) {
+// Stage-1 units: t[col] partial over the CTA's input slice, added to the
+// exchange words (lane = column).  Every CTA has a unit for every column,
+// also when its slice is empty, so each element counts one contribution
+// per CTA.
+__device__ __noinline__ void run_s1(int prog, int s, unsigned long long *xbase, float limit,
+                                    unsigned *err) {
+    const Step &st = step_at(prog, s);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
-    int cum[NJ + 1];
-    cum[0] = 0;
-#pragma unroll
-    for (int j = 0; j < NJ; ++j) cum[j + 1] = cum[j] + ((J[j].r + 31) >> 5);
-    for (int task = warp; task < cum[NJ]; task += kCW) {
-        int V = J[0].V, r = J[0].r, nw = J[0].nw, tb = J[0].tb, t = task;
-        unsigned long long *dst = J[0].dst;
-#pragma unroll
-        for (int j = 1; j < NJ; ++j)
-            if (task >= cum[j]) {
-                V = J[j].V;
-                r = J[j].r;
-                nw = J[j].nw;
-                tb = J[j].tb;
-                dst = J[j].dst;
-                t = task - cum[j];
-            }
-        const int col = 32 * t + lane;
-        if (col < r) {
-            float acc = 0.f;
-            const uint32_t *Vw = sm_u32(V) + col;
-            for (int w = 0; w < nw; ++w) {
-                uint32_t lo, hi;
-                split_word(Vw[w * r], copy, lo, hi);
-                acc += lut8(lo, hi, (uint32_t)(tb + w * 1024));
-            }
-            red_fix(dst + col, acc, limit, err);
+    const int u1 = st.first + st.wo[warp + 1];
+    for (int u = st.first + st.wo[warp]; u < u1; ++u) {
+        int4 a, b;
+        item_at(prog, u, a, b);
+        const int r = a.y, nw = a.z, ncols = b.y;
+        const uint32_t tb = (uint32_t)a.w;
+        const uint32_t *Vw = sm_u32(a.x) + min(lane, ncols - 1);
+        float acc0 = 0.f, acc1 = 0.f;
+        int w = 0;
+        for (; w + 2 <= nw; w += 2) {
+            const uint32_t w0 = Vw[w * r], w1 = Vw[(w + 1) * r];
+            acc0 += lut_word(w0, copy, tb + w * 1024);
+            acc1 += lut_word(w1, copy, tb + (w + 1) * 1024);
         }
+        if (w < nw) acc0 += lut_word(Vw[w * r], copy, tb + w * 1024);
+        if (lane < ncols) red_add_u64(xbase + b.x + lane, enc_fix(acc0 + acc1, limit, err));
     }
 }
 
@@ -376,25 +377,6 @@ __device__ __forceinline__ int csync_and(int pred) {
         : "r"(pred), "n"(kCT)
         : "memory");
     return r;
-}
-
-// Sum of v over the compute threads, returned to each of them (one barrier:
-// the partials are read back before any later barrier lets them be rewritten).
-__device__ float csum(float v) {
-    __shared__ float s_part[kCW];
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    if ((threadIdx.x & 31) == 0) s_part[threadIdx.x >> 5] = v;
-    csync();
-    float t = 0.f;
-#pragma unroll
-    for (int w = 0; w < kCW; ++w) t += s_part[w];
-    return t;
-}
-
-__device__ __forceinline__ float sum_sq(const float *v, int n) {
-    float s = 0.f;
-    for (int i = threadIdx.x; i < n; i += kCT) s += v[i] * v[i];
-    return csum(s);
 }
 
 __device__ __forceinline__ void zero_f(float *p, int n) {
@@ -457,6 +439,7 @@ __device__ bool wait_full(unsigned long long *bar, unsigned parity, unsigned *ws
     if (!mbar_try_wait(bar, parity)) {
         const unsigned long long t0 = globaltimer_ns();
         while (!mbar_try_wait(bar, parity)) {
+            __nanosleep(32);
             if (globaltimer_ns() - t0 > kWaitLimitNs) {
                 record(ws_words, LB_ERR_TIMEOUT);
                 ok = 0;
@@ -467,7 +450,6 @@ __device__ bool wait_full(unsigned long long *bar, unsigned parity, unsigned *ws
     return csync_and(ok) != 0;
 }
 
-__device__ __forceinline__ float silu(float x) { return x / (1.f + __expf(-x)); }
 
 // ---------------------------------------------------------------- the kernel
 
@@ -604,8 +586,12 @@ __device__ void producer(const Loader &ld, unsigned long long *empty, unsigned *
             if (b > 0 && l == L) break;  // the final phase needs only buffer A
             const unsigned parity = (unsigned)((l - 1) & 1);
             unsigned long long t0 = 0;
+            // the compute warps hold the buffer for most of a layer: poll it
+            // gently, so the wait does not take issue slots and shared-memory
+            // bandwidth from them
             for (int spin = 0; !mbar_try_wait(empty + b, parity); ++spin) {
-                if ((spin & 63) == 63) {
+                __nanosleep(128);
+                if ((spin & 15) == 15) {
                     if (sticky(ws_words)) {
                         ok = false;
                         break;
@@ -669,286 +655,150 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
     }
 
     // ------------------------------------------------------------ compute warps
-    const int nd = s.nd, nf = s.nf, nkv = s.nkv;
-    const int rows_d = 32 * nd, rows_f = 32 * nf;
     const Offsets &o = P.o;
-    float *res = sm_f(o.res), *xs = sm_f(o.xs), *ys = sm_f(o.ys), *yq = sm_f(o.yq);
-    float *tz = sm_f(o.tz);
-    for (int i = threadIdx.x; i < rows_d; i += kCT)
-        res[i] = bf16_bits_to_float(P.x0[32 * s.dw0 + i]);
+    {
+        const int4 *src = reinterpret_cast<const int4 *>(P.prog) + (size_t)c * (kProgBytes / 16);
+        int4 *dst = reinterpret_cast<int4 *>(g_smem + o.prog);
+        for (int i = threadIdx.x; i < kProgBytes / 16; i += kCT) dst[i] = src[i];
+    }
+    const int pg = o.prog;
+    const int rows_d = 32 * s.nd, rows_f = 32 * s.nf, nkv = s.nkv;
+    float *res0 = sm_f(o.res0), *y = sm_f(o.y), *xa = sm_f(o.xa), *yq = sm_f(o.yq);
+    float *yk = sm_f(o.yk), *yv = sm_f(o.yv), *yg = sm_f(o.yg), *yu = sm_f(o.yu);
+    float *tz = sm_f(o.tz), *tsave = sm_f(o.tsave), *ssacc = sm_f(o.ssacc);
+    for (int i = threadIdx.x; i < rows_d; i += kCT) {
+        res0[i] = bf16_bits_to_float(P.x0[32 * s.dw0 + i]);
+        y[i] = xa[i] = yq[i] = 0.f;
+    }
+    zero_f(yk, nkv);
+    zero_f(yv, nkv);
+    zero_f(yg, rows_f);
+    zero_f(yu, rows_f);
+    if (threadIdx.x == 0) *ssacc = 0.f;
+    csync();
     int nr[7];
 #pragma unroll
     for (int k = 0; k < 7; ++k) nr[k] = P.r[k][0] + (P.np[k] > 1 ? P.r[k][1] : 0);
     const int ssA = nr[LQ] + nr[LK] + nr[LV], ssC = nr[LG] + nr[LU];
+    const int rq0 = P.r[LQ][0], rq1 = P.np[LQ] > 1 ? P.r[LQ][1] : 0;
     const bool lead = threadIdx.x == 0;
-    // rank and presence of path p of linear k
-    auto rk = [&](int k, int p) { return p < P.np[k] ? P.r[k][p] : 0; };
+    const float lim = P.fix_limit;
     auto release = [&](int b) {
         csync();
         if (lead) mbar_arrive(empty + b);
     };
-    // stage 2 of down (both paths) on R_c into ys, from t in tz
-    auto down_rows = [&]() {
-        TJ T[2];
-        UJ U[2];
-        int tb = o.tables, off = 0;
-#pragma unroll
-        for (int p = 0; p < 2; ++p) {
-            const int r = rk(LD, p), R = r ? wordsR(r) : 1;
-            T[p] = TJ{tb, r ? 8 * R : 0, r, o.tz + 4 * off, o.a_ld[p], 1.f};
-            U[p] = UJ{o.a_Ud[p], o.a_hd[p], R, r ? rows_d : 0, tb, o.ys};
-            tb += r ? R * 1024 : 0;
-            off += r;
+    auto send_ss = [&](unsigned long long *p) {
+        if (lead) {
+            red_add_u64(p, enc_fix(*ssacc, lim, err));
+            *ssacc = 0.f;
         }
-        zero_f(ys, rows_d);
-        build_tables(T);
-        csync();
-        u_stage(U);
-        csync();
     };
 #define FAIL_EXIT() return
 
     for (int l = 0; l < P.n_layers; ++l) {
-        unsigned long long *xA = P.xacc + (size_t)l * P.acc_layer + P.offA;
-        unsigned long long *xB = P.xacc + (size_t)l * P.acc_layer + P.offB;
-        unsigned long long *xC = P.xacc + (size_t)l * P.acc_layer + P.offC;
-        unsigned long long *xD = P.xacc + (size_t)l * P.acc_layer + P.offD;
+        unsigned long long *xl = P.xacc + (size_t)l * P.acc_layer;
+        unsigned long long *xA = xl + P.offA, *xB = xl + P.offB, *xC = xl + P.offC,
+                           *xD = xl + P.offD;
         const unsigned par = (unsigned)(l & 1);
 
         // ================= phase A: a = h + Down_{l-1}(m) on R_c; stage 1 of q, k, v
         if (l > 0) {
-            if (!poll_decode(xD - P.acc_layer, nr[LD], n_ctas, tz, P.ws_words)) FAIL_EXIT();
+            if (!poll_decode(xD - P.acc_layer, P.lenD, n_ctas, tz, P.ws_words)) FAIL_EXIT();
             zero_stripe(xC - P.acc_layer, P.lenC);
         }
         if (!wait_full(full + 0, par, P.ws_words)) FAIL_EXIT();
         if (l > 0) {
-            down_rows();
-            for (int i = threadIdx.x; i < rows_d; i += kCT) res[i] += ys[i];
+            run_tables(pg, A_T2, 1.f, o.ssacc);
+            csync();
+            run_s2(pg, A_S2);
             csync();
         }
-        {
-            const float ss = sum_sq(res, rows_d);
-            if (lead) red_fix(xA + ssA, ss, P.fix_limit, err);
-            TJ T[6];
-            VJ V[6];
-            int tb = o.tables;
-            unsigned long long *dst = xA;
-#pragma unroll
-            for (int k = 0; k < 3; ++k)
-#pragma unroll
-                for (int p = 0; p < 2; ++p) {
-                    const int r = rk(k, p);
-                    T[2 * k + p] = TJ{tb, r ? 8 * nd : 0, rows_d, o.res, o.a_g[k][p], 1.f};
-                    V[2 * k + p] = VJ{o.a_V[k][p], r, nd, tb, dst};
-                    tb += r ? nd * 1024 : 0;
-                    dst += r;
-                }
-            build_tables(T);
-            csync();
-            v_stage(V, P.fix_limit, err);
-        }
+        run_tables(pg, A_T1, 1.f, o.ssacc);  // a = res0 + y -> res1
+        csync();
+        send_ss(xA + ssA);
+        run_s1(pg, A_S1, xl, lim, err);
+        zero_f(y, rows_d);
         release(0);
 
         // ================= phase B: v rows for attention, stage 1 of o; then q, k, v out
-        if (!poll_decode(xA, ssA + 1, n_ctas, tz, P.ws_words)) FAIL_EXIT();
+        if (!poll_decode(xA, P.lenA, n_ctas, tz, P.ws_words)) FAIL_EXIT();
         if (l > 0) zero_stripe(xD - P.acc_layer, P.lenD);
         if (!wait_full(full + 1, par, P.ws_words)) FAIL_EXIT();
         {
             const float inv = rsqrtf(tz[ssA] / (float)P.d);
-            int tb = o.tables;
-            const int tb_v = tb;
-            {
-                TJ T[2];
-                UJ U[2];
-#pragma unroll
-                for (int p = 0, off = nr[LQ] + nr[LK]; p < 2; ++p) {
-                    const int r = rk(LV, p), R = r ? wordsR(r) : 1;
-                    T[p] = TJ{tb, r ? 8 * R : 0, r, o.tz + 4 * off, o.b_lv[p], inv};
-                    U[p] = UJ{o.b_Uat[p], o.b_hat[p], R, r ? rows_d : 0, tb, o.xs};
-                    tb += r ? R * 1024 : 0;
-                    off += r;
-                }
-                zero_f(xs, rows_d);
-                build_tables(T);
-                csync();
-                u_stage(U);
-                csync();
+            if (rq1) {
+                for (int i = threadIdx.x; i < rq1; i += kCT) tsave[i] = tz[rq0 + i];
+                if (lead) tsave[rq1] = inv;
             }
-            {
-                TJ T[2];
-                VJ V[2];
-                unsigned long long *dst = xB;
-#pragma unroll
-                for (int p = 0; p < 2; ++p) {
-                    const int r = rk(LO, p);
-                    T[p] = TJ{tb, r ? 8 * nd : 0, rows_d, o.xs, o.b_go[p], 1.f};
-                    V[p] = VJ{o.b_Vo[p], r, nd, tb, dst};
-                    tb += r ? nd * 1024 : 0;
-                    dst += r;
+            run_tables(pg, B_T2V, inv, o.ssacc);
+            csync();
+            run_s2(pg, B_S2V);  // -> xa
+            csync();
+            run_tables(pg, B_T1, 1.f, o.ssacc);
+            csync();
+            run_s1(pg, B_S1, xl, lim, err);
+            zero_f(xa, rows_d);
+            // ---- off the critical path, while exchange B is in flight: k and
+            //      v on K_c, path 0 of q on R_c (path 1 of q runs after
+            //      exchange C is sent, from the saved t and rms)
+            run_tables(pg, B_T2QK, inv, o.ssacc);
+            csync();
+            run_s2(pg, B_S2QKV);  // -> yq, yk, yv
+            csync();
+            for (int i = threadIdx.x; i < nkv; i += kCT) {
+                if (P.kv_out) {
+                    P.kv_out[((size_t)l * 2 + 0) * P.dkv + s.k0 + i] = yk[i];
+                    P.kv_out[((size_t)l * 2 + 1) * P.dkv + s.k0 + i] = yv[i];
                 }
-                build_tables(T);
-                csync();
-                v_stage(V, P.fix_limit, err);
+                yk[i] = yv[i] = 0.f;
             }
-            // ---- off the critical path, while exchange B is in flight:
-            //      k and v on K_c, and path 0 of q on R_c (path 1 of q runs
-            //      after exchange C is sent, from the saved t and rms)
-            {
-                const int rq1 = rk(LQ, 1);
-                if (rq1) {
-                    float *sv = sm_f(o.tsave);
-                    for (int i = threadIdx.x; i < rq1; i += kCT) sv[i] = tz[rk(LQ, 0) + i];
-                    if (lead) sv[rq1] = inv;
+            if (!rq1)
+                for (int i = threadIdx.x; i < rows_d; i += kCT) {
+                    if (P.q_out) P.q_out[(size_t)l * P.d + 32 * s.dw0 + i] = yq[i];
+                    yq[i] = 0.f;
                 }
-                TJ T[3];
-                UJ U[5];
-                int tbv = tb_v;
-                {
-                    const int r = rk(LQ, 0), R = wordsR(r);
-                    T[0] = TJ{tb, 8 * R, r, o.tz, o.b_lq[0], inv};
-                    U[0] = UJ{o.b_Uq[0], o.b_hq[0], R, rows_d, tb, o.yq};
-                    tb += R * 1024;
-                }
-#pragma unroll
-                for (int p = 0, off = nr[LQ]; p < 2; ++p) {
-                    const int r = rk(LK, p), R = r ? wordsR(r) : 1;
-                    T[1 + p] = TJ{tb, r ? 8 * R : 0, r, o.tz + 4 * off, o.b_lk[p], inv};
-                    U[1 + p] = UJ{o.b_Uk[p], o.b_hk[p], R, r ? nkv : 0, tb, o.ys};
-                    tb += r ? R * 1024 : 0;
-                    off += r;
-                }
-#pragma unroll
-                for (int p = 0; p < 2; ++p) {  // v on K_c reuses v's tables
-                    const int r = rk(LV, p), R = r ? wordsR(r) : 1;
-                    U[3 + p] = UJ{o.b_Uvk[p], o.b_hvk[p], R, r ? nkv : 0, tbv, o.ys + 4 * nkv};
-                    tbv += r ? R * 1024 : 0;
-                }
-                zero_f(yq, rows_d);
-                zero_f(ys, 2 * nkv);
-                build_tables(T);
-                csync();
-                u_stage(U);
-                csync();
-                if (P.kv_out)
-                    for (int i = threadIdx.x; i < nkv; i += kCT) {
-                        P.kv_out[((size_t)l * 2 + 0) * P.dkv + s.k0 + i] = ys[i];
-                        P.kv_out[((size_t)l * 2 + 1) * P.dkv + s.k0 + i] = ys[nkv + i];
-                    }
-                if (!rq1 && P.q_out)
-                    for (int i = threadIdx.x; i < rows_d; i += kCT)
-                        P.q_out[(size_t)l * P.d + 32 * s.dw0 + i] = yq[i];
-            }
         }
 
         // ================= phase C: h = a + O(attn) on R_c; stage 1 of gate, up
-        if (!poll_decode(xB, nr[LO], n_ctas, tz, P.ws_words)) FAIL_EXIT();
+        if (!poll_decode(xB, P.lenB, n_ctas, tz, P.ws_words)) FAIL_EXIT();
         zero_stripe(xA, P.lenA);
         if (!wait_full(full + 2, par, P.ws_words)) FAIL_EXIT();
-        {
-            {
-                TJ T[2];
-                UJ U[2];
-                int tb = o.tables;
-#pragma unroll
-                for (int p = 0, off = 0; p < 2; ++p) {
-                    const int r = rk(LO, p), R = r ? wordsR(r) : 1;
-                    T[p] = TJ{tb, r ? 8 * R : 0, r, o.tz + 4 * off, o.c_lo[p], 1.f};
-                    U[p] = UJ{o.c_Uo[p], o.c_ho[p], R, r ? rows_d : 0, tb, o.ys};
-                    tb += r ? R * 1024 : 0;
-                    off += r;
-                }
-                zero_f(ys, rows_d);
-                build_tables(T);
-                csync();
-                u_stage(U);
-                csync();
-            }
-            for (int i = threadIdx.x; i < rows_d; i += kCT) res[i] += ys[i];
-            csync();
-            const float ss = sum_sq(res, rows_d);
-            if (lead) red_fix(xC + ssC, ss, P.fix_limit, err);
-            TJ T[4];
-            VJ V[4];
-            int tb = o.tables;
-            unsigned long long *dst = xC;
-#pragma unroll
-            for (int k = 0; k < 2; ++k)
-#pragma unroll
-                for (int p = 0; p < 2; ++p) {
-                    const int r = rk(LG + k, p);
-                    const int g = k ? o.c_gu[p] : o.c_gg[p], Vw = k ? o.c_Vu[p] : o.c_Vg[p];
-                    T[2 * k + p] = TJ{tb, r ? 8 * nd : 0, rows_d, o.res, g, 1.f};
-                    V[2 * k + p] = VJ{Vw, r, nd, tb, dst};
-                    tb += r ? nd * 1024 : 0;
-                    dst += r;
-                }
-            build_tables(T);
-            csync();
-            v_stage(V, P.fix_limit, err);
-        }
+        run_tables(pg, C_T2, 1.f, o.ssacc);
+        csync();
+        run_s2(pg, C_S2);  // -> y
+        csync();
+        run_tables(pg, C_T1, 1.f, o.ssacc);  // h = res1 + y -> res0
+        csync();
+        send_ss(xC + ssC);
+        run_s1(pg, C_S1, xl, lim, err);
+        zero_f(y, rows_d);
         // ---- off the critical path, while exchange C is in flight: path 1 of q
-        if (rk(LQ, 1)) {
+        if (rq1) {
+            run_tables(pg, C_T2Q1, tsave[rq1], o.ssacc);
             csync();
-            const int r = rk(LQ, 1), R = wordsR(r);
-            TJ T[1] = {TJ{o.tables, 8 * R, r, o.tsave, o.b_lq[1], sm_f(o.tsave)[r]}};
-            UJ U[1] = {UJ{o.b_Uq[1], o.b_hq[1], R, rows_d, o.tables, o.yq}};
-            build_tables(T);
+            run_s2(pg, C_S2Q1);  // -> yq
             csync();
-            u_stage(U);
-            csync();
-            if (P.q_out)
-                for (int i = threadIdx.x; i < rows_d; i += kCT)
-                    P.q_out[(size_t)l * P.d + 32 * s.dw0 + i] = yq[i];
+            for (int i = threadIdx.x; i < rows_d; i += kCT) {
+                if (P.q_out) P.q_out[(size_t)l * P.d + 32 * s.dw0 + i] = yq[i];
+                yq[i] = 0.f;
+            }
         }
         release(1);
         release(2);
 
         // ================= phase D: m = silu(gate) * up on F_c; stage 1 of down
-        if (!poll_decode(xC, ssC + 1, n_ctas, tz, P.ws_words)) FAIL_EXIT();
+        if (!poll_decode(xC, P.lenC, n_ctas, tz, P.ws_words)) FAIL_EXIT();
         zero_stripe(xB, P.lenB);
         if (!wait_full(full + 3, par, P.ws_words)) FAIL_EXIT();
-        {
-            const float inv = rsqrtf(tz[ssC] / (float)P.d);
-            {
-                TJ T[4];
-                UJ U[4];
-                int tb = o.tables;
-#pragma unroll
-                for (int k = 0; k < 2; ++k)
-#pragma unroll
-                    for (int p = 0; p < 2; ++p) {
-                        const int r = rk(LG + k, p), R = r ? wordsR(r) : 1;
-                        const int off = (k ? nr[LG] : 0) + (p ? rk(LG + k, 0) : 0);
-                        const int lo16 = k ? o.d_lu[p] : o.d_lg[p];
-                        const int Uw = k ? o.d_Uu[p] : o.d_Ug[p], h = k ? o.d_hu[p] : o.d_hg[p];
-                        T[2 * k + p] = TJ{tb, r ? 8 * R : 0, r, o.tz + 4 * off, lo16, inv};
-                        U[2 * k + p] = UJ{Uw, h, R, r ? rows_f : 0, tb, o.ys + (k ? 4 * rows_f : 0)};
-                        tb += r ? R * 1024 : 0;
-                    }
-                zero_f(ys, 2 * rows_f);
-                build_tables(T);
-                csync();
-                u_stage(U);
-                csync();
-            }
-            for (int i = threadIdx.x; i < rows_f; i += kCT) xs[i] = silu(ys[i]) * ys[rows_f + i];
-            csync();
-            TJ T[2];
-            VJ V[2];
-            int tb = o.tables;
-            unsigned long long *dst = xD;
-#pragma unroll
-            for (int p = 0; p < 2; ++p) {
-                const int r = rk(LD, p);
-                T[p] = TJ{tb, r ? 8 * nf : 0, rows_f, o.xs, o.d_gd[p], 1.f};
-                V[p] = VJ{o.d_Vd[p], r, nf, tb, dst};
-                tb += r ? nf * 1024 : 0;
-                dst += r;
-            }
-            build_tables(T);
-            csync();
-            v_stage(V, P.fix_limit, err);
-        }
+        run_tables(pg, D_T2, rsqrtf(tz[ssC] / (float)P.d), o.ssacc);
+        csync();
+        run_s2(pg, D_S2);  // -> yg, yu
+        csync();
+        run_tables(pg, D_T1, 1.f, o.ssacc);  // m = silu(yg) * yu
+        csync();
+        run_s1(pg, D_S1, xl, lim, err);
+        zero_f(yg, rows_f);
+        zero_f(yu, rows_f);
         release(3);
     }
 
@@ -956,11 +806,14 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
     {
         const int l = P.n_layers;
         unsigned long long *xDl = P.xacc + (size_t)(l - 1) * P.acc_layer + P.offD;
-        if (!poll_decode(xDl, nr[LD], n_ctas, tz, P.ws_words)) FAIL_EXIT();
+        if (!poll_decode(xDl, P.lenD, n_ctas, tz, P.ws_words)) FAIL_EXIT();
         zero_stripe(P.xacc + (size_t)(l - 1) * P.acc_layer + P.offC, P.lenC);
         if (!wait_full(full + 0, (unsigned)(l & 1), P.ws_words)) FAIL_EXIT();
-        down_rows();
-        for (int i = threadIdx.x; i < rows_d; i += kCT) P.out[32 * s.dw0 + i] = res[i] + ys[i];
+        run_tables(pg, A_T2, 1.f, o.ssacc);
+        csync();
+        run_s2(pg, A_S2);
+        csync();
+        for (int i = threadIdx.x; i < rows_d; i += kCT) P.out[32 * s.dw0 + i] = res0[i] + y[i];
         // The last CTA to finish has seen every other CTA's reads of the final
         // region: it clears that region and the counters for the next launch.
         if (lead) {
@@ -1102,35 +955,350 @@ SmemPlan smem_plan(const lb_linear *lin, const StackShape &sh, int N) {
         o.d_Vd[p] = take(dd ? nf * r(LD, p) * 4 : 0);
         o.d_gd[p] = take(dd ? 64 * nf : 0);
     }
-    // nibble tables: the largest set one phase holds at once
-    auto utab = [&](int k) {
+    // nibble tables (1 KB per 32 values): the largest set a phase holds at once
+    auto utab = [&](int k, int p0, int p1) {
         int b = 0;
-        for (int p = 0; p < lin[k].n_paths; ++p) b += R(k, p) * 1024;
+        for (int p = p0; p < std::min(p1, lin[k].n_paths); ++p) b += R(k, p) * 1024;
         return b;
     };
     auto vtab = [&](int k, int nw) { return lin[k].n_paths * nw * 1024; };
-    int tabs = utab(LD);
-    tabs = std::max(tabs, vtab(LQ, nd) + vtab(LK, nd) + vtab(LV, nd));
-    tabs = std::max(tabs, utab(LV) + vtab(LO, nd) + utab(LQ) + utab(LK));
-    tabs = std::max(tabs, utab(LO));
-    tabs = std::max(tabs, vtab(LG, nd) + vtab(LU, nd));
-    tabs = std::max(tabs, utab(LG) + utab(LU));
-    tabs = std::max(tabs, vtab(LD, nf));
-    at = up(at, 256);
-    o.tables = at;
-    at += tabs;
+    int t2 = utab(LD, 0, 2);
+    t2 = std::max(t2, utab(LV, 0, 2) + utab(LQ, 0, 1) + utab(LK, 0, 2));
+    t2 = std::max(t2, utab(LO, 0, 2));
+    t2 = std::max(t2, utab(LQ, 1, 2));
+    t2 = std::max(t2, utab(LG, 0, 2) + utab(LU, 0, 2));
+    int t1 = vtab(LQ, nd) + vtab(LK, nd) + vtab(LV, nd);
+    t1 = std::max(t1, vtab(LO, nd));
+    t1 = std::max(t1, vtab(LG, nd) + vtab(LU, nd));
+    t1 = std::max(t1, vtab(LD, nf));
+    at = up(at, 1024);
+    o.t2 = at;
+    at += up(t2, 1024);
+    o.t1 = at;
+    at += up(t1, 1024);
     int tz_n = rsum(lin[LQ]) + rsum(lin[LK]) + rsum(lin[LV]) + 1;
     tz_n = std::max(tz_n, rsum(lin[LO]));
     tz_n = std::max(tz_n, rsum(lin[LG]) + rsum(lin[LU]) + 1);
     tz_n = std::max(tz_n, rsum(lin[LD]));
     o.tz = take(4 * (tz_n + 1));
-    o.res = take(4 * 32 * nd);
-    o.xs = take(4 * 32 * std::max(nd, nf));
-    o.ys = take(4 * std::max(32 * nd, std::max(2 * nkv, 2 * 32 * nf)));
+    o.res0 = take(4 * 32 * nd);
+    o.res1 = take(4 * 32 * nd);
+    o.y = take(4 * 32 * nd);
+    o.xa = take(4 * 32 * nd);
     o.yq = take(4 * 32 * nd);
+    o.yk = take(4 * nkv);
+    o.yv = take(4 * nkv);
+    o.yg = take(4 * 32 * nf);
+    o.yu = take(4 * 32 * nf);
     o.tsave = take(4 * (lin[LQ].path[lin[LQ].n_paths - 1].r + 4));
+    o.ssacc = take(16);
+    o.prog = take(kProgBytes);
     S.bytes = up(at, 128);
     return S;
+}
+
+// ---------------------------------------------------------------- the program
+
+Item tab(int tb, int n_tab, int n_vals, int mode, int s0, int s1, int s2, int scale) {
+    return Item{{tb, n_tab, n_vals, mode, s0, s1, s2, scale}};
+}
+
+struct Costed {
+    Item it;
+    double cost;
+};
+
+// Longest-processing-time assignment of units to the compute warps; returns
+// the units grouped by warp (warp-start offsets in wo) and the makespan.
+double lpt(const std::vector<Costed> &us, std::vector<Item> &out, int (&wo)[kCW + 1]) {
+    std::vector<int> idx(us.size());
+    for (size_t i = 0; i < us.size(); ++i) idx[i] = (int)i;
+    std::stable_sort(idx.begin(), idx.end(),
+                     [&](int a, int b) { return us[a].cost > us[b].cost; });
+    std::vector<std::vector<int>> per(kCW);
+    double load[kCW] = {};
+    for (int i : idx) {
+        int w = 0;
+        for (int k = 1; k < kCW; ++k)
+            if (load[k] < load[w]) w = k;
+        load[w] += us[i].cost;
+        per[w].push_back(i);
+    }
+    out.clear();
+    wo[0] = 0;
+    double mk = 0;
+    for (int w = 0; w < kCW; ++w) {
+        for (int i : per[w]) out.push_back(us[i].it);
+        wo[w + 1] = (int)out.size();
+        mk = std::max(mk, load[w]);
+    }
+    return mk;
+}
+
+struct S2Job {
+    int U, h, R, rows, tb, out;
+};
+struct S1Job {
+    int V, r, nw, tb, dst;
+};
+
+struct ProgBuild {
+    Step step[N_STEPS] = {};
+    std::vector<Item> items;
+
+    // Up to 32 tables of one job per unit, one unit per warp where possible.
+    void tables(int s, const std::vector<Item> &jobs) {
+        std::vector<Costed> us;
+        for (const Item &J : jobs) {
+            const int tb = J.f[0], nt = J.f[1], nv = J.f[2], mode = J.f[3];
+            for (int t0 = 0; t0 < nt; t0 += 32) {
+                auto sh = [&](int off, int per) { return off + per * t0; };  // unused: never read
+                us.push_back({Item{{tb + 128 * t0, std::min(32, nt - t0), nv - 4 * t0, mode,
+                                    sh(J.f[4], 16), sh(J.f[5], 16), sh(J.f[6], 16),
+                                    sh(J.f[7], 8)}},
+                              1.0 + std::min(32, nt - t0) / 32.0});
+            }
+        }
+        std::vector<Item> g;
+        int wo[kCW + 1];
+        lpt(us, g, wo);
+        place(s, g, wo);
+    }
+    void place(int s, const std::vector<Item> &grouped, const int (&wo)[kCW + 1]) {
+        step[s].first = (int)items.size();
+        for (int w = 0; w <= kCW; ++w) step[s].wo[w] = wo[w];
+        items.insert(items.end(), grouped.begin(), grouped.end());
+    }
+    // 32-row blocks x runs of words, the run length chosen to balance warps
+    // (cost of a unit: its words plus a fixed overhead).
+    void s2(int s, const std::vector<S2Job> &jobs) {
+        int maxR = 1;
+        for (const S2Job &J : jobs) maxR = std::max(maxR, J.R);
+        std::vector<Item> best;
+        int best_wo[kCW + 1] = {};
+        double best_mk = 1e300;
+        for (int run = 1; run <= maxR; ++run) {
+            std::vector<Costed> us;
+            for (const S2Job &J : jobs)
+                for (int r0 = 0; r0 < J.rows; r0 += 32)
+                    for (int w0 = 0; w0 < J.R; w0 += run) {
+                        const int nw = std::min(run, J.R - w0);
+                        us.push_back({Item{{J.U + (r0 * J.R + w0) * 4, J.R, nw, J.tb + w0 * 1024,
+                                            J.h + 2 * r0, J.out + 4 * r0,
+                                            std::min(32, J.rows - r0), 0}},
+                                      nw + 1.5});
+                    }
+            if (us.size() > 160 && run < maxR) continue;
+            std::vector<Item> g;
+            int wo[kCW + 1];
+            const double mk = lpt(us, g, wo);
+            if (mk < best_mk - 1e-9) {
+                best_mk = mk;
+                best = g;
+                std::copy(wo, wo + kCW + 1, best_wo);
+            }
+        }
+        place(s, best, best_wo);
+    }
+    // 32-column blocks over the whole input slice.
+    void s1(int s, const std::vector<S1Job> &jobs) {
+        std::vector<Costed> us;
+        for (const S1Job &J : jobs)
+            for (int c0 = 0; c0 < J.r; c0 += 32)
+                us.push_back({Item{{J.V + 4 * c0, J.r, J.nw, J.tb, J.dst + c0,
+                                    std::min(32, J.r - c0), 0, 0}},
+                              J.nw + 1.0});
+        std::vector<Item> g;
+        int wo[kCW + 1];
+        lpt(us, g, wo);
+        place(s, g, wo);
+    }
+};
+
+// The program of CTA c (kProgBytes, zero-padded); false when it does not fit.
+bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, const Offsets &o,
+                   const XLayout &X, std::vector<int> &prog_out) {
+    const int Wd = sh.d / 32, Wf = sh.dff / 32, Ukv = sh.dkv / 8;
+    const int dw0 = (int)((long long)c * Wd / N), nd = (int)((long long)(c + 1) * Wd / N) - dw0;
+    const int fw0 = (int)((long long)c * Wf / N), nf = (int)((long long)(c + 1) * Wf / N) - fw0;
+    const int nkv = 8 * ((int)((long long)(c + 1) * Ukv / N) - (int)((long long)c * Ukv / N));
+    const int rows_d = 32 * nd, rows_f = 32 * nf;
+    auto np = [&](int k) { return lin[k].n_paths; };
+    auto rk = [&](int k, int p) { return lin[k].path[p].r; };
+    auto Rk = [&](int k, int p) { return (lin[k].path[p].r + 31) / 32; };
+    ProgBuild B;
+    std::vector<Item> T;
+    std::vector<S2Job> U;
+    std::vector<S1Job> V;
+    auto flush_t = [&](int s) {
+        B.tables(s, T);
+        T.clear();
+    };
+    auto flush_u = [&](int s) {
+        B.s2(s, U);
+        U.clear();
+    };
+    auto flush_v = [&](int s) {
+        B.s1(s, V);
+        V.clear();
+    };
+    // phase A: stage 2 of down (previous layer) -> y; stage 1 of q, k, v of
+    // a = res0 + y (written to res1)
+    {
+        int tb = o.t2, off = 0;
+        for (int p = 0; p < np(LD); ++p) {
+            T.push_back(tab(tb, 8 * Rk(LD, p), rk(LD, p), TAB_PLAIN, o.tz + 4 * off, 0, 0,
+                            o.a_ld[p]));
+            U.push_back({o.a_Ud[p], o.a_hd[p], Rk(LD, p), rows_d, tb, o.y});
+            tb += Rk(LD, p) * 1024;
+            off += rk(LD, p);
+        }
+        flush_t(A_T2);
+        flush_u(A_S2);
+        int tb1 = o.t1, dst = X.offA, mode = TAB_RES | TAB_WRITER;
+        for (int k = 0; k < 3; ++k)
+            for (int p = 0; p < np(k); ++p) {
+                T.push_back(tab(tb1, 8 * nd, rows_d, mode, o.res0, o.y, o.res1, o.a_g[k][p]));
+                V.push_back({o.a_V[k][p], rk(k, p), nd, tb1, dst});
+                mode = TAB_RES;
+                tb1 += nd * 1024;
+                dst += rk(k, p);
+            }
+        flush_t(A_T1);
+        flush_v(A_S1);
+    }
+    // phase B: v on the attention rows of R_c -> xa; stage 1 of o; then
+    // path 0 of q -> yq, k -> yk, v on K_c -> yv
+    {
+        const int nq = rsum(lin[LQ]), nk = rsum(lin[LK]);
+        int tb = o.t2, off = nq + nk, tbv[2] = {0, 0};
+        for (int p = 0; p < np(LV); ++p) {
+            T.push_back(tab(tb, 8 * Rk(LV, p), rk(LV, p), TAB_PLAIN | TAB_MUL, o.tz + 4 * off, 0,
+                            0, o.b_lv[p]));
+            U.push_back({o.b_Uat[p], o.b_hat[p], Rk(LV, p), rows_d, tb, o.xa});
+            tbv[p] = tb;
+            tb += Rk(LV, p) * 1024;
+            off += rk(LV, p);
+        }
+        flush_t(B_T2V);
+        flush_u(B_S2V);
+        int tb1 = o.t1, dst = X.offB;
+        for (int p = 0; p < np(LO); ++p) {
+            T.push_back(tab(tb1, 8 * nd, rows_d, TAB_PLAIN, o.xa, 0, 0, o.b_go[p]));
+            V.push_back({o.b_Vo[p], rk(LO, p), nd, tb1, dst});
+            tb1 += nd * 1024;
+            dst += rk(LO, p);
+        }
+        flush_t(B_T1);
+        flush_v(B_S1);
+        T.push_back(tab(tb, 8 * Rk(LQ, 0), rk(LQ, 0), TAB_PLAIN | TAB_MUL, o.tz, 0, 0, o.b_lq[0]));
+        U.push_back({o.b_Uq[0], o.b_hq[0], Rk(LQ, 0), rows_d, tb, o.yq});
+        tb += Rk(LQ, 0) * 1024;
+        off = nq;
+        for (int p = 0; p < np(LK); ++p) {
+            T.push_back(tab(tb, 8 * Rk(LK, p), rk(LK, p), TAB_PLAIN | TAB_MUL, o.tz + 4 * off, 0,
+                            0, o.b_lk[p]));
+            U.push_back({o.b_Uk[p], o.b_hk[p], Rk(LK, p), nkv, tb, o.yk});
+            tb += Rk(LK, p) * 1024;
+            off += rk(LK, p);
+        }
+        for (int p = 0; p < np(LV); ++p)
+            U.push_back({o.b_Uvk[p], o.b_hvk[p], Rk(LV, p), nkv, tbv[p], o.yv});
+        flush_t(B_T2QK);
+        flush_u(B_S2QKV);
+    }
+    // phase C: stage 2 of o -> y; stage 1 of gate, up of h = res1 + y
+    // (written to res0); path 1 of q from the saved t -> yq
+    {
+        int tb = o.t2, off = 0;
+        for (int p = 0; p < np(LO); ++p) {
+            T.push_back(tab(tb, 8 * Rk(LO, p), rk(LO, p), TAB_PLAIN, o.tz + 4 * off, 0, 0,
+                            o.c_lo[p]));
+            U.push_back({o.c_Uo[p], o.c_ho[p], Rk(LO, p), rows_d, tb, o.y});
+            tb += Rk(LO, p) * 1024;
+            off += rk(LO, p);
+        }
+        flush_t(C_T2);
+        flush_u(C_S2);
+        int tb1 = o.t1, dst = X.offC, mode = TAB_RES | TAB_WRITER;
+        for (int k = LG; k <= LU; ++k)
+            for (int p = 0; p < np(k); ++p) {
+                T.push_back(tab(tb1, 8 * nd, rows_d, mode, o.res1, o.y, o.res0,
+                                k == LG ? o.c_gg[p] : o.c_gu[p]));
+                V.push_back({k == LG ? o.c_Vg[p] : o.c_Vu[p], rk(k, p), nd, tb1, dst});
+                mode = TAB_RES;
+                tb1 += nd * 1024;
+                dst += rk(k, p);
+            }
+        flush_t(C_T1);
+        flush_v(C_S1);
+        if (np(LQ) > 1) {
+            T.push_back(tab(o.t2, 8 * Rk(LQ, 1), rk(LQ, 1), TAB_PLAIN | TAB_MUL, o.tsave, 0, 0,
+                            o.b_lq[1]));
+            U.push_back({o.b_Uq[1], o.b_hq[1], Rk(LQ, 1), rows_d, o.t2, o.yq});
+        }
+        flush_t(C_T2Q1);
+        flush_u(C_S2Q1);
+    }
+    // phase D: stage 2 of gate, up on F_c -> yg, yu; stage 1 of down of
+    // m = silu(yg) * yu
+    {
+        int tb = o.t2, off = 0;
+        for (int k = LG; k <= LU; ++k)
+            for (int p = 0; p < np(k); ++p) {
+                T.push_back(tab(tb, 8 * Rk(k, p), rk(k, p), TAB_PLAIN | TAB_MUL, o.tz + 4 * off,
+                                0, 0, k == LG ? o.d_lg[p] : o.d_lu[p]));
+                U.push_back({k == LG ? o.d_Ug[p] : o.d_Uu[p], k == LG ? o.d_hg[p] : o.d_hu[p],
+                             Rk(k, p), rows_f, tb, k == LG ? o.yg : o.yu});
+                tb += Rk(k, p) * 1024;
+                off += rk(k, p);
+            }
+        flush_t(D_T2);
+        flush_u(D_S2);
+        int tb1 = o.t1, dst = X.offD;
+        for (int p = 0; p < np(LD); ++p) {
+            T.push_back(tab(tb1, 8 * nf, rows_f, TAB_SILU, o.yg, o.yu, 0, o.d_gd[p]));
+            V.push_back({o.d_Vd[p], rk(LD, p), nf, tb1, dst});
+            tb1 += nf * 1024;
+            dst += rk(LD, p);
+        }
+        flush_t(D_T1);
+        flush_v(D_S1);
+    }
+    if ((int)B.items.size() > kMaxItems) return false;
+    prog_out.assign(kProgBytes / 4, 0);
+    std::memcpy(prog_out.data(), B.step, sizeof(B.step));
+    std::memcpy(prog_out.data() + kStepBytes / 4, B.items.data(), B.items.size() * sizeof(Item));
+    return true;
+}
+
+bool build_programs(const lb_linear *lin, const StackShape &sh, int N, std::vector<int> &all) {
+    const SmemPlan S = smem_plan(lin, sh, N);
+    const XLayout X = xlayout(lin);
+    all.assign((size_t)N * (kProgBytes / 4), 0);
+    std::vector<int> one;
+    for (int c = 0; c < N; ++c) {
+        if (!build_program(lin, sh, N, c, S.o, X, one)) return false;
+        std::copy(one.begin(), one.end(), all.begin() + (size_t)c * (kProgBytes / 4));
+    }
+    return true;
+}
+
+bool smem_fits(const lb_linear *lin, const StackShape &sh, int num_sms) {
+    const SmemPlan S = smem_plan(lin, sh, num_sms);
+    int max_optin = 0, dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&max_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
+            cudaSuccess)
+        return false;
+    return S.bytes + 1024 <= max_optin;
+}
+
+bool shapes_ok(const lb_linear *lin, const StackShape &sh, int num_sms) {
+    for (int k = 0; k < 7; ++k)
+        for (int p = 0; p < lin[k].n_paths; ++p)
+            if (lin[k].path[p].r % 8 != 0) return false;
+    return sh.head_dim % 32 == 0 && sh.dkv % 8 == 0 && num_sms >= 1 && num_sms <= kMaxCtas;
 }
 
 }  // namespace
@@ -1139,11 +1307,24 @@ static_assert(sizeof(LinDesc) % sizeof(uint32_t) == 0, "descriptor is copied as 
 
 size_t stack_ws_bytes_after_header(const lb_linear *lin, int n_layers) {
     const XLayout X = xlayout(lin);
-    return desc_bytes_for(n_layers) + (size_t)n_layers * X.acc_layer * sizeof(unsigned long long);
+    return desc_bytes_for(n_layers) + (size_t)n_layers * X.acc_layer * sizeof(unsigned long long) +
+           (size_t)kMaxCtas * kProgBytes;
 }
 
-cudaError_t launch_stack_prepare(const lb_linear *lin, int n_layers, unsigned long long plan,
-                                 unsigned *ws_words, char *ws_after_header, cudaStream_t s) {
+namespace {
+char *programs_at(const lb_linear *lin, int n_layers, char *ws_after_header) {
+    const XLayout X = xlayout(lin);
+    return ws_after_header + desc_bytes_for(n_layers) +
+           (size_t)n_layers * X.acc_layer * sizeof(unsigned long long);
+}
+}  // namespace
+
+cudaError_t launch_stack_prepare(const lb_linear *lin, int n_layers, const StackShape &sh,
+                                 int num_sms, unsigned long long plan, unsigned *ws_words,
+                                 char *ws_after_header, cudaStream_t s) {
+    if (!shapes_ok(lin, sh, num_sms) || !smem_fits(lin, sh, num_sms)) return cudaErrorNotSupported;
+    std::vector<int> progs;
+    if (!build_programs(lin, sh, num_sms, progs)) return cudaErrorNotSupported;
     const XLayout X = xlayout(lin);
     LinDesc *desc = reinterpret_cast<LinDesc *>(ws_after_header);
     char *xacc = ws_after_header + desc_bytes_for(n_layers);
@@ -1151,6 +1332,10 @@ cudaError_t launch_stack_prepare(const lb_linear *lin, int n_layers, unsigned lo
     if (e == cudaSuccess)
         e = cudaMemsetAsync(xacc, 0, (size_t)n_layers * X.acc_layer * sizeof(unsigned long long),
                             s);
+    // pageable source: the call returns once the data is staged
+    if (e == cudaSuccess)
+        e = cudaMemcpyAsync(programs_at(lin, n_layers, ws_after_header), progs.data(),
+                            progs.size() * sizeof(int), cudaMemcpyHostToDevice, s);
     if (e != cudaSuccess) return e;
     const int n_lin = 7 * n_layers;
     for (int first = 0; first < n_lin; first += kDescChunk) {
@@ -1166,17 +1351,7 @@ cudaError_t launch_stack_prepare(const lb_linear *lin, int n_layers, unsigned lo
 }
 
 bool stack_supported(const lb_linear *lin, const StackShape &sh, int num_sms) {
-    for (int k = 0; k < 7; ++k)
-        for (int p = 0; p < lin[k].n_paths; ++p)
-            if (lin[k].path[p].r % 8 != 0) return false;
-    if (sh.head_dim % 32 != 0 || sh.dkv % 8 != 0 || num_sms > 255) return false;
-    const SmemPlan S = smem_plan(lin, sh, num_sms);
-    int max_optin = 0, dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess ||
-        cudaDeviceGetAttribute(&max_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
-            cudaSuccess)
-        return false;
-    return S.bytes + 1024 <= max_optin;
+    return shapes_ok(lin, sh, num_sms) && smem_fits(lin, sh, num_sms);
 }
 
 cudaError_t launch_stack(const lb_linear *lin, int n_layers, const StackShape &sh,
@@ -1187,6 +1362,7 @@ cudaError_t launch_stack(const lb_linear *lin, int n_layers, const StackShape &s
     const SmemPlan S = smem_plan(lin, sh, num_sms);
     Params P{};
     P.lin = reinterpret_cast<const LinDesc *>(ws_after_header);
+    P.prog = reinterpret_cast<const int *>(programs_at(lin, n_layers, ws_after_header));
     P.n_layers = n_layers;
     P.d = sh.d;
     P.dkv = sh.dkv;
