@@ -111,6 +111,12 @@ __device__ __forceinline__ void red_add_u64(unsigned long long *p, unsigned long
     asm volatile("red.relaxed.gpu.global.add.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
 
+__device__ __forceinline__ unsigned long long ld_relaxed_u64(const unsigned long long *p) {
+    unsigned long long v;
+    asm volatile("ld.relaxed.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+
 __device__ __forceinline__ void ld_relaxed_v2_u64(const unsigned long long *p,
                                                   unsigned long long &a, unsigned long long &b) {
     asm volatile("ld.relaxed.gpu.global.v2.u64 {%0, %1}, [%2];"
@@ -139,15 +145,17 @@ struct Offsets {
     // stream (two buffers: phase A reads 0 and writes 1, phase C the reverse),
     // stage-2 outputs (added into, zeroed by their consumer), saved t of q's
     // second path, the sum-of-squares accumulator, the program
-    int t2, t1, tz, res0, res1, y, xa, yq, yk, yv, yg, yu, tsave, ssacc, prog;
+    int t2, t1, res0, res1, y, xa, yq, yk, yv, yg, yu, ssacc, prog;
 };
 
 // Steps of the per-CTA program (one per table build or unit loop).
+// (*_P2: stage-2 tables straight from the exchange words; *_T1: stage-1
+// tables; *_S2 / *_S1: stage-2 / stage-1 units.)
 enum StepId {
-    A_T2, A_S2, A_T1, A_S1,
-    B_T2V, B_S2V, B_T1, B_S1, B_T2QK, B_S2QKV,
-    C_T2, C_S2, C_T1, C_S1, C_T2Q1, C_S2Q1,
-    D_T2, D_S2, D_T1, D_S1,
+    A_P2, A_S2, A_T1, A_S1,
+    B_P2, B_S2V, B_T1, B_S1, B_S2QKV,
+    C_P2, C_S2, C_T1, C_S1,
+    D_P2, D_S2, D_T1, D_S1,
     N_STEPS
 };
 
@@ -155,6 +163,8 @@ enum StepId {
 //   table unit  : tb, n_tab, n_vals, mode, s0, s1, s2, scale   (up to 32
 //                 tables of one job, from its table t0 on; the offsets and
 //                 n_vals are those of table t0)
+//   poll-table  : tb, n_tab, n_vals, mode, e0, scale, ss_el, -  (e0, ss_el:
+//                 exchange word indices in the layer; ss_el < 0: none)
 //   stage-2 unit: U, R, nw, tb, h, out, nrows, -
 //   stage-1 unit: V, r, nw, tb, dst, ncols, -, -
 struct Item {
@@ -183,7 +193,7 @@ struct Params {
     unsigned *ws_words;
     unsigned long long plan;
     unsigned long long *xacc;  // exchange words, n_layers * acc_layer
-    int acc_layer, offA, offB, offC, offD, lenA, lenB, lenC, lenD;
+    int acc_layer, offA, offQ, offB, offC, offD, lenA, lenQ, lenB, lenC, lenD;
     float fix_limit;  // |contribution| bound that keeps the fixed-point sum in range
     Offsets o;
 };
@@ -398,23 +408,65 @@ __device__ __forceinline__ void record(unsigned *ws_words, lb_status st) {
     atomicCAS(ws_words + kErrWord, 0u, static_cast<unsigned>(st));
 }
 
-// Wait until each of region[0..n) counts n_ctas contributions and decode the
-// sums into out[0..n).  Bounded; returns false (to every compute thread) on
-// failure.
-__device__ __noinline__ bool poll_decode(const unsigned long long *region, int n, unsigned n_ctas,
-                                         float *out, unsigned *ws_words) {
+__device__ __forceinline__ float dec_fix(unsigned long long w) {
+    return __ll2float_rn((long long)w >> 8) * kFixInv;
+}
+__device__ __forceinline__ bool counted(unsigned long long w, unsigned n_ctas) {
+    return (unsigned)(w & 0xffull) == n_ctas;
+}
+
+// Stores table n of a unit at T from its four values (see run_tables).
+__device__ __forceinline__ void store_table(unsigned char *T, float4 x, int lane) {
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        const int q = (k + lane) & 7;
+        // chunk q: entries 4(q&3) .. +3; high bits (e3 e2) = q & 3
+        const float qv = ((q & 1) ? -x.z : x.z) + ((q & 2) ? -x.w : x.w);
+        *reinterpret_cast<float4 *>(T + 16 * q) =
+            make_float4(x.x + x.y + qv, x.y - x.x + qv, x.x - x.y + qv, -x.x - x.y + qv);
+    }
+}
+
+// Poll-table units: the stage-2 tables of a phase built straight from the
+// exchange words.  Lane n waits until the words e0 + 4n .. +3 (those below
+// n_vals) -- and the word ss_el, for a TAB_MUL unit that has one -- count
+// n_ctas contributions, decodes them and builds table n of v_i = t_i * l_i
+// (* inv with TAB_MUL, inv = rsqrt(ss * inv_d) of word ss_el, or the
+// argument when the unit has no ss_el).  Bounded; returns false (to every
+// compute thread) on failure.
+__device__ __noinline__ bool run_poll_tables(int prog, int s, const unsigned long long *xbase,
+                                             unsigned n_ctas, float inv, float inv_d,
+                                             unsigned *ws_words) {
+    const Step &st = step_at(prog, s);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     int ok = 1;
-    for (int i = 2 * threadIdx.x; i < n && ok; i += 2 * kCT) {
-        unsigned long long t0 = 0;
-        for (int spin = 0;; ++spin) {
-            unsigned long long a, b;
-            ld_relaxed_v2_u64(region + i, a, b);
-            const bool done = (a & 0xffull) == n_ctas && (i + 1 >= n || (b & 0xffull) == n_ctas);
-            if (done) {
-                out[i] = __ll2float_rn((long long)a >> 8) * kFixInv;
-                if (i + 1 < n) out[i + 1] = __ll2float_rn((long long)b >> 8) * kFixInv;
-                break;
+    const int u1 = st.first + st.wo[warp + 1];
+    for (int u = st.first + st.wo[warp]; u < u1 && ok; ++u) {
+        int4 a, b;
+        item_at(prog, u, a, b);
+        // lane 0 first waits, gently, for the unit's first word: the words
+        // of a region complete at about the same time, and one poller per
+        // warp keeps the L2 free for the contributions still arriving
+        if (lane == 0 && a.z > 0) {
+            const unsigned long long t0 = globaltimer_ns();
+            while (!counted(ld_relaxed_u64(xbase + b.x), n_ctas)) {
+                __nanosleep(64);
+                if (globaltimer_ns() - t0 > kWaitLimitNs) break;  // the full wait below decides
             }
+        }
+        __syncwarp();
+        if (lane >= a.y) continue;
+        const bool have = a.z - 4 * lane > 0;
+        const bool need_ss = have && (a.w & TAB_MUL) && b.z >= 0;
+        const unsigned long long *w = xbase + b.x + 4 * lane;
+        unsigned long long v0 = 0, v1 = 0, v2 = 0, v3 = 0, vs = 0, t0 = 0;
+        for (int spin = 0; have; ++spin) {
+            ld_relaxed_v2_u64(w, v0, v1);
+            ld_relaxed_v2_u64(w + 2, v2, v3);
+            if (need_ss) vs = ld_relaxed_u64(xbase + b.z);
+            if (counted(v0, n_ctas) && counted(v1, n_ctas) && counted(v2, n_ctas) &&
+                counted(v3, n_ctas) && (!need_ss || counted(vs, n_ctas)))
+                break;
             if ((spin & 15) == 15) {
                 if (sticky(ws_words)) {
                     ok = 0;
@@ -429,6 +481,17 @@ __device__ __noinline__ bool poll_decode(const unsigned long long *region, int n
                 }
             }
         }
+        if (!ok) break;
+        float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (have) {
+            const uint2 hb = *reinterpret_cast<const uint2 *>(g_smem + b.y + 8 * lane);
+            const float m = (a.w & TAB_MUL) ? (need_ss ? rsqrtf(dec_fix(vs) * inv_d) : inv) : 1.f;
+            x.x = dec_fix(v0) * half_bits_to_float((uint16_t)(hb.x & 0xffffu)) * m;
+            x.y = dec_fix(v1) * half_bits_to_float((uint16_t)(hb.x >> 16)) * m;
+            x.z = dec_fix(v2) * half_bits_to_float((uint16_t)(hb.y & 0xffffu)) * m;
+            x.w = dec_fix(v3) * half_bits_to_float((uint16_t)(hb.y >> 16)) * m;
+        }
+        store_table(g_smem + a.x + lane * 128, x, lane);
     }
     return csync_and(ok) != 0;
 }
@@ -665,7 +728,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
     const int rows_d = 32 * s.nd, rows_f = 32 * s.nf, nkv = s.nkv;
     float *res0 = sm_f(o.res0), *y = sm_f(o.y), *xa = sm_f(o.xa), *yq = sm_f(o.yq);
     float *yk = sm_f(o.yk), *yv = sm_f(o.yv), *yg = sm_f(o.yg), *yu = sm_f(o.yu);
-    float *tz = sm_f(o.tz), *tsave = sm_f(o.tsave), *ssacc = sm_f(o.ssacc);
+    float *ssacc = sm_f(o.ssacc);  // sum of squares of this CTA's slice
     for (int i = threadIdx.x; i < rows_d; i += kCT) {
         res0[i] = bf16_bits_to_float(P.x0[32 * s.dw0 + i]);
         y[i] = xa[i] = yq[i] = 0.f;
@@ -674,124 +737,92 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
     zero_f(yv, nkv);
     zero_f(yg, rows_f);
     zero_f(yu, rows_f);
-    if (threadIdx.x == 0) *ssacc = 0.f;
+    if (threadIdx.x == 0) ssacc[0] = 0.f;
     csync();
     int nr[7];
 #pragma unroll
     for (int k = 0; k < 7; ++k) nr[k] = P.r[k][0] + (P.np[k] > 1 ? P.r[k][1] : 0);
-    const int ssA = nr[LQ] + nr[LK] + nr[LV], ssC = nr[LG] + nr[LU];
-    const int rq0 = P.r[LQ][0], rq1 = P.np[LQ] > 1 ? P.r[LQ][1] : 0;
+    const int ssA = nr[LV], ssC = nr[LG] + nr[LU];
     const bool lead = threadIdx.x == 0;
-    const float lim = P.fix_limit;
+    const float lim = P.fix_limit, inv_d = 1.f / (float)P.d;
     auto release = [&](int b) {
         csync();
         if (lead) mbar_arrive(empty + b);
     };
     auto send_ss = [&](unsigned long long *p) {
         if (lead) {
-            red_add_u64(p, enc_fix(*ssacc, lim, err));
-            *ssacc = 0.f;
+            red_add_u64(p, enc_fix(ssacc[0], lim, err));
+            ssacc[0] = 0.f;
         }
     };
 #define FAIL_EXIT() return
 
     for (int l = 0; l < P.n_layers; ++l) {
         unsigned long long *xl = P.xacc + (size_t)l * P.acc_layer;
-        unsigned long long *xA = xl + P.offA, *xB = xl + P.offB, *xC = xl + P.offC,
-                           *xD = xl + P.offD;
+        unsigned long long *xp = xl - P.acc_layer;  // the previous layer's words
         const unsigned par = (unsigned)(l & 1);
 
         // ================= phase A: a = h + Down_{l-1}(m) on R_c; stage 1 of q, k, v
-        if (l > 0) {
-            if (!poll_decode(xD - P.acc_layer, P.lenD, n_ctas, tz, P.ws_words)) FAIL_EXIT();
-            zero_stripe(xC - P.acc_layer, P.lenC);
-        }
         if (!wait_full(full + 0, par, P.ws_words)) FAIL_EXIT();
         if (l > 0) {
-            run_tables(pg, A_T2, 1.f, o.ssacc);
-            csync();
+            if (!run_poll_tables(pg, A_P2, xp, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
+            zero_stripe(xp + P.offC, P.lenC);
+            zero_stripe(xp + P.offQ, P.lenQ);
             run_s2(pg, A_S2);
             csync();
         }
         run_tables(pg, A_T1, 1.f, o.ssacc);  // a = res0 + y -> res1
         csync();
-        send_ss(xA + ssA);
+        send_ss(xl + P.offA + ssA);
         run_s1(pg, A_S1, xl, lim, err);
         zero_f(y, rows_d);
         release(0);
 
         // ================= phase B: v rows for attention, stage 1 of o; then q, k, v out
-        if (!poll_decode(xA, P.lenA, n_ctas, tz, P.ws_words)) FAIL_EXIT();
-        if (l > 0) zero_stripe(xD - P.acc_layer, P.lenD);
         if (!wait_full(full + 1, par, P.ws_words)) FAIL_EXIT();
-        {
-            const float inv = rsqrtf(tz[ssA] / (float)P.d);
-            if (rq1) {
-                for (int i = threadIdx.x; i < rq1; i += kCT) tsave[i] = tz[rq0 + i];
-                if (lead) tsave[rq1] = inv;
+        // tables of v (critical) and of q, k (region Q, sent with region A)
+        if (!run_poll_tables(pg, B_P2, xl, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
+        if (l > 0) zero_stripe(xp + P.offD, P.lenD);
+        run_s2(pg, B_S2V);  // -> xa
+        csync();
+        run_tables(pg, B_T1, 1.f, o.ssacc);
+        csync();
+        run_s1(pg, B_S1, xl, lim, err);
+        zero_f(xa, rows_d);
+        // ---- off the critical path, while exchange B is in flight: q on R_c,
+        //      k and v on K_c (their tables were built with v's)
+        run_s2(pg, B_S2QKV);  // -> yq, yk, yv
+        csync();
+        for (int i = threadIdx.x; i < nkv; i += kCT) {
+            if (P.kv_out) {
+                P.kv_out[((size_t)l * 2 + 0) * P.dkv + s.k0 + i] = yk[i];
+                P.kv_out[((size_t)l * 2 + 1) * P.dkv + s.k0 + i] = yv[i];
             }
-            run_tables(pg, B_T2V, inv, o.ssacc);
-            csync();
-            run_s2(pg, B_S2V);  // -> xa
-            csync();
-            run_tables(pg, B_T1, 1.f, o.ssacc);
-            csync();
-            run_s1(pg, B_S1, xl, lim, err);
-            zero_f(xa, rows_d);
-            // ---- off the critical path, while exchange B is in flight: k and
-            //      v on K_c, path 0 of q on R_c (path 1 of q runs after
-            //      exchange C is sent, from the saved t and rms)
-            run_tables(pg, B_T2QK, inv, o.ssacc);
-            csync();
-            run_s2(pg, B_S2QKV);  // -> yq, yk, yv
-            csync();
-            for (int i = threadIdx.x; i < nkv; i += kCT) {
-                if (P.kv_out) {
-                    P.kv_out[((size_t)l * 2 + 0) * P.dkv + s.k0 + i] = yk[i];
-                    P.kv_out[((size_t)l * 2 + 1) * P.dkv + s.k0 + i] = yv[i];
-                }
-                yk[i] = yv[i] = 0.f;
-            }
-            if (!rq1)
-                for (int i = threadIdx.x; i < rows_d; i += kCT) {
-                    if (P.q_out) P.q_out[(size_t)l * P.d + 32 * s.dw0 + i] = yq[i];
-                    yq[i] = 0.f;
-                }
+            yk[i] = yv[i] = 0.f;
         }
+        for (int i = threadIdx.x; i < rows_d; i += kCT) {
+            if (P.q_out) P.q_out[(size_t)l * P.d + 32 * s.dw0 + i] = yq[i];
+            yq[i] = 0.f;
+        }
+        release(1);
 
         // ================= phase C: h = a + O(attn) on R_c; stage 1 of gate, up
-        if (!poll_decode(xB, P.lenB, n_ctas, tz, P.ws_words)) FAIL_EXIT();
-        zero_stripe(xA, P.lenA);
         if (!wait_full(full + 2, par, P.ws_words)) FAIL_EXIT();
-        run_tables(pg, C_T2, 1.f, o.ssacc);
-        csync();
+        if (!run_poll_tables(pg, C_P2, xl, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
+        zero_stripe(xl + P.offA, P.lenA);
         run_s2(pg, C_S2);  // -> y
         csync();
         run_tables(pg, C_T1, 1.f, o.ssacc);  // h = res1 + y -> res0
         csync();
-        send_ss(xC + ssC);
+        send_ss(xl + P.offC + ssC);
         run_s1(pg, C_S1, xl, lim, err);
         zero_f(y, rows_d);
-        // ---- off the critical path, while exchange C is in flight: path 1 of q
-        if (rq1) {
-            run_tables(pg, C_T2Q1, tsave[rq1], o.ssacc);
-            csync();
-            run_s2(pg, C_S2Q1);  // -> yq
-            csync();
-            for (int i = threadIdx.x; i < rows_d; i += kCT) {
-                if (P.q_out) P.q_out[(size_t)l * P.d + 32 * s.dw0 + i] = yq[i];
-                yq[i] = 0.f;
-            }
-        }
-        release(1);
         release(2);
 
         // ================= phase D: m = silu(gate) * up on F_c; stage 1 of down
-        if (!poll_decode(xC, P.lenC, n_ctas, tz, P.ws_words)) FAIL_EXIT();
-        zero_stripe(xB, P.lenB);
         if (!wait_full(full + 3, par, P.ws_words)) FAIL_EXIT();
-        run_tables(pg, D_T2, rsqrtf(tz[ssC] / (float)P.d), o.ssacc);
-        csync();
+        if (!run_poll_tables(pg, D_P2, xl, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
+        zero_stripe(xl + P.offB, P.lenB);
         run_s2(pg, D_S2);  // -> yg, yu
         csync();
         run_tables(pg, D_T1, 1.f, o.ssacc);  // m = silu(yg) * yu
@@ -805,12 +836,11 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
     // ================= final: out = h + Down_{L-1}(m) on R_c
     {
         const int l = P.n_layers;
-        unsigned long long *xDl = P.xacc + (size_t)(l - 1) * P.acc_layer + P.offD;
-        if (!poll_decode(xDl, P.lenD, n_ctas, tz, P.ws_words)) FAIL_EXIT();
-        zero_stripe(P.xacc + (size_t)(l - 1) * P.acc_layer + P.offC, P.lenC);
+        unsigned long long *xp = P.xacc + (size_t)(l - 1) * P.acc_layer;
         if (!wait_full(full + 0, (unsigned)(l & 1), P.ws_words)) FAIL_EXIT();
-        run_tables(pg, A_T2, 1.f, o.ssacc);
-        csync();
+        if (!run_poll_tables(pg, A_P2, xp, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
+        zero_stripe(xp + P.offC, P.lenC);
+        zero_stripe(xp + P.offQ, P.lenQ);
         run_s2(pg, A_S2);
         csync();
         for (int i = threadIdx.x; i < rows_d; i += kCT) P.out[32 * s.dw0 + i] = res0[i] + y[i];
@@ -823,7 +853,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         csync();
         if (s_last) {
             __threadfence();
-            for (int i = threadIdx.x; i < P.lenD; i += kCT) xDl[i] = 0ull;
+            for (int i = threadIdx.x; i < P.lenD; i += kCT) xp[P.offD + i] = 0ull;
             if (lead) P.ws_words[kDoneWord] = 0u;
         }
     }
@@ -860,20 +890,23 @@ int rsum(const lb_linear &L) {
 
 int up(int n, int a) { return (n + a - 1) / a * a; }
 
-// Exchange words per layer: A = t of q, k, v + ss(a); B = t of o;
-// C = t of gate, up + ss(h); D = t of down; each region padded to 32 words.
+// Exchange words per layer: A = t of v + ss(a); Q = t of q, k (read off
+// the critical path); B = t of o; C = t of gate, up + ss(h); D = t of down;
+// each region padded to 32 words.
 struct XLayout {
-    int acc_layer, offA, offB, offC, offD, lenA, lenB, lenC, lenD;
+    int acc_layer, offA, offQ, offB, offC, offD, lenA, lenQ, lenB, lenC, lenD;
 };
 
 XLayout xlayout(const lb_linear *lin) {
     XLayout X{};
-    X.lenA = rsum(lin[LQ]) + rsum(lin[LK]) + rsum(lin[LV]) + 1;
+    X.lenA = rsum(lin[LV]) + 1;
+    X.lenQ = rsum(lin[LQ]) + rsum(lin[LK]);
     X.lenB = rsum(lin[LO]);
     X.lenC = rsum(lin[LG]) + rsum(lin[LU]) + 1;
     X.lenD = rsum(lin[LD]);
     X.offA = 0;
-    X.offB = X.offA + up(X.lenA, 32);
+    X.offQ = X.offA + up(X.lenA, 32);
+    X.offB = X.offQ + up(X.lenQ, 32);
     X.offC = X.offB + up(X.lenB, 32);
     X.offD = X.offC + up(X.lenC, 32);
     X.acc_layer = X.offD + up(X.lenD, 32);
@@ -963,9 +996,8 @@ SmemPlan smem_plan(const lb_linear *lin, const StackShape &sh, int N) {
     };
     auto vtab = [&](int k, int nw) { return lin[k].n_paths * nw * 1024; };
     int t2 = utab(LD, 0, 2);
-    t2 = std::max(t2, utab(LV, 0, 2) + utab(LQ, 0, 1) + utab(LK, 0, 2));
+    t2 = std::max(t2, utab(LV, 0, 2) + utab(LQ, 0, 2) + utab(LK, 0, 2));
     t2 = std::max(t2, utab(LO, 0, 2));
-    t2 = std::max(t2, utab(LQ, 1, 2));
     t2 = std::max(t2, utab(LG, 0, 2) + utab(LU, 0, 2));
     int t1 = vtab(LQ, nd) + vtab(LK, nd) + vtab(LV, nd);
     t1 = std::max(t1, vtab(LO, nd));
@@ -976,11 +1008,6 @@ SmemPlan smem_plan(const lb_linear *lin, const StackShape &sh, int N) {
     at += up(t2, 1024);
     o.t1 = at;
     at += up(t1, 1024);
-    int tz_n = rsum(lin[LQ]) + rsum(lin[LK]) + rsum(lin[LV]) + 1;
-    tz_n = std::max(tz_n, rsum(lin[LO]));
-    tz_n = std::max(tz_n, rsum(lin[LG]) + rsum(lin[LU]) + 1);
-    tz_n = std::max(tz_n, rsum(lin[LD]));
-    o.tz = take(4 * (tz_n + 1));
     o.res0 = take(4 * 32 * nd);
     o.res1 = take(4 * 32 * nd);
     o.y = take(4 * 32 * nd);
@@ -990,7 +1017,6 @@ SmemPlan smem_plan(const lb_linear *lin, const StackShape &sh, int N) {
     o.yv = take(4 * nkv);
     o.yg = take(4 * 32 * nf);
     o.yu = take(4 * 32 * nf);
-    o.tsave = take(4 * (lin[LQ].path[lin[LQ].n_paths - 1].r + 4));
     o.ssacc = take(16);
     o.prog = take(kProgBytes);
     S.bytes = up(at, 128);
@@ -1001,6 +1027,10 @@ SmemPlan smem_plan(const lb_linear *lin, const StackShape &sh, int N) {
 
 Item tab(int tb, int n_tab, int n_vals, int mode, int s0, int s1, int s2, int scale) {
     return Item{{tb, n_tab, n_vals, mode, s0, s1, s2, scale}};
+}
+// e0, ss_el: exchange word indices within a layer (ss_el < 0: none)
+Item ptab(int tb, int n_tab, int n_vals, int mode, int e0, int scale, int ss_el) {
+    return Item{{tb, n_tab, n_vals, mode, e0, scale, ss_el, 0}};
 }
 
 struct Costed {
@@ -1069,6 +1099,21 @@ struct ProgBuild {
         for (int w = 0; w <= kCW; ++w) step[s].wo[w] = wo[w];
         items.insert(items.end(), grouped.begin(), grouped.end());
     }
+    // Poll-table units: the same split, word indices instead of offsets.
+    void ptables(int s, const std::vector<Item> &jobs) {
+        std::vector<Costed> us;
+        for (const Item &J : jobs) {
+            const int nt = J.f[1];
+            for (int t0 = 0; t0 < nt; t0 += 32)
+                us.push_back({Item{{J.f[0] + 128 * t0, std::min(32, nt - t0), J.f[2] - 4 * t0,
+                                    J.f[3], J.f[4] + 4 * t0, J.f[5] + 8 * t0, J.f[6], 0}},
+                              1.0 + std::min(32, nt - t0) / 32.0});
+        }
+        std::vector<Item> g;
+        int wo[kCW + 1];
+        lpt(us, g, wo);
+        place(s, g, wo);
+    }
     // 32-row blocks x runs of words, the run length chosen to balance warps
     // (cost of a unit: its words plus a fixed overhead).
     void s2(int s, const std::vector<S2Job> &jobs) {
@@ -1134,6 +1179,10 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
         B.tables(s, T);
         T.clear();
     };
+    auto flush_p = [&](int s) {
+        B.ptables(s, T);
+        T.clear();
+    };
     auto flush_u = [&](int s) {
         B.s2(s, U);
         U.clear();
@@ -1145,20 +1194,21 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
     // phase A: stage 2 of down (previous layer) -> y; stage 1 of q, k, v of
     // a = res0 + y (written to res1)
     {
-        int tb = o.t2, off = 0;
+        int tb = o.t2, off = X.offD;  // words of the previous layer
         for (int p = 0; p < np(LD); ++p) {
-            T.push_back(tab(tb, 8 * Rk(LD, p), rk(LD, p), TAB_PLAIN, o.tz + 4 * off, 0, 0,
-                            o.a_ld[p]));
+            T.push_back(ptab(tb, 8 * Rk(LD, p), rk(LD, p), TAB_PLAIN, off, o.a_ld[p], -1));
             U.push_back({o.a_Ud[p], o.a_hd[p], Rk(LD, p), rows_d, tb, o.y});
             tb += Rk(LD, p) * 1024;
             off += rk(LD, p);
         }
-        flush_t(A_T2);
+        flush_p(A_P2);
         flush_u(A_S2);
-        int tb1 = o.t1, dst = X.offA, mode = TAB_RES | TAB_WRITER;
+        // q, k -> region Q; v -> region A
+        int tb1 = o.t1, dq = X.offQ, dv = X.offA, mode = TAB_RES | TAB_WRITER;
         for (int k = 0; k < 3; ++k)
             for (int p = 0; p < np(k); ++p) {
                 T.push_back(tab(tb1, 8 * nd, rows_d, mode, o.res0, o.y, o.res1, o.a_g[k][p]));
+                int &dst = k == LV ? dv : dq;
                 V.push_back({o.a_V[k][p], rk(k, p), nd, tb1, dst});
                 mode = TAB_RES;
                 tb1 += nd * 1024;
@@ -1167,20 +1217,39 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
         flush_t(A_T1);
         flush_v(A_S1);
     }
-    // phase B: v on the attention rows of R_c -> xa; stage 1 of o; then
-    // path 0 of q -> yq, k -> yk, v on K_c -> yv
+    // phase B: tables of v, q, k (scaled by the rms factor of a); v on the
+    // attention rows of R_c -> xa; stage 1 of o; then q -> yq, k -> yk and
+    // v on K_c -> yv
     {
-        const int nq = rsum(lin[LQ]), nk = rsum(lin[LK]);
-        int tb = o.t2, off = nq + nk, tbv[2] = {0, 0};
+        const int ssA = X.offA + rsum(lin[LV]);
+        int tb = o.t2, tbv[2] = {0, 0}, off = X.offA;
         for (int p = 0; p < np(LV); ++p) {
-            T.push_back(tab(tb, 8 * Rk(LV, p), rk(LV, p), TAB_PLAIN | TAB_MUL, o.tz + 4 * off, 0,
-                            0, o.b_lv[p]));
+            T.push_back(ptab(tb, 8 * Rk(LV, p), rk(LV, p), TAB_PLAIN | TAB_MUL, off, o.b_lv[p],
+                             ssA));
             U.push_back({o.b_Uat[p], o.b_hat[p], Rk(LV, p), rows_d, tb, o.xa});
             tbv[p] = tb;
             tb += Rk(LV, p) * 1024;
             off += rk(LV, p);
         }
-        flush_t(B_T2V);
+        std::vector<S2Job> Uqkv;
+        off = X.offQ;
+        for (int p = 0; p < np(LQ); ++p) {
+            T.push_back(ptab(tb, 8 * Rk(LQ, p), rk(LQ, p), TAB_PLAIN | TAB_MUL, off, o.b_lq[p],
+                             ssA));
+            Uqkv.push_back({o.b_Uq[p], o.b_hq[p], Rk(LQ, p), rows_d, tb, o.yq});
+            tb += Rk(LQ, p) * 1024;
+            off += rk(LQ, p);
+        }
+        for (int p = 0; p < np(LK); ++p) {
+            T.push_back(ptab(tb, 8 * Rk(LK, p), rk(LK, p), TAB_PLAIN | TAB_MUL, off, o.b_lk[p],
+                             ssA));
+            Uqkv.push_back({o.b_Uk[p], o.b_hk[p], Rk(LK, p), nkv, tb, o.yk});
+            tb += Rk(LK, p) * 1024;
+            off += rk(LK, p);
+        }
+        for (int p = 0; p < np(LV); ++p)
+            Uqkv.push_back({o.b_Uvk[p], o.b_hvk[p], Rk(LV, p), nkv, tbv[p], o.yv});
+        flush_p(B_P2);
         flush_u(B_S2V);
         int tb1 = o.t1, dst = X.offB;
         for (int p = 0; p < np(LO); ++p) {
@@ -1191,34 +1260,20 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
         }
         flush_t(B_T1);
         flush_v(B_S1);
-        T.push_back(tab(tb, 8 * Rk(LQ, 0), rk(LQ, 0), TAB_PLAIN | TAB_MUL, o.tz, 0, 0, o.b_lq[0]));
-        U.push_back({o.b_Uq[0], o.b_hq[0], Rk(LQ, 0), rows_d, tb, o.yq});
-        tb += Rk(LQ, 0) * 1024;
-        off = nq;
-        for (int p = 0; p < np(LK); ++p) {
-            T.push_back(tab(tb, 8 * Rk(LK, p), rk(LK, p), TAB_PLAIN | TAB_MUL, o.tz + 4 * off, 0,
-                            0, o.b_lk[p]));
-            U.push_back({o.b_Uk[p], o.b_hk[p], Rk(LK, p), nkv, tb, o.yk});
-            tb += Rk(LK, p) * 1024;
-            off += rk(LK, p);
-        }
-        for (int p = 0; p < np(LV); ++p)
-            U.push_back({o.b_Uvk[p], o.b_hvk[p], Rk(LV, p), nkv, tbv[p], o.yv});
-        flush_t(B_T2QK);
+        U = Uqkv;
         flush_u(B_S2QKV);
     }
     // phase C: stage 2 of o -> y; stage 1 of gate, up of h = res1 + y
     // (written to res0); path 1 of q from the saved t -> yq
     {
-        int tb = o.t2, off = 0;
+        int tb = o.t2, off = X.offB;
         for (int p = 0; p < np(LO); ++p) {
-            T.push_back(tab(tb, 8 * Rk(LO, p), rk(LO, p), TAB_PLAIN, o.tz + 4 * off, 0, 0,
-                            o.c_lo[p]));
+            T.push_back(ptab(tb, 8 * Rk(LO, p), rk(LO, p), TAB_PLAIN, off, o.c_lo[p], -1));
             U.push_back({o.c_Uo[p], o.c_ho[p], Rk(LO, p), rows_d, tb, o.y});
             tb += Rk(LO, p) * 1024;
             off += rk(LO, p);
         }
-        flush_t(C_T2);
+        flush_p(C_P2);
         flush_u(C_S2);
         int tb1 = o.t1, dst = X.offC, mode = TAB_RES | TAB_WRITER;
         for (int k = LG; k <= LU; ++k)
@@ -1232,28 +1287,22 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
             }
         flush_t(C_T1);
         flush_v(C_S1);
-        if (np(LQ) > 1) {
-            T.push_back(tab(o.t2, 8 * Rk(LQ, 1), rk(LQ, 1), TAB_PLAIN | TAB_MUL, o.tsave, 0, 0,
-                            o.b_lq[1]));
-            U.push_back({o.b_Uq[1], o.b_hq[1], Rk(LQ, 1), rows_d, o.t2, o.yq});
-        }
-        flush_t(C_T2Q1);
-        flush_u(C_S2Q1);
     }
     // phase D: stage 2 of gate, up on F_c -> yg, yu; stage 1 of down of
     // m = silu(yg) * yu
     {
-        int tb = o.t2, off = 0;
+        const int ssC = X.offC + rsum(lin[LG]) + rsum(lin[LU]);
+        int tb = o.t2, off = X.offC;
         for (int k = LG; k <= LU; ++k)
             for (int p = 0; p < np(k); ++p) {
-                T.push_back(tab(tb, 8 * Rk(k, p), rk(k, p), TAB_PLAIN | TAB_MUL, o.tz + 4 * off,
-                                0, 0, k == LG ? o.d_lg[p] : o.d_lu[p]));
+                T.push_back(ptab(tb, 8 * Rk(k, p), rk(k, p), TAB_PLAIN | TAB_MUL, off,
+                                 k == LG ? o.d_lg[p] : o.d_lu[p], ssC));
                 U.push_back({k == LG ? o.d_Ug[p] : o.d_Uu[p], k == LG ? o.d_hg[p] : o.d_hu[p],
                              Rk(k, p), rows_f, tb, k == LG ? o.yg : o.yu});
                 tb += Rk(k, p) * 1024;
                 off += rk(k, p);
             }
-        flush_t(D_T2);
+        flush_p(D_P2);
         flush_u(D_S2);
         int tb1 = o.t1, dst = X.offD;
         for (int p = 0; p < np(LD); ++p) {
@@ -1381,6 +1430,8 @@ cudaError_t launch_stack(const lb_linear *lin, int n_layers, const StackShape &s
     P.xacc = reinterpret_cast<unsigned long long *>(ws_after_header + desc_bytes_for(n_layers));
     P.acc_layer = X.acc_layer;
     P.offA = X.offA;
+    P.offQ = X.offQ;
+    P.lenQ = X.lenQ;
     P.offB = X.offB;
     P.offC = X.offC;
     P.offD = X.offD;
