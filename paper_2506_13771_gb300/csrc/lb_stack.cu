@@ -173,10 +173,13 @@ struct Item {
 // Table-job modes: source kind in bits 0-1, flags above.
 enum { TAB_PLAIN = 0, TAB_RES = 1, TAB_SILU = 2, TAB_WRITER = 4, TAB_MUL = 8 };
 
-// Warp w runs units [first + wo[w], first + wo[w + 1]) of its step.
+// Warp w runs units [first + wo[w], first + wo[w + 1]) of its step.  In a
+// stage-2 step fused with the stage-1 tables of the same rows, team[w] =
+// (named barrier id << 16) | threads of warp w's team (0: no team).
 struct Step {
     int first;
     int wo[kCW + 1];
+    int team[kCW];
 };
 constexpr int kStepBytes = (int)((N_STEPS * sizeof(Step) + 15) / 16 * 16);
 constexpr int kProgBytes = 16384;  // per CTA, in the workspace and in shared memory
@@ -248,6 +251,13 @@ __device__ __forceinline__ void item_at(int prog, int u, int4 &a, int4 &b) {
     const unsigned char *p = g_smem + prog + kStepBytes + u * (int)sizeof(Item);
     a = *reinterpret_cast<const int4 *>(p);
     b = *reinterpret_cast<const int4 *>(p + 16);
+}
+
+// Barrier of warp w's team in a fused step (the warps that own the same
+// 32-row blocks): their stage-2 sums are complete after it.
+__device__ __forceinline__ void team_sync(int prog, int s) {
+    const int t = step_at(prog, s).team[threadIdx.x >> 5];
+    if (t) asm volatile("bar.sync %0, %1;" ::"r"(t >> 16), "r"(t & 0xffff) : "memory");
 }
 
 // Table units: lane n builds table n of the unit.  Table n holds, for
@@ -769,7 +779,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
             zero_stripe(xp + P.offC, P.lenC);
             zero_stripe(xp + P.offQ, P.lenQ);
             run_s2(pg, A_S2);
-            csync();
+            team_sync(pg, A_S2);
         }
         run_tables(pg, A_T1, 1.f, o.ssacc);  // a = res0 + y -> res1
         csync();
@@ -784,7 +794,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         if (!run_poll_tables(pg, B_P2, xl, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
         if (l > 0) zero_stripe(xp + P.offD, P.lenD);
         run_s2(pg, B_S2V);  // -> xa
-        csync();
+        team_sync(pg, B_S2V);
         run_tables(pg, B_T1, 1.f, o.ssacc);
         csync();
         run_s1(pg, B_S1, xl, lim, err);
@@ -811,7 +821,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         if (!run_poll_tables(pg, C_P2, xl, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
         zero_stripe(xl + P.offA, P.lenA);
         run_s2(pg, C_S2);  // -> y
-        csync();
+        team_sync(pg, C_S2);
         run_tables(pg, C_T1, 1.f, o.ssacc);  // h = res1 + y -> res0
         csync();
         send_ss(xl + P.offC + ssC);
@@ -824,7 +834,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         if (!run_poll_tables(pg, D_P2, xl, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
         zero_stripe(xl + P.offB, P.lenB);
         run_s2(pg, D_S2);  // -> yg, yu
-        csync();
+        team_sync(pg, D_S2);
         run_tables(pg, D_T1, 1.f, o.ssacc);  // m = silu(yg) * yu
         csync();
         run_s1(pg, D_S1, xl, lim, err);
@@ -1040,27 +1050,36 @@ struct Costed {
 
 // Longest-processing-time assignment of units to the compute warps; returns
 // the units grouped by warp (warp-start offsets in wo) and the makespan.
-double lpt(const std::vector<Costed> &us, std::vector<Item> &out, int (&wo)[kCW + 1]) {
+// Longest-processing-time assignment of units to warps [w0, w1): appends
+// to the per-warp lists, returns the makespan.
+using PerWarp = std::vector<Item>[kCW];
+double lpt_into(const std::vector<Costed> &us, int w0, int w1, PerWarp &per) {
     std::vector<int> idx(us.size());
     for (size_t i = 0; i < us.size(); ++i) idx[i] = (int)i;
     std::stable_sort(idx.begin(), idx.end(),
                      [&](int a, int b) { return us[a].cost > us[b].cost; });
-    std::vector<std::vector<int>> per(kCW);
     double load[kCW] = {};
     for (int i : idx) {
-        int w = 0;
-        for (int k = 1; k < kCW; ++k)
+        int w = w0;
+        for (int k = w0 + 1; k < w1; ++k)
             if (load[k] < load[w]) w = k;
         load[w] += us[i].cost;
-        per[w].push_back(i);
+        per[w].push_back(us[i].it);
     }
+    double mk = 0;
+    for (int w = w0; w < w1; ++w) mk = std::max(mk, load[w]);
+    return mk;
+}
+
+// The same over all compute warps, grouped by warp (warp-start offsets in wo).
+double lpt(const std::vector<Costed> &us, std::vector<Item> &out, int (&wo)[kCW + 1]) {
+    PerWarp per;
+    const double mk = lpt_into(us, 0, kCW, per);
     out.clear();
     wo[0] = 0;
-    double mk = 0;
     for (int w = 0; w < kCW; ++w) {
-        for (int i : per[w]) out.push_back(us[i].it);
+        out.insert(out.end(), per[w].begin(), per[w].end());
         wo[w + 1] = (int)out.size();
-        mk = std::max(mk, load[w]);
     }
     return mk;
 }
@@ -1079,16 +1098,7 @@ struct ProgBuild {
     // Up to 32 tables of one job per unit, one unit per warp where possible.
     void tables(int s, const std::vector<Item> &jobs) {
         std::vector<Costed> us;
-        for (const Item &J : jobs) {
-            const int tb = J.f[0], nt = J.f[1], nv = J.f[2], mode = J.f[3];
-            for (int t0 = 0; t0 < nt; t0 += 32) {
-                auto sh = [&](int off, int per) { return off + per * t0; };  // unused: never read
-                us.push_back({Item{{tb + 128 * t0, std::min(32, nt - t0), nv - 4 * t0, mode,
-                                    sh(J.f[4], 16), sh(J.f[5], 16), sh(J.f[6], 16),
-                                    sh(J.f[7], 8)}},
-                              1.0 + std::min(32, nt - t0) / 32.0});
-            }
-        }
+        for (const Item &J : jobs) table_units(J, 0, J.f[1], us);
         std::vector<Item> g;
         int wo[kCW + 1];
         lpt(us, g, wo);
@@ -1098,6 +1108,69 @@ struct ProgBuild {
         step[s].first = (int)items.size();
         for (int w = 0; w <= kCW; ++w) step[s].wo[w] = wo[w];
         items.insert(items.end(), grouped.begin(), grouped.end());
+    }
+    void place(int s, const PerWarp &per) {
+        step[s].first = (int)items.size();
+        step[s].wo[0] = 0;
+        for (int w = 0; w < kCW; ++w) {
+            items.insert(items.end(), per[w].begin(), per[w].end());
+            step[s].wo[w + 1] = (int)items.size() - step[s].first;
+        }
+    }
+    // Table units of one job's tables [t_lo, t_hi), up to 32 per unit.
+    static void table_units(const Item &J, int t_lo, int t_hi, std::vector<Costed> &us) {
+        for (int t0 = t_lo; t0 < std::min(t_hi, J.f[1]); t0 += 32) {
+            const int nt = std::min(32, std::min(t_hi, J.f[1]) - t0);
+            auto sh = [&](int off, int per) { return off + per * t0; };  // unused: never read
+            us.push_back({Item{{J.f[0] + 128 * t0, nt, J.f[2] - 4 * t0, J.f[3], sh(J.f[4], 16),
+                                sh(J.f[5], 16), sh(J.f[6], 16), sh(J.f[7], 8)}},
+                          1.0 + nt / 32.0});
+        }
+    }
+    // Stage 2 fused with the stage-1 tables of its output rows: the 32-row
+    // blocks are split into teams of warps (one named barrier each, ids from
+    // 2); a team computes its blocks' stage-2 sums, meets at its barrier and
+    // builds the tables of those rows (8 per block and job).
+    void fused(int s2s, int t1s, const std::vector<S2Job> &jobs, int rows,
+               const std::vector<Item> &t1jobs) {
+        PerWarp p2, p1;
+        const int nb = (rows + 31) / 32, nteam = std::min(nb, std::min(kCW, 14));
+        int maxR = 1;
+        for (const S2Job &J : jobs) maxR = std::max(maxR, J.R);
+        for (int t = 0; t < nteam; ++t) {
+            const int b0 = nb * t / nteam, b1 = nb * (t + 1) / nteam;
+            const int w0 = kCW * t / nteam, w1 = kCW * (t + 1) / nteam;
+            PerWarp best;
+            double best_mk = 1e300;
+            for (int run = 1; run <= maxR; ++run) {
+                std::vector<Costed> us;
+                for (const S2Job &J : jobs)
+                    for (int b = b0; b < b1; ++b) {
+                        const int r0 = 32 * b;
+                        if (r0 >= J.rows) continue;
+                        for (int q = 0; q < J.R; q += run) {
+                            const int nw = std::min(run, J.R - q);
+                            us.push_back({Item{{J.U + (r0 * J.R + q) * 4, J.R, nw, J.tb + q * 1024,
+                                                J.h + 2 * r0, J.out + 4 * r0,
+                                                std::min(32, J.rows - r0), 0}},
+                                          nw + 1.5});
+                        }
+                    }
+                PerWarp trial;
+                const double mk = lpt_into(us, w0, w1, trial);
+                if (mk < best_mk - 1e-9) {
+                    best_mk = mk;
+                    for (int w = w0; w < w1; ++w) best[w] = trial[w];
+                }
+            }
+            for (int w = w0; w < w1; ++w) p2[w] = best[w];
+            std::vector<Costed> ts;
+            for (const Item &J : t1jobs) table_units(J, 8 * b0, 8 * b1, ts);
+            lpt_into(ts, w0, w1, p1);
+            for (int w = w0; w < w1; ++w) step[s2s].team[w] = ((2 + t) << 16) | (32 * (w1 - w0));
+        }
+        place(s2s, p2);
+        place(t1s, p1);
     }
     // Poll-table units: the same split, word indices instead of offsets.
     void ptables(int s, const std::vector<Item> &jobs) {
@@ -1202,7 +1275,6 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
             off += rk(LD, p);
         }
         flush_p(A_P2);
-        flush_u(A_S2);
         // q, k -> region Q; v -> region A
         int tb1 = o.t1, dq = X.offQ, dv = X.offA, mode = TAB_RES | TAB_WRITER;
         for (int k = 0; k < 3; ++k)
@@ -1214,7 +1286,9 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
                 tb1 += nd * 1024;
                 dst += rk(k, p);
             }
-        flush_t(A_T1);
+        B.fused(A_S2, A_T1, U, rows_d, T);
+        U.clear();
+        T.clear();
         flush_v(A_S1);
     }
     // phase B: tables of v, q, k (scaled by the rms factor of a); v on the
@@ -1250,7 +1324,6 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
         for (int p = 0; p < np(LV); ++p)
             Uqkv.push_back({o.b_Uvk[p], o.b_hvk[p], Rk(LV, p), nkv, tbv[p], o.yv});
         flush_p(B_P2);
-        flush_u(B_S2V);
         int tb1 = o.t1, dst = X.offB;
         for (int p = 0; p < np(LO); ++p) {
             T.push_back(tab(tb1, 8 * nd, rows_d, TAB_PLAIN, o.xa, 0, 0, o.b_go[p]));
@@ -1258,7 +1331,9 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
             tb1 += nd * 1024;
             dst += rk(LO, p);
         }
-        flush_t(B_T1);
+        B.fused(B_S2V, B_T1, U, rows_d, T);
+        U.clear();
+        T.clear();
         flush_v(B_S1);
         U = Uqkv;
         flush_u(B_S2QKV);
@@ -1274,7 +1349,6 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
             off += rk(LO, p);
         }
         flush_p(C_P2);
-        flush_u(C_S2);
         int tb1 = o.t1, dst = X.offC, mode = TAB_RES | TAB_WRITER;
         for (int k = LG; k <= LU; ++k)
             for (int p = 0; p < np(k); ++p) {
@@ -1285,7 +1359,9 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
                 tb1 += nd * 1024;
                 dst += rk(k, p);
             }
-        flush_t(C_T1);
+        B.fused(C_S2, C_T1, U, rows_d, T);
+        U.clear();
+        T.clear();
         flush_v(C_S1);
     }
     // phase D: stage 2 of gate, up on F_c -> yg, yu; stage 1 of down of
@@ -1303,7 +1379,6 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
                 off += rk(k, p);
             }
         flush_p(D_P2);
-        flush_u(D_S2);
         int tb1 = o.t1, dst = X.offD;
         for (int p = 0; p < np(LD); ++p) {
             T.push_back(tab(tb1, 8 * nf, rows_f, TAB_SILU, o.yg, o.yu, 0, o.d_gd[p]));
@@ -1311,7 +1386,9 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
             tb1 += nf * 1024;
             dst += rk(LD, p);
         }
-        flush_t(D_T1);
+        B.fused(D_S2, D_T1, U, rows_f, T);
+        U.clear();
+        T.clear();
         flush_v(D_S1);
     }
     if ((int)B.items.size() > kMaxItems) return false;
