@@ -132,7 +132,7 @@ bool use_decode(const lb_linear &, int64_t T) { return T == 1; }
 
 // From this many tokens on, the layer is a dense contraction worth the
 // tensor cores (tcgen05, 128-token tiles).
-constexpr int64_t kPrefillMinTokens = 32;
+constexpr int64_t kPrefillMinTokens = 16;
 bool use_prefill(const lb_linear &L, int64_t T) {
     return T >= kPrefillMinTokens && lb::prefill_supported(L, T);
 }

@@ -14,7 +14,7 @@
 // arrives by TMA (bf16) and is converted to fp16 in shared memory (exact for
 // |x| < 65504); z goes to the workspace as fp16 and comes back by TMA.
 //
-// One CTA = 4 warps computes a 128 x BN tile (BN <= 256 fp32 TMEM columns).
+// One CTA = 8 warps computes a 128 x BN tile (BN <= 256 fp32 TMEM columns).
 // K runs in 64-element stages through a 4-deep shared-memory ring: the TMA
 // of stage k+2 and the unpacking of stage k overlap the MMAs of stage k-1.
 // Thread 0 issues the TMA copies and the MMAs (tcgen05.mma, one thread per
@@ -24,6 +24,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <mutex>
 
 #include "lb_common.cuh"
@@ -37,7 +38,7 @@ constexpr int BM = 128;       // tokens per tile (MMA M)
 constexpr int BN = 256;       // columns per tile (MMA N)
 constexpr int BK = 64;        // K per stage: 64 fp16 = one 128-byte swizzle row
 constexpr int STAGES = 4;
-constexpr int kThreads = 128;
+constexpr int kThreads = 256;  // 8 warps unpack and convert each K-stage
 constexpr int A_BYTES = BM * BK * 2;   // 16 KB
 constexpr int B_BYTES = BN * BK * 2;   // 32 KB
 // stage 1: per stage, the two V word rows of the stage's 64 inputs for the
@@ -186,6 +187,8 @@ struct PrefillParams {
     int bn1;           // stage-1 tile width: N1 if N1 <= 256, else 256
     int off1;          // column offset of path 1 in the N1 concatenation (= r_0)
     uint16_t *z;       // stage 1 output / stage 2 input, fp16 [T][N1]
+    float *zpart;      // split stage 1: fp32 partial sums [split][T][N1] (before l)
+    int split;         // stage-1 K slices (gridDim.z of stage 1)
     void *y;           // stage 2 output [T][d_out]
     int y_fp32;
     unsigned *ws_words;
@@ -278,7 +281,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     unsigned char *slab = smem + RING_BYTES;
     const int m0 = blockIdx.x * BM, n0 = blockIdx.y * BN;
     const int K = STAGE1 ? P.L.d_in : P.N1;
-    const int KC = K / BK;
+    // stage 1 may be split along K: slice z of split takes chunks [kbeg, kbeg + KC)
+    const int KT = K / BK, nsplit = STAGE1 ? P.split : 1;
+    const int kbeg = (int)((long long)blockIdx.z * KT / nsplit);
+    const int KC = (int)((long long)(blockIdx.z + 1) * KT / nsplit) - kbeg;
     const int warp = threadIdx.x >> 5;
     const bool t0 = threadIdx.x == 0;
     const int bn = STAGE1 ? P.bn1 : BN;
@@ -310,10 +316,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto B_of = [&](int s) { return smem + s * SB + A_BYTES; };
     auto S_of = [&](int s) { return smem + RING_BYTES + s * SRC_BYTES; };
     int loads_issued = 0, mmas_issued = 0;  // K-chunks loaded / multiplied (thread 0)
-    // The x / z tile of K-chunk kc by TMA; in stage 1 also the chunk's two V
-    // word rows for the tile's columns and the chunk's g values, by bulk copy.
-    auto issue_load = [&](int kc) {
-        const int s = kc % STAGES;
+    // The x / z tile of the CTA's K-chunk i (chunk kbeg + i of the layer) by
+    // TMA; in stage 1 also the chunk's two V word rows for the tile's columns
+    // and the chunk's g values, by bulk copy.
+    auto issue_load = [&](int i) {
+        const int s = i % STAGES, kc = kbeg + i;
         uint64_t *b = full + s;
         if (STAGE1) {
             unsigned char *src = S_of(s);
@@ -381,7 +388,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             ok = false;
             break;
         }
-        unpack_b<STAGE1>(P, B_of(s), S_of(s), slab, kc, n0, bn);
+        unpack_b<STAGE1>(P, B_of(s), S_of(s), slab, kbeg + kc, n0, bn);
         if (s_fail) {
             ok = false;
             break;
@@ -419,14 +426,26 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncthreads();
     } else {
         tc_fence_after();
-        // epilogue: warp w reads TMEM lanes 32w..32w+31 = tile rows
-        const int row = m0 + 32 * warp + (threadIdx.x & 31);
-        const uint32_t lane_base = tmem + ((uint32_t)(32 * warp) << 16);
-        for (int cb = 0; cb < bn; cb += 32) {
+        // epilogue: warp w reads TMEM lanes 32(w%4) .. +31 (tile rows) and
+        // the (w/4)-th half of the tile's 32-column chunks
+        const int wq = warp & 3, half = warp >> 2, nchunk = bn / 32;
+        const int row = m0 + 32 * wq + (threadIdx.x & 31);
+        const uint32_t lane_base = tmem + ((uint32_t)(32 * wq) << 16);
+        const int cb0 = 32 * (half * nchunk / 2), cb1 = 32 * ((half + 1) * nchunk / 2);
+        for (int cb = cb0; cb < cb1; cb += 32) {
             float v[32];
             tmem_ld32(lane_base + cb, v);
             if (row >= P.T) continue;
-            if (STAGE1) {
+            if (STAGE1 && nsplit > 1) {
+                // fp32 partial sums of this K slice; the reduction applies l
+                if (n0 + cb < P.N1) {
+                    float4 *dst = reinterpret_cast<float4 *>(
+                        P.zpart + ((size_t)blockIdx.z * P.T + row) * P.N1 + n0 + cb);
+#pragma unroll
+                    for (int q = 0; q < 8; ++q)
+                        dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                }
+            } else if (STAGE1) {
                 // z = l . t as fp16
                 uint32_t packed[16];
 #pragma unroll
@@ -493,6 +512,34 @@ __global__ void __launch_bounds__(kThreads, 1)
                      : "memory");
 }
 
+// z = fp16(l . sum over the K slices of the partial t), four columns per thread.
+__global__ void k_reduce_z(const __grid_constant__ PrefillParams P) {
+    const int groups = P.N1 / 4;
+    const long long n = (long long)P.T * groups;
+    for (long long g = blockIdx.x * (long long)blockDim.x + threadIdx.x; g < n;
+         g += (long long)gridDim.x * blockDim.x) {
+        const int row = (int)(g / groups), c = 4 * (int)(g % groups);
+        float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int z = 0; z < P.split; ++z) {
+            const float4 b = *reinterpret_cast<const float4 *>(
+                P.zpart + ((size_t)z * P.T + row) * P.N1 + c);
+            a.x += b.x;
+            a.y += b.y;
+            a.z += b.z;
+            a.w += b.w;
+        }
+        const int p = c >= P.off1 ? 1 : 0, j = c - (p ? P.off1 : 0);  // 4 | off1
+        const uint2 lb = *reinterpret_cast<const uint2 *>((p ? P.L.l[1] : P.L.l[0]) + j);
+        const __half2 h0 = __floats2half2_rn(a.x * half_bits_to_float(lb.x & 0xffffu),
+                                             a.y * half_bits_to_float(lb.x >> 16));
+        const __half2 h1 = __floats2half2_rn(a.z * half_bits_to_float(lb.y & 0xffffu),
+                                             a.w * half_bits_to_float(lb.y >> 16));
+        *reinterpret_cast<uint2 *>(P.z + (size_t)row * P.N1 + c) =
+            make_uint2(*reinterpret_cast<const uint32_t *>(&h0),
+                       *reinterpret_cast<const uint32_t *>(&h1));
+    }
+}
+
 // ---------------------------------------------------------------- host side
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
@@ -526,6 +573,25 @@ bool make_map(CUtensorMap *m, const void *base, CUtensorMapDataType dt, int64_t 
 
 }  // namespace
 
+// The kernels' shared-memory opt-in, once per device (a host call that
+// would otherwise sit between the launches of every forward).
+static cudaError_t set_smem_attributes() {
+    static std::mutex mu;
+    static bool done[64];
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(mu);
+    if (dev >= 0 && dev < 64 && done[dev]) return cudaSuccess;
+    e = cudaFuncSetAttribute(k_prefill<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             smem_bytes<true>());
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_prefill<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 smem_bytes<false>());
+    if (e == cudaSuccess && dev >= 0 && dev < 64) done[dev] = true;
+    return e;
+}
+
 bool prefill_supported(const lb_linear &L, int64_t T) {
     if (T < 1 || T > (1LL << 30)) return false;
     if (L.d_in % BK != 0 || L.d_out % 8 != 0) return false;
@@ -534,10 +600,32 @@ bool prefill_supported(const lb_linear &L, int64_t T) {
     return encoder();
 }
 
-size_t prefill_ws_bytes(const lb_linear &L, int64_t T) {
+namespace {
+size_t n1_of(const lb_linear &L) {
     size_t n1 = 0;
     for (int p = 0; p < L.n_paths; ++p) n1 += (size_t)L.path[p].r;
-    return ((size_t)T * n1 * 2 + 255) & ~(size_t)255;
+    return n1;
+}
+// Stage-1 K slices: enough CTAs to fill about 148 SMs, at least two K-chunks
+// per slice, at most 32 slices (a function of the shapes only, so the
+// workspace size does not depend on the device).
+int split_of(const lb_linear &L, int64_t T) {
+    const int64_t n1 = (int64_t)n1_of(L), bn1 = n1 <= BN ? n1 : BN;
+    const int64_t tiles = ((T + BM - 1) / BM) * ((n1 + bn1 - 1) / bn1);
+    const int64_t kc = L.d_in / BK;
+    int64_t s = 148 / tiles;
+    s = std::min<int64_t>(s, kc / 2);
+    s = std::min<int64_t>(s, 32);
+    return s < 2 ? 1 : (int)s;
+}
+size_t z16_bytes(const lb_linear &L, int64_t T) {
+    return ((size_t)T * n1_of(L) * 2 + 255) & ~(size_t)255;
+}
+}  // namespace
+
+size_t prefill_ws_bytes(const lb_linear &L, int64_t T) {
+    const int S = split_of(L, T);
+    return z16_bytes(L, T) + (S > 1 ? (size_t)S * T * n1_of(L) * 4 : 0);
 }
 
 cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, void *y, int y_fp32,
@@ -552,6 +640,8 @@ cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, voi
     P.bn1 = P.N1 <= BN ? P.N1 : BN;
     P.d_out = L.d_out;
     P.z = static_cast<uint16_t *>(z_ws);
+    P.split = split_of(L, T);
+    P.zpart = reinterpret_cast<float *>(static_cast<char *>(z_ws) + z16_bytes(L, T));
     P.y = y;
     P.y_fp32 = y_fp32;
     P.ws_words = ws_words;
@@ -559,17 +649,20 @@ cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, voi
     if (!make_map(&xmap, x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, T, L.d_in) ||
         !make_map(&zmap, z_ws, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, T, P.N1))
         return cudaErrorInvalidValue;
-    cudaError_t e;
-    e = cudaFuncSetAttribute(k_prefill<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             smem_bytes<true>());
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_prefill<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 smem_bytes<false>());
+    cudaError_t e = set_smem_attributes();
     if (e != cudaSuccess) return e;
-    const dim3 g1((unsigned)((T + BM - 1) / BM), (unsigned)((P.N1 + P.bn1 - 1) / P.bn1));
+    const dim3 g1((unsigned)((T + BM - 1) / BM), (unsigned)((P.N1 + P.bn1 - 1) / P.bn1),
+                  (unsigned)P.split);
     k_prefill<true><<<g1, kThreads, smem_bytes<true>(), s>>>(xmap, P);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
+    if (P.split > 1) {
+        const long long groups = (long long)T * (P.N1 / 4);
+        const int blocks = (int)std::min<long long>((groups + 255) / 256, 148 * 8);
+        k_reduce_z<<<blocks, 256, 0, s>>>(P);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
     const dim3 g2((unsigned)((T + BM - 1) / BM), (unsigned)((L.d_out + BN - 1) / BN));
     k_prefill<false><<<g2, kThreads, smem_bytes<false>(), s>>>(zmap, P);
     return cudaGetLastError();

@@ -1248,10 +1248,6 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
     std::vector<Item> T;
     std::vector<S2Job> U;
     std::vector<S1Job> V;
-    auto flush_t = [&](int s) {
-        B.tables(s, T);
-        T.clear();
-    };
     auto flush_p = [&](int s) {
         B.ptables(s, T);
         T.clear();

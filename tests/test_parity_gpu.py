@@ -116,8 +116,8 @@ def test_config2_4096_r64(T, out_dtype):
 @pytest.mark.parametrize("T", [1, 16, 64])
 def test_config3_ffn_triple(r, T):
     lins, x, x_down = inputs.config3(r, T)
-    # T >= 32 runs on the tensor cores with fp16 operands (z rounded to fp16)
-    tol = 1e-3 if T >= 32 else TOL_FP32
+    # T >= 16 runs on the tensor cores with fp16 operands (z rounded to fp16)
+    tol = 1e-3 if T >= 16 else TOL_FP32
     for name in ("gate", "up", "down"):
         L = lins[name]
         xin = x_down if name == "down" else x
@@ -147,7 +147,7 @@ STRESS = [
     (32, 17, (1,), 1), (32, 1000, (16, 33), 2), (4128, 17, (96, 1), 3), (4128, 1000, (33, 96), 7),
     (64, 64, (96,), 8), (4128, 1000, (16,), 9), (1024, 300, (33, 16), 65), (4128, 40, (1, 1), 1),
     (96, 2048, (1000, 24), 1), (8192, 8, (64, 64), 1),
-    # T >= 32 but d_out % 8 != 0 or r > 512: the CUDA-core path
+    # T >= 16 but d_out % 8 != 0 or r > 512: the CUDA-core path
     (512, 2100, (192,), 300), (256, 512, (576,), 40),
 ]
 
@@ -158,16 +158,18 @@ def test_stress_shapes(d_in, d_out, rs, T):
     L = inputs.make_linear(rng, d_in, d_out, list(rs), len(rs), 0.1)
     x = inputs.bf16_normal(rng, (T, d_in))
     D = lb.DeviceLinear(L, DEV)
-    tol = 1e-3 if T >= 32 and all(r % 64 == 0 for r in rs) and d_in % 64 == 0 else TOL_FP32
+    tol = 1e-3 if T >= 16 and all(r % 64 == 0 for r in rs) and d_in % 64 == 0 else TOL_FP32
     check(gpu_forward(D, x, torch.float32), oracle.forward_factored(L, x), torch.float32, tol)
 
 
 PREFILL = [
-    # d_in, d_out, ranks, T   (the tensor-core path: T >= 32, ranks multiples of 64
+    # d_in, d_out, ranks, T   (the tensor-core path: T >= 16, ranks multiples of 64
     # up to 512, d_out a multiple of 8)
     (64, 256, (64,), 128), (128, 512, (64, 64), 256), (4096, 4096, (64, 64), 200),
     (256, 1000, (128, 64), 77), (512, 2104, (192,), 300), (1024, 768, (512, 512), 130),
     (4096, 11008, (128, 128), 64), (64, 8, (64, 64), 33),
+    # stage 1 split along d_in into K slices (long d_in, few token tiles)
+    (11008, 4096, (128, 128), 16), (4096, 2048, (512, 512), 300), (2048, 64, (64,), 20),
 ]
 
 
