@@ -13,6 +13,13 @@ on a bounded sample (cpu_baseline), and the SM clocks seen while timing.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                   [--layers L]
+  python bench.py --config 2|3|4 [--steps K] [--warmup W]
+
+--config times the single-linear workloads instead (one JSON line per case,
+not the bench line): 2 = 4096x4096 r64 at T = 1, 8; 3 = the FFN triple at
+r = 128, 512 and T = 1, 16, 64; 4 = prefill at T = 2048, 8192.  Cases 2 and 3
+report algorithmic GB/s with L2 flushed before every call; case 4 reports
+TFLOP/s (2 flops per +-1 MAC, both paths) against the dense bf16 peak.
 
 --impl reference times the CPU oracle (the reference of this build) on the
 same metric; under torchrun only rank 0 runs it.  N > 1 runs independent
@@ -46,6 +53,10 @@ def parse_args():
     ap.add_argument("--layers", type=int, default=80,
                     help="stack depth (80 = the Llama2-70B workload; smaller only for profiling)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--config", type=int, choices=[2, 3, 4], default=None,
+                    help="time a single-linear workload instead of the stack")
+    ap.add_argument("--only", default=None,
+                    help="with --config: only the cases whose 'name:T' contains this text")
     return ap.parse_args()
 
 
@@ -383,10 +394,100 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+# ----------------------------------------------------------------- single-linear workloads
+
+
+def run_config(args):
+    import torch
+
+    from paper_2506_13771_gb300 import build as lb_build
+    from paper_2506_13771_gb300 import inputs
+    from paper_2506_13771_gb300 import littlebit as lb
+
+    lb_build.build()
+    dev = torch.device("cuda", 0)
+    peaks = measured_peaks()
+    hbm = float(peaks.get("hbm_gbs", 6800.0))
+    tc = float(peaks.get("bf16_tflops", 1900.0))
+    l2 = torch.cuda.get_device_properties(dev).L2_cache_size or L2_BYTES
+    flush = torch.empty(2 * l2, dtype=torch.uint8, device=dev)
+    steps = max(1, min(args.steps, 200))
+
+    def weight_bytes(L):
+        return sum(P["v_words"].nbytes + P["u_words"].nbytes + 2 * (L["d_in"] + L["d_out"] + P["r"])
+                   for P in L["paths"])
+
+    def time_case(L, x_bits, T, cold):
+        D = lb.DeviceLinear(L, dev)
+        x = lb.bf16_tensor(x_bits, dev)
+        y = torch.empty((T, D.d_out), dtype=torch.bfloat16, device=dev)
+        ws = lb.new_workspace(lb.workspace_size(D, T), dev)
+        for _ in range(max(3, args.warmup)):
+            lb.linear_forward(D, x, y=y, ws=ws)
+        torch.cuda.synchronize(dev)
+        ts = []
+        for _ in range(steps):
+            if cold:
+                flush.zero_()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record()
+            lb.linear_forward(D, x, y=y, ws=ws)
+            e1.record()
+            torch.cuda.synchronize(dev)
+            ts.append(e0.elapsed_time(e1))
+        if lb.poll_error(ws) != lb.LB_OK:
+            raise RuntimeError("kernel reported an error")
+        return statistics.median(ts)
+
+    def wanted(name, T):
+        return args.only is None or args.only in f"{name}:{T}"
+
+    def emit(name, cfg, T, L, ms, flops_mode):
+        wb = weight_bytes(L)
+        act = T * (L["d_in"] + L["d_out"]) * 2
+        flops = sum(2 * T * P["r"] * (L["d_in"] + L["d_out"]) for P in L["paths"])
+        line = {"config": cfg, "case": name, "tokens": T, "ms": ms,
+                "us": ms * 1e3, "bytes": wb + act, "flops": flops,
+                "gbs": (wb + act) / ms / 1e6, "tflops": flops / ms / 1e9}
+        if flops_mode:
+            line["roofline"] = {"bound": "tensor", "achieved": line["tflops"], "peak": tc,
+                                "unit": "TFLOP/s", "frac": line["tflops"] / tc,
+                                "peak_source": "MEASURED_PEAKS.json bf16_tflops (burst)"}
+        else:
+            line["roofline"] = {"bound": "hbm", "achieved": line["gbs"], "peak": hbm,
+                                "unit": "GB/s", "frac": line["gbs"] / hbm,
+                                "peak_source": "MEASURED_PEAKS.json hbm_gbs"}
+        print(json.dumps(line), flush=True)
+
+    if args.config == 2:
+        for T in (1, 8):
+            if wanted("4096x4096 r64", T):
+                L, x = inputs.config2(T)
+                emit("4096x4096 r64", 2, T, L, time_case(L, x, T, True), False)
+    elif args.config == 3:
+        for r in (128, 512):
+            for T in (1, 16, 64):
+                lins, x, xd = inputs.config3(r, T)
+                for nm in ("gate", "up", "down"):
+                    if not wanted(f"{nm} r{r}", T):
+                        continue
+                    xin = xd if nm == "down" else x
+                    emit(f"{nm} r{r}", 3, T, lins[nm], time_case(lins[nm], xin, T, True), False)
+    else:
+        for shape in inputs.PREFILL_SHAPES:
+            for T in (2048, 8192):
+                if wanted(shape, T):
+                    L, x = inputs.config4(shape, T)
+                    emit(shape, 4, T, L, time_case(L, x, T, True), True)
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         run_reference(args)
+    elif args.config is not None:
+        run_config(args)
     else:
         run_ours(args)
 
