@@ -14,13 +14,16 @@
 // arrives by TMA (bf16) and is converted to fp16 in shared memory (exact for
 // |x| < 65504); z goes to the workspace as fp16 and comes back by TMA.
 //
-// One CTA = 8 warps computes a 128 x BN tile (BN <= 256 fp32 TMEM columns).
-// K runs in 64-element stages through a 4-deep shared-memory ring: the TMA
-// of stage k+2 and the unpacking of stage k overlap the MMAs of stage k-1.
-// Thread 0 issues the TMA copies and the MMAs (tcgen05.mma, one thread per
-// CTA); tcgen05.commit releases a stage.  Every wait is bounded (about one
-// second); on a timeout the CTA records LB_ERR_TIMEOUT, waits for its own
-// copies and MMAs in flight, frees its TMEM and returns.
+// One CTA computes a 128 x BN tile (BN <= 256 fp32 TMEM columns) with
+// specialised warps: warp 0 issues the TMA / bulk copies of each 64-element
+// K-stage into a 4-deep shared-memory ring, warps 2..9 unpack and convert a
+// stage as soon as it lands, and warp 1 issues its MMAs (tcgen05.mma, one
+// thread) as soon as it is unpacked; tcgen05.commit hands the stage back to
+// the copy warp.  Per stage, full / ready / empty mbarriers order the three
+// roles, so no CTA-wide barrier sits in the K loop.  Every wait is bounded
+// (about one second); on a timeout the CTA records LB_ERR_TIMEOUT, the other
+// roles stop, the CTA waits for its own copies and MMAs in flight, frees its
+// TMEM and returns.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -38,7 +41,11 @@ constexpr int BM = 128;       // tokens per tile (MMA M)
 constexpr int BN = 256;       // columns per tile (MMA N)
 constexpr int BK = 64;        // K per stage: 64 fp16 = one 128-byte swizzle row
 constexpr int STAGES = 4;
-constexpr int kThreads = 256;  // 8 warps unpack and convert each K-stage
+// Warp roles: 0 issues the TMA / bulk copies, 1 issues the MMAs, 2..9 unpack
+// and convert each K-stage and then read the accumulator out.
+constexpr int kThreads = 320;
+constexpr int kWork = 256;     // threads of the unpacking / epilogue warps
+constexpr int kWorkWarps = kWork / 32;
 constexpr int A_BYTES = BM * BK * 2;   // 16 KB
 constexpr int B_BYTES = BN * BK * 2;   // 32 KB
 // stage 1: per stage, the two V word rows of the stage's 64 inputs for the
@@ -90,6 +97,17 @@ __device__ bool mb_wait(uint64_t *b, unsigned parity) {
     const unsigned long long t0 = globaltimer_ns();
     while (!mb_try(b, parity))
         if (globaltimer_ns() - t0 > kWaitLimitNs) return false;
+    return true;
+}
+
+// The same, giving up early once another role of the CTA has failed.
+__device__ bool mb_wait_role(uint64_t *b, unsigned parity, volatile int *fail) {
+    if (mb_try(b, parity)) return true;
+    const unsigned long long t0 = globaltimer_ns();
+    while (!mb_try(b, parity)) {
+        if (*fail) return false;
+        if (globaltimer_ns() - t0 > kWaitLimitNs) return false;
+    }
     return true;
 }
 
@@ -189,6 +207,9 @@ struct PrefillParams {
     uint16_t *z;       // stage 1 output / stage 2 input, fp16 [T][N1]
     float *zpart;      // split stage 1: fp32 partial sums [split][T][N1] (before l)
     int split;         // stage-1 K slices (gridDim.z of stage 1)
+    int expanded;      // B operands pre-expanded to fp16 (bv, bu) and loaded by TMA
+    uint16_t *bv;      // [N1][d_in]: +-g_p[k] at (column n of path p, input k)
+    uint16_t *bu;      // [d_out][N1]: +-h_p[o] at (output o, column n of path p)
     void *y;           // stage 2 output [T][d_out]
     int y_fp32;
     unsigned *ws_words;
@@ -200,11 +221,11 @@ struct PrefillParams {
 template <bool STAGE1>
 __device__ __forceinline__ void unpack_b(const PrefillParams &P, unsigned char *Bs,
                                          const unsigned char *src, const unsigned char *slab,
-                                         int kc, int n0, int bn) {
+                                         int kc, int n0, int bn, int tid) {
     const uint32_t *words = reinterpret_cast<const uint32_t *>(src);
     const uint16_t *gs = reinterpret_cast<const uint16_t *>(src + 2 * BN * 4);
     // each item = one 16-byte chunk (8 K values) of one B row
-    for (int item = threadIdx.x; item < bn * 8; item += kThreads) {
+    for (int item = tid; item < bn * 8; item += kWork) {
         const int n = item >> 3, c = item & 7;
         uint4 v = make_uint4(0, 0, 0, 0);
         if (STAGE1) {
@@ -253,8 +274,8 @@ __device__ __forceinline__ void mb_expect_only(uint64_t *b, unsigned bytes) {
 }
 
 // In-place bf16 -> fp16 of the A stage (layout-preserving, elementwise).
-__device__ __forceinline__ void convert_a(unsigned char *As) {
-    for (int i = threadIdx.x; i < A_BYTES / 16; i += kThreads) {
+__device__ __forceinline__ void convert_a(unsigned char *As, int tid) {
+    for (int i = tid; i < A_BYTES / 16; i += kWork) {
         uint4 *p = reinterpret_cast<uint4 *>(As) + i;
         uint4 u = *p;
         uint32_t w[4] = {u.x, u.y, u.z, u.w};
@@ -270,11 +291,12 @@ __device__ __forceinline__ void convert_a(unsigned char *As) {
 
 template <bool STAGE1>
 __global__ void __launch_bounds__(kThreads, 1)
-    k_prefill(const __grid_constant__ CUtensorMap amap, const __grid_constant__ PrefillParams P) {
-    __shared__ __align__(8) uint64_t full[STAGES], done[STAGES];
+    k_prefill(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
+              const __grid_constant__ PrefillParams P) {
+    __shared__ __align__(8) uint64_t full[STAGES], ready[STAGES], empty[STAGES];
+    __shared__ __align__(8) uint64_t slab_bar, acc_bar;
     __shared__ uint32_t s_tmem;
     __shared__ int s_fail;
-    __shared__ __align__(8) uint64_t slab_bar;
     unsigned char *smem = reinterpret_cast<unsigned char *>(
         (reinterpret_cast<uintptr_t>(p_smem) + 1023) & ~(uintptr_t)1023);
     constexpr int SB = A_BYTES + B_BYTES;
@@ -285,21 +307,23 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int KT = K / BK, nsplit = STAGE1 ? P.split : 1;
     const int kbeg = (int)((long long)blockIdx.z * KT / nsplit);
     const int KC = (int)((long long)(blockIdx.z + 1) * KT / nsplit) - kbeg;
-    const int warp = threadIdx.x >> 5;
-    const bool t0 = threadIdx.x == 0;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int bn = STAGE1 ? P.bn1 : BN;
+    volatile int *fail = &s_fail;
     if (ld_relaxed_gpu(P.ws_words + kErrWord) != 0u) return;
 
-    if (t0) {
+    if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             mb_init(full + s, 1);
-            mb_init(done + s, 1);
+            mb_init(ready + s, kWorkWarps);
+            mb_init(empty + s, 1);
         }
         mb_init(&slab_bar, 1);
+        mb_init(&acc_bar, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         s_fail = 0;
     }
-    if (warp == 0) {
+    if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                          su32(&s_tmem)),
                      "r"(BN)
@@ -315,13 +339,24 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto A_of = [&](int s) { return smem + s * SB; };
     auto B_of = [&](int s) { return smem + s * SB + A_BYTES; };
     auto S_of = [&](int s) { return smem + RING_BYTES + s * SRC_BYTES; };
-    int loads_issued = 0, mmas_issued = 0;  // K-chunks loaded / multiplied (thread 0)
+    auto give_up = [&]() {
+        *fail = 1;
+        atomicCAS(P.ws_words + kErrWord, 0u, static_cast<unsigned>(LB_ERR_TIMEOUT));
+    };
+    int loads_issued = 0, mmas_issued = 0;  // K-chunks loaded / multiplied
     // The x / z tile of the CTA's K-chunk i (chunk kbeg + i of the layer) by
     // TMA; in stage 1 also the chunk's two V word rows for the tile's columns
     // and the chunk's g values, by bulk copy.
     auto issue_load = [&](int i) {
         const int s = i % STAGES, kc = kbeg + i;
         uint64_t *b = full + s;
+        if (P.expanded) {
+            // both operands by TMA: the B tile is rows [n0, n0 + bn) of bv / bu
+            mb_expect_tx(b, (unsigned)(A_BYTES + bn * BK * 2));
+            tma_load_2d(A_of(s), &amap, kc * BK, m0, b);
+            tma_load_2d(B_of(s), &bmap, kc * BK, n0, b);
+            return;
+        }
         if (STAGE1) {
             unsigned char *src = S_of(s);
             for (int p = 0; p < P.L.n_paths; ++p) {
@@ -343,93 +378,103 @@ __global__ void __launch_bounds__(kThreads, 1)
         mb_expect_tx(b, A_BYTES);
         tma_load_2d(A_of(s), &amap, kc * BK, m0, b);
     };
-    if (t0) {
-        if (!STAGE1) {
-            // the tile's U rows and h of every path, once
-            const int nrows = min(BN, P.d_out - n0);
-            for (int p = 0; p < P.L.n_paths; ++p) {
-                const int R = ((p ? P.L.r[1] : P.L.r[0]) + 31) >> 5;
-                mb_expect_only(&slab_bar, (unsigned)(nrows * R * 4 + nrows * 2));
-                bulk_g2s(slab + p * SLAB_U_BYTES, (p ? P.L.u[1] : P.L.u[0]) + (size_t)n0 * R,
-                         (unsigned)(nrows * R * 4), &slab_bar);
-                bulk_g2s(slab + 2 * SLAB_U_BYTES + p * BN * 2, (p ? P.L.h[1] : P.L.h[0]) + n0,
-                         (unsigned)(nrows * 2), &slab_bar);
-            }
-            asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(&slab_bar))
-                         : "memory");
-        }
-        for (int kc = 0; kc < 2 && kc < KC; ++kc) issue_load(kc);
-        loads_issued = KC < 2 ? KC : 2;
-    }
-    bool slab_ok = true;
-    if (!STAGE1) slab_ok = mb_wait(&slab_bar, 0);
 
-    bool ok = __syncthreads_and(slab_ok) != 0;
-    for (int kc = 0; kc < KC && ok; ++kc) {
-        const int s = kc % STAGES;
-        // refill two stages ahead once the MMAs that last read that stage finished
-        if (t0 && kc + 2 < KC) {
-            const int kr = kc + 2;
-            if (kr >= STAGES && !mb_wait(done + (kr % STAGES), (unsigned)(((kr / STAGES) - 1) & 1)))
-                s_fail = 1;
-            else {
-                issue_load(kr);
+    if (warp == 0) {
+        // ---------------- producer: copies for chunk i once the MMAs of
+        //                  chunk i - STAGES have released its stage
+        if (lane == 0) {
+            if (!STAGE1 && !P.expanded) {
+                // the tile's U rows and h of every path, once
+                const int nrows = min(BN, P.d_out - n0);
+                for (int p = 0; p < P.L.n_paths; ++p) {
+                    const int R = ((p ? P.L.r[1] : P.L.r[0]) + 31) >> 5;
+                    mb_expect_only(&slab_bar, (unsigned)(nrows * R * 4 + nrows * 2));
+                    bulk_g2s(slab + p * SLAB_U_BYTES, (p ? P.L.u[1] : P.L.u[0]) + (size_t)n0 * R,
+                             (unsigned)(nrows * R * 4), &slab_bar);
+                    bulk_g2s(slab + 2 * SLAB_U_BYTES + p * BN * 2,
+                             (p ? P.L.h[1] : P.L.h[0]) + n0, (unsigned)(nrows * 2), &slab_bar);
+                }
+                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(&slab_bar))
+                             : "memory");
+            }
+            for (int i = 0; i < KC; ++i) {
+                const int s = i % STAGES;
+                if (i >= STAGES &&
+                    !mb_wait_role(empty + s, (unsigned)((i / STAGES - 1) & 1), fail)) {
+                    give_up();
+                    break;
+                }
+                issue_load(i);
                 ++loads_issued;
             }
         }
-        __syncthreads();
-        if (s_fail) {
-            ok = false;
-            break;
-        }
-        if (!mb_wait(full + s, (unsigned)((kc / STAGES) & 1))) s_fail = 1;
-        __syncthreads();
-        if (s_fail) {
-            ok = false;
-            break;
-        }
-        unpack_b<STAGE1>(P, B_of(s), S_of(s), slab, kbeg + kc, n0, bn);
-        if (s_fail) {
-            ok = false;
-            break;
-        }
-        if (STAGE1) convert_a(A_of(s));
-        fence_proxy_async_smem();
-        __syncthreads();
-        if (t0) {
-            tc_fence_after();
-            const uint32_t a0 = su32(A_of(s)), b0 = su32(B_of(s));
+        __syncwarp();
+    } else if (warp == 1) {
+        // ---------------- MMA issuer
+        if (lane == 0) {
+            for (int i = 0; i < KC; ++i) {
+                const int s = i % STAGES;
+                if (!mb_wait_role(ready + s, (unsigned)((i / STAGES) & 1), fail)) {
+                    give_up();
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t a0 = su32(A_of(s)), b0 = su32(B_of(s));
 #pragma unroll
-            for (int k = 0; k < BK / 16; ++k)
-                mma_f16(tmem, smem_desc(a0 + 32 * k), smem_desc(b0 + 32 * k), idesc,
-                        (kc > 0 || k > 0) ? 1u : 0u);
-            mma_commit(done + s);
-            ++mmas_issued;
+                for (int k = 0; k < BK / 16; ++k)
+                    mma_f16(tmem, smem_desc(a0 + 32 * k), smem_desc(b0 + 32 * k), idesc,
+                            (i > 0 || k > 0) ? 1u : 0u);
+                mma_commit(empty + s);
+                ++mmas_issued;
+            }
+            if (mmas_issued == KC) mma_commit(&acc_bar);
         }
-    }
-    // wait for the last MMA (the accumulator is complete when its commit lands)
-    if (ok && KC > 0) {
-        const int kl = KC - 1;
-        if (!mb_wait(done + (kl % STAGES), (unsigned)((kl / STAGES) & 1))) ok = false;
-    }
-    if (!ok) {
-        if (t0) {
-            atomicCAS(P.ws_words + kErrWord, 0u, static_cast<unsigned>(LB_ERR_TIMEOUT));
-            // let every issued copy and MMA land before the CTA goes away: for
-            // each stage wait for the phase of its last issued use
-            for (int kc = loads_issued - STAGES; kc < loads_issued; ++kc)
-                if (kc >= 0) mb_wait(full + kc % STAGES, (unsigned)((kc / STAGES) & 1));
-            for (int kc = mmas_issued - STAGES; kc < mmas_issued; ++kc)
-                if (kc >= 0) mb_wait(done + kc % STAGES, (unsigned)((kc / STAGES) & 1));
-            if (!STAGE1) mb_wait(&slab_bar, 0);
-        }
-        __syncthreads();
+        __syncwarp();
     } else {
+        // ---------------- unpacking warps: +-scale B and fp16 A of each stage
+        const int tid = threadIdx.x - 64;
+        bool ok = STAGE1 || P.expanded || mb_wait_role(&slab_bar, 0, fail);
+        if (!ok) give_up();
+        for (int i = 0; i < KC && ok; ++i) {
+            const int s = i % STAGES;
+            if (!mb_wait_role(full + s, (unsigned)((i / STAGES) & 1), fail)) {
+                give_up();
+                break;
+            }
+            if (!P.expanded) unpack_b<STAGE1>(P, B_of(s), S_of(s), slab, kbeg + i, n0, bn, tid);
+            if (STAGE1) convert_a(A_of(s), tid);
+            fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0)
+                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(ready + s))
+                             : "memory");
+        }
+    }
+    // the accumulator is complete when the last commit lands
+    bool ok = true;
+    if (warp >= 2 && KC > 0 && !mb_wait_role(&acc_bar, 0, fail)) {
+        if (lane == 0) give_up();
+        ok = false;
+    }
+    ok = __syncthreads_and(ok && !*fail) != 0;
+    if (!ok) {
+        // let every issued copy and MMA land before the CTA goes away: for
+        // each stage wait (bounded) for the phase of its last issued use
+        if (threadIdx.x == 0) {
+            for (int i = loads_issued - STAGES; i < loads_issued; ++i)
+                if (i >= 0) mb_wait(full + i % STAGES, (unsigned)((i / STAGES) & 1));
+            if (!STAGE1 && !P.expanded) mb_wait(&slab_bar, 0);
+        }
+        if (threadIdx.x == 32)
+            for (int i = mmas_issued - STAGES; i < mmas_issued; ++i)
+                if (i >= 0) mb_wait(empty + i % STAGES, (unsigned)((i / STAGES) & 1));
+        __syncthreads();
+    } else if (warp >= 2) {
         tc_fence_after();
         // epilogue: warp w reads TMEM lanes 32(w%4) .. +31 (tile rows) and
-        // the (w/4)-th half of the tile's 32-column chunks
-        const int wq = warp & 3, half = warp >> 2, nchunk = bn / 32;
-        const int row = m0 + 32 * wq + (threadIdx.x & 31);
+        // one half of the tile's 32-column chunks
+        const int wq = warp & 3, half = (warp - 2) >> 2, nchunk = bn / 32;
+        const int row = m0 + 32 * wq + lane;
         const uint32_t lane_base = tmem + ((uint32_t)(32 * wq) << 16);
         const int cb0 = 32 * (half * nchunk / 2), cb1 = 32 * ((half + 1) * nchunk / 2);
         for (int cb = cb0; cb < cb1; cb += 32) {
@@ -506,7 +551,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     tc_fence_before();
     __syncthreads();
-    if (warp == 0)
+    if (warp == 1)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                      "r"(BN)
                      : "memory");
@@ -540,6 +585,41 @@ __global__ void k_reduce_z(const __grid_constant__ PrefillParams P) {
     }
 }
 
+// bv[n][k] = +-g_p[k]: input k of column n (column j of path p) of V_sign,
+// eight inputs (one 16-byte chunk) per thread.
+__global__ void k_expand_v(const __grid_constant__ PrefillParams P) {
+    const int kq = P.L.d_in / 8;
+    const long long n_items = (long long)P.N1 * kq;
+    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < n_items;
+         idx += (long long)gridDim.x * blockDim.x) {
+        const int n = (int)(idx / kq), k0 = 8 * (int)(idx % kq);
+        const int p = n >= P.off1 ? 1 : 0, j = n - (p ? P.off1 : 0);
+        const int r = p ? P.L.r[1] : P.L.r[0];
+        const uint32_t word = __ldg((p ? P.L.v[1] : P.L.v[0]) + (size_t)(k0 >> 5) * r + j);
+        const uint4 mag = *reinterpret_cast<const uint4 *>((p ? P.L.g[1] : P.L.g[0]) + k0);
+        *reinterpret_cast<uint4 *>(P.bv + (size_t)n * P.L.d_in + k0) =
+            signed8((word >> (k0 & 31)) & 0xffu, mag);
+    }
+}
+
+// bu[o][n] = +-h_p[o]: column n (column j of path p) of row o of U_sign,
+// eight columns per thread.
+__global__ void k_expand_u(const __grid_constant__ PrefillParams P) {
+    const int nq = P.N1 / 8;
+    const long long n_items = (long long)P.d_out * nq;
+    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < n_items;
+         idx += (long long)gridDim.x * blockDim.x) {
+        const int o = (int)(idx / nq), n0 = 8 * (int)(idx % nq);
+        const int p = n0 >= P.off1 ? 1 : 0, j0 = n0 - (p ? P.off1 : 0);
+        const int R = ((p ? P.L.r[1] : P.L.r[0]) + 31) >> 5;
+        const uint32_t word = __ldg((p ? P.L.u[1] : P.L.u[0]) + (size_t)o * R + (j0 >> 5));
+        const uint32_t hb = __ldg((p ? P.L.h[1] : P.L.h[0]) + o);
+        const uint32_t hh = hb | (hb << 16);
+        *reinterpret_cast<uint4 *>(P.bu + (size_t)o * P.N1 + n0) =
+            signed8((word >> (j0 & 31)) & 0xffu, make_uint4(hh, hh, hh, hh));
+    }
+}
+
 // ---------------------------------------------------------------- host side
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
@@ -560,10 +640,10 @@ bool encoder() {
 // 2-D map over a row-major [rows][cols] 16-bit matrix, box BK x BM, 128B swizzle,
 // out-of-range rows read as zero.
 bool make_map(CUtensorMap *m, const void *base, CUtensorMapDataType dt, int64_t rows,
-              int64_t cols) {
+              int64_t cols, int box_rows = BM) {
     const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
     const cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
-    const cuuint32_t box[2] = {BK, BM};
+    const cuuint32_t box[2] = {BK, (cuuint32_t)box_rows};
     const cuuint32_t estr[2] = {1, 1};
     return g_encode(m, dt, 2, const_cast<void *>(base), dims, strides, box, estr,
                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -621,11 +701,20 @@ int split_of(const lb_linear &L, int64_t T) {
 size_t z16_bytes(const lb_linear &L, int64_t T) {
     return ((size_t)T * n1_of(L) * 2 + 255) & ~(size_t)255;
 }
+size_t zpart_bytes(const lb_linear &L, int64_t T) {
+    const int S = split_of(L, T);
+    return S > 1 ? ((size_t)S * T * n1_of(L) * 4 + 255) & ~(size_t)255 : 0;
+}
+// From four token tiles on, every tile would unpack the same sign bits: the
+// B operands are expanded to fp16 once per call instead (workspace).
+bool expanded_of(const lb_linear &, int64_t T) { return (T + BM - 1) / BM >= 4; }
+size_t bv_bytes(const lb_linear &L) { return ((size_t)n1_of(L) * L.d_in * 2 + 255) & ~(size_t)255; }
+size_t bu_bytes(const lb_linear &L) { return ((size_t)L.d_out * n1_of(L) * 2 + 255) & ~(size_t)255; }
 }  // namespace
 
 size_t prefill_ws_bytes(const lb_linear &L, int64_t T) {
-    const int S = split_of(L, T);
-    return z16_bytes(L, T) + (S > 1 ? (size_t)S * T * n1_of(L) * 4 : 0);
+    return z16_bytes(L, T) + zpart_bytes(L, T) +
+           (expanded_of(L, T) ? bv_bytes(L) + bu_bytes(L) : 0);
 }
 
 cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, void *y, int y_fp32,
@@ -641,19 +730,34 @@ cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, voi
     P.d_out = L.d_out;
     P.z = static_cast<uint16_t *>(z_ws);
     P.split = split_of(L, T);
-    P.zpart = reinterpret_cast<float *>(static_cast<char *>(z_ws) + z16_bytes(L, T));
+    char *wsb = static_cast<char *>(z_ws);
+    P.zpart = reinterpret_cast<float *>(wsb + z16_bytes(L, T));
+    P.expanded = expanded_of(L, T) ? 1 : 0;
+    P.bv = reinterpret_cast<uint16_t *>(wsb + z16_bytes(L, T) + zpart_bytes(L, T));
+    P.bu = reinterpret_cast<uint16_t *>(wsb + z16_bytes(L, T) + zpart_bytes(L, T) + bv_bytes(L));
     P.y = y;
     P.y_fp32 = y_fp32;
     P.ws_words = ws_words;
-    CUtensorMap xmap, zmap;
+    CUtensorMap xmap, zmap, bvmap{}, bumap{};
     if (!make_map(&xmap, x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, T, L.d_in) ||
         !make_map(&zmap, z_ws, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, T, P.N1))
         return cudaErrorInvalidValue;
+    if (P.expanded &&
+        (!make_map(&bvmap, P.bv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, P.N1, L.d_in, P.bn1) ||
+         !make_map(&bumap, P.bu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, L.d_out, P.N1, BN)))
+        return cudaErrorInvalidValue;
     cudaError_t e = set_smem_attributes();
     if (e != cudaSuccess) return e;
+    if (P.expanded) {
+        const long long nv = (long long)P.N1 * (L.d_in / 8), nu = (long long)L.d_out * (P.N1 / 8);
+        k_expand_v<<<(int)std::min<long long>((nv + 255) / 256, 148 * 16), 256, 0, s>>>(P);
+        k_expand_u<<<(int)std::min<long long>((nu + 255) / 256, 148 * 16), 256, 0, s>>>(P);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
     const dim3 g1((unsigned)((T + BM - 1) / BM), (unsigned)((P.N1 + P.bn1 - 1) / P.bn1),
                   (unsigned)P.split);
-    k_prefill<true><<<g1, kThreads, smem_bytes<true>(), s>>>(xmap, P);
+    k_prefill<true><<<g1, kThreads, smem_bytes<true>(), s>>>(xmap, bvmap, P);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     if (P.split > 1) {
@@ -664,7 +768,7 @@ cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, voi
         if (e != cudaSuccess) return e;
     }
     const dim3 g2((unsigned)((T + BM - 1) / BM), (unsigned)((L.d_out + BN - 1) / BN));
-    k_prefill<false><<<g2, kThreads, smem_bytes<false>(), s>>>(zmap, P);
+    k_prefill<false><<<g2, kThreads, smem_bytes<false>(), s>>>(zmap, bumap, P);
     return cudaGetLastError();
 }
 
