@@ -137,6 +137,11 @@ bool use_prefill(const lb_linear &L, int64_t T) {
     return T >= kPrefillMinTokens && lb::prefill_supported(L, T);
 }
 
+// Workspace of a linear: header | the single-token kernel's exchange words
+// (a region no other path writes, so it stays clean between its launches) |
+// the data of the path a call takes.
+size_t linear_data_offset(const lb_linear &L) { return kWsHeader + lb::decode_ws_bytes(L); }
+
 }  // namespace
 
 lb_status lb::validate_linear(const lb_linear *L) { return check_linear(L); }
@@ -169,14 +174,12 @@ lb_status littlebit_pack(const int8_t *signs, int64_t rows, int64_t cols, int32_
 
 size_t littlebit_workspace_size(const lb_linear *L, int64_t T) {
     if (check_linear(L) != LB_OK || T < 0) return 0;
-    size_t floats = lb::generic_ws_floats(*L, T);
-    // the decode path falls back to the two-launch path when its grid cannot
-    // be co-resident, so size for both
-    if (use_decode(*L, T) && lb::decode_ws_floats(*L) > floats) floats = lb::decode_ws_floats(*L);
+    const size_t floats = lb::generic_ws_floats(*L, T);
     size_t bytes = (floats * sizeof(float) + 255) & ~(size_t)255;
     if (use_prefill(*L, T) && lb::prefill_ws_bytes(*L, T) > bytes) bytes = lb::prefill_ws_bytes(*L, T);
-    return kWsHeader + bytes;
+    return linear_data_offset(*L) + bytes;
 }
+
 
 lb_status littlebit_linear_forward(const lb_linear *L, const uint16_t *x, int64_t T, void *y,
                                    int32_t y_dtype, void *ws, size_t ws_bytes,
@@ -194,12 +197,13 @@ lb_status littlebit_linear_forward(const lb_linear *L, const uint16_t *x, int64_
     if ((st = num_sms(&sms)) != LB_OK) return st;
     cudaStream_t s = (cudaStream_t)stream;
     unsigned *words = static_cast<unsigned *>(ws);
-    float *data = reinterpret_cast<float *>(static_cast<char *>(ws) + kWsHeader);
+    float *data = reinterpret_cast<float *>(static_cast<char *>(ws) + linear_data_offset(*L));
     const int fp32 = y_dtype == LB_OUT_FP32;
-    if (use_decode(*L, T)) {
-        cudaError_t e = lb::launch_decode(*L, x, y, fp32, words, data, sms, s);
+    if (use_decode(*L, T) && lb::decode_supported(*L, sms)) {
+        cudaError_t e = lb::launch_decode(*L, x, y, fp32, words,
+                                          static_cast<char *>(ws) + kWsHeader, sms, s);
         if (e != cudaErrorCooperativeLaunchTooLarge) return from_cuda(e);
-        cudaGetLastError();  // grid cannot be co-resident here: take the two-launch path
+        cudaGetLastError();  // too large for one co-resident grid: take the two-launch path
     }
     if (use_prefill(*L, T)) return from_cuda(lb::launch_prefill(*L, x, T, y, fp32, words, data, s));
     return from_cuda(lb::launch_generic(*L, x, T, y, fp32, data, sms, s));

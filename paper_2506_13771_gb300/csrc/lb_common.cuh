@@ -19,12 +19,15 @@ constexpr unsigned long long kWaitLimitNs = 1000000000ull;  // 1 s per grid-wide
 //               only by littlebit_poll_error
 //   word 1    : grid-barrier arrival counter
 //   word 2    : count of CTAs that finished a stack launch
+//   word 3    : launch epoch of the single-token kernel (selects which of its
+//               two exchange-word buffers a launch uses)
 //   words 4-5 : 64-bit fingerprint of the linears a stack workspace was
 //               prepared for (littlebit_stack_prepare)
 constexpr size_t kWsHeader = 256;
 constexpr int kErrWord = 0;
 constexpr int kCounterWord = 1;
 constexpr int kDoneWord = 2;
+constexpr int kEpochWord = 3;  // launches of the single-token kernel on this workspace
 constexpr int kPlanWord = 4;
 
 // Device copy of one linear (paths 0..n_paths-1).

@@ -20,11 +20,14 @@ size_t generic_ws_floats(const lb_linear &L, int64_t T);
 cudaError_t launch_generic(const lb_linear &L, const uint16_t *x, int64_t T, void *y, int y_fp32,
                            float *t_acc, int num_sms, cudaStream_t s);
 
-// Single-launch persistent decode of one linear, T = 1 (lb_persistent.cu).
-size_t decode_ws_floats(const lb_linear &L);
+// Single-launch decode of one linear, T = 1 (lb_decode.cu): ranks multiples
+// of 8, d_out a multiple of 8.  xw: decode_ws_bytes of exchange words (two
+// buffers), zero before the first launch; completed launches keep them so.
 // Returns cudaErrorCooperativeLaunchTooLarge when the grid cannot be co-resident.
+bool decode_supported(const lb_linear &L, int num_sms);
+size_t decode_ws_bytes(const lb_linear &L);
 cudaError_t launch_decode(const lb_linear &L, const uint16_t *x, void *y, int y_fp32,
-                          unsigned *ws_words, float *acc, int num_sms, cudaStream_t s);
+                          unsigned *ws_words, void *xw, int num_sms, cudaStream_t s);
 
 // Persistent decode of the seven-linear-per-layer stack (lb_stack.cu).
 struct StackShape {
