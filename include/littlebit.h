@@ -45,6 +45,8 @@
  *     record LB_ERR_TIMEOUT in the workspace's sticky error word and return;
  *     while that word is set, kernels using the workspace return at once
  *     without writing outputs; littlebit_poll_error reads and clears it.
+ *     A launch that timed out may leave exchange words behind: zero-fill the
+ *     workspace again (or prepare a stack workspace again) before reusing it.
  */
 #ifndef LITTLEBIT_H
 #define LITTLEBIT_H
@@ -113,7 +115,13 @@ size_t littlebit_workspace_size(const lb_linear *L, int64_t T);
 /* Y = X W^T for one LittleBit linear (Prop. 1 per path, paths summed by
  * Eq. 6).  L is a HOST struct holding device pointers.  x: bf16 [T][d_in];
  * y: [T][d_out] in y_dtype.  T = 0 is a no-op.  Requires d_in % 32 == 0 and
- * 1 <= r <= 1024 for every path (else LB_ERR_UNSUPPORTED). */
+ * 1 <= r <= 1024 for every path (else LB_ERR_UNSUPPORTED).
+ * Paths taken: T = 1 with every r % 8 == 0 and d_out % 8 == 0 -> one launch
+ * of the single-token kernel (it keeps its exchange words in ws between
+ * calls, so a workspace must not be shared by concurrent calls); T >= 16
+ * with d_in and every r multiples of 64, r <= 512 and d_out % 8 == 0 -> the
+ * tensor-core path (fp16 operands, see its tolerance in the design notes);
+ * otherwise the two-launch CUDA-core path. */
 lb_status littlebit_linear_forward(const lb_linear *L, const uint16_t *x, int64_t T, void *y,
                                    int32_t y_dtype, void *ws, size_t ws_bytes,
                                    lb_stream_t stream);
