@@ -970,15 +970,6 @@ struct ProgBuild {
     Step step[N_STEPS] = {};
     std::vector<Item> items;
 
-    // Up to 32 tables of one job per unit, one unit per warp where possible.
-    void tables(int s, const std::vector<Item> &jobs) {
-        std::vector<Costed> us;
-        for (const Item &J : jobs) table_units(J, 0, J.f[1], us);
-        std::vector<Item> g;
-        int wo[kCW + 1];
-        lpt(us, g, wo);
-        place(s, g, wo);
-    }
     void place(int s, const std::vector<Item> &grouped, const int (&wo)[kCW + 1]) {
         step[s].first = (int)items.size();
         for (int w = 0; w <= kCW; ++w) step[s].wo[w] = wo[w];
