@@ -78,6 +78,10 @@ def _bind(lib):
     lib.lbo_forward_factored.restype = ctypes.c_int
     lib.lbo_apply_factored.argtypes = [ctypes.POINTER(Linear), vp, i64, vp, vp]
     lib.lbo_apply_factored.restype = ctypes.c_int
+    lib.lbo_latent.argtypes = [ctypes.POINTER(Linear), vp, i64, vp]
+    lib.lbo_latent.restype = ctypes.c_int
+    lib.lbo_expand.argtypes = [ctypes.POINTER(Linear), vp, i64, vp]
+    lib.lbo_expand.restype = None
     lib.lbo_stack_forward.argtypes = [ctypes.POINTER(Linear), ctypes.c_int32, ctypes.c_int32,
                                       vp, vp, vp, vp]
     lib.lbo_stack_forward.restype = ctypes.c_int
@@ -211,6 +215,26 @@ class Oracle:
             off += T * r
         return y, ts
 
+    def latent(self, layer: dict, x_bf16: np.ndarray) -> np.ndarray:
+        """Latent states z [T][r_0 + r_1] (l_p . (X . g_p) V_p,sign per path), fp64."""
+        hold = _Holder(layer)
+        x = _c(x_bf16, np.uint16)
+        n1 = sum(int(P["r"]) for P in layer["paths"])
+        z = np.zeros((x.shape[0], n1), dtype=np.float64)
+        if self.lib.lbo_latent(ctypes.byref(hold.c), _ptr(x), x.shape[0], _ptr(z)):
+            raise MemoryError("oracle latent failed")
+        return z
+
+    def expand(self, layer: dict, z: np.ndarray) -> np.ndarray:
+        """Y [T][d_out] = sum_p h_p . (U_p,sign z_p) from latents in latent()'s layout."""
+        hold = _Holder(layer)
+        Z = _c(z, np.float64)
+        n1 = sum(int(P["r"]) for P in layer["paths"])
+        assert Z.ndim == 2 and Z.shape[1] == n1
+        y = np.zeros((Z.shape[0], layer["d_out"]), dtype=np.float64)
+        self.lib.lbo_expand(ctypes.byref(hold.c), _ptr(Z), Z.shape[0], _ptr(y))
+        return y
+
     def stack_forward(self, layers: list, x0_bf16: np.ndarray, head_dim: int = 128,
                       want_q: bool = True, want_kv: bool = True):
         """Decode step at position 0 through n_layers x (q,k,v,o,gate,up,down);
@@ -265,7 +289,8 @@ def _forward(name):
 
 
 for _name in ("half_to_double", "bf16_to_double", "pack_u", "pack_v", "unpack_u", "unpack_v",
-              "forward_dense", "forward_factored", "apply_factored", "stack_forward",
+              "forward_dense", "forward_factored", "apply_factored", "latent", "expand",
+              "stack_forward",
               "bpw", "rank_for_bpw", "flops", "set_threads", "get_threads"):
     globals()[_name] = _forward(_name)
 del _name

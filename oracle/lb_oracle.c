@@ -263,6 +263,63 @@ int lbo_forward_factored(const lbo_linear *L, const uint16_t *x, int64_t T, doub
 }
 
 /* ------------------------------------------------------------------------ */
+/* Latent states (Sec. 5 "KV Cache Compression", Fig. 5, Table 4)          */
+/* ------------------------------------------------------------------------ */
+
+/* The rank-r latent of each path, the bracketed inner product of Prop. 1
+ * after the latent scale: z_p[t][j] = l_p[j] * sum_i V_p,sign[i][j] g_p[i] X[t][i].
+ * Stored as [T][r_0 + r_1]: path 0 in columns 0..r_0-1, path 1 after it. */
+int lbo_latent(const lbo_linear *L, const uint16_t *x, int64_t T, double *z)
+{
+    int64_t din = L->d_in, n1 = 0;
+    for (int p = 0; p < L->n_paths; p++)
+        n1 += L->path[p].r;
+    double *X = decode_bf16_array(x, T * din);
+    if (!X)
+        return -1;
+    int64_t off = 0;
+    for (int p = 0; p < L->n_paths; p++) {
+        const lbo_path *P = &L->path[p];
+        int64_t r = P->r;
+#pragma omp parallel for schedule(static)
+        for (int64_t tj = 0; tj < T * r; tj++) {
+            int64_t tt = tj / r, j = tj % r;
+            double s = 0.0;
+            for (int64_t i = 0; i < din; i++)
+                s += X[tt * din + i] * lbo_half_to_double(P->g[i]) * sign_v(P->v_words, r, i, j);
+            z[tt * n1 + off + j] = lbo_half_to_double(P->l[j]) * s;
+        }
+        off += r;
+    }
+    free(X);
+    return 0;
+}
+
+/* The output rebuilt from cached latents, Prop. 1's outer part per path,
+ * summed over paths (Eq. 6): y[t][o] = sum_p h_p[o] sum_j U_p,sign[o][j] z_p[t][j],
+ * z in the layout lbo_latent writes. */
+void lbo_expand(const lbo_linear *L, const double *z, int64_t T, double *y)
+{
+    int64_t dout = L->d_out, n1 = 0;
+    for (int p = 0; p < L->n_paths; p++)
+        n1 += L->path[p].r;
+#pragma omp parallel for schedule(static)
+    for (int64_t to = 0; to < T * dout; to++) {
+        int64_t tt = to / dout, o = to % dout, off = 0;
+        double acc = 0.0;
+        for (int p = 0; p < L->n_paths; p++) {
+            const lbo_path *P = &L->path[p];
+            double s = 0.0;
+            for (int64_t j = 0; j < P->r; j++)
+                s += z[tt * n1 + off + j] * sign_u(P->u_words, P->r, o, j);
+            acc += lbo_half_to_double(P->h[o]) * s;
+            off += P->r;
+        }
+        y[to] = acc;
+    }
+}
+
+/* ------------------------------------------------------------------------ */
 /* Decode chain of the 70B-shaped stack                                     */
 /* ------------------------------------------------------------------------ */
 

@@ -76,6 +76,14 @@ int lbo_forward_factored(const lbo_linear *L, const uint16_t *x, int64_t T, doub
 int lbo_apply_factored(const lbo_linear *L, const double *x, int64_t T, double *y,
                        double *t_out);
 
+/* Latent states (Sec. 5, KV cache compression; Prop. 1's inner product after
+ * the latent scale): z[t][off_p + j] = l_p[j] * ((X[t] . g_p) V_p,sign)[j],
+ * off_0 = 0, off_1 = r_0; z is [T][r_0 + r_1].  x: bf16 [T][d_in].  0 / -1. */
+int lbo_latent(const lbo_linear *L, const uint16_t *x, int64_t T, double *z);
+/* The output from latents: y[t][o] = sum_p h_p[o] (U_p,sign z_p[t])[o], z in
+ * lbo_latent's layout, y: [T][d_out]. */
+void lbo_expand(const lbo_linear *L, const double *z, int64_t T, double *y);
+
 /* One decode step of a Llama-shaped decoder stack at sequence position 0,
  * n_layers x (q, k, v, o, gate, up, down), seven linears per layer in that
  * order, only the linears being LittleBit (the paper's end-to-end setting

@@ -12,7 +12,8 @@ Sources of truth used here, none of which is the oracle:
   * closed forms of Prop. 1 / Eq. 4 for special parameter choices (rank 1,
     all-equal signs, Sylvester-Hadamard factors with unit scales)
   * a hand-expanded quadruple sum over every sign pattern of a tiny layer
-  * the worked examples of App. E and App. I.1 (tests/golden/)
+  * the worked examples of App. E and App. I.1, and Table 4's KV-cache ranks
+    (tests/golden/)
   * algebraic invariants: path-swap symmetry of Eq. 6, h_res = 0 reducing to
     one path
   * for the decoder chain: textbook softmax attention over the one cached
@@ -319,6 +320,116 @@ def pin_padding_ignored(orc):
     assert np.array_equal(orc.forward_dense(Lp, x), orc.forward_dense(L, x))
 
 
+# ------------------------------------------------------------------ pins: latent states
+
+
+def pin_latent_hadamard(orc):
+    """Unit scales, V = U = the first r columns of a Sylvester matrix H: the
+    latent is the first r Walsh-Hadamard coefficients of X, and expanding
+    coefficients c gives FWHT(c padded with zeros).  With two paths that
+    split the columns of H (r_0 + r_1 = d), the latent is the whole transform
+    in column order and expanding it gives d X (H H^T = d I)."""
+    rng = np.random.default_rng(21)
+    d = 256
+    H = sylvester(d)
+    one = lambda n: np.full(n, 0x3C00, np.uint16)  # fp16 1.0
+    x = rand_x(rng, 3, d)
+    c = fwht(np_bf16(x))
+    for r in (200, 1):
+        L = layer_from_signs(orc, d, d, [{"u_signs": H[:, :r].copy(), "v_signs": H[:, :r].copy(),
+                                          "g": one(d), "l": one(r), "h": one(d)}])
+        z = orc.latent(L, x)
+        assert np.array_equal(z, c[:, :r])
+        zp = np.zeros_like(c)
+        zp[:, :r] = z
+        assert np.array_equal(orc.expand(L, z), fwht(zp))
+    r0 = 72
+    L = layer_from_signs(orc, d, d, [
+        {"u_signs": H[:, :r0].copy(), "v_signs": H[:, :r0].copy(), "g": one(d), "l": one(r0),
+         "h": one(d)},
+        {"u_signs": H[:, r0:].copy(), "v_signs": H[:, r0:].copy(), "g": one(d),
+         "l": one(d - r0), "h": one(d)}])
+    z = orc.latent(L, x)
+    assert np.array_equal(z, c)
+    assert np.array_equal(orc.expand(L, z), d * np_bf16(x))
+
+
+def pin_latent_closed_forms(orc):
+    """r = 1: z[t] = l v.(g X[t]); all-equal V signs s: z[t][j] = s l_j sum_i g_i X[t][i];
+    expanding a one-hot latent e_j gives the column h . U[:, j] * 1."""
+    rng = np.random.default_rng(22)
+    d_in, d_out, T = 61, 29, 3
+    x = rand_x(rng, T, d_in)
+    X = np_bf16(x)
+    P = rand_path(rng, d_in, d_out, 1)
+    L = layer_from_signs(orc, d_in, d_out, [P])
+    v = P["v_signs"][:, 0].astype(np.float64)
+    ref = (X @ (v * np_half(P["g"])))[:, None] * np_half(P["l"])[0]
+    assert rel(orc.latent(L, x), ref) <= 1e-14
+    for sv in (1, -1):
+        P = rand_path(rng, d_in, d_out, 9)
+        P["v_signs"] = np.full((d_in, 9), sv, np.int8)
+        L = layer_from_signs(orc, d_in, d_out, [P])
+        ref = sv * np.outer(X @ np_half(P["g"]), np_half(P["l"]))
+        assert rel(orc.latent(L, x), ref) <= 1e-14
+        for j in (0, 4, 8):
+            e = np.zeros((1, 9))
+            e[0, j] = 1.0
+            col = np_half(P["h"]) * P["u_signs"][:, j]
+            assert np.array_equal(orc.expand(L, e)[0], col)
+
+
+def pin_latent_brute_force(orc):
+    """Every V sign pattern of a 2-input rank-2 path: the latent agrees with a
+    hand-expanded l_j sum_i V[i][j] g_i X[t][i]; every U pattern of a 2 x 2 U:
+    the expansion agrees with h_o sum_j U[o][j] z[t][j]."""
+    rng = np.random.default_rng(23)
+    d_in, d_out, r, T = 2, 2, 2, 2
+    P = rand_path(rng, d_in, d_out, r)
+    x = rand_x(rng, T, d_in)
+    X = np_bf16(x)
+    g, l, h = np_half(P["g"]), np_half(P["l"]), np_half(P["h"])
+    Z = rng.standard_normal((T, r))
+    for pattern in range(1 << (d_in * r)):
+        S = np.array([1 - 2 * ((pattern >> k) & 1) for k in range(d_in * r)],
+                     np.int8).reshape(d_in, r)
+        L = layer_from_signs(orc, d_in, d_out, [dict(P, v_signs=S, u_signs=S)])
+        zref = np.zeros((T, r))
+        yref = np.zeros((T, d_out))
+        for t in range(T):
+            for j in range(r):
+                for i in range(d_in):
+                    zref[t, j] += l[j] * S[i, j] * g[i] * X[t, i]
+            for o in range(d_out):
+                for j in range(r):
+                    yref[t, o] += h[o] * S[o, j] * Z[t, j]
+        assert rel(orc.latent(L, x), zref) <= 1e-15, pattern
+        assert rel(orc.expand(L, Z), yref) <= 1e-15, pattern
+
+
+def pin_latent_expand_composition(orc):
+    """Expanding the latent gives the forward (Prop. 1 split at its latent),
+    checked against the dense Eq. 4-6 weight; a two-path latent is the two
+    one-path latents side by side, and its expansion the sum of theirs."""
+    rng = np.random.default_rng(24)
+    for (d_in, d_out, rs, T) in [(40, 24, (3, 5), 3), (96, 17, (40,), 2), (64, 33, (17, 16), 2)]:
+        paths = [rand_path(rng, d_in, d_out, r) for r in rs]
+        L = layer_from_signs(orc, d_in, d_out, paths)
+        x = rand_x(rng, T, d_in)
+        z = orc.latent(L, x)
+        assert z.shape == (T, sum(rs))
+        y = orc.expand(L, z)
+        yd = orc.forward_dense(L, x)
+        assert rel(y, yd) <= 1e-12, rel(y, yd)
+        if len(rs) == 2:
+            L0 = layer_from_signs(orc, d_in, d_out, paths[:1])
+            L1 = layer_from_signs(orc, d_in, d_out, paths[1:])
+            z0, z1 = orc.latent(L0, x), orc.latent(L1, x)
+            assert np.array_equal(z, np.concatenate([z0, z1], axis=1))
+            ys = orc.expand(L0, z[:, :rs[0]]) + orc.expand(L1, z[:, rs[0]:])
+            assert rel(y, ys) <= 1e-15
+
+
 # ------------------------------------------------------------------ pins: accounting
 
 
@@ -352,6 +463,19 @@ def pin_theoretical_cost(orc):
     for T, d_out, d_in, r, mflops in _golden_rows("theoretical_cost.txt"):
         f = orc.flops(int(T), int(d_out), int(d_in), int(r), 1)
         assert abs(f / 1e6 - float(mflops)) < 0.05, f
+
+
+def pin_kv_cache_table4(orc):
+    """Table 4: the single-path rank for each target bits per weight of a
+    d_model x d_model key/value projection (rounded up to a multiple of 8)
+    and the reduction d_model / r of the cache when the latent replaces the
+    d_model-wide key or value."""
+    for d, b, r, factor in _golden_rows("kv_cache_table4.txt"):
+        d, b, r, factor = int(d), float(b), int(r), float(factor)
+        r_real = orc.rank_for_bpw(b, d, d, 1)
+        assert int(np.ceil(r_real / 8.0)) * 8 == r, (b, r_real, r)
+        assert orc.bpw(d, d, r, 1) >= b
+        assert round(d / r, 1) == factor
 
 
 # ------------------------------------------------------------------ pins: decode chain
@@ -459,5 +583,7 @@ def pin_stack_attention_closed_form(orc):
 ALL_PINS = [pin_fp16_exhaustive, pin_bf16_exhaustive, pin_pack_structured, pin_pack_vs_numpy,
             pin_dense_equals_factored, pin_rank1_closed_form, pin_all_equal_signs,
             pin_hadamard_identity, pin_brute_force, pin_residual_paths, pin_padding_ignored,
-            pin_bpw_worked_examples, pin_theoretical_cost, pin_stack_chain,
+            pin_latent_hadamard, pin_latent_closed_forms, pin_latent_brute_force,
+            pin_latent_expand_composition, pin_bpw_worked_examples, pin_theoretical_cost,
+            pin_kv_cache_table4, pin_stack_chain,
             pin_stack_zero_branches, pin_stack_attention_closed_form]

@@ -42,6 +42,16 @@ MUTATIONS = [
     ("chain_silu_sign", "return x / (1.0 + exp(-x));", "return x / (1.0 + exp(x));"),
     ("bpw_drops_latent_scale", "+ 16.0 * (double)(d_out + d_in + r);", "+ 16.0 * (double)(d_out + d_in);"),
     ("rank_solve_one_path", "(n_paths * s + n_paths * 16.0);", "(s + n_paths * 16.0);"),
+    ("latent_drops_l", "z[tt * n1 + off + j] = lbo_half_to_double(P->l[j]) * s;",
+     "z[tt * n1 + off + j] = s;"),
+    ("latent_drops_g",
+     "s += X[tt * din + i] * lbo_half_to_double(P->g[i]) * sign_v(P->v_words, r, i, j);",
+     "s += X[tt * din + i] * sign_v(P->v_words, r, i, j);"),
+    ("latent_path_offset", "        off += r;\n    }\n    free(X);", "        off += 1;\n    }\n    free(X);"),
+    ("expand_drops_h", "acc += lbo_half_to_double(P->h[o]) * s;", "acc += s;"),
+    ("expand_path_offset", "            off += P->r;", "            off += 0;"),
+    ("expand_u_transposed", "s += z[tt * n1 + off + j] * sign_u(P->u_words, P->r, o, j);",
+     "s += z[tt * n1 + off + j] * sign_u(P->u_words, P->r, j % L->d_out, o % P->r);"),
     ("flops_factor", "return (double)n_paths * 2.0 * (double)T", "return (double)n_paths * 1.0 * (double)T"),
 ]
 
