@@ -13,13 +13,16 @@ on a bounded sample (cpu_baseline), and the SM clocks seen while timing.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                   [--layers L]
-  python bench.py --config 2|3|4 [--steps K] [--warmup W]
+  python bench.py --config 2|3|4|6 [--steps K] [--warmup W]
 
 --config times the single-linear workloads instead (one JSON line per case,
 not the bench line): 2 = 4096x4096 r64 at T = 1, 8; 3 = the FFN triple at
-r = 128, 512 and T = 1, 16, 64; 4 = prefill at T = 2048, 8192.  Cases 2 and 3
-report algorithmic GB/s with L2 flushed before every call; case 4 reports
-TFLOP/s (2 flops per +-1 MAC, both paths) against the dense bf16 peak.
+r = 128, 512 and T = 1, 16, 64; 4 = prefill at T = 2048, 8192; 6 = the
+latent-state halves (littlebit_linear_latent / _expand: the 70B key
+projection at T = 1 and a 4096-token cache, 4096x4096 r512 at T = 2048).
+Cases 2, 3 and the CUDA-core cases of 6 report algorithmic GB/s with L2
+flushed before every call; 4 and the tensor-core cases of 6 report TFLOP/s
+(2 flops per +-1 MAC, both paths) against the dense bf16 peak.
 
 --impl reference times the CPU oracle (the reference of this build) on the
 same metric; under torchrun only rank 0 runs it.  N > 1 runs independent
@@ -53,7 +56,7 @@ def parse_args():
     ap.add_argument("--layers", type=int, default=80,
                     help="stack depth (80 = the Llama2-70B workload; smaller only for profiling)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--config", type=int, choices=[2, 3, 4], default=None,
+    ap.add_argument("--config", type=int, choices=[2, 3, 4, 6], default=None,
                     help="time a single-linear workload instead of the stack")
     ap.add_argument("--only", default=None,
                     help="with --config: only the cases whose 'name:T' contains this text")
@@ -417,13 +420,26 @@ def run_config(args):
         return sum(P["v_words"].nbytes + P["u_words"].nbytes + 2 * (L["d_in"] + L["d_out"] + P["r"])
                    for P in L["paths"])
 
-    def time_case(L, x_bits, T, cold):
+    def time_case(L, x_bits, T, cold, op="forward"):
+        """Median ms of one call: the forward, the latent (z fp16) or the
+        expansion of an fp16 latent, L2 flushed before each call when cold."""
         D = lb.DeviceLinear(L, dev)
         x = lb.bf16_tensor(x_bits, dev)
         y = torch.empty((T, D.d_out), dtype=torch.bfloat16, device=dev)
         ws = lb.new_workspace(lb.workspace_size(D, T), dev)
+        z = torch.empty((T, sum(D.ranks)), dtype=torch.float16, device=dev)
+        lb.linear_latent(D, x, z=z, ws=ws)
+        if op == "forward":
+            def call():
+                lb.linear_forward(D, x, y=y, ws=ws)
+        elif op == "latent":
+            def call():
+                lb.linear_latent(D, x, z=z, ws=ws)
+        else:
+            def call():
+                lb.linear_expand(D, z, y=y, ws=ws)
         for _ in range(max(3, args.warmup)):
-            lb.linear_forward(D, x, y=y, ws=ws)
+            call()
         torch.cuda.synchronize(dev)
         ts = []
         for _ in range(steps):
@@ -432,7 +448,7 @@ def run_config(args):
             e0 = torch.cuda.Event(enable_timing=True)
             e1 = torch.cuda.Event(enable_timing=True)
             e0.record()
-            lb.linear_forward(D, x, y=y, ws=ws)
+            call()
             e1.record()
             torch.cuda.synchronize(dev)
             ts.append(e0.elapsed_time(e1))
@@ -443,11 +459,21 @@ def run_config(args):
     def wanted(name, T):
         return args.only is None or args.only in f"{name}:{T}"
 
-    def emit(name, cfg, T, L, ms, flops_mode):
-        wb = weight_bytes(L)
-        act = T * (L["d_in"] + L["d_out"]) * 2
-        flops = sum(2 * T * P["r"] * (L["d_in"] + L["d_out"]) for P in L["paths"])
-        line = {"config": cfg, "case": name, "tokens": T, "ms": ms,
+    def emit(name, cfg, T, L, ms, flops_mode, op="forward"):
+        n1 = sum(P["r"] for P in L["paths"])
+        if op == "forward":
+            wb = weight_bytes(L)
+            act = T * (L["d_in"] + L["d_out"]) * 2
+            flops = sum(2 * T * P["r"] * (L["d_in"] + L["d_out"]) for P in L["paths"])
+        elif op == "latent":   # V bits, g, l; x in, z (fp16) out
+            wb = sum(P["v_words"].nbytes + 2 * (L["d_in"] + P["r"]) for P in L["paths"])
+            act = T * (L["d_in"] + n1) * 2
+            flops = sum(2 * T * P["r"] * L["d_in"] for P in L["paths"])
+        else:                  # U bits, h; z (fp16) in, y out
+            wb = sum(P["u_words"].nbytes + 2 * L["d_out"] for P in L["paths"])
+            act = T * (n1 + L["d_out"]) * 2
+            flops = sum(2 * T * P["r"] * L["d_out"] for P in L["paths"])
+        line = {"config": cfg, "case": name, "op": op, "tokens": T, "ms": ms,
                 "us": ms * 1e3, "bytes": wb + act, "flops": flops,
                 "gbs": (wb + act) / ms / 1e6, "tflops": flops / ms / 1e9}
         if flops_mode:
@@ -474,6 +500,23 @@ def run_config(args):
                         continue
                     xin = xd if nm == "down" else x
                     emit(f"{nm} r{r}", 3, T, lins[nm], time_case(lins[nm], xin, T, True), False)
+    elif args.config == 6:
+        # latent states (KV cache compression): the 70B key projection's latent
+        # for one new token and the expansion of a 4096-token latent cache
+        # (CUDA-core stages), and the 4096 x 4096 r512 halves at 2048 tokens
+        # (tensor cores)
+        rng = inputs.rng_for(6)
+        kproj = inputs.make_linear(rng, 8192, 1024, [32, 32], 2, 0.02)
+        cases = [("kv 8192->1024 r32", kproj, 1, "latent", False),
+                 ("kv 8192->1024 r32", kproj, 4096, "expand", False)]
+        L4, x4 = inputs.config4("4096x4096_r512", 2048)
+        cases += [("4096x4096_r512", L4, 2048, "latent", True),
+                  ("4096x4096_r512", L4, 2048, "expand", True)]
+        for name, L, T, op, fl in cases:
+            if not wanted(f"{name} {op}", T):
+                continue
+            x = x4 if T == 2048 else inputs.bf16_normal(rng, (T, L["d_in"]))
+            emit(name, 6, T, L, time_case(L, x, T, True, op), fl, op)
     else:
         for shape in inputs.PREFILL_SHAPES:
             for T in (2048, 8192):

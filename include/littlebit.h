@@ -126,6 +126,40 @@ lb_status littlebit_linear_forward(const lb_linear *L, const uint16_t *x, int64_
                                    int32_t y_dtype, void *ws, size_t ws_bytes,
                                    lb_stream_t stream);
 
+/* Element type of a latent-state buffer (littlebit_linear_latent / _expand). */
+typedef enum { LB_LATENT_FP32 = 0, LB_LATENT_FP16 = 1 } lb_latent_dtype;
+
+/* Latent states of a LittleBit linear (Sec. 5, KV cache compression; Fig. 5,
+ * Table 4): Prop. 1 split after its latent scale.  Per path,
+ *     z_p[t][j] = l_p[j] * sum_i V_p,sign[i][j] g_p[i] X[t][i]
+ * written row-major as z [T][r_0 + r_1] (path 0's r_0 columns, then path
+ * 1's).  Caching z of the key and value projections in place of their
+ * outputs divides the KV cache by d_kv / (r_0 + r_1) (Table 4 lists
+ * d_model / r for one path); littlebit_linear_expand turns z back into the
+ * projection's output.
+ * x: bf16 [T][d_in]; z: device, 16-byte aligned, in z_dtype: LB_LATENT_FP32,
+ * or LB_LATENT_FP16 (round to nearest even; a magnitude above 65504 becomes
+ * inf).  ws: littlebit_workspace_size(L, T) bytes, rules as for the forward.
+ * T = 0 is a no-op.  Shape rules and the choice of path (tensor-core stage 1
+ * with fp16 operands, or the CUDA-core stage 1 with an fp32 reduction) are
+ * those of littlebit_linear_forward for the same L and T, except that one
+ * token also takes the CUDA-core stage. */
+lb_status littlebit_linear_latent(const lb_linear *L, const uint16_t *x, int64_t T, void *z,
+                                  int32_t z_dtype, void *ws, size_t ws_bytes,
+                                  lb_stream_t stream);
+
+/* The projection's output from latent states in littlebit_linear_latent's
+ * layout: Y[t][o] = sum_p h_p[o] sum_j U_p,sign[o][j] z_p[t][j] (Prop. 1's
+ * outer part, paths summed by Eq. 6), so that expanding the latent of X
+ * gives the forward of X up to rounding.  z: device [T][r_0 + r_1] in
+ * z_dtype, 16-byte aligned; y: [T][d_out] in y_dtype.  ws:
+ * littlebit_workspace_size(L, T) bytes.  T = 0 is a no-op.  Path: the
+ * tensor-core stage 2 where the forward would take it (an fp32 z is first
+ * rounded to fp16 in ws), else the CUDA-core stage 2 (fp32 arithmetic). */
+lb_status littlebit_linear_expand(const lb_linear *L, const void *z, int32_t z_dtype, int64_t T,
+                                  void *y, int32_t y_dtype, void *ws, size_t ws_bytes,
+                                  lb_stream_t stream);
+
 /* Workspace bytes littlebit_stack_prepare / littlebit_stack_forward need
  * (0 if the arguments are invalid). */
 size_t littlebit_stack_workspace_size(const lb_linear *lin, int32_t n_layers, int32_t head_dim);

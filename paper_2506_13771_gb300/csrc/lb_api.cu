@@ -209,6 +209,71 @@ lb_status littlebit_linear_forward(const lb_linear *L, const uint16_t *x, int64_
     return from_cuda(lb::launch_generic(*L, x, T, y, fp32, data, sms, s));
 }
 
+lb_status littlebit_linear_latent(const lb_linear *L, const uint16_t *x, int64_t T, void *z,
+                                  int32_t z_dtype, void *ws, size_t ws_bytes,
+                                  lb_stream_t stream) {
+    lb_status st = check_linear(L);
+    if (st != LB_OK) return st;
+    if (T < 0 || (z_dtype != LB_LATENT_FP32 && z_dtype != LB_LATENT_FP16)) return LB_ERR_INVALID_ARG;
+    if (T == 0) return LB_OK;
+    if (T > INT32_MAX / 8) return LB_ERR_UNSUPPORTED;
+    if (!x || !z || !aligned16(x) || !aligned16(z)) return LB_ERR_INVALID_ARG;
+    if (!ws || ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) ||
+        ws_bytes < littlebit_workspace_size(L, T))
+        return LB_ERR_WORKSPACE;
+    int sms = 0;
+    if ((st = num_sms(&sms)) != LB_OK) return st;
+    cudaStream_t s = (cudaStream_t)stream;
+    unsigned *words = static_cast<unsigned *>(ws);
+    char *data = static_cast<char *>(ws) + linear_data_offset(*L);
+    const bool half = z_dtype == LB_LATENT_FP16;
+    if (use_prefill(*L, T))
+        return from_cuda(lb::launch_prefill_latent(
+            *L, x, T, half ? static_cast<uint16_t *>(z) : nullptr,
+            half ? nullptr : static_cast<float *>(z), words, data, s));
+    if (!half) return from_cuda(lb::launch_latent_generic(*L, x, T, static_cast<float *>(z), sms, s));
+    float *z32 = reinterpret_cast<float *>(data);
+    cudaError_t e = lb::launch_latent_generic(*L, x, T, z32, sms, s);
+    if (e == cudaSuccess)
+        e = lb::launch_to_half(z32, static_cast<uint16_t *>(z),
+                               (long long)lb::generic_ws_floats(*L, T), s);
+    return from_cuda(e);
+}
+
+lb_status littlebit_linear_expand(const lb_linear *L, const void *z, int32_t z_dtype, int64_t T,
+                                  void *y, int32_t y_dtype, void *ws, size_t ws_bytes,
+                                  lb_stream_t stream) {
+    lb_status st = check_linear(L);
+    if (st != LB_OK) return st;
+    if (T < 0 || (z_dtype != LB_LATENT_FP32 && z_dtype != LB_LATENT_FP16) ||
+        (y_dtype != LB_OUT_BF16 && y_dtype != LB_OUT_FP32))
+        return LB_ERR_INVALID_ARG;
+    if (T == 0) return LB_OK;
+    if (T > INT32_MAX / 8) return LB_ERR_UNSUPPORTED;
+    if (!z || !y || !aligned16(z) || !aligned16(y)) return LB_ERR_INVALID_ARG;
+    if (!ws || ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) ||
+        ws_bytes < littlebit_workspace_size(L, T))
+        return LB_ERR_WORKSPACE;
+    cudaStream_t s = (cudaStream_t)stream;
+    unsigned *words = static_cast<unsigned *>(ws);
+    char *data = static_cast<char *>(ws) + linear_data_offset(*L);
+    const int fp32 = y_dtype == LB_OUT_FP32;
+    const bool half = z_dtype == LB_LATENT_FP16;
+    if (use_prefill(*L, T)) {
+        const uint16_t *z16 = static_cast<const uint16_t *>(z);
+        if (!half) {
+            // the tensor-core stage takes fp16 operands: round z at the start of ws
+            uint16_t *zc = reinterpret_cast<uint16_t *>(data);
+            const cudaError_t e = lb::launch_to_half(static_cast<const float *>(z), zc,
+                                                     (long long)lb::generic_ws_floats(*L, T), s);
+            if (e != cudaSuccess) return from_cuda(e);
+            z16 = zc;
+        }
+        return from_cuda(lb::launch_prefill_expand(*L, z16, T, y, fp32, words, data, s));
+    }
+    return from_cuda(lb::launch_expand_generic(*L, z, half ? 1 : 0, T, y, fp32, s));
+}
+
 size_t littlebit_stack_workspace_size(const lb_linear *lin, int32_t n_layers, int32_t head_dim) {
     lb::StackShape shape;
     if (check_stack(lin, n_layers, head_dim, &shape) != LB_OK) return 0;

@@ -14,11 +14,19 @@ struct LinDesc;
 // Shape and pointer checks of one linear, as littlebit_linear_forward does them.
 lb_status validate_linear(const lb_linear *L);
 
-// Two-launch CUDA-core path for any T (lb_generic.cu).  t_acc: workspace
-// floats, generic_ws_floats() of them.
+// Two-launch CUDA-core path for any T (lb_generic.cu).  Stage 1 writes the
+// latent z = l . ((X . g) V_sign) as fp32 [T][r_0 + r_1] (z32 is zeroed by the
+// launcher), stage 2 reads z (fp32, or fp16 when z_half) and writes Y.
+// launch_generic runs both with z in z_ws: generic_ws_floats() floats.
 size_t generic_ws_floats(const lb_linear &L, int64_t T);
 cudaError_t launch_generic(const lb_linear &L, const uint16_t *x, int64_t T, void *y, int y_fp32,
-                           float *t_acc, int num_sms, cudaStream_t s);
+                           float *z_ws, int num_sms, cudaStream_t s);
+cudaError_t launch_latent_generic(const lb_linear &L, const uint16_t *x, int64_t T, float *z32,
+                                  int num_sms, cudaStream_t s);
+cudaError_t launch_expand_generic(const lb_linear &L, const void *z, int z_half, int64_t T,
+                                  void *y, int y_fp32, cudaStream_t s);
+// z16[i] = fp16(z32[i]) (round to nearest even), n elements.
+cudaError_t launch_to_half(const float *z32, uint16_t *z16, long long n, cudaStream_t s);
 
 // Single-launch decode of one linear, T = 1 (lb_decode.cu): ranks multiples
 // of 8, d_out a multiple of 8.  xw: decode_ws_bytes of exchange words (two
@@ -50,12 +58,18 @@ cudaError_t launch_stack(const lb_linear *lin, int n_layers, const StackShape &s
                          float *kv_out, unsigned *ws_words, char *ws_after_header, int num_sms,
                          cudaStream_t s);
 
-// Many-token path on the tensor cores (lb_prefill.cu): stage 1 writes z
-// (fp16 [T][sum r]) into z_ws, stage 2 reads it.
+// Many-token path on the tensor cores (lb_prefill.cu).  The latent half
+// writes z = l . ((X . g) V_sign) as fp16 into z16, or as fp32 into z32 when
+// that is not null; the expansion half reads an fp16 z ([T][r_0 + r_1],
+// 16-byte aligned).  ws: prefill_ws_bytes; launch_prefill keeps z at its start.
 bool prefill_supported(const lb_linear &L, int64_t T);
 size_t prefill_ws_bytes(const lb_linear &L, int64_t T);
 cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, void *y, int y_fp32,
-                           unsigned *ws_words, void *z_ws, cudaStream_t s);
+                           unsigned *ws_words, void *ws, cudaStream_t s);
+cudaError_t launch_prefill_latent(const lb_linear &L, const uint16_t *x, int64_t T, uint16_t *z16,
+                                  float *z32, unsigned *ws_words, void *ws, cudaStream_t s);
+cudaError_t launch_prefill_expand(const lb_linear &L, const uint16_t *z16, int64_t T, void *y,
+                                  int y_fp32, unsigned *ws_words, void *ws, cudaStream_t s);
 
 // Bounded-wait diagnostic (lb_persistent.cu).
 cudaError_t launch_wait_timeout(unsigned *ws_words, cudaStream_t s);

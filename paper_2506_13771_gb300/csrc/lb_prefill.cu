@@ -5,25 +5,30 @@
 //   stage 1   z = fp16( l . (X diag(g) V_sign) )     [T x N1],  N1 = sum_p r_p
 //   stage 2   Y = z [diag(h_p) U_p,sign]_p^T          [T x d_out]  (Eq. 6 sum
 //             over the paths is the K dimension of this GEMM)
-// The sign factors never exist in memory as numbers: each CTA unpacks the
-// +-1 bits of its K-slice into shared memory as +-g (stage 1) or +-h (stage
-// 2) fp16 values, in the tensor cores' 128-byte-swizzled K-major layout.
-// The bits come from shared memory too: stage 1 bulk-copies each K-stage's
-// two V word rows (and its 64 g values) on the stage's mbarrier beside the
-// TMA of X; stage 2 bulk-copies the tile's U rows and h once per CTA.  X
-// arrives by TMA (bf16) and is converted to fp16 in shared memory (exact for
-// |x| < 65504); z goes to the workspace as fp16 and comes back by TMA.
+// Below four token tiles the sign factors never exist in memory as numbers:
+// each CTA unpacks the +-1 bits of its K-slice into shared memory as +-g
+// (stage 1) or +-h (stage 2) fp16 values, in the tensor cores' 128-byte-
+// swizzled K-major layout.  The bits come from shared memory too: stage 1
+// bulk-copies each K-stage's two V word rows (and its 64 g values) on the
+// stage's mbarrier beside the TMA of X; stage 2 bulk-copies the tile's U rows
+// and h once per CTA.  X arrives by TMA (bf16) and is converted to fp16 in
+// shared memory (exact for |x| < 65504).  From four token tiles on, every
+// tile would repeat that work, so one pre-pass writes the +-g / +-h operands
+// and an fp16 copy of X to the workspace and both GEMMs stream plain fp16
+// tiles by TMA.  z goes to the workspace as fp16 and comes back by TMA.
 //
 // One CTA computes a 128 x BN tile (BN <= 256 fp32 TMEM columns) with
 // specialised warps: warp 0 issues the TMA / bulk copies of each 64-element
 // K-stage into a 4-deep shared-memory ring, warps 2..9 unpack and convert a
-// stage as soon as it lands, and warp 1 issues its MMAs (tcgen05.mma, one
-// thread) as soon as it is unpacked; tcgen05.commit hands the stage back to
-// the copy warp.  Per stage, full / ready / empty mbarriers order the three
-// roles, so no CTA-wide barrier sits in the K loop.  Every wait is bounded
-// (about one second); on a timeout the CTA records LB_ERR_TIMEOUT, the other
-// roles stop, the CTA waits for its own copies and MMAs in flight, frees its
-// TMEM and returns.
+// stage as soon as it lands (only without the pre-pass), and warp 1 issues
+// its MMAs (tcgen05.mma, one thread) as soon as the stage is ready;
+// tcgen05.commit hands the stage back to the copy warp.  Per stage, full /
+// ready / empty mbarriers order the three roles, so no CTA-wide barrier sits
+// in the K loop; the two single-thread roles poll with test_wait, which
+// notices a completed phase sooner than a suspended try_wait.  Every wait is
+// bounded (about one second); on a timeout the CTA records LB_ERR_TIMEOUT, the
+// other roles stop, the CTA waits for its own copies and MMAs in flight,
+// frees its TMEM and returns.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -63,6 +68,7 @@ __host__ __device__ constexpr int smem_bytes() {
     return RING_BYTES + (STAGE1 ? STAGES * SRC_BYTES : SLAB_BYTES) + 1024;
 }
 static_assert(smem_bytes<true>() <= 232448 && smem_bytes<false>() <= 232448, "shared memory");
+constexpr int kTilesSmem = RING_BYTES + 1024;  // the persistent form: the A|B ring only
 
 extern __shared__ __align__(1024) unsigned char p_smem[];
 
@@ -105,6 +111,30 @@ __device__ bool mb_wait_role(uint64_t *b, unsigned parity, volatile int *fail) {
     if (mb_try(b, parity)) return true;
     const unsigned long long t0 = globaltimer_ns();
     while (!mb_try(b, parity)) {
+        if (*fail) return false;
+        if (globaltimer_ns() - t0 > kWaitLimitNs) return false;
+    }
+    return true;
+}
+
+__device__ __forceinline__ bool mb_test(uint64_t *b, unsigned parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tmbarrier.test_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(su32(b)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// mb_wait_role for the single-thread roles on the pipeline's critical path
+// (copy issuer, MMA issuer): a test_wait spin, which sees a completed phase
+// sooner than a suspended try_wait wakes up.
+__device__ bool mb_spin_role(uint64_t *b, unsigned parity, volatile int *fail) {
+    if (mb_test(b, parity)) return true;
+    const unsigned long long t0 = globaltimer_ns();
+    while (!mb_test(b, parity)) {
         if (*fail) return false;
         if (globaltimer_ns() - t0 > kWaitLimitNs) return false;
     }
@@ -205,11 +235,14 @@ struct PrefillParams {
     int bn1;           // stage-1 tile width: N1 if N1 <= 256, else 256
     int off1;          // column offset of path 1 in the N1 concatenation (= r_0)
     uint16_t *z;       // stage 1 output / stage 2 input, fp16 [T][N1]
+    float *z32;        // stage 1 output in fp32 instead of z (latent entry point), or null
     float *zpart;      // split stage 1: fp32 partial sums [split][T][N1] (before l)
     int split;         // stage-1 K slices (gridDim.z of stage 1)
     int expanded;      // B operands pre-expanded to fp16 (bv, bu) and loaded by TMA
     uint16_t *bv;      // [N1][d_in]: +-g_p[k] at (column n of path p, input k)
     uint16_t *bu;      // [d_out][N1]: +-h_p[o] at (output o, column n of path p)
+    const uint16_t *x; // stage 1 input, bf16 [T][d_in]
+    uint16_t *xh;      // expanded stage 1: x converted to fp16 once per call [T][d_in]
     void *y;           // stage 2 output [T][d_out]
     int y_fp32;
     unsigned *ws_words;
@@ -286,6 +319,93 @@ __device__ __forceinline__ void convert_a(unsigned char *As, int tid) {
             w[k] = *reinterpret_cast<const uint32_t *>(&h);
         }
         *p = make_uint4(w[0], w[1], w[2], w[3]);
+    }
+}
+
+// One 32-column chunk of a finished accumulator row: columns c0 .. c0 + 31 of
+// output row `row` (stage 1: z, or the fp32 partial sums of K slice zslice
+// when nsplit > 1; stage 2: y).
+template <bool STAGE1>
+__device__ __forceinline__ void store_chunk(const PrefillParams &P, const float (&v)[32], int row,
+                                            int c0, int zslice, int nsplit) {
+    if (STAGE1 && nsplit > 1) {
+        // fp32 partial sums of this K slice; the reduction applies l
+        if (c0 < P.N1) {
+            float4 *dst = reinterpret_cast<float4 *>(
+                P.zpart + ((size_t)zslice * P.T + row) * P.N1 + c0);
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+        }
+    } else if (STAGE1 && P.z32) {
+        // z = l . t as fp32
+        if (c0 < P.N1) {
+            const int p = c0 >= P.off1 ? 1 : 0;  // 32 | off1
+            const int j0 = c0 - (p ? P.off1 : 0);
+            const uint16_t *lp = (p ? P.L.l[1] : P.L.l[0]) + j0;
+            float4 *dst = reinterpret_cast<float4 *>(P.z32 + (size_t)row * P.N1 + c0);
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                dst[q] = make_float4(v[4 * q] * half_bits_to_float(__ldg(lp + 4 * q)),
+                                     v[4 * q + 1] * half_bits_to_float(__ldg(lp + 4 * q + 1)),
+                                     v[4 * q + 2] * half_bits_to_float(__ldg(lp + 4 * q + 2)),
+                                     v[4 * q + 3] * half_bits_to_float(__ldg(lp + 4 * q + 3)));
+        }
+    } else if (STAGE1) {
+        // z = l . t as fp16
+        uint32_t packed[16];
+#pragma unroll
+        for (int i = 0; i < 32; i += 2) {
+            float a = 0.f, b = 0.f;
+            const int c = c0 + i;
+            if (c < P.N1) {
+                const int p = c >= P.off1 ? 1 : 0;
+                const int j = c - (p ? P.off1 : 0);
+                const uint16_t *lp = p ? P.L.l[1] : P.L.l[0];
+                a = v[i] * half_bits_to_float(__ldg(lp + j));
+                b = v[i + 1] * half_bits_to_float(__ldg(lp + j + 1));
+            }
+            const __half2 h = __floats2half2_rn(a, b);
+            packed[i >> 1] = *reinterpret_cast<const uint32_t *>(&h);
+        }
+        if (c0 < P.N1) {
+            uint4 *dst = reinterpret_cast<uint4 *>(P.z + (size_t)row * P.N1 + c0);
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+                dst[q] = make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2],
+                                    packed[4 * q + 3]);
+        }
+    } else {
+        if (P.y_fp32) {
+            float *dst = static_cast<float *>(P.y) + (size_t)row * P.d_out + c0;
+            if (c0 + 32 <= P.d_out && (P.d_out & 3) == 0) {
+#pragma unroll
+                for (int q = 0; q < 8; ++q)
+                    reinterpret_cast<float4 *>(dst)[q] =
+                        make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            } else {
+#pragma unroll
+                for (int i = 0; i < 32; ++i)
+                    if (c0 + i < P.d_out) dst[i] = v[i];
+            }
+        } else {
+            uint16_t *dst = static_cast<uint16_t *>(P.y) + (size_t)row * P.d_out + c0;
+            if (c0 + 32 <= P.d_out && (P.d_out & 7) == 0) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    uint32_t w[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e)
+                        w[e] = (uint32_t)float_to_bf16_bits(v[8 * q + 2 * e]) |
+                               ((uint32_t)float_to_bf16_bits(v[8 * q + 2 * e + 1]) << 16);
+                    reinterpret_cast<uint4 *>(dst)[q] = make_uint4(w[0], w[1], w[2], w[3]);
+                }
+            } else {
+#pragma unroll
+                for (int i = 0; i < 32; ++i)
+                    if (c0 + i < P.d_out) dst[i] = float_to_bf16_bits(v[i]);
+            }
+        }
     }
 }
 
@@ -400,7 +520,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int i = 0; i < KC; ++i) {
                 const int s = i % STAGES;
                 if (i >= STAGES &&
-                    !mb_wait_role(empty + s, (unsigned)((i / STAGES - 1) & 1), fail)) {
+                    !mb_spin_role(empty + s, (unsigned)((i / STAGES - 1) & 1), fail)) {
                     give_up();
                     break;
                 }
@@ -414,7 +534,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
             for (int i = 0; i < KC; ++i) {
                 const int s = i % STAGES;
-                if (!mb_wait_role(ready + s, (unsigned)((i / STAGES) & 1), fail)) {
+                // with both operands pre-expanded a stage is ready as soon as it lands
+                if (!mb_spin_role(P.expanded ? full + s : ready + s, (unsigned)((i / STAGES) & 1),
+                                  fail)) {
                     give_up();
                     break;
                 }
@@ -435,13 +557,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int tid = threadIdx.x - 64;
         bool ok = STAGE1 || P.expanded || mb_wait_role(&slab_bar, 0, fail);
         if (!ok) give_up();
-        for (int i = 0; i < KC && ok; ++i) {
+        for (int i = 0; i < KC && ok && !P.expanded; ++i) {
             const int s = i % STAGES;
             if (!mb_wait_role(full + s, (unsigned)((i / STAGES) & 1), fail)) {
                 give_up();
                 break;
             }
-            if (!P.expanded) unpack_b<STAGE1>(P, B_of(s), S_of(s), slab, kbeg + i, n0, bn, tid);
+            unpack_b<STAGE1>(P, B_of(s), S_of(s), slab, kbeg + i, n0, bn, tid);
             if (STAGE1) convert_a(A_of(s), tid);
             fence_proxy_async_smem();
             __syncwarp();
@@ -481,72 +603,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             float v[32];
             tmem_ld32(lane_base + cb, v);
             if (row >= P.T) continue;
-            if (STAGE1 && nsplit > 1) {
-                // fp32 partial sums of this K slice; the reduction applies l
-                if (n0 + cb < P.N1) {
-                    float4 *dst = reinterpret_cast<float4 *>(
-                        P.zpart + ((size_t)blockIdx.z * P.T + row) * P.N1 + n0 + cb);
-#pragma unroll
-                    for (int q = 0; q < 8; ++q)
-                        dst[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-                }
-            } else if (STAGE1) {
-                // z = l . t as fp16
-                uint32_t packed[16];
-#pragma unroll
-                for (int i = 0; i < 32; i += 2) {
-                    float a = 0.f, b = 0.f;
-                    const int c0 = n0 + cb + i;
-                    if (c0 < P.N1) {
-                        const int p = c0 >= P.off1 ? 1 : 0;
-                        const int j = c0 - (p ? P.off1 : 0);
-                        const uint16_t *lp = p ? P.L.l[1] : P.L.l[0];
-                        a = v[i] * half_bits_to_float(__ldg(lp + j));
-                        b = v[i + 1] * half_bits_to_float(__ldg(lp + j + 1));
-                    }
-                    const __half2 h = __floats2half2_rn(a, b);
-                    packed[i >> 1] = *reinterpret_cast<const uint32_t *>(&h);
-                }
-                if (n0 + cb < P.N1) {
-                    uint4 *dst = reinterpret_cast<uint4 *>(P.z + (size_t)row * P.N1 + n0 + cb);
-#pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        dst[q] = make_uint4(packed[4 * q], packed[4 * q + 1], packed[4 * q + 2],
-                                            packed[4 * q + 3]);
-                }
-            } else {
-                const int o0 = n0 + cb;
-                if (P.y_fp32) {
-                    float *dst = static_cast<float *>(P.y) + (size_t)row * P.d_out + o0;
-                    if (o0 + 32 <= P.d_out && (P.d_out & 3) == 0) {
-#pragma unroll
-                        for (int q = 0; q < 8; ++q)
-                            reinterpret_cast<float4 *>(dst)[q] =
-                                make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-                    } else {
-#pragma unroll
-                        for (int i = 0; i < 32; ++i)
-                            if (o0 + i < P.d_out) dst[i] = v[i];
-                    }
-                } else {
-                    uint16_t *dst = static_cast<uint16_t *>(P.y) + (size_t)row * P.d_out + o0;
-                    if (o0 + 32 <= P.d_out && (P.d_out & 7) == 0) {
-#pragma unroll
-                        for (int q = 0; q < 4; ++q) {
-                            uint32_t w[4];
-#pragma unroll
-                            for (int e = 0; e < 4; ++e)
-                                w[e] = (uint32_t)float_to_bf16_bits(v[8 * q + 2 * e]) |
-                                       ((uint32_t)float_to_bf16_bits(v[8 * q + 2 * e + 1]) << 16);
-                            reinterpret_cast<uint4 *>(dst)[q] = make_uint4(w[0], w[1], w[2], w[3]);
-                        }
-                    } else {
-#pragma unroll
-                        for (int i = 0; i < 32; ++i)
-                            if (o0 + i < P.d_out) dst[i] = float_to_bf16_bits(v[i]);
-                    }
-                }
-            }
+            store_chunk<STAGE1>(P, v, row, n0 + cb, blockIdx.z, nsplit);
         }
     }
     tc_fence_before();
@@ -557,7 +614,178 @@ __global__ void __launch_bounds__(kThreads, 1)
                      : "memory");
 }
 
-// z = fp16(l . sum over the K slices of the partial t), four columns per thread.
+// Persistent form for pre-expanded operands (both A and B stream by TMA):
+// gridDim.x CTAs walk the tiles t = blockIdx.x, blockIdx.x + gridDim.x, ...
+// (column tile fastest, then K slice, then token tile) and keep two fp32
+// accumulators in TMEM (2 x BN columns), so the epilogue warps read out tile
+// t while the MMA warp already accumulates tile t + gridDim.x and the copy
+// warp keeps streaming K-stages across tile boundaries.  acc_full[b] is
+// committed by the MMA warp when accumulator b holds a finished tile;
+// acc_empty[b] collects one arrival per epilogue warp once it has read b.
+template <bool STAGE1>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_tiles(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
+            const __grid_constant__ PrefillParams P, int tiles_n, int nsplit, int n_tiles) {
+    __shared__ __align__(8) uint64_t full[STAGES], empty[STAGES], acc_full[2], acc_empty[2];
+    __shared__ uint32_t s_tmem;
+    __shared__ int s_fail;
+    unsigned char *smem = reinterpret_cast<unsigned char *>(
+        (reinterpret_cast<uintptr_t>(p_smem) + 1023) & ~(uintptr_t)1023);
+    constexpr int SB = A_BYTES + B_BYTES;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int bn = STAGE1 ? P.bn1 : BN;
+    const int KT = (STAGE1 ? P.L.d_in : P.N1) / BK;
+    volatile int *fail = &s_fail;
+    if (ld_relaxed_gpu(P.ws_words + kErrWord) != 0u) return;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mb_init(full + s, 1);
+            mb_init(empty + s, 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mb_init(acc_full + b, 1);
+            mb_init(acc_empty + b, kWorkWarps);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        s_fail = 0;
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         su32(&s_tmem)),
+                     "r"(2 * BN)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = s_tmem;
+    const uint32_t idesc = instr_desc(BM, bn);
+    auto give_up = [&]() {
+        *fail = 1;
+        atomicCAS(P.ws_words + kErrWord, 0u, static_cast<unsigned>(LB_ERR_TIMEOUT));
+    };
+    // tile t -> token tile origin m0, column origin n0, K chunks [kbeg, kbeg + kc)
+    auto tile = [&](int t, int &m0, int &n0, int &z, int &kbeg, int &kc) {
+        const int nt = t % tiles_n, rest = t / tiles_n;
+        z = rest % nsplit;
+        m0 = (rest / nsplit) * BM;
+        n0 = nt * bn;
+        kbeg = (int)((long long)z * KT / nsplit);
+        kc = (int)((long long)(z + 1) * KT / nsplit) - kbeg;
+    };
+    int loads_issued = 0, mmas_issued = 0;  // K-stages over all of this CTA's tiles
+
+    if (warp == 0) {
+        // ---------------- copy warp
+        if (lane == 0) {
+            bool ok = true;
+            for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+                int m0, n0, z, kbeg, kc;
+                tile(t, m0, n0, z, kbeg, kc);
+                for (int i = 0; i < kc; ++i) {
+                    const int it = loads_issued, s = it % STAGES;
+                    if (it >= STAGES &&
+                        !mb_spin_role(empty + s, (unsigned)((it / STAGES - 1) & 1), fail)) {
+                        give_up();
+                        ok = false;
+                        break;
+                    }
+                    uint64_t *b = full + s;
+                    mb_expect_tx(b, (unsigned)(A_BYTES + bn * BK * 2));
+                    tma_load_2d(smem + s * SB, &amap, (kbeg + i) * BK, m0, b);
+                    tma_load_2d(smem + s * SB + A_BYTES, &bmap, (kbeg + i) * BK, n0, b);
+                    ++loads_issued;
+                }
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        // ---------------- MMA warp
+        if (lane == 0) {
+            bool ok = true;
+            int ti = 0;
+            for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++ti) {
+                int m0, n0, z, kbeg, kc;
+                tile(t, m0, n0, z, kbeg, kc);
+                const int b = ti & 1;
+                if (ti >= 2 &&
+                    !mb_spin_role(acc_empty + b, (unsigned)(((ti >> 1) - 1) & 1), fail)) {
+                    give_up();
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t d = tmem + (uint32_t)(b * BN);
+                for (int i = 0; i < kc; ++i) {
+                    const int it = mmas_issued, s = it % STAGES;
+                    if (!mb_spin_role(full + s, (unsigned)((it / STAGES) & 1), fail)) {
+                        give_up();
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a0 = su32(smem + s * SB), b0 = su32(smem + s * SB + A_BYTES);
+#pragma unroll
+                    for (int k = 0; k < BK / 16; ++k)
+                        mma_f16(d, smem_desc(a0 + 32 * k), smem_desc(b0 + 32 * k), idesc,
+                                (i > 0 || k > 0) ? 1u : 0u);
+                    mma_commit(empty + s);
+                    ++mmas_issued;
+                }
+                if (ok) mma_commit(acc_full + b);
+            }
+        }
+        __syncwarp();
+    } else {
+        // ---------------- epilogue warps: warp w reads TMEM lanes 32(w%4) ..
+        //                  +31 (tile rows) and one half of the tile's columns
+        const int wq = warp & 3, half = (warp - 2) >> 2, nchunk = bn / 32;
+        const uint32_t lane_base = tmem + ((uint32_t)(32 * wq) << 16);
+        const int cb0 = 32 * (half * nchunk / 2), cb1 = 32 * ((half + 1) * nchunk / 2);
+        int ti = 0;
+        for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++ti) {
+            int m0, n0, z, kbeg, kc;
+            tile(t, m0, n0, z, kbeg, kc);
+            const int b = ti & 1;
+            if (!mb_wait_role(acc_full + b, (unsigned)((ti >> 1) & 1), fail)) {
+                if (lane == 0) give_up();
+                break;
+            }
+            tc_fence_after();
+            const int row = m0 + 32 * wq + lane;
+            for (int cb = cb0; cb < cb1; cb += 32) {
+                float v[32];
+                tmem_ld32(lane_base + (uint32_t)(b * BN + cb), v);
+                if (row < P.T) store_chunk<STAGE1>(P, v, row, n0 + cb, z, nsplit);
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0)
+                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(acc_empty + b))
+                             : "memory");
+        }
+    }
+    if (__syncthreads_or(*fail)) {
+        // let every issued copy and MMA land before the CTA goes away
+        if (threadIdx.x == 0)
+            for (int i = loads_issued - STAGES; i < loads_issued; ++i)
+                if (i >= 0) mb_wait(full + i % STAGES, (unsigned)((i / STAGES) & 1));
+        if (threadIdx.x == 32)
+            for (int i = mmas_issued - STAGES; i < mmas_issued; ++i)
+                if (i >= 0) mb_wait(empty + i % STAGES, (unsigned)((i / STAGES) & 1));
+        __syncthreads();
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                     "r"(2 * BN)
+                     : "memory");
+}
+
+// z = l . (sum over the K slices of the partial t), as fp16 (or fp32 into z32),
+// four columns per thread.
 __global__ void k_reduce_z(const __grid_constant__ PrefillParams P) {
     const int groups = P.N1 / 4;
     const long long n = (long long)P.T * groups;
@@ -575,6 +803,14 @@ __global__ void k_reduce_z(const __grid_constant__ PrefillParams P) {
         }
         const int p = c >= P.off1 ? 1 : 0, j = c - (p ? P.off1 : 0);  // 4 | off1
         const uint2 lb = *reinterpret_cast<const uint2 *>((p ? P.L.l[1] : P.L.l[0]) + j);
+        if (P.z32) {
+            *reinterpret_cast<float4 *>(P.z32 + (size_t)row * P.N1 + c) =
+                make_float4(a.x * half_bits_to_float(lb.x & 0xffffu),
+                            a.y * half_bits_to_float(lb.x >> 16),
+                            a.z * half_bits_to_float(lb.y & 0xffffu),
+                            a.w * half_bits_to_float(lb.y >> 16));
+            continue;
+        }
         const __half2 h0 = __floats2half2_rn(a.x * half_bits_to_float(lb.x & 0xffffu),
                                              a.y * half_bits_to_float(lb.x >> 16));
         const __half2 h1 = __floats2half2_rn(a.z * half_bits_to_float(lb.y & 0xffffu),
@@ -586,7 +822,7 @@ __global__ void k_reduce_z(const __grid_constant__ PrefillParams P) {
 }
 
 // bv[n][k] = +-g_p[k]: input k of column n (column j of path p) of V_sign,
-// eight inputs (one 16-byte chunk) per thread.
+// eight inputs (one 16-byte chunk) per thread; then x converted to fp16.
 __global__ void k_expand_v(const __grid_constant__ PrefillParams P) {
     const int kq = P.L.d_in / 8;
     const long long n_items = (long long)P.N1 * kq;
@@ -599,6 +835,21 @@ __global__ void k_expand_v(const __grid_constant__ PrefillParams P) {
         const uint4 mag = *reinterpret_cast<const uint4 *>((p ? P.L.g[1] : P.L.g[0]) + k0);
         *reinterpret_cast<uint4 *>(P.bv + (size_t)n * P.L.d_in + k0) =
             signed8((word >> (k0 & 31)) & 0xffu, mag);
+    }
+    // and x as fp16, eight values per thread (the same rounding as the
+    // in-loop conversion of the unexpanded path)
+    const long long nx = (long long)P.T * kq;
+    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < nx;
+         idx += (long long)gridDim.x * blockDim.x) {
+        const uint4 u = __ldcs(reinterpret_cast<const uint4 *>(P.x) + idx);
+        uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const __half2 h = __floats2half2_rn(__uint_as_float(w[k] << 16),
+                                                __uint_as_float(w[k] & 0xffff0000u));
+            w[k] = *reinterpret_cast<const uint32_t *>(&h);
+        }
+        reinterpret_cast<uint4 *>(P.xh)[idx] = make_uint4(w[0], w[1], w[2], w[3]);
     }
 }
 
@@ -666,10 +917,30 @@ static cudaError_t set_smem_attributes() {
     e = cudaFuncSetAttribute(k_prefill<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              smem_bytes<true>());
     if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_tiles<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 kTilesSmem);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_tiles<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 kTilesSmem);
+    if (e == cudaSuccess)
         e = cudaFuncSetAttribute(k_prefill<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  smem_bytes<false>());
     if (e == cudaSuccess && dev >= 0 && dev < 64) done[dev] = true;
     return e;
+}
+
+// SM count of the current device (cached per device).
+static int device_sms() {
+    static int sms[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+    if (sms[dev] == 0) {
+        int n = 0;
+        if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+            return 148;
+        sms[dev] = n;
+    }
+    return sms[dev];
 }
 
 bool prefill_supported(const lb_linear &L, int64_t T) {
@@ -710,66 +981,114 @@ size_t zpart_bytes(const lb_linear &L, int64_t T) {
 bool expanded_of(const lb_linear &, int64_t T) { return (T + BM - 1) / BM >= 4; }
 size_t bv_bytes(const lb_linear &L) { return ((size_t)n1_of(L) * L.d_in * 2 + 255) & ~(size_t)255; }
 size_t bu_bytes(const lb_linear &L) { return ((size_t)L.d_out * n1_of(L) * 2 + 255) & ~(size_t)255; }
+size_t xh_bytes(const lb_linear &L, int64_t T) { return ((size_t)T * L.d_in * 2 + 255) & ~(size_t)255; }
 }  // namespace
 
 size_t prefill_ws_bytes(const lb_linear &L, int64_t T) {
     return z16_bytes(L, T) + zpart_bytes(L, T) +
-           (expanded_of(L, T) ? bv_bytes(L) + bu_bytes(L) : 0);
+           (expanded_of(L, T) ? bv_bytes(L) + bu_bytes(L) + xh_bytes(L, T) : 0);
 }
 
-cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, void *y, int y_fp32,
-                           unsigned *ws_words, void *z_ws, cudaStream_t s) {
-    if (!encoder()) return cudaErrorNotSupported;
+namespace {
+PrefillParams params_of(const lb_linear &L, int64_t T, unsigned *ws_words, void *ws) {
     PrefillParams P{};
     P.L = make_desc(L);
     P.T = (int)T;
-    P.N1 = 0;
-    for (int p = 0; p < L.n_paths; ++p) P.N1 += L.path[p].r;
+    P.N1 = (int)n1_of(L);
     P.off1 = L.path[0].r;
     P.bn1 = P.N1 <= BN ? P.N1 : BN;
     P.d_out = L.d_out;
-    P.z = static_cast<uint16_t *>(z_ws);
+    char *wsb = static_cast<char *>(ws);
+    P.z = reinterpret_cast<uint16_t *>(wsb);
     P.split = split_of(L, T);
-    char *wsb = static_cast<char *>(z_ws);
     P.zpart = reinterpret_cast<float *>(wsb + z16_bytes(L, T));
     P.expanded = expanded_of(L, T) ? 1 : 0;
     P.bv = reinterpret_cast<uint16_t *>(wsb + z16_bytes(L, T) + zpart_bytes(L, T));
     P.bu = reinterpret_cast<uint16_t *>(wsb + z16_bytes(L, T) + zpart_bytes(L, T) + bv_bytes(L));
-    P.y = y;
-    P.y_fp32 = y_fp32;
+    P.xh = reinterpret_cast<uint16_t *>(wsb + z16_bytes(L, T) + zpart_bytes(L, T) + bv_bytes(L) +
+                                        bu_bytes(L));
     P.ws_words = ws_words;
-    CUtensorMap xmap, zmap, bvmap{}, bumap{};
-    if (!make_map(&xmap, x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, T, L.d_in) ||
-        !make_map(&zmap, z_ws, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, T, P.N1))
+    return P;
+}
+}  // namespace
+
+cudaError_t launch_prefill_latent(const lb_linear &L, const uint16_t *x, int64_t T, uint16_t *z16,
+                                  float *z32, unsigned *ws_words, void *ws, cudaStream_t s) {
+    if (!encoder()) return cudaErrorNotSupported;
+    PrefillParams P = params_of(L, T, ws_words, ws);
+    P.z = z16;
+    P.z32 = z32;
+    P.x = x;
+    CUtensorMap xmap, bvmap{};
+    // the expanded path multiplies the fp16 copy of x, the other one converts in shared memory
+    if (!(P.expanded ? make_map(&xmap, P.xh, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, T, L.d_in)
+                     : make_map(&xmap, x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, T, L.d_in)))
         return cudaErrorInvalidValue;
     if (P.expanded &&
-        (!make_map(&bvmap, P.bv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, P.N1, L.d_in, P.bn1) ||
-         !make_map(&bumap, P.bu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, L.d_out, P.N1, BN)))
+        !make_map(&bvmap, P.bv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, P.N1, L.d_in, P.bn1))
         return cudaErrorInvalidValue;
     cudaError_t e = set_smem_attributes();
     if (e != cudaSuccess) return e;
     if (P.expanded) {
-        const long long nv = (long long)P.N1 * (L.d_in / 8), nu = (long long)L.d_out * (P.N1 / 8);
+        const long long nv = std::max<long long>((long long)P.N1, T) * (L.d_in / 8);
         k_expand_v<<<(int)std::min<long long>((nv + 255) / 256, 148 * 16), 256, 0, s>>>(P);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    const int tm = (int)((T + BM - 1) / BM), tn = (P.N1 + P.bn1 - 1) / P.bn1;
+    if (P.expanded) {
+        const int n_tiles = tm * tn * P.split;
+        k_tiles<true><<<std::min(n_tiles, device_sms()), kThreads, kTilesSmem, s>>>(
+            xmap, bvmap, P, tn, P.split, n_tiles);
+    } else {
+        const dim3 g1((unsigned)tm, (unsigned)tn, (unsigned)P.split);
+        k_prefill<true><<<g1, kThreads, smem_bytes<true>(), s>>>(xmap, bvmap, P);
+    }
+    e = cudaGetLastError();
+    if (e != cudaSuccess || P.split <= 1) return e;
+    const long long groups = (long long)T * (P.N1 / 4);
+    const int blocks = (int)std::min<long long>((groups + 255) / 256, 148 * 8);
+    k_reduce_z<<<blocks, 256, 0, s>>>(P);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_prefill_expand(const lb_linear &L, const uint16_t *z16, int64_t T, void *y,
+                                  int y_fp32, unsigned *ws_words, void *ws, cudaStream_t s) {
+    if (!encoder()) return cudaErrorNotSupported;
+    PrefillParams P = params_of(L, T, ws_words, ws);
+    P.z = const_cast<uint16_t *>(z16);
+    P.y = y;
+    P.y_fp32 = y_fp32;
+    CUtensorMap zmap, bumap{};
+    if (!make_map(&zmap, z16, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, T, P.N1)) return cudaErrorInvalidValue;
+    if (P.expanded && !make_map(&bumap, P.bu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, L.d_out, P.N1, BN))
+        return cudaErrorInvalidValue;
+    cudaError_t e = set_smem_attributes();
+    if (e != cudaSuccess) return e;
+    if (P.expanded) {
+        const long long nu = (long long)L.d_out * (P.N1 / 8);
         k_expand_u<<<(int)std::min<long long>((nu + 255) / 256, 148 * 16), 256, 0, s>>>(P);
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
-    const dim3 g1((unsigned)((T + BM - 1) / BM), (unsigned)((P.N1 + P.bn1 - 1) / P.bn1),
-                  (unsigned)P.split);
-    k_prefill<true><<<g1, kThreads, smem_bytes<true>(), s>>>(xmap, bvmap, P);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    if (P.split > 1) {
-        const long long groups = (long long)T * (P.N1 / 4);
-        const int blocks = (int)std::min<long long>((groups + 255) / 256, 148 * 8);
-        k_reduce_z<<<blocks, 256, 0, s>>>(P);
-        e = cudaGetLastError();
-        if (e != cudaSuccess) return e;
+    const int tm = (int)((T + BM - 1) / BM), tn = (L.d_out + BN - 1) / BN;
+    if (P.expanded) {
+        const int n_tiles = tm * tn;
+        k_tiles<false><<<std::min(n_tiles, device_sms()), kThreads, kTilesSmem, s>>>(
+            zmap, bumap, P, tn, 1, n_tiles);
+    } else {
+        const dim3 g2((unsigned)tm, (unsigned)tn);
+        k_prefill<false><<<g2, kThreads, smem_bytes<false>(), s>>>(zmap, bumap, P);
     }
-    const dim3 g2((unsigned)((T + BM - 1) / BM), (unsigned)((L.d_out + BN - 1) / BN));
-    k_prefill<false><<<g2, kThreads, smem_bytes<false>(), s>>>(zmap, bumap, P);
     return cudaGetLastError();
+}
+
+cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, void *y, int y_fp32,
+                           unsigned *ws_words, void *ws, cudaStream_t s) {
+    uint16_t *z16 = static_cast<uint16_t *>(ws);  // the workspace starts with z
+    cudaError_t e = launch_prefill_latent(L, x, T, z16, nullptr, ws_words, ws, s);
+    if (e != cudaSuccess) return e;
+    return launch_prefill_expand(L, z16, T, y, y_fp32, ws_words, ws, s);
 }
 
 }  // namespace lb

@@ -19,10 +19,12 @@ LIB_PATH = os.path.join(_HERE, "_build", "liblittlebit.so")
 (LB_OK, LB_ERR_INVALID_ARG, LB_ERR_UNSUPPORTED, LB_ERR_CUDA, LB_ERR_TIMEOUT, LB_ERR_WORKSPACE,
  LB_ERR_PLAN, LB_ERR_RANGE) = range(8)
 LB_OUT_BF16, LB_OUT_FP32 = 0, 1
+LB_LATENT_FP32, LB_LATENT_FP16 = 0, 1
 LB_PACK_U, LB_PACK_V = 0, 1
 
 EXPORTED = ["littlebit_status_string", "littlebit_pack", "littlebit_workspace_size",
-            "littlebit_linear_forward", "littlebit_stack_workspace_size",
+            "littlebit_linear_forward", "littlebit_linear_latent", "littlebit_linear_expand",
+            "littlebit_stack_workspace_size",
             "littlebit_stack_prepare", "littlebit_stack_forward", "littlebit_poll_error",
             "littlebit_selftest_wait_timeout", "littlebit_linear_forward_noalloc"]
 
@@ -73,6 +75,12 @@ def lib(path: str | None = None):
         L.littlebit_linear_forward.argtypes = [ctypes.POINTER(lb_linear), vp, i64, vp, i32, vp,
                                                sz, vp]
         L.littlebit_linear_forward.restype = ctypes.c_int
+        L.littlebit_linear_latent.argtypes = [ctypes.POINTER(lb_linear), vp, i64, vp, i32, vp,
+                                              sz, vp]
+        L.littlebit_linear_latent.restype = ctypes.c_int
+        L.littlebit_linear_expand.argtypes = [ctypes.POINTER(lb_linear), vp, i32, i64, vp, i32,
+                                              vp, sz, vp]
+        L.littlebit_linear_expand.restype = ctypes.c_int
         L.littlebit_stack_workspace_size.argtypes = [ctypes.POINTER(lb_linear), i32, i32]
         L.littlebit_stack_workspace_size.restype = sz
         L.littlebit_stack_prepare.argtypes = [ctypes.POINTER(lb_linear), i32, i32, vp, sz, vp]
@@ -136,6 +144,7 @@ class DeviceLinear:
         self.d_in = int(layer["d_in"])
         self.d_out = int(layer["d_out"])
         self.paths = []
+        self.ranks = []
         self.c = lb_linear()
         self.c.d_in = self.d_in
         self.c.d_out = self.d_out
@@ -151,6 +160,7 @@ class DeviceLinear:
             t = {"v_bits": v, "u_bits": u, "g": to_device_bits(P["g"], device),
                  "l": to_device_bits(P["l"], device), "h": to_device_bits(P["h"], device)}
             self.paths.append(t)
+            self.ranks.append(r)
             cp = self.c.path[p]
             cp.r = r
             for k, ten in t.items():
@@ -203,6 +213,47 @@ def linear_forward(L: DeviceLinear, x: torch.Tensor, out_dtype=torch.bfloat16,
     _check(lib().littlebit_linear_forward(ctypes.byref(L.c), x.data_ptr(), T, y.data_ptr(),
                                           y_dtype, ws.data_ptr(), ws.numel(), _stream(stream)),
            "littlebit_linear_forward")
+    return y
+
+
+def linear_latent(L: DeviceLinear, x: torch.Tensor, z_dtype=torch.float32,
+                  z: torch.Tensor | None = None, ws: torch.Tensor | None = None,
+                  stream=None) -> torch.Tensor:
+    """Latent states z [T][r_0 + r_1] = l_p . ((X . g_p) V_p,sign) per path
+    (Sec. 5, KV cache compression) for x bf16 [T][d_in] on device."""
+    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.shape[1] == L.d_in
+    x = x.contiguous()
+    T = x.shape[0]
+    if z is None:
+        z = torch.empty((T, sum(L.ranks)), dtype=z_dtype, device=x.device)
+    assert z.dtype in (torch.float32, torch.float16) and z.is_contiguous()
+    code = LB_LATENT_FP16 if z.dtype == torch.float16 else LB_LATENT_FP32
+    if ws is None:
+        ws = new_workspace(workspace_size(L, T), x.device)
+    _check(lib().littlebit_linear_latent(ctypes.byref(L.c), x.data_ptr(), T, z.data_ptr(), code,
+                                         ws.data_ptr(), ws.numel(), _stream(stream)),
+           "littlebit_linear_latent")
+    return z
+
+
+def linear_expand(L: DeviceLinear, z: torch.Tensor, out_dtype=torch.bfloat16,
+                  y: torch.Tensor | None = None, ws: torch.Tensor | None = None,
+                  stream=None) -> torch.Tensor:
+    """Y [T][d_out] = sum_p h_p . (U_p,sign z_p) from latents z [T][r_0 + r_1]
+    (fp32 or fp16) on device."""
+    assert z.dtype in (torch.float32, torch.float16) and z.dim() == 2
+    assert z.shape[1] == sum(L.ranks)
+    z = z.contiguous()
+    T = z.shape[0]
+    code = LB_LATENT_FP16 if z.dtype == torch.float16 else LB_LATENT_FP32
+    if y is None:
+        y = torch.empty((T, L.d_out), dtype=out_dtype, device=z.device)
+    y_dtype = LB_OUT_FP32 if y.dtype == torch.float32 else LB_OUT_BF16
+    if ws is None:
+        ws = new_workspace(workspace_size(L, T), z.device)
+    _check(lib().littlebit_linear_expand(ctypes.byref(L.c), z.data_ptr(), code, T, y.data_ptr(),
+                                         y_dtype, ws.data_ptr(), ws.numel(), _stream(stream)),
+           "littlebit_linear_expand")
     return y
 
 

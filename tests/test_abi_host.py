@@ -98,6 +98,27 @@ def test_forward_argument_validation(L):
     assert fwd(L, fake_linear(rs=(2000, 64))) == lb.LB_ERR_UNSUPPORTED
 
 
+def test_latent_and_expand_argument_validation(L):
+    c = fake_linear()
+    lat, exp = L.littlebit_linear_latent, L.littlebit_linear_expand
+    ref = ctypes.byref(c)
+    assert lat(None, FAKE, 1, FAKE, 0, FAKE, 1 << 30, None) == lb.LB_ERR_INVALID_ARG
+    assert lat(ref, FAKE, -1, FAKE, 0, FAKE, 1 << 30, None) == lb.LB_ERR_INVALID_ARG
+    assert lat(ref, FAKE, 1, FAKE, 2, FAKE, 1 << 30, None) == lb.LB_ERR_INVALID_ARG  # z dtype
+    assert lat(ref, FAKE, 0, FAKE, 0, FAKE, 1 << 30, None) == lb.LB_OK              # T = 0
+    assert lat(ref, FAKE, 1, 0, 0, FAKE, 1 << 30, None) == lb.LB_ERR_INVALID_ARG
+    assert lat(ref, FAKE, 1, FAKE + 8, 1, FAKE, 1 << 30, None) == lb.LB_ERR_INVALID_ARG
+    assert lat(ref, FAKE, 1, FAKE, 0, FAKE, 64, None) == lb.LB_ERR_WORKSPACE
+    assert lat(ctypes.byref(fake_linear(d_in=40)), FAKE, 1, FAKE, 0, FAKE, 1 << 30,
+               None) == lb.LB_ERR_UNSUPPORTED
+    assert exp(None, FAKE, 0, 1, FAKE, 0, FAKE, 1 << 30, None) == lb.LB_ERR_INVALID_ARG
+    assert exp(ref, FAKE, 2, 1, FAKE, 0, FAKE, 1 << 30, None) == lb.LB_ERR_INVALID_ARG  # z dtype
+    assert exp(ref, FAKE, 0, 1, FAKE, 5, FAKE, 1 << 30, None) == lb.LB_ERR_INVALID_ARG  # y dtype
+    assert exp(ref, FAKE, 0, 0, FAKE, 0, FAKE, 1 << 30, None) == lb.LB_OK              # T = 0
+    assert exp(ref, FAKE + 4, 0, 1, FAKE, 0, FAKE, 1 << 30, None) == lb.LB_ERR_INVALID_ARG
+    assert exp(ref, FAKE, 0, 1, FAKE, 0, FAKE + 16, 1 << 30, None) == lb.LB_ERR_WORKSPACE
+
+
 def fake_stack(n_layers=2, d=256, dkv=64, dff=512, rq=16, rk=8, rm=24):
     shapes = [(d, d, rq), (d, dkv, rk), (d, dkv, rk), (d, d, rq), (d, dff, rm), (d, dff, rm),
               (dff, d, rm)]

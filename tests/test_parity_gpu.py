@@ -201,6 +201,101 @@ def test_padding_bits_are_ignored(T):
     check(gpu_forward(D, x, torch.float32), y_ref, torch.float32)
 
 
+# ------------------------------------------------------------------ latent states (Sec. 5)
+
+LATENT = [
+    # d_in, d_out, ranks, T   (CUDA-core stages unless T >= 16 and the ranks and
+    # d_in are multiples of 64)
+    (256, 96, (33, 16), 1), (512, 40, (7,), 3), (4128, 1000, (96, 1), 9), (1024, 300, (33, 16), 65),
+    (8192, 1024, (32, 32), 1), (8192, 1024, (32, 32), 64),
+    (128, 512, (64, 64), 256), (256, 1000, (128, 64), 77), (4096, 2048, (512, 512), 300),
+    (11008, 4096, (128, 128), 16), (4096, 4096, (64, 64), 600),
+]
+
+
+def _tensor_path(d_in, rs, T):
+    return T >= 16 and d_in % 64 == 0 and all(r % 64 == 0 and r <= 512 for r in rs)
+
+
+@pytest.mark.parametrize("d_in,d_out,rs,T", LATENT)
+@pytest.mark.parametrize("z_dtype", [torch.float32, torch.float16])
+def test_latent_and_expand(d_in, d_out, rs, T, z_dtype):
+    """z = l . ((X . g) V_sign) per path as [T][r_0 + r_1], and its expansion,
+    each against the oracle; expanding the GPU latent gives the forward."""
+    rng = inputs.rng_for(106, salt=d_in + d_out + T)
+    L = inputs.make_linear(rng, d_in, d_out, list(rs), len(rs), 0.05)
+    x = inputs.bf16_normal(rng, (T, d_in))
+    D = lb.DeviceLinear(L, DEV)
+    ws = lb.new_workspace(lb.workspace_size(D, T), DEV)
+    xin = lb.bf16_tensor(x, DEV)
+    z = torch.full((T, sum(rs)), float("nan"), dtype=z_dtype, device=DEV)
+    lb.linear_latent(D, xin, z=z, ws=ws)
+    torch.cuda.synchronize()
+    zg = z.float().cpu().numpy().astype(np.float64)
+    z_ref = oracle.latent(L, x)
+    assert np.all(np.isfinite(zg))
+    # fp32: fp32 sums (1e-4 as for the forward); fp16: the fp16 rounding of z
+    # itself, relative RMS 2^-11 / sqrt(3) ~ 2.8e-4
+    e = rel(zg, z_ref)
+    assert e <= (1e-4 if z_dtype == torch.float32 else 1e-3), e
+    # the expansion alone, on the oracle's latent in the same element type
+    z_in = torch.from_numpy(z_ref.astype(np.float32)).to(z_dtype)
+    z_exp = z_in.double().numpy()
+    y = torch.full((T, d_out), float("nan"), dtype=torch.float32, device=DEV)
+    lb.linear_expand(D, z_in.to(DEV), y=y, ws=ws)
+    torch.cuda.synchronize()
+    yg = y.cpu().numpy().astype(np.float64)
+    assert np.all(np.isfinite(yg))
+    # the tensor-core stage rounds an fp32 z to fp16 operands
+    tol = 1e-3 if (_tensor_path(d_in, rs, T) and z_dtype == torch.float32) else 1e-4
+    e = rel(yg, oracle.expand(L, z_exp))
+    assert e <= tol, e
+    # expand(latent(X)) against the oracle's forward (fp32 output: with a few
+    # hundred outputs the bf16 rounding alone can exceed 2e-3 by chance)
+    yc = torch.full((T, d_out), float("nan"), dtype=torch.float32, device=DEV)
+    lb.linear_expand(D, z, y=yc, ws=ws)
+    torch.cuda.synchronize()
+    tol = 1e-3 if (_tensor_path(d_in, rs, T) or z_dtype == torch.float16) else 1e-4
+    check(yc.cpu().numpy().astype(np.float64), oracle.forward_factored(L, x), torch.float32, tol)
+
+
+def test_latent_kv_cache_70b_kv_projection():
+    """The 70B key projection (8192 -> 1024, two paths of rank 32): a 512-token
+    fp16 latent cache is 16x smaller than the bf16 keys, and its expansion
+    matches the forward of each cached token."""
+    rng = inputs.rng_for(107)
+    T, d, dkv, r = 512, 8192, 1024, 32
+    L = inputs.make_linear(rng, d, dkv, [r, r], 2, 0.02)
+    x = inputs.bf16_normal(rng, (T, d))
+    D = lb.DeviceLinear(L, DEV)
+    xin = lb.bf16_tensor(x, DEV)
+    z = lb.linear_latent(D, xin, z_dtype=torch.float16)
+    keys = lb.linear_forward(D, xin, out_dtype=torch.bfloat16)
+    assert z.numel() * z.element_size() * 16 == keys.numel() * keys.element_size()
+    y = lb.linear_expand(D, z, out_dtype=torch.float32)
+    torch.cuda.synchronize()
+    rows = np.array([0, 1, 77, 300, T - 1])
+    zg = z.float().cpu().numpy().astype(np.float64)
+    assert rel(zg[rows], oracle.latent(L, x[rows])) <= 1e-3
+    ref = oracle.forward_factored(L, x[rows])
+    assert rel(y.cpu().numpy().astype(np.float64)[rows], ref) <= TOL
+    assert rel(keys.float().cpu().numpy().astype(np.float64)[rows], ref) <= TOL
+
+
+def test_latent_full_size_prefill_sampled_tokens():
+    """4096 x 4096, two paths of rank 512, 2048 tokens: the tensor-core
+    latent (split along d_in or not, as the forward) on sampled tokens."""
+    L, x = inputs.config4("4096x4096_r512", 2048)
+    D = lb.DeviceLinear(L, DEV)
+    xin = lb.bf16_tensor(x, DEV)
+    for z_dtype, tol in ((torch.float32, 1e-4), (torch.float16, 1e-3)):
+        z = lb.linear_latent(D, xin, z_dtype=z_dtype)
+        torch.cuda.synchronize()
+        rows = np.array([0, 5, 127, 128, 1000, 2047])
+        zg = z.float().cpu().numpy().astype(np.float64)[rows]
+        assert rel(zg, oracle.latent(L, x[rows])) <= tol
+
+
 # ------------------------------------------------------------------ stack
 
 
