@@ -13,9 +13,11 @@
 // stage's mbarrier beside the TMA of X; stage 2 bulk-copies the tile's U rows
 // and h once per CTA.  X arrives by TMA (bf16) and is converted to fp16 in
 // shared memory (exact for |x| < 65504).  From four token tiles on, every
-// tile would repeat that work, so one pre-pass writes the +-g / +-h operands
-// and an fp16 copy of X to the workspace and both GEMMs stream plain fp16
-// tiles by TMA.  z goes to the workspace as fp16 and comes back by TMA.
+// tile would repeat the unpacking, so one pre-pass writes the +-g / +-h
+// operands to the workspace, both GEMMs stream them by TMA, and a persistent
+// kernel (k_tiles) walks the tiles with two TMEM accumulators so the
+// epilogue of one tile overlaps the K loop of the next.  z goes to the
+// workspace as fp16 and comes back by TMA.
 //
 // One CTA computes a 128 x BN tile (BN <= 256 fp32 TMEM columns) with
 // specialised warps: warp 0 issues the TMA / bulk copies of each 64-element
@@ -68,7 +70,14 @@ __host__ __device__ constexpr int smem_bytes() {
     return RING_BYTES + (STAGE1 ? STAGES * SRC_BYTES : SLAB_BYTES) + 1024;
 }
 static_assert(smem_bytes<true>() <= 232448 && smem_bytes<false>() <= 232448, "shared memory");
-constexpr int kTilesSmem = RING_BYTES + 1024;  // the persistent form: the A|B ring only
+// The persistent form: the A|B ring, then (stage 2) one 32 x 16 fp32 staging
+// tile per epilogue warp, rows padded to 20 floats so that each quarter-warp
+// float4 access hits distinct banks.
+constexpr int kStagePitch = 20;
+constexpr int kMaxStages = 8;
+constexpr int kStageBytes = 32 * kStagePitch * 4;
+constexpr int kTilesSmem = RING_BYTES + kWorkWarps * kStageBytes + 1024;
+static_assert(kTilesSmem <= 232448, "shared memory");
 
 extern __shared__ __align__(1024) unsigned char p_smem[];
 
@@ -194,20 +203,23 @@ __device__ __forceinline__ void tc_fence_after() {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 
-// 32 consecutive fp32 columns of this thread's TMEM lane.
+// 32 consecutive fp32 columns of this thread's TMEM lane.  The load and its
+// wait are one asm statement: tcgen05.ld fills the registers asynchronously,
+// so no instruction may read (or copy) them before tcgen05.wait::ld.
 __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
     uint32_t r[32];
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
-        "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        "%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n\t"
+        "tcgen05.wait::ld.sync.aligned;"
         : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
           "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
           "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]),
           "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
           "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]),
           "=r"(r[31])
-        : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+        : "r"(taddr)
+        : "memory");
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
 }
@@ -241,8 +253,6 @@ struct PrefillParams {
     int expanded;      // B operands pre-expanded to fp16 (bv, bu) and loaded by TMA
     uint16_t *bv;      // [N1][d_in]: +-g_p[k] at (column n of path p, input k)
     uint16_t *bu;      // [d_out][N1]: +-h_p[o] at (output o, column n of path p)
-    const uint16_t *x; // stage 1 input, bf16 [T][d_in]
-    uint16_t *xh;      // expanded stage 1: x converted to fp16 once per call [T][d_in]
     void *y;           // stage 2 output [T][d_out]
     int y_fp32;
     unsigned *ws_words;
@@ -306,9 +316,11 @@ __device__ __forceinline__ void mb_expect_only(uint64_t *b, unsigned bytes) {
                  : "memory");
 }
 
-// In-place bf16 -> fp16 of the A stage (layout-preserving, elementwise).
+// In-place bf16 -> fp16 of the A stage (layout-preserving, elementwise),
+// NT threads.
+template <int NT = kWork>
 __device__ __forceinline__ void convert_a(unsigned char *As, int tid) {
-    for (int i = tid; i < A_BYTES / 16; i += kWork) {
+    for (int i = tid; i < A_BYTES / 16; i += NT) {
         uint4 *p = reinterpret_cast<uint4 *>(As) + i;
         uint4 u = *p;
         uint32_t w[4] = {u.x, u.y, u.z, u.w};
@@ -614,7 +626,48 @@ __global__ void __launch_bounds__(kThreads, 1)
                      : "memory");
 }
 
-// Persistent form for pre-expanded operands (both A and B stream by TMA):
+// Stage 2 output of one warp's 32 x 32 accumulator chunk (thread = row, v =
+// its 32 columns starting at c0) written through shared memory so that each
+// store instruction covers whole row segments: per 16-column half, every
+// thread parks its row in stg (32 rows x kStagePitch floats), then in four
+// passes reads back four columns of row 8i + lane/4 and writes them (8 bytes
+// bf16 / 16 bytes fp32), four lanes per row, eight rows per pass.
+__device__ __forceinline__ void store_y_coalesced(const PrefillParams &P, const float (&v)[32],
+                                                  float *stg, int row0, int c0, int lane) {
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        float4 *mine = reinterpret_cast<float4 *>(stg + lane * kStagePitch);
+#pragma unroll
+        for (int q = 0; q < 4; ++q)
+            mine[q] = make_float4(v[16 * h + 4 * q], v[16 * h + 4 * q + 1], v[16 * h + 4 * q + 2],
+                                  v[16 * h + 4 * q + 3]);
+        __syncwarp();
+        const int j = lane & 3;
+        const int col = c0 + 16 * h + 4 * j;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int r = 8 * i + (lane >> 2);
+            const float4 f = *reinterpret_cast<const float4 *>(stg + r * kStagePitch + 4 * j);
+            const int row = row0 + r;
+            if (row >= P.T || col >= P.d_out) continue;  // d_out % 8 == 0: whole groups of 4
+            if (P.y_fp32) {
+                *reinterpret_cast<float4 *>(static_cast<float *>(P.y) + (size_t)row * P.d_out +
+                                            col) = f;
+            } else {
+                const uint32_t w0 = (uint32_t)float_to_bf16_bits(f.x) |
+                                    ((uint32_t)float_to_bf16_bits(f.y) << 16);
+                const uint32_t w1 = (uint32_t)float_to_bf16_bits(f.z) |
+                                    ((uint32_t)float_to_bf16_bits(f.w) << 16);
+                *reinterpret_cast<uint2 *>(static_cast<uint16_t *>(P.y) + (size_t)row * P.d_out +
+                                           col) = make_uint2(w0, w1);
+            }
+        }
+        __syncwarp();
+    }
+}
+
+// Persistent form for pre-expanded B operands (A and B both stream by TMA;
+// in stage 1 four warps convert each bf16 x stage to fp16 in place):
 // gridDim.x CTAs walk the tiles t = blockIdx.x, blockIdx.x + gridDim.x, ...
 // (column tile fastest, then K slice, then token tile) and keep two fp32
 // accumulators in TMEM (2 x BN columns), so the epilogue warps read out tile
@@ -626,26 +679,34 @@ template <bool STAGE1>
 __global__ void __launch_bounds__(kThreads, 1)
     k_tiles(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
             const __grid_constant__ PrefillParams P, int tiles_n, int nsplit, int n_tiles) {
-    __shared__ __align__(8) uint64_t full[STAGES], empty[STAGES], acc_full[2], acc_empty[2];
+    __shared__ __align__(8) uint64_t full[kMaxStages], ready[kMaxStages], empty[kMaxStages],
+        acc_full[2], acc_empty[2];
     __shared__ uint32_t s_tmem;
     __shared__ int s_fail;
     unsigned char *smem = reinterpret_cast<unsigned char *>(
         (reinterpret_cast<uintptr_t>(p_smem) + 1023) & ~(uintptr_t)1023);
-    constexpr int SB = A_BYTES + B_BYTES;
+    // stage 1 streams x as bf16: warps 2..5 convert each A stage to fp16 in
+    // place and warps 6..9 run the epilogue; stage 2 uses all eight for it
+    constexpr int kEpiWarps = STAGE1 ? 4 : kWorkWarps;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int bn = STAGE1 ? P.bn1 : BN;
     const int KT = (STAGE1 ? P.L.d_in : P.N1) / BK;
+    // the ring holds as many stages as fit: narrower B tiles, deeper ring
+    // (bn 64 / 128 / 192 / 256 -> 8 / 6 / 4 / 4 stages of 24 / 32 / 40 / 48 KB)
+    const int SB = A_BYTES + bn * BK * 2;
+    const int nst = min(kMaxStages, RING_BYTES / SB);
     volatile int *fail = &s_fail;
     if (ld_relaxed_gpu(P.ws_words + kErrWord) != 0u) return;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < STAGES; ++s) {
+        for (int s = 0; s < nst; ++s) {
             mb_init(full + s, 1);
+            mb_init(ready + s, 4);
             mb_init(empty + s, 1);
         }
         for (int b = 0; b < 2; ++b) {
             mb_init(acc_full + b, 1);
-            mb_init(acc_empty + b, kWorkWarps);
+            mb_init(acc_empty + b, kEpiWarps);
         }
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         s_fail = 0;
@@ -676,27 +737,36 @@ __global__ void __launch_bounds__(kThreads, 1)
         kc = (int)((long long)(z + 1) * KT / nsplit) - kbeg;
     };
     int loads_issued = 0, mmas_issued = 0;  // K-stages over all of this CTA's tiles
+    // ring cursor: stage s and the parity ph of its current use
+    auto advance = [&](int &s, unsigned &ph) {
+        if (++s == nst) {
+            s = 0;
+            ph ^= 1u;
+        }
+    };
 
     if (warp == 0) {
         // ---------------- copy warp
         if (lane == 0) {
             bool ok = true;
+            int s = 0;
+            unsigned ph = 0;
             for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
                 int m0, n0, z, kbeg, kc;
                 tile(t, m0, n0, z, kbeg, kc);
                 for (int i = 0; i < kc; ++i) {
-                    const int it = loads_issued, s = it % STAGES;
-                    if (it >= STAGES &&
-                        !mb_spin_role(empty + s, (unsigned)((it / STAGES - 1) & 1), fail)) {
+                    // a stage's previous use must have been multiplied
+                    if (loads_issued >= nst && !mb_spin_role(empty + s, ph ^ 1u, fail)) {
                         give_up();
                         ok = false;
                         break;
                     }
                     uint64_t *b = full + s;
-                    mb_expect_tx(b, (unsigned)(A_BYTES + bn * BK * 2));
+                    mb_expect_tx(b, (unsigned)SB);
                     tma_load_2d(smem + s * SB, &amap, (kbeg + i) * BK, m0, b);
                     tma_load_2d(smem + s * SB + A_BYTES, &bmap, (kbeg + i) * BK, n0, b);
                     ++loads_issued;
+                    advance(s, ph);
                 }
             }
         }
@@ -705,7 +775,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---------------- MMA warp
         if (lane == 0) {
             bool ok = true;
-            int ti = 0;
+            int ti = 0, s = 0;
+            unsigned ph = 0;
             for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++ti) {
                 int m0, n0, z, kbeg, kc;
                 tile(t, m0, n0, z, kbeg, kc);
@@ -718,8 +789,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_fence_after();
                 const uint32_t d = tmem + (uint32_t)(b * BN);
                 for (int i = 0; i < kc; ++i) {
-                    const int it = mmas_issued, s = it % STAGES;
-                    if (!mb_spin_role(full + s, (unsigned)((it / STAGES) & 1), fail)) {
+                    // stage 1: the stage is ready once its A half is fp16
+                    if (!mb_spin_role(STAGE1 ? ready + s : full + s, ph, fail)) {
                         give_up();
                         ok = false;
                         break;
@@ -732,23 +803,54 @@ __global__ void __launch_bounds__(kThreads, 1)
                                 (i > 0 || k > 0) ? 1u : 0u);
                     mma_commit(empty + s);
                     ++mmas_issued;
+                    advance(s, ph);
                 }
                 if (ok) mma_commit(acc_full + b);
             }
         }
         __syncwarp();
+    } else if (STAGE1 && warp < 6) {
+        // ---------------- conversion warps: bf16 -> fp16 of each A stage
+        const int tid = threadIdx.x - 64;
+        int s = 0;
+        unsigned ph = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+            int m0, n0, z, kbeg, kc;
+            tile(t, m0, n0, z, kbeg, kc);
+            for (int i = 0; i < kc; ++i, advance(s, ph)) {
+                const bool got = mb_wait_role(full + s, ph, fail);
+                if (!__all_sync(0xffffffffu, got)) {
+                    if (lane == 0) give_up();
+                    ok = false;
+                    break;
+                }
+                convert_a<128>(smem + s * SB, tid);
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0)
+                    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(ready + s))
+                                 : "memory");
+            }
+        }
     } else {
         // ---------------- epilogue warps: warp w reads TMEM lanes 32(w%4) ..
-        //                  +31 (tile rows) and one half of the tile's columns
-        const int wq = warp & 3, half = (warp - 2) >> 2, nchunk = bn / 32;
+        //                  +31 (tile rows) and its share of the tile's columns
+        //                  (all of them in stage 1, one half in stage 2)
+        const int wq = warp & 3, nchunk = bn / 32;
+        const int half = STAGE1 ? 0 : (warp - 2) >> 2, halves = STAGE1 ? 1 : 2;
         const uint32_t lane_base = tmem + ((uint32_t)(32 * wq) << 16);
-        const int cb0 = 32 * (half * nchunk / 2), cb1 = 32 * ((half + 1) * nchunk / 2);
+        const int cb0 = 32 * (half * nchunk / halves), cb1 = 32 * ((half + 1) * nchunk / halves);
         int ti = 0;
         for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++ti) {
             int m0, n0, z, kbeg, kc;
             tile(t, m0, n0, z, kbeg, kc);
             const int b = ti & 1;
-            if (!mb_wait_role(acc_full + b, (unsigned)((ti >> 1) & 1), fail)) {
+            // the vote reconverges the warp (each lane leaves the wait on its
+            // own) before the warp-collective tcgen05.ld, and makes the
+            // outcome uniform
+            const bool got = mb_wait_role(acc_full + b, (unsigned)((ti >> 1) & 1), fail);
+            if (!__all_sync(0xffffffffu, got)) {
                 if (lane == 0) give_up();
                 break;
             }
@@ -757,7 +859,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int cb = cb0; cb < cb1; cb += 32) {
                 float v[32];
                 tmem_ld32(lane_base + (uint32_t)(b * BN + cb), v);
-                if (row < P.T) store_chunk<STAGE1>(P, v, row, n0 + cb, z, nsplit);
+                if (STAGE1) {
+                    if (row < P.T) store_chunk<STAGE1>(P, v, row, n0 + cb, z, nsplit);
+                } else {
+                    float *stg = reinterpret_cast<float *>(smem + RING_BYTES +
+                                                           (warp - 2) * kStageBytes);
+                    store_y_coalesced(P, v, stg, m0 + 32 * wq, n0 + cb, lane);
+                }
             }
             tc_fence_before();
             __syncwarp();
@@ -769,11 +877,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (__syncthreads_or(*fail)) {
         // let every issued copy and MMA land before the CTA goes away
         if (threadIdx.x == 0)
-            for (int i = loads_issued - STAGES; i < loads_issued; ++i)
-                if (i >= 0) mb_wait(full + i % STAGES, (unsigned)((i / STAGES) & 1));
+            for (int i = loads_issued - nst; i < loads_issued; ++i)
+                if (i >= 0) mb_wait(full + i % nst, (unsigned)((i / nst) & 1));
         if (threadIdx.x == 32)
-            for (int i = mmas_issued - STAGES; i < mmas_issued; ++i)
-                if (i >= 0) mb_wait(empty + i % STAGES, (unsigned)((i / STAGES) & 1));
+            for (int i = mmas_issued - nst; i < mmas_issued; ++i)
+                if (i >= 0) mb_wait(empty + i % nst, (unsigned)((i / nst) & 1));
         __syncthreads();
     }
     tc_fence_before();
@@ -822,7 +930,7 @@ __global__ void k_reduce_z(const __grid_constant__ PrefillParams P) {
 }
 
 // bv[n][k] = +-g_p[k]: input k of column n (column j of path p) of V_sign,
-// eight inputs (one 16-byte chunk) per thread; then x converted to fp16.
+// eight inputs (one 16-byte chunk) per thread.
 __global__ void k_expand_v(const __grid_constant__ PrefillParams P) {
     const int kq = P.L.d_in / 8;
     const long long n_items = (long long)P.N1 * kq;
@@ -835,21 +943,6 @@ __global__ void k_expand_v(const __grid_constant__ PrefillParams P) {
         const uint4 mag = *reinterpret_cast<const uint4 *>((p ? P.L.g[1] : P.L.g[0]) + k0);
         *reinterpret_cast<uint4 *>(P.bv + (size_t)n * P.L.d_in + k0) =
             signed8((word >> (k0 & 31)) & 0xffu, mag);
-    }
-    // and x as fp16, eight values per thread (the same rounding as the
-    // in-loop conversion of the unexpanded path)
-    const long long nx = (long long)P.T * kq;
-    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < nx;
-         idx += (long long)gridDim.x * blockDim.x) {
-        const uint4 u = __ldcs(reinterpret_cast<const uint4 *>(P.x) + idx);
-        uint32_t w[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const __half2 h = __floats2half2_rn(__uint_as_float(w[k] << 16),
-                                                __uint_as_float(w[k] & 0xffff0000u));
-            w[k] = *reinterpret_cast<const uint32_t *>(&h);
-        }
-        reinterpret_cast<uint4 *>(P.xh)[idx] = make_uint4(w[0], w[1], w[2], w[3]);
     }
 }
 
@@ -981,12 +1074,11 @@ size_t zpart_bytes(const lb_linear &L, int64_t T) {
 bool expanded_of(const lb_linear &, int64_t T) { return (T + BM - 1) / BM >= 4; }
 size_t bv_bytes(const lb_linear &L) { return ((size_t)n1_of(L) * L.d_in * 2 + 255) & ~(size_t)255; }
 size_t bu_bytes(const lb_linear &L) { return ((size_t)L.d_out * n1_of(L) * 2 + 255) & ~(size_t)255; }
-size_t xh_bytes(const lb_linear &L, int64_t T) { return ((size_t)T * L.d_in * 2 + 255) & ~(size_t)255; }
 }  // namespace
 
 size_t prefill_ws_bytes(const lb_linear &L, int64_t T) {
     return z16_bytes(L, T) + zpart_bytes(L, T) +
-           (expanded_of(L, T) ? bv_bytes(L) + bu_bytes(L) + xh_bytes(L, T) : 0);
+           (expanded_of(L, T) ? bv_bytes(L) + bu_bytes(L) : 0);
 }
 
 namespace {
@@ -1005,8 +1097,6 @@ PrefillParams params_of(const lb_linear &L, int64_t T, unsigned *ws_words, void 
     P.expanded = expanded_of(L, T) ? 1 : 0;
     P.bv = reinterpret_cast<uint16_t *>(wsb + z16_bytes(L, T) + zpart_bytes(L, T));
     P.bu = reinterpret_cast<uint16_t *>(wsb + z16_bytes(L, T) + zpart_bytes(L, T) + bv_bytes(L));
-    P.xh = reinterpret_cast<uint16_t *>(wsb + z16_bytes(L, T) + zpart_bytes(L, T) + bv_bytes(L) +
-                                        bu_bytes(L));
     P.ws_words = ws_words;
     return P;
 }
@@ -1018,19 +1108,15 @@ cudaError_t launch_prefill_latent(const lb_linear &L, const uint16_t *x, int64_t
     PrefillParams P = params_of(L, T, ws_words, ws);
     P.z = z16;
     P.z32 = z32;
-    P.x = x;
     CUtensorMap xmap, bvmap{};
-    // the expanded path multiplies the fp16 copy of x, the other one converts in shared memory
-    if (!(P.expanded ? make_map(&xmap, P.xh, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, T, L.d_in)
-                     : make_map(&xmap, x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, T, L.d_in)))
-        return cudaErrorInvalidValue;
+    if (!make_map(&xmap, x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, T, L.d_in)) return cudaErrorInvalidValue;
     if (P.expanded &&
         !make_map(&bvmap, P.bv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, P.N1, L.d_in, P.bn1))
         return cudaErrorInvalidValue;
     cudaError_t e = set_smem_attributes();
     if (e != cudaSuccess) return e;
     if (P.expanded) {
-        const long long nv = std::max<long long>((long long)P.N1, T) * (L.d_in / 8);
+        const long long nv = (long long)P.N1 * (L.d_in / 8);
         k_expand_v<<<(int)std::min<long long>((nv + 255) / 256, 148 * 16), 256, 0, s>>>(P);
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
