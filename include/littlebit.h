@@ -119,9 +119,10 @@ size_t littlebit_workspace_size(const lb_linear *L, int64_t T);
  * Paths taken: T = 1 with every r % 8 == 0 and d_out % 8 == 0 -> one launch
  * of the single-token kernel (it keeps its exchange words in ws between
  * calls, so a workspace must not be shared by concurrent calls); T >= 16
- * with d_in and every r multiples of 64, r <= 512 and d_out % 8 == 0 -> the
- * tensor-core path (fp16 operands, see its tolerance in the design notes);
- * otherwise the two-launch CUDA-core path. */
+ * and T * (r_0 + r_1) > 8192, with d_in and every r multiples of 64,
+ * r <= 512 and d_out % 8 == 0 -> the tensor-core path (fp16 operands, see
+ * its tolerance in the design notes); otherwise the two-launch CUDA-core
+ * path. */
 lb_status littlebit_linear_forward(const lb_linear *L, const uint16_t *x, int64_t T, void *y,
                                    int32_t y_dtype, void *ws, size_t ws_bytes,
                                    lb_stream_t stream);

@@ -130,11 +130,18 @@ unsigned long long stack_fingerprint(const lb_linear *lin, int32_t n_layers, int
 // One token goes through the single-launch persistent kernel.
 bool use_decode(const lb_linear &, int64_t T) { return T == 1; }
 
-// From this many tokens on, the layer is a dense contraction worth the
-// tensor cores (tcgen05, 128-token tiles).
+// From this many tokens on, and once the stage-1 output (T x sum of ranks)
+// fills a few tensor-core tiles, the layer is a dense contraction worth the
+// tensor cores (tcgen05, 128-token tiles).  Below that the two-launch
+// CUDA-core path finishes first (measured on GB300 for the 4096 <-> 11008
+// shapes: at rank sums 256 and T = 16 it takes 25 us against 30-37 us, at
+// T = 32 they tie, from T = 64 or rank sum 1024 on the tensor cores win).
 constexpr int64_t kPrefillMinTokens = 16;
+constexpr int64_t kPrefillMinLatent = 8192;
 bool use_prefill(const lb_linear &L, int64_t T) {
-    return T >= kPrefillMinTokens && lb::prefill_supported(L, T);
+    int64_t n1 = 0;
+    for (int p = 0; p < L.n_paths; ++p) n1 += L.path[p].r;
+    return T >= kPrefillMinTokens && T * n1 > kPrefillMinLatent && lb::prefill_supported(L, T);
 }
 
 // Workspace of a linear: header | the single-token kernel's exchange words

@@ -158,18 +158,18 @@ def test_stress_shapes(d_in, d_out, rs, T):
     L = inputs.make_linear(rng, d_in, d_out, list(rs), len(rs), 0.1)
     x = inputs.bf16_normal(rng, (T, d_in))
     D = lb.DeviceLinear(L, DEV)
-    tol = 1e-3 if T >= 16 and all(r % 64 == 0 for r in rs) and d_in % 64 == 0 else TOL_FP32
+    tol = 1e-3 if _tensor_path(d_in, rs, T) else TOL_FP32
     check(gpu_forward(D, x, torch.float32), oracle.forward_factored(L, x), torch.float32, tol)
 
 
 PREFILL = [
-    # d_in, d_out, ranks, T   (the tensor-core path: T >= 16, ranks multiples of 64
-    # up to 512, d_out a multiple of 8)
-    (64, 256, (64,), 128), (128, 512, (64, 64), 256), (4096, 4096, (64, 64), 200),
+    # d_in, d_out, ranks, T   (the tensor-core path: T >= 16 and T x sum of ranks
+    # above 8192, ranks multiples of 64 up to 512, d_out a multiple of 8)
+    (64, 256, (64,), 160), (128, 512, (64, 64), 256), (4096, 4096, (64, 64), 200),
     (256, 1000, (128, 64), 77), (512, 2104, (192,), 300), (1024, 768, (512, 512), 130),
-    (4096, 11008, (128, 128), 64), (64, 8, (64, 64), 33),
+    (4096, 11008, (128, 128), 64), (64, 8, (64, 64), 65), (512, 1000, (512,), 17),
     # stage 1 split along d_in into K slices (long d_in, few token tiles)
-    (11008, 4096, (128, 128), 16), (4096, 2048, (512, 512), 300), (2048, 64, (64,), 20),
+    (11008, 4096, (128, 128), 48), (4096, 2048, (512, 512), 300), (2048, 64, (64, 64), 72),
 ]
 
 
@@ -209,12 +209,13 @@ LATENT = [
     (256, 96, (33, 16), 1), (512, 40, (7,), 3), (4128, 1000, (96, 1), 9), (1024, 300, (33, 16), 65),
     (8192, 1024, (32, 32), 1), (8192, 1024, (32, 32), 64),
     (128, 512, (64, 64), 256), (256, 1000, (128, 64), 77), (4096, 2048, (512, 512), 300),
-    (11008, 4096, (128, 128), 16), (4096, 4096, (64, 64), 600),
+    (11008, 4096, (128, 128), 48), (4096, 4096, (64, 64), 600), (4096, 1000, (128,), 16),
 ]
 
 
 def _tensor_path(d_in, rs, T):
-    return T >= 16 and d_in % 64 == 0 and all(r % 64 == 0 and r <= 512 for r in rs)
+    return (T >= 16 and T * sum(rs) > 8192 and d_in % 64 == 0
+            and all(r % 64 == 0 and r <= 512 for r in rs))
 
 
 @pytest.mark.parametrize("d_in,d_out,rs,T", LATENT)
