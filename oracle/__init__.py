@@ -7,7 +7,7 @@ the product package never does, and this package never imports the product.
 
 The arithmetic lives in ``lb_oracle.c`` (plain C, fp64, one function per
 definition of the paper: Eq. 2 packing, Eq. 4-6 dense weight, Prop. 1 factored
-forward, App. E bit accounting).  This module only builds it with gcc and
+forward, latent states, Dual-SVID initialisation, App. E bit accounting).  This module only builds it with gcc and
 marshals numpy arrays through ctypes.
 """
 from __future__ import annotations
@@ -82,6 +82,12 @@ def _bind(lib):
     lib.lbo_latent.restype = ctypes.c_int
     lib.lbo_expand.argtypes = [ctypes.POINTER(Linear), vp, i64, vp]
     lib.lbo_expand.restype = None
+    lib.lbo_svd_top.argtypes = [vp, i64, i64, i64, vp, vp, vp]
+    lib.lbo_svd_top.restype = ctypes.c_int
+    lib.lbo_dual_svid_path.argtypes = [vp, i64, i64, i64, vp, vp, vp, vp, vp]
+    lib.lbo_dual_svid_path.restype = ctypes.c_int
+    lib.lbo_path_weight.argtypes = [vp, vp, vp, vp, vp, i64, i64, i64, vp]
+    lib.lbo_path_weight.restype = None
     lib.lbo_stack_forward.argtypes = [ctypes.POINTER(Linear), ctypes.c_int32, ctypes.c_int32,
                                       vp, vp, vp, vp]
     lib.lbo_stack_forward.restype = ctypes.c_int
@@ -254,6 +260,60 @@ class Oracle:
             raise MemoryError("oracle stack forward failed")
         return out, q, kv
 
+    # ------------------------------------------------------------ Dual-SVID (Sec. 3.2, 3.3)
+    def svd_top(self, A: np.ndarray, r: int):
+        """The r largest singular triples of A by one-sided Jacobi: (s[r], U[m][r], V[n][r])."""
+        A = _c(A, np.float64)
+        m, n = A.shape
+        s = np.zeros(r)
+        U = np.zeros((m, r))
+        V = np.zeros((n, r))
+        if self.lib.lbo_svd_top(_ptr(A), m, n, r, _ptr(s), _ptr(U), _ptr(V)):
+            raise ValueError("svd_top: rank out of range or no memory")
+        return s, U, V
+
+    def dual_svid_path(self, R: np.ndarray, r: int):
+        """Dual-SVID of one path (Sec. 3.2): (usign [d_out][r], vsign [d_in][r], h, g, l) in fp64."""
+        R = _c(R, np.float64)
+        d_out, d_in = R.shape
+        us = np.zeros((d_out, r), np.int8)
+        vs = np.zeros((d_in, r), np.int8)
+        h, g, l = np.zeros(d_out), np.zeros(d_in), np.zeros(r)
+        if self.lib.lbo_dual_svid_path(_ptr(R), d_out, d_in, r, _ptr(us), _ptr(vs), _ptr(h),
+                                       _ptr(g), _ptr(l)):
+            raise ValueError("dual_svid_path: rank out of range or no memory")
+        return us, vs, h, g, l
+
+    def path_weight(self, us, vs, h, g, l) -> np.ndarray:
+        """W_hat = diag(h) U_sign diag(l) V_sign^T diag(g) (Eq. 4), fp64."""
+        us, vs = _c(us, np.int8), _c(vs, np.int8)
+        h, g, l = _c(h, np.float64), _c(g, np.float64), _c(l, np.float64)
+        d_out, r = us.shape
+        d_in = vs.shape[0]
+        W = np.zeros((d_out, d_in))
+        self.lib.lbo_path_weight(_ptr(us), _ptr(vs), _ptr(h), _ptr(g), _ptr(l), d_out, d_in, r,
+                                 _ptr(W))
+        return W
+
+    def dual_svid(self, W: np.ndarray, ranks) -> dict:
+        """Dual-SVID initialisation with Residual Compensation (Sec. 3.2, 3.3): path 0 from
+        W, each further path from the residual W - sum of the previous paths' W_hat, where a
+        path's W_hat uses its scales as stored (rounded to fp16, nearest even).  Returns a
+        layer dict (packed words, fp16 scale bits) plus 'signs' (usign, vsign per path)."""
+        W = _c(W, np.float64)
+        R = W.copy()
+        paths, signs = [], []
+        for r in ranks:
+            us, vs, h, g, l = self.dual_svid_path(R, int(r))
+            h16, g16, l16 = (np.asarray(a, np.float64).astype(np.float16) for a in (h, g, l))
+            paths.append({"r": int(r), "u_words": self.pack_u(us), "v_words": self.pack_v(vs),
+                          "h": h16.view(np.uint16), "g": g16.view(np.uint16),
+                          "l": l16.view(np.uint16)})
+            signs.append((us, vs))
+            R = R - self.path_weight(us, vs, h16.astype(np.float64), g16.astype(np.float64),
+                                     l16.astype(np.float64))
+        return {"d_in": W.shape[1], "d_out": W.shape[0], "paths": paths, "signs": signs}
+
     # ------------------------------------------------------------ accounting (App. E, I.1)
     def bpw(self, d_out: int, d_in: int, r: int, n_paths: int = 2) -> float:
         return self.lib.lbo_bpw(d_out, d_in, r, n_paths)
@@ -290,7 +350,7 @@ def _forward(name):
 
 for _name in ("half_to_double", "bf16_to_double", "pack_u", "pack_v", "unpack_u", "unpack_v",
               "forward_dense", "forward_factored", "apply_factored", "latent", "expand",
-              "stack_forward",
+              "svd_top", "dual_svid_path", "path_weight", "dual_svid", "stack_forward",
               "bpw", "rank_for_bpw", "flops", "set_threads", "get_threads"):
     globals()[_name] = _forward(_name)
 del _name

@@ -412,6 +412,230 @@ done:
 }
 
 /* ------------------------------------------------------------------------ */
+/* Dual-SVID initialisation (Sec. 3.2) and Residual Compensation (Sec. 3.3)  */
+/* ------------------------------------------------------------------------ */
+
+/* Truncated SVD by one-sided Jacobi (Hestenes).  Plane rotations G act on
+ * pairs of columns of A until all columns are mutually orthogonal:
+ * A G_1 G_2 ... = B with B's columns b_j = sigma_j u_j, and V = G_1 G_2 ...,
+ * so A = sum_j sigma_j u_j v_j^T.  Kept transposed: row j of Bt is column j
+ * of A G..., row j of J is column j of V (J starts as I).  For columns x, y
+ * with alpha = x.x, beta = y.y, gamma = x.y the rotation x' = c x - s y,
+ * y' = s x + c y makes x'.y' = 0 for t = s/c, the smaller root of
+ * t^2 + 2 zeta t - 1 = 0, zeta = (beta - alpha) / (2 gamma).
+ * Returns the r largest singular values in decreasing order (s[r]) with
+ * U[m][r], V[n][r].  Sign convention (u_j, v_j are defined up to a joint
+ * sign): the entry of largest magnitude of each v_j, the first one on a tie,
+ * is positive.  0, or -1 (r out of range or no memory). */
+int lbo_svd_top(const double *A, int64_t m, int64_t n, int64_t r, double *s, double *U, double *V)
+{
+    if (r < 1 || r > m || r > n)
+        return -1;
+    double *Bt = (double *)malloc((size_t)(n * m) * sizeof(double));
+    double *J = (double *)calloc((size_t)(n * n), sizeof(double));
+    double *nrm = (double *)malloc((size_t)n * sizeof(double));
+    char *used = (char *)calloc((size_t)n, 1);
+    if (!Bt || !J || !nrm || !used) {
+        free(Bt);
+        free(J);
+        free(nrm);
+        free(used);
+        return -1;
+    }
+    for (int64_t i = 0; i < m; i++)
+        for (int64_t j = 0; j < n; j++)
+            Bt[j * m + i] = A[i * n + j];
+    for (int64_t j = 0; j < n; j++)
+        J[j * n + j] = 1.0;
+    for (int sweep = 0; sweep < 60; sweep++) {
+        double off = 0.0;
+        for (int64_t p = 0; p < n - 1; p++)
+            for (int64_t q = p + 1; q < n; q++) {
+                double *x = Bt + p * m, *y = Bt + q * m;
+                double alpha = 0.0, beta = 0.0, gamma = 0.0;
+                for (int64_t i = 0; i < m; i++) {
+                    alpha += x[i] * x[i];
+                    beta += y[i] * y[i];
+                    gamma += x[i] * y[i];
+                }
+                if (gamma == 0.0)
+                    continue;
+                double rel = fabs(gamma) / sqrt(alpha * beta);
+                if (rel > off)
+                    off = rel;
+                if (rel < 1e-15)
+                    continue;
+                double zeta = (beta - alpha) / (2.0 * gamma);
+                double t = (zeta >= 0 ? 1.0 : -1.0) / (fabs(zeta) + sqrt(1.0 + zeta * zeta));
+                double c = 1.0 / sqrt(1.0 + t * t), sn = c * t;
+                for (int64_t i = 0; i < m; i++) {
+                    double a = x[i], b = y[i];
+                    x[i] = c * a - sn * b;
+                    y[i] = sn * a + c * b;
+                }
+                double *jp = J + p * n, *jq = J + q * n;
+                for (int64_t i = 0; i < n; i++) {
+                    double a = jp[i], b = jq[i];
+                    jp[i] = c * a - sn * b;
+                    jq[i] = sn * a + c * b;
+                }
+            }
+        if (off < 1e-14)
+            break;
+    }
+    for (int64_t j = 0; j < n; j++) {
+        double ss = 0.0;
+        for (int64_t i = 0; i < m; i++)
+            ss += Bt[j * m + i] * Bt[j * m + i];
+        nrm[j] = sqrt(ss);
+    }
+    for (int64_t a = 0; a < r; a++) {
+        /* the largest remaining column norm (lowest index on a tie) */
+        int64_t best = -1;
+        for (int64_t b = 0; b < n; b++)
+            if (!used[b] && (best < 0 || nrm[b] > nrm[best]))
+                best = b;
+        used[best] = 1;
+        s[a] = nrm[best];
+        int64_t imax = 0;
+        for (int64_t i = 1; i < n; i++)
+            if (fabs(J[best * n + i]) > fabs(J[best * n + imax]))
+                imax = i;
+        double sg = J[best * n + imax] < 0 ? -1.0 : 1.0;
+        for (int64_t i = 0; i < n; i++)
+            V[i * r + a] = sg * J[best * n + i];
+        for (int64_t i = 0; i < m; i++)
+            U[i * r + a] = nrm[best] > 0 ? sg * Bt[best * m + i] / nrm[best] : 0.0;
+    }
+    free(used);
+    free(Bt);
+    free(J);
+    free(nrm);
+    return 0;
+}
+
+/* Best rank-1 approximation of a nonnegative matrix M (rows x cols, all
+ * entries >= 0) as a b^T with a, b >= 0: its leading singular pair, found
+ * by power iteration from b = 1 (for a nonnegative matrix the leading
+ * singular vectors can be taken nonnegative, Perron-Frobenius).  The
+ * singular value sigma is split evenly: a = sqrt(sigma) u, b = sqrt(sigma) v.
+ * A zero matrix gives a = b = 0. */
+static void rank1_nonneg(const double *M, int64_t rows, int64_t cols, double *a, double *b)
+{
+    double *u = (double *)malloc((size_t)rows * sizeof(double));
+    double *v = (double *)malloc((size_t)cols * sizeof(double));
+    if (!u || !v) {
+        free(u);
+        free(v);
+        return;
+    }
+    for (int64_t j = 0; j < cols; j++)
+        v[j] = 1.0 / sqrt((double)cols);
+    double sigma = 0.0;
+    for (int it = 0; it < 500; it++) {
+        double nu = 0.0, nv = 0.0;
+        for (int64_t i = 0; i < rows; i++) {
+            double acc = 0.0;
+            for (int64_t j = 0; j < cols; j++)
+                acc += M[i * cols + j] * v[j];
+            u[i] = acc;
+            nu += acc * acc;
+        }
+        nu = sqrt(nu);
+        if (nu == 0.0) {
+            sigma = 0.0;
+            break;
+        }
+        for (int64_t i = 0; i < rows; i++)
+            u[i] /= nu;
+        double change = 0.0;
+        for (int64_t j = 0; j < cols; j++) {
+            double acc = 0.0;
+            for (int64_t i = 0; i < rows; i++)
+                acc += M[i * cols + j] * u[i];
+            change += (acc - nu * v[j]) * (acc - nu * v[j]);
+            v[j] = acc;
+            nv += acc * acc;
+        }
+        nv = sqrt(nv);
+        for (int64_t j = 0; j < cols; j++)
+            v[j] /= nv;
+        sigma = nv;
+        if (sqrt(change) <= 1e-15 * nv)
+            break;
+    }
+    double sq = sqrt(sigma);
+    for (int64_t i = 0; i < rows; i++)
+        a[i] = sigma > 0 ? sq * u[i] : 0.0;
+    for (int64_t j = 0; j < cols; j++)
+        b[j] = sigma > 0 ? sq * v[j] : 0.0;
+    free(u);
+    free(v);
+}
+
+/* Dual-SVID of one path (Sec. 3.2): from R (d_out x d_in, row-major) and
+ * rank r,
+ *   (1) truncated SVD R ~ U' V'^T with U' = U_r diag(sqrt s), V' = V_r diag(sqrt s)
+ *       (the singular values split evenly between the two factors);
+ *   (2) U_sign = sign(U'), V_sign = sign(V') (sign(0) = +1);
+ *   (3) |U'| ~ h0 l_u^T, |V'| ~ g0 l_v^T (best rank-1, rank1_nonneg), l0 = l_u . l_v.
+ * Outputs usign[d_out][r], vsign[d_in][r] (+-1), h[d_out], g[d_in], l[r].
+ * 0, or -1. */
+int lbo_dual_svid_path(const double *R, int64_t d_out, int64_t d_in, int64_t r, int8_t *usign,
+                       int8_t *vsign, double *h, double *g, double *l)
+{
+    double *s = (double *)malloc((size_t)r * sizeof(double));
+    double *U = (double *)malloc((size_t)(d_out * r) * sizeof(double));
+    double *V = (double *)malloc((size_t)(d_in * r) * sizeof(double));
+    double *lu = (double *)malloc((size_t)r * sizeof(double));
+    double *lv = (double *)malloc((size_t)r * sizeof(double));
+    int rc = -1;
+    if (!s || !U || !V || !lu || !lv || lbo_svd_top(R, d_out, d_in, r, s, U, V) != 0)
+        goto out;
+    for (int64_t j = 0; j < r; j++) {
+        double q = sqrt(s[j]);
+        for (int64_t i = 0; i < d_out; i++)
+            U[i * r + j] *= q;
+        for (int64_t i = 0; i < d_in; i++)
+            V[i * r + j] *= q;
+    }
+    for (int64_t k = 0; k < d_out * r; k++) {
+        usign[k] = U[k] < 0 ? -1 : 1;
+        U[k] = fabs(U[k]);
+    }
+    for (int64_t k = 0; k < d_in * r; k++) {
+        vsign[k] = V[k] < 0 ? -1 : 1;
+        V[k] = fabs(V[k]);
+    }
+    rank1_nonneg(U, d_out, r, h, lu);
+    rank1_nonneg(V, d_in, r, g, lv);
+    for (int64_t j = 0; j < r; j++)
+        l[j] = lu[j] * lv[j];
+    rc = 0;
+out:
+    free(s);
+    free(U);
+    free(V);
+    free(lu);
+    free(lv);
+    return rc;
+}
+
+/* W_hat of one path from signs and scales, Eq. 4: h_o u_oj l_j v_ij g_i. */
+void lbo_path_weight(const int8_t *usign, const int8_t *vsign, const double *h, const double *g,
+                     const double *l, int64_t d_out, int64_t d_in, int64_t r, double *What)
+{
+#pragma omp parallel for schedule(static)
+    for (int64_t o = 0; o < d_out; o++)
+        for (int64_t i = 0; i < d_in; i++) {
+            double acc = 0.0;
+            for (int64_t j = 0; j < r; j++)
+                acc += usign[o * r + j] * l[j] * vsign[i * r + j];
+            What[o * d_in + i] = h[o] * acc * g[i];
+        }
+}
+
+/* ------------------------------------------------------------------------ */
 /* Accounting (App. E, App. I.1)                                            */
 /* ------------------------------------------------------------------------ */
 

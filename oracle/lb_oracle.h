@@ -100,6 +100,21 @@ void lbo_expand(const lbo_linear *L, const double *z, int64_t T, double *y);
 int lbo_stack_forward(const lbo_linear *lin, int32_t n_layers, int32_t head_dim,
                       const uint16_t *x0, double *out, double *q_out, double *kv_out);
 
+/* Dual-SVID initialisation (Sec. 3.2).
+ * lbo_svd_top: the r largest singular triples of A (m x n, row-major) by
+ * one-sided Jacobi; s[r] decreasing, U[m][r], V[n][r]; each v_j has its
+ * largest-magnitude entry (first on a tie) positive.  0 / -1.
+ * lbo_dual_svid_path: truncated SVD R ~ U' V'^T (U' = U diag(sqrt s), V' =
+ * V diag(sqrt s)), U_sign = sign(U'), V_sign = sign(V') (sign(0) = +1), best
+ * rank-1 |U'| ~ h l_u^T and |V'| ~ g l_v^T (singular value split evenly),
+ * l = l_u . l_v.  usign[d_out][r], vsign[d_in][r] (+-1).  0 / -1.
+ * lbo_path_weight: W_hat = diag(h) U_sign diag(l) V_sign^T diag(g) (Eq. 4). */
+int lbo_svd_top(const double *A, int64_t m, int64_t n, int64_t r, double *s, double *U, double *V);
+int lbo_dual_svid_path(const double *R, int64_t d_out, int64_t d_in, int64_t r, int8_t *usign,
+                       int8_t *vsign, double *h, double *g, double *l);
+void lbo_path_weight(const int8_t *usign, const int8_t *vsign, const double *h, const double *g,
+                     const double *l, int64_t d_out, int64_t d_in, int64_t r, double *What);
+
 /* App. E bits per weight: total parameter bits / (d_out * d_in), where each
  * path stores r*(d_out+d_in) sign bits and 16*(d_out+d_in+r) scale bits. */
 double lbo_bpw(int64_t d_out, int64_t d_in, int64_t r, int32_t n_paths);

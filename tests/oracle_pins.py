@@ -16,6 +16,8 @@ Sources of truth used here, none of which is the oracle:
     (tests/golden/)
   * algebraic invariants: path-swap symmetry of Eq. 6, h_res = 0 reducing to
     one path
+  * numpy's LAPACK SVD for the Dual-SVID steps; exact recovery of a rank-1
+    matrix and of a Sylvester-Hadamard LittleBit weight
   * for the decoder chain: textbook softmax attention over the one cached
     position, and closed forms with branches switched off or made the identity
 """
@@ -465,6 +467,107 @@ def pin_theoretical_cost(orc):
         assert abs(f / 1e6 - float(mflops)) < 0.05, f
 
 
+# ------------------------------------------------------------------ pins: Dual-SVID (Sec. 3.2, 3.3)
+
+
+def pin_svd_top_vs_numpy(orc):
+    """The Jacobi SVD's r largest singular triples against numpy's LAPACK SVD
+    (values, vectors up to the joint sign), orthonormality, the sign
+    convention, and Eckart-Young: the rank-r error is the tail of the spectrum."""
+    rng = np.random.default_rng(25)
+    for m, n, r in [(40, 30, 5), (30, 40, 7), (24, 24, 24), (50, 17, 1)]:
+        A = rng.standard_normal((m, n))
+        s, U, V = orc.svd_top(A, r)
+        Un, sn, Vtn = np.linalg.svd(A)
+        assert np.allclose(s, sn[:r], rtol=1e-12, atol=0), (m, n, r)
+        assert np.allclose(np.abs(np.sum(U * Un[:, :r], axis=0)), 1.0, atol=1e-10)
+        assert np.allclose(np.abs(np.sum(V * Vtn[:r].T, axis=0)), 1.0, atol=1e-10)
+        assert np.allclose(U.T @ U, np.eye(r), atol=1e-12)
+        assert np.allclose(V.T @ V, np.eye(r), atol=1e-12)
+        for j in range(r):
+            k = int(np.argmax(np.abs(V[:, j])))
+            assert V[k, j] > 0
+        err = np.linalg.norm(A - (U * s) @ V.T) ** 2
+        tail = float(np.sum(sn[r:] ** 2))
+        assert abs(err - tail) <= 1e-10 * max(1.0, tail), (err, tail)
+
+
+def pin_dual_svid_rank1(orc):
+    """A rank-1 W = a b^T: the signs are those of a and b (jointly flipped so
+    that the largest |b_i| is positive), |U'| and |V'| are rank-1 already, and
+    the primary path reproduces W; the residual path then has nothing left."""
+    rng = np.random.default_rng(26)
+    a = rng.standard_normal(23)
+    a[5] = 0.0  # a zero row of W: U' is 0 there, sign(0) = +1 and h = 0
+    b = rng.standard_normal(19)
+    W = np.outer(a, b)
+    us, vs, h, g, l = orc.dual_svid_path(W, 1)
+    flip = 1 if b[np.argmax(np.abs(b))] > 0 else -1
+    assert us[5, 0] == 1 and h[5] == 0.0
+    assert np.array_equal(us[:, 0], np.where(flip * a < 0, -1, 1).astype(np.int8))
+    assert np.array_equal(vs[:, 0], np.where(flip * b < 0, -1, 1).astype(np.int8))
+    assert rel(orc.path_weight(us, vs, h, g, l), W) <= 1e-13
+    L = orc.dual_svid(W, [1, 1])
+    h1 = np_half(L["paths"][1]["h"])
+    g1 = np_half(L["paths"][1]["g"])
+    # the residual is W minus the fp16-rounded primary path: small, and the
+    # second path's W_hat is of its size, not of W's
+    us1, vs1 = L["signs"][1]
+    W1 = orc.path_weight(us1, vs1, h1, g1, np_half(L["paths"][1]["l"]))
+    assert np.linalg.norm(W1) <= 5e-3 * np.linalg.norm(W)
+
+
+def pin_dual_svid_hadamard(orc):
+    """W = H_r diag(lam) H_r^T (Sylvester columns, distinct lam > 0) is a
+    LittleBit weight with h = g = 1: Dual-SVID finds U_sign = V_sign = H_r up
+    to one joint sign per column (all entries of a column tie in magnitude,
+    so the sign convention falls to rounding there) and W_hat = W."""
+    d, r = 64, 8
+    H = sylvester(d)[:, :r].astype(np.float64)
+    lam = np.array([9.0, 7.5, 6.0, 5.0, 4.0, 3.0, 2.0, 1.5])
+    W = (H * lam) @ H.T
+    us, vs, h, g, l = orc.dual_svid_path(W, r)
+    flip = (us[0] * H[0]).astype(np.int8)
+    assert np.array_equal(us, (H * flip).astype(np.int8))
+    assert np.array_equal(vs, (H * flip).astype(np.int8))
+    assert rel(orc.path_weight(us, vs, h, g, l), W) <= 1e-12
+    # the scales factor the magnitudes: h and g constant, l proportional to lam
+    assert np.ptp(h) <= 1e-12 * h.mean() and np.ptp(g) <= 1e-12 * g.mean()
+    assert np.allclose(l / l[0], lam / lam[0], rtol=1e-12)
+
+
+def pin_dual_svid_vs_lapack(orc):
+    """Dual-SVID assembled from numpy's SVD (truncated SVD, then the leading
+    singular pair of |U'| and |V'|) gives the same signs and W_hat as the
+    oracle's Jacobi / power-iteration steps; and scaling W by c scales W_hat by
+    c with the same signs."""
+    rng = np.random.default_rng(27)
+    m, n, r = 36, 28, 6
+    A = rng.standard_normal((m, n)) * np.linspace(2.0, 0.5, n)
+    us, vs, h, g, l = orc.dual_svid_path(A, r)
+    Un, sn, Vtn = np.linalg.svd(A)
+    Ur, Vr = Un[:, :r] * np.sqrt(sn[:r]), Vtn[:r].T * np.sqrt(sn[:r])
+    for j in range(r):  # the oracle's joint sign convention
+        if Vr[np.argmax(np.abs(Vr[:, j])), j] < 0:
+            Ur[:, j], Vr[:, j] = -Ur[:, j], -Vr[:, j]
+    assert np.array_equal(us, np.where(Ur < 0, -1, 1).astype(np.int8))
+    assert np.array_equal(vs, np.where(Vr < 0, -1, 1).astype(np.int8))
+
+    def rank1(M):
+        u, s1, vt = np.linalg.svd(M)
+        a, b = np.abs(u[:, 0]) * np.sqrt(s1[0]), np.abs(vt[0]) * np.sqrt(s1[0])
+        return a, b
+    hu, lu = rank1(np.abs(Ur))
+    gv, lv = rank1(np.abs(Vr))
+    W_ref = (hu[:, None] * np.where(Ur < 0, -1.0, 1.0) * (lu * lv)) @ \
+        (gv[:, None] * np.where(Vr < 0, -1.0, 1.0)).T
+    assert rel(orc.path_weight(us, vs, h, g, l), W_ref) <= 1e-9
+    assert rel(h * g.mean() * l.mean(), hu * gv.mean() * (lu * lv).mean()) <= 1e-9
+    us2, vs2, h2, g2, l2 = orc.dual_svid_path(3.0 * A, r)
+    assert np.array_equal(us2, us) and np.array_equal(vs2, vs)
+    assert rel(orc.path_weight(us2, vs2, h2, g2, l2), 3.0 * orc.path_weight(us, vs, h, g, l)) <= 1e-12
+
+
 def pin_kv_cache_table4(orc):
     """Table 4: the single-path rank for each target bits per weight of a
     d_model x d_model key/value projection (rounded up to a multiple of 8)
@@ -585,5 +688,6 @@ ALL_PINS = [pin_fp16_exhaustive, pin_bf16_exhaustive, pin_pack_structured, pin_p
             pin_hadamard_identity, pin_brute_force, pin_residual_paths, pin_padding_ignored,
             pin_latent_hadamard, pin_latent_closed_forms, pin_latent_brute_force,
             pin_latent_expand_composition, pin_bpw_worked_examples, pin_theoretical_cost,
-            pin_kv_cache_table4, pin_stack_chain,
+            pin_kv_cache_table4, pin_svd_top_vs_numpy, pin_dual_svid_rank1,
+            pin_dual_svid_hadamard, pin_dual_svid_vs_lapack, pin_stack_chain,
             pin_stack_zero_branches, pin_stack_attention_closed_form]

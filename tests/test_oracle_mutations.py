@@ -52,6 +52,14 @@ MUTATIONS = [
     ("expand_path_offset", "            off += P->r;", "            off += 0;"),
     ("expand_u_transposed", "s += z[tt * n1 + off + j] * sign_u(P->u_words, P->r, o, j);",
      "s += z[tt * n1 + off + j] * sign_u(P->u_words, P->r, j % L->d_out, o % P->r);"),
+    ("dsvid_no_sqrt_split", "double q = sqrt(s[j]);", "double q = s[j];"),
+    ("dsvid_latent_lu_only", "l[j] = lu[j] * lv[j];", "l[j] = lu[j];"),
+    ("dsvid_sign_of_zero", "usign[k] = U[k] < 0 ? -1 : 1;", "usign[k] = U[k] <= 0 ? -1 : 1;"),
+    ("dsvid_no_abs", "        U[k] = fabs(U[k]);", "        U[k] = U[k];"),
+    ("jacobi_rotation_sign", "y[i] = sn * a + c * b;", "y[i] = -sn * a + c * b;"),
+    ("svd_sign_convention", "double sg = J[best * n + imax] < 0 ? -1.0 : 1.0;",
+     "double sg = J[best * n + imax] > 0 ? -1.0 : 1.0;"),
+    ("path_weight_drops_g", "What[o * d_in + i] = h[o] * acc * g[i];", "What[o * d_in + i] = h[o] * acc;"),
     ("flops_factor", "return (double)n_paths * 2.0 * (double)T", "return (double)n_paths * 1.0 * (double)T"),
 ]
 
