@@ -13,13 +13,14 @@ on a bounded sample (cpu_baseline), and the SM clocks seen while timing.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                   [--layers L]
-  python bench.py --config 2|3|4|6 [--steps K] [--warmup W]
+  python bench.py --config 2|3|4|6|7 [--steps K] [--warmup W]
 
 --config times the single-linear workloads instead (one JSON line per case,
 not the bench line): 2 = 4096x4096 r64 at T = 1, 8; 3 = the FFN triple at
 r = 128, 512 and T = 1, 16, 64; 4 = prefill at T = 2048, 8192; 6 = the
 latent-state halves (littlebit_linear_latent / _expand: the 70B key
-projection at T = 1 and a 4096-token cache, 4096x4096 r512 at T = 2048).
+projection at T = 1 and a 4096-token cache, 4096x4096 r512 at T = 2048);
+7 = Dual-SVID initialisation of a dense weight into two paths (ms per layer).
 Cases 2, 3 and the CUDA-core cases of 6 report algorithmic GB/s with L2
 flushed before every call; 4 and the tensor-core cases of 6 report TFLOP/s
 (2 flops per +-1 MAC, both paths) against the dense bf16 peak.
@@ -56,7 +57,7 @@ def parse_args():
     ap.add_argument("--layers", type=int, default=80,
                     help="stack depth (80 = the Llama2-70B workload; smaller only for profiling)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--config", type=int, choices=[2, 3, 4, 6], default=None,
+    ap.add_argument("--config", type=int, choices=[2, 3, 4, 6, 7], default=None,
                     help="time a single-linear workload instead of the stack")
     ap.add_argument("--only", default=None,
                     help="with --config: only the cases whose 'name:T' contains this text")
@@ -500,6 +501,46 @@ def run_config(args):
                         continue
                     xin = xd if nm == "down" else x
                     emit(f"{nm} r{r}", 3, T, lins[nm], time_case(lins[nm], xin, T, True), False)
+    elif args.config == 7:
+        # Dual-SVID initialisation (one dense weight -> two LittleBit paths):
+        # the 4096 x 4096 r64 layer and the 70B gate shape (8192 -> 28672, r320),
+        # synthetic weights with a power-law singular spectrum built on the device
+        g = torch.Generator(device=dev)
+        g.manual_seed(20250607)
+        fp32_peak = 152 * 128 * 2 * 1.92e9 / 1e12  # FP32 FMA lanes x 2 flops x SM clock
+        for name, m, n, r in (("4096x4096 r64x2", 4096, 4096, 64),
+                              ("gate 8192->28672 r320x2", 28672, 8192, 320)):
+            if not wanted(name, 0):
+                continue
+            k0 = 1024
+            A = torch.randn((m, k0), generator=g, device=dev) / m ** 0.5
+            B = torch.randn((n, k0), generator=g, device=dev) / n ** 0.5
+            sig = (1.0 + torch.arange(k0, device=dev, dtype=torch.float32)) ** -0.6
+            W = (A * sig) @ B.t() + 1e-3 * torch.randn((m, n), generator=g, device=dev) / n ** 0.5
+            del A, B
+            lb.dual_svid(W, [r, r], iters=8)  # warm-up (cuBLAS handle, workspace)
+            torch.cuda.synchronize(dev)
+            ts = []
+            for _ in range(max(1, min(steps, 3))):
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record()
+                lb.dual_svid(W, [r, r], iters=8)
+                e1.record()
+                torch.cuda.synchronize(dev)
+                ts.append(e0.elapsed_time(e1))
+            ms = statistics.median(ts)
+            k = min(r + 8, m, n)
+            # GEMM flops of two paths: per path 8 iterations of R Q and R^T Y
+            # (2 m n k each), the Rayleigh-Ritz R Q, the Ritz vectors, the residual
+            flops = 2 * (8 * 2 * 2 * m * n * k + 2 * m * n * k + 2 * (m + n) * k * r) + 2 * m * n * r
+            line = {"config": 7, "case": name, "op": "dual_svid", "ms": ms,
+                    "gemm_tflops": flops / ms / 1e9,
+                    "roofline": {"bound": "alu", "achieved": flops / ms / 1e9,
+                                 "peak": fp32_peak, "unit": "TFLOP/s",
+                                 "frac": flops / ms / 1e9 / fp32_peak,
+                                 "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 x 1.92 GHz"}}
+            print(json.dumps(line), flush=True)
     elif args.config == 6:
         # latent states (KV cache compression): the 70B key projection's latent
         # for one new token and the expansion of a 4096-token latent cache

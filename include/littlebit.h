@@ -161,6 +161,45 @@ lb_status littlebit_linear_expand(const lb_linear *L, const void *z, int32_t z_d
                                   void *y, int32_t y_dtype, void *ws, size_t ws_bytes,
                                   lb_stream_t stream);
 
+/* Output buffers of one path for littlebit_dual_svid: device memory in the
+ * layouts of lb_path (the caller allocates them). */
+typedef struct {
+    int32_t r;           /* rank of this path, 1 <= r <= min(d_out, d_in), r <= 1024 */
+    uint32_t *v_bits;    /* V_sign, [ceil(d_in/32)][r] words */
+    uint32_t *u_bits;    /* U_sign, [d_out][ceil(r/32)] words */
+    uint16_t *g;         /* fp16 [d_in] */
+    uint16_t *l;         /* fp16 [r] */
+    uint16_t *h;         /* fp16 [d_out] */
+} lb_path_init;
+
+/* Workspace bytes littlebit_dual_svid needs (0 if the arguments are invalid). */
+size_t littlebit_dual_svid_workspace_size(int32_t d_out, int32_t d_in, int32_t n_paths,
+                                          const lb_path_init *paths);
+
+/* Dual-SVID initialisation (Sec. 3.2) of a LittleBit linear from a dense
+ * weight, with Residual Compensation (Sec. 3.3): path 0 from W, path 1 (if
+ * n_paths = 2) from the residual W - W_hat_0, where W_hat_0 uses path 0's
+ * scales as stored (fp16).  Per path, with the path's rank r:
+ *   (1) truncated SVD R ~ U' V'^T, the singular values split evenly
+ *       (U' = U_r diag(sqrt s), V' = V_r diag(sqrt s)); the joint sign of each
+ *       singular pair makes the largest-magnitude entry of v_j positive;
+ *   (2) U_sign = sign(U'), V_sign = sign(V'), sign(0) = +1;
+ *   (3) |U'| ~ h l_u^T and |V'| ~ g l_v^T, each the leading singular pair of
+ *       the nonnegative matrix with its singular value split evenly, and
+ *       l = l_u . l_v; h, g, l rounded to fp16 (nearest even).
+ * The SVD is computed by subspace iteration (iters >= 1 passes of
+ * Y = R Q, Q = R^T Y with Cholesky-QR re-orthonormalisation, 8 columns of
+ * oversampling, then a Rayleigh-Ritz step); it converges to the exact
+ * truncated SVD when the r-th and (r + 9)-th singular values are apart.
+ * W: DEVICE fp32 row-major [d_out][d_in]; paths: HOST array of n_paths
+ * (1 or 2) output descriptors.  ws: littlebit_dual_svid_workspace_size
+ * bytes, 256-byte aligned (no zero fill needed).  Uses cuBLAS for its GEMMs
+ * on the given stream.  Errors: LB_ERR_INVALID_ARG (shapes, ranks,
+ * pointers), LB_ERR_WORKSPACE, LB_ERR_CUDA. */
+lb_status littlebit_dual_svid(const float *W, int32_t d_out, int32_t d_in, int32_t n_paths,
+                              const lb_path_init *paths, int32_t iters, void *ws, size_t ws_bytes,
+                              lb_stream_t stream);
+
 /* Workspace bytes littlebit_stack_prepare / littlebit_stack_forward need
  * (0 if the arguments are invalid). */
 size_t littlebit_stack_workspace_size(const lb_linear *lin, int32_t n_layers, int32_t head_dim);

@@ -281,6 +281,54 @@ lb_status littlebit_linear_expand(const lb_linear *L, const void *z, int32_t z_d
     return from_cuda(lb::launch_expand_generic(*L, z, half ? 1 : 0, T, y, fp32, s));
 }
 
+namespace {
+bool check_svid(int32_t d_out, int32_t d_in, int32_t n_paths, const lb_path_init *paths) {
+    if (d_out <= 0 || d_in <= 0 || (n_paths != 1 && n_paths != 2) || !paths) return false;
+    for (int p = 0; p < n_paths; ++p) {
+        const lb_path_init &P = paths[p];
+        if (P.r < 1 || P.r > lb::kMaxRank || P.r > d_out || P.r > d_in) return false;
+    }
+    return true;
+}
+}  // namespace
+
+size_t littlebit_dual_svid_workspace_size(int32_t d_out, int32_t d_in, int32_t n_paths,
+                                          const lb_path_init *paths) {
+    if (!check_svid(d_out, d_in, n_paths, paths)) return 0;
+    int ranks[2] = {paths[0].r, n_paths > 1 ? paths[1].r : 0};
+    return lb::svid_ws_bytes(d_out, d_in, ranks, n_paths);
+}
+
+lb_status littlebit_dual_svid(const float *W, int32_t d_out, int32_t d_in, int32_t n_paths,
+                              const lb_path_init *paths, int32_t iters, void *ws, size_t ws_bytes,
+                              lb_stream_t stream) {
+    if (!check_svid(d_out, d_in, n_paths, paths) || !W || !aligned16(W) || iters < 1 ||
+        iters > 1000)
+        return LB_ERR_INVALID_ARG;
+    for (int p = 0; p < n_paths; ++p) {
+        const lb_path_init &P = paths[p];
+        if (!P.v_bits || !P.u_bits || !P.g || !P.l || !P.h || !aligned16(P.v_bits) ||
+            !aligned16(P.u_bits) || !aligned16(P.g) || !aligned16(P.l) || !aligned16(P.h))
+            return LB_ERR_INVALID_ARG;
+    }
+    if (!ws || ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) ||
+        ws_bytes < littlebit_dual_svid_workspace_size(d_out, d_in, n_paths, paths))
+        return LB_ERR_WORKSPACE;
+    int ranks[2];
+    uint32_t *vb[2], *ub[2];
+    uint16_t *g[2], *l[2], *h[2];
+    for (int p = 0; p < n_paths; ++p) {
+        ranks[p] = paths[p].r;
+        vb[p] = paths[p].v_bits;
+        ub[p] = paths[p].u_bits;
+        g[p] = paths[p].g;
+        l[p] = paths[p].l;
+        h[p] = paths[p].h;
+    }
+    return from_cuda(lb::launch_dual_svid(W, d_out, d_in, n_paths, ranks, vb, ub, g, l, h, iters,
+                                          ws, (cudaStream_t)stream));
+}
+
 size_t littlebit_stack_workspace_size(const lb_linear *lin, int32_t n_layers, int32_t head_dim) {
     lb::StackShape shape;
     if (check_stack(lin, n_layers, head_dim, &shape) != LB_OK) return 0;

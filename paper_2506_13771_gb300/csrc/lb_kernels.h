@@ -71,6 +71,15 @@ cudaError_t launch_prefill_latent(const lb_linear &L, const uint16_t *x, int64_t
 cudaError_t launch_prefill_expand(const lb_linear &L, const uint16_t *z16, int64_t T, void *y,
                                   int y_fp32, unsigned *ws_words, void *ws, cudaStream_t s);
 
+// Dual-SVID initialisation (lb_svid.cu): W fp32 row-major [d_out][d_in],
+// per path the output sign words and fp16 scales; ws: svid_ws_bytes.
+int svid_k(int r, int d_out, int d_in);
+size_t svid_ws_bytes(int d_out, int d_in, const int *ranks, int n_paths);
+cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, const int *ranks,
+                             uint32_t *const *v_bits, uint32_t *const *u_bits, uint16_t *const *g,
+                             uint16_t *const *l, uint16_t *const *h, int iters, void *ws,
+                             cudaStream_t s);
+
 // Bounded-wait diagnostic (lb_persistent.cu).
 cudaError_t launch_wait_timeout(unsigned *ws_words, cudaStream_t s);
 

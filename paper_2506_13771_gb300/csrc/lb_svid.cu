@@ -1,0 +1,571 @@
+// lb_svid.cu -- Dual-SVID initialisation (Sec. 3.2) with Residual
+// Compensation (Sec. 3.3) on the GPU.
+//
+// Per path p (rank r), from the residual R (path 0: W; path p: W minus the
+// W_hat of the paths before it, with their scales as stored in fp16):
+//   (1) truncated SVD R ~ U_r diag(s) V_r^T by subspace iteration: Q (d_in x k,
+//       k = r + oversampling) starts random; each iteration Y = R Q, Y = orth(Y),
+//       Q = R^T Y, Q = orth(Q), orth being Cholesky QR applied twice with the
+//       Gram matrix in fp64; then Rayleigh-Ritz: B = R Q, B^T B = E diag(lam) E^T
+//       (Jacobi, fp64), s = sqrt(lam), V_r = Q E_r, U_r = B E_r diag(1/s).
+//       Sign convention: each v_j has its largest-magnitude entry positive.
+//   (2) U' = U_r diag(sqrt s), V' = V_r diag(sqrt s); U_sign = sign(U'),
+//       V_sign = sign(V') (sign(0) = +1), packed in the lb_path layouts.
+//   (3) |U'| ~ h l_u^T, |V'| ~ g l_v^T, the leading singular pair of each
+//       nonnegative matrix by power iteration (fp64), the singular value split
+//       evenly; l = l_u . l_v.  h, g, l are rounded to fp16 (nearest even).
+// The GEMMs are cuBLAS (plain fp32 / fp64 GEMMs); the small dense problems
+// (Cholesky and triangular inverse of a k x k Gram matrix, the k x k Jacobi
+// eigenproblem) run in one CTA each; the rest are elementwise / reduction
+// kernels below.
+#include <cublas_v2.h>
+
+#include <algorithm>
+#include <cmath>
+#include <mutex>
+#include <vector>
+
+#include "lb_common.cuh"
+#include "lb_kernels.h"
+
+namespace lb {
+
+namespace {
+
+constexpr int kOversample = 8;
+constexpr int kPowerIters = 100;  // rank-1 power iterations on |U'|, |V'|
+constexpr int kJacobiSweeps = 40;
+constexpr int kSmallThreads = 1024;
+
+// Sum of v over the block, returned to every thread (blockDim.x <= 1024).
+__device__ double block_sum_d(double v) {
+    __shared__ double s_part[32];
+    __shared__ double s_total;
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (lane == 0) s_part[warp] = v;
+    __syncthreads();
+    if (warp == 0) {
+        const int nw = (blockDim.x + 31) >> 5;
+        double t = lane < nw ? s_part[lane] : 0.0;
+        for (int o = 16; o > 0; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
+        if (lane == 0) s_total = t;
+    }
+    __syncthreads();
+    const double total = s_total;
+    __syncthreads();
+    return total;
+}
+
+// ---------------------------------------------------------------- random start
+
+// Q[i] uniform in [-1, 1) from a 64-bit counter hash (splitmix64 finaliser).
+__global__ void k_rand(float *Q, long long n, unsigned long long seed) {
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n;
+         i += (long long)gridDim.x * blockDim.x) {
+        unsigned long long z = seed + 0x9E3779B97F4A7C15ull * (unsigned long long)(i + 1);
+        z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+        z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+        z ^= z >> 31;
+        Q[i] = (float)((double)(z >> 11) * (1.0 / 9007199254740992.0) * 2.0 - 1.0);
+    }
+}
+
+__global__ void k_to_f64(const float *a, double *b, long long n) {
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < n;
+         i += (long long)gridDim.x * blockDim.x)
+        b[i] = (double)a[i];
+}
+
+// ---------------------------------------------------------------- Cholesky QR
+
+// G (k x k, column-major, fp64, symmetric positive semidefinite) -> Lt
+// (fp32, k x k column-major) = (L^{-1})^T where G = L L^T, so that Y Lt has
+// orthonormal columns when G = Y^T Y.  One CTA; X (k x k fp64) is scratch for
+// L^{-1}.  A pivot at or below 1e-14 of the mean diagonal (a column of Y in
+// the span of the previous ones, or Y = 0) is set to zero, and so are the
+// entries of L below it and of L^{-1} that depend on it: that column of Y
+// maps to zero instead of blowing up.
+__global__ void __launch_bounds__(kSmallThreads) k_chol_inv(double *G, int k, double *X, float *Lt) {
+    __shared__ double s_piv;
+    double trace = 0.0;
+    for (int j = 0; j < k; ++j) trace += G[(size_t)j * k + j];
+    const double floor_piv = 1e-14 * fmax(trace, 0.0) / k;
+    // Cholesky in place: L(i, j) at G[j * k + i], i >= j
+    for (int j = 0; j < k; ++j) {
+        if (threadIdx.x == 0) {
+            double d = G[(size_t)j * k + j];
+            for (int p = 0; p < j; ++p) d -= G[(size_t)p * k + j] * G[(size_t)p * k + j];
+            s_piv = d > floor_piv && d > 0.0 ? sqrt(d) : 0.0;
+            G[(size_t)j * k + j] = s_piv;
+        }
+        __syncthreads();
+        const double piv = s_piv;
+        for (int i = j + 1 + threadIdx.x; i < k; i += blockDim.x) {
+            double a = G[(size_t)j * k + i];
+            for (int p = 0; p < j; ++p) a -= G[(size_t)p * k + i] * G[(size_t)p * k + j];
+            G[(size_t)j * k + i] = piv > 0.0 ? a / piv : 0.0;
+        }
+        __syncthreads();
+    }
+    // column c of L^{-1} by forward substitution (one thread per column):
+    // x_i = (delta_ic - sum_{c <= p < i} L(i, p) x_p) / L(i, i), x in X[c * k + .];
+    // Lt(c, i) = L^{-1}(i, c) goes to Lt[i * k + c]
+    for (int c = threadIdx.x; c < k; c += blockDim.x) {
+        double *x = X + (size_t)c * k;
+        for (int i = 0; i < k; ++i) {
+            double xi = 0.0;
+            if (i >= c) {
+                double a = (i == c) ? 1.0 : 0.0;
+                for (int p = c; p < i; ++p) a -= G[(size_t)p * k + i] * x[p];
+                const double piv = G[(size_t)i * k + i];
+                xi = piv > 0.0 ? a / piv : 0.0;
+            }
+            x[i] = xi;
+            Lt[(size_t)i * k + c] = (float)xi;
+        }
+    }
+}
+
+// ---------------------------------------------------------------- Jacobi eigen
+
+// Symmetric M (k x k, fp64, column-major, overwritten) -> eigenvalues lam (k,
+// decreasing) and eigenvectors E (fp32, k x k column-major, column j for
+// lam[j]).  Cyclic Jacobi with the round-robin pairing: each round rotates
+// k/2 disjoint pairs (p, q) at once, M <- J^T M J, V <- V J.  One CTA; V is
+// fp64 scratch (k x k).  Sweeps stop once the largest |off-diagonal| is at
+// most 1e-15 of the largest |diagonal| (or after kJacobiSweeps).
+__global__ void __launch_bounds__(kSmallThreads) k_jacobi(double *M, double *V, int k, double *cs,
+                                                          double *lam, float *E) {
+    __shared__ double s_red[32];
+    __shared__ int s_done;
+    const int kk = (k + 1) & ~1;  // even count: index k is a dummy when k is odd
+    for (int idx = threadIdx.x; idx < k * k; idx += blockDim.x)
+        V[idx] = (idx / k == idx % k) ? 1.0 : 0.0;
+    __syncthreads();
+    for (int sweep = 0; sweep < kJacobiSweeps; ++sweep) {
+        // convergence test
+        double off = 0.0, dia = 0.0;
+        for (int idx = threadIdx.x; idx < k * k; idx += blockDim.x) {
+            const int c = idx / k, i = idx % k;
+            const double a = fabs(M[idx]);
+            if (i == c) dia = fmax(dia, a);
+            else off = fmax(off, a);
+        }
+        for (int o = 16; o > 0; o >>= 1) {
+            off = fmax(off, __shfl_xor_sync(0xffffffffu, off, o));
+            dia = fmax(dia, __shfl_xor_sync(0xffffffffu, dia, o));
+        }
+        if ((threadIdx.x & 31) == 0) {
+            s_red[threadIdx.x >> 5] = off;
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            double m = 0.0;
+            for (int w = 0; w < (int)(blockDim.x >> 5); ++w) m = fmax(m, s_red[w]);
+            s_red[0] = m;
+        }
+        __syncthreads();
+        const double off_all = s_red[0];
+        __syncthreads();
+        if ((threadIdx.x & 31) == 0) s_red[threadIdx.x >> 5] = dia;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            double m = 0.0;
+            for (int w = 0; w < (int)(blockDim.x >> 5); ++w) m = fmax(m, s_red[w]);
+            s_done = off_all <= 1e-15 * m || m == 0.0;
+        }
+        __syncthreads();
+        if (s_done) break;
+        for (int round = 0; round < kk - 1; ++round) {
+            // pairs of this round: position 0 fixed, the others rotate
+            for (int t = threadIdx.x; t < kk / 2; t += blockDim.x) {
+                int a = t == 0 ? 0 : 1 + (t - 1 + round) % (kk - 1);
+                int b = 1 + (kk - 2 - t + round) % (kk - 1);
+                if (a > b) { const int x = a; a = b; b = x; }
+                double c = 1.0, s = 0.0;
+                if (b < k) {
+                    const double app = M[(size_t)a * k + a], aqq = M[(size_t)b * k + b];
+                    const double apq = M[(size_t)b * k + a];
+                    if (apq != 0.0) {
+                        const double zeta = (aqq - app) / (2.0 * apq);
+                        const double tt = (zeta >= 0 ? 1.0 : -1.0) / (fabs(zeta) + sqrt(1.0 + zeta * zeta));
+                        c = 1.0 / sqrt(1.0 + tt * tt);
+                        s = c * tt;
+                    }
+                }
+                cs[4 * t] = (double)a;
+                cs[4 * t + 1] = (double)b;
+                cs[4 * t + 2] = c;
+                cs[4 * t + 3] = s;
+            }
+            __syncthreads();
+            // columns: M <- M J, V <- V J (pair t rotates columns a, b)
+            for (int idx = threadIdx.x; idx < (kk / 2) * k; idx += blockDim.x) {
+                const int t = idx / k, i = idx % k;
+                const int a = (int)cs[4 * t], b = (int)cs[4 * t + 1];
+                if (b >= k) continue;
+                const double c = cs[4 * t + 2], s = cs[4 * t + 3];
+                const double x = M[(size_t)a * k + i], y = M[(size_t)b * k + i];
+                M[(size_t)a * k + i] = c * x - s * y;
+                M[(size_t)b * k + i] = s * x + c * y;
+                const double vx = V[(size_t)a * k + i], vy = V[(size_t)b * k + i];
+                V[(size_t)a * k + i] = c * vx - s * vy;
+                V[(size_t)b * k + i] = s * vx + c * vy;
+            }
+            __syncthreads();
+            // rows: M <- J^T M
+            for (int idx = threadIdx.x; idx < (kk / 2) * k; idx += blockDim.x) {
+                const int t = idx / k, col = idx % k;
+                const int a = (int)cs[4 * t], b = (int)cs[4 * t + 1];
+                if (b >= k) continue;
+                const double c = cs[4 * t + 2], s = cs[4 * t + 3];
+                const double x = M[(size_t)col * k + a], y = M[(size_t)col * k + b];
+                M[(size_t)col * k + a] = c * x - s * y;
+                M[(size_t)col * k + b] = s * x + c * y;
+            }
+            __syncthreads();
+        }
+    }
+    // sort by decreasing eigenvalue: the rank of each (ties by index)
+    for (int j = threadIdx.x; j < k; j += blockDim.x) {
+        const double lj = M[(size_t)j * k + j];
+        int rank = 0;
+        for (int i = 0; i < k; ++i) {
+            const double li = M[(size_t)i * k + i];
+            rank += (li > lj) || (li == lj && i < j);
+        }
+        lam[rank] = lj;
+        for (int i = 0; i < k; ++i) E[(size_t)rank * k + i] = (float)V[(size_t)j * k + i];
+    }
+}
+
+// ---------------------------------------------------------------- Ritz vectors
+
+// s_j = sqrt(max(lam_j, 0)); U (m x r, column-major) /= s_j (0 where s_j = 0).
+__global__ void k_ritz_scale(const double *lam, float *U, int m, int r, double *s) {
+    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < (long long)m * r;
+         idx += (long long)gridDim.x * blockDim.x) {
+        const int j = (int)(idx / m);
+        const double sj = sqrt(fmax(lam[j], 0.0));
+        if (idx % m == 0) s[j] = sj;
+        U[idx] = sj > 0.0 ? (float)((double)U[idx] / sj) : 0.0f;
+    }
+}
+
+// Sign convention and the even split: for column j, the entry of V (n x r)
+// of largest magnitude (first on a tie) decides a joint sign; then
+// U' = sign * U * sqrt(s_j), V' = sign * V * sqrt(s_j).  One block per column.
+__global__ void k_sign_split(float *U, float *V, int m, int n, const double *s) {
+    const int j = blockIdx.x;
+    __shared__ float s_v[32];
+    __shared__ int s_i[32];
+    float best = -1.f;
+    int bi = 0x7fffffff;
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+        const float a = fabsf(V[(size_t)j * n + i]);
+        if (a > best || (a == best && i < bi)) {
+            best = a;
+            bi = i;
+        }
+    }
+    for (int o = 16; o > 0; o >>= 1) {
+        const float ob = __shfl_xor_sync(0xffffffffu, best, o);
+        const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+        if (ob > best || (ob == best && oi < bi)) {
+            best = ob;
+            bi = oi;
+        }
+    }
+    if ((threadIdx.x & 31) == 0) {
+        s_v[threadIdx.x >> 5] = best;
+        s_i[threadIdx.x >> 5] = bi;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        for (int w = 1; w < (int)(blockDim.x >> 5); ++w)
+            if (s_v[w] > s_v[0] || (s_v[w] == s_v[0] && s_i[w] < s_i[0])) {
+                s_v[0] = s_v[w];
+                s_i[0] = s_i[w];
+            }
+    }
+    __syncthreads();
+    const int imax = s_i[0];
+    const float sg = (imax < n && V[(size_t)j * n + imax] < 0.f) ? -1.f : 1.f;
+    __syncthreads();
+    const float f = sg * (float)sqrt(s[j]);
+    for (int i = threadIdx.x; i < n; i += blockDim.x) V[(size_t)j * n + i] *= f;
+    for (int i = threadIdx.x; i < m; i += blockDim.x) U[(size_t)j * m + i] *= f;
+}
+
+// ---------------------------------------------------------------- signs
+
+// u_bits[o][w] from U' (d_out x r, column-major): bit k = U'(o, 32w + k) < 0.
+__global__ void k_pack_u_cm(const float *U, int d_out, int r, uint32_t *u_bits) {
+    const int R = (r + 31) >> 5;
+    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < (long long)d_out * R;
+         idx += (long long)gridDim.x * blockDim.x) {
+        const int o = (int)(idx / R), w = (int)(idx % R);
+        uint32_t word = 0;
+        for (int b = 0; b < 32 && 32 * w + b < r; ++b)
+            if (U[(size_t)(32 * w + b) * d_out + o] < 0.f) word |= 1u << b;
+        u_bits[idx] = word;
+    }
+}
+
+// v_bits[w][j] from V' (d_in x r, column-major): bit k = V'(32w + k, j) < 0.
+__global__ void k_pack_v_cm(const float *V, int d_in, int r, uint32_t *v_bits) {
+    const int W = (d_in + 31) >> 5;
+    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < (long long)W * r;
+         idx += (long long)gridDim.x * blockDim.x) {
+        const int w = (int)(idx / r), j = (int)(idx % r);
+        uint32_t word = 0;
+        for (int b = 0; b < 32 && 32 * w + b < d_in; ++b)
+            if (V[(size_t)j * d_in + 32 * w + b] < 0.f) word |= 1u << b;
+        v_bits[idx] = word;
+    }
+}
+
+// ---------------------------------------------------------------- rank-1 of |M|
+
+// y[i] = sum_j |M(i, j)| x[j], M rows x cols column-major; one thread per row.
+__global__ void k_abs_mv(const float *M, int rows, int cols, const double *x, double *y) {
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < rows; i += gridDim.x * blockDim.x) {
+        double acc = 0.0;
+        for (int j = 0; j < cols; ++j) acc += fabs((double)M[(size_t)j * rows + i]) * x[j];
+        y[i] = acc;
+    }
+}
+
+// x[j] = sum_i |M(i, j)| y[i]; one block per column.
+__global__ void k_abs_mtv(const float *M, int rows, const double *y, double *x) {
+    const int j = blockIdx.x;
+    double acc = 0.0;
+    for (int i = threadIdx.x; i < rows; i += blockDim.x)
+        acc += fabs((double)M[(size_t)j * rows + i]) * y[i];
+    acc = block_sum_d(acc);
+    if (threadIdx.x == 0) x[j] = acc;
+}
+
+// v <- v / |v| (one block); the norm goes to *nrm.
+__global__ void k_normalize(double *v, int n, double *nrm) {
+    double ss = 0.0;
+    for (int i = threadIdx.x; i < n; i += blockDim.x) ss += v[i] * v[i];
+    ss = block_sum_d(ss);
+    const double nv = sqrt(ss);
+    for (int i = threadIdx.x; i < n; i += blockDim.x) v[i] = nv > 0.0 ? v[i] / nv : 0.0;
+    if (threadIdx.x == 0) *nrm = nv;
+}
+
+__global__ void k_fill(double *v, int n, double val) {
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) v[i] = val;
+}
+
+// a = sqrt(sigma) u as fp16 (a zero sigma gives zeros); optionally keep the
+// fp64 values in keep[] as well.
+__global__ void k_split_half(const double *u, int n, const double *sigma, uint16_t *out,
+                             double *keep) {
+    const double sq = sqrt(fmax(*sigma, 0.0));
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) {
+        const double a = *sigma > 0.0 ? sq * u[i] : 0.0;
+        if (keep) keep[i] = a;
+        else out[i] = __half_as_ushort(__double2half(a));
+    }
+}
+
+// l = l_u . l_v as fp16.
+__global__ void k_latent_half(const double *lu, const double *lv, int r, uint16_t *l) {
+    for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < r; j += gridDim.x * blockDim.x)
+        l[j] = __half_as_ushort(__double2half(lu[j] * lv[j]));
+}
+
+// ---------------------------------------------------------------- residual
+
+// A1 (d_out x r, cm) = h_o * sign(U'(o, j)) * l_j, B1 (d_in x r, cm) =
+// g_i * sign(V'(i, j)), from the stored fp16 scales, so that
+// W_hat = A1 B1^T (Eq. 4).
+__global__ void k_what_factors(const float *U, const float *V, int d_out, int d_in, int r,
+                               const uint16_t *h, const uint16_t *g, const uint16_t *l, float *A1,
+                               float *B1) {
+    const long long na = (long long)d_out * r, nb = (long long)d_in * r;
+    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < na + nb;
+         idx += (long long)gridDim.x * blockDim.x) {
+        if (idx < na) {
+            const int j = (int)(idx / d_out), o = (int)(idx % d_out);
+            const float sg = U[idx] < 0.f ? -1.f : 1.f;
+            A1[idx] = half_bits_to_float(h[o]) * sg * half_bits_to_float(l[j]);
+        } else {
+            const long long e = idx - na;
+            const int i = (int)(e % d_in);
+            const float sg = V[e] < 0.f ? -1.f : 1.f;
+            B1[e] = half_bits_to_float(g[i]) * sg;
+        }
+    }
+}
+
+// ---------------------------------------------------------------- cuBLAS
+
+std::mutex g_blas_mu;
+cublasHandle_t g_blas[64];
+
+cublasHandle_t blas_handle() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    std::lock_guard<std::mutex> lock(g_blas_mu);
+    if (!g_blas[dev] && cublasCreate(&g_blas[dev]) != CUBLAS_STATUS_SUCCESS) g_blas[dev] = nullptr;
+    return g_blas[dev];
+}
+
+int grid_for(long long n) { return (int)std::min<long long>((n + 255) / 256, 152 * 8); }
+
+struct Buf {
+    char *p;
+    size_t off = 0;
+    template <class T>
+    T *take(size_t n) {
+        T *r = reinterpret_cast<T *>(p + off);
+        off += (n * sizeof(T) + 255) & ~(size_t)255;
+        return r;
+    }
+};
+
+}  // namespace
+
+int svid_k(int r, int d_out, int d_in) { return std::min(r + kOversample, std::min(d_out, d_in)); }
+
+size_t svid_ws_bytes(int d_out, int d_in, const int *ranks, int n_paths) {
+    int kmax = 0;
+    for (int p = 0; p < n_paths; ++p) kmax = std::max(kmax, svid_k(ranks[p], d_out, d_in));
+    Buf b{nullptr};
+    const size_t m = (size_t)d_out, n = (size_t)d_in, k = (size_t)kmax;
+    b.take<float>(m * n);                  // R (residual, column-major n x m = row-major W)
+    b.take<float>(n * k);                  // Q
+    b.take<float>(n * k);                  // Q2
+    b.take<float>(m * k);                  // Y
+    b.take<float>(m * k);                  // Y2
+    b.take<double>(std::max(m, n) * k);    // fp64 copy for the Gram matrix
+    b.take<double>(k * k);                 // G / M
+    b.take<double>(k * k);                 // Jacobi V
+    b.take<double>(4 * ((k + 2) / 2));     // Jacobi rotations
+    b.take<float>(k * k);                  // L^-T / E
+    b.take<double>(k);                     // lam
+    b.take<double>(k);                     // s
+    b.take<double>(m + n);                 // power iteration y
+    b.take<double>(2 * k);                 // x, l_u / l_v (fp64)
+    b.take<double>(4);                     // norms
+    return b.off + 256;
+}
+
+cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, const int *ranks,
+                             uint32_t *const *v_bits, uint32_t *const *u_bits, uint16_t *const *g,
+                             uint16_t *const *l, uint16_t *const *h, int iters, void *ws,
+                             cudaStream_t s) {
+    cublasHandle_t H = blas_handle();
+    if (!H) return cudaErrorNotSupported;
+    if (cublasSetStream(H, s) != CUBLAS_STATUS_SUCCESS) return cudaErrorUnknown;
+    cublasSetPointerMode(H, CUBLAS_POINTER_MODE_HOST);
+    const int m = d_out, n = d_in;
+    int kmax = 0;
+    for (int p = 0; p < n_paths; ++p) kmax = std::max(kmax, svid_k(ranks[p], d_out, d_in));
+    Buf b{static_cast<char *>(ws)};
+    float *R = b.take<float>((size_t)m * n);
+    float *Q = b.take<float>((size_t)n * kmax);
+    float *Q2 = b.take<float>((size_t)n * kmax);
+    float *Y = b.take<float>((size_t)m * kmax);
+    float *Y2 = b.take<float>((size_t)m * kmax);
+    double *D = b.take<double>((size_t)std::max(m, n) * kmax);
+    double *G = b.take<double>((size_t)kmax * kmax);
+    double *JV = b.take<double>((size_t)kmax * kmax);
+    double *rot = b.take<double>(4 * ((size_t)(kmax + 2) / 2));
+    float *Lt = b.take<float>((size_t)kmax * kmax);
+    double *lam = b.take<double>(kmax);
+    double *sv = b.take<double>(kmax);
+    double *py = b.take<double>((size_t)m + n);
+    double *px = b.take<double>(2 * (size_t)kmax);
+    double *nrm = b.take<double>(4);
+    // R = W (row-major m x n is the column-major n x m matrix R^T)
+    cudaError_t e = cudaMemcpyAsync(R, W, (size_t)m * n * sizeof(float), cudaMemcpyDeviceToDevice, s);
+    if (e != cudaSuccess) return e;
+    const float one = 1.f, zero = 0.f, minus = -1.f;
+    const double done = 1.0, dzero = 0.0;
+    bool blas_ok = true;
+    auto gemm = [&](cublasOperation_t ta, cublasOperation_t tb, int mm, int nn, int kk,
+                    const float *A, int lda, const float *B, int ldb, const float *beta, float *C,
+                    int ldc, const float *alpha) {
+        blas_ok = blas_ok && cublasSgemm(H, ta, tb, mm, nn, kk, alpha, A, lda, B, ldb, beta, C, ldc) ==
+                                 CUBLAS_STATUS_SUCCESS;
+    };
+    // orthonormalise the columns of X (rows x k, column-major) into X (via Xt)
+    auto orth = [&](float *X, float *Xt, int rows, int k) {
+        for (int pass = 0; pass < 2; ++pass) {
+            k_to_f64<<<grid_for((long long)rows * k), 256, 0, s>>>(X, D, (long long)rows * k);
+            blas_ok = blas_ok && cublasDgemm(H, CUBLAS_OP_T, CUBLAS_OP_N, k, k, rows, &done, D, rows,
+                                             D, rows, &dzero, G, k) == CUBLAS_STATUS_SUCCESS;
+            k_chol_inv<<<1, kSmallThreads, 0, s>>>(G, k, JV, Lt);
+            gemm(CUBLAS_OP_N, CUBLAS_OP_N, rows, k, k, X, rows, Lt, k, &zero, Xt, rows, &one);
+            cudaMemcpyAsync(X, Xt, (size_t)rows * k * sizeof(float), cudaMemcpyDeviceToDevice, s);
+        }
+    };
+    for (int p = 0; p < n_paths && blas_ok; ++p) {
+        const int r = ranks[p], k = svid_k(r, m, n);
+        k_rand<<<grid_for((long long)n * k), 256, 0, s>>>(Q, (long long)n * k,
+                                                          0x5EEDull + 7919ull * (unsigned)p);
+        orth(Q, Q2, n, k);
+        for (int it = 0; it < iters; ++it) {
+            // Y = R Q  (R is n x m column-major: op T gives m x n)
+            gemm(CUBLAS_OP_T, CUBLAS_OP_N, m, k, n, R, n, Q, n, &zero, Y, m, &one);
+            orth(Y, Y2, m, k);
+            // Q = R^T Y
+            gemm(CUBLAS_OP_N, CUBLAS_OP_N, n, k, m, R, n, Y, m, &zero, Q, n, &one);
+            orth(Q, Q2, n, k);
+        }
+        // Rayleigh-Ritz: B = R Q (in Y), M = B^T B (fp64), eigen
+        gemm(CUBLAS_OP_T, CUBLAS_OP_N, m, k, n, R, n, Q, n, &zero, Y, m, &one);
+        k_to_f64<<<grid_for((long long)m * k), 256, 0, s>>>(Y, D, (long long)m * k);
+        blas_ok = blas_ok && cublasDgemm(H, CUBLAS_OP_T, CUBLAS_OP_N, k, k, m, &done, D, m, D, m,
+                                         &dzero, G, k) == CUBLAS_STATUS_SUCCESS;
+        k_jacobi<<<1, kSmallThreads, 0, s>>>(G, JV, k, rot, lam, Lt);
+        // V_r = Q E_r (into Q2, n x r), U_r = B E_r / s (into Y2, m x r)
+        gemm(CUBLAS_OP_N, CUBLAS_OP_N, n, r, k, Q, n, Lt, k, &zero, Q2, n, &one);
+        gemm(CUBLAS_OP_N, CUBLAS_OP_N, m, r, k, Y, m, Lt, k, &zero, Y2, m, &one);
+        k_ritz_scale<<<grid_for((long long)m * r), 256, 0, s>>>(lam, Y2, m, r, sv);
+        k_sign_split<<<r, 256, 0, s>>>(Y2, Q2, m, n, sv);
+        k_pack_u_cm<<<grid_for((long long)m * ((r + 31) / 32)), 256, 0, s>>>(Y2, m, r, u_bits[p]);
+        k_pack_v_cm<<<grid_for((long long)((n + 31) / 32) * r), 256, 0, s>>>(Q2, n, r, v_bits[p]);
+        // rank-1 of |U'| (m x r) and |V'| (n x r): power iteration from x = 1
+        double *lu = px, *lv = px + kmax;
+        for (int side = 0; side < 2; ++side) {
+            const float *M = side == 0 ? Y2 : Q2;
+            const int rows = side == 0 ? m : n;
+            k_fill<<<1, 256, 0, s>>>(px + side * kmax, r, 1.0 / sqrt((double)r));
+            double *x = px + side * kmax;
+            for (int it = 0; it < kPowerIters; ++it) {
+                k_abs_mv<<<grid_for(rows), 256, 0, s>>>(M, rows, r, x, py);
+                k_normalize<<<1, 1024, 0, s>>>(py, rows, nrm);
+                k_abs_mtv<<<r, 256, 0, s>>>(M, rows, py, x);
+                k_normalize<<<1, 1024, 0, s>>>(x, r, nrm + 1);
+            }
+            // x = v (unit), py = u (unit), sigma = |M^T u| in nrm[1]
+            if (side == 0) {
+                k_split_half<<<grid_for(rows), 256, 0, s>>>(py, rows, nrm + 1, h[p], nullptr);
+                k_split_half<<<1, 256, 0, s>>>(x, r, nrm + 1, nullptr, lu);
+            } else {
+                k_split_half<<<grid_for(rows), 256, 0, s>>>(py, rows, nrm + 1, g[p], nullptr);
+                k_split_half<<<1, 256, 0, s>>>(x, r, nrm + 1, nullptr, lv);
+            }
+        }
+        k_latent_half<<<1, 256, 0, s>>>(lu, lv, r, l[p]);
+        if (p + 1 < n_paths) {
+            // R <- R - W_hat_p: R^T (n x m) -= B1 A1^T with A1 = h.U_sign.l, B1 = g.V_sign
+            float *A1 = Y, *B1 = Q;
+            k_what_factors<<<grid_for((long long)(m + n) * r), 256, 0, s>>>(Y2, Q2, m, n, r, h[p],
+                                                                             g[p], l[p], A1, B1);
+            gemm(CUBLAS_OP_N, CUBLAS_OP_T, n, m, r, B1, n, A1, m, &one, R, n, &minus);
+        }
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    return blas_ok ? cudaSuccess : cudaErrorUnknown;
+}
+
+}  // namespace lb

@@ -181,3 +181,14 @@ def make_stack(n_layers: int = 80, d_model: int = 8192, d_kv: int = 1024, d_ff: 
 def config5(n_layers: int = 80):
     kw = {k: v for k, v in STACK_70B.items() if k not in ("n_layers", "head_dim")}
     return make_stack(n_layers=n_layers, **kw)
+
+
+def spectral_weight(rng: np.random.Generator, d_out: int, d_in: int,
+                    spectrum: np.ndarray) -> np.ndarray:
+    """A dense fp64 weight A diag(spectrum) B^T with random orthonormal A, B
+    (QR of Gaussian matrices): a synthetic stand-in for a trained weight with
+    a prescribed singular spectrum (the Dual-SVID workloads)."""
+    k = min(d_out, d_in)
+    A, _ = np.linalg.qr(rng.standard_normal((d_out, k)))
+    B, _ = np.linalg.qr(rng.standard_normal((d_in, k)))
+    return (A * np.asarray(spectrum, np.float64)[:k]) @ B.T

@@ -24,6 +24,7 @@ LB_PACK_U, LB_PACK_V = 0, 1
 
 EXPORTED = ["littlebit_status_string", "littlebit_pack", "littlebit_workspace_size",
             "littlebit_linear_forward", "littlebit_linear_latent", "littlebit_linear_expand",
+            "littlebit_dual_svid_workspace_size", "littlebit_dual_svid",
             "littlebit_stack_workspace_size",
             "littlebit_stack_prepare", "littlebit_stack_forward", "littlebit_poll_error",
             "littlebit_selftest_wait_timeout", "littlebit_linear_forward_noalloc"]
@@ -49,6 +50,12 @@ class lb_linear(ctypes.Structure):
                 ("d_out", ctypes.c_int32),
                 ("n_paths", ctypes.c_int32),
                 ("path", lb_path * 2)]
+
+
+class lb_path_init(ctypes.Structure):
+    """Output buffers of one path for littlebit_dual_svid (device pointers)."""
+    _fields_ = [("r", ctypes.c_int32), ("v_bits", ctypes.c_void_p), ("u_bits", ctypes.c_void_p),
+                ("g", ctypes.c_void_p), ("l", ctypes.c_void_p), ("h", ctypes.c_void_p)]
 
 
 _lib = None
@@ -81,6 +88,11 @@ def lib(path: str | None = None):
         L.littlebit_linear_expand.argtypes = [ctypes.POINTER(lb_linear), vp, i32, i64, vp, i32,
                                               vp, sz, vp]
         L.littlebit_linear_expand.restype = ctypes.c_int
+        L.littlebit_dual_svid_workspace_size.argtypes = [i32, i32, i32, ctypes.POINTER(lb_path_init)]
+        L.littlebit_dual_svid_workspace_size.restype = sz
+        L.littlebit_dual_svid.argtypes = [vp, i32, i32, i32, ctypes.POINTER(lb_path_init), i32, vp,
+                                          sz, vp]
+        L.littlebit_dual_svid.restype = ctypes.c_int
         L.littlebit_stack_workspace_size.argtypes = [ctypes.POINTER(lb_linear), i32, i32]
         L.littlebit_stack_workspace_size.restype = sz
         L.littlebit_stack_prepare.argtypes = [ctypes.POINTER(lb_linear), i32, i32, vp, sz, vp]
@@ -255,6 +267,52 @@ def linear_expand(L: DeviceLinear, z: torch.Tensor, out_dtype=torch.bfloat16,
                                          y_dtype, ws.data_ptr(), ws.numel(), _stream(stream)),
            "littlebit_linear_expand")
     return y
+
+
+def dual_svid(W: torch.Tensor, ranks, iters: int = 8, ws: torch.Tensor | None = None,
+              stream=None) -> dict:
+    """Dual-SVID initialisation (Sec. 3.2) with Residual Compensation (Sec. 3.3) of a dense
+    fp32 weight W [d_out][d_in] on the device.  Returns a layer dict of device tensors:
+    {'d_in', 'd_out', 'paths': [{'r', 'v_words', 'u_words', 'g', 'l', 'h'}]} (int32 words,
+    int16 fp16 bit patterns)."""
+    assert W.dtype == torch.float32 and W.dim() == 2 and W.is_cuda
+    W = W.contiguous()
+    d_out, d_in = W.shape
+    outs = []
+    arr = (lb_path_init * len(ranks))()
+    for p, r in enumerate(ranks):
+        t = {"r": int(r),
+             "v_words": torch.empty(((d_in + 31) // 32, r), dtype=torch.int32, device=W.device),
+             "u_words": torch.empty((d_out, (r + 31) // 32), dtype=torch.int32, device=W.device),
+             "g": torch.empty(d_in, dtype=torch.int16, device=W.device),
+             "l": torch.empty(r, dtype=torch.int16, device=W.device),
+             "h": torch.empty(d_out, dtype=torch.int16, device=W.device)}
+        outs.append(t)
+        arr[p].r = int(r)
+        arr[p].v_bits, arr[p].u_bits = t["v_words"].data_ptr(), t["u_words"].data_ptr()
+        arr[p].g, arr[p].l, arr[p].h = t["g"].data_ptr(), t["l"].data_ptr(), t["h"].data_ptr()
+    n = int(lib().littlebit_dual_svid_workspace_size(d_out, d_in, len(ranks), arr))
+    if n == 0:
+        raise LittleBitError(LB_ERR_INVALID_ARG, "littlebit_dual_svid_workspace_size")
+    if ws is None:
+        ws = torch.empty(n, dtype=torch.uint8, device=W.device)
+    _check(lib().littlebit_dual_svid(W.data_ptr(), d_out, d_in, len(ranks), arr, int(iters),
+                                     ws.data_ptr(), ws.numel(), _stream(stream)),
+           "littlebit_dual_svid")
+    return {"d_in": d_in, "d_out": d_out, "paths": outs}
+
+
+def layer_to_host(layer: dict) -> dict:
+    """A layer dict of device tensors as numpy arrays in the inputs.make_linear layout."""
+    paths = []
+    for P in layer["paths"]:
+        paths.append({"r": P["r"],
+                      "v_words": P["v_words"].cpu().numpy().view(np.uint32),
+                      "u_words": P["u_words"].cpu().numpy().view(np.uint32),
+                      "g": P["g"].cpu().numpy().view(np.uint16),
+                      "l": P["l"].cpu().numpy().view(np.uint16),
+                      "h": P["h"].cpu().numpy().view(np.uint16)})
+    return {"d_in": layer["d_in"], "d_out": layer["d_out"], "paths": paths}
 
 
 class DeviceStack:

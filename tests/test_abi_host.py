@@ -119,6 +119,30 @@ def test_latent_and_expand_argument_validation(L):
     assert exp(ref, FAKE, 0, 1, FAKE, 0, FAKE + 16, 1 << 30, None) == lb.LB_ERR_WORKSPACE
 
 
+def test_dual_svid_argument_validation(L):
+    arr = (lb.lb_path_init * 2)()
+    for p in range(2):
+        arr[p].r = 16
+        arr[p].v_bits = arr[p].u_bits = arr[p].g = arr[p].l = arr[p].h = FAKE
+    ws_size = L.littlebit_dual_svid_workspace_size
+    n = ws_size(256, 384, 2, arr)
+    assert n > 256 * 384 * 4                       # holds the residual copy of W
+    assert ws_size(256, 384, 3, arr) == 0          # n_paths
+    assert ws_size(0, 384, 2, arr) == 0
+    assert ws_size(256, 384, 2, None) == 0
+    arr[1].r = 300
+    assert ws_size(256, 384, 2, arr) == 0          # r > min(d_out, d_in)
+    arr[1].r = 16
+    svid = L.littlebit_dual_svid
+    assert svid(None, 256, 384, 2, arr, 8, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    assert svid(FAKE + 4, 256, 384, 2, arr, 8, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    assert svid(FAKE, 256, 384, 2, arr, 0, FAKE, n, None) == lb.LB_ERR_INVALID_ARG   # iters
+    assert svid(FAKE, 256, 384, 2, arr, 8, FAKE, n - 256, None) == lb.LB_ERR_WORKSPACE
+    assert svid(FAKE, 256, 384, 2, arr, 8, FAKE + 16, n, None) == lb.LB_ERR_WORKSPACE
+    arr[0].h = 0
+    assert svid(FAKE, 256, 384, 2, arr, 8, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+
+
 def fake_stack(n_layers=2, d=256, dkv=64, dff=512, rq=16, rk=8, rm=24):
     shapes = [(d, d, rq), (d, dkv, rk), (d, dkv, rk), (d, d, rq), (d, dff, rm), (d, dff, rm),
               (dff, d, rm)]

@@ -297,6 +297,85 @@ def test_latent_full_size_prefill_sampled_tokens():
         assert rel(zg, oracle.latent(L, x[rows])) <= tol
 
 
+# ------------------------------------------------------------------ Dual-SVID (Sec. 3.2, 3.3)
+
+
+def _svid_weights(layer):
+    """W_hat of each path of a host layer dict (oracle unpacker and decoders)."""
+    out = []
+    for P in layer["paths"]:
+        r = P["r"]
+        us = oracle.unpack_u(P["u_words"], layer["d_out"], r)
+        vs = oracle.unpack_v(P["v_words"], layer["d_in"], r)
+        dec = lambda b: np.asarray(b, np.uint16).view(np.float16).astype(np.float64)
+        out.append((us, vs, oracle.path_weight(us, vs, dec(P["h"]), dec(P["g"]), dec(P["l"]))))
+    return out
+
+
+@pytest.mark.parametrize("d_out,d_in,ranks", [(256, 384, (16, 16)), (384, 256, (24,)),
+                                              (200, 136, (8, 40)), (96, 96, (96,))])
+def test_dual_svid_vs_oracle(d_out, d_in, ranks):
+    """Dual-SVID on the GPU (subspace iteration) against the oracle (exact
+    Jacobi SVD) on weights whose singular values fall by 0.85 per index:
+    path-0 signs equal wherever |U'| and |V'| are not tiny, scales within
+    fp16 rounding, each path's W_hat and the total reconstruction error match."""
+    rng = inputs.rng_for(108, salt=d_out + d_in)
+    W = inputs.spectral_weight(rng, d_out, d_in, 0.85 ** np.arange(min(d_out, d_in)))
+    ref = oracle.dual_svid(W, ranks)
+    got = lb.layer_to_host(lb.dual_svid(torch.from_numpy(W.astype(np.float32)).to(DEV), ranks,
+                                        iters=10))
+    torch.cuda.synchronize()
+    gw, rw = _svid_weights(got), _svid_weights(ref)
+    r0 = ranks[0]
+    s, U, V = oracle.svd_top(W, r0)
+    Up, Vp = U * np.sqrt(s), V * np.sqrt(s)
+    for mine, theirs, F in ((gw[0][0], ref["signs"][0][0], Up), (gw[0][1], ref["signs"][0][1], Vp)):
+        bad = mine != theirs
+        assert np.all(np.abs(F[bad]) < 1e-3 * np.abs(F).max()), int(bad.sum())
+    dec = lambda b: np.asarray(b, np.uint16).view(np.float16).astype(np.float64)
+    for key in ("h", "g", "l"):
+        a, b = dec(got["paths"][0][key]), dec(ref["paths"][0][key])
+        assert rel(a, b) <= 2e-3, (key, rel(a, b))
+    assert rel(gw[0][2], rw[0][2]) <= 2e-3, rel(gw[0][2], rw[0][2])
+    Wg = sum(p[2] for p in gw)
+    Wr = sum(p[2] for p in rw)
+    eg, er = rel(Wg, W), rel(Wr, W)
+    assert abs(eg - er) <= 0.02 * er + 1e-4, (eg, er)
+    if len(ranks) == 2:
+        assert rel(Wg, W) < rel(gw[0][2], W)  # the residual path helps
+
+
+def test_dual_svid_exact_cases():
+    """A Sylvester-Hadamard LittleBit weight (h = g = 1) is recovered (signs up
+    to one joint flip per column, W_hat = W within fp16 scale rounding); an
+    all-zero weight gives +1 signs and zero scales."""
+    d, r = 64, 8
+    H = np.array([[1.0]])
+    while H.shape[0] < d:
+        H = np.block([[H, H], [H, -H]])
+    H = H[:, :r]
+    lam = np.array([9.0, 7.5, 6.0, 5.0, 4.0, 3.0, 2.0, 1.5])
+    W = (H * lam) @ H.T
+    got = lb.layer_to_host(lb.dual_svid(torch.from_numpy(W.astype(np.float32)).to(DEV), [r]))
+    ((us, vs, Wg),) = _svid_weights(got)
+    flip = (us[0] * H[0]).astype(np.int8)
+    assert np.array_equal(us, (H * flip).astype(np.int8))
+    assert np.array_equal(vs, (H * flip).astype(np.int8))
+    assert rel(Wg, W) <= 2e-3
+    Z = torch.zeros((48, 80), dtype=torch.float32, device=DEV)
+    got = lb.layer_to_host(lb.dual_svid(Z, [4, 4]))
+    for P in got["paths"]:
+        assert not P["u_words"].any() and not P["v_words"].any()
+        for key in ("h", "g", "l"):
+            assert np.all(np.asarray(P[key], np.uint16).view(np.float16) == 0)
+
+
+def test_dual_svid_512x384_two_paths():
+    """A larger weight, 512 x 384 with ranks (40, 40): the same checks as the
+    small cases against the oracle's exact SVD (a few seconds of CPU work)."""
+    test_dual_svid_vs_oracle(512, 384, (40, 40))
+
+
 # ------------------------------------------------------------------ stack
 
 
