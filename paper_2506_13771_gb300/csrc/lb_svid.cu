@@ -5,9 +5,11 @@
 // W_hat of the paths before it, with their scales as stored in fp16):
 //   (1) truncated SVD R ~ U_r diag(s) V_r^T by subspace iteration: Q (d_in x k,
 //       k = r + oversampling) starts random; each iteration Y = R Q, Y = orth(Y),
-//       Q = R^T Y, Q = orth(Q), orth being Cholesky QR applied twice with the
-//       Gram matrix in fp64; then Rayleigh-Ritz: B = R Q, B^T B = E diag(lam) E^T
-//       (Jacobi, fp64), s = sqrt(lam), V_r = Q E_r, U_r = B E_r diag(1/s).
+//       Q = R^T Y, Q = orth(Q), orth being Cholesky QR with the Gram matrix in
+//       fp64 followed by a second pass in fp32; then Rayleigh-Ritz: B = R Q,
+//       B = Y' L^T (L the Cholesky factor of B^T B), L^T = U_C diag(s) E^T by
+//       one-sided Jacobi (fp32, no squaring of the spectrum), V_r = Q E_r,
+//       U_r = B E_r diag(1/s).
 //       Sign convention: each v_j has its largest-magnitude entry positive.
 //   (2) U' = U_r diag(sqrt s), V' = V_r diag(sqrt s); U_sign = sign(U'),
 //       V_sign = sign(V') (sign(0) = +1), packed in the lb_path layouts.
@@ -16,8 +18,8 @@
 //       evenly; l = l_u . l_v.  h, g, l are rounded to fp16 (nearest even).
 // The GEMMs are cuBLAS (plain fp32 / fp64 GEMMs); the small dense problems
 // (Cholesky and triangular inverse of a k x k Gram matrix, the k x k Jacobi
-// eigenproblem) run in one CTA each; the rest are elementwise / reduction
-// kernels below.
+// SVD) run in one CTA each; the rest are elementwise / reduction kernels
+// below.
 #include <cublas_v2.h>
 
 #include <algorithm>
@@ -36,6 +38,7 @@ constexpr int kOversample = 8;
 constexpr int kPowerIters = 100;  // rank-1 power iterations on |U'|, |V'|
 constexpr int kJacobiSweeps = 40;
 constexpr int kSmallThreads = 1024;
+constexpr int kMaxK = 1024 + 16;  // rank + oversampling
 
 // Sum of v over the block, returned to every thread (blockDim.x <= 1024).
 __device__ double block_sum_d(double v) {
@@ -79,47 +82,57 @@ __global__ void k_to_f64(const float *a, double *b, long long n) {
 
 // ---------------------------------------------------------------- Cholesky QR
 
-// G (k x k, column-major, fp64, symmetric positive semidefinite) -> Lt
-// (fp32, k x k column-major) = (L^{-1})^T where G = L L^T, so that Y Lt has
-// orthonormal columns when G = Y^T Y.  One CTA; X (k x k fp64) is scratch for
-// L^{-1}.  A pivot at or below 1e-14 of the mean diagonal (a column of Y in
-// the span of the previous ones, or Y = 0) is set to zero, and so are the
-// entries of L below it and of L^{-1} that depend on it: that column of Y
-// maps to zero instead of blowing up.
-__global__ void __launch_bounds__(kSmallThreads) k_chol_inv(double *G, int k, double *X, float *Lt) {
-    __shared__ double s_piv;
-    double trace = 0.0;
+// G (k x k, column-major, symmetric positive semidefinite, type T) ->
+// FACTOR ? Lt = L^T : Lt = (L^{-1})^T (fp32, k x k column-major) where
+// G = L L^T, so that Y (L^{-1})^T has orthonormal columns when G = Y^T Y.
+// One CTA; X (k x k, T) is scratch for L^{-1}.  A pivot at or below 1e-14
+// (fp64) / 1e-6 (fp32) of the mean diagonal (a column of Y in the span of the
+// previous ones, or Y = 0) is set to zero, and so are the entries of L below
+// it and of L^{-1} that depend on it: that column of Y maps to zero instead
+// of blowing up.
+template <typename T, bool FACTOR>
+__global__ void __launch_bounds__(kSmallThreads) k_chol(T *G, int k, T *X, float *Lt) {
+    __shared__ T s_piv;
+    T trace = 0;
     for (int j = 0; j < k; ++j) trace += G[(size_t)j * k + j];
-    const double floor_piv = 1e-14 * fmax(trace, 0.0) / k;
+    const T floor_piv = (sizeof(T) == 8 ? (T)1e-14 : (T)1e-6) * (trace > 0 ? trace : 0) / k;
     // Cholesky in place: L(i, j) at G[j * k + i], i >= j
     for (int j = 0; j < k; ++j) {
         if (threadIdx.x == 0) {
-            double d = G[(size_t)j * k + j];
+            T d = G[(size_t)j * k + j];
             for (int p = 0; p < j; ++p) d -= G[(size_t)p * k + j] * G[(size_t)p * k + j];
-            s_piv = d > floor_piv && d > 0.0 ? sqrt(d) : 0.0;
+            s_piv = d > floor_piv && d > 0 ? sqrt(d) : 0;
             G[(size_t)j * k + j] = s_piv;
         }
         __syncthreads();
-        const double piv = s_piv;
+        const T piv = s_piv;
         for (int i = j + 1 + threadIdx.x; i < k; i += blockDim.x) {
-            double a = G[(size_t)j * k + i];
+            T a = G[(size_t)j * k + i];
             for (int p = 0; p < j; ++p) a -= G[(size_t)p * k + i] * G[(size_t)p * k + j];
-            G[(size_t)j * k + i] = piv > 0.0 ? a / piv : 0.0;
+            G[(size_t)j * k + i] = piv > 0 ? a / piv : 0;
         }
         __syncthreads();
+    }
+    if (FACTOR) {
+        // Lt(c, i) = L(i, c) for i >= c, else 0
+        for (int idx = threadIdx.x; idx < k * k; idx += blockDim.x) {
+            const int i = idx / k, c = idx % k;  // Lt column i, row c
+            Lt[idx] = i >= c ? (float)G[(size_t)c * k + i] : 0.f;
+        }
+        return;
     }
     // column c of L^{-1} by forward substitution (one thread per column):
     // x_i = (delta_ic - sum_{c <= p < i} L(i, p) x_p) / L(i, i), x in X[c * k + .];
     // Lt(c, i) = L^{-1}(i, c) goes to Lt[i * k + c]
     for (int c = threadIdx.x; c < k; c += blockDim.x) {
-        double *x = X + (size_t)c * k;
+        T *x = X + (size_t)c * k;
         for (int i = 0; i < k; ++i) {
-            double xi = 0.0;
+            T xi = 0;
             if (i >= c) {
-                double a = (i == c) ? 1.0 : 0.0;
+                T a = (i == c) ? 1 : 0;
                 for (int p = c; p < i; ++p) a -= G[(size_t)p * k + i] * x[p];
-                const double piv = G[(size_t)i * k + i];
-                xi = piv > 0.0 ? a / piv : 0.0;
+                const T piv = G[(size_t)i * k + i];
+                xi = piv > 0 ? a / piv : 0;
             }
             x[i] = xi;
             Lt[(size_t)i * k + c] = (float)xi;
@@ -129,126 +142,101 @@ __global__ void __launch_bounds__(kSmallThreads) k_chol_inv(double *G, int k, do
 
 // ---------------------------------------------------------------- Jacobi eigen
 
-// Symmetric M (k x k, fp64, column-major, overwritten) -> eigenvalues lam (k,
-// decreasing) and eigenvectors E (fp32, k x k column-major, column j for
-// lam[j]).  Cyclic Jacobi with the round-robin pairing: each round rotates
-// k/2 disjoint pairs (p, q) at once, M <- J^T M J, V <- V J.  One CTA; V is
-// fp64 scratch (k x k).  Sweeps stop once the largest |off-diagonal| is at
-// most 1e-15 of the largest |diagonal| (or after kJacobiSweeps).
-__global__ void __launch_bounds__(kSmallThreads) k_jacobi(double *M, double *V, int k, double *cs,
-                                                          double *lam, float *E) {
-    __shared__ double s_red[32];
+// SVD of a small square A (k x k, fp32, column-major, overwritten) by
+// one-sided Jacobi: plane rotations of column pairs until the columns are
+// mutually orthogonal (A V = U diag(s), the rotations accumulated in V).
+// Round-robin pairing: each round rotates k/2 disjoint pairs, one warp per
+// pair, so the rounds need one CTA barrier each.  For columns x, y with
+// alpha = |x|^2, beta = |y|^2, gamma = x.y, t is the smaller root of
+// t^2 + 2 zeta t - 1 = 0, zeta = (beta - alpha) / (2 gamma), and
+// x' = c x - s y, y' = s x + c y.  Outputs s (k, decreasing, fp64) and the
+// right singular vectors E (fp32, k x k column-major, column j for s[j]).
+// Sweeps stop when no pair of a sweep is more than 1e-6 from orthogonal (or
+// after kJacobiSweeps).  One CTA; V is fp32 scratch (k x k).
+__global__ void __launch_bounds__(kSmallThreads) k_svd_jacobi(float *A, float *V, int k, double *sv,
+                                                              float *E) {
+    __shared__ float s_off[32];
     __shared__ int s_done;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
     const int kk = (k + 1) & ~1;  // even count: index k is a dummy when k is odd
     for (int idx = threadIdx.x; idx < k * k; idx += blockDim.x)
-        V[idx] = (idx / k == idx % k) ? 1.0 : 0.0;
+        V[idx] = (idx / k == idx % k) ? 1.f : 0.f;
     __syncthreads();
     for (int sweep = 0; sweep < kJacobiSweeps; ++sweep) {
-        // convergence test
-        double off = 0.0, dia = 0.0;
-        for (int idx = threadIdx.x; idx < k * k; idx += blockDim.x) {
-            const int c = idx / k, i = idx % k;
-            const double a = fabs(M[idx]);
-            if (i == c) dia = fmax(dia, a);
-            else off = fmax(off, a);
-        }
-        for (int o = 16; o > 0; o >>= 1) {
-            off = fmax(off, __shfl_xor_sync(0xffffffffu, off, o));
-            dia = fmax(dia, __shfl_xor_sync(0xffffffffu, dia, o));
-        }
-        if ((threadIdx.x & 31) == 0) {
-            s_red[threadIdx.x >> 5] = off;
-        }
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            double m = 0.0;
-            for (int w = 0; w < (int)(blockDim.x >> 5); ++w) m = fmax(m, s_red[w]);
-            s_red[0] = m;
-        }
-        __syncthreads();
-        const double off_all = s_red[0];
-        __syncthreads();
-        if ((threadIdx.x & 31) == 0) s_red[threadIdx.x >> 5] = dia;
-        __syncthreads();
-        if (threadIdx.x == 0) {
-            double m = 0.0;
-            for (int w = 0; w < (int)(blockDim.x >> 5); ++w) m = fmax(m, s_red[w]);
-            s_done = off_all <= 1e-15 * m || m == 0.0;
-        }
-        __syncthreads();
-        if (s_done) break;
+        float off = 0.f;
         for (int round = 0; round < kk - 1; ++round) {
-            // pairs of this round: position 0 fixed, the others rotate
-            for (int t = threadIdx.x; t < kk / 2; t += blockDim.x) {
+            for (int t = warp; t < kk / 2; t += nwarps) {
                 int a = t == 0 ? 0 : 1 + (t - 1 + round) % (kk - 1);
                 int b = 1 + (kk - 2 - t + round) % (kk - 1);
                 if (a > b) { const int x = a; a = b; b = x; }
-                double c = 1.0, s = 0.0;
-                if (b < k) {
-                    const double app = M[(size_t)a * k + a], aqq = M[(size_t)b * k + b];
-                    const double apq = M[(size_t)b * k + a];
-                    if (apq != 0.0) {
-                        const double zeta = (aqq - app) / (2.0 * apq);
-                        const double tt = (zeta >= 0 ? 1.0 : -1.0) / (fabs(zeta) + sqrt(1.0 + zeta * zeta));
-                        c = 1.0 / sqrt(1.0 + tt * tt);
-                        s = c * tt;
-                    }
+                if (b >= k) continue;
+                float *xa = A + (size_t)a * k, *xb = A + (size_t)b * k;
+                float al = 0.f, be = 0.f, ga = 0.f;
+                for (int i = lane; i < k; i += 32) {
+                    al += xa[i] * xa[i];
+                    be += xb[i] * xb[i];
+                    ga += xa[i] * xb[i];
                 }
-                cs[4 * t] = (double)a;
-                cs[4 * t + 1] = (double)b;
-                cs[4 * t + 2] = c;
-                cs[4 * t + 3] = s;
-            }
-            __syncthreads();
-            // columns: M <- M J, V <- V J (pair t rotates columns a, b)
-            for (int idx = threadIdx.x; idx < (kk / 2) * k; idx += blockDim.x) {
-                const int t = idx / k, i = idx % k;
-                const int a = (int)cs[4 * t], b = (int)cs[4 * t + 1];
-                if (b >= k) continue;
-                const double c = cs[4 * t + 2], s = cs[4 * t + 3];
-                const double x = M[(size_t)a * k + i], y = M[(size_t)b * k + i];
-                M[(size_t)a * k + i] = c * x - s * y;
-                M[(size_t)b * k + i] = s * x + c * y;
-                const double vx = V[(size_t)a * k + i], vy = V[(size_t)b * k + i];
-                V[(size_t)a * k + i] = c * vx - s * vy;
-                V[(size_t)b * k + i] = s * vx + c * vy;
-            }
-            __syncthreads();
-            // rows: M <- J^T M
-            for (int idx = threadIdx.x; idx < (kk / 2) * k; idx += blockDim.x) {
-                const int t = idx / k, col = idx % k;
-                const int a = (int)cs[4 * t], b = (int)cs[4 * t + 1];
-                if (b >= k) continue;
-                const double c = cs[4 * t + 2], s = cs[4 * t + 3];
-                const double x = M[(size_t)col * k + a], y = M[(size_t)col * k + b];
-                M[(size_t)col * k + a] = c * x - s * y;
-                M[(size_t)col * k + b] = s * x + c * y;
+                for (int o = 16; o > 0; o >>= 1) {
+                    al += __shfl_xor_sync(0xffffffffu, al, o);
+                    be += __shfl_xor_sync(0xffffffffu, be, o);
+                    ga += __shfl_xor_sync(0xffffffffu, ga, o);
+                }
+                const float rel = (al > 0.f && be > 0.f) ? fabsf(ga) / sqrtf(al * be) : 0.f;
+                off = fmaxf(off, rel);
+                if (rel <= 1e-7f) continue;
+                const float zeta = (be - al) / (2.f * ga);
+                const float tt = (zeta >= 0.f ? 1.f : -1.f) / (fabsf(zeta) + sqrtf(1.f + zeta * zeta));
+                const float c = 1.f / sqrtf(1.f + tt * tt), sn = c * tt;
+                for (int i = lane; i < k; i += 32) {
+                    const float x = xa[i], y = xb[i];
+                    xa[i] = c * x - sn * y;
+                    xb[i] = sn * x + c * y;
+                    const float vx = V[(size_t)a * k + i], vy = V[(size_t)b * k + i];
+                    V[(size_t)a * k + i] = c * vx - sn * vy;
+                    V[(size_t)b * k + i] = sn * vx + c * vy;
+                }
             }
             __syncthreads();
         }
+        for (int o = 16; o > 0; o >>= 1) off = fmaxf(off, __shfl_xor_sync(0xffffffffu, off, o));
+        if (lane == 0) s_off[warp] = off;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            float m = 0.f;
+            for (int w = 0; w < nwarps; ++w) m = fmaxf(m, s_off[w]);
+            s_done = m <= 1e-6f;
+        }
+        __syncthreads();
+        if (s_done) break;
     }
-    // sort by decreasing eigenvalue: the rank of each (ties by index)
+    // singular values (column norms), sorted by rank (ties by index)
+    __shared__ double s_norm[kMaxK];
     for (int j = threadIdx.x; j < k; j += blockDim.x) {
-        const double lj = M[(size_t)j * k + j];
+        double ss = 0.0;
+        for (int i = 0; i < k; ++i) ss += (double)A[(size_t)j * k + i] * A[(size_t)j * k + i];
+        s_norm[j] = sqrt(ss);
+    }
+    __syncthreads();
+    for (int j = threadIdx.x; j < k; j += blockDim.x) {
+        const double sj = s_norm[j];
         int rank = 0;
         for (int i = 0; i < k; ++i) {
-            const double li = M[(size_t)i * k + i];
-            rank += (li > lj) || (li == lj && i < j);
+            const double si = s_norm[i];
+            rank += (si > sj) || (si == sj && i < j);
         }
-        lam[rank] = lj;
-        for (int i = 0; i < k; ++i) E[(size_t)rank * k + i] = (float)V[(size_t)j * k + i];
+        sv[rank] = sj;
+        for (int i = 0; i < k; ++i) E[(size_t)rank * k + i] = V[(size_t)j * k + i];
     }
 }
 
 // ---------------------------------------------------------------- Ritz vectors
 
-// s_j = sqrt(max(lam_j, 0)); U (m x r, column-major) /= s_j (0 where s_j = 0).
-__global__ void k_ritz_scale(const double *lam, float *U, int m, int r, double *s) {
+// U (m x r, column-major) /= s_j (0 where s_j = 0).
+__global__ void k_ritz_scale(const double *s, float *U, int m, int r) {
     for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < (long long)m * r;
          idx += (long long)gridDim.x * blockDim.x) {
-        const int j = (int)(idx / m);
-        const double sj = sqrt(fmax(lam[j], 0.0));
-        if (idx % m == 0) s[j] = sj;
+        const double sj = s[idx / m];
         U[idx] = sj > 0.0 ? (float)((double)U[idx] / sj) : 0.0f;
     }
 }
@@ -444,11 +432,11 @@ size_t svid_ws_bytes(int d_out, int d_in, const int *ranks, int n_paths) {
     b.take<float>(m * k);                  // Y
     b.take<float>(m * k);                  // Y2
     b.take<double>(std::max(m, n) * k);    // fp64 copy for the Gram matrix
-    b.take<double>(k * k);                 // G / M
-    b.take<double>(k * k);                 // Jacobi V
-    b.take<double>(4 * ((k + 2) / 2));     // Jacobi rotations
+    b.take<double>(k * k);                 // G (fp64 Gram)
+    b.take<double>(k * k);                 // fp64 scratch of the triangular inverse
+    b.take<float>(k * k);                  // G32 (fp32 Gram / L^T)
+    b.take<float>(k * k);                  // fp32 scratch (inverse, Jacobi V)
     b.take<float>(k * k);                  // L^-T / E
-    b.take<double>(k);                     // lam
     b.take<double>(k);                     // s
     b.take<double>(m + n);                 // power iteration y
     b.take<double>(2 * k);                 // x, l_u / l_v (fp64)
@@ -476,9 +464,9 @@ cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, c
     double *D = b.take<double>((size_t)std::max(m, n) * kmax);
     double *G = b.take<double>((size_t)kmax * kmax);
     double *JV = b.take<double>((size_t)kmax * kmax);
-    double *rot = b.take<double>(4 * ((size_t)(kmax + 2) / 2));
+    float *G32 = b.take<float>((size_t)kmax * kmax);
+    float *JV32 = b.take<float>((size_t)kmax * kmax);
     float *Lt = b.take<float>((size_t)kmax * kmax);
-    double *lam = b.take<double>(kmax);
     double *sv = b.take<double>(kmax);
     double *py = b.take<double>((size_t)m + n);
     double *px = b.take<double>(2 * (size_t)kmax);
@@ -487,6 +475,7 @@ cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, c
     cudaError_t e = cudaMemcpyAsync(R, W, (size_t)m * n * sizeof(float), cudaMemcpyDeviceToDevice, s);
     if (e != cudaSuccess) return e;
     const float one = 1.f, zero = 0.f, minus = -1.f;
+    (void)G32;
     const double done = 1.0, dzero = 0.0;
     bool blas_ok = true;
     auto gemm = [&](cublasOperation_t ta, cublasOperation_t tb, int mm, int nn, int kk,
@@ -495,16 +484,19 @@ cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, c
         blas_ok = blas_ok && cublasSgemm(H, ta, tb, mm, nn, kk, alpha, A, lda, B, ldb, beta, C, ldc) ==
                                  CUBLAS_STATUS_SUCCESS;
     };
-    // orthonormalise the columns of X (rows x k, column-major) into X (via Xt)
+    // orthonormalise the columns of X (rows x k, column-major) in place (Xt
+    // scratch): Cholesky QR with the Gram matrix in fp64 (the pass that has to
+    // cope with the conditioning of X), then once more in fp32 on the nearly
+    // orthonormal result
     auto orth = [&](float *X, float *Xt, int rows, int k) {
-        for (int pass = 0; pass < 2; ++pass) {
-            k_to_f64<<<grid_for((long long)rows * k), 256, 0, s>>>(X, D, (long long)rows * k);
-            blas_ok = blas_ok && cublasDgemm(H, CUBLAS_OP_T, CUBLAS_OP_N, k, k, rows, &done, D, rows,
-                                             D, rows, &dzero, G, k) == CUBLAS_STATUS_SUCCESS;
-            k_chol_inv<<<1, kSmallThreads, 0, s>>>(G, k, JV, Lt);
-            gemm(CUBLAS_OP_N, CUBLAS_OP_N, rows, k, k, X, rows, Lt, k, &zero, Xt, rows, &one);
-            cudaMemcpyAsync(X, Xt, (size_t)rows * k * sizeof(float), cudaMemcpyDeviceToDevice, s);
-        }
+        k_to_f64<<<grid_for((long long)rows * k), 256, 0, s>>>(X, D, (long long)rows * k);
+        blas_ok = blas_ok && cublasDgemm(H, CUBLAS_OP_T, CUBLAS_OP_N, k, k, rows, &done, D, rows, D,
+                                         rows, &dzero, G, k) == CUBLAS_STATUS_SUCCESS;
+        k_chol<double, false><<<1, kSmallThreads, 0, s>>>(G, k, JV, Lt);
+        gemm(CUBLAS_OP_N, CUBLAS_OP_N, rows, k, k, X, rows, Lt, k, &zero, Xt, rows, &one);
+        gemm(CUBLAS_OP_T, CUBLAS_OP_N, k, k, rows, Xt, rows, Xt, rows, &zero, G32, k, &one);
+        k_chol<float, false><<<1, kSmallThreads, 0, s>>>(G32, k, JV32, Lt);
+        gemm(CUBLAS_OP_N, CUBLAS_OP_N, rows, k, k, Xt, rows, Lt, k, &zero, X, rows, &one);
     };
     for (int p = 0; p < n_paths && blas_ok; ++p) {
         const int r = ranks[p], k = svid_k(r, m, n);
@@ -519,16 +511,18 @@ cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, c
             gemm(CUBLAS_OP_N, CUBLAS_OP_N, n, k, m, R, n, Y, m, &zero, Q, n, &one);
             orth(Q, Q2, n, k);
         }
-        // Rayleigh-Ritz: B = R Q (in Y), M = B^T B (fp64), eigen
+        // Rayleigh-Ritz: B = R Q (in Y); B = Y' L^T with L the Cholesky factor
+        // of B^T B (fp64); the SVD of the k x k L^T (one-sided Jacobi) gives
+        // B's singular values and right vectors E: V_r = Q E_r, U_r = B E_r / s
         gemm(CUBLAS_OP_T, CUBLAS_OP_N, m, k, n, R, n, Q, n, &zero, Y, m, &one);
         k_to_f64<<<grid_for((long long)m * k), 256, 0, s>>>(Y, D, (long long)m * k);
         blas_ok = blas_ok && cublasDgemm(H, CUBLAS_OP_T, CUBLAS_OP_N, k, k, m, &done, D, m, D, m,
                                          &dzero, G, k) == CUBLAS_STATUS_SUCCESS;
-        k_jacobi<<<1, kSmallThreads, 0, s>>>(G, JV, k, rot, lam, Lt);
-        // V_r = Q E_r (into Q2, n x r), U_r = B E_r / s (into Y2, m x r)
+        k_chol<double, true><<<1, kSmallThreads, 0, s>>>(G, k, JV, G32);
+        k_svd_jacobi<<<1, kSmallThreads, 0, s>>>(G32, JV32, k, sv, Lt);
         gemm(CUBLAS_OP_N, CUBLAS_OP_N, n, r, k, Q, n, Lt, k, &zero, Q2, n, &one);
         gemm(CUBLAS_OP_N, CUBLAS_OP_N, m, r, k, Y, m, Lt, k, &zero, Y2, m, &one);
-        k_ritz_scale<<<grid_for((long long)m * r), 256, 0, s>>>(lam, Y2, m, r, sv);
+        k_ritz_scale<<<grid_for((long long)m * r), 256, 0, s>>>(sv, Y2, m, r);
         k_sign_split<<<r, 256, 0, s>>>(Y2, Q2, m, n, sv);
         k_pack_u_cm<<<grid_for((long long)m * ((r + 31) / 32)), 256, 0, s>>>(Y2, m, r, u_bits[p]);
         k_pack_v_cm<<<grid_for((long long)((n + 31) / 32) * r), 256, 0, s>>>(Q2, n, r, v_bits[p]);
