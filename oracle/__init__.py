@@ -88,6 +88,11 @@ def _bind(lib):
     lib.lbo_dual_svid_path.restype = ctypes.c_int
     lib.lbo_path_weight.argtypes = [vp, vp, vp, vp, vp, i64, i64, i64, vp]
     lib.lbo_path_weight.restype = None
+    lib.lbo_train_forward.argtypes = [ctypes.POINTER(TrainLinear), vp, i64, vp, ctypes.c_int]
+    lib.lbo_train_forward.restype = ctypes.c_int
+    lib.lbo_train_backward.argtypes = [ctypes.POINTER(TrainLinear), vp, vp, i64, d, ctypes.c_int,
+                                       ctypes.POINTER(TrainGrad), vp]
+    lib.lbo_train_backward.restype = ctypes.c_int
     lib.lbo_stack_forward.argtypes = [ctypes.POINTER(Linear), ctypes.c_int32, ctypes.c_int32,
                                       vp, vp, vp, vp]
     lib.lbo_stack_forward.restype = ctypes.c_int
@@ -130,6 +135,38 @@ class _Holder:
                 "l": _c(P["l"], np.uint16),
                 "h": _c(P["h"], np.uint16),
             }
+            self.keep.append(arrs)
+            cp = self.c.path[p]
+            cp.r = int(P["r"])
+            for k, a in arrs.items():
+                setattr(cp, k, _ptr(a))
+
+
+class TrainPath(ctypes.Structure):
+    _fields_ = [("r", ctypes.c_int32), ("u", ctypes.c_void_p), ("v", ctypes.c_void_p),
+                ("g", ctypes.c_void_p), ("l", ctypes.c_void_p), ("h", ctypes.c_void_p)]
+
+
+class TrainLinear(ctypes.Structure):
+    _fields_ = [("d_in", ctypes.c_int32), ("d_out", ctypes.c_int32), ("n_paths", ctypes.c_int32),
+                ("path", TrainPath * 2)]
+
+
+class TrainGrad(ctypes.Structure):
+    _fields_ = [("du", ctypes.c_void_p), ("dv", ctypes.c_void_p), ("dg", ctypes.c_void_p),
+                ("dl", ctypes.c_void_p), ("dh", ctypes.c_void_p)]
+
+
+class _TrainHolder:
+    """Keeps the fp64 arrays referenced by a ctypes TrainLinear alive."""
+
+    def __init__(self, layer: dict):
+        self.keep = []
+        self.c = TrainLinear()
+        self.c.d_in, self.c.d_out = int(layer["d_in"]), int(layer["d_out"])
+        self.c.n_paths = len(layer["paths"])
+        for p, P in enumerate(layer["paths"]):
+            arrs = {k: _c(P[k], np.float64) for k in ("u", "v", "g", "l", "h")}
             self.keep.append(arrs)
             cp = self.c.path[p]
             cp.r = int(P["r"])
@@ -314,6 +351,38 @@ class Oracle:
                                      l16.astype(np.float64))
         return {"d_in": W.shape[1], "d_out": W.shape[0], "paths": paths, "signs": signs}
 
+    # ------------------------------------------------------------ QAT with SmoothSign
+    def train_forward(self, layer: dict, x: np.ndarray, relaxed: bool = False) -> np.ndarray:
+        """Y = sum_p Prop. 1 with sign(U), sign(V) of the latent factors (identity if relaxed)."""
+        hold = _TrainHolder(layer)
+        X = _c(x, np.float64)
+        Y = np.zeros((X.shape[0], layer["d_out"]))
+        if self.lib.lbo_train_forward(ctypes.byref(hold.c), _ptr(X), X.shape[0], _ptr(Y),
+                                      1 if relaxed else 0):
+            raise MemoryError("oracle train forward failed")
+        return Y
+
+    def train_backward(self, layer: dict, x: np.ndarray, dy: np.ndarray, k: float = 100.0,
+                       relaxed: bool = False):
+        """Gradients of sum(Y . dY): (list of per-path dicts du, dv, dg, dl, dh; dX)."""
+        hold = _TrainHolder(layer)
+        X, DY = _c(x, np.float64), _c(dy, np.float64)
+        T = X.shape[0]
+        grads = (TrainGrad * len(layer["paths"]))()
+        out = []
+        for p, P in enumerate(layer["paths"]):
+            r = int(P["r"])
+            g = {"du": np.zeros((layer["d_out"], r)), "dv": np.zeros((layer["d_in"], r)),
+                 "dg": np.zeros(layer["d_in"]), "dl": np.zeros(r), "dh": np.zeros(layer["d_out"])}
+            out.append(g)
+            for key, a in g.items():
+                setattr(grads[p], key, _ptr(a))
+        dX = np.zeros((T, layer["d_in"]))
+        if self.lib.lbo_train_backward(ctypes.byref(hold.c), _ptr(X), _ptr(DY), T, float(k),
+                                       1 if relaxed else 0, grads, _ptr(dX)):
+            raise MemoryError("oracle train backward failed")
+        return out, dX
+
     # ------------------------------------------------------------ accounting (App. E, I.1)
     def bpw(self, d_out: int, d_in: int, r: int, n_paths: int = 2) -> float:
         return self.lib.lbo_bpw(d_out, d_in, r, n_paths)
@@ -350,7 +419,8 @@ def _forward(name):
 
 for _name in ("half_to_double", "bf16_to_double", "pack_u", "pack_v", "unpack_u", "unpack_v",
               "forward_dense", "forward_factored", "apply_factored", "latent", "expand",
-              "svd_top", "dual_svid_path", "path_weight", "dual_svid", "stack_forward",
+              "svd_top", "dual_svid_path", "path_weight", "dual_svid", "train_forward",
+              "train_backward", "stack_forward",
               "bpw", "rank_for_bpw", "flops", "set_threads", "get_threads"):
     globals()[_name] = _forward(_name)
 del _name

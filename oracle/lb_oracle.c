@@ -636,6 +636,173 @@ void lbo_path_weight(const int8_t *usign, const int8_t *vsign, const double *h, 
 }
 
 /* ------------------------------------------------------------------------ */
+/* QAT forward / backward with SmoothSign (Sec. 4 settings, App. "SmoothSign") */
+/* ------------------------------------------------------------------------ */
+
+/* Sign of a latent entry as the forward uses it: +1 for x >= 0, else -1;
+ * with relaxed != 0 the latent value itself (the continuous relaxation used
+ * to check the gradients with respect to the sign matrices). */
+static double qat_sign(double x, int relaxed) { return relaxed ? x : (x < 0 ? -1.0 : 1.0); }
+
+/* Y = sum_p ((((X . g) S(V)) . l) S(U)^T) . h with S the sign (Prop. 1 on the
+ * latent factors).  X [T][d_in], Y [T][d_out]. */
+int lbo_train_forward(const lbo_train_linear *L, const double *X, int64_t T, double *Y, int relaxed)
+{
+    int64_t din = L->d_in, dout = L->d_out;
+    for (int64_t k = 0; k < T * dout; k++)
+        Y[k] = 0.0;
+    for (int p = 0; p < L->n_paths; p++) {
+        const lbo_train_path *P = &L->path[p];
+        int64_t r = P->r;
+        double *z = (double *)malloc((size_t)(T * r > 0 ? T * r : 1) * sizeof(double));
+        if (!z)
+            return -1;
+#pragma omp parallel for schedule(static)
+        for (int64_t tj = 0; tj < T * r; tj++) {
+            int64_t t = tj / r, j = tj % r;
+            double s = 0.0;
+            for (int64_t i = 0; i < din; i++)
+                s += X[t * din + i] * P->g[i] * qat_sign(P->v[i * r + j], relaxed);
+            z[tj] = s * P->l[j];
+        }
+#pragma omp parallel for schedule(static)
+        for (int64_t to = 0; to < T * dout; to++) {
+            int64_t t = to / dout, o = to % dout;
+            double s = 0.0;
+            for (int64_t j = 0; j < r; j++)
+                s += z[t * r + j] * qat_sign(P->u[o * r + j], relaxed);
+            Y[to] += s * P->h[o];
+        }
+        free(z);
+    }
+    return 0;
+}
+
+/* Gradients of the loss sum(Y . dY) through the forward above, by the chain
+ * rule along Prop. 1's steps, per path (a = X . g, t = a S(V), z = t . l,
+ * q = z S(U)^T, y = q . h):
+ *   dh_o = sum_t dY_to q_to          dq = dY . h
+ *   dS(U) = dq^T z                   dz = dq S(U)
+ *   dl_j = sum_t dz_tj t_tj          dt = dz . l
+ *   dS(V) = a^T dt                   da = dt S(V)^T
+ *   dg_i = sum_t da_ti X_ti          dX += da . g
+ * and through the sign by SmoothSign, d sign(x)/dx := k (1 - tanh(k x)^2)
+ * (the derivative of tanh(k x)): dU = dS(U) . k (1 - tanh^2(k U)), likewise
+ * dV.  With relaxed != 0 the sign is the identity and dU = dS(U).
+ * Outputs per path (arrays of the path's shapes, overwritten) and dX [T][d_in]
+ * (may be NULL). */
+int lbo_train_backward(const lbo_train_linear *L, const double *X, const double *dY, int64_t T,
+                       double k, int relaxed, lbo_train_grad *G, double *dX)
+{
+    int64_t din = L->d_in, dout = L->d_out;
+    if (dX)
+        for (int64_t q = 0; q < T * din; q++)
+            dX[q] = 0.0;
+    for (int p = 0; p < L->n_paths; p++) {
+        const lbo_train_path *P = &L->path[p];
+        lbo_train_grad *D = &G[p];
+        int64_t r = P->r;
+        double *t = (double *)malloc((size_t)(T * r + 1) * sizeof(double));
+        double *z = (double *)malloc((size_t)(T * r + 1) * sizeof(double));
+        double *dz = (double *)malloc((size_t)(T * r + 1) * sizeof(double));
+        double *q = (double *)malloc((size_t)(T * dout + 1) * sizeof(double));
+        double *da = (double *)malloc((size_t)(T * din + 1) * sizeof(double));
+        if (!t || !z || !dz || !q || !da) {
+            free(t);
+            free(z);
+            free(dz);
+            free(q);
+            free(da);
+            return -1;
+        }
+        /* forward intermediates */
+#pragma omp parallel for schedule(static)
+        for (int64_t tj = 0; tj < T * r; tj++) {
+            int64_t tt = tj / r, j = tj % r;
+            double s = 0.0;
+            for (int64_t i = 0; i < din; i++)
+                s += X[tt * din + i] * P->g[i] * qat_sign(P->v[i * r + j], relaxed);
+            t[tj] = s;
+            z[tj] = s * P->l[j];
+        }
+#pragma omp parallel for schedule(static)
+        for (int64_t to = 0; to < T * dout; to++) {
+            int64_t tt = to / dout, o = to % dout;
+            double s = 0.0;
+            for (int64_t j = 0; j < r; j++)
+                s += z[tt * r + j] * qat_sign(P->u[o * r + j], relaxed);
+            q[to] = s;
+        }
+        /* dh, dS(U) -> dU */
+        for (int64_t o = 0; o < dout; o++) {
+            double s = 0.0;
+            for (int64_t tt = 0; tt < T; tt++)
+                s += dY[tt * dout + o] * q[tt * dout + o];
+            D->dh[o] = s;
+        }
+#pragma omp parallel for schedule(static)
+        for (int64_t oj = 0; oj < dout * r; oj++) {
+            int64_t o = oj / r, j = oj % r;
+            double s = 0.0;
+            for (int64_t tt = 0; tt < T; tt++)
+                s += dY[tt * dout + o] * P->h[o] * z[tt * r + j];
+            double th = tanh(k * P->u[oj]);
+            D->du[oj] = relaxed ? s : s * k * (1.0 - th * th);
+        }
+        /* dz, dl, dt */
+#pragma omp parallel for schedule(static)
+        for (int64_t tj = 0; tj < T * r; tj++) {
+            int64_t tt = tj / r, j = tj % r;
+            double s = 0.0;
+            for (int64_t o = 0; o < dout; o++)
+                s += dY[tt * dout + o] * P->h[o] * qat_sign(P->u[o * r + j], relaxed);
+            dz[tj] = s;
+        }
+        for (int64_t j = 0; j < r; j++) {
+            double s = 0.0;
+            for (int64_t tt = 0; tt < T; tt++)
+                s += dz[tt * r + j] * t[tt * r + j];
+            D->dl[j] = s;
+        }
+        for (int64_t tj = 0; tj < T * r; tj++)
+            dz[tj] *= P->l[tj % r]; /* dz now holds dt */
+        /* dS(V) -> dV, da, dg, dX */
+#pragma omp parallel for schedule(static)
+        for (int64_t ij = 0; ij < din * r; ij++) {
+            int64_t i = ij / r, j = ij % r;
+            double s = 0.0;
+            for (int64_t tt = 0; tt < T; tt++)
+                s += X[tt * din + i] * P->g[i] * dz[tt * r + j];
+            double th = tanh(k * P->v[ij]);
+            D->dv[ij] = relaxed ? s : s * k * (1.0 - th * th);
+        }
+#pragma omp parallel for schedule(static)
+        for (int64_t ti = 0; ti < T * din; ti++) {
+            int64_t tt = ti / din, i = ti % din;
+            double s = 0.0;
+            for (int64_t j = 0; j < r; j++)
+                s += dz[tt * r + j] * qat_sign(P->v[i * r + j], relaxed);
+            da[ti] = s;
+        }
+        for (int64_t i = 0; i < din; i++) {
+            double s = 0.0;
+            for (int64_t tt = 0; tt < T; tt++)
+                s += da[tt * din + i] * X[tt * din + i];
+            D->dg[i] = s;
+        }
+        if (dX)
+            for (int64_t ti = 0; ti < T * din; ti++)
+                dX[ti] += da[ti] * P->g[ti % din];
+        free(t);
+        free(z);
+        free(dz);
+        free(q);
+        free(da);
+    }
+    return 0;
+}
+
+/* ------------------------------------------------------------------------ */
 /* Accounting (App. E, App. I.1)                                            */
 /* ------------------------------------------------------------------------ */
 

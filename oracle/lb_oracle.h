@@ -115,6 +115,29 @@ int lbo_dual_svid_path(const double *R, int64_t d_out, int64_t d_in, int64_t r, 
 void lbo_path_weight(const int8_t *usign, const int8_t *vsign, const double *h, const double *g,
                      const double *l, int64_t d_out, int64_t d_in, int64_t r, double *What);
 
+/* QAT (training) form of a linear: latent fp64 factors U [d_out][r],
+ * V [d_in][r] and scales, the forward using their signs (Eq. 2). */
+typedef struct {
+    int32_t r;
+    const double *u, *v, *g, *l, *h;
+} lbo_train_path;
+typedef struct {
+    int32_t d_in, d_out, n_paths;
+    lbo_train_path path[2];
+} lbo_train_linear;
+/* Gradients of one path (shapes of u, v, g, l, h). */
+typedef struct {
+    double *du, *dv, *dg, *dl, *dh;
+} lbo_train_grad;
+/* Y = sum_p Prop. 1 with S(U), S(V); S = sign (x >= 0 -> +1), or the identity
+ * when relaxed != 0.  X [T][d_in], Y [T][d_out].  0 / -1. */
+int lbo_train_forward(const lbo_train_linear *L, const double *X, int64_t T, double *Y, int relaxed);
+/* Gradients of sum(Y . dY): chain rule along Prop. 1, SmoothSign
+ * k (1 - tanh^2(k x)) through the sign (identity when relaxed).  dX may be
+ * NULL.  0 / -1. */
+int lbo_train_backward(const lbo_train_linear *L, const double *X, const double *dY, int64_t T,
+                       double k, int relaxed, lbo_train_grad *G, double *dX);
+
 /* App. E bits per weight: total parameter bits / (d_out * d_in), where each
  * path stores r*(d_out+d_in) sign bits and 16*(d_out+d_in+r) scale bits. */
 double lbo_bpw(int64_t d_out, int64_t d_in, int64_t r, int32_t n_paths);

@@ -568,6 +568,98 @@ def pin_dual_svid_vs_lapack(orc):
     assert rel(orc.path_weight(us2, vs2, h2, g2, l2), 3.0 * orc.path_weight(us, vs, h, g, l)) <= 1e-12
 
 
+# ------------------------------------------------------------------ pins: QAT backward (SmoothSign)
+
+
+def _train_layer(rng, d_in, d_out, rs, signs_only=False):
+    paths = []
+    for r in rs:
+        u = rng.standard_normal((d_out, r))
+        v = rng.standard_normal((d_in, r))
+        if signs_only:
+            u, v = np.where(u < 0, -1.0, 1.0), np.where(v < 0, -1.0, 1.0)
+        paths.append({"r": r, "u": u, "v": v, "g": 0.2 + rng.random(d_in),
+                      "l": 0.2 + rng.random(r), "h": 0.2 + rng.random(d_out)})
+    return {"d_in": d_in, "d_out": d_out, "paths": paths}
+
+
+def pin_train_forward_is_inference(orc):
+    """The training forward on latent factors equals the inference forward
+    (Prop. 1, pinned above) on their packed signs, for scales and inputs that
+    fp16 / bf16 hold exactly."""
+    rng = np.random.default_rng(28)
+    d_in, d_out, T = 64, 40, 3
+    L = _train_layer(rng, d_in, d_out, (8, 5))
+    for P in L["paths"]:
+        for key in ("g", "l", "h"):
+            P[key] = np.asarray(P[key]).astype(np.float16).astype(np.float64)
+    x = rand_x(rng, T, d_in)
+    inf = {"d_in": d_in, "d_out": d_out, "paths": [
+        {"r": P["r"], "u_words": orc.pack_u(np.where(P["u"] < 0, -1, 1).astype(np.int8)),
+         "v_words": orc.pack_v(np.where(P["v"] < 0, -1, 1).astype(np.int8)),
+         "g": half_bits(P["g"]), "l": half_bits(P["l"]), "h": half_bits(P["h"])}
+        for P in L["paths"]]}
+    assert rel(orc.train_forward(L, np_bf16(x)), orc.forward_factored(inf, x)) <= 1e-13
+
+
+def pin_train_backward_central_differences(orc):
+    """With the signs relaxed to the identity the loss sum(Y . dY) is linear in
+    every single entry of h, g, l, X, S(U) and S(V), so a central difference
+    of the forward gives each gradient entry up to rounding."""
+    rng = np.random.default_rng(29)
+    d_in, d_out, T = 24, 18, 5
+    L = _train_layer(rng, d_in, d_out, (4, 3))
+    X = rng.standard_normal((T, d_in))
+    dY = rng.standard_normal((T, d_out))
+    grads, dX = orc.train_backward(L, X, dY, relaxed=True)
+    loss = lambda LL, XX: float(np.sum(orc.train_forward(LL, XX, relaxed=True) * dY))
+    eps = 1e-3
+    for p in range(2):
+        for key, gkey in (("h", "dh"), ("g", "dg"), ("l", "dl"), ("u", "du"), ("v", "dv")):
+            arr = L["paths"][p][key]
+            for _ in range(3):
+                idx = tuple(rng.integers(0, n) for n in arr.shape)
+                old = arr[idx]
+                arr[idx] = old + eps
+                lp = loss(L, X)
+                arr[idx] = old - eps
+                lm = loss(L, X)
+                arr[idx] = old
+                fd = (lp - lm) / (2 * eps)
+                assert abs(fd - grads[p][gkey][idx]) <= 1e-8 * max(1.0, abs(fd)), (p, key, fd)
+    for _ in range(4):
+        idx = (rng.integers(0, T), rng.integers(0, d_in))
+        Xp, Xm = X.copy(), X.copy()
+        Xp[idx] += eps
+        Xm[idx] -= eps
+        fd = (loss(L, Xp) - loss(L, Xm)) / (2 * eps)
+        assert abs(fd - dX[idx]) <= 1e-8 * max(1.0, abs(fd))
+
+
+def pin_smoothsign_factor(orc):
+    """Through the sign the gradient is the sign-matrix gradient times the
+    derivative of tanh(k x), k = 100: at latent U' = S(U) . a (a > 0, so the
+    signs and the forward do not change) the backward equals the relaxed
+    backward at S(U) times a central difference of numpy's tanh at U'."""
+    rng = np.random.default_rng(30)
+    d_in, d_out, T, k = 20, 16, 4, 100.0
+    L = _train_layer(rng, d_in, d_out, (5,), signs_only=True)
+    X = rng.standard_normal((T, d_in))
+    dY = rng.standard_normal((T, d_out))
+    ref, _ = orc.train_backward(L, X, dY, k=k, relaxed=True)
+    P = L["paths"][0]
+    au = rng.uniform(0.001, 0.03, P["u"].shape)
+    av = rng.uniform(0.001, 0.03, P["v"].shape)
+    L2 = {"d_in": d_in, "d_out": d_out, "paths": [dict(P, u=P["u"] * au, v=P["v"] * av)]}
+    got, _ = orc.train_backward(L2, X, dY, k=k)
+    hstep = 1e-7
+    for lat, key in ((L2["paths"][0]["u"], "du"), (L2["paths"][0]["v"], "dv")):
+        dtanh = (np.tanh(k * (lat + hstep)) - np.tanh(k * (lat - hstep))) / (2 * hstep)
+        assert rel(got[0][key], ref[0][key] * dtanh) <= 1e-6, key
+    for key in ("dg", "dl", "dh"):
+        assert rel(got[0][key], ref[0][key]) <= 1e-13, key
+
+
 def pin_kv_cache_table4(orc):
     """Table 4: the single-path rank for each target bits per weight of a
     d_model x d_model key/value projection (rounded up to a multiple of 8)
@@ -689,5 +781,6 @@ ALL_PINS = [pin_fp16_exhaustive, pin_bf16_exhaustive, pin_pack_structured, pin_p
             pin_latent_hadamard, pin_latent_closed_forms, pin_latent_brute_force,
             pin_latent_expand_composition, pin_bpw_worked_examples, pin_theoretical_cost,
             pin_kv_cache_table4, pin_svd_top_vs_numpy, pin_dual_svid_rank1,
-            pin_dual_svid_hadamard, pin_dual_svid_vs_lapack, pin_stack_chain,
+            pin_dual_svid_hadamard, pin_dual_svid_vs_lapack, pin_train_forward_is_inference,
+            pin_train_backward_central_differences, pin_smoothsign_factor, pin_stack_chain,
             pin_stack_zero_branches, pin_stack_attention_closed_form]

@@ -60,6 +60,14 @@ MUTATIONS = [
     ("svd_sign_convention", "double sg = J[best * n + imax] < 0 ? -1.0 : 1.0;",
      "double sg = J[best * n + imax] > 0 ? -1.0 : 1.0;"),
     ("path_weight_drops_g", "What[o * d_in + i] = h[o] * acc * g[i];", "What[o * d_in + i] = h[o] * acc;"),
+    ("qat_du_drops_h", "s += dY[tt * dout + o] * P->h[o] * z[tt * r + j];",
+     "s += dY[tt * dout + o] * z[tt * r + j];"),
+    ("qat_tanh_sign", "D->du[oj] = relaxed ? s : s * k * (1.0 - th * th);",
+     "D->du[oj] = relaxed ? s : s * k * (1.0 + th * th);"),
+    ("qat_dt_drops_l", "dz[tj] *= P->l[tj % r]; /* dz now holds dt */", "dz[tj] *= 1.0;"),
+    ("qat_dg_drops_x", "s += da[tt * din + i] * X[tt * din + i];", "s += da[tt * din + i];"),
+    ("qat_dx_drops_g", "dX[ti] += da[ti] * P->g[ti % din];", "dX[ti] += da[ti];"),
+    ("qat_dl_index", "s += dz[tt * r + j] * t[tt * r + j];", "s += dz[tt * r + j] * t[tt * r + (r - 1 - j)];"),
     ("flops_factor", "return (double)n_paths * 2.0 * (double)T", "return (double)n_paths * 1.0 * (double)T"),
 ]
 
