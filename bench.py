@@ -13,14 +13,16 @@ on a bounded sample (cpu_baseline), and the SM clocks seen while timing.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                   [--layers L]
-  python bench.py --config 2|3|4|6|7 [--steps K] [--warmup W]
+  python bench.py --config 2|3|4|6|7|8 [--steps K] [--warmup W]
 
 --config times the single-linear workloads instead (one JSON line per case,
 not the bench line): 2 = 4096x4096 r64 at T = 1, 8; 3 = the FFN triple at
 r = 128, 512 and T = 1, 16, 64; 4 = prefill at T = 2048, 8192; 6 = the
 latent-state halves (littlebit_linear_latent / _expand: the 70B key
 projection at T = 1 and a 4096-token cache, 4096x4096 r512 at T = 2048);
-7 = Dual-SVID initialisation of a dense weight into two paths (ms per layer).
+7 = Dual-SVID initialisation of a dense weight into two paths (ms per layer);
+8 = one QAT step (forward + SmoothSign backward) at 2048 tokens (TFLOP/s
+against the TF32 tensor peak).
 Cases 2, 3 and the CUDA-core cases of 6 report algorithmic GB/s with L2
 flushed before every call; 4 and the tensor-core cases of 6 report TFLOP/s
 (2 flops per +-1 MAC, both paths) against the dense bf16 peak.
@@ -57,7 +59,7 @@ def parse_args():
     ap.add_argument("--layers", type=int, default=80,
                     help="stack depth (80 = the Llama2-70B workload; smaller only for profiling)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--config", type=int, choices=[2, 3, 4, 6, 7], default=None,
+    ap.add_argument("--config", type=int, choices=[2, 3, 4, 6, 7, 8], default=None,
                     help="time a single-linear workload instead of the stack")
     ap.add_argument("--only", default=None,
                     help="with --config: only the cases whose 'name:T' contains this text")
@@ -540,6 +542,51 @@ def run_config(args):
                                  "peak": fp32_peak, "unit": "TFLOP/s",
                                  "frac": flops / ms / 1e9 / fp32_peak,
                                  "peak_source": "derived: 152 SMs x 128 FP32 lanes x 2 x 1.92 GHz"}}
+            print(json.dumps(line), flush=True)
+    elif args.config == 8:
+        # one QAT step (forward + SmoothSign backward) of a LittleBit linear on
+        # latent fp32 factors, 2048 tokens (the paper's training sequence length)
+        g = torch.Generator(device=dev)
+        g.manual_seed(20250608)
+        tf32_peak = tc * 1.1 / 2.25  # measured dense bf16 x nominal TF32 / bf16 ratio
+        for name, d_in, d_out, r in (("4096x4096 r512x2", 4096, 4096, 512),
+                                     ("gate 8192->28672 r320x2", 8192, 28672, 320)):
+            T = 2048
+            if not wanted(name, T):
+                continue
+            layer = {"d_in": d_in, "d_out": d_out, "paths": [
+                {"r": r, "u": 0.02 * torch.randn((d_out, r), generator=g, device=dev),
+                 "v": 0.02 * torch.randn((d_in, r), generator=g, device=dev),
+                 "g": 0.5 + torch.rand(d_in, generator=g, device=dev),
+                 "l": 0.5 + torch.rand(r, generator=g, device=dev),
+                 "h": 0.5 + torch.rand(d_out, generator=g, device=dev)} for _ in range(2)]}
+            TL = lb.TrainLinear(layer, dev)
+            x = torch.randn((T, d_in), generator=g, device=dev)
+            dy = torch.randn((T, d_out), generator=g, device=dev)
+            ws = TL.workspace(T, dev)
+            for _ in range(3):
+                lb.train_forward(TL, x, ws=ws)
+                lb.train_backward(TL, x, dy, ws=ws)
+            torch.cuda.synchronize(dev)
+            ts = []
+            for _ in range(max(3, min(steps, 20))):
+                flush.zero_()
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record()
+                lb.train_forward(TL, x, ws=ws)
+                lb.train_backward(TL, x, dy, ws=ws)
+                e1.record()
+                torch.cuda.synchronize(dev)
+                ts.append(e0.elapsed_time(e1))
+            ms = statistics.median(ts)
+            flops = 2 * (2 * T * r * (d_in + d_out) + 2 * T * r * (3 * d_in + 2 * d_out))
+            line = {"config": 8, "case": name, "op": "qat_step", "tokens": T, "ms": ms,
+                    "tflops": flops / ms / 1e9,
+                    "roofline": {"bound": "tensor", "achieved": flops / ms / 1e9,
+                                 "peak": tf32_peak, "unit": "TFLOP/s",
+                                 "frac": flops / ms / 1e9 / tf32_peak,
+                                 "peak_source": "MEASURED_PEAKS.json bf16_tflops x 1.1/2.25 (TF32)"}}
             print(json.dumps(line), flush=True)
     elif args.config == 6:
         # latent states (KV cache compression): the 70B key projection's latent

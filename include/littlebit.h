@@ -200,6 +200,54 @@ lb_status littlebit_dual_svid(const float *W, int32_t d_out, int32_t d_in, int32
                               const lb_path_init *paths, int32_t iters, void *ws, size_t ws_bytes,
                               lb_stream_t stream);
 
+/* QAT (quantization-aware training) form of one path: the latent full-
+ * precision factors the forward binarises (Eq. 2) and fp32 scales.  All
+ * pointers are device memory, fp32, row-major. */
+typedef struct {
+    int32_t r;           /* rank, 1 <= r <= 1024 */
+    const float *u;      /* latent U, [d_out][r] */
+    const float *v;      /* latent V, [d_in][r] */
+    const float *g;      /* [d_in] */
+    const float *l;      /* [r] */
+    const float *h;      /* [d_out] */
+} lb_train_path;
+
+typedef struct {
+    int32_t d_in, d_out, n_paths;   /* n_paths 1 or 2 */
+    lb_train_path path[2];
+} lb_train_linear;
+
+/* Gradient buffers of one path (device, fp32, the shapes of u, v, g, l, h);
+ * overwritten. */
+typedef struct {
+    float *du, *dv, *dg, *dl, *dh;
+} lb_train_grad;
+
+/* Workspace bytes littlebit_train_forward / littlebit_train_backward need for
+ * T tokens (0 if the arguments are invalid). */
+size_t littlebit_train_workspace_size(const lb_train_linear *L, int64_t T);
+
+/* QAT forward: Y = sum_p Prop. 1 with U_sign = sign(U), V_sign = sign(V)
+ * (sign(0) = +1) of the latent factors.  x: fp32 [T][d_in]; y: fp32
+ * [T][d_out].  The two products per path run on the tensor cores with TF32
+ * inputs (the +-1 factors are exact; x and the latent z = l . (X . g) V_sign
+ * round to 10 mantissa bits) and fp32 accumulation.  T = 0 is a no-op. */
+lb_status littlebit_train_forward(const lb_train_linear *L, const float *x, int64_t T, float *y,
+                                  void *ws, size_t ws_bytes, lb_stream_t stream);
+
+/* QAT backward (the paper's training, SmoothSign): given dy = dLoss/dY
+ * (fp32 [T][d_out]) and the forward's input x, writes per path dLoss/dU,
+ * dLoss/dV, dLoss/dg, dLoss/dl, dLoss/dh into grads[p] (HOST array of
+ * n_paths descriptors) and dLoss/dX into dx (fp32 [T][d_in], may be NULL).
+ * Through the sign the derivative is SmoothSign's proxy
+ * d tanh(k x)/dx = k (1 - tanh^2(k x)) with k = k_smooth (the paper: 100).
+ * Five GEMM-shaped products per path on the tensor cores (TF32 inputs, fp32
+ * accumulation); the scale gradients and the SmoothSign factor are fused into
+ * the reductions that follow them. */
+lb_status littlebit_train_backward(const lb_train_linear *L, const float *x, const float *dy,
+                                   int64_t T, float k_smooth, const lb_train_grad *grads,
+                                   float *dx, void *ws, size_t ws_bytes, lb_stream_t stream);
+
 /* Workspace bytes littlebit_stack_prepare / littlebit_stack_forward need
  * (0 if the arguments are invalid). */
 size_t littlebit_stack_workspace_size(const lb_linear *lin, int32_t n_layers, int32_t head_dim);

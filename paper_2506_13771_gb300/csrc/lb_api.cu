@@ -329,6 +329,66 @@ lb_status littlebit_dual_svid(const float *W, int32_t d_out, int32_t d_in, int32
                                           ws, (cudaStream_t)stream));
 }
 
+namespace {
+lb_status check_train(const lb_train_linear *L) {
+    if (!L || L->d_in <= 0 || L->d_out <= 0 || (L->n_paths != 1 && L->n_paths != 2))
+        return LB_ERR_INVALID_ARG;
+    for (int p = 0; p < L->n_paths; ++p) {
+        const lb_train_path &P = L->path[p];
+        if (P.r < 1 || P.r > lb::kMaxRank) return LB_ERR_INVALID_ARG;
+        if (!P.u || !P.v || !P.g || !P.l || !P.h || !aligned16(P.u) || !aligned16(P.v) ||
+            !aligned16(P.g) || !aligned16(P.l) || !aligned16(P.h))
+            return LB_ERR_INVALID_ARG;
+    }
+    return LB_OK;
+}
+int train_rmax(const lb_train_linear &L) {
+    int r = 0;
+    for (int p = 0; p < L.n_paths; ++p) r = r > L.path[p].r ? r : L.path[p].r;
+    return r;
+}
+}  // namespace
+
+size_t littlebit_train_workspace_size(const lb_train_linear *L, int64_t T) {
+    if (check_train(L) != LB_OK || T < 0 || T > INT32_MAX) return 0;
+    return lb::qat_ws_bytes(L->d_in, L->d_out, train_rmax(*L), T);
+}
+
+lb_status littlebit_train_forward(const lb_train_linear *L, const float *x, int64_t T, float *y,
+                                  void *ws, size_t ws_bytes, lb_stream_t stream) {
+    lb_status st = check_train(L);
+    if (st != LB_OK) return st;
+    if (T < 0 || T > INT32_MAX) return LB_ERR_INVALID_ARG;
+    if (T == 0) return LB_OK;
+    if (!x || !y || !aligned16(x) || !aligned16(y)) return LB_ERR_INVALID_ARG;
+    if (!ws || ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) ||
+        ws_bytes < littlebit_train_workspace_size(L, T))
+        return LB_ERR_WORKSPACE;
+    return from_cuda(lb::launch_train_forward(*L, x, T, y, ws, (cudaStream_t)stream));
+}
+
+lb_status littlebit_train_backward(const lb_train_linear *L, const float *x, const float *dy,
+                                   int64_t T, float k_smooth, const lb_train_grad *grads,
+                                   float *dx, void *ws, size_t ws_bytes, lb_stream_t stream) {
+    lb_status st = check_train(L);
+    if (st != LB_OK) return st;
+    if (T < 0 || T > INT32_MAX || !grads || !(k_smooth > 0.f)) return LB_ERR_INVALID_ARG;
+    if (T == 0) return LB_OK;
+    if (!x || !dy || !aligned16(x) || !aligned16(dy) || (dx && !aligned16(dx)))
+        return LB_ERR_INVALID_ARG;
+    for (int p = 0; p < L->n_paths; ++p) {
+        const lb_train_grad &G = grads[p];
+        if (!G.du || !G.dv || !G.dg || !G.dl || !G.dh || !aligned16(G.du) || !aligned16(G.dv) ||
+            !aligned16(G.dg) || !aligned16(G.dl) || !aligned16(G.dh))
+            return LB_ERR_INVALID_ARG;
+    }
+    if (!ws || ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) ||
+        ws_bytes < littlebit_train_workspace_size(L, T))
+        return LB_ERR_WORKSPACE;
+    return from_cuda(lb::launch_train_backward(*L, x, dy, T, k_smooth, grads, dx, ws,
+                                               (cudaStream_t)stream));
+}
+
 size_t littlebit_stack_workspace_size(const lb_linear *lin, int32_t n_layers, int32_t head_dim) {
     lb::StackShape shape;
     if (check_stack(lin, n_layers, head_dim, &shape) != LB_OK) return 0;

@@ -7,7 +7,13 @@
 
 #include "littlebit.h"
 
+struct cublasContext;
+
 namespace lb {
+
+// The library's cuBLAS handle for the current device (created on first use,
+// one per device, shared by the calls that run plain GEMMs).
+cublasContext *blas_handle();
 
 struct LinDesc;
 
@@ -79,6 +85,15 @@ cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, c
                              uint32_t *const *v_bits, uint32_t *const *u_bits, uint16_t *const *g,
                              uint16_t *const *l, uint16_t *const *h, int iters, void *ws,
                              cudaStream_t s);
+
+// QAT forward / backward on latent factors (lb_qat.cu); ws: qat_ws_bytes for
+// the largest rank.
+size_t qat_ws_bytes(int d_in, int d_out, int rmax, long long T);
+cudaError_t launch_train_forward(const lb_train_linear &L, const float *x, long long T, float *y,
+                                 void *ws, cudaStream_t s);
+cudaError_t launch_train_backward(const lb_train_linear &L, const float *x, const float *dy,
+                                  long long T, float k, const lb_train_grad *G, float *dx, void *ws,
+                                  cudaStream_t s);
 
 // Bounded-wait diagnostic (lb_persistent.cu).
 cudaError_t launch_wait_timeout(unsigned *ws_words, cudaStream_t s);

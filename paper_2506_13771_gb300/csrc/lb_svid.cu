@@ -393,17 +393,6 @@ __global__ void k_what_factors(const float *U, const float *V, int d_out, int d_
 
 // ---------------------------------------------------------------- cuBLAS
 
-std::mutex g_blas_mu;
-cublasHandle_t g_blas[64];
-
-cublasHandle_t blas_handle() {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-    std::lock_guard<std::mutex> lock(g_blas_mu);
-    if (!g_blas[dev] && cublasCreate(&g_blas[dev]) != CUBLAS_STATUS_SUCCESS) g_blas[dev] = nullptr;
-    return g_blas[dev];
-}
-
 int grid_for(long long n) { return (int)std::min<long long>((n + 255) / 256, 152 * 8); }
 
 struct Buf {
@@ -418,6 +407,17 @@ struct Buf {
 };
 
 }  // namespace
+
+static std::mutex g_blas_mu;
+static cublasHandle_t g_blas[64];
+
+cublasHandle_t blas_handle() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    std::lock_guard<std::mutex> lock(g_blas_mu);
+    if (!g_blas[dev] && cublasCreate(&g_blas[dev]) != CUBLAS_STATUS_SUCCESS) g_blas[dev] = nullptr;
+    return g_blas[dev];
+}
 
 int svid_k(int r, int d_out, int d_in) { return std::min(r + kOversample, std::min(d_out, d_in)); }
 

@@ -25,6 +25,8 @@ LB_PACK_U, LB_PACK_V = 0, 1
 EXPORTED = ["littlebit_status_string", "littlebit_pack", "littlebit_workspace_size",
             "littlebit_linear_forward", "littlebit_linear_latent", "littlebit_linear_expand",
             "littlebit_dual_svid_workspace_size", "littlebit_dual_svid",
+            "littlebit_train_workspace_size", "littlebit_train_forward",
+            "littlebit_train_backward",
             "littlebit_stack_workspace_size",
             "littlebit_stack_prepare", "littlebit_stack_forward", "littlebit_poll_error",
             "littlebit_selftest_wait_timeout", "littlebit_linear_forward_noalloc"]
@@ -50,6 +52,21 @@ class lb_linear(ctypes.Structure):
                 ("d_out", ctypes.c_int32),
                 ("n_paths", ctypes.c_int32),
                 ("path", lb_path * 2)]
+
+
+class lb_train_path(ctypes.Structure):
+    _fields_ = [("r", ctypes.c_int32), ("u", ctypes.c_void_p), ("v", ctypes.c_void_p),
+                ("g", ctypes.c_void_p), ("l", ctypes.c_void_p), ("h", ctypes.c_void_p)]
+
+
+class lb_train_linear(ctypes.Structure):
+    _fields_ = [("d_in", ctypes.c_int32), ("d_out", ctypes.c_int32), ("n_paths", ctypes.c_int32),
+                ("path", lb_train_path * 2)]
+
+
+class lb_train_grad(ctypes.Structure):
+    _fields_ = [("du", ctypes.c_void_p), ("dv", ctypes.c_void_p), ("dg", ctypes.c_void_p),
+                ("dl", ctypes.c_void_p), ("dh", ctypes.c_void_p)]
 
 
 class lb_path_init(ctypes.Structure):
@@ -93,6 +110,15 @@ def lib(path: str | None = None):
         L.littlebit_dual_svid.argtypes = [vp, i32, i32, i32, ctypes.POINTER(lb_path_init), i32, vp,
                                           sz, vp]
         L.littlebit_dual_svid.restype = ctypes.c_int
+        L.littlebit_train_workspace_size.argtypes = [ctypes.POINTER(lb_train_linear), i64]
+        L.littlebit_train_workspace_size.restype = sz
+        L.littlebit_train_forward.argtypes = [ctypes.POINTER(lb_train_linear), vp, i64, vp, vp, sz,
+                                              vp]
+        L.littlebit_train_forward.restype = ctypes.c_int
+        L.littlebit_train_backward.argtypes = [ctypes.POINTER(lb_train_linear), vp, vp, i64,
+                                               ctypes.c_float, ctypes.POINTER(lb_train_grad), vp,
+                                               vp, sz, vp]
+        L.littlebit_train_backward.restype = ctypes.c_int
         L.littlebit_stack_workspace_size.argtypes = [ctypes.POINTER(lb_linear), i32, i32]
         L.littlebit_stack_workspace_size.restype = sz
         L.littlebit_stack_prepare.argtypes = [ctypes.POINTER(lb_linear), i32, i32, vp, sz, vp]
@@ -313,6 +339,68 @@ def layer_to_host(layer: dict) -> dict:
                       "l": P["l"].cpu().numpy().view(np.uint16),
                       "h": P["h"].cpu().numpy().view(np.uint16)})
     return {"d_in": layer["d_in"], "d_out": layer["d_out"], "paths": paths}
+
+
+class TrainLinear:
+    """A LittleBit linear in QAT form on the device: latent fp32 factors and scales.
+    Built from {'d_in', 'd_out', 'paths': [{'r', 'u', 'v', 'g', 'l', 'h'}]} (numpy or torch)."""
+
+    def __init__(self, layer: dict, device="cuda"):
+        self.d_in, self.d_out = int(layer["d_in"]), int(layer["d_out"])
+        self.c = lb_train_linear()
+        self.c.d_in, self.c.d_out, self.c.n_paths = self.d_in, self.d_out, len(layer["paths"])
+        self.paths, self.ranks = [], []
+        for p, P in enumerate(layer["paths"]):
+            t = {k: torch.as_tensor(np.asarray(P[k]) if not torch.is_tensor(P[k]) else P[k],
+                                    dtype=torch.float32).to(device).contiguous()
+                 for k in ("u", "v", "g", "l", "h")}
+            self.paths.append(t)
+            self.ranks.append(int(P["r"]))
+            cp = self.c.path[p]
+            cp.r = int(P["r"])
+            for k, ten in t.items():
+                setattr(cp, k, ten.data_ptr())
+
+    def workspace(self, T: int, device="cuda") -> torch.Tensor:
+        n = int(lib().littlebit_train_workspace_size(ctypes.byref(self.c), int(T)))
+        return torch.empty(max(n, 256), dtype=torch.uint8, device=device)
+
+
+def train_forward(L: TrainLinear, x: torch.Tensor, ws: torch.Tensor | None = None,
+                  stream=None) -> torch.Tensor:
+    """QAT forward (signs of the latent factors), fp32 x [T][d_in] -> y [T][d_out]."""
+    assert x.dtype == torch.float32 and x.dim() == 2 and x.shape[1] == L.d_in
+    x = x.contiguous()
+    T = x.shape[0]
+    y = torch.empty((T, L.d_out), dtype=torch.float32, device=x.device)
+    ws = ws if ws is not None else L.workspace(T, x.device)
+    _check(lib().littlebit_train_forward(ctypes.byref(L.c), x.data_ptr(), T, y.data_ptr(),
+                                         ws.data_ptr(), ws.numel(), _stream(stream)),
+           "littlebit_train_forward")
+    return y
+
+
+def train_backward(L: TrainLinear, x: torch.Tensor, dy: torch.Tensor, k: float = 100.0,
+                   want_dx: bool = True, ws: torch.Tensor | None = None, stream=None):
+    """QAT backward with SmoothSign: (per-path dicts du, dv, dg, dl, dh; dX or None)."""
+    x, dy = x.contiguous(), dy.contiguous()
+    T = x.shape[0]
+    grads = (lb_train_grad * len(L.paths))()
+    out = []
+    for p, P in enumerate(L.paths):
+        g = {"du": torch.empty_like(P["u"]), "dv": torch.empty_like(P["v"]),
+             "dg": torch.empty_like(P["g"]), "dl": torch.empty_like(P["l"]),
+             "dh": torch.empty_like(P["h"])}
+        out.append(g)
+        for key, ten in g.items():
+            setattr(grads[p], key, ten.data_ptr())
+    dx = torch.empty_like(x) if want_dx else None
+    ws = ws if ws is not None else L.workspace(T, x.device)
+    _check(lib().littlebit_train_backward(ctypes.byref(L.c), x.data_ptr(), dy.data_ptr(), T,
+                                          float(k), grads, dx.data_ptr() if want_dx else None,
+                                          ws.data_ptr(), ws.numel(), _stream(stream)),
+           "littlebit_train_backward")
+    return out, dx
 
 
 class DeviceStack:

@@ -143,6 +143,28 @@ def test_dual_svid_argument_validation(L):
     assert svid(FAKE, 256, 384, 2, arr, 8, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
 
 
+def test_train_argument_validation(L):
+    c = lb.lb_train_linear()
+    c.d_in, c.d_out, c.n_paths = 64, 32, 1
+    c.path[0].r = 8
+    c.path[0].u = c.path[0].v = c.path[0].g = c.path[0].l = c.path[0].h = FAKE
+    ref = ctypes.byref(c)
+    n = L.littlebit_train_workspace_size(ref, 16)
+    assert n > 0
+    g = (lb.lb_train_grad * 1)()
+    g[0].du = g[0].dv = g[0].dg = g[0].dl = g[0].dh = FAKE
+    fwd, bwd = L.littlebit_train_forward, L.littlebit_train_backward
+    assert fwd(ref, FAKE, 0, FAKE, FAKE, n, None) == lb.LB_OK                    # T = 0
+    assert fwd(ref, FAKE + 4, 16, FAKE, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    assert fwd(ref, FAKE, 16, FAKE, FAKE, 64, None) == lb.LB_ERR_WORKSPACE
+    assert bwd(ref, FAKE, FAKE, 16, 0.0, g, None, FAKE, n, None) == lb.LB_ERR_INVALID_ARG  # k
+    assert bwd(ref, FAKE, FAKE, 16, 100.0, None, None, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    g[0].dl = 0
+    assert bwd(ref, FAKE, FAKE, 16, 100.0, g, None, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    c.n_paths = 3
+    assert L.littlebit_train_workspace_size(ref, 16) == 0
+
+
 def fake_stack(n_layers=2, d=256, dkv=64, dff=512, rq=16, rk=8, rm=24):
     shapes = [(d, d, rq), (d, dkv, rk), (d, dkv, rk), (d, d, rq), (d, dff, rm), (d, dff, rm),
               (dff, d, rm)]

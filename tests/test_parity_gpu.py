@@ -376,6 +376,54 @@ def test_dual_svid_512x384_two_paths():
     test_dual_svid_vs_oracle(512, 384, (40, 40))
 
 
+# ------------------------------------------------------------------ QAT backward (SmoothSign)
+
+# TF32 rounds the non-sign GEMM operands to 10 mantissa bits (relative error
+# up to 2^-11 per element, about 2^-11 / sqrt(3) ~ 2.8e-4 RMS); a product
+# with two rounded operands (dY^T z, X^T dt) carries about 4e-4 relative L2.
+# fp32 accumulation adds ~1e-6.  Bar: 2e-3 relative L2 per gradient.
+TOL_TF32 = 2e-3
+
+
+def _train_case(rng, d_in, d_out, rs):
+    paths = []
+    for r in rs:
+        paths.append({"r": r,
+                      "u": (rng.standard_normal((d_out, r)) * 0.02).astype(np.float32),
+                      "v": (rng.standard_normal((d_in, r)) * 0.02).astype(np.float32),
+                      "g": (0.5 + rng.random(d_in)).astype(np.float32),
+                      "l": (0.5 + rng.random(r)).astype(np.float32),
+                      "h": (0.5 + rng.random(d_out)).astype(np.float32)})
+    return {"d_in": d_in, "d_out": d_out, "paths": paths}
+
+
+@pytest.mark.parametrize("d_in,d_out,rs,T", [(256, 192, (16, 16), 64), (512, 1024, (64,), 130),
+                                             (1000, 520, (33, 7), 37), (4096, 4096, (64, 64), 256)])
+def test_train_forward_backward_vs_oracle(d_in, d_out, rs, T):
+    """QAT forward and every gradient of the backward against the fp64 oracle
+    on the same fp32 latent factors (signs decided on identical values)."""
+    rng = inputs.rng_for(109, salt=d_in + d_out + T)
+    layer = _train_case(rng, d_in, d_out, rs)
+    x = rng.standard_normal((T, d_in)).astype(np.float32)
+    dy = rng.standard_normal((T, d_out)).astype(np.float32)
+    TL = lb.TrainLinear(layer, DEV)
+    xd, dyd = torch.from_numpy(x).to(DEV), torch.from_numpy(dy).to(DEV)
+    y = lb.train_forward(TL, xd)
+    grads, dx = lb.train_backward(TL, xd, dyd, k=100.0)
+    torch.cuda.synchronize()
+    L64 = {"d_in": d_in, "d_out": d_out,
+           "paths": [{k: (P[k].astype(np.float64) if k != "r" else P[k]) for k in P}
+                     for P in layer["paths"]]}
+    y_ref = oracle.train_forward(L64, x.astype(np.float64))
+    g_ref, dx_ref = oracle.train_backward(L64, x.astype(np.float64), dy.astype(np.float64), k=100.0)
+    assert rel(y.cpu().numpy(), y_ref) <= TOL_TF32
+    assert rel(dx.cpu().numpy(), dx_ref) <= TOL_TF32
+    for p in range(len(rs)):
+        for key in ("du", "dv", "dg", "dl", "dh"):
+            e = rel(grads[p][key].cpu().numpy(), g_ref[p][key])
+            assert e <= TOL_TF32, (p, key, e)
+
+
 # ------------------------------------------------------------------ stack
 
 
