@@ -5,8 +5,9 @@
 // W_hat of the paths before it, with their scales as stored in fp16):
 //   (1) truncated SVD R ~ U_r diag(s) V_r^T by subspace iteration: Q (d_in x k,
 //       k = r + oversampling) starts random; each iteration Y = R Q, Y = orth(Y),
-//       Q = R^T Y, Q = orth(Q), orth being Cholesky QR with the Gram matrix in
-//       fp64 followed by a second pass in fp32; then Rayleigh-Ritz: B = R Q,
+//       Q = R^T Y, Q = orth(Q), orth being Cholesky QR (X <- X L^{-T}, G = X^T X
+//       = L L^T) with the Gram matrix in fp64 followed by a second pass in
+//       fp32; then Rayleigh-Ritz: B = R Q,
 //       B = Y' L^T (L the Cholesky factor of B^T B), L^T = U_C diag(s) E^T by
 //       one-sided Jacobi (fp32, no squaring of the spectrum), V_r = Q E_r,
 //       U_r = B E_r diag(1/s).
@@ -14,12 +15,13 @@
 //   (2) U' = U_r diag(sqrt s), V' = V_r diag(sqrt s); U_sign = sign(U'),
 //       V_sign = sign(V') (sign(0) = +1), packed in the lb_path layouts.
 //   (3) |U'| ~ h l_u^T, |V'| ~ g l_v^T, the leading singular pair of each
-//       nonnegative matrix by power iteration (fp64), the singular value split
+//       nonnegative matrix by power iteration (fp64, 50 steps), the singular value split
 //       evenly; l = l_u . l_v.  h, g, l are rounded to fp16 (nearest even).
-// The GEMMs are cuBLAS (plain fp32 / fp64 GEMMs); the small dense problems
-// (Cholesky and triangular inverse of a k x k Gram matrix, the k x k Jacobi
-// SVD) run in one CTA each; the rest are elementwise / reduction kernels
-// below.
+// The GEMMs are cuBLAS (plain fp32 / fp64 GEMMs); the Cholesky factor of
+// a k x k Gram matrix and the triangular solve with it are blocked (64-wide
+// diagonal blocks in one CTA each, rows below by many CTAs, updates by GEMM);
+// the k x k Jacobi SVD runs in one CTA; the rest are elementwise / reduction
+// kernels below.
 #include <cublas_v2.h>
 
 #include <algorithm>
@@ -35,7 +37,7 @@ namespace lb {
 namespace {
 
 constexpr int kOversample = 8;
-constexpr int kPowerIters = 100;  // rank-1 power iterations on |U'|, |V'|
+constexpr int kPowerIters = 50;  // rank-1 power iterations on |U'|, |V'|
 constexpr int kJacobiSweeps = 40;
 constexpr int kSmallThreads = 1024;
 constexpr int kMaxK = 1024 + 16;  // rank + oversampling
@@ -82,61 +84,112 @@ __global__ void k_to_f64(const float *a, double *b, long long n) {
 
 // ---------------------------------------------------------------- Cholesky QR
 
-// G (k x k, column-major, symmetric positive semidefinite, type T) ->
-// FACTOR ? Lt = L^T : Lt = (L^{-1})^T (fp32, k x k column-major) where
-// G = L L^T, so that Y (L^{-1})^T has orthonormal columns when G = Y^T Y.
-// One CTA; X (k x k, T) is scratch for L^{-1}.  A pivot at or below 1e-14
-// (fp64) / 1e-6 (fp32) of the mean diagonal (a column of Y in the span of the
-// previous ones, or Y = 0) is set to zero, and so are the entries of L below
-// it and of L^{-1} that depend on it: that column of Y maps to zero instead
-// of blowing up.
-template <typename T, bool FACTOR>
-__global__ void __launch_bounds__(kSmallThreads) k_chol(T *G, int k, T *X, float *Lt) {
-    __shared__ T s_piv;
-    T trace = 0;
-    for (int j = 0; j < k; ++j) trace += G[(size_t)j * k + j];
-    const T floor_piv = (sizeof(T) == 8 ? (T)1e-14 : (T)1e-6) * (trace > 0 ? trace : 0) / k;
-    // Cholesky in place: L(i, j) at G[j * k + i], i >= j
-    for (int j = 0; j < k; ++j) {
-        if (threadIdx.x == 0) {
-            T d = G[(size_t)j * k + j];
-            for (int p = 0; p < j; ++p) d -= G[(size_t)p * k + j] * G[(size_t)p * k + j];
-            s_piv = d > floor_piv && d > 0 ? sqrt(d) : 0;
-            G[(size_t)j * k + j] = s_piv;
+// ---------------------------------------------------------------- blocked Cholesky
+
+constexpr int kNB = 64;  // block width of the blocked Cholesky / triangular solve
+
+// floor = eps_rel * trace(G) / k (one block): pivots at or below it count as zero.
+template <typename T>
+__global__ void k_pivot_floor(const T *G, int k, T eps_rel, T *floor_out) {
+    T acc = 0;
+    for (int j = threadIdx.x; j < k; j += blockDim.x) acc += G[(size_t)j * k + j];
+    __shared__ T s_part[32];
+    for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if ((threadIdx.x & 31) == 0) s_part[threadIdx.x >> 5] = acc;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        T t = 0;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += s_part[w];
+        *floor_out = eps_rel * (t > 0 ? t : 0) / k;
+    }
+}
+
+// Factor the diagonal block G[jb:jb+b, jb:jb+b] (already updated by the
+// blocks to its left) in place, lower triangle, in shared memory; one CTA of
+// kNB threads.  A pivot at or below *floor becomes 0, and so does the column
+// below it.
+template <typename T>
+__global__ void __launch_bounds__(kNB) k_potrf_diag(T *G, int k, int jb, int b, const T *floor_p) {
+    __shared__ T a[kNB][kNB + 1];
+    const int c = threadIdx.x;
+    for (int i = 0; i < b; ++i)
+        if (c < b) a[i][c] = G[(size_t)(jb + c) * k + jb + i];
+    __syncthreads();
+    const T fl = *floor_p;
+    for (int j = 0; j < b; ++j) {
+        if (c == 0) {
+            T d = a[j][j];
+            for (int p = 0; p < j; ++p) d -= a[j][p] * a[j][p];
+            a[j][j] = d > fl && d > 0 ? sqrt(d) : 0;
         }
         __syncthreads();
-        const T piv = s_piv;
-        for (int i = j + 1 + threadIdx.x; i < k; i += blockDim.x) {
-            T a = G[(size_t)j * k + i];
-            for (int p = 0; p < j; ++p) a -= G[(size_t)p * k + i] * G[(size_t)p * k + j];
-            G[(size_t)j * k + i] = piv > 0 ? a / piv : 0;
+        const T piv = a[j][j];
+        if (c > j && c < b) {
+            T v = a[c][j];
+            for (int p = 0; p < j; ++p) v -= a[c][p] * a[j][p];
+            a[c][j] = piv > 0 ? v / piv : 0;
         }
         __syncthreads();
     }
-    if (FACTOR) {
-        // Lt(c, i) = L(i, c) for i >= c, else 0
-        for (int idx = threadIdx.x; idx < k * k; idx += blockDim.x) {
-            const int i = idx / k, c = idx % k;  // Lt column i, row c
-            Lt[idx] = i >= c ? (float)G[(size_t)c * k + i] : 0.f;
-        }
-        return;
+    for (int i = 0; i < b; ++i)
+        if (c < b && c <= i) G[(size_t)(jb + c) * k + jb + i] = a[i][c];
+}
+
+// Panel rows i in [jb+b, k): L[i, jb:jb+b] = G[i, jb:jb+b] L_jj^{-T}, one
+// thread per row, L_jj in shared memory (column-major G).
+template <typename T>
+__global__ void k_trsm_panel(T *G, int k, int jb, int b) {
+    __shared__ T l[kNB][kNB + 1];
+    for (int idx = threadIdx.x; idx < b * b; idx += blockDim.x) {
+        const int i = idx / b, j = idx % b;
+        l[i][j] = j <= i ? G[(size_t)(jb + j) * k + jb + i] : 0;
     }
-    // column c of L^{-1} by forward substitution (one thread per column):
-    // x_i = (delta_ic - sum_{c <= p < i} L(i, p) x_p) / L(i, i), x in X[c * k + .];
-    // Lt(c, i) = L^{-1}(i, c) goes to Lt[i * k + c]
-    for (int c = threadIdx.x; c < k; c += blockDim.x) {
-        T *x = X + (size_t)c * k;
-        for (int i = 0; i < k; ++i) {
-            T xi = 0;
-            if (i >= c) {
-                T a = (i == c) ? 1 : 0;
-                for (int p = c; p < i; ++p) a -= G[(size_t)p * k + i] * x[p];
-                const T piv = G[(size_t)i * k + i];
-                xi = piv > 0 ? a / piv : 0;
-            }
-            x[i] = xi;
-            Lt[(size_t)i * k + c] = (float)xi;
-        }
+    __syncthreads();
+    const int i = jb + b + blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= k) return;
+    T x[kNB];
+#pragma unroll 4
+    for (int j = 0; j < kNB; ++j) {
+        if (j >= b) break;
+        T v = G[(size_t)(jb + j) * k + i];
+        for (int p = 0; p < j; ++p) v -= x[p] * l[j][p];
+        x[j] = l[j][j] > 0 ? v / l[j][j] : 0;
+        G[(size_t)(jb + j) * k + i] = x[j];
+    }
+}
+
+// In-place rows of X (rows x k column-major, fp32): columns jb:jb+b solved
+// against L_jj^T, x L_jj^T = y, one thread per row (the columns left of jb
+// have been subtracted by a GEMM already).  L is fp32 column-major k x k.
+__global__ void k_trsm_cols(float *X, int rows, const float *L, int k, int jb, int b) {
+    __shared__ float l[kNB][kNB + 1];
+    for (int idx = threadIdx.x; idx < b * b; idx += blockDim.x) {
+        const int i = idx / b, j = idx % b;
+        l[i][j] = j <= i ? L[(size_t)(jb + j) * k + jb + i] : 0.f;
+    }
+    __syncthreads();
+    const int row = blockIdx.x * blockDim.x + threadIdx.x;
+    if (row >= rows) return;
+    float x[kNB];
+#pragma unroll 4
+    for (int j = 0; j < kNB; ++j) {
+        if (j >= b) break;
+        float v = X[(size_t)(jb + j) * rows + row];
+        for (int p = 0; p < j; ++p) v -= x[p] * l[j][p];
+        x[j] = l[j][j] > 0.f ? v / l[j][j] : 0.f;
+        X[(size_t)(jb + j) * rows + row] = x[j];
+    }
+}
+
+// fp32 copy of the lower triangle of G (zeros above), column-major; with
+// transpose, Lt = L^T instead.
+template <typename T>
+__global__ void k_lower_f32(const T *G, int k, float *L, int transpose) {
+    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < (long long)k * k;
+         idx += (long long)gridDim.x * blockDim.x) {
+        const int c = (int)(idx / k), i = (int)(idx % k);  // column c, row i of the output
+        const int gi = transpose ? c : i, gc = transpose ? i : c;  // element (gi, gc) of L
+        L[idx] = gi >= gc ? (float)G[(size_t)gc * k + gi] : 0.f;
     }
 }
 
@@ -151,8 +204,9 @@ __global__ void __launch_bounds__(kSmallThreads) k_chol(T *G, int k, T *X, float
 // t^2 + 2 zeta t - 1 = 0, zeta = (beta - alpha) / (2 gamma), and
 // x' = c x - s y, y' = s x + c y.  Outputs s (k, decreasing, fp64) and the
 // right singular vectors E (fp32, k x k column-major, column j for s[j]).
-// Sweeps stop when no pair of a sweep is more than 1e-6 from orthogonal (or
-// after kJacobiSweeps).  One CTA; V is fp32 scratch (k x k).
+// Pairs within 1e-6 of orthogonal are left alone; sweeps stop when no pair
+// of a sweep is more than 4e-6 from orthogonal (fp32 dot products of length
+// k carry ~sqrt(k) 6e-8 of noise) or after kJacobiSweeps.  One CTA; V is fp32 scratch (k x k).
 __global__ void __launch_bounds__(kSmallThreads) k_svd_jacobi(float *A, float *V, int k, double *sv,
                                                               float *E) {
     __shared__ float s_off[32];
@@ -184,7 +238,7 @@ __global__ void __launch_bounds__(kSmallThreads) k_svd_jacobi(float *A, float *V
                 }
                 const float rel = (al > 0.f && be > 0.f) ? fabsf(ga) / sqrtf(al * be) : 0.f;
                 off = fmaxf(off, rel);
-                if (rel <= 1e-7f) continue;
+                if (rel <= 1e-6f) continue;
                 const float zeta = (be - al) / (2.f * ga);
                 const float tt = (zeta >= 0.f ? 1.f : -1.f) / (fabsf(zeta) + sqrtf(1.f + zeta * zeta));
                 const float c = 1.f / sqrtf(1.f + tt * tt), sn = c * tt;
@@ -205,7 +259,7 @@ __global__ void __launch_bounds__(kSmallThreads) k_svd_jacobi(float *A, float *V
         if (threadIdx.x == 0) {
             float m = 0.f;
             for (int w = 0; w < nwarps; ++w) m = fmaxf(m, s_off[w]);
-            s_done = m <= 1e-6f;
+            s_done = m <= 4e-6f;
         }
         __syncthreads();
         if (s_done) break;
@@ -433,10 +487,9 @@ size_t svid_ws_bytes(int d_out, int d_in, const int *ranks, int n_paths) {
     b.take<float>(m * k);                  // Y2
     b.take<double>(std::max(m, n) * k);    // fp64 copy for the Gram matrix
     b.take<double>(k * k);                 // G (fp64 Gram)
-    b.take<double>(k * k);                 // fp64 scratch of the triangular inverse
     b.take<float>(k * k);                  // G32 (fp32 Gram / L^T)
-    b.take<float>(k * k);                  // fp32 scratch (inverse, Jacobi V)
-    b.take<float>(k * k);                  // L^-T / E
+    b.take<float>(k * k);                  // fp32 scratch (Jacobi V)
+    b.take<float>(k * k);                  // L (fp32) / E
     b.take<double>(k);                     // s
     b.take<double>(m + n);                 // power iteration y
     b.take<double>(2 * k);                 // x, l_u / l_v (fp64)
@@ -463,7 +516,6 @@ cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, c
     float *Y2 = b.take<float>((size_t)m * kmax);
     double *D = b.take<double>((size_t)std::max(m, n) * kmax);
     double *G = b.take<double>((size_t)kmax * kmax);
-    double *JV = b.take<double>((size_t)kmax * kmax);
     float *G32 = b.take<float>((size_t)kmax * kmax);
     float *JV32 = b.take<float>((size_t)kmax * kmax);
     float *Lt = b.take<float>((size_t)kmax * kmax);
@@ -484,19 +536,65 @@ cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, c
         blas_ok = blas_ok && cublasSgemm(H, ta, tb, mm, nn, kk, alpha, A, lda, B, ldb, beta, C, ldc) ==
                                  CUBLAS_STATUS_SUCCESS;
     };
-    // orthonormalise the columns of X (rows x k, column-major) in place (Xt
-    // scratch): Cholesky QR with the Gram matrix in fp64 (the pass that has to
-    // cope with the conditioning of X), then once more in fp32 on the nearly
-    // orthonormal result
-    auto orth = [&](float *X, float *Xt, int rows, int k) {
+    // blocked Cholesky of the k x k Gram matrix Gm (lower, in place): per
+    // 64-wide block, the diagonal block in one CTA, the rows below it by a
+    // triangular solve, the trailing matrix by a GEMM
+    double *dfloor = reinterpret_cast<double *>(nrm + 2);
+    float *ffloor = reinterpret_cast<float *>(nrm + 3);
+    auto chol64 = [&](double *Gm, int k) {
+        k_pivot_floor<double><<<1, 256, 0, s>>>(Gm, k, 1e-14, dfloor);
+        for (int jb = 0; jb < k; jb += kNB) {
+            const int bw = std::min(kNB, k - jb), rest = k - jb - bw;
+            k_potrf_diag<double><<<1, kNB, 0, s>>>(Gm, k, jb, bw, dfloor);
+            if (rest > 0) {
+                k_trsm_panel<double><<<(rest + 127) / 128, 128, 0, s>>>(Gm, k, jb, bw);
+                const double dminus = -1.0;
+                blas_ok = blas_ok &&
+                          cublasDgemm(H, CUBLAS_OP_N, CUBLAS_OP_T, rest, rest, bw, &dminus,
+                                      Gm + (size_t)jb * k + jb + bw, k, Gm + (size_t)jb * k + jb + bw,
+                                      k, &done, Gm + (size_t)(jb + bw) * k + jb + bw, k) ==
+                              CUBLAS_STATUS_SUCCESS;
+            }
+        }
+    };
+    auto chol32 = [&](float *Gm, int k) {
+        k_pivot_floor<float><<<1, 256, 0, s>>>(Gm, k, 1e-6f, ffloor);
+        for (int jb = 0; jb < k; jb += kNB) {
+            const int bw = std::min(kNB, k - jb), rest = k - jb - bw;
+            k_potrf_diag<float><<<1, kNB, 0, s>>>(Gm, k, jb, bw, ffloor);
+            if (rest > 0) {
+                k_trsm_panel<float><<<(rest + 127) / 128, 128, 0, s>>>(Gm, k, jb, bw);
+                gemm(CUBLAS_OP_N, CUBLAS_OP_T, rest, rest, bw, Gm + (size_t)jb * k + jb + bw, k,
+                     Gm + (size_t)jb * k + jb + bw, k, &one, Gm + (size_t)(jb + bw) * k + jb + bw,
+                     k, &minus);
+            }
+        }
+    };
+    // X (rows x k) <- X L^{-T} in place, block column by block column
+    auto trsm_right = [&](float *X, int rows, const float *L32, int k) {
+        for (int jb = 0; jb < k; jb += kNB) {
+            const int bw = std::min(kNB, k - jb);
+            if (jb > 0)
+                gemm(CUBLAS_OP_N, CUBLAS_OP_T, rows, bw, jb, X, rows, L32 + jb, k, &one,
+                     X + (size_t)jb * rows, rows, &minus);
+            k_trsm_cols<<<(rows + 127) / 128, 128, 0, s>>>(X, rows, L32, k, jb, bw);
+        }
+    };
+    // orthonormalise the columns of X (rows x k, column-major) in place:
+    // Cholesky QR with the Gram matrix in fp64 (the pass that copes with the
+    // conditioning of X), then once more in fp32 on the nearly orthonormal
+    // result
+    auto orth = [&](float *X, float *, int rows, int k) {
         k_to_f64<<<grid_for((long long)rows * k), 256, 0, s>>>(X, D, (long long)rows * k);
         blas_ok = blas_ok && cublasDgemm(H, CUBLAS_OP_T, CUBLAS_OP_N, k, k, rows, &done, D, rows, D,
                                          rows, &dzero, G, k) == CUBLAS_STATUS_SUCCESS;
-        k_chol<double, false><<<1, kSmallThreads, 0, s>>>(G, k, JV, Lt);
-        gemm(CUBLAS_OP_N, CUBLAS_OP_N, rows, k, k, X, rows, Lt, k, &zero, Xt, rows, &one);
-        gemm(CUBLAS_OP_T, CUBLAS_OP_N, k, k, rows, Xt, rows, Xt, rows, &zero, G32, k, &one);
-        k_chol<float, false><<<1, kSmallThreads, 0, s>>>(G32, k, JV32, Lt);
-        gemm(CUBLAS_OP_N, CUBLAS_OP_N, rows, k, k, Xt, rows, Lt, k, &zero, X, rows, &one);
+        chol64(G, k);
+        k_lower_f32<double><<<grid_for((long long)k * k), 256, 0, s>>>(G, k, Lt, 0);
+        trsm_right(X, rows, Lt, k);
+        gemm(CUBLAS_OP_T, CUBLAS_OP_N, k, k, rows, X, rows, X, rows, &zero, G32, k, &one);
+        chol32(G32, k);
+        k_lower_f32<float><<<grid_for((long long)k * k), 256, 0, s>>>(G32, k, Lt, 0);
+        trsm_right(X, rows, Lt, k);
     };
     for (int p = 0; p < n_paths && blas_ok; ++p) {
         const int r = ranks[p], k = svid_k(r, m, n);
@@ -518,7 +616,8 @@ cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, c
         k_to_f64<<<grid_for((long long)m * k), 256, 0, s>>>(Y, D, (long long)m * k);
         blas_ok = blas_ok && cublasDgemm(H, CUBLAS_OP_T, CUBLAS_OP_N, k, k, m, &done, D, m, D, m,
                                          &dzero, G, k) == CUBLAS_STATUS_SUCCESS;
-        k_chol<double, true><<<1, kSmallThreads, 0, s>>>(G, k, JV, G32);
+        chol64(G, k);
+        k_lower_f32<double><<<grid_for((long long)k * k), 256, 0, s>>>(G, k, G32, 1);
         k_svd_jacobi<<<1, kSmallThreads, 0, s>>>(G32, JV32, k, sv, Lt);
         gemm(CUBLAS_OP_N, CUBLAS_OP_N, n, r, k, Q, n, Lt, k, &zero, Q2, n, &one);
         gemm(CUBLAS_OP_N, CUBLAS_OP_N, m, r, k, Y, m, Lt, k, &zero, Y2, m, &one);
