@@ -250,7 +250,7 @@ struct PrefillParams {
     float *z32;        // stage 1 output in fp32 instead of z (latent entry point), or null
     float *zpart;      // split stage 1: fp32 partial sums [split][T][N1] (before l)
     int split;         // stage-1 K slices (gridDim.z of stage 1)
-    int expanded;      // B operands pre-expanded to fp16 (bv, bu) and loaded by TMA
+    int expanded;      // B operands pre-expanded to fp16 (bv, bu): the k_tiles path
     uint16_t *bv;      // [N1][d_in]: +-g_p[k] at (column n of path p, input k)
     uint16_t *bu;      // [d_out][N1]: +-h_p[o] at (output o, column n of path p)
     void *y;           // stage 2 output [T][d_out]
@@ -423,8 +423,7 @@ __device__ __forceinline__ void store_chunk(const PrefillParams &P, const float 
 
 template <bool STAGE1>
 __global__ void __launch_bounds__(kThreads, 1)
-    k_prefill(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
-              const __grid_constant__ PrefillParams P) {
+    k_prefill(const __grid_constant__ CUtensorMap amap, const __grid_constant__ PrefillParams P) {
     __shared__ __align__(8) uint64_t full[STAGES], ready[STAGES], empty[STAGES];
     __shared__ __align__(8) uint64_t slab_bar, acc_bar;
     __shared__ uint32_t s_tmem;
@@ -482,13 +481,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     auto issue_load = [&](int i) {
         const int s = i % STAGES, kc = kbeg + i;
         uint64_t *b = full + s;
-        if (P.expanded) {
-            // both operands by TMA: the B tile is rows [n0, n0 + bn) of bv / bu
-            mb_expect_tx(b, (unsigned)(A_BYTES + bn * BK * 2));
-            tma_load_2d(A_of(s), &amap, kc * BK, m0, b);
-            tma_load_2d(B_of(s), &bmap, kc * BK, n0, b);
-            return;
-        }
         if (STAGE1) {
             unsigned char *src = S_of(s);
             for (int p = 0; p < P.L.n_paths; ++p) {
@@ -515,7 +507,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // ---------------- producer: copies for chunk i once the MMAs of
         //                  chunk i - STAGES have released its stage
         if (lane == 0) {
-            if (!STAGE1 && !P.expanded) {
+            if (!STAGE1) {
                 // the tile's U rows and h of every path, once
                 const int nrows = min(BN, P.d_out - n0);
                 for (int p = 0; p < P.L.n_paths; ++p) {
@@ -546,9 +538,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
             for (int i = 0; i < KC; ++i) {
                 const int s = i % STAGES;
-                // with both operands pre-expanded a stage is ready as soon as it lands
-                if (!mb_spin_role(P.expanded ? full + s : ready + s, (unsigned)((i / STAGES) & 1),
-                                  fail)) {
+                if (!mb_spin_role(ready + s, (unsigned)((i / STAGES) & 1), fail)) {
                     give_up();
                     break;
                 }
@@ -567,9 +557,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     } else {
         // ---------------- unpacking warps: +-scale B and fp16 A of each stage
         const int tid = threadIdx.x - 64;
-        bool ok = STAGE1 || P.expanded || mb_wait_role(&slab_bar, 0, fail);
+        bool ok = STAGE1 || mb_wait_role(&slab_bar, 0, fail);
         if (!ok) give_up();
-        for (int i = 0; i < KC && ok && !P.expanded; ++i) {
+        for (int i = 0; i < KC && ok; ++i) {
             const int s = i % STAGES;
             if (!mb_wait_role(full + s, (unsigned)((i / STAGES) & 1), fail)) {
                 give_up();
@@ -597,7 +587,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (threadIdx.x == 0) {
             for (int i = loads_issued - STAGES; i < loads_issued; ++i)
                 if (i >= 0) mb_wait(full + i % STAGES, (unsigned)((i / STAGES) & 1));
-            if (!STAGE1 && !P.expanded) mb_wait(&slab_bar, 0);
+            if (!STAGE1) mb_wait(&slab_bar, 0);
         }
         if (threadIdx.x == 32)
             for (int i = mmas_issued - STAGES; i < mmas_issued; ++i)
@@ -1128,7 +1118,7 @@ cudaError_t launch_prefill_latent(const lb_linear &L, const uint16_t *x, int64_t
             xmap, bvmap, P, tn, P.split, n_tiles);
     } else {
         const dim3 g1((unsigned)tm, (unsigned)tn, (unsigned)P.split);
-        k_prefill<true><<<g1, kThreads, smem_bytes<true>(), s>>>(xmap, bvmap, P);
+        k_prefill<true><<<g1, kThreads, smem_bytes<true>(), s>>>(xmap, P);
     }
     e = cudaGetLastError();
     if (e != cudaSuccess || P.split <= 1) return e;
@@ -1164,7 +1154,7 @@ cudaError_t launch_prefill_expand(const lb_linear &L, const uint16_t *z16, int64
             zmap, bumap, P, tn, 1, n_tiles);
     } else {
         const dim3 g2((unsigned)tm, (unsigned)tn);
-        k_prefill<false><<<g2, kThreads, smem_bytes<false>(), s>>>(zmap, bumap, P);
+        k_prefill<false><<<g2, kThreads, smem_bytes<false>(), s>>>(zmap, P);
     }
     return cudaGetLastError();
 }
