@@ -16,7 +16,9 @@ on a bounded sample (cpu_baseline), and the SM clocks seen while timing.
   python bench.py --config 2|3|4|6|7|8 [--steps K] [--warmup W]
 
 --config times the single-linear workloads instead (one JSON line per case,
-not the bench line): 2 = 4096x4096 r64 at T = 1, 8; 3 = the FFN triple at
+not the bench line): 2 = 4096x4096 r64 at T = 1, 8 (each also as "graph64":
+64 distinct weight copies, one forward each, replayed as one CUDA graph, per
+forward); 3 = the FFN triple at
 r = 128, 512 and T = 1, 16, 64; 4 = prefill at T = 2048, 8192; 6 = the
 latent-state halves (littlebit_linear_latent / _expand: the 70B key
 projection at T = 1 and a 4096-token cache, 4096x4096 r512 at T = 2048);
@@ -459,10 +461,48 @@ def run_config(args):
             raise RuntimeError("kernel reported an error")
         return statistics.median(ts)
 
+    def time_graph(L, x_bits, T, copies=64):
+        """Sustained single-linear throughput: `copies` distinct device copies of
+        the weights (so each forward streams its own), one forward each, captured
+        in one CUDA graph; L2 flushed before each replay.  Median ms per forward,
+        or None if the forwards cannot be captured."""
+        devs = [lb.DeviceLinear(L, dev) for _ in range(copies)]
+        x = lb.bf16_tensor(x_bits, dev)
+        y = torch.empty((T, devs[0].d_out), dtype=torch.bfloat16, device=dev)
+        ws = lb.new_workspace(max(lb.workspace_size(D, T) for D in devs), dev)
+        side = torch.cuda.Stream(dev)
+        side.wait_stream(torch.cuda.current_stream(dev))
+        with torch.cuda.stream(side):
+            for D in devs:
+                lb.linear_forward(D, x, y=y, ws=ws)
+        torch.cuda.current_stream(dev).wait_stream(side)
+        torch.cuda.synchronize(dev)
+        graph = torch.cuda.CUDAGraph()
+        try:
+            with torch.cuda.graph(graph):
+                for D in devs:
+                    lb.linear_forward(D, x, y=y, ws=ws)
+        except Exception as exc:  # noqa: BLE001 - reported, not fatal
+            print(f"# graph capture unavailable: {exc}", file=sys.stderr)
+            return None
+        ts = []
+        for _ in range(max(5, min(steps, 50))):
+            flush.zero_()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record()
+            graph.replay()
+            e1.record()
+            torch.cuda.synchronize(dev)
+            ts.append(e0.elapsed_time(e1) / copies)
+        if lb.poll_error(ws) != lb.LB_OK:
+            raise RuntimeError("kernel reported an error")
+        return statistics.median(ts)
+
     def wanted(name, T):
         return args.only is None or args.only in f"{name}:{T}"
 
-    def emit(name, cfg, T, L, ms, flops_mode, op="forward"):
+    def emit(name, cfg, T, L, ms, flops_mode, op="forward", mode="single"):
         n1 = sum(P["r"] for P in L["paths"])
         if op == "forward":
             wb = weight_bytes(L)
@@ -476,7 +516,7 @@ def run_config(args):
             wb = sum(P["u_words"].nbytes + 2 * L["d_out"] for P in L["paths"])
             act = T * (n1 + L["d_out"]) * 2
             flops = sum(2 * T * P["r"] * L["d_out"] for P in L["paths"])
-        line = {"config": cfg, "case": name, "op": op, "tokens": T, "ms": ms,
+        line = {"config": cfg, "case": name, "op": op, "mode": mode, "tokens": T, "ms": ms,
                 "us": ms * 1e3, "bytes": wb + act, "flops": flops,
                 "gbs": (wb + act) / ms / 1e6, "tflops": flops / ms / 1e9}
         if flops_mode:
@@ -494,6 +534,9 @@ def run_config(args):
             if wanted("4096x4096 r64", T):
                 L, x = inputs.config2(T)
                 emit("4096x4096 r64", 2, T, L, time_case(L, x, T, True), False)
+                ms = time_graph(L, x, T)
+                if ms is not None:
+                    emit("4096x4096 r64", 2, T, L, ms, False, mode="graph64")
     elif args.config == 3:
         for r in (128, 512):
             for T in (1, 16, 64):
@@ -503,6 +546,10 @@ def run_config(args):
                         continue
                     xin = xd if nm == "down" else x
                     emit(f"{nm} r{r}", 3, T, lins[nm], time_case(lins[nm], xin, T, True), False)
+                    if T == 1:
+                        ms = time_graph(lins[nm], xin, T)
+                        if ms is not None:
+                            emit(f"{nm} r{r}", 3, T, lins[nm], ms, False, mode="graph64")
     elif args.config == 7:
         # Dual-SVID initialisation (one dense weight -> two LittleBit paths):
         # the 4096 x 4096 r64 layer and the 70B gate shape (8192 -> 28672, r320),
