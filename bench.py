@@ -75,6 +75,25 @@ def dist_env():
     return world, rank, local
 
 
+def max_over_ranks(value: float, world: int, device=None) -> float:
+    """The largest of `value` over the ranks of the default process group (the
+    slowest rank's time), or `value` itself when there is one rank.  The
+    tensor lives on `device` (a CUDA device under NCCL, the CPU under gloo)."""
+    if world <= 1:
+        return float(value)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def replica_throughput(world: int, units_per_rank: int, slowest_ms: float) -> float:
+    """Whole-job units per second of `world` independent replicas, each doing
+    `units_per_rank` units, timed by the slowest rank (weak scaling)."""
+    return world * units_per_rank / (slowest_ms / 1e3)
+
+
 def workload_config(n_layers: int) -> dict:
     from paper_2506_13771_gb300 import inputs
     s = inputs.STACK_70B
@@ -321,11 +340,7 @@ def run_ours(args):
     if status != lb.LB_OK:
         raise RuntimeError(f"stack kernel reported {lb.status_string(status)}")
     per_launch_ms = [evs[i].elapsed_time(evs[i + 1]) for i in range(args.steps)]
-    total_ms = evs[0].elapsed_time(evs[-1])
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(evs[0].elapsed_time(evs[-1]), world, dev)
     clocks = sampler.summary(t_wall0, t_wall1)
     sampler.stop()
 
@@ -353,16 +368,12 @@ def run_ours(args):
         out_host.copy_(out, non_blocking=True)
     e1.record(stream)
     torch.cuda.synchronize(dev)
-    e2e_ms = e0.elapsed_time(e1)
-    if world > 1:
-        t = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
     if lb.poll_error(ws) != lb.LB_OK:
         raise RuntimeError("stack kernel reported an error in the end-to-end loop")
 
     ms_per_step = total_ms / args.steps
-    value = world * args.steps / (total_ms / 1e3)
+    value = replica_throughput(world, args.steps, total_ms)
     kernel_ms = statistics.mean(per_launch_ms)
     peaks = measured_peaks()
     peak = peaks.get("hbm_gbs")
@@ -387,7 +398,7 @@ def run_ours(args):
                      "frac": achieved / peak, "traffic": traffic,
                      "algorithmic_bytes_per_launch": step_bytes,
                      "kernel_ms": kernel_ms, "kernel_source_sha": sha},
-        "e2e": {"value": world * e2e_steps / (e2e_ms / 1e3), "unit": "tokens/s",
+        "e2e": {"value": replica_throughput(world, e2e_steps, e2e_ms), "unit": "tokens/s",
                 "h2d_bytes_per_step": x_host.numel() * 2,
                 "d2h_bytes_per_step": out_host.numel() * 4},
         "gpu_launches": args.steps,
