@@ -442,8 +442,10 @@ lb_status littlebit_poll_error(void *ws, lb_stream_t stream) {
     if (cudaMemcpy(&err, ws, sizeof(unsigned), cudaMemcpyDeviceToHost) != cudaSuccess)
         return LB_ERR_CUDA;
     if (err != 0u) {
-        const unsigned zero = 0;
-        if (cudaMemcpy(ws, &zero, sizeof(unsigned), cudaMemcpyHostToDevice) != cudaSuccess)
+        // the error word, and the grid-barrier counters a failed launch may
+        // have left behind
+        const unsigned zero[3] = {0u, 0u, 0u};
+        if (cudaMemcpy(ws, zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess)
             return LB_ERR_CUDA;
         return (lb_status)err;
     }

@@ -13,11 +13,14 @@
 // stage's mbarrier beside the TMA of X; stage 2 bulk-copies the tile's U rows
 // and h once per CTA.  X arrives by TMA (bf16) and is converted to fp16 in
 // shared memory (exact for |x| < 65504).  From four token tiles on, every
-// tile would repeat the unpacking, so one pre-pass writes the +-g / +-h
-// operands to the workspace, both GEMMs stream them by TMA, and a persistent
-// kernel (k_tiles) walks the tiles with two TMEM accumulators so the
-// epilogue of one tile overlaps the K loop of the next.  z goes to the
-// workspace as fp16 and comes back by TMA.
+// tile would repeat the unpacking, so the operands are expanded to +-g / +-h
+// fp16 matrices in the workspace once per call and both GEMMs stream them by
+// TMA.  That path is ONE cooperative launch (k_fused, one CTA per SM): the
+// expansion, stage 1 over all its tiles, the reduction of its K slices and
+// stage 2 run as phases separated by grid barriers, and each tile phase is
+// persistent, with two TMEM accumulators so the epilogue of one tile overlaps
+// the K loop of the next.  z goes to the workspace as fp16 and comes back by
+// TMA.
 //
 // One CTA computes a 128 x BN tile (BN <= 256 fp32 TMEM columns) with
 // specialised warps: warp 0 issues the TMA / bulk copies of each 64-element
@@ -159,6 +162,13 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, i
         : "memory");
 }
 
+// Fire-and-forget prefetch of one TMA box into L2.
+__device__ __forceinline__ void tma_prefetch_2d(const CUtensorMap *map, int x, int y) {
+    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(map),
+                 "r"(x), "r"(y)
+                 : "memory");
+}
+
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
@@ -250,7 +260,7 @@ struct PrefillParams {
     float *z32;        // stage 1 output in fp32 instead of z (latent entry point), or null
     float *zpart;      // split stage 1: fp32 partial sums [split][T][N1] (before l)
     int split;         // stage-1 K slices (gridDim.z of stage 1)
-    int expanded;      // B operands pre-expanded to fp16 (bv, bu): the k_tiles path
+    int expanded;      // B operands pre-expanded to fp16 (bv, bu): the k_fused path
     uint16_t *bv;      // [N1][d_in]: +-g_p[k] at (column n of path p, input k)
     uint16_t *bu;      // [d_out][N1]: +-h_p[o] at (output o, column n of path p)
     void *y;           // stage 2 output [T][d_out]
@@ -656,28 +666,167 @@ __device__ __forceinline__ void store_y_coalesced(const PrefillParams &P, const 
     }
 }
 
-// Persistent form for pre-expanded B operands (A and B both stream by TMA;
-// in stage 1 four warps convert each bf16 x stage to fp16 in place):
-// gridDim.x CTAs walk the tiles t = blockIdx.x, blockIdx.x + gridDim.x, ...
+// The item loops below run inside k_fused at ten warps per SM, so each
+// thread gathers the inputs of kBatch items (independent loads in flight)
+// before it computes and stores them, and walks its items of a [rows][cols]
+// index space by stepping (row, col) instead of dividing a flat index.
+constexpr int kBatch = 8;
+
+struct ItemWalk {
+    int row, col, drow, dcol, cols;
+    __device__ ItemWalk(long long i0, long long di, int cols_)
+        : row((int)(i0 / cols_)), col((int)(i0 % cols_)), drow((int)(di / cols_)),
+          dcol((int)(di % cols_)), cols(cols_) {}
+    __device__ __forceinline__ void step() {
+        row += drow;
+        col += dcol;
+        if (col >= cols) {
+            col -= cols;
+            ++row;
+        }
+    }
+};
+
+// z = l . (sum over the K slices of the partial t), as fp16 (or fp32 into z32),
+// four columns per item; items i0, i0 + di, ... of [T][N1 / 4].
+__device__ __forceinline__ void reduce_z_items(const PrefillParams &P, long long i0, long long di) {
+    constexpr int kB = kBatch / 2;
+    ItemWalk w(i0, di, P.N1 / 4);
+    const size_t slice = (size_t)P.T * P.N1;
+    while (w.row < P.T) {
+        int row[kB], c[kB];
+        float4 a[kB];
+#pragma unroll
+        for (int k = 0; k < kB; ++k) {
+            row[k] = w.row;
+            c[k] = 4 * w.col;
+            a[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+            w.step();
+        }
+        for (int z = 0; z < P.split; ++z) {
+#pragma unroll
+            for (int k = 0; k < kB; ++k) {
+                if (row[k] < P.T) {
+                    const float4 b = *reinterpret_cast<const float4 *>(
+                        P.zpart + z * slice + (size_t)row[k] * P.N1 + c[k]);
+                    a[k].x += b.x;
+                    a[k].y += b.y;
+                    a[k].z += b.z;
+                    a[k].w += b.w;
+                }
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < kB; ++k) {
+            if (row[k] >= P.T) continue;
+            const int p = c[k] >= P.off1 ? 1 : 0, j = c[k] - (p ? P.off1 : 0);  // 4 | off1
+            const uint2 lb = __ldg(reinterpret_cast<const uint2 *>((p ? P.L.l[1] : P.L.l[0]) + j));
+            const float l0 = half_bits_to_float(lb.x & 0xffffu), l1 = half_bits_to_float(lb.x >> 16);
+            const float l2 = half_bits_to_float(lb.y & 0xffffu), l3 = half_bits_to_float(lb.y >> 16);
+            const size_t e = (size_t)row[k] * P.N1 + c[k];
+            if (P.z32) {
+                *reinterpret_cast<float4 *>(P.z32 + e) =
+                    make_float4(a[k].x * l0, a[k].y * l1, a[k].z * l2, a[k].w * l3);
+                continue;
+            }
+            const __half2 h0 = __floats2half2_rn(a[k].x * l0, a[k].y * l1);
+            const __half2 h1 = __floats2half2_rn(a[k].z * l2, a[k].w * l3);
+            *reinterpret_cast<uint2 *>(P.z + e) =
+                make_uint2(*reinterpret_cast<const uint32_t *>(&h0),
+                           *reinterpret_cast<const uint32_t *>(&h1));
+        }
+    }
+}
+
+// bv[n][k] = +-g_p[k]: input k of column n (column j of path p) of V_sign,
+// eight inputs (one 16-byte chunk) per item; items of [N1][d_in / 8].
+__device__ __forceinline__ void expand_v_items(const PrefillParams &P, long long i0, long long di) {
+    ItemWalk w(i0, di, P.L.d_in / 8);
+    while (w.row < P.N1) {
+        int n[kBatch], k0[kBatch];
+        uint32_t word[kBatch];
+        uint4 mag[kBatch];
+#pragma unroll
+        for (int k = 0; k < kBatch; ++k) {
+            n[k] = w.row;
+            k0[k] = 8 * w.col;
+            w.step();
+            word[k] = 0u;
+            mag[k] = make_uint4(0u, 0u, 0u, 0u);
+            if (n[k] < P.N1) {
+                const int p = n[k] >= P.off1 ? 1 : 0, j = n[k] - (p ? P.off1 : 0);
+                const int r = p ? P.L.r[1] : P.L.r[0];
+                word[k] = __ldg((p ? P.L.v[1] : P.L.v[0]) + (size_t)(k0[k] >> 5) * r + j);
+                mag[k] = __ldg(reinterpret_cast<const uint4 *>((p ? P.L.g[1] : P.L.g[0]) + k0[k]));
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < kBatch; ++k)
+            if (n[k] < P.N1)
+                *reinterpret_cast<uint4 *>(P.bv + (size_t)n[k] * P.L.d_in + k0[k]) =
+                    signed8((word[k] >> (k0[k] & 31)) & 0xffu, mag[k]);
+    }
+}
+
+// bu[o][n] = +-h_p[o]: column n (column j of path p) of row o of U_sign,
+// eight columns per item; items of [d_out][N1 / 8].
+__device__ __forceinline__ void expand_u_items(const PrefillParams &P, long long i0, long long di) {
+    ItemWalk w(i0, di, P.N1 / 8);
+    while (w.row < P.d_out) {
+        int o[kBatch], n0[kBatch];
+        uint32_t word[kBatch], hb[kBatch];
+#pragma unroll
+        for (int k = 0; k < kBatch; ++k) {
+            o[k] = w.row;
+            n0[k] = 8 * w.col;
+            w.step();
+            word[k] = hb[k] = 0u;
+            if (o[k] < P.d_out) {
+                const int p = n0[k] >= P.off1 ? 1 : 0, j0 = n0[k] - (p ? P.off1 : 0);
+                const int R = ((p ? P.L.r[1] : P.L.r[0]) + 31) >> 5;
+                word[k] = __ldg((p ? P.L.u[1] : P.L.u[0]) + (size_t)o[k] * R + (j0 >> 5));
+                hb[k] = __ldg((p ? P.L.h[1] : P.L.h[0]) + o[k]);
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < kBatch; ++k) {
+            if (o[k] >= P.d_out) continue;
+            const int p = n0[k] >= P.off1 ? 1 : 0, j0 = n0[k] - (p ? P.off1 : 0);
+            const uint32_t hh = hb[k] | (hb[k] << 16);
+            *reinterpret_cast<uint4 *>(P.bu + (size_t)o[k] * P.N1 + n0[k]) =
+                signed8((word[k] >> (j0 & 31)) & 0xffu, make_uint4(hh, hh, hh, hh));
+        }
+    }
+}
+
+// mbarriers of one persistent tile phase.  Each phase of the fused kernel has
+// its own set, so that no late arrival of one phase lands on the other's.
+struct PhaseBars {
+    uint64_t full[kMaxStages], ready[kMaxStages], empty[kMaxStages], acc_full[2], acc_empty[2];
+};
+
+__device__ __forceinline__ void fence_proxy_async_global() {
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+// One persistent tile phase over pre-expanded B operands (A and B both
+// stream by TMA; in stage 1 four warps convert each bf16 x stage to fp16 in
+// place): the CTAs walk the tiles t = blockIdx.x, blockIdx.x + gridDim.x, ...
 // (column tile fastest, then K slice, then token tile) and keep two fp32
 // accumulators in TMEM (2 x BN columns), so the epilogue warps read out tile
 // t while the MMA warp already accumulates tile t + gridDim.x and the copy
 // warp keeps streaming K-stages across tile boundaries.  acc_full[b] is
 // committed by the MMA warp when accumulator b holds a finished tile;
 // acc_empty[b] collects one arrival per epilogue warp once it has read b.
+// Every thread of the CTA calls this; false once a wait of this CTA ran out
+// (every copy and MMA it issued has landed by then).
 template <bool STAGE1>
-__global__ void __launch_bounds__(kThreads, 1)
-    k_tiles(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
-            const __grid_constant__ PrefillParams P, int tiles_n, int nsplit, int n_tiles) {
-    __shared__ __align__(8) uint64_t full[kMaxStages], ready[kMaxStages], empty[kMaxStages],
-        acc_full[2], acc_empty[2];
-    __shared__ uint32_t s_tmem;
-    __shared__ int s_fail;
-    unsigned char *smem = reinterpret_cast<unsigned char *>(
-        (reinterpret_cast<uintptr_t>(p_smem) + 1023) & ~(uintptr_t)1023);
+__device__ bool run_tiles(const CUtensorMap *amap, const CUtensorMap *bmap,
+                          const PrefillParams &P, int tiles_n, int nsplit, int n_tiles,
+                          PhaseBars &B, uint32_t tmem, unsigned char *smem, volatile int *fail,
+                          bool expand_u_meanwhile = false) {
     // stage 1 streams x as bf16: warps 2..5 convert each A stage to fp16 in
     // place and warps 6..9 run the epilogue; stage 2 uses all eight for it
-    constexpr int kEpiWarps = STAGE1 ? 4 : kWorkWarps;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int bn = STAGE1 ? P.bn1 : BN;
     const int KT = (STAGE1 ? P.L.d_in : P.N1) / BK;
@@ -685,33 +834,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     // (bn 64 / 128 / 192 / 256 -> 8 / 6 / 4 / 4 stages of 24 / 32 / 40 / 48 KB)
     const int SB = A_BYTES + bn * BK * 2;
     const int nst = min(kMaxStages, RING_BYTES / SB);
-    volatile int *fail = &s_fail;
-    if (ld_relaxed_gpu(P.ws_words + kErrWord) != 0u) return;
-
-    if (threadIdx.x == 0) {
-        for (int s = 0; s < nst; ++s) {
-            mb_init(full + s, 1);
-            mb_init(ready + s, 4);
-            mb_init(empty + s, 1);
-        }
-        for (int b = 0; b < 2; ++b) {
-            mb_init(acc_full + b, 1);
-            mb_init(acc_empty + b, kEpiWarps);
-        }
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-        s_fail = 0;
-    }
-    if (warp == 1) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                         su32(&s_tmem)),
-                     "r"(2 * BN)
-                     : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem = s_tmem;
     const uint32_t idesc = instr_desc(BM, bn);
     auto give_up = [&]() {
         *fail = 1;
@@ -738,6 +860,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 0) {
         // ---------------- copy warp
         if (lane == 0) {
+            // the operands may have been written by other CTAs of this launch
+            // (generic proxy) before the grid barrier that led here
+            fence_proxy_async_global();
             bool ok = true;
             int s = 0;
             unsigned ph = 0;
@@ -746,15 +871,15 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tile(t, m0, n0, z, kbeg, kc);
                 for (int i = 0; i < kc; ++i) {
                     // a stage's previous use must have been multiplied
-                    if (loads_issued >= nst && !mb_spin_role(empty + s, ph ^ 1u, fail)) {
+                    if (loads_issued >= nst && !mb_spin_role(B.empty + s, ph ^ 1u, fail)) {
                         give_up();
                         ok = false;
                         break;
                     }
-                    uint64_t *b = full + s;
+                    uint64_t *b = B.full + s;
                     mb_expect_tx(b, (unsigned)SB);
-                    tma_load_2d(smem + s * SB, &amap, (kbeg + i) * BK, m0, b);
-                    tma_load_2d(smem + s * SB + A_BYTES, &bmap, (kbeg + i) * BK, n0, b);
+                    tma_load_2d(smem + s * SB, amap, (kbeg + i) * BK, m0, b);
+                    tma_load_2d(smem + s * SB + A_BYTES, bmap, (kbeg + i) * BK, n0, b);
                     ++loads_issued;
                     advance(s, ph);
                 }
@@ -772,7 +897,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tile(t, m0, n0, z, kbeg, kc);
                 const int b = ti & 1;
                 if (ti >= 2 &&
-                    !mb_spin_role(acc_empty + b, (unsigned)(((ti >> 1) - 1) & 1), fail)) {
+                    !mb_spin_role(B.acc_empty + b, (unsigned)(((ti >> 1) - 1) & 1), fail)) {
                     give_up();
                     break;
                 }
@@ -780,7 +905,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 const uint32_t d = tmem + (uint32_t)(b * BN);
                 for (int i = 0; i < kc; ++i) {
                     // stage 1: the stage is ready once its A half is fp16
-                    if (!mb_spin_role(STAGE1 ? ready + s : full + s, ph, fail)) {
+                    if (!mb_spin_role(STAGE1 ? B.ready + s : B.full + s, ph, fail)) {
                         give_up();
                         ok = false;
                         break;
@@ -791,11 +916,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                     for (int k = 0; k < BK / 16; ++k)
                         mma_f16(d, smem_desc(a0 + 32 * k), smem_desc(b0 + 32 * k), idesc,
                                 (i > 0 || k > 0) ? 1u : 0u);
-                    mma_commit(empty + s);
+                    mma_commit(B.empty + s);
                     ++mmas_issued;
                     advance(s, ph);
                 }
-                if (ok) mma_commit(acc_full + b);
+                if (ok) mma_commit(B.acc_full + b);
             }
         }
         __syncwarp();
@@ -809,7 +934,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             int m0, n0, z, kbeg, kc;
             tile(t, m0, n0, z, kbeg, kc);
             for (int i = 0; i < kc; ++i, advance(s, ph)) {
-                const bool got = mb_wait_role(full + s, ph, fail);
+                const bool got = mb_wait_role(B.full + s, ph, fail);
                 if (!__all_sync(0xffffffffu, got)) {
                     if (lane == 0) give_up();
                     ok = false;
@@ -819,7 +944,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 fence_proxy_async_smem();
                 __syncwarp();
                 if (lane == 0)
-                    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(ready + s))
+                    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(B.ready + s))
                                  : "memory");
             }
         }
@@ -831,6 +956,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int half = STAGE1 ? 0 : (warp - 2) >> 2, halves = STAGE1 ? 1 : 2;
         const uint32_t lane_base = tmem + ((uint32_t)(32 * wq) << 16);
         const int cb0 = 32 * (half * nchunk / halves), cb1 = 32 * ((half + 1) * nchunk / halves);
+        // stage 1 of a forward: the epilogue warps of all CTAs expand stage
+        // 2's +-h operand while the first tiles accumulate
+        if (STAGE1 && expand_u_meanwhile)
+            expand_u_items(P, blockIdx.x * 128LL + (threadIdx.x - 192), gridDim.x * 128LL);
         int ti = 0;
         for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++ti) {
             int m0, n0, z, kbeg, kc;
@@ -839,7 +968,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             // the vote reconverges the warp (each lane leaves the wait on its
             // own) before the warp-collective tcgen05.ld, and makes the
             // outcome uniform
-            const bool got = mb_wait_role(acc_full + b, (unsigned)((ti >> 1) & 1), fail);
+            const bool got = mb_wait_role(B.acc_full + b, (unsigned)((ti >> 1) & 1), fail);
             if (!__all_sync(0xffffffffu, got)) {
                 if (lane == 0) give_up();
                 break;
@@ -860,7 +989,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_before();
             __syncwarp();
             if (lane == 0)
-                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(acc_empty + b))
+                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(B.acc_empty + b))
                              : "memory");
         }
     }
@@ -868,11 +997,130 @@ __global__ void __launch_bounds__(kThreads, 1)
         // let every issued copy and MMA land before the CTA goes away
         if (threadIdx.x == 0)
             for (int i = loads_issued - nst; i < loads_issued; ++i)
-                if (i >= 0) mb_wait(full + i % nst, (unsigned)((i / nst) & 1));
+                if (i >= 0) mb_wait(B.full + i % nst, (unsigned)((i / nst) & 1));
         if (threadIdx.x == 32)
             for (int i = mmas_issued - nst; i < mmas_issued; ++i)
-                if (i >= 0) mb_wait(empty + i % nst, (unsigned)((i / nst) & 1));
+                if (i >= 0) mb_wait(B.empty + i % nst, (unsigned)((i / nst) & 1));
         __syncthreads();
+        return false;
+    }
+    return true;
+}
+
+// The split stage 1 of the non-persistent path (k_prefill) reduces its K
+// slices in a launch of its own.
+__global__ void k_reduce_z(const __grid_constant__ PrefillParams P) {
+    reduce_z_items(P, blockIdx.x * (long long)blockDim.x + threadIdx.x,
+                   (long long)gridDim.x * blockDim.x);
+}
+
+// What one launch of k_fused does, in this order: expand V and / or U, stage
+// 1 (and the reduction of its K slices), stage 2.
+enum : int { kDoExpandV = 1, kDoExpandU = 2, kDoStage1 = 4, kDoStage2 = 8 };
+struct FusedPlan {
+    int flags;
+    int tiles_n1, split, n_tiles1;  // stage 1: column tiles, K slices, work units
+    int tiles_n2, n_tiles2;         // stage 2: column tiles, tiles
+};
+
+// The many-token forward (or either half of it) in ONE cooperative launch of
+// one CTA per SM: the +-g / +-h operand expansion, stage 1 over all its
+// tiles, the reduction of its K slices, and stage 2, separated by grid
+// barriers.  Writes that a later phase reads by TMA are published with a
+// proxy fence before the barrier.  The last CTA out resets the barrier
+// counter, so the next launch on the workspace starts from zero; a launch
+// that fails leaves the sticky error word set, and littlebit_poll_error
+// clears both.
+__global__ void __launch_bounds__(kThreads, 1)
+    k_fused(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap bvmap,
+            const __grid_constant__ CUtensorMap zmap, const __grid_constant__ CUtensorMap bumap,
+            const __grid_constant__ PrefillParams P, const __grid_constant__ FusedPlan F) {
+    __shared__ PhaseBars bars[2];
+    __shared__ uint32_t s_tmem;
+    __shared__ int s_fail;
+    unsigned char *smem = reinterpret_cast<unsigned char *>(
+        (reinterpret_cast<uintptr_t>(p_smem) + 1023) & ~(uintptr_t)1023);
+    const int warp = threadIdx.x >> 5;
+    volatile int *fail = &s_fail;
+    if (ld_relaxed_gpu(P.ws_words + kErrWord) != 0u) return;
+    const unsigned n_ctas = gridDim.x;
+
+    if (threadIdx.x == 0) {
+        for (int ph = 0; ph < 2; ++ph) {
+            PhaseBars &B = bars[ph];
+            for (int s = 0; s < kMaxStages; ++s) {
+                mb_init(B.full + s, 1);
+                mb_init(B.ready + s, 4);
+                mb_init(B.empty + s, 1);
+            }
+            for (int b = 0; b < 2; ++b) {
+                mb_init(B.acc_full + b, 1);
+                mb_init(B.acc_empty + b, ph == 0 ? 4 : kWorkWarps);
+            }
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        s_fail = 0;
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         su32(&s_tmem)),
+                     "r"(2 * BN)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = s_tmem;
+    const long long gi = blockIdx.x * (long long)blockDim.x + threadIdx.x;
+    const long long gn = (long long)gridDim.x * blockDim.x;
+    unsigned nbar = 0;  // grid barriers passed
+    bool ok = true;
+
+    // U is expanded up front only without a stage 1 to hide it in
+    const bool u_in_stage1 = (F.flags & kDoStage1) && (F.flags & kDoExpandU);
+    if (F.flags & (kDoExpandV | kDoExpandU)) {
+        if (threadIdx.x == 32) {
+            // while the operands expand: the A stages of this CTA's first tile
+            // (x or z, inputs of the call) into L2
+            const bool s1 = F.flags & kDoStage1;
+            const int t = blockIdx.x, tiles_n = s1 ? F.tiles_n1 : F.tiles_n2;
+            const int nsplit = s1 ? F.split : 1, KT = (s1 ? P.L.d_in : P.N1) / BK;
+            if (t < (s1 ? F.n_tiles1 : F.n_tiles2)) {
+                const int rest = t / tiles_n, z = rest % nsplit, m0 = (rest / nsplit) * BM;
+                const int kbeg = (int)((long long)z * KT / nsplit);
+                const int kc = (int)((long long)(z + 1) * KT / nsplit) - kbeg;
+                for (int i = 0; i < kc && i < 16; ++i)
+                    tma_prefetch_2d(s1 ? &xmap : &zmap, (kbeg + i) * BK, m0);
+            }
+        }
+        if (F.flags & kDoExpandV) expand_v_items(P, gi, gn);
+        if ((F.flags & kDoExpandU) && !u_in_stage1) expand_u_items(P, gi, gn);
+        fence_proxy_async_global();
+        ok = grid_barrier(P.ws_words, n_ctas * ++nbar);
+    }
+    if (ok && (F.flags & kDoStage1)) {
+        ok = run_tiles<true>(&xmap, &bvmap, P, F.tiles_n1, F.split, F.n_tiles1, bars[0], tmem,
+                             smem, fail, u_in_stage1);
+        if (ok && F.split > 1) {
+            ok = grid_barrier(P.ws_words, n_ctas * ++nbar);
+            if (ok) reduce_z_items(P, gi, gn);
+        }
+        if (ok && (F.flags & kDoStage2)) {
+            fence_proxy_async_global();
+            ok = grid_barrier(P.ws_words, n_ctas * ++nbar);
+        }
+    }
+    if (ok && (F.flags & kDoStage2))
+        ok = run_tiles<false>(&zmap, &bumap, P, F.tiles_n2, 1, F.n_tiles2, bars[1], tmem, smem,
+                              fail);
+    if (ok && threadIdx.x == 0) {
+        // every CTA counted here has passed its last barrier
+        __threadfence();
+        if (atomicAdd(P.ws_words + kDoneWord, 1u) == n_ctas - 1) {
+            atomicExch(P.ws_words + kCounterWord, 0u);
+            atomicExch(P.ws_words + kDoneWord, 0u);
+        }
     }
     tc_fence_before();
     __syncthreads();
@@ -880,78 +1128,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                      "r"(2 * BN)
                      : "memory");
-}
-
-// z = l . (sum over the K slices of the partial t), as fp16 (or fp32 into z32),
-// four columns per thread.
-__global__ void k_reduce_z(const __grid_constant__ PrefillParams P) {
-    const int groups = P.N1 / 4;
-    const long long n = (long long)P.T * groups;
-    for (long long g = blockIdx.x * (long long)blockDim.x + threadIdx.x; g < n;
-         g += (long long)gridDim.x * blockDim.x) {
-        const int row = (int)(g / groups), c = 4 * (int)(g % groups);
-        float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int z = 0; z < P.split; ++z) {
-            const float4 b = *reinterpret_cast<const float4 *>(
-                P.zpart + ((size_t)z * P.T + row) * P.N1 + c);
-            a.x += b.x;
-            a.y += b.y;
-            a.z += b.z;
-            a.w += b.w;
-        }
-        const int p = c >= P.off1 ? 1 : 0, j = c - (p ? P.off1 : 0);  // 4 | off1
-        const uint2 lb = *reinterpret_cast<const uint2 *>((p ? P.L.l[1] : P.L.l[0]) + j);
-        if (P.z32) {
-            *reinterpret_cast<float4 *>(P.z32 + (size_t)row * P.N1 + c) =
-                make_float4(a.x * half_bits_to_float(lb.x & 0xffffu),
-                            a.y * half_bits_to_float(lb.x >> 16),
-                            a.z * half_bits_to_float(lb.y & 0xffffu),
-                            a.w * half_bits_to_float(lb.y >> 16));
-            continue;
-        }
-        const __half2 h0 = __floats2half2_rn(a.x * half_bits_to_float(lb.x & 0xffffu),
-                                             a.y * half_bits_to_float(lb.x >> 16));
-        const __half2 h1 = __floats2half2_rn(a.z * half_bits_to_float(lb.y & 0xffffu),
-                                             a.w * half_bits_to_float(lb.y >> 16));
-        *reinterpret_cast<uint2 *>(P.z + (size_t)row * P.N1 + c) =
-            make_uint2(*reinterpret_cast<const uint32_t *>(&h0),
-                       *reinterpret_cast<const uint32_t *>(&h1));
-    }
-}
-
-// bv[n][k] = +-g_p[k]: input k of column n (column j of path p) of V_sign,
-// eight inputs (one 16-byte chunk) per thread.
-__global__ void k_expand_v(const __grid_constant__ PrefillParams P) {
-    const int kq = P.L.d_in / 8;
-    const long long n_items = (long long)P.N1 * kq;
-    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < n_items;
-         idx += (long long)gridDim.x * blockDim.x) {
-        const int n = (int)(idx / kq), k0 = 8 * (int)(idx % kq);
-        const int p = n >= P.off1 ? 1 : 0, j = n - (p ? P.off1 : 0);
-        const int r = p ? P.L.r[1] : P.L.r[0];
-        const uint32_t word = __ldg((p ? P.L.v[1] : P.L.v[0]) + (size_t)(k0 >> 5) * r + j);
-        const uint4 mag = *reinterpret_cast<const uint4 *>((p ? P.L.g[1] : P.L.g[0]) + k0);
-        *reinterpret_cast<uint4 *>(P.bv + (size_t)n * P.L.d_in + k0) =
-            signed8((word >> (k0 & 31)) & 0xffu, mag);
-    }
-}
-
-// bu[o][n] = +-h_p[o]: column n (column j of path p) of row o of U_sign,
-// eight columns per thread.
-__global__ void k_expand_u(const __grid_constant__ PrefillParams P) {
-    const int nq = P.N1 / 8;
-    const long long n_items = (long long)P.d_out * nq;
-    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < n_items;
-         idx += (long long)gridDim.x * blockDim.x) {
-        const int o = (int)(idx / nq), n0 = 8 * (int)(idx % nq);
-        const int p = n0 >= P.off1 ? 1 : 0, j0 = n0 - (p ? P.off1 : 0);
-        const int R = ((p ? P.L.r[1] : P.L.r[0]) + 31) >> 5;
-        const uint32_t word = __ldg((p ? P.L.u[1] : P.L.u[0]) + (size_t)o * R + (j0 >> 5));
-        const uint32_t hb = __ldg((p ? P.L.h[1] : P.L.h[0]) + o);
-        const uint32_t hh = hb | (hb << 16);
-        *reinterpret_cast<uint4 *>(P.bu + (size_t)o * P.N1 + n0) =
-            signed8((word >> (j0 & 31)) & 0xffu, make_uint4(hh, hh, hh, hh));
-    }
 }
 
 // ---------------------------------------------------------------- host side
@@ -1000,11 +1176,7 @@ static cudaError_t set_smem_attributes() {
     e = cudaFuncSetAttribute(k_prefill<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              smem_bytes<true>());
     if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_tiles<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 kTilesSmem);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(k_tiles<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 kTilesSmem);
+        e = cudaFuncSetAttribute(k_fused, cudaFuncAttributeMaxDynamicSharedMemorySize, kTilesSmem);
     if (e == cudaSuccess)
         e = cudaFuncSetAttribute(k_prefill<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  smem_bytes<false>());
@@ -1092,13 +1264,40 @@ PrefillParams params_of(const lb_linear &L, int64_t T, unsigned *ws_words, void 
 }
 }  // namespace
 
+namespace {
+// One cooperative launch of k_fused, one CTA per SM (the grid barriers need
+// every CTA resident).  Maps of phases the plan skips are never read.
+cudaError_t launch_fused(const CUtensorMap &xmap, const CUtensorMap &bvmap,
+                         const CUtensorMap &zmap, const CUtensorMap &bumap,
+                         const PrefillParams &P, const FusedPlan &F, cudaStream_t s) {
+    void *args[] = {const_cast<CUtensorMap *>(&xmap), const_cast<CUtensorMap *>(&bvmap),
+                    const_cast<CUtensorMap *>(&zmap), const_cast<CUtensorMap *>(&bumap),
+                    const_cast<PrefillParams *>(&P), const_cast<FusedPlan *>(&F)};
+    return cudaLaunchCooperativeKernel((const void *)k_fused, dim3(device_sms()), dim3(kThreads),
+                                       args, kTilesSmem, s);
+}
+
+// Stage-1 and stage-2 tilings of the persistent phases.
+void plan_stage1(const PrefillParams &P, FusedPlan &F) {
+    const int tm = (P.T + BM - 1) / BM, tn = (P.N1 + P.bn1 - 1) / P.bn1;
+    F.tiles_n1 = tn;
+    F.split = P.split;
+    F.n_tiles1 = tm * tn * P.split;
+}
+void plan_stage2(const PrefillParams &P, FusedPlan &F) {
+    const int tm = (P.T + BM - 1) / BM, tn = (P.d_out + BN - 1) / BN;
+    F.tiles_n2 = tn;
+    F.n_tiles2 = tm * tn;
+}
+}  // namespace
+
 cudaError_t launch_prefill_latent(const lb_linear &L, const uint16_t *x, int64_t T, uint16_t *z16,
                                   float *z32, unsigned *ws_words, void *ws, cudaStream_t s) {
     if (!encoder()) return cudaErrorNotSupported;
     PrefillParams P = params_of(L, T, ws_words, ws);
     P.z = z16;
     P.z32 = z32;
-    CUtensorMap xmap, bvmap{};
+    CUtensorMap xmap, bvmap{}, none{};
     if (!make_map(&xmap, x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, T, L.d_in)) return cudaErrorInvalidValue;
     if (P.expanded &&
         !make_map(&bvmap, P.bv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, P.N1, L.d_in, P.bn1))
@@ -1106,20 +1305,14 @@ cudaError_t launch_prefill_latent(const lb_linear &L, const uint16_t *x, int64_t
     cudaError_t e = set_smem_attributes();
     if (e != cudaSuccess) return e;
     if (P.expanded) {
-        const long long nv = (long long)P.N1 * (L.d_in / 8);
-        k_expand_v<<<(int)std::min<long long>((nv + 255) / 256, 148 * 16), 256, 0, s>>>(P);
-        e = cudaGetLastError();
-        if (e != cudaSuccess) return e;
+        FusedPlan F{};
+        F.flags = kDoExpandV | kDoStage1;
+        plan_stage1(P, F);
+        return launch_fused(xmap, bvmap, none, none, P, F, s);
     }
     const int tm = (int)((T + BM - 1) / BM), tn = (P.N1 + P.bn1 - 1) / P.bn1;
-    if (P.expanded) {
-        const int n_tiles = tm * tn * P.split;
-        k_tiles<true><<<std::min(n_tiles, device_sms()), kThreads, kTilesSmem, s>>>(
-            xmap, bvmap, P, tn, P.split, n_tiles);
-    } else {
-        const dim3 g1((unsigned)tm, (unsigned)tn, (unsigned)P.split);
-        k_prefill<true><<<g1, kThreads, smem_bytes<true>(), s>>>(xmap, P);
-    }
+    const dim3 g1((unsigned)tm, (unsigned)tn, (unsigned)P.split);
+    k_prefill<true><<<g1, kThreads, smem_bytes<true>(), s>>>(xmap, P);
     e = cudaGetLastError();
     if (e != cudaSuccess || P.split <= 1) return e;
     const long long groups = (long long)T * (P.N1 / 4);
@@ -1135,36 +1328,51 @@ cudaError_t launch_prefill_expand(const lb_linear &L, const uint16_t *z16, int64
     P.z = const_cast<uint16_t *>(z16);
     P.y = y;
     P.y_fp32 = y_fp32;
-    CUtensorMap zmap, bumap{};
+    CUtensorMap zmap, bumap{}, none{};
     if (!make_map(&zmap, z16, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, T, P.N1)) return cudaErrorInvalidValue;
     if (P.expanded && !make_map(&bumap, P.bu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, L.d_out, P.N1, BN))
         return cudaErrorInvalidValue;
     cudaError_t e = set_smem_attributes();
     if (e != cudaSuccess) return e;
     if (P.expanded) {
-        const long long nu = (long long)L.d_out * (P.N1 / 8);
-        k_expand_u<<<(int)std::min<long long>((nu + 255) / 256, 148 * 16), 256, 0, s>>>(P);
-        e = cudaGetLastError();
-        if (e != cudaSuccess) return e;
+        FusedPlan F{};
+        F.flags = kDoExpandU | kDoStage2;
+        plan_stage2(P, F);
+        return launch_fused(none, none, zmap, bumap, P, F, s);
     }
     const int tm = (int)((T + BM - 1) / BM), tn = (L.d_out + BN - 1) / BN;
-    if (P.expanded) {
-        const int n_tiles = tm * tn;
-        k_tiles<false><<<std::min(n_tiles, device_sms()), kThreads, kTilesSmem, s>>>(
-            zmap, bumap, P, tn, 1, n_tiles);
-    } else {
-        const dim3 g2((unsigned)tm, (unsigned)tn);
-        k_prefill<false><<<g2, kThreads, smem_bytes<false>(), s>>>(zmap, P);
-    }
+    const dim3 g2((unsigned)tm, (unsigned)tn);
+    k_prefill<false><<<g2, kThreads, smem_bytes<false>(), s>>>(zmap, P);
     return cudaGetLastError();
 }
 
 cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, void *y, int y_fp32,
                            unsigned *ws_words, void *ws, cudaStream_t s) {
     uint16_t *z16 = static_cast<uint16_t *>(ws);  // the workspace starts with z
-    cudaError_t e = launch_prefill_latent(L, x, T, z16, nullptr, ws_words, ws, s);
+    if (!encoder()) return cudaErrorNotSupported;
+    PrefillParams P = params_of(L, T, ws_words, ws);
+    if (!P.expanded) {
+        cudaError_t e = launch_prefill_latent(L, x, T, z16, nullptr, ws_words, ws, s);
+        if (e != cudaSuccess) return e;
+        return launch_prefill_expand(L, z16, T, y, y_fp32, ws_words, ws, s);
+    }
+    // both stages in one launch
+    P.z = z16;
+    P.y = y;
+    P.y_fp32 = y_fp32;
+    CUtensorMap xmap, bvmap, zmap, bumap;
+    if (!make_map(&xmap, x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, T, L.d_in) ||
+        !make_map(&bvmap, P.bv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, P.N1, L.d_in, P.bn1) ||
+        !make_map(&zmap, z16, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, T, P.N1) ||
+        !make_map(&bumap, P.bu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, L.d_out, P.N1, BN))
+        return cudaErrorInvalidValue;
+    cudaError_t e = set_smem_attributes();
     if (e != cudaSuccess) return e;
-    return launch_prefill_expand(L, z16, T, y, y_fp32, ws_words, ws, s);
+    FusedPlan F{};
+    F.flags = kDoExpandV | kDoExpandU | kDoStage1 | kDoStage2;
+    plan_stage1(P, F);
+    plan_stage2(P, F);
+    return launch_fused(xmap, bvmap, zmap, bumap, P, F, s);
 }
 
 }  // namespace lb

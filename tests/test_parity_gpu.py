@@ -503,6 +503,56 @@ def test_stack_70b_full():
     check_stack(run_stack(layers, x0, 128), oracle.stack_forward(layers, x0, head_dim=128))
 
 
+def test_fused_launch_reuses_workspace():
+    """From four token tiles on, the forward (and each of latent / expand) is
+    one cooperative launch whose grid barriers count on workspace words 1 and
+    2.  Repeated calls on one workspace give bit-identical outputs and leave
+    both words at zero; after a timed-out wait and its poll (which clears
+    them) the launch works again."""
+    rng = inputs.rng_for(108, salt=0)
+    # 4 token tiles x 4 column tiles: stage 1 is split into K slices, so the
+    # launch runs three grid barriers (expansion, slices, stage 2)
+    T, d_in, d_out = 512, 4096, 2048
+    L = inputs.make_linear(rng, d_in, d_out, [512, 512], 2, 0.05)
+    x = inputs.bf16_normal(rng, (T, d_in))
+    D = lb.DeviceLinear(L, DEV)
+    ws = lb.new_workspace(lb.workspace_size(D, T), DEV)
+    xin = lb.bf16_tensor(x, DEV)
+
+    def forward():
+        y = torch.full((T, d_out), float("nan"), dtype=torch.float32, device=DEV)
+        lb.linear_forward(D, xin, y=y, ws=ws)
+        torch.cuda.synchronize()
+        return y
+
+    def words():
+        return ws[:16].view(torch.int32).cpu().tolist()
+
+    y0 = forward()
+    rows = np.array([0, 1, 127, 128, 300, T - 1])
+    check(y0.cpu().numpy().astype(np.float64)[rows], oracle.forward_factored(L, x[rows]),
+          torch.float32, 1e-3)
+    assert words()[:3] == [0, 0, 0]
+    z = torch.empty((T, 1024), dtype=torch.float16, device=DEV)
+    for _ in range(3):
+        lb.linear_latent(D, xin, z=z, ws=ws)
+        yc = torch.empty((T, d_out), dtype=torch.float32, device=DEV)
+        lb.linear_expand(D, z, y=yc, ws=ws)
+        torch.cuda.synchronize()
+        assert torch.equal(yc, y0)
+        assert torch.equal(forward(), y0)
+    assert lb.poll_error(ws) == lb.LB_OK
+    assert words()[:3] == [0, 0, 0]
+    lb.selftest_wait_timeout(ws)
+    y = torch.full((T, d_out), float("nan"), dtype=torch.float32, device=DEV)
+    lb.linear_forward(D, xin, y=y, ws=ws)
+    assert lb.poll_error(ws) == lb.LB_ERR_TIMEOUT
+    assert torch.isnan(y).all(), "a kernel wrote outputs while the error word was set"
+    assert words()[:3] == [0, 0, 0]
+    assert torch.equal(forward(), y0)
+    assert lb.poll_error(ws) == lb.LB_OK
+
+
 # ------------------------------------------------------------------ bounded waits
 
 
