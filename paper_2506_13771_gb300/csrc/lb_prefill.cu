@@ -260,6 +260,7 @@ struct PrefillParams {
     float *z32;        // stage 1 output in fp32 instead of z (latent entry point), or null
     float *zpart;      // split stage 1: fp32 partial sums [split][T][N1] (before l)
     int split;         // stage-1 K slices (gridDim.z of stage 1)
+    int pair;          // stage 1 in 128 x 512 column-pair tiles (k_fused)
     int expanded;      // B operands pre-expanded to fp16 (bv, bu): the k_fused path
     uint16_t *bv;      // [N1][d_in]: +-g_p[k] at (column n of path p, input k)
     uint16_t *bu;      // [d_out][N1]: +-h_p[o] at (output o, column n of path p)
@@ -1014,6 +1015,197 @@ __global__ void k_reduce_z(const __grid_constant__ PrefillParams P) {
                    (long long)gridDim.x * blockDim.x);
 }
 
+// Column-pair form of stage 1 for long token runs (N1 a multiple of 512):
+// one CTA computes a 128 x 512 tile as two 256-wide MMAs that share each
+// converted A stage, which halves the shared-memory traffic of A and of the
+// bf16 -> fp16 conversion per flop.  The two accumulators fill all of TMEM,
+// so a tile's epilogue does not overlap the next tile's K loop (stage 1's K
+// loop is long: d_in).  K-stages are 32 wide (64-byte rows, 64-byte
+// swizzle): 8 KB of A and 2 x 16 KB of B, five in the ring.
+constexpr int BK2 = 32;
+constexpr int A2_BYTES = BM * BK2 * 2;
+constexpr int B2_HALF = BN * BK2 * 2;
+constexpr int SB2 = A2_BYTES + 2 * B2_HALF;
+constexpr int NST2 = 5;
+static_assert(NST2 * SB2 + 1024 <= kTilesSmem && NST2 <= kMaxStages, "pair ring");
+
+// Shared-memory matrix descriptor: K-major, 64-byte swizzle, 8-row groups
+// 512 bytes apart, descriptor version 1.
+__device__ __forceinline__ uint64_t smem_desc_sw64(uint32_t saddr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFF) >> 4);  // start address
+    d |= (uint64_t)1 << 16;                    // leading byte offset (unused when swizzled)
+    d |= (uint64_t)(512 >> 4) << 32;           // stride byte offset
+    d |= (uint64_t)1 << 46;                    // version
+    d |= (uint64_t)4 << 61;                    // 64-byte swizzle
+    return d;
+}
+
+__device__ bool run_tiles_pair(const CUtensorMap *amap, const CUtensorMap *bmap,
+                               const PrefillParams &P, int n_pairs, int n_tiles, PhaseBars &B,
+                               uint32_t tmem, unsigned char *smem, volatile int *fail,
+                               bool expand_u_meanwhile) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int KT = P.L.d_in / BK2;
+    const uint32_t idesc = instr_desc(BM, BN);
+    auto give_up = [&]() {
+        *fail = 1;
+        atomicCAS(P.ws_words + kErrWord, 0u, static_cast<unsigned>(LB_ERR_TIMEOUT));
+    };
+    // tile t -> token tile origin m0, column origin n0 (512 columns)
+    auto tile = [&](int t, int &m0, int &n0) {
+        m0 = (t / n_pairs) * BM;
+        n0 = (t % n_pairs) * 2 * BN;
+    };
+    int loads_issued = 0, mmas_issued = 0;
+    auto advance = [&](int &s, unsigned &ph) {
+        if (++s == NST2) {
+            s = 0;
+            ph ^= 1u;
+        }
+    };
+
+    if (warp == 0) {
+        // ---------------- copy warp
+        if (lane == 0) {
+            fence_proxy_async_global();
+            bool ok = true;
+            int s = 0;
+            unsigned ph = 0;
+            for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+                int m0, n0;
+                tile(t, m0, n0);
+                for (int i = 0; i < KT; ++i) {
+                    if (loads_issued >= NST2 && !mb_spin_role(B.empty + s, ph ^ 1u, fail)) {
+                        give_up();
+                        ok = false;
+                        break;
+                    }
+                    uint64_t *b = B.full + s;
+                    unsigned char *st = smem + s * SB2;
+                    mb_expect_tx(b, (unsigned)SB2);
+                    tma_load_2d(st, amap, i * BK2, m0, b);
+                    tma_load_2d(st + A2_BYTES, bmap, i * BK2, n0, b);
+                    tma_load_2d(st + A2_BYTES + B2_HALF, bmap, i * BK2, n0 + BN, b);
+                    ++loads_issued;
+                    advance(s, ph);
+                }
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        // ---------------- MMA warp: both halves of the tile per K-step
+        if (lane == 0) {
+            bool ok = true;
+            int ti = 0, s = 0;
+            unsigned ph = 0;
+            for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x, ++ti) {
+                if (ti >= 1 &&
+                    !mb_spin_role(B.acc_empty, (unsigned)((ti - 1) & 1), fail)) {
+                    give_up();
+                    break;
+                }
+                tc_fence_after();
+                for (int i = 0; i < KT; ++i) {
+                    if (!mb_spin_role(B.ready + s, ph, fail)) {
+                        give_up();
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a0 = su32(smem + s * SB2), b0 = a0 + A2_BYTES;
+#pragma unroll
+                    for (int k = 0; k < BK2 / 16; ++k) {
+                        const uint64_t ad = smem_desc_sw64(a0 + 32 * k);
+                        const uint32_t acc = (i > 0 || k > 0) ? 1u : 0u;
+                        mma_f16(tmem, ad, smem_desc_sw64(b0 + 32 * k), idesc, acc);
+                        mma_f16(tmem + BN, ad, smem_desc_sw64(b0 + B2_HALF + 32 * k), idesc, acc);
+                    }
+                    mma_commit(B.empty + s);
+                    ++mmas_issued;
+                    advance(s, ph);
+                }
+                if (ok) mma_commit(B.acc_full);
+            }
+        }
+        __syncwarp();
+    } else if (warp < 6) {
+        // ---------------- conversion warps: bf16 -> fp16 of each A stage
+        const int tid = threadIdx.x - 64;
+        int s = 0;
+        unsigned ph = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; t < n_tiles && ok; t += gridDim.x) {
+            for (int i = 0; i < KT; ++i, advance(s, ph)) {
+                const bool got = mb_wait_role(B.full + s, ph, fail);
+                if (!__all_sync(0xffffffffu, got)) {
+                    if (lane == 0) give_up();
+                    ok = false;
+                    break;
+                }
+                uint4 *a = reinterpret_cast<uint4 *>(smem + s * SB2);
+                for (int q = tid; q < A2_BYTES / 16; q += 128) {
+                    uint4 u = a[q];
+                    uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float lo = __uint_as_float(w[e] << 16),
+                                    hi = __uint_as_float(w[e] & 0xffff0000u);
+                        const __half2 h = __floats2half2_rn(lo, hi);
+                        w[e] = *reinterpret_cast<const uint32_t *>(&h);
+                    }
+                    a[q] = make_uint4(w[0], w[1], w[2], w[3]);
+                }
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0)
+                    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(B.ready + s))
+                                 : "memory");
+            }
+        }
+    } else {
+        // ---------------- epilogue warps: TMEM lanes 32(w%4) .. +31, all 512 columns
+        const int wq = warp & 3;
+        const uint32_t lane_base = tmem + ((uint32_t)(32 * wq) << 16);
+        if (expand_u_meanwhile)
+            expand_u_items(P, blockIdx.x * 128LL + (threadIdx.x - 192), gridDim.x * 128LL);
+        int ti = 0;
+        for (int t = blockIdx.x; t < n_tiles; t += gridDim.x, ++ti) {
+            int m0, n0;
+            tile(t, m0, n0);
+            const bool got = mb_wait_role(B.acc_full, (unsigned)(ti & 1), fail);
+            if (!__all_sync(0xffffffffu, got)) {
+                if (lane == 0) give_up();
+                break;
+            }
+            tc_fence_after();
+            const int row = m0 + 32 * wq + lane;
+            for (int cb = 0; cb < 2 * BN; cb += 32) {
+                float v[32];
+                tmem_ld32(lane_base + (uint32_t)cb, v);
+                if (row < P.T) store_chunk<true>(P, v, row, n0 + cb, 0, 1);
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0)
+                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(B.acc_empty))
+                             : "memory");
+        }
+    }
+    if (__syncthreads_or(*fail)) {
+        if (threadIdx.x == 0)
+            for (int i = loads_issued - NST2; i < loads_issued; ++i)
+                if (i >= 0) mb_wait(B.full + i % NST2, (unsigned)((i / NST2) & 1));
+        if (threadIdx.x == 32)
+            for (int i = mmas_issued - NST2; i < mmas_issued; ++i)
+                if (i >= 0) mb_wait(B.empty + i % NST2, (unsigned)((i / NST2) & 1));
+        __syncthreads();
+        return false;
+    }
+    return true;
+}
+
+
 // What one launch of k_fused does, in this order: expand V and / or U, stage
 // 1 (and the reduction of its K slices), stage 2.
 enum : int { kDoExpandV = 1, kDoExpandU = 2, kDoStage1 = 4, kDoStage2 = 8 };
@@ -1085,13 +1277,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             // (x or z, inputs of the call) into L2
             const bool s1 = F.flags & kDoStage1;
             const int t = blockIdx.x, tiles_n = s1 ? F.tiles_n1 : F.tiles_n2;
-            const int nsplit = s1 ? F.split : 1, KT = (s1 ? P.L.d_in : P.N1) / BK;
+            const int kstep = (s1 && P.pair) ? BK2 : BK;
+            const int nsplit = s1 ? F.split : 1, KT = (s1 ? P.L.d_in : P.N1) / kstep;
             if (t < (s1 ? F.n_tiles1 : F.n_tiles2)) {
                 const int rest = t / tiles_n, z = rest % nsplit, m0 = (rest / nsplit) * BM;
                 const int kbeg = (int)((long long)z * KT / nsplit);
                 const int kc = (int)((long long)(z + 1) * KT / nsplit) - kbeg;
                 for (int i = 0; i < kc && i < 16; ++i)
-                    tma_prefetch_2d(s1 ? &xmap : &zmap, (kbeg + i) * BK, m0);
+                    tma_prefetch_2d(s1 ? &xmap : &zmap, (kbeg + i) * kstep, m0);
             }
         }
         if (F.flags & kDoExpandV) expand_v_items(P, gi, gn);
@@ -1100,8 +1293,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         ok = grid_barrier(P.ws_words, n_ctas * ++nbar);
     }
     if (ok && (F.flags & kDoStage1)) {
-        ok = run_tiles<true>(&xmap, &bvmap, P, F.tiles_n1, F.split, F.n_tiles1, bars[0], tmem,
-                             smem, fail, u_in_stage1);
+        ok = P.pair ? run_tiles_pair(&xmap, &bvmap, P, F.tiles_n1, F.n_tiles1, bars[0], tmem,
+                                     smem, fail, u_in_stage1)
+                    : run_tiles<true>(&xmap, &bvmap, P, F.tiles_n1, F.split, F.n_tiles1, bars[0],
+                                      tmem, smem, fail, u_in_stage1);
         if (ok && F.split > 1) {
             ok = grid_barrier(P.ws_words, n_ctas * ++nbar);
             if (ok) reduce_z_items(P, gi, gn);
@@ -1147,16 +1342,18 @@ bool encoder() {
     return g_encode != nullptr;
 }
 
-// 2-D map over a row-major [rows][cols] 16-bit matrix, box BK x BM, 128B swizzle,
-// out-of-range rows read as zero.
+// 2-D map over a row-major [rows][cols] 16-bit matrix, box BK x BM with the
+// 128-byte swizzle (or, narrow, BK2 x BM with the 64-byte swizzle of the
+// column-pair stage 1), out-of-range rows read as zero.
 bool make_map(CUtensorMap *m, const void *base, CUtensorMapDataType dt, int64_t rows,
-              int64_t cols, int box_rows = BM) {
+              int64_t cols, int box_rows = BM, bool narrow = false) {
     const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
     const cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
-    const cuuint32_t box[2] = {BK, (cuuint32_t)box_rows};
+    const cuuint32_t box[2] = {(cuuint32_t)(narrow ? BK2 : BK), (cuuint32_t)box_rows};
     const cuuint32_t estr[2] = {1, 1};
     return g_encode(m, dt, 2, const_cast<void *>(base), dims, strides, box, estr,
-                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE,
+                    narrow ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B,
                     CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -1215,7 +1412,10 @@ size_t n1_of(const lb_linear &L) {
 // Stage-1 K slices: enough CTAs to fill about 148 SMs, at least two K-chunks
 // per slice, at most 32 slices (a function of the shapes only, so the
 // workspace size does not depend on the device).
+bool expanded_of(const lb_linear &, int64_t T);
+bool pair_of(const lb_linear &L, int64_t T);
 int split_of(const lb_linear &L, int64_t T) {
+    if (pair_of(L, T)) return 1;
     const int64_t n1 = (int64_t)n1_of(L), bn1 = n1 <= BN ? n1 : BN;
     const int64_t tiles = ((T + BM - 1) / BM) * ((n1 + bn1 - 1) / bn1);
     const int64_t kc = L.d_in / BK;
@@ -1234,6 +1434,12 @@ size_t zpart_bytes(const lb_linear &L, int64_t T) {
 // From four token tiles on, every tile would unpack the same sign bits: the
 // B operands are expanded to fp16 once per call instead (workspace).
 bool expanded_of(const lb_linear &, int64_t T) { return (T + BM - 1) / BM >= 4; }
+// Stage 1 in 128 x 512 column-pair tiles once there are enough of them to
+// fill most SMs without splitting K.
+bool pair_of(const lb_linear &L, int64_t T) {
+    const int64_t n1 = (int64_t)n1_of(L);
+    return expanded_of(L, T) && n1 % (2 * BN) == 0 && ((T + BM - 1) / BM) * (n1 / (2 * BN)) >= 96;
+}
 size_t bv_bytes(const lb_linear &L) { return ((size_t)n1_of(L) * L.d_in * 2 + 255) & ~(size_t)255; }
 size_t bu_bytes(const lb_linear &L) { return ((size_t)L.d_out * n1_of(L) * 2 + 255) & ~(size_t)255; }
 }  // namespace
@@ -1255,6 +1461,7 @@ PrefillParams params_of(const lb_linear &L, int64_t T, unsigned *ws_words, void 
     char *wsb = static_cast<char *>(ws);
     P.z = reinterpret_cast<uint16_t *>(wsb);
     P.split = split_of(L, T);
+    P.pair = pair_of(L, T) ? 1 : 0;
     P.zpart = reinterpret_cast<float *>(wsb + z16_bytes(L, T));
     P.expanded = expanded_of(L, T) ? 1 : 0;
     P.bv = reinterpret_cast<uint16_t *>(wsb + z16_bytes(L, T) + zpart_bytes(L, T));
@@ -1279,7 +1486,8 @@ cudaError_t launch_fused(const CUtensorMap &xmap, const CUtensorMap &bvmap,
 
 // Stage-1 and stage-2 tilings of the persistent phases.
 void plan_stage1(const PrefillParams &P, FusedPlan &F) {
-    const int tm = (P.T + BM - 1) / BM, tn = (P.N1 + P.bn1 - 1) / P.bn1;
+    const int tm = (P.T + BM - 1) / BM;
+    const int tn = P.pair ? P.N1 / (2 * BN) : (P.N1 + P.bn1 - 1) / P.bn1;
     F.tiles_n1 = tn;
     F.split = P.split;
     F.n_tiles1 = tm * tn * P.split;
@@ -1298,9 +1506,10 @@ cudaError_t launch_prefill_latent(const lb_linear &L, const uint16_t *x, int64_t
     P.z = z16;
     P.z32 = z32;
     CUtensorMap xmap, bvmap{}, none{};
-    if (!make_map(&xmap, x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, T, L.d_in)) return cudaErrorInvalidValue;
+    if (!make_map(&xmap, x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, T, L.d_in, BM, P.pair))
+        return cudaErrorInvalidValue;
     if (P.expanded &&
-        !make_map(&bvmap, P.bv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, P.N1, L.d_in, P.bn1))
+        !make_map(&bvmap, P.bv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, P.N1, L.d_in, P.bn1, P.pair))
         return cudaErrorInvalidValue;
     cudaError_t e = set_smem_attributes();
     if (e != cudaSuccess) return e;
@@ -1361,8 +1570,8 @@ cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, voi
     P.y = y;
     P.y_fp32 = y_fp32;
     CUtensorMap xmap, bvmap, zmap, bumap;
-    if (!make_map(&xmap, x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, T, L.d_in) ||
-        !make_map(&bvmap, P.bv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, P.N1, L.d_in, P.bn1) ||
+    if (!make_map(&xmap, x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, T, L.d_in, BM, P.pair) ||
+        !make_map(&bvmap, P.bv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, P.N1, L.d_in, P.bn1, P.pair) ||
         !make_map(&zmap, z16, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, T, P.N1) ||
         !make_map(&bumap, P.bu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, L.d_out, P.N1, BN))
         return cudaErrorInvalidValue;

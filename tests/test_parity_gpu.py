@@ -187,6 +187,45 @@ def test_prefill_tensor_core_shapes(d_in, d_out, rs, T, out_dtype):
     assert np.all(np.isfinite(y)) and e <= (TOL if out_dtype == torch.bfloat16 else 1e-3), e
 
 
+PAIR = [
+    # d_in, d_out, ranks, T: N1 a multiple of 512 and at least 96 column-pair
+    # tiles, ragged last token tile
+    (1024, 264, (512, 512), 6100), (512, 136, (256, 256), 12200), (4096, 512, (512,), 12290),
+]
+
+
+@pytest.mark.parametrize("d_in,d_out,rs,T", PAIR)
+def test_prefill_column_pair_tiles(d_in, d_out, rs, T):
+    """Long token runs with N1 a multiple of 512 take stage 1 in 128 x 512
+    tiles (two 256-wide MMAs per converted x stage, 64-byte swizzle): sampled
+    rows of the forward and of both latent types against the oracle."""
+    rng = inputs.rng_for(109, salt=d_in + T)
+    L = inputs.make_linear(rng, d_in, d_out, list(rs), len(rs), 0.05)
+    x = inputs.bf16_normal(rng, (T, d_in))
+    D = lb.DeviceLinear(L, DEV)
+    ws = lb.new_workspace(lb.workspace_size(D, T), DEV)
+    xin = lb.bf16_tensor(x, DEV)
+    rows = np.unique(np.concatenate([[0, 1, 127, 128, T - 85, T - 1],
+                                     rng.choice(T, 10, replace=False)]))
+    y = torch.full((T, d_out), float("nan"), dtype=torch.float32, device=DEV)
+    lb.linear_forward(D, xin, y=y, ws=ws)
+    torch.cuda.synchronize()
+    yg = y.cpu().numpy().astype(np.float64)
+    assert np.all(np.isfinite(yg))
+    e = rel(yg[rows], oracle.forward_factored(L, x[rows]))
+    assert e <= 1e-3, e
+    z_ref = oracle.latent(L, x[rows])
+    for zt, tol in ((torch.float32, 1e-4), (torch.float16, 1e-3)):
+        z = torch.full((T, sum(rs)), float("nan"), dtype=zt, device=DEV)
+        lb.linear_latent(D, xin, z=z, ws=ws)
+        torch.cuda.synchronize()
+        zg = z.float().cpu().numpy().astype(np.float64)
+        assert np.all(np.isfinite(zg))
+        e = rel(zg[rows], z_ref)
+        assert e <= tol, e
+    assert lb.poll_error(ws) == lb.LB_OK
+
+
 @pytest.mark.parametrize("T", [1, 4])
 def test_padding_bits_are_ignored(T):
     """U words with every padding bit set (r = 33, 16) give the same output."""
