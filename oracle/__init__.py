@@ -96,6 +96,14 @@ def _bind(lib):
     lib.lbo_stack_forward.argtypes = [ctypes.POINTER(Linear), ctypes.c_int32, ctypes.c_int32,
                                       vp, vp, vp, vp]
     lib.lbo_stack_forward.restype = ctypes.c_int
+    lib.lbo_round_bf16.argtypes = [d]
+    lib.lbo_round_bf16.restype = d
+    lib.lbo_rope.argtypes = [vp, i64, i64, d]
+    lib.lbo_rope.restype = None
+    i32 = ctypes.c_int32
+    lib.lbo_decoder_step.argtypes = [ctypes.POINTER(Linear), i32, i32, i32, i32, d, i64, i64, i32,
+                                     vp, vp, vp, vp, vp, vp]
+    lib.lbo_decoder_step.restype = ctypes.c_int
     lib.lbo_bpw.argtypes = [i64, i64, i64, ctypes.c_int32]
     lib.lbo_bpw.restype = d
     lib.lbo_rank_for_bpw.argtypes = [d, i64, i64, ctypes.c_int32]
@@ -296,6 +304,46 @@ class Oracle:
                                       _ptr(kv) if want_kv else None):
             raise MemoryError("oracle stack forward failed")
         return out, q, kv
+
+    # ------------------------------------------------------------ decode step at position p (App. I.3)
+    def round_bf16(self, v) -> np.ndarray:
+        """The nearest bf16 value of each element (ties to even), as float64."""
+        v = np.asarray(v, dtype=np.float64)
+        return np.array([self.lib.lbo_round_bf16(float(e)) for e in v.ravel()]).reshape(v.shape)
+
+    def rope(self, x: np.ndarray, p: int, base: float = 10000.0) -> np.ndarray:
+        """One head rotated to position p (half-split pairing)."""
+        y = _c(np.array(x, dtype=np.float64), np.float64)
+        self.lib.lbo_rope(_ptr(y), y.shape[0], int(p), float(base))
+        return y
+
+    def decoder_step(self, layers: list, shape: dict, pos: int, x_bf16: np.ndarray,
+                     kcache: np.ndarray, vcache: np.ndarray, round_inputs: bool = True,
+                     want_attn: bool = False, want_qk: bool = False):
+        """One decode step at position pos; kcache / vcache [n_layers][max_pos][d_kv]
+        (float64, updated in place at row pos).  shape: n_heads, n_kv_heads,
+        head_dim, rope_base.  Returns (out [d], attn [n_layers][d] or None,
+        qk [n_layers][d + d_kv] or None)."""
+        assert len(layers) % 7 == 0
+        n_layers = len(layers) // 7
+        holders = [_Holder(L) for L in layers]
+        arr = (Linear * len(layers))(*[h.c for h in holders])
+        H, G, D = shape["n_heads"], shape["n_kv_heads"], shape["head_dim"]
+        d, dkv = H * D, G * D
+        assert kcache.dtype == np.float64 and kcache.flags.c_contiguous
+        assert vcache.dtype == np.float64 and vcache.flags.c_contiguous
+        assert kcache.shape == vcache.shape and kcache.shape[0] == n_layers and kcache.shape[2] == dkv
+        x = _c(x_bf16, np.uint16)
+        out = np.zeros(d, dtype=np.float64)
+        attn = np.zeros((n_layers, d)) if want_attn else None
+        qk = np.zeros((n_layers, d + dkv)) if want_qk else None
+        if self.lib.lbo_decoder_step(arr, n_layers, H, G, D, float(shape.get("rope_base", 10000.0)),
+                                     int(pos), kcache.shape[1], 1 if round_inputs else 0,
+                                     _ptr(x), _ptr(kcache), _ptr(vcache), _ptr(out),
+                                     _ptr(attn) if want_attn else None,
+                                     _ptr(qk) if want_qk else None):
+            raise ValueError("decoder_step: position out of range, bad shape or no memory")
+        return out, attn, qk
 
     # ------------------------------------------------------------ Dual-SVID (Sec. 3.2, 3.3)
     def svd_top(self, A: np.ndarray, r: int):

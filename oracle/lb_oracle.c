@@ -412,6 +412,166 @@ done:
 }
 
 /* ------------------------------------------------------------------------ */
+/* Decode step at position p of a Llama-shaped decoder (App. I.3: only the  */
+/* linears are LittleBit; attention and the norms stay dense)              */
+/* ------------------------------------------------------------------------ */
+
+/* The bf16 value nearest to v, ties to the even significand: bf16 keeps 8
+ * significant bits, so v = m 2^e with 0.5 <= |m| < 1 is rounded to a
+ * multiple of 2^(e - 8) (the exponent floor -125 covers the subnormals).
+ * This is the rounding applied to the input of each LittleBit linear when the
+ * GPU feeds it bf16. */
+double lbo_round_bf16(double v)
+{
+    if (v == 0.0 || !isfinite(v))
+        return v;
+    int e;
+    frexp(v, &e);
+    if (e < -125)
+        e = -125;
+    double q = ldexp(1.0, e - 8);
+    double t = v / q, f = floor(t), rem = t - f;
+    double n = f;
+    if (rem > 0.5 || (rem == 0.5 && fmod(f, 2.0) != 0.0))
+        n = f + 1.0;
+    return n * q;
+}
+
+/* Rotary position embedding of one head of width D at position p (the
+ * half-split pairing): for i < D/2, (x_i, x_{i + D/2}) is rotated by
+ * theta_i = p * base^(-2i / D). */
+void lbo_rope(double *x, int64_t D, int64_t p, double base)
+{
+    int64_t h = D / 2;
+    for (int64_t i = 0; i < h; i++) {
+        double th = (double)p * pow(base, -2.0 * (double)i / (double)D);
+        double c = cos(th), sn = sin(th), a = x[i], b = x[i + h];
+        x[i] = a * c - b * sn;
+        x[i + h] = a * sn + b * c;
+    }
+}
+
+/* One decode step: the token x (bf16 [d]) at position pos, with the keys and
+ * values of positions 0 .. pos-1 in the caches ([n_layers][max_pos][d_kv],
+ * d_kv = n_kv_heads * head_dim; this step writes row pos of every layer).
+ * Per layer, with rho the unit-weight RMS normalisation:
+ *   n = rho(a); q, k, v = Q(n), K(n), V(n); q, k rotated (lbo_rope) per head
+ *   cache[pos] = (k, v); per query head h of kv head g = h / (n_heads / n_kv_heads)
+ *   s_t = q_h . k_t,g / sqrt(head_dim), w = softmax_t(s) over t = 0..pos,
+ *   attn_h = sum_t w_t v_t,g;  a += O(attn)
+ *   n = rho(a); a += Down(silu(Gate(n)) . Up(n))
+ * round_inputs = 1 rounds n, attn and the MLP product to bf16 before their
+ * linears (lbo_round_bf16), as the GPU feeds them; 0 keeps them exact.
+ * Optional outputs per layer: attn_out [n_layers][d], qk_out [n_layers][d + d_kv]
+ * (the rotated q and k).  0, or -1 (pos out of range or no memory). */
+int lbo_decoder_step(const lbo_linear *lin, int32_t n_layers, int32_t n_heads,
+                     int32_t n_kv_heads, int32_t head_dim, double rope_base, int64_t pos,
+                     int64_t max_pos, int32_t round_inputs, const uint16_t *x, double *kcache,
+                     double *vcache, double *out, double *attn_out, double *qk_out)
+{
+    int64_t d = (int64_t)n_heads * head_dim, dkv = (int64_t)n_kv_heads * head_dim;
+    int64_t dff = lin[4].d_out, group = n_heads / n_kv_heads;
+    if (pos < 0 || pos >= max_pos || n_kv_heads <= 0 || n_heads % n_kv_heads != 0)
+        return -1;
+    double *a = decode_bf16_array(x, d);
+    double *n = (double *)malloc((size_t)d * sizeof(double));
+    double *q = (double *)malloc((size_t)d * sizeof(double));
+    double *k = (double *)malloc((size_t)dkv * sizeof(double));
+    double *v = (double *)malloc((size_t)dkv * sizeof(double));
+    double *attn = (double *)malloc((size_t)d * sizeof(double));
+    double *o = (double *)malloc((size_t)d * sizeof(double));
+    double *gt = (double *)malloc((size_t)dff * sizeof(double));
+    double *up = (double *)malloc((size_t)dff * sizeof(double));
+    double *w = (double *)malloc((size_t)(pos + 1) * sizeof(double));
+    int rc = -1;
+    if (!a || !n || !q || !k || !v || !attn || !o || !gt || !up || !w)
+        goto done;
+    for (int32_t layer = 0; layer < n_layers; layer++) {
+        const lbo_linear *L = &lin[7 * (int64_t)layer];
+        double *Kc = kcache + (int64_t)layer * max_pos * dkv;
+        double *Vc = vcache + (int64_t)layer * max_pos * dkv;
+        rms_normalize(a, d, n);
+        if (round_inputs)
+            for (int64_t i = 0; i < d; i++)
+                n[i] = lbo_round_bf16(n[i]);
+        if (lbo_apply_factored(&L[0], n, 1, q, NULL) || lbo_apply_factored(&L[1], n, 1, k, NULL) ||
+            lbo_apply_factored(&L[2], n, 1, v, NULL))
+            goto done;
+        for (int32_t h = 0; h < n_heads; h++)
+            lbo_rope(q + (int64_t)h * head_dim, head_dim, pos, rope_base);
+        for (int32_t g = 0; g < n_kv_heads; g++)
+            lbo_rope(k + (int64_t)g * head_dim, head_dim, pos, rope_base);
+        if (qk_out) {
+            memcpy(qk_out + (int64_t)layer * (d + dkv), q, (size_t)d * sizeof(double));
+            memcpy(qk_out + (int64_t)layer * (d + dkv) + d, k, (size_t)dkv * sizeof(double));
+        }
+        memcpy(Kc + pos * dkv, k, (size_t)dkv * sizeof(double));
+        memcpy(Vc + pos * dkv, v, (size_t)dkv * sizeof(double));
+        for (int32_t h = 0; h < n_heads; h++) {
+            int64_t g = h / group;
+            const double *qh = q + (int64_t)h * head_dim;
+            double mx = -INFINITY, sum = 0.0;
+            for (int64_t t = 0; t <= pos; t++) {
+                double s = 0.0;
+                for (int64_t c = 0; c < head_dim; c++)
+                    s += qh[c] * Kc[t * dkv + g * head_dim + c];
+                w[t] = s / sqrt((double)head_dim);
+                if (w[t] > mx)
+                    mx = w[t];
+            }
+            for (int64_t t = 0; t <= pos; t++) {
+                w[t] = exp(w[t] - mx);
+                sum += w[t];
+            }
+            for (int64_t c = 0; c < head_dim; c++) {
+                double acc = 0.0;
+                for (int64_t t = 0; t <= pos; t++)
+                    acc += w[t] * Vc[t * dkv + g * head_dim + c];
+                attn[(int64_t)h * head_dim + c] = acc / sum;
+            }
+        }
+        if (attn_out)
+            memcpy(attn_out + (int64_t)layer * d, attn, (size_t)d * sizeof(double));
+        if (round_inputs)
+            for (int64_t i = 0; i < d; i++)
+                attn[i] = lbo_round_bf16(attn[i]);
+        if (lbo_apply_factored(&L[3], attn, 1, o, NULL))
+            goto done;
+        for (int64_t i = 0; i < d; i++)
+            a[i] += o[i];
+        rms_normalize(a, d, n);
+        if (round_inputs)
+            for (int64_t i = 0; i < d; i++)
+                n[i] = lbo_round_bf16(n[i]);
+        if (lbo_apply_factored(&L[4], n, 1, gt, NULL) || lbo_apply_factored(&L[5], n, 1, up, NULL))
+            goto done;
+        for (int64_t i = 0; i < dff; i++) {
+            gt[i] = silu(gt[i]) * up[i];
+            if (round_inputs)
+                gt[i] = lbo_round_bf16(gt[i]);
+        }
+        if (lbo_apply_factored(&L[6], gt, 1, o, NULL))
+            goto done;
+        for (int64_t i = 0; i < d; i++)
+            a[i] += o[i];
+    }
+    memcpy(out, a, (size_t)d * sizeof(double));
+    rc = 0;
+done:
+    free(a);
+    free(n);
+    free(q);
+    free(k);
+    free(v);
+    free(attn);
+    free(o);
+    free(gt);
+    free(up);
+    free(w);
+    return rc;
+}
+
+/* ------------------------------------------------------------------------ */
 /* Dual-SVID initialisation (Sec. 3.2) and Residual Compensation (Sec. 3.3)  */
 /* ------------------------------------------------------------------------ */
 

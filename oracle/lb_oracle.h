@@ -147,6 +147,17 @@ double lbo_rank_for_bpw(double b, int64_t d_out, int64_t d_in, int32_t n_paths);
 double lbo_flops(int64_t T, int64_t d_out, int64_t d_in, int64_t r, int32_t n_paths);
 
 /* Threads used by the OpenMP loops (0 = the OpenMP default). */
+/* Decode step at position pos of a Llama-shaped decoder (App. I.3): RMS
+ * norms, rotary embedding, softmax attention over the KV cache, SiLU MLP,
+ * residual stream; the linears are LittleBit (lin[7 * layer + 0..6] = q, k,
+ * v, o, gate, up, down).  See lb_oracle.c for the exact definition. */
+double lbo_round_bf16(double v);
+void lbo_rope(double *x, int64_t D, int64_t p, double base);
+int lbo_decoder_step(const lbo_linear *lin, int32_t n_layers, int32_t n_heads,
+                     int32_t n_kv_heads, int32_t head_dim, double rope_base, int64_t pos,
+                     int64_t max_pos, int32_t round_inputs, const uint16_t *x, double *kcache,
+                     double *vcache, double *out, double *attn_out, double *qk_out);
+
 void lbo_set_threads(int32_t n);
 int32_t lbo_get_threads(void);
 

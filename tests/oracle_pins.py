@@ -775,6 +775,184 @@ def pin_stack_attention_closed_form(orc):
     assert rel(out, a) <= 1e-13, rel(out, a)
 
 
+# ------------------------------------------------------------------ pins: decode step at position p
+
+
+def _bf16_rne_of_f32(f32: np.ndarray) -> np.ndarray:
+    """bf16 rounding of float32 values by the integer carry trick (ties to even)."""
+    u = np.asarray(f32, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    r = ((u + 0x7FFF + ((u >> 16) & 1)) >> 16) << 16
+    return r.astype(np.uint32).view(np.float32).astype(np.float64)
+
+
+def pin_round_bf16(orc):
+    """Nearest-even bf16 rounding: equal to the integer carry trick on float32
+    inputs (random values, exact ties with even and odd kept bits, tiny and
+    subnormal magnitudes); for float64 inputs between float32 values the
+    result is a bf16 value within half a bf16 step, and just above a tie it
+    rounds away from the tie's even neighbour."""
+    rng = np.random.default_rng(30)
+    f = np.concatenate([rng.standard_normal(3000) * 10.0 ** rng.integers(-30, 30, 3000),
+                        rng.standard_normal(200) * 1e-39]).astype(np.float32)
+    # exact ties: the low 16 bits of finite float32 values set to 0x8000, with
+    # the last kept bit both even and odd
+    u = (rng.standard_normal(400).astype(np.float32).view(np.uint32) & 0xFFFF0000) | 0x8000
+    ties = np.concatenate([u, u ^ 0x00010000]).view(np.float32)
+    f = np.concatenate([f, ties])
+    assert np.array_equal(orc.round_bf16(f.astype(np.float64)), _bf16_rne_of_f32(f))
+    v = rng.standard_normal(500) * 3.0
+    r = orc.round_bf16(v)
+    assert np.array_equal(_bf16_rne_of_f32(r.astype(np.float32)), r)  # representable
+    e = np.floor(np.log2(np.abs(v)))
+    assert np.all(np.abs(v - r) <= np.ldexp(1.0, (e - 8).astype(int)) * (1 + 1e-12))
+    # 1 + 2^-8 is a tie between 1 and 1 + 2^-7 (kept bit even: down); a hair above it rounds up
+    assert orc.round_bf16(1 + 2.0 ** -8) == 1.0
+    assert orc.round_bf16(1 + 2.0 ** -8 + 2.0 ** -40) == 1 + 2.0 ** -7
+
+
+def pin_rope(orc):
+    """Rotary embedding: the half-split pairing and frequencies on unit vectors
+    (closed forms), identity at position 0, norm preservation, composition of
+    rotations, and scores that depend only on the position difference."""
+    c1, s1 = np.cos(1.0), np.sin(1.0)
+    assert np.allclose(orc.rope([1.0, 0.0], 1), [c1, s1], rtol=0, atol=1e-15)
+    assert np.allclose(orc.rope([1.0, 0.0, 0.0, 0.0], 1), [c1, 0.0, s1, 0.0], rtol=0, atol=1e-15)
+    th = 10000.0 ** -0.5
+    assert np.allclose(orc.rope([0.0, 1.0, 0.0, 0.0], 1), [0.0, np.cos(th), 0.0, np.sin(th)],
+                       rtol=0, atol=1e-15)
+    assert np.allclose(orc.rope([0.0, 0.0, 0.0, 1.0], 3), [0.0, -np.sin(3 * th), 0.0, np.cos(3 * th)],
+                       rtol=0, atol=1e-15)
+    rng = np.random.default_rng(31)
+    x, y = rng.standard_normal(128), rng.standard_normal(128)
+    assert np.array_equal(orc.rope(x, 0), x)
+    assert abs(np.linalg.norm(orc.rope(x, 77)) - np.linalg.norm(x)) <= 1e-12
+    assert np.allclose(orc.rope(orc.rope(x, 5), 9), orc.rope(x, 14), rtol=0, atol=1e-12)
+    for p, t, sh in ((9, 3, 40), (100, 0, 7), (5, 5, 1000)):
+        a = orc.rope(x, p) @ orc.rope(y, t)
+        b = orc.rope(x, p + sh) @ orc.rope(y, t + sh)
+        assert abs(a - b) <= 1e-10 * (1 + abs(a)), (a, b)
+
+
+DEC = {"n_heads": 8, "n_kv_heads": 2, "head_dim": 8, "rope_base": 10000.0}
+
+
+def _decode_tokens(orc, layers, xs, max_pos, round_inputs=True):
+    n_layers = len(layers) // 7
+    dkv = layers[1]["d_out"]
+    kc = np.zeros((n_layers, max_pos, dkv))
+    vc = np.zeros((n_layers, max_pos, dkv))
+    outs = []
+    for p, x in enumerate(xs):
+        outs.append(orc.decoder_step(layers, DEC, p, x, kc, vc, round_inputs)[0])
+    return outs, kc, vc
+
+
+def pin_decoder_pos0_is_stack(orc):
+    """At position 0 (exact inputs) the rotation is the identity and the
+    softmax of one score is 1: the step equals the position-0 stack chain."""
+    rng = np.random.default_rng(32)
+    layers, x0 = small_stack(rng)
+    out_s, _, kv = orc.stack_forward(layers, x0, head_dim=8)
+    kc = np.zeros((3, 4, 16))
+    vc = np.zeros((3, 4, 16))
+    out, _, _ = orc.decoder_step(layers, DEC, 0, x0, kc, vc, round_inputs=False)
+    assert rel(out, out_s) <= 1e-12, rel(out, out_s)
+    assert rel(kc[:, 0], kv[:, 0]) <= 1e-12 and rel(vc[:, 0], kv[:, 1]) <= 1e-12
+    assert not kc[:, 1:].any() and not vc[:, 1:].any()
+
+
+def pin_decoder_composition(orc):
+    """Step 3 rebuilt from single-linear oracle calls, numpy RMS, the pinned
+    bf16 rounding and rotation, and textbook attention over cache rows 0..3."""
+    rng = np.random.default_rng(33)
+    layers, _ = small_stack(rng)
+    xs = [inputs_bf16(rng, 64) for _ in range(4)]
+    _, kc, vc = _decode_tokens(orc, layers, xs[:3], 6)
+    kc0, vc0 = kc.copy(), vc.copy()
+    out, attn, qk = orc.decoder_step(layers, DEC, 3, xs[3], kc, vc, True, True, True)
+    a = np_bf16(xs[3])
+    D = DEC["head_dim"]
+    for l in range(3):
+        Q, K, V, O, G, Up, Dn = layers[7 * l:7 * l + 7]
+        n = orc.round_bf16(_rho(a))[None, :]
+        q = orc.apply_factored(Q, n)[0]
+        k = orc.apply_factored(K, n)[0]
+        v = orc.apply_factored(V, n)[0]
+        q = np.concatenate([orc.rope(q[h * D:(h + 1) * D], 3) for h in range(8)])
+        k = np.concatenate([orc.rope(k[g * D:(g + 1) * D], 3) for g in range(2)])
+        assert rel(qk[l], np.concatenate([q, k])) <= 1e-12
+        assert rel(kc[l, 3], k) <= 1e-12 and rel(vc[l, 3], v) <= 1e-12
+        assert np.array_equal(kc[l, :3], kc0[l, :3]) and not kc[l, 4:].any()
+        at = _attention(q, np.vstack([kc0[l, :3], k]), np.vstack([vc0[l, :3], v]), D)
+        assert rel(attn[l], at) <= 1e-12, rel(attn[l], at)
+        h = a + orc.apply_factored(O, orc.round_bf16(at)[None, :])[0]
+        n = orc.round_bf16(_rho(h))[None, :]
+        gt = orc.apply_factored(G, n)[0]
+        m = orc.round_bf16(gt / (1.0 + np.exp(-gt)) * orc.apply_factored(Up, n)[0])
+        a = h + orc.apply_factored(Dn, m[None, :])[0]
+    assert rel(out, a) <= 1e-12, rel(out, a)
+
+
+def inputs_bf16(rng, n):
+    return rand_x(rng, 1, n)[0]
+
+
+def pin_decoder_attention_closed_forms(orc):
+    """One layer, two kv heads shared by four query heads each.  (a) Cached
+    keys equal to the new key: uniform weights, each head reads the mean of
+    its kv head's values.  (b) Position 1 with a zero key at row 0: the
+    weights are a logistic function of q . k / sqrt(head_dim)."""
+    rng = np.random.default_rng(34)
+    layers, _ = small_stack(rng, n_layers=1)
+    x = inputs_bf16(rng, 64)
+    D, p = DEC["head_dim"], 5
+    kc = np.zeros((1, 8, 16))
+    vc = rng.standard_normal((1, 8, 16))
+    _, _, qk = orc.decoder_step(layers, DEC, p, x, kc.copy(), vc.copy(), True, False, True)
+    kc[0, :p] = qk[0, 64:]
+    _, attn, _ = orc.decoder_step(layers, DEC, p, x, kc, vc, True, True, False)
+    for h in range(8):
+        g = h // 4
+        want = vc[0, :p + 1, g * D:(g + 1) * D].mean(axis=0)
+        assert rel(attn[0, h * D:(h + 1) * D], want) <= 1e-12
+    kc = np.zeros((1, 4, 16))
+    vc = np.zeros((1, 4, 16))
+    vc[0, 0] = rng.standard_normal(16)
+    _, attn, qk = orc.decoder_step(layers, DEC, 1, x, kc, vc, True, True, True)
+    q, k = qk[0, :64], qk[0, 64:]
+    for h in range(8):
+        g = h // 4
+        s = q[h * D:(h + 1) * D] @ k[g * D:(g + 1) * D] / np.sqrt(D)
+        w1 = 1.0 / (1.0 + np.exp(-s))
+        want = (1 - w1) * vc[0, 0, g * D:(g + 1) * D] + w1 * vc[0, 1, g * D:(g + 1) * D]
+        assert rel(attn[0, h * D:(h + 1) * D], want) <= 1e-12
+
+
+def pin_decoder_causal(orc):
+    """Cache rows after the current position are never read (NaN there
+    changes nothing), and position max_pos is refused."""
+    rng = np.random.default_rng(35)
+    layers, _ = small_stack(rng, n_layers=2)
+    xs = [inputs_bf16(rng, 64) for _ in range(3)]
+    outs, kc, vc = _decode_tokens(orc, layers, xs, 5)
+    kc2, vc2 = kc.copy(), vc.copy()
+    kc2[:, 3:] = np.nan
+    vc2[:, 3:] = np.nan
+    kc[:, 2:] = 0.0
+    vc[:, 2:] = 0.0
+    kc2[:, 2] = 0.0
+    vc2[:, 2] = 0.0
+    a = orc.decoder_step(layers, DEC, 2, xs[2], kc, vc)[0]
+    b = orc.decoder_step(layers, DEC, 2, xs[2], kc2, vc2)[0]
+    assert np.all(np.isfinite(b)) and np.array_equal(a, b) and np.array_equal(a, outs[2])
+    try:
+        orc.decoder_step(layers, DEC, 5, xs[0], kc, vc)
+    except ValueError:
+        pass
+    else:
+        raise AssertionError("position max_pos accepted")
+
+
 ALL_PINS = [pin_fp16_exhaustive, pin_bf16_exhaustive, pin_pack_structured, pin_pack_vs_numpy,
             pin_dense_equals_factored, pin_rank1_closed_form, pin_all_equal_signs,
             pin_hadamard_identity, pin_brute_force, pin_residual_paths, pin_padding_ignored,
@@ -783,4 +961,6 @@ ALL_PINS = [pin_fp16_exhaustive, pin_bf16_exhaustive, pin_pack_structured, pin_p
             pin_kv_cache_table4, pin_svd_top_vs_numpy, pin_dual_svid_rank1,
             pin_dual_svid_hadamard, pin_dual_svid_vs_lapack, pin_train_forward_is_inference,
             pin_train_backward_central_differences, pin_smoothsign_factor, pin_stack_chain,
-            pin_stack_zero_branches, pin_stack_attention_closed_form]
+            pin_stack_zero_branches, pin_stack_attention_closed_form, pin_round_bf16, pin_rope,
+            pin_decoder_pos0_is_stack, pin_decoder_composition,
+            pin_decoder_attention_closed_forms, pin_decoder_causal]

@@ -69,6 +69,25 @@ MUTATIONS = [
     ("qat_dx_drops_g", "dX[ti] += da[ti] * P->g[ti % din];", "dX[ti] += da[ti];"),
     ("qat_dl_index", "s += dz[tt * r + j] * t[tt * r + j];", "s += dz[tt * r + j] * t[tt * r + (r - 1 - j)];"),
     ("flops_factor", "return (double)n_paths * 2.0 * (double)T", "return (double)n_paths * 1.0 * (double)T"),
+    ("bf16_ties_away", "if (rem > 0.5 || (rem == 0.5 && fmod(f, 2.0) != 0.0))", "if (rem >= 0.5)"),
+    ("bf16_one_bit_short", "double q = ldexp(1.0, e - 8);", "double q = ldexp(1.0, e - 7);"),
+    ("rope_frequency", "double th = (double)p * pow(base, -2.0 * (double)i / (double)D);",
+     "double th = (double)p * pow(base, -1.0 * (double)i / (double)D);"),
+    ("rope_rotation_sign", "x[i] = a * c - b * sn;", "x[i] = a * c + b * sn;"),
+    ("rope_interleaved", "double c = cos(th), sn = sin(th), a = x[i], b = x[i + h];",
+     "double c = cos(th), sn = sin(th), a = x[i], b = x[(i + 1) % D];"),
+    ("attn_no_scale", "w[t] = s / sqrt((double)head_dim);", "w[t] = s;"),
+    ("attn_group_index", "int64_t g = h / group;", "int64_t g = h % n_kv_heads;"),
+    ("attn_not_normalised", "attn[(int64_t)h * head_dim + c] = acc / sum;",
+     "attn[(int64_t)h * head_dim + c] = acc;"),
+    ("attn_skips_new_row", "for (int64_t t = 0; t <= pos; t++) {\n                double s = 0.0;",
+     "for (int64_t t = 0; t < pos; t++) {\n                double s = 0.0;"),
+    ("decoder_cache_row", "memcpy(Kc + pos * dkv, k, (size_t)dkv * sizeof(double));",
+     "memcpy(Kc + 0 * dkv, k, (size_t)dkv * sizeof(double));"),
+    ("decoder_unrounded_attn", "                attn[i] = lbo_round_bf16(attn[i]);",
+     "                attn[i] = attn[i];"),
+    ("decoder_k_not_rotated", "            lbo_rope(k + (int64_t)g * head_dim, head_dim, pos, rope_base);",
+     "            (void)g;"),
 ]
 
 
