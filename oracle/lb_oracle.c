@@ -546,7 +546,7 @@ int lbo_decoder_step(const lbo_linear *lin, int32_t n_layers, int32_t n_heads,
         if (lbo_apply_factored(&L[4], n, 1, gt, NULL) || lbo_apply_factored(&L[5], n, 1, up, NULL))
             goto done;
         for (int64_t i = 0; i < dff; i++) {
-            gt[i] = silu(gt[i]) * up[i];
+            gt[i] = up[i] * silu(gt[i]);
             if (round_inputs)
                 gt[i] = lbo_round_bf16(gt[i]);
         }

@@ -86,6 +86,7 @@ MUTATIONS = [
      "memcpy(Kc + 0 * dkv, k, (size_t)dkv * sizeof(double));"),
     ("decoder_unrounded_attn", "                attn[i] = lbo_round_bf16(attn[i]);",
      "                attn[i] = attn[i];"),
+    ("decoder_no_silu", "gt[i] = up[i] * silu(gt[i]);", "gt[i] = up[i] * gt[i];"),
     ("decoder_k_not_rotated", "            lbo_rope(k + (int64_t)g * head_dim, head_dim, pos, rope_base);",
      "            (void)g;"),
 ]
