@@ -61,7 +61,7 @@ def parse_args():
     ap.add_argument("--layers", type=int, default=80,
                     help="stack depth (80 = the Llama2-70B workload; smaller only for profiling)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--config", type=int, choices=[2, 3, 4, 6, 7, 8], default=None,
+    ap.add_argument("--config", type=int, choices=[2, 3, 4, 6, 7, 8, 9], default=None,
                     help="time a single-linear workload instead of the stack")
     ap.add_argument("--only", default=None,
                     help="with --config: only the cases whose 'name:T' contains this text")
@@ -646,6 +646,64 @@ def run_config(args):
                                  "frac": flops / ms / 1e9 / tf32_peak,
                                  "peak_source": "MEASURED_PEAKS.json bf16_tflops x 1.1/2.25 (TF32)"}}
             print(json.dumps(line), flush=True)
+    elif args.config == 9:
+        # end-to-end decoding of a Llama2-7B-shaped decoder whose linears are
+        # LittleBit (the paper's tokens-per-second setting, shape only): 128
+        # and 256 new tokens from an empty cache, one decode step per token
+        # replayed as a CUDA graph (inputs resident; the step's 353 launches
+        # are the per-token critical path)
+        S = inputs.DECODER_7B
+        for n_new in (128, 256):
+            name = f"llama2-7b-shape {n_new} new tokens"
+            if not wanted(name, n_new):
+                continue
+            layers, xs = inputs.decoder7b(n_new)
+            dec = lb.DeviceDecoder(layers, S["n_heads"], S["n_kv_heads"], S["head_dim"], n_new,
+                                   10000.0, dev)
+            xt = lb.bf16_tensor(xs, dev)
+            x_static = torch.empty(S["d_model"], dtype=torch.bfloat16, device=dev)
+            out = torch.empty(S["d_model"], dtype=torch.float32, device=dev)
+            x_static.copy_(xt[0])
+            dec.step(x_static, out)  # warm-up outside the capture
+            torch.cuda.synchronize(dev)
+            cs = torch.cuda.Stream(device=dev)
+            with torch.cuda.stream(cs):
+                graph = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(graph, stream=cs):
+                    dec.step(x_static, out, stream=cs)
+            runs = []
+            for _ in range(2):
+                dec.pos.zero_()
+                dec.kcache.zero_()
+                dec.vcache.zero_()
+                torch.cuda.synchronize(dev)
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record()
+                for t in range(n_new):
+                    x_static.copy_(xt[t])
+                    graph.replay()
+                e1.record()
+                torch.cuda.synchronize(dev)
+                runs.append(e0.elapsed_time(e1))
+            if dec.poll_error() != lb.LB_OK or int(dec.pos.item()) != n_new:
+                raise RuntimeError("decoder reported an error")
+            ms = min(runs)
+            # bytes per run: every linear's words and scales per token, plus the
+            # cache rows read (positions 0..p-1 of keys and values, fp32) and written
+            wbytes = dec.nbytes * n_new
+            cache = 4 * 2 * S["n_layers"] * S["d_kv"] * (n_new * (n_new - 1) // 2 + n_new)
+            gbs = (wbytes + cache) / ms / 1e6
+            line = {"config": 9, "case": name, "op": "decode", "tokens": n_new, "ms": ms,
+                    "tokens_per_s": n_new / ms * 1e3, "ms_per_token": ms / n_new,
+                    "bytes_per_token": (wbytes + cache) / n_new, "gbs": gbs,
+                    "launches_per_token": 1 + 11 * S["n_layers"],
+                    "roofline": {"bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s",
+                                 "frac": gbs / hbm, "peak_source": "MEASURED_PEAKS.json hbm_gbs"},
+                    "context": "paper Table 12 (A100, Llama2-7B, 0.1 BPW, 128 new tokens): 203.20 "
+                               "tokens/s; other hardware and a trained model"}
+            print(json.dumps(line), flush=True)
+            del dec, graph
     elif args.config == 6:
         # latent states (KV cache compression): the 70B key projection's latent
         # for one new token and the expansion of a 4096-token latent cache

@@ -69,7 +69,8 @@ typedef enum {
     LB_ERR_TIMEOUT = 4,      /* a device-side grid wait ran out (see poll) */
     LB_ERR_WORKSPACE = 5,    /* ws is NULL, misaligned or too small */
     LB_ERR_PLAN = 6,         /* stack workspace not prepared for these linears */
-    LB_ERR_RANGE = 7         /* a stack intermediate left the exchange's range */
+    LB_ERR_RANGE = 7         /* a stack intermediate left the exchange's range, or a
+                                decode position lies outside the KV cache */
 } lb_status;
 
 typedef enum { LB_OUT_BF16 = 0, LB_OUT_FP32 = 1 } lb_out_dtype;
@@ -289,6 +290,56 @@ lb_status littlebit_stack_prepare(const lb_linear *lin, int32_t n_layers, int32_
 lb_status littlebit_stack_forward(const lb_linear *lin, int32_t n_layers, int32_t head_dim,
                                   const uint16_t *x0, float *out, float *q_out, float *kv_out,
                                   void *ws, size_t ws_bytes, lb_stream_t stream);
+
+/* ---------------------------------------------------------------- decode at position p
+ * The paper's end-to-end decoding setting (App. I.3, Table 12: Llama2
+ * decoding with only nn.Linear replaced by LittleBit, attention and the norms
+ * left dense) as one decode step at any position p of a KV cache.
+ * n_heads query heads and n_kv_heads key/value heads of head_dim dimensions:
+ * d = n_heads * head_dim, d_kv = n_kv_heads * head_dim.  The linears are
+ * lin[7*l + {0..6}] = q, k, v, o, gate, up, down of layer l (HOST array of
+ * structs holding device pointers), shapes as for littlebit_stack_forward
+ * and the same in every layer (else LB_ERR_UNSUPPORTED). */
+typedef struct {
+    int32_t n_layers, n_heads, n_kv_heads;
+    int32_t head_dim;   /* 64, 128 or 256 */
+    int32_t max_pos;    /* KV cache rows per layer, 1 .. 8192 */
+    float rope_base;    /* rotary base, > 1 (10000 for Llama 2) */
+} lb_decoder_shape;
+
+/* Workspace bytes littlebit_decoder_step needs (0 if the arguments are invalid). */
+size_t littlebit_decoder_workspace_size(const lb_linear *lin, const lb_decoder_shape *S);
+
+/* One decode step of the token x (bf16 [d]) at position p = *pos (a DEVICE
+ * int32, read by the step's kernels and incremented by its last one, so the
+ * same sequence of launches serves every token and can be captured once as a
+ * CUDA graph).  With rho(v) = v / sqrt(mean(v^2)) and a = x, each layer:
+ *     n = rho(a);  q, k, v = Q(n), K(n), V(n)
+ *     rotary embedding of q and k at p, per head: the pair (i, i + head_dim/2)
+ *       rotated by theta_i = p * rope_base^(-2i/head_dim)
+ *     kcache[l][p] = k;  vcache[l][p] = v
+ *     attn_h = sum_{t<=p} softmax_t(q_h . k_{t,g} / sqrt(head_dim)) v_{t,g},
+ *       g = h / (n_heads / n_kv_heads)
+ *     a += O(attn);  n = rho(a);  a += Down(silu(Gate(n)) * Up(n))
+ * All activations are fp32 (the linears take them as fp32 inputs).  kcache,
+ * vcache: fp32 [n_layers][max_pos][d_kv]; rows < p must hold the earlier
+ * steps' keys and values, rows > p are not read.  out: fp32 [d], the last a.
+ * A position outside [0, max_pos) records LB_ERR_RANGE in the decoder
+ * workspace's error word and the step writes nothing (read it with
+ * littlebit_decoder_poll_error).  Every linear's d_out and ranks must be
+ * multiples of 8 (else LB_ERR_UNSUPPORTED).  ws: zero-filled before first
+ * use, not shared with concurrent calls.  Enqueues 1 + 11 * n_layers
+ * launches on the stream: seven single-token LittleBit linears per layer
+ * (the cooperative kernel of littlebit_linear_forward at T = 1) and the
+ * attention, norm and SiLU kernels. */
+lb_status littlebit_decoder_step(const lb_linear *lin, const lb_decoder_shape *S,
+                                 const uint16_t *x, float *kcache, float *vcache, int32_t *pos,
+                                 float *out, void *ws, size_t ws_bytes, lb_stream_t stream);
+
+/* littlebit_poll_error over a decoder workspace: the step's own error word
+ * and each linear's, all cleared; returns the first error found, or LB_OK. */
+lb_status littlebit_decoder_poll_error(const lb_linear *lin, const lb_decoder_shape *S, void *ws,
+                                       lb_stream_t stream);
 
 /* The forward of littlebit_linear_forward for callers that cannot allocate
  * device memory.  The paper has no counterpart: this exists for hosts such as

@@ -461,7 +461,8 @@ void lbo_rope(double *x, int64_t D, int64_t p, double base)
  *   attn_h = sum_t w_t v_t,g;  a += O(attn)
  *   n = rho(a); a += Down(silu(Gate(n)) . Up(n))
  * round_inputs = 1 rounds n, attn and the MLP product to bf16 before their
- * linears (lbo_round_bf16), as the GPU feeds them; 0 keeps them exact.
+ * linears (lbo_round_bf16): the chain with bf16 linear inputs; 0 keeps every
+ * activation exact (the GPU decode step keeps them in fp32).
  * Optional outputs per layer: attn_out [n_layers][d], qk_out [n_layers][d + d_kv]
  * (the rotated q and k).  0, or -1 (pos out of range or no memory). */
 int lbo_decoder_step(const lbo_linear *lin, int32_t n_layers, int32_t n_heads,

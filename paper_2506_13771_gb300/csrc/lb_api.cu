@@ -207,7 +207,7 @@ lb_status littlebit_linear_forward(const lb_linear *L, const uint16_t *x, int64_
     float *data = reinterpret_cast<float *>(static_cast<char *>(ws) + linear_data_offset(*L));
     const int fp32 = y_dtype == LB_OUT_FP32;
     if (use_decode(*L, T) && lb::decode_supported(*L, sms)) {
-        cudaError_t e = lb::launch_decode(*L, x, y, fp32, words,
+        cudaError_t e = lb::launch_decode(*L, x, 0, y, fp32, words,
                                           static_cast<char *>(ws) + kWsHeader, sms, s);
         if (e != cudaErrorCooperativeLaunchTooLarge) return from_cuda(e);
         cudaGetLastError();  // too large for one co-resident grid: take the two-launch path

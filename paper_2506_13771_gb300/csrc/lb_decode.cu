@@ -37,7 +37,8 @@ struct DecodeLayout {
 
 struct DecodeParams {
     LinDesc L;
-    const uint16_t *x;
+    const void *x;     // bf16 [d_in], or fp32 when x_fp32
+    int x_fp32;
     void *y;
     int y_fp32;
     unsigned *ws_words;
@@ -114,7 +115,9 @@ __global__ void __launch_bounds__(kDT, 1) k_decode(const __grid_constant__ Decod
         const uint16_t *g = p ? L.g[1] : L.g[0];
         float *xg = reinterpret_cast<float *>(g_smem + o.xg[p]);
         for (int i = tid; i < 32 * nw; i += kDT)
-            xg[i] = bf16_bits_to_float(P.x[32 * iw0 + i]) * half_bits_to_float(g[32 * iw0 + i]);
+            xg[i] = (P.x_fp32 ? static_cast<const float *>(P.x)[32 * iw0 + i]
+                              : bf16_bits_to_float(static_cast<const uint16_t *>(P.x)[32 * iw0 + i])) *
+                    half_bits_to_float(g[32 * iw0 + i]);
     }
     float *y = reinterpret_cast<float *>(g_smem + o.y);
     for (int i = tid; i < nrows; i += kDT) y[i] = 0.f;
@@ -309,7 +312,7 @@ size_t decode_ws_bytes(const lb_linear &L) {
     return ((size_t)2 * rsum_of(L) * sizeof(unsigned long long) + 255) & ~(size_t)255;
 }
 
-cudaError_t launch_decode(const lb_linear &L, const uint16_t *x, void *y, int y_fp32,
+cudaError_t launch_decode(const lb_linear &L, const void *x, int x_fp32, void *y, int y_fp32,
                           unsigned *ws_words, void *xw, int num_sms, cudaStream_t s) {
     int max_smem = 0;
     cudaError_t e = device_setup(&max_smem);
@@ -317,6 +320,7 @@ cudaError_t launch_decode(const lb_linear &L, const uint16_t *x, void *y, int y_
     DecodeParams P{};
     P.L = make_desc(L);
     P.x = x;
+    P.x_fp32 = x_fp32;
     P.y = y;
     P.y_fp32 = y_fp32;
     P.ws_words = ws_words;

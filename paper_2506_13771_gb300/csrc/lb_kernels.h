@@ -40,7 +40,7 @@ cudaError_t launch_to_half(const float *z32, uint16_t *z16, long long n, cudaStr
 // Returns cudaErrorCooperativeLaunchTooLarge when the grid cannot be co-resident.
 bool decode_supported(const lb_linear &L, int num_sms);
 size_t decode_ws_bytes(const lb_linear &L);
-cudaError_t launch_decode(const lb_linear &L, const uint16_t *x, void *y, int y_fp32,
+cudaError_t launch_decode(const lb_linear &L, const void *x, int x_fp32, void *y, int y_fp32,
                           unsigned *ws_words, void *xw, int num_sms, cudaStream_t s);
 
 // Persistent decode of the seven-linear-per-layer stack (lb_stack.cu).

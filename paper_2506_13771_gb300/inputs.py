@@ -178,6 +178,24 @@ def make_stack(n_layers: int = 80, d_model: int = 8192, d_kv: int = 1024, d_ff: 
     return layers, x0
 
 
+# Llama2-7B-shaped decoder (the model of the paper's end-to-end decoding
+# table, shape only): 32 layers, d_model 4096 = 32 heads x 128, MHA, d_ff
+# 11008, with the ranks of the single-linear workloads (q/k/v/o 4096^2 at
+# r = 64 per path, ~0.08 BPW; the MLP at r = 128, ~0.1 BPW).
+DECODER_7B = dict(n_layers=32, d_model=4096, d_kv=4096, d_ff=11008, r_qo=64, r_kv=64, r_mlp=128,
+                  n_heads=32, n_kv_heads=32, head_dim=128)
+
+
+def decoder7b(n_tokens: int, n_layers: int = 32, config_id: int = 9):
+    """The 7B-shaped decoder's linears (two paths each, random sign words,
+    unit-gain scales) and n_tokens token embeddings, bf16 N(0,1) [n_tokens][4096]."""
+    kw = {k: v for k, v in DECODER_7B.items()
+          if k not in ("n_layers", "n_heads", "n_kv_heads", "head_dim")}
+    layers, _ = make_stack(n_layers=n_layers, config_id=config_id, **kw)
+    xs = bf16_normal(rng_for(config_id, salt=1), (n_tokens, DECODER_7B["d_model"]))
+    return layers, xs
+
+
 def config5(n_layers: int = 80):
     kw = {k: v for k, v in STACK_70B.items() if k not in ("n_layers", "head_dim")}
     return make_stack(n_layers=n_layers, **kw)

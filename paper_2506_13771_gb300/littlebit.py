@@ -29,7 +29,15 @@ EXPORTED = ["littlebit_status_string", "littlebit_pack", "littlebit_workspace_si
             "littlebit_train_backward",
             "littlebit_stack_workspace_size",
             "littlebit_stack_prepare", "littlebit_stack_forward", "littlebit_poll_error",
-            "littlebit_selftest_wait_timeout", "littlebit_linear_forward_noalloc"]
+            "littlebit_selftest_wait_timeout", "littlebit_linear_forward_noalloc",
+            "littlebit_decoder_workspace_size", "littlebit_decoder_step",
+            "littlebit_decoder_poll_error"]
+
+
+class lb_decoder_shape(ctypes.Structure):
+    _fields_ = [("n_layers", ctypes.c_int32), ("n_heads", ctypes.c_int32),
+                ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("max_pos", ctypes.c_int32), ("rope_base", ctypes.c_float)]
 
 
 class LittleBitError(RuntimeError):
@@ -126,6 +134,16 @@ def lib(path: str | None = None):
         L.littlebit_stack_forward.argtypes = [ctypes.POINTER(lb_linear), i32, i32, vp, vp, vp, vp,
                                               vp, sz, vp]
         L.littlebit_stack_forward.restype = ctypes.c_int
+        L.littlebit_decoder_workspace_size.argtypes = [ctypes.POINTER(lb_linear),
+                                                       ctypes.POINTER(lb_decoder_shape)]
+        L.littlebit_decoder_workspace_size.restype = sz
+        L.littlebit_decoder_step.argtypes = [ctypes.POINTER(lb_linear),
+                                             ctypes.POINTER(lb_decoder_shape), vp, vp, vp, vp, vp,
+                                             vp, sz, vp]
+        L.littlebit_decoder_step.restype = ctypes.c_int
+        L.littlebit_decoder_poll_error.argtypes = [ctypes.POINTER(lb_linear),
+                                                   ctypes.POINTER(lb_decoder_shape), vp, vp]
+        L.littlebit_decoder_poll_error.restype = ctypes.c_int
         L.littlebit_poll_error.argtypes = [vp, vp]
         L.littlebit_poll_error.restype = ctypes.c_int
         L.littlebit_selftest_wait_timeout.argtypes = [vp, vp]
@@ -483,3 +501,53 @@ def linear_forward_noalloc(L: DeviceLinear, x: torch.Tensor, out_dtype=torch.bfl
                                                   y_dtype, _stream(stream)),
            "littlebit_linear_forward_noalloc")
     return y
+
+
+# ------------------------------------------------------------------ decode at position p (App. I.3)
+
+
+class DeviceDecoder:
+    """A Llama-shaped decoder whose n_layers x (q, k, v, o, gate, up, down)
+    linears are LittleBit linears on the device, with its fp32 KV cache
+    ([n_layers][max_pos][d_kv] each for keys and values), the device position
+    counter and a workspace (all zero-filled: the cache starts empty)."""
+
+    def __init__(self, layers: list, n_heads: int, n_kv_heads: int, head_dim: int = 128,
+                 max_pos: int = 512, rope_base: float = 10000.0, device="cuda"):
+        assert len(layers) % 7 == 0
+        self.n_layers = len(layers) // 7
+        self.linears = [DeviceLinear(L, device) for L in layers]
+        self.carray = (lb_linear * len(self.linears))(*[L.c for L in self.linears])
+        self.shape = lb_decoder_shape(self.n_layers, int(n_heads), int(n_kv_heads), int(head_dim),
+                                      int(max_pos), float(rope_base))
+        self.d_model = int(n_heads) * int(head_dim)
+        self.d_kv = int(n_kv_heads) * int(head_dim)
+        nbytes = int(lib().littlebit_decoder_workspace_size(self.carray, ctypes.byref(self.shape)))
+        if nbytes == 0:
+            raise LittleBitError(LB_ERR_INVALID_ARG, "littlebit_decoder_workspace_size")
+        self.ws = new_workspace(nbytes, device)
+        self.kcache = torch.zeros((self.n_layers, max_pos, self.d_kv), dtype=torch.float32,
+                                  device=device)
+        self.vcache = torch.zeros_like(self.kcache)
+        self.pos = torch.zeros(1, dtype=torch.int32, device=device)
+
+    @property
+    def nbytes(self) -> int:
+        return sum(L.nbytes for L in self.linears)
+
+    def step(self, x: torch.Tensor, out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+        """Decodes the token x (bf16 [d_model]) at the current position and
+        advances it; returns the last hidden state (fp32 [d_model])."""
+        assert x.dtype == torch.bfloat16 and x.numel() == self.d_model and x.is_contiguous()
+        if out is None:
+            out = torch.empty(self.d_model, dtype=torch.float32, device=x.device)
+        _check(lib().littlebit_decoder_step(self.carray, ctypes.byref(self.shape), x.data_ptr(),
+                                            self.kcache.data_ptr(), self.vcache.data_ptr(),
+                                            self.pos.data_ptr(), out.data_ptr(), self.ws.data_ptr(),
+                                            self.ws.numel(), _stream(stream)),
+               "littlebit_decoder_step")
+        return out
+
+    def poll_error(self, stream=None) -> int:
+        return int(lib().littlebit_decoder_poll_error(self.carray, ctypes.byref(self.shape),
+                                                      self.ws.data_ptr(), _stream(stream)))

@@ -207,6 +207,48 @@ def test_stack_argument_validation(L):
     assert prep(uneven, 2, hd, FAKE, n, None) == lb.LB_ERR_UNSUPPORTED
 
 
+def test_decoder_argument_validation(L):
+    arr = fake_stack()                 # d 256 = 4 heads x 64, d_kv 64 = 1 kv head
+    S = lb.lb_decoder_shape(2, 4, 1, 64, 64, 10000.0)
+    n = L.littlebit_decoder_workspace_size(arr, ctypes.byref(S))
+    assert n > 256 and n % 256 == 0
+    st = L.littlebit_decoder_step
+    ok = dict(x=FAKE, k=FAKE, v=FAKE, pos=FAKE, out=FAKE, ws=FAKE, nb=n)
+
+    def call(a=arr, shape=S, **kw):
+        v = dict(ok, **kw)
+        return st(a, ctypes.byref(shape), v["x"], v["k"], v["v"], v["pos"], v["out"], v["ws"],
+                  v["nb"], None)
+
+    def shape(**kw):
+        f = dict(n_layers=2, n_heads=4, n_kv_heads=1, head_dim=64, max_pos=64, rope_base=10000.0)
+        f.update(kw)
+        return lb.lb_decoder_shape(*f.values())
+
+    assert call(shape=shape(n_layers=0)) == lb.LB_ERR_INVALID_ARG
+    assert call(shape=shape(n_kv_heads=3)) == lb.LB_ERR_INVALID_ARG     # 4 % 3 != 0
+    assert call(shape=shape(n_heads=8, head_dim=32)) == lb.LB_ERR_INVALID_ARG  # 64, 128 or 256
+    assert call(shape=shape(max_pos=0)) == lb.LB_ERR_INVALID_ARG
+    assert call(shape=shape(max_pos=8193)) == lb.LB_ERR_INVALID_ARG
+    assert call(shape=shape(rope_base=1.0)) == lb.LB_ERR_INVALID_ARG
+    assert call(x=0) == lb.LB_ERR_INVALID_ARG
+    assert call(x=FAKE + 8) == lb.LB_ERR_INVALID_ARG
+    assert call(pos=0) == lb.LB_ERR_INVALID_ARG
+    assert call(pos=FAKE + 2) == lb.LB_ERR_INVALID_ARG
+    assert call(ws=FAKE + 16) == lb.LB_ERR_WORKSPACE
+    assert call(nb=n - 256) == lb.LB_ERR_WORKSPACE
+    broken = fake_stack()
+    broken[1] = fake_linear(256, 128, (8, 8))                         # k must be d -> d_kv
+    assert L.littlebit_decoder_workspace_size(broken, ctypes.byref(S)) == 0
+    assert call(a=broken) == lb.LB_ERR_UNSUPPORTED
+    uneven = fake_stack()
+    uneven[7] = fake_linear(256, 256, (32, 16))                       # layer 1 q differs
+    assert call(a=uneven) == lb.LB_ERR_UNSUPPORTED
+    assert L.littlebit_decoder_poll_error(arr, ctypes.byref(shape(n_layers=0)), FAKE, None) == \
+        lb.LB_ERR_INVALID_ARG
+    assert L.littlebit_decoder_poll_error(arr, ctypes.byref(S), None, None) == lb.LB_ERR_WORKSPACE
+
+
 def test_pack_argument_validation(L):
     p = L.littlebit_pack
     assert p(None, 4, 4, lb.LB_PACK_U, FAKE, 4, None, None) == lb.LB_ERR_INVALID_ARG
