@@ -510,6 +510,46 @@ def run_config(args):
             raise RuntimeError("kernel reported an error")
         return statistics.median(ts)
 
+    def time_multi(L, x_bits, copies=64, per_launch=24):
+        """The same sustained measurement at T = 1 with the forwards grouped:
+        `copies` distinct weight copies through littlebit_linear_forward_multi,
+        `per_launch` linears per launch, all launches in one CUDA graph; L2
+        flushed before each replay.  Median ms per forward."""
+        devs = [lb.DeviceLinear(L, dev) for _ in range(copies)]
+        x = lb.bf16_tensor(x_bits, dev)[0]
+        y = torch.empty((copies, devs[0].d_out), dtype=torch.bfloat16, device=dev)
+        groups = [devs[i:i + per_launch] for i in range(0, copies, per_launch)]
+        wss = [lb.new_workspace(lb.multi_workspace_size(g), dev) for g in groups]
+
+        def run():
+            o = 0
+            for g, w in zip(groups, wss):
+                lb.linear_forward_multi(g, x, y=y[o:o + len(g)], ws=w)
+                o += len(g)
+        side = torch.cuda.Stream(dev)
+        side.wait_stream(torch.cuda.current_stream(dev))
+        with torch.cuda.stream(side):
+            run()
+        torch.cuda.current_stream(dev).wait_stream(side)
+        torch.cuda.synchronize(dev)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph):
+            run()
+        ts = []
+        for _ in range(max(5, min(steps, 50))):
+            flush.zero_()
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record()
+            graph.replay()
+            e1.record()
+            torch.cuda.synchronize(dev)
+            ts.append(e0.elapsed_time(e1) / copies)
+        for w in wss:
+            if lb.poll_error(w) != lb.LB_OK:
+                raise RuntimeError("kernel reported an error")
+        return statistics.median(ts)
+
     def wanted(name, T):
         return args.only is None or args.only in f"{name}:{T}"
 
@@ -548,6 +588,8 @@ def run_config(args):
                 ms = time_graph(L, x, T)
                 if ms is not None:
                     emit("4096x4096 r64", 2, T, L, ms, False, mode="graph64")
+                if T == 1:
+                    emit("4096x4096 r64", 2, T, L, time_multi(L, x), False, mode="multi64")
     elif args.config == 3:
         for r in (128, 512):
             for T in (1, 16, 64):
@@ -561,6 +603,8 @@ def run_config(args):
                         ms = time_graph(lins[nm], xin, T)
                         if ms is not None:
                             emit(f"{nm} r{r}", 3, T, lins[nm], ms, False, mode="graph64")
+                        emit(f"{nm} r{r}", 3, T, lins[nm], time_multi(lins[nm], xin), False,
+                             mode="multi64")
     elif args.config == 7:
         # Dual-SVID initialisation (one dense weight -> two LittleBit paths):
         # the 4096 x 4096 r64 layer and the 70B gate shape (8192 -> 28672, r320),
@@ -650,7 +694,7 @@ def run_config(args):
         # end-to-end decoding of a Llama2-7B-shaped decoder whose linears are
         # LittleBit (the paper's tokens-per-second setting, shape only): 128
         # and 256 new tokens from an empty cache, one decode step per token
-        # replayed as a CUDA graph (inputs resident; the step's 353 launches
+        # replayed as a CUDA graph (inputs resident; the step's 257 launches
         # are the per-token critical path)
         S = inputs.DECODER_7B
         for n_new in (128, 256):
@@ -697,7 +741,7 @@ def run_config(args):
             line = {"config": 9, "case": name, "op": "decode", "tokens": n_new, "ms": ms,
                     "tokens_per_s": n_new / ms * 1e3, "ms_per_token": ms / n_new,
                     "bytes_per_token": (wbytes + cache) / n_new, "gbs": gbs,
-                    "launches_per_token": 1 + 11 * S["n_layers"],
+                    "launches_per_token": 1 + 8 * S["n_layers"],  # q/k/v and gate/up grouped
                     "roofline": {"bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s",
                                  "frac": gbs / hbm, "peak_source": "MEASURED_PEAKS.json hbm_gbs"},
                     "context": "paper Table 12 (A100, Llama2-7B, 0.1 BPW, 128 new tokens): 203.20 "

@@ -328,10 +328,11 @@ size_t littlebit_decoder_workspace_size(const lb_linear *lin, const lb_decoder_s
  * workspace's error word and the step writes nothing (read it with
  * littlebit_decoder_poll_error).  Every linear's d_out and ranks must be
  * multiples of 8 (else LB_ERR_UNSUPPORTED).  ws: zero-filled before first
- * use, not shared with concurrent calls.  Enqueues 1 + 11 * n_layers
- * launches on the stream: seven single-token LittleBit linears per layer
- * (the cooperative kernel of littlebit_linear_forward at T = 1) and the
- * attention, norm and SiLU kernels. */
+ * use, not shared with concurrent calls.  Enqueues 1 + (8 .. 11) * n_layers
+ * launches on the stream: per layer the single-token LittleBit linears, with
+ * q / k / v (or k / v) and gate / up each grouped into one launch when they
+ * share a shape (as littlebit_linear_forward_multi), and the attention, norm
+ * and SiLU kernels. */
 lb_status littlebit_decoder_step(const lb_linear *lin, const lb_decoder_shape *S,
                                  const uint16_t *x, float *kcache, float *vcache, int32_t *pos,
                                  float *out, void *ws, size_t ws_bytes, lb_stream_t stream);
@@ -340,6 +341,24 @@ lb_status littlebit_decoder_step(const lb_linear *lin, const lb_decoder_shape *S
  * and each linear's, all cleared; returns the first error found, or LB_OK. */
 lb_status littlebit_decoder_poll_error(const lb_linear *lin, const lb_decoder_shape *S, void *ws,
                                        lb_stream_t stream);
+
+/* One token (T = 1) through M LittleBit linears of one shape that read the
+ * same input, in one launch: a decoder layer's q / k / v or gate / up
+ * projections, or M independent weight sets (Prop. 1 and Eq. 6 per linear,
+ * as littlebit_linear_forward).  L: HOST array of M structs (device
+ * pointers), 1 <= M <= 24, all with the same d_in, d_out, n_paths and ranks,
+ * d_out and the ranks multiples of 8 (else LB_ERR_UNSUPPORTED; other shape
+ * errors LB_ERR_INVALID_ARG).  x: bf16 [d_in]; y: [M][d_out] in y_dtype,
+ * row m the output of L[m].  One persistent launch of one CTA per SM that
+ * streams the linears' factors through shared memory and overlaps each
+ * linear's exchange with the next linears' work; the results equal M calls
+ * of littlebit_linear_forward at T = 1.  ws: littlebit_multi_workspace_size
+ * bytes, zero-filled before first use; a workspace serves one (shape, M) and
+ * calls on it must not overlap in time. */
+size_t littlebit_multi_workspace_size(const lb_linear *L, int32_t M);
+lb_status littlebit_linear_forward_multi(const lb_linear *L, int32_t M, const uint16_t *x,
+                                         void *y, int32_t y_dtype, void *ws, size_t ws_bytes,
+                                         lb_stream_t stream);
 
 /* The forward of littlebit_linear_forward for callers that cannot allocate
  * device memory.  The paper has no counterpart: this exists for hosts such as

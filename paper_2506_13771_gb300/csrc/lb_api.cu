@@ -216,6 +216,36 @@ lb_status littlebit_linear_forward(const lb_linear *L, const uint16_t *x, int64_
     return from_cuda(lb::launch_generic(*L, x, T, y, fp32, data, sms, s));
 }
 
+size_t littlebit_multi_workspace_size(const lb_linear *L, int32_t M) {
+    if (!L || M < 1 || M > lb::kMaxMultiLinears) return 0;
+    for (int m = 0; m < M; ++m)
+        if (check_linear(&L[m]) != LB_OK) return 0;
+    return kWsHeader + lb::multi_ws_bytes(L[0], M);
+}
+
+lb_status littlebit_linear_forward_multi(const lb_linear *L, int32_t M, const uint16_t *x,
+                                         void *y, int32_t y_dtype, void *ws, size_t ws_bytes,
+                                         lb_stream_t stream) {
+    if (!L || M < 1 || M > lb::kMaxMultiLinears) return LB_ERR_INVALID_ARG;
+    for (int m = 0; m < M; ++m) {
+        const lb_status st = check_linear(&L[m]);
+        if (st != LB_OK) return st;
+    }
+    if (y_dtype != LB_OUT_BF16 && y_dtype != LB_OUT_FP32) return LB_ERR_INVALID_ARG;
+    if (!x || !y || !aligned16(x) || !aligned16(y)) return LB_ERR_INVALID_ARG;
+    if (!ws || ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) ||
+        ws_bytes < littlebit_multi_workspace_size(L, M))
+        return LB_ERR_WORKSPACE;
+    int sms = 0;
+    lb_status st = num_sms(&sms);
+    if (st != LB_OK) return st;
+    if (!lb::multi_supported(L, M, sms)) return LB_ERR_UNSUPPORTED;
+    const cudaError_t e = lb::launch_decode_multi(
+        L, M, x, 0, y, y_dtype == LB_OUT_FP32, static_cast<unsigned *>(ws),
+        static_cast<char *>(ws) + kWsHeader, sms, (cudaStream_t)stream);
+    return e == cudaErrorCooperativeLaunchTooLarge ? LB_ERR_UNSUPPORTED : from_cuda(e);
+}
+
 lb_status littlebit_linear_latent(const lb_linear *L, const uint16_t *x, int64_t T, void *z,
                                   int32_t z_dtype, void *ws, size_t ws_bytes,
                                   lb_stream_t stream) {

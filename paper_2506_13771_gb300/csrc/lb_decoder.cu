@@ -226,9 +226,17 @@ __global__ void __launch_bounds__(HD)
 size_t align256(size_t b) { return (b + 255) & ~(size_t)255; }
 
 struct DecLayout {
-    size_t slot[7];        // byte offsets of the seven linear workspaces
+    size_t slot[7];        // byte offsets of the seven single-linear workspaces
     size_t slot_bytes[7];
+    size_t qkv_ws, qkv_bytes, gu_ws, gu_bytes;  // the two multi-linear workspaces
     size_t n, attn, m, q, k, v, y, g, u, a, end;
+};
+
+// The grouped launches of a layer: q with k and v when all three have one
+// shape (else k and v together, q alone), gate with up.
+struct DecGroups {
+    int qkv;  // 3: q, k, v in one launch; 2: k, v in one launch; 0: none
+    bool gu;
 };
 
 DecLayout dec_layout(const lb_linear *lin, const lb_decoder_shape &S) {
@@ -239,6 +247,12 @@ DecLayout dec_layout(const lb_linear *lin, const lb_decoder_shape &S) {
         o.slot_bytes[j] = kWsHeader + align256(decode_ws_bytes(lin[j]));
         off += o.slot_bytes[j];
     }
+    o.qkv_ws = off;
+    o.qkv_bytes = kWsHeader + align256(multi_ws_bytes(lin[1], 3));
+    off += o.qkv_bytes;
+    o.gu_ws = off;
+    o.gu_bytes = kWsHeader + align256(multi_ws_bytes(lin[4], 2));
+    off += o.gu_bytes;
     const size_t d = (size_t)S.n_heads * S.head_dim, dkv = (size_t)S.n_kv_heads * S.head_dim;
     const size_t dff = (size_t)lin[4].d_out;
     auto take = [&](size_t bytes) {
@@ -249,12 +263,12 @@ DecLayout dec_layout(const lb_linear *lin, const lb_decoder_shape &S) {
     o.n = take(d * 4);
     o.attn = take(d * 4);
     o.m = take(dff * 4);
-    o.q = take(d * 4);
-    o.k = take(dkv * 4);
-    o.v = take(dkv * 4);
+    o.q = take((d + 2 * dkv) * 4);  // q, k, v back to back (the rows of a grouped launch)
+    o.k = o.q + d * 4;
+    o.v = o.k + dkv * 4;
     o.y = take(d * 4);
-    o.g = take(dff * 4);
-    o.u = take(dff * 4);
+    o.g = take(2 * dff * 4);        // gate, up back to back
+    o.u = o.g + dff * 4;
     o.a = take(d * 4);
     o.end = off;
     return o;
@@ -293,6 +307,16 @@ lb_status check_decoder(const lb_linear *lin, const lb_decoder_shape *S) {
 }
 
 lb_status from_err(cudaError_t e) { return e == cudaSuccess ? LB_OK : LB_ERR_CUDA; }
+
+DecGroups groups_of(const lb_linear *lin, int sms) {
+    DecGroups G{};
+    const lb_linear qkv[3] = {lin[0], lin[1], lin[2]};
+    if (multi_supported(qkv, 3, sms)) G.qkv = 3;
+    else if (multi_supported(qkv + 1, 2, sms)) G.qkv = 2;
+    const lb_linear gu[2] = {lin[4], lin[5]};
+    G.gu = multi_supported(gu, 2, sms);
+    return G;
+}
 
 // SM count of the current device (cached per device).
 int sm_count() {
@@ -358,14 +382,29 @@ lb_status littlebit_decoder_step(const lb_linear *lin, const lb_decoder_shape *S
                                             sms, s);
         return e == cudaErrorCooperativeLaunchTooLarge ? LB_ERR_UNSUPPORTED : from_err(e);
     };
+    // linears j .. j + M - 1 of layer l in one launch (outputs back to back)
+    auto group = [&](int l, int j, int M, size_t ws_off, const float *xin, float *yout) {
+        char *gw = w + ws_off;
+        const cudaError_t e = launch_decode_multi(&lin[7 * (size_t)l + j], M, xin, 1, yout, 1,
+                                                  reinterpret_cast<unsigned *>(gw),
+                                                  gw + kWsHeader, sms, s);
+        return e == cudaErrorCooperativeLaunchTooLarge ? LB_ERR_UNSUPPORTED : from_err(e);
+    };
+    const DecGroups G = groups_of(lin, sms);
     k_dec_start<<<1, kNormThreads, 0, s>>>(x, a, n, d, pos, S->max_pos, hdr);
     if ((st = from_err(cudaGetLastError())) != LB_OK) return st;
     const int silu_blocks = (dff + 255) / 256;
     for (int l = 0; l < S->n_layers; ++l) {
         const bool last = l + 1 == S->n_layers;
-        if ((st = linear(l, 0, n, q)) != LB_OK || (st = linear(l, 1, n, k)) != LB_OK ||
-            (st = linear(l, 2, n, v)) != LB_OK)
+        if (G.qkv == 3) {
+            if ((st = group(l, 0, 3, o.qkv_ws, n, q)) != LB_OK) return st;
+        } else if (G.qkv == 2) {
+            if ((st = linear(l, 0, n, q)) != LB_OK || (st = group(l, 1, 2, o.qkv_ws, n, k)) != LB_OK)
+                return st;
+        } else if ((st = linear(l, 0, n, q)) != LB_OK || (st = linear(l, 1, n, k)) != LB_OK ||
+                   (st = linear(l, 2, n, v)) != LB_OK) {
             return st;
+        }
         float *kl = kcache + l * layer_rows, *vl = vcache + l * layer_rows;
         if (D == 64)
             k_dec_attention<64><<<S->n_heads, 64, attn_smem, s>>>(
@@ -380,7 +419,11 @@ lb_status littlebit_decoder_step(const lb_linear *lin, const lb_decoder_shape *S
         if ((st = linear(l, 3, attn, y)) != LB_OK) return st;
         k_dec_residual<<<1, kNormThreads, 0, s>>>(a, y, n, d, nullptr, nullptr, hdr);
         if ((st = from_err(cudaGetLastError())) != LB_OK) return st;
-        if ((st = linear(l, 4, n, g)) != LB_OK || (st = linear(l, 5, n, u)) != LB_OK) return st;
+        if (G.gu) {
+            if ((st = group(l, 4, 2, o.gu_ws, n, g)) != LB_OK) return st;
+        } else if ((st = linear(l, 4, n, g)) != LB_OK || (st = linear(l, 5, n, u)) != LB_OK) {
+            return st;
+        }
         k_dec_silu<<<silu_blocks, 256, 0, s>>>(g, u, m, dff, hdr);
         if ((st = from_err(cudaGetLastError())) != LB_OK) return st;
         if ((st = linear(l, 6, m, y)) != LB_OK) return st;
@@ -401,8 +444,9 @@ lb_status littlebit_decoder_poll_error(const lb_linear *lin, const lb_decoder_sh
     char *w = static_cast<char *>(ws);
     // the decoder's own word first, then each linear slot's workspace
     lb_status first = littlebit_poll_error(w, stream);
-    for (int j = 0; j < 7; ++j) {
-        const lb_status e = littlebit_poll_error(w + o.slot[j], stream);
+    for (int j = 0; j < 9; ++j) {
+        const size_t at = j < 7 ? o.slot[j] : (j == 7 ? o.qkv_ws : o.gu_ws);
+        const lb_status e = littlebit_poll_error(w + at, stream);
         if (first == LB_OK) first = e;
     }
     return first;

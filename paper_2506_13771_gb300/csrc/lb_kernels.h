@@ -43,6 +43,14 @@ size_t decode_ws_bytes(const lb_linear &L);
 cudaError_t launch_decode(const lb_linear &L, const void *x, int x_fp32, void *y, int y_fp32,
                           unsigned *ws_words, void *xw, int num_sms, cudaStream_t s);
 
+// T = 1 through M linears of one shape that read the same x (lb_multi.cu).
+constexpr int kMaxMultiLinears = 24;
+bool multi_supported(const lb_linear *L, int M, int num_sms);
+size_t multi_ws_bytes(const lb_linear &L, int M);
+cudaError_t launch_decode_multi(const lb_linear *L, int M, const void *x, int x_fp32, void *y,
+                                int y_fp32, unsigned *ws_words, void *xw, int num_sms,
+                                cudaStream_t s);
+
 // Persistent decode of the seven-linear-per-layer stack (lb_stack.cu).
 struct StackShape {
     int n_layers, d, dkv, dff, head_dim;

@@ -1,0 +1,421 @@
+// lb_multi.cu -- one token (T = 1) through M LittleBit linears of one shape
+// that read the same input x, in ONE persistent launch: the q / k / v (or
+// gate / up) projections of a decoder layer, or M independent weight sets.
+//
+// Per linear and path, Prop. 1 (LittleBit, arXiv 2506.13771): stage 1
+// t = V_sign^T (g . x), a +-1 reduction over d_in split across the CTAs and
+// summed through self-counting exchange words; stage 2 y = h . (U_sign (l . t))
+// over each CTA's output rows; Eq. 6 sums the paths.  The single-linear
+// kernel (k_decode) runs the two stages back to back and waits for its
+// exchange in between.  Here the linears are software-pipelined: iteration i
+// runs stage 1 of linear i and stage 2 of linear i - kAhead, so each
+// exchange has kAhead - 1 whole iterations of other linears' work to
+// complete behind.  Thread 0 bulk-copies (cp.async.bulk) each linear's V
+// slice, g slice, U rows and h into a ring of kSlots shared-memory slots, a
+// slot being refilled once its linear's stage 2 is done (kSlots - kAhead
+// iterations ahead of its stage 1).  The exchange words of all M linears are
+// double-buffered by the workspace's launch epoch as in k_decode: every CTA
+// clears its stripe of the previous launch's buffer.  Every wait is bounded;
+// on a timeout the CTA records LB_ERR_TIMEOUT, lets its own copies land and
+// returns.
+#include <mutex>
+
+#include "lb_common.cuh"
+#include "lb_kernels.h"
+#include "lb_lut.cuh"
+
+namespace lb {
+
+namespace {
+
+constexpr int kMT = 512;  // threads per CTA
+constexpr int kMW = kMT / 32;
+constexpr int kSlots = 6;
+constexpr int kAhead = 4;
+static_assert(kSlots > kAhead, "a slot must be refilled before its next stage 1");
+
+struct MultiPtrs {
+    const uint32_t *v[2], *u[2];
+    const uint16_t *g[2], *l[2], *h[2];
+};
+
+// Shared-memory byte offsets; V / g / U / h are offsets inside a slot.
+struct MultiLayout {
+    int V[2], g[2], U[2], h[2], slot_bytes, slots, xs, t1, t2, y, bytes;
+};
+
+struct MultiParams {
+    int d_in, d_out, np, r[2], M, N1, off1;
+    const void *x;  // bf16 [d_in], or fp32 when x_fp32
+    int x_fp32;
+    void *y;        // [M][d_out], bf16 or fp32
+    int y_fp32;
+    unsigned *ws_words;
+    unsigned long long *xw;  // exchange words: two buffers of M * N1
+    float fix_limit;
+    MultiLayout o;
+    MultiPtrs p[kMaxMultiLinears];
+};
+
+__device__ bool wait_bar_m(unsigned long long *bar, unsigned parity, unsigned *ws_words) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = globaltimer_ns();
+    while (!mbar_try_wait(bar, parity)) {
+        if (ld_relaxed_gpu(ws_words + kErrWord) != 0u) return false;
+        if (globaltimer_ns() - t0 > kWaitLimitNs) {
+            atomicCAS(ws_words + kErrWord, 0u, static_cast<unsigned>(LB_ERR_TIMEOUT));
+            return false;
+        }
+    }
+    return true;
+}
+
+__global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__ MultiParams P) {
+    __shared__ __align__(8) unsigned long long vbar[kSlots], ubar[kSlots];
+    __shared__ int s_ok;
+    unsigned *err = P.ws_words + kErrWord;
+    if (ld_relaxed_gpu(err) != 0u) return;
+    const unsigned epoch = ld_relaxed_gpu(P.ws_words + kEpochWord);
+    const size_t words = (size_t)P.M * P.N1;
+    unsigned long long *xw = P.xw + (size_t)(epoch & 1u) * words;
+    unsigned long long *xold = P.xw + (size_t)((epoch + 1u) & 1u) * words;
+    const MultiLayout &o = P.o;
+    const int N = gridDim.x, c = blockIdx.x, tid = threadIdx.x;
+    const int warp = tid >> 5, lane = tid & 31, np = P.np;
+    // input words [iw0, iw0 + nw), output rows [o0, o0 + nrows) (whole octets)
+    const int W = P.d_in >> 5, Q = P.d_out >> 3;
+    const int iw0 = (int)((long long)c * W / N), nw = (int)((long long)(c + 1) * W / N) - iw0;
+    const int q0 = (int)((long long)c * Q / N), nq = (int)((long long)(c + 1) * Q / N) - q0;
+    const int o0 = 8 * q0, nrows = 8 * nq;
+    // Contributions per exchange word: every CTA for linear 0 (so that no CTA
+    // can still be about to read the epoch when block 0 moves it on), only
+    // the CTAs holding input words for the others.
+    const unsigned n_contrib = (unsigned)(W < N ? W : N), n_first = (unsigned)N;
+    const int R0 = (P.r[0] + 31) >> 5, R1 = np > 1 ? (P.r[1] + 31) >> 5 : 0;
+    const int cbs = R0 + R1, nt0 = 8 * R0, ntab = 8 * (R0 + R1);
+
+    if (tid == 0) {
+        for (int s = 0; s < kSlots; ++s) {
+            mbar_init(vbar + s, 1);
+            mbar_init(ubar + s, 1);
+        }
+        fence_barrier_init();
+        s_ok = 1;
+    }
+    __syncthreads();
+    auto slot = [&](int m) { return g_smem + o.slots + (m % kSlots) * o.slot_bytes; };
+    // thread 0: the copies of linear m into its slot
+    auto issue = [&](int m) {
+        unsigned char *b = slot(m);
+        unsigned long long *vb = vbar + m % kSlots, *ub = ubar + m % kSlots;
+        const MultiPtrs &L = P.p[m];
+        for (int p = 0; p < np; ++p) {
+            const int r = P.r[p], R = (r + 31) >> 5;
+            if (nw > 0) {
+                mbar_expect_tx(vb, (unsigned)(nw * r * 4 + 64 * nw));
+                bulk_g2s(b + o.V[p], L.v[p] + (size_t)iw0 * r, (unsigned)(nw * r * 4), vb);
+                bulk_g2s(b + o.g[p], L.g[p] + 32 * iw0, (unsigned)(64 * nw), vb);
+            }
+            if (nrows > 0) {
+                mbar_expect_tx(ub, (unsigned)(nrows * R * 4 + 2 * nrows));
+                bulk_g2s(b + o.U[p], L.u[p] + (size_t)o0 * R, (unsigned)(nrows * R * 4), ub);
+                bulk_g2s(b + o.h[p], L.h[p] + o0, (unsigned)(2 * nrows), ub);
+            }
+        }
+        mbar_arrive(vb);
+        mbar_arrive(ub);
+    };
+    if (tid == 0)
+        for (int m = 0; m < P.M && m < kSlots; ++m) issue(m);
+    int issued = P.M < kSlots ? P.M : kSlots;  // linears whose copies were issued (thread 0)
+
+    // the x slice (fp32), and the previous launch's exchange words back to zero
+    float *xs = reinterpret_cast<float *>(g_smem + o.xs);
+    for (int i = tid; i < 32 * nw; i += kMT)
+        xs[i] = P.x_fp32 ? static_cast<const float *>(P.x)[32 * iw0 + i]
+                         : bf16_bits_to_float(static_cast<const uint16_t *>(P.x)[32 * iw0 + i]);
+    {
+        const size_t a = (size_t)c * words / N, b = (size_t)(c + 1) * words / N;
+        for (size_t i = a + tid; i < b; i += kMT) xold[i] = 0ull;
+    }
+    float *y = reinterpret_cast<float *>(g_smem + o.y);
+    for (int i = tid; i < nrows; i += kMT) y[i] = 0.f;
+    __syncthreads();
+    const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
+    bool ok = true;
+
+    for (int it = 0; it < P.M + kAhead && ok; ++it) {
+        // ---------------- stage 1 of linear it
+        if (it == 0 && nw == 0) {
+            // a CTA without input words still counts itself into linear 0's words
+            for (int i = tid; i < P.N1; i += kMT) red_add_u64(xw + i, 1ull);
+        }
+        if (it < P.M && nw > 0) {
+            const int m = it;
+            unsigned char *b = slot(m);
+            // tables of g . x (8 per input word and path), once the slice landed
+            bool got = true;
+            if (tid == 0) got = wait_bar_m(vbar + m % kSlots, (unsigned)((m / kSlots) & 1), P.ws_words);
+            if (tid == 0 && !got) s_ok = 0;
+            __syncthreads();
+            if (!s_ok) {
+                ok = false;
+                break;
+            }
+            if (tid != 0) mbar_try_wait(vbar + m % kSlots, (unsigned)((m / kSlots) & 1));
+            for (int idx = tid; idx < np * 8 * nw; idx += kMT) {
+                const int p = idx / (8 * nw), n = idx - p * 8 * nw;
+                const float4 xv = *reinterpret_cast<const float4 *>(xs + 4 * n);
+                const uint2 gw = *reinterpret_cast<const uint2 *>(b + o.g[p] + 8 * n);
+                const float4 v = make_float4(xv.x * half_bits_to_float((uint16_t)(gw.x & 0xffffu)),
+                                             xv.y * half_bits_to_float((uint16_t)(gw.x >> 16)),
+                                             xv.z * half_bits_to_float((uint16_t)(gw.y & 0xffffu)),
+                                             xv.w * half_bits_to_float((uint16_t)(gw.y >> 16)));
+                store_table(g_smem + o.t1 + idx * 128, v, lane);
+            }
+            __syncthreads();
+            unsigned long long *xm = xw + (size_t)m * P.N1;
+            for (int u = warp; u < cbs; u += kMW) {
+                const int p = u >= R0 ? 1 : 0, cb = u - (p ? R0 : 0);
+                const int r = P.r[p];
+                const int col = 32 * cb + lane, cc = min(col, r - 1);
+                const uint32_t *Vw = reinterpret_cast<const uint32_t *>(b + o.V[p]) + cc;
+                const uint32_t tb = (uint32_t)(o.t1 + p * 8 * nw * 128);
+                float acc0 = 0.f, acc1 = 0.f;
+                int w = 0;
+                for (; w + 2 <= nw; w += 2) {
+                    const uint32_t w0 = Vw[w * r], w1 = Vw[(w + 1) * r];
+                    acc0 += lut_word(w0, copy, tb + w * 1024);
+                    acc1 += lut_word(w1, copy, tb + (w + 1) * 1024);
+                }
+                if (w < nw) acc0 += lut_word(Vw[w * r], copy, tb + w * 1024);
+                if (col < r)
+                    red_add_u64(xm + (p ? P.off1 : 0) + col, enc_fix(acc0 + acc1, P.fix_limit, err));
+            }
+            __syncthreads();  // t1 is rebuilt by the next linear
+        }
+        // ---------------- stage 2 of linear it - kAhead
+        const int mm = it - kAhead;
+        if (mm < 0) continue;
+        {
+            const unsigned long long *xm = xw + (size_t)mm * P.N1;
+            const MultiPtrs &L = P.p[mm];
+            int pok = 1;
+            for (int idx = tid; idx < ntab && pok; idx += kMT) {
+                const int p = idx >= nt0 ? 1 : 0, n = idx - (p ? nt0 : 0);
+                const int r = P.r[p];
+                float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (4 * n < r) {
+                    const uint2 lw = __ldg(reinterpret_cast<const uint2 *>(L.l[p] + 4 * n));
+                    const unsigned long long *wd = xm + (p ? P.off1 : 0) + 4 * n;
+                    unsigned long long a0 = 0, a1 = 0, a2 = 0, a3 = 0, t0 = 0;
+                    for (int spin = 0;; ++spin) {
+                        ld_relaxed_v2_u64(wd, a0, a1);
+                        ld_relaxed_v2_u64(wd + 2, a2, a3);
+                        const unsigned want = mm == 0 ? n_first : n_contrib;
+                        if (counted(a0, want) && counted(a1, want) && counted(a2, want) &&
+                            counted(a3, want))
+                            break;
+                        if ((spin & 15) == 15) {
+                            if (ld_relaxed_gpu(err) != 0u) {
+                                pok = 0;
+                                break;
+                            }
+                            const unsigned long long now = globaltimer_ns();
+                            if (t0 == 0) t0 = now;
+                            if (now - t0 > kWaitLimitNs) {
+                                atomicCAS(err, 0u, static_cast<unsigned>(LB_ERR_TIMEOUT));
+                                pok = 0;
+                                break;
+                            }
+                        }
+                    }
+                    v = make_float4(dec_fix(a0) * half_bits_to_float((uint16_t)(lw.x & 0xffffu)),
+                                    dec_fix(a1) * half_bits_to_float((uint16_t)(lw.x >> 16)),
+                                    dec_fix(a2) * half_bits_to_float((uint16_t)(lw.y & 0xffffu)),
+                                    dec_fix(a3) * half_bits_to_float((uint16_t)(lw.y >> 16)));
+                }
+                store_table(g_smem + o.t2 + idx * 128, v, lane);
+            }
+            bool u_ok = true;
+            if (tid == 0 && nrows > 0)
+                u_ok = wait_bar_m(ubar + mm % kSlots, (unsigned)((mm / kSlots) & 1), P.ws_words);
+            if (!__syncthreads_and(pok && u_ok)) {
+                ok = false;
+                break;
+            }
+            if (tid != 0 && nrows > 0) mbar_try_wait(ubar + mm % kSlots, (unsigned)((mm / kSlots) & 1));
+            // every CTA contributed to linear 0's words before any could
+            // complete, so all have read the epoch: the next launch may use
+            // the other buffer
+            if (mm == 0 && c == 0 && tid == 0) P.ws_words[kEpochWord] = epoch + 1u;
+            unsigned char *b = slot(mm);
+            const int rb = (nrows + 31) >> 5;
+            for (int u = warp; u < np * rb; u += kMW) {
+                const int p = u / rb, blk = u - p * rb;
+                const int R = (P.r[p] + 31) >> 5;
+                const int row = 32 * blk + lane, rr = min(row, nrows - 1);
+                const float hs = half_bits_to_float(reinterpret_cast<const uint16_t *>(b + o.h[p])[rr]);
+                const uint32_t *Uw = reinterpret_cast<const uint32_t *>(b + o.U[p]) + rr * R;
+                const uint32_t tb = (uint32_t)(o.t2 + (p ? nt0 : 0) * 128);
+                float acc0 = 0.f, acc1 = 0.f;
+                int w = 0;
+                for (; w + 2 <= R; w += 2) {
+                    const uint32_t w0 = Uw[w], w1 = Uw[w + 1];
+                    acc0 += lut_word(w0, copy, tb + w * 1024);
+                    acc1 += lut_word(w1, copy, tb + (w + 1) * 1024);
+                }
+                if (w < R) acc0 += lut_word(Uw[w], copy, tb + w * 1024);
+                if (row < nrows) atomicAdd(y + row, (acc0 + acc1) * hs);
+            }
+            __syncthreads();
+            // the slot is free: refill it with linear mm + kSlots
+            if (tid == 0 && mm + kSlots < P.M) {
+                issue(mm + kSlots);
+                ++issued;
+            }
+            for (int i = tid; i < nrows; i += kMT) {
+                const size_t at = (size_t)mm * P.d_out + o0 + i;
+                if (P.y_fp32)
+                    static_cast<float *>(P.y)[at] = y[i];
+                else
+                    static_cast<uint16_t *>(P.y)[at] = float_to_bf16_bits(y[i]);
+                y[i] = 0.f;
+            }
+            __syncthreads();
+        }
+    }
+    if (!ok && tid == 0) {
+        // every copy this CTA issued must land before it goes away (the last
+        // use of each slot; earlier uses were consumed)
+        for (int m = issued > kSlots ? issued - kSlots : 0; m < issued; ++m) {
+            wait_bar_m(vbar + m % kSlots, (unsigned)((m / kSlots) & 1), P.ws_words);
+            wait_bar_m(ubar + m % kSlots, (unsigned)((m / kSlots) & 1), P.ws_words);
+        }
+    }
+}
+
+int up16(int n) { return (n + 15) & ~15; }
+
+MultiLayout layout_of(const lb_linear &L, int N) {
+    const int nw = (L.d_in / 32 + N - 1) / N, nrows = 8 * ((L.d_out / 8 + N - 1) / N);
+    MultiLayout o{};
+    int at = 0;
+    auto take = [&at](int bytes) {
+        const int off = at;
+        at += up16(bytes);
+        return off;
+    };
+    // one slot: V and g slices, U rows and h of each path
+    int ntab2 = 0;
+    for (int p = 0; p < 2; ++p) {
+        const bool on = p < L.n_paths;
+        const int r = on ? L.path[p].r : 0, R = (r + 31) / 32;
+        o.V[p] = take(nw * r * 4);
+        o.g[p] = take(on ? 64 * nw : 0);
+        o.U[p] = take(nrows * R * 4);
+        o.h[p] = take(2 * nrows);
+        ntab2 += 8 * R;
+    }
+    o.slot_bytes = up16(at);
+    at = 0;
+    o.slots = take(kSlots * o.slot_bytes);
+    o.xs = take(128 * nw);
+    // table bases are 1024-aligned: lut8 splices the entry byte into them
+    at = (at + 1023) & ~1023;
+    o.t1 = take(L.n_paths * 8 * nw * 128);
+    at = (at + 1023) & ~1023;
+    o.t2 = take(ntab2 * 128);
+    o.y = take(4 * nrows);
+    o.bytes = at;
+    return o;
+}
+
+int rsum(const lb_linear &L) {
+    int s = 0;
+    for (int p = 0; p < L.n_paths; ++p) s += L.path[p].r;
+    return s;
+}
+
+cudaError_t multi_setup(int *max_smem) {
+    static std::mutex mu;
+    static int smem_of[64];
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lock(mu);
+    if (dev >= 0 && dev < 64 && smem_of[dev] > 0) {
+        *max_smem = smem_of[dev];
+        return cudaSuccess;
+    }
+    int optin = 0;
+    e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    if (e != cudaSuccess) return e;
+    const int usable = optin - 1024;  // the kernel's static shared memory
+    e = cudaFuncSetAttribute((const void *)k_decode_multi,
+                             cudaFuncAttributeMaxDynamicSharedMemorySize, usable);
+    if (e != cudaSuccess) return e;
+    if (dev >= 0 && dev < 64) smem_of[dev] = usable;
+    *max_smem = usable;
+    return cudaSuccess;
+}
+
+}  // namespace
+
+bool multi_supported(const lb_linear *L, int M, int num_sms) {
+    if (M < 1 || M > kMaxMultiLinears || num_sms < 1 || num_sms > 255) return false;
+    const lb_linear &A = L[0];
+    if (A.d_out % 8 != 0) return false;
+    for (int m = 0; m < M; ++m) {
+        const lb_linear &B = L[m];
+        if (B.d_in != A.d_in || B.d_out != A.d_out || B.n_paths != A.n_paths) return false;
+        for (int p = 0; p < A.n_paths; ++p)
+            if (B.path[p].r != A.path[p].r || B.path[p].r % 8 != 0) return false;
+    }
+    return true;
+}
+
+size_t multi_ws_bytes(const lb_linear &L, int M) {
+    return ((size_t)2 * M * rsum(L) * sizeof(unsigned long long) + 255) & ~(size_t)255;
+}
+
+cudaError_t launch_decode_multi(const lb_linear *L, int M, const void *x, int x_fp32, void *y,
+                                int y_fp32, unsigned *ws_words, void *xw, int num_sms,
+                                cudaStream_t s) {
+    int max_smem = 0;
+    cudaError_t e = multi_setup(&max_smem);
+    if (e != cudaSuccess) return e;
+    MultiParams P{};
+    const lb_linear &A = L[0];
+    P.d_in = A.d_in;
+    P.d_out = A.d_out;
+    P.np = A.n_paths;
+    P.r[0] = A.path[0].r;
+    P.r[1] = A.n_paths > 1 ? A.path[1].r : 0;
+    P.M = M;
+    P.N1 = rsum(A);
+    P.off1 = A.path[0].r;
+    P.x = x;
+    P.x_fp32 = x_fp32;
+    P.y = y;
+    P.y_fp32 = y_fp32;
+    P.ws_words = ws_words;
+    P.xw = static_cast<unsigned long long *>(xw);
+    P.fix_limit = 2147483648.f / (float)num_sms;
+    P.o = layout_of(A, num_sms);
+    if (P.o.bytes > max_smem) return cudaErrorCooperativeLaunchTooLarge;
+    for (int m = 0; m < M; ++m)
+        for (int p = 0; p < A.n_paths; ++p) {
+            const lb_path &Q = L[m].path[p];
+            P.p[m].v[p] = Q.v_bits;
+            P.p[m].u[p] = Q.u_bits;
+            P.p[m].g[p] = Q.g;
+            P.p[m].l[p] = Q.l;
+            P.p[m].h[p] = Q.h;
+        }
+    void *args[] = {&P};
+    return cudaLaunchCooperativeKernel((const void *)k_decode_multi, dim3(num_sms), dim3(kMT), args,
+                                       (size_t)P.o.bytes, s);
+}
+
+}  // namespace lb

@@ -31,7 +31,8 @@ EXPORTED = ["littlebit_status_string", "littlebit_pack", "littlebit_workspace_si
             "littlebit_stack_prepare", "littlebit_stack_forward", "littlebit_poll_error",
             "littlebit_selftest_wait_timeout", "littlebit_linear_forward_noalloc",
             "littlebit_decoder_workspace_size", "littlebit_decoder_step",
-            "littlebit_decoder_poll_error"]
+            "littlebit_decoder_poll_error", "littlebit_multi_workspace_size",
+            "littlebit_linear_forward_multi"]
 
 
 class lb_decoder_shape(ctypes.Structure):
@@ -144,6 +145,11 @@ def lib(path: str | None = None):
         L.littlebit_decoder_poll_error.argtypes = [ctypes.POINTER(lb_linear),
                                                    ctypes.POINTER(lb_decoder_shape), vp, vp]
         L.littlebit_decoder_poll_error.restype = ctypes.c_int
+        L.littlebit_multi_workspace_size.argtypes = [ctypes.POINTER(lb_linear), i32]
+        L.littlebit_multi_workspace_size.restype = sz
+        L.littlebit_linear_forward_multi.argtypes = [ctypes.POINTER(lb_linear), i32, vp, vp, i32,
+                                                     vp, sz, vp]
+        L.littlebit_linear_forward_multi.restype = ctypes.c_int
         L.littlebit_poll_error.argtypes = [vp, vp]
         L.littlebit_poll_error.restype = ctypes.c_int
         L.littlebit_selftest_wait_timeout.argtypes = [vp, vp]
@@ -551,3 +557,31 @@ class DeviceDecoder:
     def poll_error(self, stream=None) -> int:
         return int(lib().littlebit_decoder_poll_error(self.carray, ctypes.byref(self.shape),
                                                       self.ws.data_ptr(), _stream(stream)))
+
+
+# ------------------------------------------------------------------ several linears, one token
+
+
+def multi_workspace_size(linears: list) -> int:
+    arr = (lb_linear * len(linears))(*[L.c for L in linears])
+    return int(lib().littlebit_multi_workspace_size(arr, len(linears)))
+
+
+def linear_forward_multi(linears: list, x: torch.Tensor, out_dtype=torch.bfloat16,
+                         y: torch.Tensor | None = None, ws: torch.Tensor | None = None,
+                         stream=None) -> torch.Tensor:
+    """y[m] = x W_m^T for M DeviceLinears of one shape and one bf16 token x [d_in]:
+    one launch; returns [M][d_out]."""
+    assert x.dtype == torch.bfloat16 and x.is_contiguous()
+    M = len(linears)
+    arr = (lb_linear * M)(*[L.c for L in linears])
+    if y is None:
+        y = torch.empty((M, linears[0].d_out), dtype=out_dtype, device=x.device)
+    assert y.dtype in (torch.bfloat16, torch.float32) and y.is_contiguous()
+    if ws is None:
+        ws = new_workspace(multi_workspace_size(linears), x.device)
+    code = LB_OUT_FP32 if y.dtype == torch.float32 else LB_OUT_BF16
+    _check(lib().littlebit_linear_forward_multi(arr, M, x.data_ptr(), y.data_ptr(), code,
+                                                ws.data_ptr(), ws.numel(), _stream(stream)),
+           "littlebit_linear_forward_multi")
+    return y

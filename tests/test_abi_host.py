@@ -249,6 +249,22 @@ def test_decoder_argument_validation(L):
     assert L.littlebit_decoder_poll_error(arr, ctypes.byref(S), None, None) == lb.LB_ERR_WORKSPACE
 
 
+def test_multi_argument_validation(L):
+    arr = (lb.lb_linear * 3)(*[fake_linear(1024, 512, (64, 64)) for _ in range(3)])
+    n = L.littlebit_multi_workspace_size(arr, 3)
+    assert n > 256 and n % 256 == 0
+    f = L.littlebit_linear_forward_multi
+    assert f(arr, 0, FAKE, FAKE, 0, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    assert f(arr, 25, FAKE, FAKE, 0, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    assert f(arr, 3, 0, FAKE, 0, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    assert f(arr, 3, FAKE, FAKE + 4, 0, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    assert f(arr, 3, FAKE, FAKE, 2, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    assert f(arr, 3, FAKE, FAKE, 0, FAKE, n - 256, None) == lb.LB_ERR_WORKSPACE
+    assert f(arr, 3, FAKE, FAKE, 0, FAKE + 128, n, None) == lb.LB_ERR_WORKSPACE
+    assert L.littlebit_multi_workspace_size(arr, 0) == 0
+    assert L.littlebit_multi_workspace_size(arr, 25) == 0
+
+
 def test_pack_argument_validation(L):
     p = L.littlebit_pack
     assert p(None, 4, 4, lb.LB_PACK_U, FAKE, 4, None, None) == lb.LB_ERR_INVALID_ARG
