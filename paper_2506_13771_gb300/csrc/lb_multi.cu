@@ -144,7 +144,20 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
     const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
     bool ok = true;
 
+    // the exchange words a thread polls for stage 2 (its table tid; ntab <=
+    // kMT whenever the ranks sum to at most 2048), loaded one iteration's
+    // stage 1 ahead of their use so that the L2 round trip overlaps it
+    unsigned long long pre[4] = {0ull, 0ull, 0ull, 0ull};
+    auto prefetch = [&](int mm) {
+        if (mm < 0 || mm >= P.M || tid >= ntab) return;
+        const int p = tid >= nt0 ? 1 : 0, n = tid - (p ? nt0 : 0);
+        if (4 * n >= P.r[p]) return;
+        const unsigned long long *wd = xw + (size_t)mm * P.N1 + (p ? P.off1 : 0) + 4 * n;
+        ld_relaxed_v2_u64(wd, pre[0], pre[1]);
+        ld_relaxed_v2_u64(wd + 2, pre[2], pre[3]);
+    };
     for (int it = 0; it < P.M + kAhead && ok; ++it) {
+        prefetch(it - kAhead);
         // ---------------- stage 1 of linear it
         if (it == 0 && nw == 0) {
             // a CTA without input words still counts itself into linear 0's words
@@ -210,8 +223,15 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
                     const unsigned long long *wd = xm + (p ? P.off1 : 0) + 4 * n;
                     unsigned long long a0 = 0, a1 = 0, a2 = 0, a3 = 0, t0 = 0;
                     for (int spin = 0;; ++spin) {
-                        ld_relaxed_v2_u64(wd, a0, a1);
-                        ld_relaxed_v2_u64(wd + 2, a2, a3);
+                        if (spin == 0 && idx == tid) {
+                            a0 = pre[0];
+                            a1 = pre[1];
+                            a2 = pre[2];
+                            a3 = pre[3];
+                        } else {
+                            ld_relaxed_v2_u64(wd, a0, a1);
+                            ld_relaxed_v2_u64(wd + 2, a2, a3);
+                        }
                         const unsigned want = mm == 0 ? n_first : n_contrib;
                         if (counted(a0, want) && counted(a1, want) && counted(a2, want) &&
                             counted(a3, want))
