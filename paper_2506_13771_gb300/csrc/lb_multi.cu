@@ -30,18 +30,20 @@ namespace {
 
 constexpr int kMT = 512;  // threads per CTA
 constexpr int kMW = kMT / 32;
-constexpr int kSlots = 6;
+constexpr int kSlots = 7;
 constexpr int kAhead = 4;
-static_assert(kSlots > kAhead, "a slot must be refilled before its next stage 1");
+// a slot freed by stage 2 in iteration i is refilled during iteration i + 1
+static_assert(kSlots > kAhead + 1, "a slot must be refilled before its next stage 1");
+constexpr int kIssuer = kMT - 32;  // lane 0 of the last warp issues the refills
 
 struct MultiPtrs {
     const uint32_t *v[2], *u[2];
     const uint16_t *g[2], *l[2], *h[2];
 };
 
-// Shared-memory byte offsets; V / g / U / h are offsets inside a slot.
+// Shared-memory byte offsets; V / g / U / h / l are offsets inside a slot.
 struct MultiLayout {
-    int V[2], g[2], U[2], h[2], slot_bytes, slots, xs, t1, t2, y, bytes;
+    int V[2], g[2], U[2], h[2], l[2], slot_bytes, slots, xs, t1, t2, y, bytes;
 };
 
 struct MultiParams {
@@ -72,7 +74,7 @@ __device__ bool wait_bar_m(unsigned long long *bar, unsigned parity, unsigned *w
 
 __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__ MultiParams P) {
     __shared__ __align__(8) unsigned long long vbar[kSlots], ubar[kSlots];
-    __shared__ int s_ok;
+    __shared__ int s_ok, s_issued;
     unsigned *err = P.ws_words + kErrWord;
     if (ld_relaxed_gpu(err) != 0u) return;
     const unsigned epoch = ld_relaxed_gpu(P.ws_words + kEpochWord);
@@ -101,6 +103,7 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
         }
         fence_barrier_init();
         s_ok = 1;
+        s_issued = P.M < kSlots ? P.M : kSlots;
     }
     __syncthreads();
     auto slot = [&](int m) { return g_smem + o.slots + (m % kSlots) * o.slot_bytes; };
@@ -116,8 +119,10 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
                 bulk_g2s(b + o.V[p], L.v[p] + (size_t)iw0 * r, (unsigned)(nw * r * 4), vb);
                 bulk_g2s(b + o.g[p], L.g[p] + 32 * iw0, (unsigned)(64 * nw), vb);
             }
+            // l with the U rows: stage 2's tables read it next to the exchange
+            mbar_expect_tx(ub, (unsigned)(2 * r + (nrows > 0 ? nrows * R * 4 + 2 * nrows : 0)));
+            bulk_g2s(b + o.l[p], L.l[p], (unsigned)(2 * r), ub);
             if (nrows > 0) {
-                mbar_expect_tx(ub, (unsigned)(nrows * R * 4 + 2 * nrows));
                 bulk_g2s(b + o.U[p], L.u[p] + (size_t)o0 * R, (unsigned)(nrows * R * 4), ub);
                 bulk_g2s(b + o.h[p], L.h[p] + o0, (unsigned)(2 * nrows), ub);
             }
@@ -127,7 +132,6 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
     };
     if (tid == 0)
         for (int m = 0; m < P.M && m < kSlots; ++m) issue(m);
-    int issued = P.M < kSlots ? P.M : kSlots;  // linears whose copies were issued (thread 0)
 
     // the x slice (fp32), and the previous launch's exchange words back to zero
     float *xs = reinterpret_cast<float *>(g_smem + o.xs);
@@ -212,14 +216,22 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
         if (mm < 0) continue;
         {
             const unsigned long long *xm = xw + (size_t)mm * P.N1;
-            const MultiPtrs &L = P.p[mm];
+            unsigned char *b = slot(mm);
+            // the slot's U rows, h and l (thread 0 waits, the rest observe the phase)
+            bool u_ok = true;
+            if (tid == 0) u_ok = wait_bar_m(ubar + mm % kSlots, (unsigned)((mm / kSlots) & 1), P.ws_words);
+            if (!__syncthreads_and(u_ok)) {
+                ok = false;
+                break;
+            }
+            if (tid != 0) mbar_try_wait(ubar + mm % kSlots, (unsigned)((mm / kSlots) & 1));
             int pok = 1;
             for (int idx = tid; idx < ntab && pok; idx += kMT) {
                 const int p = idx >= nt0 ? 1 : 0, n = idx - (p ? nt0 : 0);
                 const int r = P.r[p];
                 float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
                 if (4 * n < r) {
-                    const uint2 lw = __ldg(reinterpret_cast<const uint2 *>(L.l[p] + 4 * n));
+                    const uint2 lw = *reinterpret_cast<const uint2 *>(b + o.l[p] + 8 * n);
                     const unsigned long long *wd = xm + (p ? P.off1 : 0) + 4 * n;
                     unsigned long long a0 = 0, a1 = 0, a2 = 0, a3 = 0, t0 = 0;
                     for (int spin = 0;; ++spin) {
@@ -257,19 +269,20 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
                 }
                 store_table(g_smem + o.t2 + idx * 128, v, lane);
             }
-            bool u_ok = true;
-            if (tid == 0 && nrows > 0)
-                u_ok = wait_bar_m(ubar + mm % kSlots, (unsigned)((mm / kSlots) & 1), P.ws_words);
-            if (!__syncthreads_and(pok && u_ok)) {
+            if (!__syncthreads_and(pok)) {
                 ok = false;
                 break;
             }
-            if (tid != 0 && nrows > 0) mbar_try_wait(ubar + mm % kSlots, (unsigned)((mm / kSlots) & 1));
             // every CTA contributed to linear 0's words before any could
             // complete, so all have read the epoch: the next launch may use
             // the other buffer
             if (mm == 0 && c == 0 && tid == 0) P.ws_words[kEpochWord] = epoch + 1u;
-            unsigned char *b = slot(mm);
+            // the slot linear mm - 1 freed: refilled by the last warp, idle
+            // while the others sum the rows below
+            if (tid == kIssuer && mm >= 1 && mm - 1 + kSlots < P.M) {
+                issue(mm - 1 + kSlots);
+                s_issued = mm - 1 + kSlots + 1;
+            }
             const int rb = (nrows + 31) >> 5;
             for (int u = warp; u < np * rb; u += kMW) {
                 const int p = u / rb, blk = u - p * rb;
@@ -286,14 +299,10 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
                     acc1 += lut_word(w1, copy, tb + (w + 1) * 1024);
                 }
                 if (w < R) acc0 += lut_word(Uw[w], copy, tb + w * 1024);
+                // at most two paths meet in a row: 0 + a + b is exact in either order
                 if (row < nrows) atomicAdd(y + row, (acc0 + acc1) * hs);
             }
             __syncthreads();
-            // the slot is free: refill it with linear mm + kSlots
-            if (tid == 0 && mm + kSlots < P.M) {
-                issue(mm + kSlots);
-                ++issued;
-            }
             for (int i = tid; i < nrows; i += kMT) {
                 const size_t at = (size_t)mm * P.d_out + o0 + i;
                 if (P.y_fp32)
@@ -305,9 +314,11 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
             __syncthreads();
         }
     }
+    __syncthreads();
     if (!ok && tid == 0) {
         // every copy this CTA issued must land before it goes away (the last
         // use of each slot; earlier uses were consumed)
+        const int issued = s_issued;
         for (int m = issued > kSlots ? issued - kSlots : 0; m < issued; ++m) {
             wait_bar_m(vbar + m % kSlots, (unsigned)((m / kSlots) & 1), P.ws_words);
             wait_bar_m(ubar + m % kSlots, (unsigned)((m / kSlots) & 1), P.ws_words);
@@ -335,6 +346,7 @@ MultiLayout layout_of(const lb_linear &L, int N) {
         o.g[p] = take(on ? 64 * nw : 0);
         o.U[p] = take(nrows * R * 4);
         o.h[p] = take(2 * nrows);
+        o.l[p] = take(2 * r);
         ntab2 += 8 * R;
     }
     o.slot_bytes = up16(at);

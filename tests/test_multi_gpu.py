@@ -1,6 +1,7 @@
 """One token through M LittleBit linears of one shape in one launch
-(littlebit_linear_forward_multi) against the oracle, and against M calls of
-the single-linear entry point."""
+(littlebit_linear_forward_multi) against the oracle, against M calls of the
+single-linear entry point, and against itself (repeated calls on one
+workspace are bit-identical)."""
 import numpy as np
 import pytest
 import torch
@@ -61,7 +62,8 @@ def test_multi_vs_oracle_and_single(d_in, d_out, rs, M, out_dtype):
     for m in range(M):
         e = rel(yg[m], oracle.forward_factored(layers[m], x)[0])
         assert e <= (1e-4 if out_dtype == torch.float32 else 2e-3), (m, e)
-    # bit for bit the single-linear path at T = 1 (same sums, same order)
+    # bit for bit the single-linear path at T = 1 (the same exact fixed-point
+    # exchange and the same fp32 sums in the same order)
     for m in (0, M - 1):
         ys = torch.full((1, d_out), float("nan"), dtype=out_dtype, device=DEV)
         lb.linear_forward(D[m], xt[None, :], y=ys)
