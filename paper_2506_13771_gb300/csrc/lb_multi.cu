@@ -32,9 +32,9 @@ constexpr int kMT = 512;  // threads per CTA
 constexpr int kMW = kMT / 32;
 constexpr int kSlots = 7;
 constexpr int kAhead = 4;
-// a slot freed by stage 2 in iteration i is refilled during iteration i + 1
-static_assert(kSlots > kAhead + 1, "a slot must be refilled before its next stage 1");
-constexpr int kIssuer = kMT - 32;  // lane 0 of the last warp issues the refills
+static_assert(kSlots > kAhead + 1, "a slot must be refilled ahead of its next stage 1");
+constexpr int kCW = kMW - 1;       // compute warps; the last warp issues the copies
+constexpr int kCT = kCW * 32;
 
 struct MultiPtrs {
     const uint32_t *v[2], *u[2];
@@ -72,8 +72,23 @@ __device__ bool wait_bar_m(unsigned long long *bar, unsigned parity, unsigned *w
     return true;
 }
 
+__device__ __forceinline__ void csync_m() {
+    asm volatile("bar.sync 1, %0;" ::"n"(kCT) : "memory");
+}
+// AND of pred over the compute threads (named barrier 1), returned to each.
+__device__ __forceinline__ int csync_and_m(int pred) {
+    int r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\tsetp.ne.s32 p, %1, 0;\n\tbar.red.and.pred q, 1, %2, p;\n\t"
+        "selp.s32 %0, 1, 0, q;\n\t}"
+        : "=r"(r)
+        : "r"(pred), "n"(kCT)
+        : "memory");
+    return r;
+}
+
 __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__ MultiParams P) {
-    __shared__ __align__(8) unsigned long long vbar[kSlots], ubar[kSlots];
+    __shared__ __align__(8) unsigned long long vbar[kSlots], ubar[kSlots], fbar[kSlots];
     __shared__ int s_ok, s_issued;
     unsigned *err = P.ws_words + kErrWord;
     if (ld_relaxed_gpu(err) != 0u) return;
@@ -100,133 +115,140 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
         for (int s = 0; s < kSlots; ++s) {
             mbar_init(vbar + s, 1);
             mbar_init(ubar + s, 1);
+            mbar_init(fbar + s, 1);
         }
         fence_barrier_init();
         s_ok = 1;
-        s_issued = P.M < kSlots ? P.M : kSlots;
+        s_issued = 0;
     }
     __syncthreads();
     auto slot = [&](int m) { return g_smem + o.slots + (m % kSlots) * o.slot_bytes; };
-    // thread 0: the copies of linear m into its slot
-    auto issue = [&](int m) {
-        unsigned char *b = slot(m);
-        unsigned long long *vb = vbar + m % kSlots, *ub = ubar + m % kSlots;
-        const MultiPtrs &L = P.p[m];
-        for (int p = 0; p < np; ++p) {
-            const int r = P.r[p], R = (r + 31) >> 5;
-            if (nw > 0) {
-                mbar_expect_tx(vb, (unsigned)(nw * r * 4 + 64 * nw));
-                bulk_g2s(b + o.V[p], L.v[p] + (size_t)iw0 * r, (unsigned)(nw * r * 4), vb);
-                bulk_g2s(b + o.g[p], L.g[p] + 32 * iw0, (unsigned)(64 * nw), vb);
-            }
-            // l with the U rows: stage 2's tables read it next to the exchange
-            mbar_expect_tx(ub, (unsigned)(2 * r + (nrows > 0 ? nrows * R * 4 + 2 * nrows : 0)));
-            bulk_g2s(b + o.l[p], L.l[p], (unsigned)(2 * r), ub);
-            if (nrows > 0) {
-                bulk_g2s(b + o.U[p], L.u[p] + (size_t)o0 * R, (unsigned)(nrows * R * 4), ub);
-                bulk_g2s(b + o.h[p], L.h[p] + o0, (unsigned)(2 * nrows), ub);
-            }
-        }
-        mbar_arrive(vb);
-        mbar_arrive(ub);
-    };
-    if (tid == 0)
-        for (int m = 0; m < P.M && m < kSlots; ++m) issue(m);
 
-    // the x slice (fp32), and the previous launch's exchange words back to zero
-    float *xs = reinterpret_cast<float *>(g_smem + o.xs);
-    for (int i = tid; i < 32 * nw; i += kMT)
-        xs[i] = P.x_fp32 ? static_cast<const float *>(P.x)[32 * iw0 + i]
-                         : bf16_bits_to_float(static_cast<const uint16_t *>(P.x)[32 * iw0 + i]);
-    {
-        const size_t a = (size_t)c * words / N, b = (size_t)(c + 1) * words / N;
-        for (size_t i = a + tid; i < b; i += kMT) xold[i] = 0ull;
-    }
-    float *y = reinterpret_cast<float *>(g_smem + o.y);
-    for (int i = tid; i < nrows; i += kMT) y[i] = 0.f;
-    __syncthreads();
-    const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
-    bool ok = true;
-
-    // the exchange words a thread polls for stage 2 (its table tid; ntab <=
-    // kMT whenever the ranks sum to at most 2048), loaded one iteration's
-    // stage 1 ahead of their use so that the L2 round trip overlaps it
-    unsigned long long pre[4] = {0ull, 0ull, 0ull, 0ull};
-    auto prefetch = [&](int mm) {
-        if (mm < 0 || mm >= P.M || tid >= ntab) return;
-        const int p = tid >= nt0 ? 1 : 0, n = tid - (p ? nt0 : 0);
-        if (4 * n >= P.r[p]) return;
-        const unsigned long long *wd = xw + (size_t)mm * P.N1 + (p ? P.off1 : 0) + 4 * n;
-        ld_relaxed_v2_u64(wd, pre[0], pre[1]);
-        ld_relaxed_v2_u64(wd + 2, pre[2], pre[3]);
-    };
-    for (int it = 0; it < P.M + kAhead && ok; ++it) {
-        prefetch(it - kAhead);
-        // ---------------- stage 1 of linear it
-        if (it == 0 && nw == 0) {
-            // a CTA without input words still counts itself into linear 0's words
-            for (int i = tid; i < P.N1; i += kMT) red_add_u64(xw + i, 1ull);
-        }
-        if (it < P.M && nw > 0) {
-            const int m = it;
-            unsigned char *b = slot(m);
-            // tables of g . x (8 per input word and path), once the slice landed
-            bool got = true;
-            if (tid == 0) got = wait_bar_m(vbar + m % kSlots, (unsigned)((m / kSlots) & 1), P.ws_words);
-            if (tid == 0 && !got) s_ok = 0;
-            __syncthreads();
-            if (!s_ok) {
-                ok = false;
-                break;
-            }
-            if (tid != 0) mbar_try_wait(vbar + m % kSlots, (unsigned)((m / kSlots) & 1));
-            for (int idx = tid; idx < np * 8 * nw; idx += kMT) {
-                const int p = idx / (8 * nw), n = idx - p * 8 * nw;
-                const float4 xv = *reinterpret_cast<const float4 *>(xs + 4 * n);
-                const uint2 gw = *reinterpret_cast<const uint2 *>(b + o.g[p] + 8 * n);
-                const float4 v = make_float4(xv.x * half_bits_to_float((uint16_t)(gw.x & 0xffffu)),
-                                             xv.y * half_bits_to_float((uint16_t)(gw.x >> 16)),
-                                             xv.z * half_bits_to_float((uint16_t)(gw.y & 0xffffu)),
-                                             xv.w * half_bits_to_float((uint16_t)(gw.y >> 16)));
-                store_table(g_smem + o.t1 + idx * 128, v, lane);
-            }
-            __syncthreads();
-            unsigned long long *xm = xw + (size_t)m * P.N1;
-            for (int u = warp; u < cbs; u += kMW) {
-                const int p = u >= R0 ? 1 : 0, cb = u - (p ? R0 : 0);
-                const int r = P.r[p];
-                const int col = 32 * cb + lane, cc = min(col, r - 1);
-                const uint32_t *Vw = reinterpret_cast<const uint32_t *>(b + o.V[p]) + cc;
-                const uint32_t tb = (uint32_t)(o.t1 + p * 8 * nw * 128);
-                float acc0 = 0.f, acc1 = 0.f;
-                int w = 0;
-                for (; w + 2 <= nw; w += 2) {
-                    const uint32_t w0 = Vw[w * r], w1 = Vw[(w + 1) * r];
-                    acc0 += lut_word(w0, copy, tb + w * 1024);
-                    acc1 += lut_word(w1, copy, tb + (w + 1) * 1024);
+    if (warp == kCW) {
+        // ---------------- producer: the copies of every linear into its slot,
+        //                  a slot refilled once the compute warps freed it
+        if (lane == 0) {
+            for (int m = 0; m < P.M; ++m) {
+                if (m >= kSlots &&
+                    !wait_bar_m(fbar + m % kSlots, (unsigned)(((m - kSlots) / kSlots) & 1),
+                                P.ws_words))
+                    break;
+                unsigned char *b = slot(m);
+                unsigned long long *vb = vbar + m % kSlots, *ub = ubar + m % kSlots;
+                const MultiPtrs &L = P.p[m];
+                for (int p = 0; p < np; ++p) {
+                    const int r = P.r[p], R = (r + 31) >> 5;
+                    if (nw > 0) {
+                        mbar_expect_tx(vb, (unsigned)(nw * r * 4 + 64 * nw));
+                        bulk_g2s(b + o.V[p], L.v[p] + (size_t)iw0 * r, (unsigned)(nw * r * 4), vb);
+                        bulk_g2s(b + o.g[p], L.g[p] + 32 * iw0, (unsigned)(64 * nw), vb);
+                    }
+                    // l with the U rows: stage 2's tables read it next to the exchange
+                    mbar_expect_tx(ub, (unsigned)(2 * r + (nrows > 0 ? nrows * R * 4 + 2 * nrows : 0)));
+                    bulk_g2s(b + o.l[p], L.l[p], (unsigned)(2 * r), ub);
+                    if (nrows > 0) {
+                        bulk_g2s(b + o.U[p], L.u[p] + (size_t)o0 * R, (unsigned)(nrows * R * 4), ub);
+                        bulk_g2s(b + o.h[p], L.h[p] + o0, (unsigned)(2 * nrows), ub);
+                    }
                 }
-                if (w < nw) acc0 += lut_word(Vw[w * r], copy, tb + w * 1024);
-                if (col < r)
-                    red_add_u64(xm + (p ? P.off1 : 0) + col, enc_fix(acc0 + acc1, P.fix_limit, err));
+                mbar_arrive(vb);
+                mbar_arrive(ub);
+                s_issued = m + 1;
             }
-            __syncthreads();  // t1 is rebuilt by the next linear
         }
-        // ---------------- stage 2 of linear it - kAhead
-        const int mm = it - kAhead;
-        if (mm < 0) continue;
+        __syncwarp();
+    } else {
+        // ---------------- compute warps (named barrier 1)
+        // the x slice (fp32), and the previous launch's exchange words back to zero
+        float *xs = reinterpret_cast<float *>(g_smem + o.xs);
+        for (int i = tid; i < 32 * nw; i += kCT)
+            xs[i] = P.x_fp32 ? static_cast<const float *>(P.x)[32 * iw0 + i]
+                             : bf16_bits_to_float(static_cast<const uint16_t *>(P.x)[32 * iw0 + i]);
         {
+            const size_t a = (size_t)c * words / N, e = (size_t)(c + 1) * words / N;
+            for (size_t i = a + tid; i < e; i += kCT) xold[i] = 0ull;
+        }
+        float *y = reinterpret_cast<float *>(g_smem + o.y);
+        for (int i = tid; i < nrows; i += kCT) y[i] = 0.f;
+        csync_m();
+        const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
+        bool ok = true;
+        // the exchange words a thread polls for stage 2 (its table tid; ntab <=
+        // kCT whenever the ranks sum to at most 1920), loaded while the row
+        // sums of the linear before run, so that the L2 round trip overlaps them
+        unsigned long long pre[4] = {0ull, 0ull, 0ull, 0ull};
+        auto prefetch = [&](int mm) {
+            if (mm < 0 || mm >= P.M || tid >= ntab) return;
+            const int p = tid >= nt0 ? 1 : 0, n = tid - (p ? nt0 : 0);
+            if (4 * n >= P.r[p]) return;
+            const unsigned long long *wd = xw + (size_t)mm * P.N1 + (p ? P.off1 : 0) + 4 * n;
+            ld_relaxed_v2_u64(wd, pre[0], pre[1]);
+            ld_relaxed_v2_u64(wd + 2, pre[2], pre[3]);
+        };
+        for (int it = 0; it < P.M + kAhead && ok; ++it) {
+            if (it == kAhead) prefetch(0);
+            // ---------------- stage 1 of linear it
+            if (it == 0 && nw == 0) {
+                // a CTA without input words still counts itself into linear 0's words
+                for (int i = tid; i < P.N1; i += kCT) red_add_u64(xw + i, 1ull);
+            }
+            if (it < P.M && nw > 0) {
+                const int m = it;
+                unsigned char *b = slot(m);
+                // tables of g . x (8 per input word and path), once the slice landed
+                bool got = true;
+                if (tid == 0) got = wait_bar_m(vbar + m % kSlots, (unsigned)((m / kSlots) & 1), P.ws_words);
+                if (!csync_and_m(got)) {
+                    ok = false;
+                    break;
+                }
+                if (tid != 0) mbar_try_wait(vbar + m % kSlots, (unsigned)((m / kSlots) & 1));
+                for (int idx = tid; idx < np * 8 * nw; idx += kCT) {
+                    const int p = idx / (8 * nw), n = idx - p * 8 * nw;
+                    const float4 xv = *reinterpret_cast<const float4 *>(xs + 4 * n);
+                    const uint2 gw = *reinterpret_cast<const uint2 *>(b + o.g[p] + 8 * n);
+                    const float4 v = make_float4(xv.x * half_bits_to_float((uint16_t)(gw.x & 0xffffu)),
+                                                 xv.y * half_bits_to_float((uint16_t)(gw.x >> 16)),
+                                                 xv.z * half_bits_to_float((uint16_t)(gw.y & 0xffffu)),
+                                                 xv.w * half_bits_to_float((uint16_t)(gw.y >> 16)));
+                    store_table(g_smem + o.t1 + idx * 128, v, lane);
+                }
+                csync_m();
+                unsigned long long *xm = xw + (size_t)m * P.N1;
+                for (int u = warp; u < cbs; u += kCW) {
+                    const int p = u >= R0 ? 1 : 0, cb = u - (p ? R0 : 0);
+                    const int r = P.r[p];
+                    const int col = 32 * cb + lane, cc = min(col, r - 1);
+                    const uint32_t *Vw = reinterpret_cast<const uint32_t *>(b + o.V[p]) + cc;
+                    const uint32_t tb = (uint32_t)(o.t1 + p * 8 * nw * 128);
+                    float acc0 = 0.f, acc1 = 0.f;
+                    int w = 0;
+                    for (; w + 2 <= nw; w += 2) {
+                        const uint32_t w0 = Vw[w * r], w1 = Vw[(w + 1) * r];
+                        acc0 += lut_word(w0, copy, tb + w * 1024);
+                        acc1 += lut_word(w1, copy, tb + (w + 1) * 1024);
+                    }
+                    if (w < nw) acc0 += lut_word(Vw[w * r], copy, tb + w * 1024);
+                    if (col < r)
+                        red_add_u64(xm + (p ? P.off1 : 0) + col, enc_fix(acc0 + acc1, P.fix_limit, err));
+                }
+                csync_m();  // t1 is rebuilt by the next linear
+            }
+            // ---------------- stage 2 of linear it - kAhead
+            const int mm = it - kAhead;
+            if (mm < 0) continue;
             const unsigned long long *xm = xw + (size_t)mm * P.N1;
             unsigned char *b = slot(mm);
             // the slot's U rows, h and l (thread 0 waits, the rest observe the phase)
             bool u_ok = true;
             if (tid == 0) u_ok = wait_bar_m(ubar + mm % kSlots, (unsigned)((mm / kSlots) & 1), P.ws_words);
-            if (!__syncthreads_and(u_ok)) {
+            if (!csync_and_m(u_ok)) {
                 ok = false;
                 break;
             }
             if (tid != 0) mbar_try_wait(ubar + mm % kSlots, (unsigned)((mm / kSlots) & 1));
             int pok = 1;
-            for (int idx = tid; idx < ntab && pok; idx += kMT) {
+            for (int idx = tid; idx < ntab && pok; idx += kCT) {
                 const int p = idx >= nt0 ? 1 : 0, n = idx - (p ? nt0 : 0);
                 const int r = P.r[p];
                 float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -269,22 +291,17 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
                 }
                 store_table(g_smem + o.t2 + idx * 128, v, lane);
             }
-            if (!__syncthreads_and(pok)) {
+            if (!csync_and_m(pok)) {
                 ok = false;
                 break;
             }
+            prefetch(mm + 1);
             // every CTA contributed to linear 0's words before any could
             // complete, so all have read the epoch: the next launch may use
             // the other buffer
             if (mm == 0 && c == 0 && tid == 0) P.ws_words[kEpochWord] = epoch + 1u;
-            // the slot linear mm - 1 freed: refilled by the last warp, idle
-            // while the others sum the rows below
-            if (tid == kIssuer && mm >= 1 && mm - 1 + kSlots < P.M) {
-                issue(mm - 1 + kSlots);
-                s_issued = mm - 1 + kSlots + 1;
-            }
             const int rb = (nrows + 31) >> 5;
-            for (int u = warp; u < np * rb; u += kMW) {
+            for (int u = warp; u < np * rb; u += kCW) {
                 const int p = u / rb, blk = u - p * rb;
                 const int R = (P.r[p] + 31) >> 5;
                 const int row = 32 * blk + lane, rr = min(row, nrows - 1);
@@ -302,8 +319,10 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
                 // at most two paths meet in a row: 0 + a + b is exact in either order
                 if (row < nrows) atomicAdd(y + row, (acc0 + acc1) * hs);
             }
-            __syncthreads();
-            for (int i = tid; i < nrows; i += kMT) {
+            csync_m();
+            // the slot is free for the producer
+            if (tid == 0) mbar_arrive(fbar + mm % kSlots);
+            for (int i = tid; i < nrows; i += kCT) {
                 const size_t at = (size_t)mm * P.d_out + o0 + i;
                 if (P.y_fp32)
                     static_cast<float *>(P.y)[at] = y[i];
@@ -311,11 +330,12 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
                     static_cast<uint16_t *>(P.y)[at] = float_to_bf16_bits(y[i]);
                 y[i] = 0.f;
             }
-            __syncthreads();
+            csync_m();
         }
+        if (!ok && tid == 0) s_ok = 0;
     }
     __syncthreads();
-    if (!ok && tid == 0) {
+    if (!s_ok && tid == 0) {
         // every copy this CTA issued must land before it goes away (the last
         // use of each slot; earlier uses were consumed)
         const int issued = s_issued;
