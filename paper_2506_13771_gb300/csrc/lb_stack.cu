@@ -230,7 +230,28 @@ __device__ __noinline__ void run_s2(int prog, int s) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
     const int u1 = st.first + st.wo[warp + 1];
-    for (int u = st.first + st.wo[warp]; u < u1; ++u) {
+    int u = st.first + st.wo[warp];
+    // two units per pass: their word loops run side by side (a unit has at
+    // least one word; the shorter one re-reads its last word, masked out)
+    for (; u + 2 <= u1; u += 2) {
+        int4 a, b, c, d;
+        item_at(prog, u, a, b);
+        item_at(prog, u + 1, c, d);
+        const uint32_t *U0 = sm_u32(a.x) + min(lane, b.z - 1) * a.y;
+        const uint32_t *U1 = sm_u32(c.x) + min(lane, d.z - 1) * c.y;
+        const int nw = max(a.z, c.z);
+        float acc0 = 0.f, acc1 = 0.f;
+        for (int w = 0; w < nw; ++w) {
+            const int w0 = min(w, a.z - 1), w1 = min(w, c.z - 1);
+            const float v0 = lut_word(U0[w0], copy, (uint32_t)a.w + w0 * 1024);
+            const float v1 = lut_word(U1[w1], copy, (uint32_t)c.w + w1 * 1024);
+            acc0 += w < a.z ? v0 : 0.f;
+            acc1 += w < c.z ? v1 : 0.f;
+        }
+        if (lane < b.z) atomicAdd(sm_f(b.y) + lane, acc0 * half_bits_to_float(sm_u16(b.x)[lane]));
+        if (lane < d.z) atomicAdd(sm_f(d.y) + lane, acc1 * half_bits_to_float(sm_u16(d.x)[lane]));
+    }
+    if (u < u1) {
         int4 a, b;
         item_at(prog, u, a, b);
         const int R = a.y, nw = a.z, nrows = b.z;
@@ -260,7 +281,28 @@ __device__ __noinline__ void run_s1(int prog, int s, unsigned long long *xbase, 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
     const int u1 = st.first + st.wo[warp + 1];
-    for (int u = st.first + st.wo[warp]; u < u1; ++u) {
+    int u = st.first + st.wo[warp];
+    // two units per pass; a unit whose input slice is empty (no words) reads
+    // the first entries of its buffer and table, masked out, and sends zero
+    for (; u + 2 <= u1; u += 2) {
+        int4 a, b, c, d;
+        item_at(prog, u, a, b);
+        item_at(prog, u + 1, c, d);
+        const uint32_t *V0 = sm_u32(a.x) + min(lane, b.y - 1);
+        const uint32_t *V1 = sm_u32(c.x) + min(lane, d.y - 1);
+        const int nw = max(a.z, c.z);
+        float acc0 = 0.f, acc1 = 0.f;
+        for (int w = 0; w < nw; ++w) {
+            const int w0 = max(min(w, a.z - 1), 0), w1 = max(min(w, c.z - 1), 0);
+            const float v0 = lut_word(V0[w0 * a.y], copy, (uint32_t)a.w + w0 * 1024);
+            const float v1 = lut_word(V1[w1 * c.y], copy, (uint32_t)c.w + w1 * 1024);
+            acc0 += w < a.z ? v0 : 0.f;
+            acc1 += w < c.z ? v1 : 0.f;
+        }
+        if (lane < b.y) red_add_u64(xbase + b.x + lane, enc_fix(acc0, limit, err));
+        if (lane < d.y) red_add_u64(xbase + d.x + lane, enc_fix(acc1, limit, err));
+    }
+    if (u < u1) {
         int4 a, b;
         item_at(prog, u, a, b);
         const int r = a.y, nw = a.z, ncols = b.y;
@@ -297,11 +339,13 @@ __device__ __forceinline__ void zero_f(float *p, int n) {
     for (int i = threadIdx.x; i < n; i += kCT) p[i] = 0.f;
 }
 
-// Zero this CTA's stripe of an exchange region whose readers are all done.
-__device__ __forceinline__ void zero_stripe(unsigned long long *region, int len) {
-    const int a = (int)((long long)blockIdx.x * len / gridDim.x);
-    const int b = (int)((long long)(blockIdx.x + 1) * len / gridDim.x);
-    for (int i = a + threadIdx.x; i < b; i += kCT) region[i] = 0ull;
+// Exchange regions of a layer, in the order of their stripe bounds.
+enum { XR_A = 0, XR_Q, XR_B, XR_C, XR_D, XR_N };
+
+// Zero this CTA's stripe [z[0], z[1]) of an exchange region whose readers are
+// all done (the bounds are computed once per launch).
+__device__ __forceinline__ void zero_stripe(unsigned long long *region, const int *z) {
+    for (int i = z[0] + threadIdx.x; i < z[1]; i += kCT) region[i] = 0ull;
 }
 
 __device__ __forceinline__ bool sticky(const unsigned *ws_words) {
@@ -570,6 +614,7 @@ __device__ void producer(const Loader &ld, unsigned long long *empty, unsigned *
 __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params P) {
     __shared__ __align__(8) unsigned long long full[4], empty[4];
     __shared__ int s_last;
+    __shared__ int s_zs[XR_N][2];  // this CTA's stripe of each exchange region
     unsigned *err = P.ws_words + kErrWord;
     if (sticky(P.ws_words)) return;
     if (*reinterpret_cast<const volatile unsigned long long *>(P.ws_words + kPlanWord) != P.plan) {
@@ -595,6 +640,13 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
             mbar_init(empty + b, 1);
         }
         fence_barrier_init();
+    }
+    if (threadIdx.x < XR_N) {
+        const int t = threadIdx.x;
+        const int n = t == XR_A ? P.lenA : t == XR_Q ? P.lenQ : t == XR_B ? P.lenB
+                    : t == XR_C ? P.lenC : P.lenD;
+        s_zs[threadIdx.x][0] = (int)((long long)c * n / N);
+        s_zs[threadIdx.x][1] = (int)((long long)(c + 1) * n / N);
     }
     __syncthreads();
     if (threadIdx.x >= kCT) {
@@ -651,8 +703,6 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         if (!wait_full(full + 0, par, P.ws_words)) FAIL_EXIT();
         if (l > 0) {
             if (!run_poll_tables(pg, A_P2, xp, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
-            zero_stripe(xp + P.offC, P.lenC);
-            zero_stripe(xp + P.offQ, P.lenQ);
             run_s2(pg, A_S2);
             team_sync(pg, A_S2);
         }
@@ -660,6 +710,12 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         csync();
         send_ss(xl + P.offA + ssA);
         run_s1(pg, A_S1, xl, lim, err);
+        // regions C and Q of the previous layer: every CTA has passed the
+        // poll that read them (exchange D, polled above, counts all CTAs)
+        if (l > 0) {
+            zero_stripe(xp + P.offC, s_zs[XR_C]);
+            zero_stripe(xp + P.offQ, s_zs[XR_Q]);
+        }
         zero_f(y, rows_d);
         release(0);
 
@@ -667,12 +723,12 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         if (!wait_full(full + 1, par, P.ws_words)) FAIL_EXIT();
         // tables of v (critical) and of q, k (region Q, sent with region A)
         if (!run_poll_tables(pg, B_P2, xl, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
-        if (l > 0) zero_stripe(xp + P.offD, P.lenD);
         run_s2(pg, B_S2V);  // -> xa
         team_sync(pg, B_S2V);
         run_tables(pg, B_T1, 1.f, o.ssacc);
         csync();
         run_s1(pg, B_S1, xl, lim, err);
+        if (l > 0) zero_stripe(xp + P.offD, s_zs[XR_D]);  // read by phase A's poll
         zero_f(xa, rows_d);
         // ---- off the critical path, while exchange B is in flight: q on R_c,
         //      k and v on K_c (their tables were built with v's)
@@ -694,25 +750,25 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         // ================= phase C: h = a + O(attn) on R_c; stage 1 of gate, up
         if (!wait_full(full + 2, par, P.ws_words)) FAIL_EXIT();
         if (!run_poll_tables(pg, C_P2, xl, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
-        zero_stripe(xl + P.offA, P.lenA);
         run_s2(pg, C_S2);  // -> y
         team_sync(pg, C_S2);
         run_tables(pg, C_T1, 1.f, o.ssacc);  // h = res1 + y -> res0
         csync();
         send_ss(xl + P.offC + ssC);
         run_s1(pg, C_S1, xl, lim, err);
+        zero_stripe(xl + P.offA, s_zs[XR_A]);  // read by phase B's poll
         zero_f(y, rows_d);
         release(2);
 
         // ================= phase D: m = silu(gate) * up on F_c; stage 1 of down
         if (!wait_full(full + 3, par, P.ws_words)) FAIL_EXIT();
         if (!run_poll_tables(pg, D_P2, xl, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
-        zero_stripe(xl + P.offB, P.lenB);
         run_s2(pg, D_S2);  // -> yg, yu
         team_sync(pg, D_S2);
         run_tables(pg, D_T1, 1.f, o.ssacc);  // m = silu(yg) * yu
         csync();
         run_s1(pg, D_S1, xl, lim, err);
+        zero_stripe(xl + P.offB, s_zs[XR_B]);  // read by phase C's poll
         zero_f(yg, rows_f);
         zero_f(yu, rows_f);
         release(3);
@@ -724,8 +780,8 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         unsigned long long *xp = P.xacc + (size_t)(l - 1) * P.acc_layer;
         if (!wait_full(full + 0, (unsigned)(l & 1), P.ws_words)) FAIL_EXIT();
         if (!run_poll_tables(pg, A_P2, xp, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
-        zero_stripe(xp + P.offC, P.lenC);
-        zero_stripe(xp + P.offQ, P.lenQ);
+        zero_stripe(xp + P.offC, s_zs[XR_C]);
+        zero_stripe(xp + P.offQ, s_zs[XR_Q]);
         run_s2(pg, A_S2);
         csync();
         for (int i = threadIdx.x; i < rows_d; i += kCT) P.out[32 * s.dw0 + i] = res0[i] + y[i];
