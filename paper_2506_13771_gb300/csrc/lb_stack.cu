@@ -67,45 +67,49 @@ struct Offsets {
     int c_Uo[2], c_ho[2], c_lo[2], c_Vg[2], c_Vu[2], c_gg[2], c_gu[2];
     // phase D: stage 2 of gate, up, stage 1 of down
     int d_Ug[2], d_Uu[2], d_hg[2], d_hu[2], d_lg[2], d_lu[2], d_Vd[2], d_gd[2];
-    // work areas: stage-2 and stage-1 tables, decoded exchange, residual
-    // stream (two buffers: phase A reads 0 and writes 1, phase C the reverse),
-    // stage-2 outputs (added into, zeroed by their consumer), saved t of q's
-    // second path, the sum-of-squares accumulator, the program
-    int t2, t1, res0, res1, y, xa, yq, yk, yv, yg, yu, ssacc, prog;
+    // work areas: stage-2 and stage-1 tables, residual stream (two buffers:
+    // phase A reads 0 and writes 1, phase C the reverse), the off-path q, k, v
+    // outputs (added into, zeroed once stored), the sum-of-squares
+    // accumulator, the program
+    int t2, t1, res0, res1, yq, yk, yv, ssacc, prog;
 };
 
 // Steps of the per-CTA program (one per table build or unit loop).
-// (*_P2: stage-2 tables straight from the exchange words; *_T1: stage-1
-// tables; *_S2 / *_S1: stage-2 / stage-1 units.)
+// (*_P2: stage-2 tables straight from the exchange words; *_R: row units,
+// stage 2 with the stage-1 tables of its rows; *_S2 / *_S1: stage-2 /
+// stage-1 units.)
 enum StepId {
-    A_P2, A_S2, A_T1, A_S1,
-    B_P2, B_S2V, B_T1, B_S1, B_S2QKV,
-    C_P2, C_S2, C_T1, C_S1,
-    D_P2, D_S2, D_T1, D_S1,
+    A_P2, A_R, A_S1,
+    B_P2, B_R, B_S1, B_S2QKV,
+    C_P2, C_R, C_S1,
+    D_P2, D_R, D_S1,
     N_STEPS
 };
 
 // One program record (8 ints).  Meaning by step kind:
-//   table unit  : tb, n_tab, n_vals, mode, s0, s1, s2, scale   (up to 32
-//                 tables of one job, from its table t0 on; the offsets and
-//                 n_vals are those of table t0)
 //   poll-table  : tb, n_tab, n_vals, mode, e0, scale, ss_el, -  (e0, ss_el:
 //                 exchange word indices in the layer; ss_el < 0: none)
 //   stage-2 unit: U, R, nw, tb, h, out, nrows, -
 //   stage-1 unit: V, r, nw, tb, dst, ncols, -, -
+//   row unit    : a header  n_pair, n_job, mode, nrows, res_in, res_out, -, -
+//                 then per pair two segments (first for lanes 0-15, second
+//                 for lanes 16-31)  U, R, nw, tb, h, -, -, -
+//                 then per table job  tb, g, -, -, -, -, -, -
+//                 (offsets of the unit's first row)
 struct Item {
     int f[8];
 };
-// Table-job modes: source kind in bits 0-1, flags above.
-enum { TAB_PLAIN = 0, TAB_RES = 1, TAB_SILU = 2, TAB_WRITER = 4, TAB_MUL = 8 };
+// Poll-table modes.
+enum { TAB_PLAIN = 0, TAB_MUL = 8 };
+// Row-unit modes: x = A + B;  x = res_in + A + B (stored to res_out, x^2
+// added to the sum of squares);  x = silu(A) * B.
+enum { ROW_SUM = 0, ROW_RES = 1, ROW_SILU = 2 };
 
-// Warp w runs units [first + wo[w], first + wo[w + 1]) of its step.  In a
-// stage-2 step fused with the stage-1 tables of the same rows, team[w] =
-// (named barrier id << 16) | threads of warp w's team (0: no team).
+// Warp w runs units [first + wo[w], first + wo[w + 1]) of its step (records,
+// for a row step).
 struct Step {
     int first;
     int wo[kCW + 1];
-    int team[kCW];
 };
 constexpr int kStepBytes = (int)((N_STEPS * sizeof(Step) + 15) / 16 * 16);
 constexpr int kProgBytes = 16384;  // per CTA, in the workspace and in shared memory
@@ -141,9 +145,6 @@ __device__ __forceinline__ const uint16_t *sm_u16(int off) {
 
 __device__ __forceinline__ float silu(float x) { return x / (1.f + __expf(-x)); }
 
-__device__ __forceinline__ float4 ld_f4(int off) {
-    return *reinterpret_cast<const float4 *>(g_smem + off);
-}
 
 // The program lives in shared memory at byte offset prog; step and unit
 // records are read with shared-memory loads (the step functions take byte
@@ -157,69 +158,82 @@ __device__ __forceinline__ void item_at(int prog, int u, int4 &a, int4 &b) {
     b = *reinterpret_cast<const int4 *>(p + 16);
 }
 
-// Barrier of warp w's team in a fused step (the warps that own the same
-// 32-row blocks): their stage-2 sums are complete after it.
-__device__ __forceinline__ void team_sync(int prog, int s) {
-    const int t = step_at(prog, s).team[threadIdx.x >> 5];
-    if (t) asm volatile("bar.sync %0, %1;" ::"r"(t >> 16), "r"(t & 0xffff) : "memory");
-}
-
-// Table units: lane n builds table n of the unit.  Table n holds, for
-// e = 0..15, sum_{k<4} (bit k of e ? -v : +v) of v_i = x_i * scale_i
-// (* inv with TAB_MUL), i = 4n + k, where x_i is
-//   TAB_PLAIN: s0[i]    TAB_RES: s0[i] + s1[i]    TAB_SILU: silu(s0[i]) * s1[i]
-// (values at or past n_vals are 0, so padding bits add nothing).  It is
-// stored twice (entries e and 16 + e, one copy per half-warp).  A TAB_WRITER
-// unit also stores x into s2 and adds sum x^2 into the float at ss_off.
-// Each lane writes its table's eight 16-byte chunks starting at chunk
-// (lane & 7): the eight lanes of a quarter-warp hit distinct banks.
-__device__ __noinline__ void run_tables(int prog, int s, float inv, int ss_off) {
+// Row units: 16 output rows of a stage-2 step summed whole inside one warp,
+// then the stage-1 tables of those rows, with no shared accumulator and no
+// barrier in between.  Lanes 0-15 take the rows with the first segment of
+// every pair, lanes 16-31 the same rows with the second (the two halves read
+// the two copies of every table, so their lookups never share a bank); one
+// shuffle joins the halves into x (by the unit's mode).  Table job j then
+// gets the unit's four tables, table n of v_i = x_i * g_j[i], i = 4n + k,
+// built by lane 4j + n.  do_s2 = false takes A = B = 0 (the first layer has
+// no previous down); do_tab = false builds no tables (the last phase).
+__device__ __noinline__ void run_rows(int prog, int s, bool do_s2, bool do_tab, int ss_off) {
     const Step &st = step_at(prog, s);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int half = lane >> 4, r = lane & 15;
+    const uint32_t copy = half ? 0x40404040u : 0u;
     const int u1 = st.first + st.wo[warp + 1];
-    for (int u = st.first + st.wo[warp]; u < u1; ++u) {
-        int4 a, b;
-        item_at(prog, u, a, b);
-        const int n_vals = a.z - 4 * lane, mode = a.w;
-        float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
-        float ss = 0.f;
-        if (lane < a.y && n_vals > 0) {
-            x = ld_f4(b.x + 16 * lane);
-            if ((mode & 3) == TAB_RES) {
-                const float4 y = ld_f4(b.y + 16 * lane);
-                x = make_float4(x.x + y.x, x.y + y.y, x.z + y.z, x.w + y.w);
-            } else if ((mode & 3) == TAB_SILU) {
-                const float4 y = ld_f4(b.y + 16 * lane);
-                x = make_float4(silu(x.x) * y.x, silu(x.y) * y.y, silu(x.z) * y.z,
-                                silu(x.w) * y.w);
-            }
-            if (mode & TAB_WRITER) {
-                *reinterpret_cast<float4 *>(g_smem + b.z + 16 * lane) = x;
-                ss = x.x * x.x + x.y * x.y + x.z * x.z + x.w * x.w;
-            }
-            const uint2 hb = *reinterpret_cast<const uint2 *>(g_smem + b.w + 8 * lane);
-            const float m = (mode & TAB_MUL) ? inv : 1.f;
-            x.x *= half_bits_to_float((uint16_t)(hb.x & 0xffffu)) * m;
-            x.y *= half_bits_to_float((uint16_t)(hb.x >> 16)) * m;
-            x.z *= half_bits_to_float((uint16_t)(hb.y & 0xffffu)) * m;
-            x.w *= half_bits_to_float((uint16_t)(hb.y >> 16)) * m;
-        }
-        if (lane < a.y) {
-            unsigned char *T = g_smem + a.x + lane * 128;
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                const int q = (k + lane) & 7;
-                // chunk q: entries 4(q&3) .. +3; high bits (e3 e2) = q & 3
-                const float qv = ((q & 1) ? -x.z : x.z) + ((q & 2) ? -x.w : x.w);
-                *reinterpret_cast<float4 *>(T + 16 * q) = make_float4(
-                    x.x + x.y + qv, x.y - x.x + qv, x.x - x.y + qv, -x.x - x.y + qv);
+    for (int u = st.first + st.wo[warp]; u < u1;) {
+        int4 hd, he;
+        item_at(prog, u, hd, he);
+        const int npair = hd.x, njob = hd.y, mode = hd.z, nrows = hd.w;
+        const int row = min(r, nrows - 1);
+        float acc = 0.f;
+        if (do_s2) {
+            for (int k = 0; k < npair; ++k) {
+                int4 a0, b0, a1, b1;
+                item_at(prog, u + 1 + 2 * k, a0, b0);
+                item_at(prog, u + 2 + 2 * k, a1, b1);
+                // a segment without words points at its partner's rows and
+                // tables: its clamped reads stay in place and are masked out
+                const int nw = half ? a1.z : a0.z, nwm = max(a0.z, a1.z);
+                const uint32_t *Uw = sm_u32(half ? a1.x : a0.x) + row * (half ? a1.y : a0.y);
+                const uint32_t tb = (uint32_t)(half ? a1.w : a0.w);
+                float s0 = 0.f, s1 = 0.f;
+                for (int w = 0; w < nwm; w += 2) {
+                    const int wa = max(min(w, nw - 1), 0), wb = max(min(w + 1, nw - 1), 0);
+                    const float va = lut_word(Uw[wa], copy, tb + wa * 1024);
+                    const float vb = lut_word(Uw[wb], copy, tb + wb * 1024);
+                    s0 += w < nw ? va : 0.f;
+                    s1 += w + 1 < nw ? vb : 0.f;
+                }
+                const float h = half_bits_to_float(sm_u16(half ? b1.x : b0.x)[row]);
+                acc += nw > 0 ? (s0 + s1) * h : 0.f;
             }
         }
-        if (mode & TAB_WRITER) {
+        const float other = __shfl_xor_sync(0xffffffffu, acc, 16);
+        float x = mode == ROW_SILU ? silu(acc) * other : acc + other;
+        if (lane >= nrows) x = 0.f;  // also every lane of the second half
+        if (mode == ROW_RES) {
+            float ss = 0.f;
+            if (lane < nrows) {
+                x += sm_f(he.x)[lane];
+                sm_f(he.y)[lane] = x;
+                ss = x * x;
+            }
 #pragma unroll
-            for (int o = 16; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
+            for (int o = 8; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
             if (lane == 0) atomicAdd(sm_f(ss_off), ss);
         }
+        if (do_tab) {
+            const int n = lane & 3;
+            const float4 v = make_float4(__shfl_sync(0xffffffffu, x, 4 * n),
+                                         __shfl_sync(0xffffffffu, x, 4 * n + 1),
+                                         __shfl_sync(0xffffffffu, x, 4 * n + 2),
+                                         __shfl_sync(0xffffffffu, x, 4 * n + 3));
+            for (int L = lane; L < 4 * njob; L += 32) {
+                int4 ta, tz;
+                item_at(prog, u + 1 + 2 * npair + (L >> 2), ta, tz);
+                const uint2 hb = *reinterpret_cast<const uint2 *>(g_smem + ta.y + 8 * n);
+                const float4 t =
+                    make_float4(v.x * half_bits_to_float((uint16_t)(hb.x & 0xffffu)),
+                                v.y * half_bits_to_float((uint16_t)(hb.x >> 16)),
+                                v.z * half_bits_to_float((uint16_t)(hb.y & 0xffffu)),
+                                v.w * half_bits_to_float((uint16_t)(hb.y >> 16)));
+                store_table(g_smem + ta.x + 128 * n, t, lane);
+            }
+        }
+        u += 1 + 2 * npair + njob;
     }
 }
 
@@ -662,18 +676,16 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         for (int i = threadIdx.x; i < kProgBytes / 16; i += kCT) dst[i] = src[i];
     }
     const int pg = o.prog;
-    const int rows_d = 32 * s.nd, rows_f = 32 * s.nf, nkv = s.nkv;
-    float *res0 = sm_f(o.res0), *y = sm_f(o.y), *xa = sm_f(o.xa), *yq = sm_f(o.yq);
-    float *yk = sm_f(o.yk), *yv = sm_f(o.yv), *yg = sm_f(o.yg), *yu = sm_f(o.yu);
+    const int rows_d = 32 * s.nd, nkv = s.nkv;
+    float *res0 = sm_f(o.res0), *res1 = sm_f(o.res1), *yq = sm_f(o.yq);
+    float *yk = sm_f(o.yk), *yv = sm_f(o.yv);
     float *ssacc = sm_f(o.ssacc);  // sum of squares of this CTA's slice
     for (int i = threadIdx.x; i < rows_d; i += kCT) {
         res0[i] = bf16_bits_to_float(P.x0[32 * s.dw0 + i]);
-        y[i] = xa[i] = yq[i] = 0.f;
+        yq[i] = 0.f;
     }
     zero_f(yk, nkv);
     zero_f(yv, nkv);
-    zero_f(yg, rows_f);
-    zero_f(yu, rows_f);
     if (threadIdx.x == 0) ssacc[0] = 0.f;
     csync();
     int nr[7];
@@ -701,12 +713,9 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
 
         // ================= phase A: a = h + Down_{l-1}(m) on R_c; stage 1 of q, k, v
         if (!wait_full(full + 0, par, P.ws_words)) FAIL_EXIT();
-        if (l > 0) {
-            if (!run_poll_tables(pg, A_P2, xp, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
-            run_s2(pg, A_S2);
-            team_sync(pg, A_S2);
-        }
-        run_tables(pg, A_T1, 1.f, o.ssacc);  // a = res0 + y -> res1
+        if (l > 0 && !run_poll_tables(pg, A_P2, xp, n_ctas, 1.f, inv_d, P.ws_words))
+            FAIL_EXIT();
+        run_rows(pg, A_R, l > 0, true, o.ssacc);  // a = res0 + Down(m) -> res1; tables
         csync();
         send_ss(xl + P.offA + ssA);
         run_s1(pg, A_S1, xl, lim, err);
@@ -716,20 +725,16 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
             zero_stripe(xp + P.offC, s_zs[XR_C]);
             zero_stripe(xp + P.offQ, s_zs[XR_Q]);
         }
-        zero_f(y, rows_d);
         release(0);
 
         // ================= phase B: v rows for attention, stage 1 of o; then q, k, v out
         if (!wait_full(full + 1, par, P.ws_words)) FAIL_EXIT();
         // tables of v (critical) and of q, k (region Q, sent with region A)
         if (!run_poll_tables(pg, B_P2, xl, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
-        run_s2(pg, B_S2V);  // -> xa
-        team_sync(pg, B_S2V);
-        run_tables(pg, B_T1, 1.f, o.ssacc);
+        run_rows(pg, B_R, true, true, o.ssacc);  // v on the attention rows; tables of o
         csync();
         run_s1(pg, B_S1, xl, lim, err);
         if (l > 0) zero_stripe(xp + P.offD, s_zs[XR_D]);  // read by phase A's poll
-        zero_f(xa, rows_d);
         // ---- off the critical path, while exchange B is in flight: q on R_c,
         //      k and v on K_c (their tables were built with v's)
         run_s2(pg, B_S2QKV);  // -> yq, yk, yv
@@ -750,27 +755,20 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         // ================= phase C: h = a + O(attn) on R_c; stage 1 of gate, up
         if (!wait_full(full + 2, par, P.ws_words)) FAIL_EXIT();
         if (!run_poll_tables(pg, C_P2, xl, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
-        run_s2(pg, C_S2);  // -> y
-        team_sync(pg, C_S2);
-        run_tables(pg, C_T1, 1.f, o.ssacc);  // h = res1 + y -> res0
+        run_rows(pg, C_R, true, true, o.ssacc);  // h = res1 + O(attn) -> res0; tables
         csync();
         send_ss(xl + P.offC + ssC);
         run_s1(pg, C_S1, xl, lim, err);
         zero_stripe(xl + P.offA, s_zs[XR_A]);  // read by phase B's poll
-        zero_f(y, rows_d);
         release(2);
 
         // ================= phase D: m = silu(gate) * up on F_c; stage 1 of down
         if (!wait_full(full + 3, par, P.ws_words)) FAIL_EXIT();
         if (!run_poll_tables(pg, D_P2, xl, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
-        run_s2(pg, D_S2);  // -> yg, yu
-        team_sync(pg, D_S2);
-        run_tables(pg, D_T1, 1.f, o.ssacc);  // m = silu(yg) * yu
+        run_rows(pg, D_R, true, true, o.ssacc);  // m = silu(gate) * up; tables of down
         csync();
         run_s1(pg, D_S1, xl, lim, err);
         zero_stripe(xl + P.offB, s_zs[XR_B]);  // read by phase C's poll
-        zero_f(yg, rows_f);
-        zero_f(yu, rows_f);
         release(3);
     }
 
@@ -782,9 +780,9 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         if (!run_poll_tables(pg, A_P2, xp, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
         zero_stripe(xp + P.offC, s_zs[XR_C]);
         zero_stripe(xp + P.offQ, s_zs[XR_Q]);
-        run_s2(pg, A_S2);
+        run_rows(pg, A_R, true, false, o.ssacc);  // a = res0 + Down(m) -> res1
         csync();
-        for (int i = threadIdx.x; i < rows_d; i += kCT) P.out[32 * s.dw0 + i] = res0[i] + y[i];
+        for (int i = threadIdx.x; i < rows_d; i += kCT) P.out[32 * s.dw0 + i] = res1[i];
         // The last CTA to finish has seen every other CTA's reads of the final
         // region: it clears that region and the counters for the next launch.
         if (lead) {
@@ -951,13 +949,9 @@ SmemPlan smem_plan(const lb_linear *lin, const StackShape &sh, int N) {
     at += up(t1, 1024);
     o.res0 = take(4 * 32 * nd);
     o.res1 = take(4 * 32 * nd);
-    o.y = take(4 * 32 * nd);
-    o.xa = take(4 * 32 * nd);
     o.yq = take(4 * 32 * nd);
     o.yk = take(4 * nkv);
     o.yv = take(4 * nkv);
-    o.yg = take(4 * 32 * nf);
-    o.yu = take(4 * 32 * nf);
     o.ssacc = take(16);
     o.prog = take(kProgBytes);
     S.bytes = up(at, 128);
@@ -966,9 +960,6 @@ SmemPlan smem_plan(const lb_linear *lin, const StackShape &sh, int N) {
 
 // ---------------------------------------------------------------- the program
 
-Item tab(int tb, int n_tab, int n_vals, int mode, int s0, int s1, int s2, int scale) {
-    return Item{{tb, n_tab, n_vals, mode, s0, s1, s2, scale}};
-}
 // e0, ss_el: exchange word indices within a layer (ss_el < 0: none)
 Item ptab(int tb, int n_tab, int n_vals, int mode, int e0, int scale, int ss_el) {
     return Item{{tb, n_tab, n_vals, mode, e0, scale, ss_el, 0}};
@@ -1018,6 +1009,17 @@ double lpt(const std::vector<Costed> &us, std::vector<Item> &out, int (&wo)[kCW 
 struct S2Job {
     int U, h, R, rows, tb, out;
 };
+// A row-unit segment at row 0: U rows (R words each, from word 0 of the
+// segment), nw words, the stage-2 tables of word 0 and h.  A segment without
+// words keeps its partner's offsets (its reads are masked).
+struct Seg {
+    int U, R, nw, tb, h;
+};
+// A stage-1 table job of a row step: its table set (128 bytes per 4 rows) and
+// its g, at row 0.
+struct TabJob {
+    int tb, g;
+};
 struct S1Job {
     int V, r, nw, tb, dst;
 };
@@ -1039,60 +1041,62 @@ struct ProgBuild {
             step[s].wo[w + 1] = (int)items.size() - step[s].first;
         }
     }
-    // Table units of one job's tables [t_lo, t_hi), up to 32 per unit.
-    static void table_units(const Item &J, int t_lo, int t_hi, std::vector<Costed> &us) {
-        for (int t0 = t_lo; t0 < std::min(t_hi, J.f[1]); t0 += 32) {
-            const int nt = std::min(32, std::min(t_hi, J.f[1]) - t0);
-            auto sh = [&](int off, int per) { return off + per * t0; };  // unused: never read
-            us.push_back({Item{{J.f[0] + 128 * t0, nt, J.f[2] - 4 * t0, J.f[3], sh(J.f[4], 16),
-                                sh(J.f[5], 16), sh(J.f[6], 16), sh(J.f[7], 8)}},
-                          1.0 + nt / 32.0});
-        }
-    }
-    // Stage 2 fused with the stage-1 tables of its output rows: the 32-row
-    // blocks are split into teams of warps (one named barrier each, ids from
-    // 2); a team computes its blocks' stage-2 sums, meets at its barrier and
-    // builds the tables of those rows (8 per block and job).
-    void fused(int s2s, int t1s, const std::vector<S2Job> &jobs, int rows,
-               const std::vector<Item> &t1jobs) {
-        PerWarp p2, p1;
-        const int nb = (rows + 31) / 32, nteam = std::min(nb, std::min(kCW, 14));
-        int maxR = 1;
-        for (const S2Job &J : jobs) maxR = std::max(maxR, J.R);
-        for (int t = 0; t < nteam; ++t) {
-            const int b0 = nb * t / nteam, b1 = nb * (t + 1) / nteam;
-            const int w0 = kCW * t / nteam, w1 = kCW * (t + 1) / nteam;
-            PerWarp best;
-            double best_mk = 1e300;
-            for (int run = 1; run <= maxR; ++run) {
-                std::vector<Costed> us;
-                for (const S2Job &J : jobs)
-                    for (int b = b0; b < b1; ++b) {
-                        const int r0 = 32 * b;
-                        if (r0 >= J.rows) continue;
-                        for (int q = 0; q < J.R; q += run) {
-                            const int nw = std::min(run, J.R - q);
-                            us.push_back({Item{{J.U + (r0 * J.R + q) * 4, J.R, nw, J.tb + q * 1024,
-                                                J.h + 2 * r0, J.out + 4 * r0,
-                                                std::min(32, J.rows - r0), 0}},
-                                          nw + 1.5});
-                        }
-                    }
-                PerWarp trial;
-                const double mk = lpt_into(us, w0, w1, trial);
-                if (mk < best_mk - 1e-9) {
-                    best_mk = mk;
-                    for (int w = w0; w < w1; ++w) best[w] = trial[w];
-                }
+    // Row units of a stage-2 step (16 rows each, see run_rows): pairs of
+    // segments given at row 0, the table jobs of the rows, the mode and the
+    // residual buffers.  Units go to the warps longest first (cost: the words
+    // of the longer segment of each pair plus a fixed overhead).
+    void rows(int s, const std::vector<std::pair<Seg, Seg>> &pairs,
+              const std::vector<TabJob> &jobs, int mode, int res_in, int res_out, int nrows) {
+        struct Unit {
+            std::vector<Item> it;
+            double cost;
+        };
+        std::vector<Unit> us;
+        for (int r0 = 0; r0 < nrows; r0 += 16) {
+            Unit U{{}, 2.0 + jobs.size() / 8.0};
+            U.it.push_back(Item{{(int)pairs.size(), (int)jobs.size(), mode,
+                                 std::min(16, nrows - r0), res_in + 4 * r0, res_out + 4 * r0, 0,
+                                 0}});
+            for (const auto &pr : pairs) {
+                for (const Seg *g : {&pr.first, &pr.second})
+                    U.it.push_back(Item{{g->U + 4 * r0 * g->R, g->R, g->nw, g->tb, g->h + 2 * r0,
+                                         0, 0, 0}});
+                U.cost += std::max(pr.first.nw, pr.second.nw);
             }
-            for (int w = w0; w < w1; ++w) p2[w] = best[w];
-            std::vector<Costed> ts;
-            for (const Item &J : t1jobs) table_units(J, 8 * b0, 8 * b1, ts);
-            lpt_into(ts, w0, w1, p1);
-            for (int w = w0; w < w1; ++w) step[s2s].team[w] = ((2 + t) << 16) | (32 * (w1 - w0));
+            for (const TabJob &J : jobs)
+                U.it.push_back(Item{{J.tb + 128 * (r0 / 4), J.g + 2 * r0, 0, 0, 0, 0, 0, 0}});
+            us.push_back(U);
         }
-        place(s2s, p2);
-        place(t1s, p1);
+        std::vector<int> idx(us.size());
+        for (size_t i = 0; i < us.size(); ++i) idx[i] = (int)i;
+        std::stable_sort(idx.begin(), idx.end(),
+                         [&](int a, int b) { return us[a].cost > us[b].cost; });
+        PerWarp per;
+        double load[kCW] = {};
+        for (int i : idx) {
+            int w = 0;
+            for (int k = 1; k < kCW; ++k)
+                if (load[k] < load[w]) w = k;
+            load[w] += us[i].cost;
+            per[w].insert(per[w].end(), us[i].it.begin(), us[i].it.end());
+        }
+        place(s, per);
+    }
+    // The segment pair of one linear summed over its paths: path 0 beside
+    // path 1, or one path split into two runs of words.
+    static std::pair<Seg, Seg> sum_pair(const Seg &p0, const Seg *p1) {
+        if (p1) return {p0, *p1};
+        Seg a = p0, b = p0;
+        a.nw = (p0.nw + 1) / 2;
+        b.nw = p0.nw - a.nw;
+        if (b.nw > 0) {
+            b.U += 4 * a.nw;
+            b.tb += 1024 * a.nw;
+        } else {
+            b = a;
+            b.nw = 0;
+        }
+        return {a, b};
     }
     // Poll-table units: the same split, word indices instead of offsets.
     void ptables(int s, const std::vector<Item> &jobs) {
@@ -1182,43 +1186,46 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
         B.s1(s, V);
         V.clear();
     };
-    // phase A: stage 2 of down (previous layer) -> y; stage 1 of q, k, v of
-    // a = res0 + y (written to res1)
+    auto pair_of = [](const std::vector<Seg> &g) {
+        return ProgBuild::sum_pair(g[0], g.size() > 1 ? &g[1] : nullptr);
+    };
+    // phase A: stage 2 of down (previous layer) in row units, a = res0 +
+    // Down(m) written to res1, the stage-1 tables of q, k, v; stage 1 of q, k, v
     {
         int tb = o.t2, off = X.offD;  // words of the previous layer
+        std::vector<Seg> g;
         for (int p = 0; p < np(LD); ++p) {
             T.push_back(ptab(tb, 8 * Rk(LD, p), rk(LD, p), TAB_PLAIN, off, o.a_ld[p], -1));
-            U.push_back({o.a_Ud[p], o.a_hd[p], Rk(LD, p), rows_d, tb, o.y});
+            g.push_back({o.a_Ud[p], Rk(LD, p), Rk(LD, p), tb, o.a_hd[p]});
             tb += Rk(LD, p) * 1024;
             off += rk(LD, p);
         }
         flush_p(A_P2);
         // q, k -> region Q; v -> region A
-        int tb1 = o.t1, dq = X.offQ, dv = X.offA, mode = TAB_RES | TAB_WRITER;
+        std::vector<TabJob> tj;
+        int tb1 = o.t1, dq = X.offQ, dv = X.offA;
         for (int k = 0; k < 3; ++k)
             for (int p = 0; p < np(k); ++p) {
-                T.push_back(tab(tb1, 8 * nd, rows_d, mode, o.res0, o.y, o.res1, o.a_g[k][p]));
+                tj.push_back({tb1, o.a_g[k][p]});
                 int &dst = k == LV ? dv : dq;
                 V.push_back({o.a_V[k][p], rk(k, p), nd, tb1, dst});
-                mode = TAB_RES;
                 tb1 += nd * 1024;
                 dst += rk(k, p);
             }
-        B.fused(A_S2, A_T1, U, rows_d, T);
-        U.clear();
-        T.clear();
+        B.rows(A_R, {pair_of(g)}, tj, ROW_RES, o.res0, o.res1, rows_d);
         flush_v(A_S1);
     }
     // phase B: tables of v, q, k (scaled by the rms factor of a); v on the
-    // attention rows of R_c -> xa; stage 1 of o; then q -> yq, k -> yk and
-    // v on K_c -> yv
+    // attention rows of R_c in row units with the tables of o; stage 1 of o;
+    // then q -> yq, k -> yk and v on K_c -> yv
     {
         const int ssA = X.offA + rsum(lin[LV]);
         int tb = o.t2, tbv[2] = {0, 0}, off = X.offA;
+        std::vector<Seg> g;
         for (int p = 0; p < np(LV); ++p) {
             T.push_back(ptab(tb, 8 * Rk(LV, p), rk(LV, p), TAB_PLAIN | TAB_MUL, off, o.b_lv[p],
                              ssA));
-            U.push_back({o.b_Uat[p], o.b_hat[p], Rk(LV, p), rows_d, tb, o.xa});
+            g.push_back({o.b_Uat[p], Rk(LV, p), Rk(LV, p), tb, o.b_hat[p]});
             tbv[p] = tb;
             tb += Rk(LV, p) * 1024;
             off += rk(LV, p);
@@ -1242,71 +1249,76 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
         for (int p = 0; p < np(LV); ++p)
             Uqkv.push_back({o.b_Uvk[p], o.b_hvk[p], Rk(LV, p), nkv, tbv[p], o.yv});
         flush_p(B_P2);
+        std::vector<TabJob> tj;
         int tb1 = o.t1, dst = X.offB;
         for (int p = 0; p < np(LO); ++p) {
-            T.push_back(tab(tb1, 8 * nd, rows_d, TAB_PLAIN, o.xa, 0, 0, o.b_go[p]));
+            tj.push_back({tb1, o.b_go[p]});
             V.push_back({o.b_Vo[p], rk(LO, p), nd, tb1, dst});
             tb1 += nd * 1024;
             dst += rk(LO, p);
         }
-        B.fused(B_S2V, B_T1, U, rows_d, T);
-        U.clear();
-        T.clear();
+        B.rows(B_R, {pair_of(g)}, tj, ROW_SUM, 0, 0, rows_d);
         flush_v(B_S1);
         U = Uqkv;
         flush_u(B_S2QKV);
     }
-    // phase C: stage 2 of o -> y; stage 1 of gate, up of h = res1 + y
-    // (written to res0); path 1 of q from the saved t -> yq
+    // phase C: stage 2 of o in row units, h = res1 + O(attn) written to res0,
+    // the tables of gate, up; stage 1 of gate, up
     {
         int tb = o.t2, off = X.offB;
+        std::vector<Seg> g;
         for (int p = 0; p < np(LO); ++p) {
             T.push_back(ptab(tb, 8 * Rk(LO, p), rk(LO, p), TAB_PLAIN, off, o.c_lo[p], -1));
-            U.push_back({o.c_Uo[p], o.c_ho[p], Rk(LO, p), rows_d, tb, o.y});
+            g.push_back({o.c_Uo[p], Rk(LO, p), Rk(LO, p), tb, o.c_ho[p]});
             tb += Rk(LO, p) * 1024;
             off += rk(LO, p);
         }
         flush_p(C_P2);
-        int tb1 = o.t1, dst = X.offC, mode = TAB_RES | TAB_WRITER;
+        std::vector<TabJob> tj;
+        int tb1 = o.t1, dst = X.offC;
         for (int k = LG; k <= LU; ++k)
             for (int p = 0; p < np(k); ++p) {
-                T.push_back(tab(tb1, 8 * nd, rows_d, mode, o.res1, o.y, o.res0,
-                                k == LG ? o.c_gg[p] : o.c_gu[p]));
+                tj.push_back({tb1, k == LG ? o.c_gg[p] : o.c_gu[p]});
                 V.push_back({k == LG ? o.c_Vg[p] : o.c_Vu[p], rk(k, p), nd, tb1, dst});
-                mode = TAB_RES;
                 tb1 += nd * 1024;
                 dst += rk(k, p);
             }
-        B.fused(C_S2, C_T1, U, rows_d, T);
-        U.clear();
-        T.clear();
+        B.rows(C_R, {pair_of(g)}, tj, ROW_RES, o.res1, o.res0, rows_d);
         flush_v(C_S1);
     }
-    // phase D: stage 2 of gate, up on F_c -> yg, yu; stage 1 of down of
-    // m = silu(yg) * yu
+    // phase D: stage 2 of gate (lanes 0-15) and up (lanes 16-31) in row
+    // units, m = silu(gate) * up, the tables of down; stage 1 of down
     {
         const int ssC = X.offC + rsum(lin[LG]) + rsum(lin[LU]);
         int tb = o.t2, off = X.offC;
+        std::vector<Seg> gs[2];
         for (int k = LG; k <= LU; ++k)
             for (int p = 0; p < np(k); ++p) {
                 T.push_back(ptab(tb, 8 * Rk(k, p), rk(k, p), TAB_PLAIN | TAB_MUL, off,
                                  k == LG ? o.d_lg[p] : o.d_lu[p], ssC));
-                U.push_back({k == LG ? o.d_Ug[p] : o.d_Uu[p], k == LG ? o.d_hg[p] : o.d_hu[p],
-                             Rk(k, p), rows_f, tb, k == LG ? o.yg : o.yu});
+                gs[k - LG].push_back({k == LG ? o.d_Ug[p] : o.d_Uu[p], Rk(k, p), Rk(k, p), tb,
+                                      k == LG ? o.d_hg[p] : o.d_hu[p]});
                 tb += Rk(k, p) * 1024;
                 off += rk(k, p);
             }
         flush_p(D_P2);
+        std::vector<std::pair<Seg, Seg>> pairs;
+        for (size_t p = 0; p < std::max(gs[0].size(), gs[1].size()); ++p) {
+            Seg a = p < gs[0].size() ? gs[0][p] : gs[1][p];
+            Seg b = p < gs[1].size() ? gs[1][p] : gs[0][p];
+            if (p >= gs[0].size()) a.nw = 0;
+            if (p >= gs[1].size()) b.nw = 0;
+            pairs.push_back({a, b});
+        }
+        std::vector<TabJob> tj;
         int tb1 = o.t1, dst = X.offD;
         for (int p = 0; p < np(LD); ++p) {
-            T.push_back(tab(tb1, 8 * nf, rows_f, TAB_SILU, o.yg, o.yu, 0, o.d_gd[p]));
+            tj.push_back({tb1, o.d_gd[p]});
             V.push_back({o.d_Vd[p], rk(LD, p), nf, tb1, dst});
             tb1 += nf * 1024;
             dst += rk(LD, p);
         }
-        B.fused(D_S2, D_T1, U, rows_f, T);
-        U.clear();
-        T.clear();
+        B.rows(D_R, pairs, tj, ROW_SILU, 0, 0, rows_f);
         flush_v(D_S1);
     }
     if ((int)B.items.size() > kMaxItems) return false;
