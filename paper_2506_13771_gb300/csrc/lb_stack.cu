@@ -22,11 +22,13 @@
 //    values, stored twice so the two half-warps use disjoint banks; a 32-bit
 //    sign word costs 8 table lookups (PRMT forms the address, LDS reads it);
 //  * the compute warps run a per-CTA program built on the host by
-//    littlebit_stack_prepare: for every step, table jobs and warp-balanced
-//    work units (32 rows x a run of words, or 32 columns x the slice) with
-//    their shared-memory offsets.  The shapes are those of every layer, so
-//    the program is the same for all of them; the device code is a handful
-//    of generic loops, small enough to stay in the instruction cache;
+//    littlebit_stack_prepare: for every step, warp-balanced work units with
+//    their shared-memory offsets -- stage-2 tables polled from the exchange,
+//    row units (16 output rows of a critical linear summed whole by one warp,
+//    the two half-warps on the two paths (or on gate and up), followed by
+//    the stage-1 tables of those rows), 32 columns x the slice for stage 1.
+//    The shapes are those of every layer, so the program is the same for all
+//    of them; the device code is a handful of generic loops;
 //  * the all-reduce of t accumulates fixed-point values in 64-bit words whose
 //    low 8 bits count contributions: each CTA adds (round(v * 2^24) << 8) + 1
 //    with one red.add per element and readers poll the words they need until
