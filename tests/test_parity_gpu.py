@@ -506,6 +506,23 @@ def test_stack_ragged_slices():
     check_stack(run_stack(layers, x0, 32), oracle.stack_forward(layers, x0, head_dim=32))
 
 
+def test_stack_mixed_paths_and_ranks():
+    """Per-linear path counts and unequal path ranks (Eq. 6 allows both): one-path
+    linears split their words across the half-warps, a gate of two paths meets an
+    up of one, and paths of unequal rank run side by side with masked words."""
+    rng = inputs.rng_for(104)
+    d, dkv, dff = 512, 128, 1024
+    spec = [(d, d, [40]), (d, dkv, [8, 24]), (d, dkv, [16, 8]), (d, d, [48, 16]),
+            (d, dff, [56, 24]), (d, dff, [40]), (dff, d, [32, 64])]
+    layers = []
+    for _ in range(2):
+        for di, do, rs in spec:
+            c = inputs.unit_gain_scale(di, sum(rs) // len(rs), len(rs))
+            layers.append(inputs.make_linear(rng, di, do, rs, len(rs), c))
+    x0 = inputs.bf16_normal(rng, (d,))
+    check_stack(run_stack(layers, x0, 64), oracle.stack_forward(layers, x0, head_dim=64))
+
+
 def test_stack_workspace_reuse_and_plan_check():
     """Back-to-back launches on one prepared workspace agree (the launch leaves
     it clean); a workspace prepared for other linears is refused on the
