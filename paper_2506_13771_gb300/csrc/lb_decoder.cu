@@ -118,23 +118,39 @@ struct RopeFreq {
     double inv_freq[kMaxHeadDim / 2];
 };
 
-// Attention of query head h = blockIdx.x, thread i = dimension i of the head
-// (HD = head_dim threads).  kc / vc: this layer's cache rows [max_pos][d_kv].
-// Rows t < p come from the cache (earlier steps); row p is this step's rotated
-// k and v, which the first query head of each kv head also writes into the
+// Attention splits per query head: the positions 0..p are cut into kSplits
+// runs handled by kSplits CTAs (flash-decoding), so that a long context
+// spreads over the SMs instead of one CTA per head.
+constexpr int kSplits = 8;
+
+// Attention of query head h = blockIdx.x over its run sp = blockIdx.y of the
+// positions, thread i = dimension i of the head (HD = head_dim threads).
+// kc / vc: this layer's cache rows [max_pos][d_kv].  Rows t < p come from the
+// cache (earlier steps); row p is this step's rotated k and v, which the run
+// holding p of the first query head of each kv head also writes into the
 // cache.  Scores and the weighted values each take kU positions per warp at a
-// time with every load of those positions in flight together.
+// time with every load of those positions in flight together.  Each run
+// leaves (sum_t e^(s_t - m) v_t, m, sum_t e^(s_t - m)) over its positions in
+// part; the last run of a head to finish (a counter in cnt, which it resets)
+// rescales the runs to their common maximum and writes the head's output.
 template <int HD>
 __global__ void __launch_bounds__(HD)
     k_dec_attention(const float *q, const float *k, const float *v, float *kc, float *vc,
-                    float *attn, int n_heads, int n_kv_heads, int max_pos,
-                    const __grid_constant__ RopeFreq F, const int *pos, const unsigned *hdr) {
+                    float *attn, float *part, unsigned *cnt, int n_heads, int n_kv_heads,
+                    int max_pos, const __grid_constant__ RopeFreq F, const int *pos,
+                    const unsigned *hdr) {
     constexpr int kU = 8, NW = HD / 32, PER = HD / 32;
     extern __shared__ float sm[];
+    __shared__ int s_last;
     if (!dec_ok(hdr)) return;
     const int half = HD / 2, i = threadIdx.x;
-    const int h = blockIdx.x, group = n_heads / n_kv_heads, g = h / group;
+    const int h = blockIdx.x, sp = blockIdx.y, S = gridDim.y;
+    const int group = n_heads / n_kv_heads, g = h / group;
     const int dkv = n_kv_heads * HD, p = *pos;
+    // this run's positions [t_lo, t_hi), possibly none
+    const int n = p + 1, chunk = (n + S - 1) / S;
+    const int t_lo = min(n, sp * chunk), t_hi = min(n, t_lo + chunk);
+    const bool has_p = t_lo <= p && p < t_hi;
     float *qs = sm, *ks = sm + HD, *red = sm + 2 * HD, *sc = sm + 2 * HD + 32;
     float *vsum = sc + max_pos;  // [NW][HD]
     qs[i] = q[h * HD + i];
@@ -153,7 +169,7 @@ __global__ void __launch_bounds__(HD)
     __syncthreads();
     qs[i] = qr;
     ks[i] = kr;
-    if (h % group == 0) {
+    if (has_p && h % group == 0) {
         kc[(size_t)p * dkv + g * HD + i] = kr;
         vc[(size_t)p * dkv + g * HD + i] = vi;
     }
@@ -163,7 +179,7 @@ __global__ void __launch_bounds__(HD)
 #pragma unroll
     for (int e = 0; e < PER; ++e) qreg[e] = qs[lane + 32 * e];
     const float scale = 1.f / sqrtf((float)HD);
-    for (int t0 = warp * kU; t0 <= p; t0 += NW * kU) {
+    for (int t0 = t_lo + warp * kU; t0 < t_hi; t0 += NW * kU) {
         float kv[kU][PER];
 #pragma unroll
         for (int u = 0; u < kU; ++u) {
@@ -171,7 +187,8 @@ __global__ void __launch_bounds__(HD)
             const float *kt = t < p ? kc + (size_t)t * dkv + g * HD : ks;
 #pragma unroll
             for (int e = 0; e < PER; ++e)
-                kv[u][e] = t < p ? __ldg(kt + lane + 32 * e) : (t == p ? kt[lane + 32 * e] : 0.f);
+                kv[u][e] = t < min(p, t_hi) ? __ldg(kt + lane + 32 * e)
+                                            : (t == p ? kt[lane + 32 * e] : 0.f);
         }
 #pragma unroll
         for (int u = 0; u < kU; ++u) {
@@ -179,15 +196,16 @@ __global__ void __launch_bounds__(HD)
 #pragma unroll
             for (int e = 0; e < PER; ++e) acc += qreg[e] * kv[u][e];
             acc = warp_sum(acc);
-            if (lane == 0 && t0 + u <= p) sc[t0 + u] = acc * scale;
+            if (lane == 0 && t0 + u < t_hi) sc[t0 + u - t_lo] = acc * scale;
         }
     }
     __syncthreads();
+    const int len = t_hi - t_lo;
     float mx = -INFINITY;
-    for (int t = i; t <= p; t += HD) mx = fmaxf(mx, sc[t]);
+    for (int t = i; t < len; t += HD) mx = fmaxf(mx, sc[t]);
     mx = cta_reduce<true>(mx, red);
     float sum = 0.f;
-    for (int t = i; t <= p; t += HD) {
+    for (int t = i; t < len; t += HD) {
         const float e = expf(sc[t] - mx);
         sc[t] = e;
         sum += e;
@@ -195,32 +213,56 @@ __global__ void __launch_bounds__(HD)
     sum = cta_reduce<false>(sum, red);  // its barriers also publish sc
     // weighted values: the same split of positions over warps; the warps'
     // partial vectors meet in shared memory
-    float part[PER];
+    float pv[PER];
 #pragma unroll
-    for (int e = 0; e < PER; ++e) part[e] = 0.f;
-    for (int t0 = warp * kU; t0 < p; t0 += NW * kU) {
+    for (int e = 0; e < PER; ++e) pv[e] = 0.f;
+    const int t_end = min(t_hi, p);  // cached rows of the run
+    for (int t0 = t_lo + warp * kU; t0 < t_end; t0 += NW * kU) {
         float vv[kU][PER];
 #pragma unroll
         for (int u = 0; u < kU; ++u) {
             const int t = t0 + u;
-            const float *vt = vc + (size_t)(t < p ? t : 0) * dkv + g * HD + lane;
+            const float *vt = vc + (size_t)(t < t_end ? t : t_lo) * dkv + g * HD + lane;
 #pragma unroll
-            for (int e = 0; e < PER; ++e) vv[u][e] = t < p ? __ldg(vt + 32 * e) : 0.f;
+            for (int e = 0; e < PER; ++e) vv[u][e] = t < t_end ? __ldg(vt + 32 * e) : 0.f;
         }
 #pragma unroll
         for (int u = 0; u < kU; ++u) {
-            const float w = t0 + u < p ? sc[t0 + u] : 0.f;
+            const float w = t0 + u < t_end ? sc[t0 + u - t_lo] : 0.f;
 #pragma unroll
-            for (int e = 0; e < PER; ++e) part[e] += w * vv[u][e];
+            for (int e = 0; e < PER; ++e) pv[e] += w * vv[u][e];
         }
     }
 #pragma unroll
-    for (int e = 0; e < PER; ++e) vsum[warp * HD + lane + 32 * e] = part[e];
+    for (int e = 0; e < PER; ++e) vsum[warp * HD + lane + 32 * e] = pv[e];
     __syncthreads();
-    float acc = sc[p] * vi;
+    float acc = has_p ? sc[p - t_lo] * vi : 0.f;
 #pragma unroll
     for (int w = 0; w < NW; ++w) acc += vsum[w * HD + i];
-    attn[h * HD + i] = acc / sum;
+    float *mine = part + ((size_t)h * S + sp) * (HD + 2);
+    mine[i] = acc;
+    if (i == 0) {
+        mine[HD] = mx;    // -inf for a run without positions
+        mine[HD + 1] = sum;
+    }
+    __threadfence();
+    __syncthreads();
+    if (i == 0) s_last = atomicAdd(cnt + h, 1u) == (unsigned)(S - 1);
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    const float *runs = part + (size_t)h * S * (HD + 2);
+    float M = -INFINITY;
+    for (int r = 0; r < S; ++r) M = fmaxf(M, __ldcg(runs + r * (HD + 2) + HD));
+    float L = 0.f, O = 0.f;
+    for (int r = 0; r < S; ++r) {
+        const float m_r = __ldcg(runs + r * (HD + 2) + HD);
+        const float w = m_r == -INFINITY ? 0.f : expf(m_r - M);
+        L += w * __ldcg(runs + r * (HD + 2) + HD + 1);
+        O += w * __ldcg(runs + r * (HD + 2) + i);
+    }
+    attn[h * HD + i] = O / L;
+    if (i == 0) cnt[h] = 0u;
 }
 
 size_t align256(size_t b) { return (b + 255) & ~(size_t)255; }
@@ -229,7 +271,7 @@ struct DecLayout {
     size_t slot[7];        // byte offsets of the seven single-linear workspaces
     size_t slot_bytes[7];
     size_t qkv_ws, qkv_bytes, gu_ws, gu_bytes;  // the two multi-linear workspaces
-    size_t n, attn, m, q, k, v, y, g, u, a, end;
+    size_t n, attn, m, q, k, v, y, g, u, a, part, cnt, end;
 };
 
 // The grouped launches of a layer: q with k and v when all three have one
@@ -270,6 +312,8 @@ DecLayout dec_layout(const lb_linear *lin, const lb_decoder_shape &S) {
     o.g = take(2 * dff * 4);        // gate, up back to back
     o.u = o.g + dff * 4;
     o.a = take(d * 4);
+    o.part = take((size_t)S.n_heads * kSplits * (S.head_dim + 2) * 4);  // attention runs
+    o.cnt = take((size_t)S.n_heads * 4);                                 // zero between steps
     o.end = off;
     return o;
 }
@@ -366,6 +410,8 @@ lb_status littlebit_decoder_step(const lb_linear *lin, const lb_decoder_shape *S
     float *v = reinterpret_cast<float *>(w + o.v), *y = reinterpret_cast<float *>(w + o.y);
     float *g = reinterpret_cast<float *>(w + o.g), *u = reinterpret_cast<float *>(w + o.u);
     float *a = reinterpret_cast<float *>(w + o.a);
+    float *part = reinterpret_cast<float *>(w + o.part);
+    unsigned *cnt = reinterpret_cast<unsigned *>(w + o.cnt);
     const int d = S->n_heads * S->head_dim, dkv = S->n_kv_heads * S->head_dim;
     const int dff = lin[4].d_out, D = S->head_dim;
     const size_t layer_rows = (size_t)S->max_pos * dkv;
@@ -406,15 +452,19 @@ lb_status littlebit_decoder_step(const lb_linear *lin, const lb_decoder_shape *S
             return st;
         }
         float *kl = kcache + l * layer_rows, *vl = vcache + l * layer_rows;
+        const dim3 agrid(S->n_heads, kSplits);
         if (D == 64)
-            k_dec_attention<64><<<S->n_heads, 64, attn_smem, s>>>(
-                q, k, v, kl, vl, attn, S->n_heads, S->n_kv_heads, S->max_pos, freq, pos, hdr);
+            k_dec_attention<64><<<agrid, 64, attn_smem, s>>>(q, k, v, kl, vl, attn, part, cnt,
+                                                            S->n_heads, S->n_kv_heads,
+                                                            S->max_pos, freq, pos, hdr);
         else if (D == 128)
-            k_dec_attention<128><<<S->n_heads, 128, attn_smem, s>>>(
-                q, k, v, kl, vl, attn, S->n_heads, S->n_kv_heads, S->max_pos, freq, pos, hdr);
+            k_dec_attention<128><<<agrid, 128, attn_smem, s>>>(q, k, v, kl, vl, attn, part, cnt,
+                                                              S->n_heads, S->n_kv_heads,
+                                                              S->max_pos, freq, pos, hdr);
         else
-            k_dec_attention<256><<<S->n_heads, 256, attn_smem, s>>>(
-                q, k, v, kl, vl, attn, S->n_heads, S->n_kv_heads, S->max_pos, freq, pos, hdr);
+            k_dec_attention<256><<<agrid, 256, attn_smem, s>>>(q, k, v, kl, vl, attn, part, cnt,
+                                                              S->n_heads, S->n_kv_heads,
+                                                              S->max_pos, freq, pos, hdr);
         if ((st = from_err(cudaGetLastError())) != LB_OK) return st;
         if ((st = linear(l, 3, attn, y)) != LB_OK) return st;
         k_dec_residual<<<1, kNormThreads, 0, s>>>(a, y, n, d, nullptr, nullptr, hdr);

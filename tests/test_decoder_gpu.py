@@ -118,6 +118,17 @@ def test_decoder_step_replays_as_a_graph(orc):
     run_and_compare(orc, layers, shape, xs, max_pos=6, graph=True)
 
 
+def test_decoder_long_context(orc):
+    """200 tokens through one GQA layer with heads of 128 (the benchmark's head
+    size): attention over up to 200 cached positions, many times the positions
+    one pass of the attention kernel's warps covers, checked at every step."""
+    rng = inputs.rng_for(112)
+    layers, shape = small(rng, n_layers=1, n_heads=4, n_kv_heads=2, head_dim=128, d_ff=256,
+                          r=(32, 32, 32))
+    xs = inputs.bf16_normal(rng, (200, 512))
+    run_and_compare(orc, layers, shape, xs, max_pos=256)
+
+
 def test_decoder_7b_shape_first_tokens(orc):
     """The Llama2-7B-shaped workload of the benchmark (32 layers, 32 heads of
     128, d_ff 11008, two LittleBit paths per linear): its first three tokens."""
