@@ -37,8 +37,8 @@ struct DecodeLayout {
 
 struct DecodeParams {
     LinDesc L;
-    const void *x;     // bf16 [d_in], or fp32 when x_fp32
-    int x_fp32;
+    const void *x;     // bf16 [d_in]; fp32 [d_in] (x_fp32 = 1); fp32 [2][d_in] (x_fp32 = 2)
+    int x_fp32;        // 2: the input is silu(x[0][i]) * x[1][i] (a decoder MLP's gate, up)
     void *y;
     int y_fp32;
     unsigned *ws_words;
@@ -114,10 +114,19 @@ __global__ void __launch_bounds__(kDT, 1) k_decode(const __grid_constant__ Decod
     for (int p = 0; p < np; ++p) {
         const uint16_t *g = p ? L.g[1] : L.g[0];
         float *xg = reinterpret_cast<float *>(g_smem + o.xg[p]);
-        for (int i = tid; i < 32 * nw; i += kDT)
-            xg[i] = (P.x_fp32 ? static_cast<const float *>(P.x)[32 * iw0 + i]
-                              : bf16_bits_to_float(static_cast<const uint16_t *>(P.x)[32 * iw0 + i])) *
-                    half_bits_to_float(g[32 * iw0 + i]);
+        for (int i = tid; i < 32 * nw; i += kDT) {
+            const int e = 32 * iw0 + i;
+            float xe;
+            if (P.x_fp32 == 2) {
+                const float *xf = static_cast<const float *>(P.x);
+                const float gt = xf[e];
+                xe = xf[L.d_in + e] * (gt / (1.f + expf(-gt)));
+            } else {
+                xe = P.x_fp32 ? static_cast<const float *>(P.x)[e]
+                              : bf16_bits_to_float(static_cast<const uint16_t *>(P.x)[e]);
+            }
+            xg[i] = xe * half_bits_to_float(g[e]);
+        }
     }
     float *y = reinterpret_cast<float *>(g_smem + o.y);
     for (int i = tid; i < nrows; i += kDT) y[i] = 0.f;

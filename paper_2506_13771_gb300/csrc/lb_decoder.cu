@@ -102,16 +102,6 @@ __global__ void __launch_bounds__(kNormThreads)
     }
 }
 
-// m = up . silu(gate), silu(x) = x / (1 + e^-x).
-__global__ void k_dec_silu(const float *gate, const float *up, float *m, int n,
-                           const unsigned *hdr) {
-    if (!dec_ok(hdr)) return;
-    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) {
-        const float g = gate[i];
-        m[i] = up[i] * (g / (1.f + expf(-g)));
-    }
-}
-
 // Rotary inverse frequencies base^(-2j/D), j < D/2, computed on the host in
 // fp64 (a kernel argument).
 struct RopeFreq {
@@ -271,7 +261,7 @@ struct DecLayout {
     size_t slot[7];        // byte offsets of the seven single-linear workspaces
     size_t slot_bytes[7];
     size_t qkv_ws, qkv_bytes, gu_ws, gu_bytes;  // the two multi-linear workspaces
-    size_t n, attn, m, q, k, v, y, g, u, a, part, cnt, end;
+    size_t n, attn, q, k, v, y, g, u, a, part, cnt, end;
 };
 
 // The grouped launches of a layer: q with k and v when all three have one
@@ -304,7 +294,6 @@ DecLayout dec_layout(const lb_linear *lin, const lb_decoder_shape &S) {
     };
     o.n = take(d * 4);
     o.attn = take(d * 4);
-    o.m = take(dff * 4);
     o.q = take((d + 2 * dkv) * 4);  // q, k, v back to back (the rows of a grouped launch)
     o.k = o.q + d * 4;
     o.v = o.k + dkv * 4;
@@ -405,7 +394,6 @@ lb_status littlebit_decoder_step(const lb_linear *lin, const lb_decoder_shape *S
     unsigned *hdr = reinterpret_cast<unsigned *>(w);
     float *n = reinterpret_cast<float *>(w + o.n);
     float *attn = reinterpret_cast<float *>(w + o.attn);
-    float *m = reinterpret_cast<float *>(w + o.m);
     float *q = reinterpret_cast<float *>(w + o.q), *k = reinterpret_cast<float *>(w + o.k);
     float *v = reinterpret_cast<float *>(w + o.v), *y = reinterpret_cast<float *>(w + o.y);
     float *g = reinterpret_cast<float *>(w + o.g), *u = reinterpret_cast<float *>(w + o.u);
@@ -421,9 +409,10 @@ lb_status littlebit_decoder_step(const lb_linear *lin, const lb_decoder_shape *S
         freq.inv_freq[j] = std::pow((double)S->rope_base, -2.0 * (double)j / (double)D);
     const int sms = sm_count();
     if (sms < 1 || !decode_supported(lin[0], sms)) return LB_ERR_UNSUPPORTED;
-    auto linear = [&](int l, int j, const float *xin, float *yout) {
+    // x_mode 1: fp32 input; 2: silu(xin[i]) * xin[d_in + i] (gate, up back to back)
+    auto linear = [&](int l, int j, const float *xin, float *yout, int x_mode = 1) {
         char *slot = w + o.slot[j];
-        const cudaError_t e = launch_decode(lin[7 * (size_t)l + j], xin, 1, yout, 1,
+        const cudaError_t e = launch_decode(lin[7 * (size_t)l + j], xin, x_mode, yout, 1,
                                             reinterpret_cast<unsigned *>(slot), slot + kWsHeader,
                                             sms, s);
         return e == cudaErrorCooperativeLaunchTooLarge ? LB_ERR_UNSUPPORTED : from_err(e);
@@ -439,7 +428,6 @@ lb_status littlebit_decoder_step(const lb_linear *lin, const lb_decoder_shape *S
     const DecGroups G = groups_of(lin, sms);
     k_dec_start<<<1, kNormThreads, 0, s>>>(x, a, n, d, pos, S->max_pos, hdr);
     if ((st = from_err(cudaGetLastError())) != LB_OK) return st;
-    const int silu_blocks = (dff + 255) / 256;
     for (int l = 0; l < S->n_layers; ++l) {
         const bool last = l + 1 == S->n_layers;
         if (G.qkv == 3) {
@@ -474,9 +462,8 @@ lb_status littlebit_decoder_step(const lb_linear *lin, const lb_decoder_shape *S
         } else if ((st = linear(l, 4, n, g)) != LB_OK || (st = linear(l, 5, n, u)) != LB_OK) {
             return st;
         }
-        k_dec_silu<<<silu_blocks, 256, 0, s>>>(g, u, m, dff, hdr);
-        if ((st = from_err(cudaGetLastError())) != LB_OK) return st;
-        if ((st = linear(l, 6, m, y)) != LB_OK) return st;
+        // down reads silu(gate) * up straight from the gate / up outputs
+        if ((st = linear(l, 6, g, y, 2)) != LB_OK) return st;
         k_dec_residual<<<1, kNormThreads, 0, s>>>(a, y, last ? nullptr : n, d, last ? out : nullptr,
                                                   last ? pos : nullptr, hdr);
         if ((st = from_err(cudaGetLastError())) != LB_OK) return st;
