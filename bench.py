@@ -694,7 +694,7 @@ def run_config(args):
         # end-to-end decoding of a Llama2-7B-shaped decoder whose linears are
         # LittleBit (the paper's tokens-per-second setting, shape only): 128
         # and 256 new tokens from an empty cache, one decode step per token
-        # replayed as a CUDA graph (inputs resident; the step's 225 launches
+        # replayed as a CUDA graph (inputs resident; the step's 162 launches
         # are the per-token critical path)
         S = inputs.DECODER_7B
         for n_new in (128, 256):
@@ -741,8 +741,10 @@ def run_config(args):
             line = {"config": 9, "case": name, "op": "decode", "tokens": n_new, "ms": ms,
                     "tokens_per_s": n_new / ms * 1e3, "ms_per_token": ms / n_new,
                     "bytes_per_token": (wbytes + cache) / n_new, "gbs": gbs,
-                    # q/k/v and gate/up grouped, SiLU read inside down
-                    "launches_per_token": 1 + 7 * S["n_layers"],
+                    # per layer q/k/v (grouped, the residual add and norm
+                    # folded in), attention, o, gate/up (likewise), down
+                    # (SiLU read inside); plus the first norm and the last add
+                    "launches_per_token": 2 + 5 * S["n_layers"],
                     "roofline": {"bound": "hbm", "achieved": gbs, "peak": hbm, "unit": "GB/s",
                                  "frac": gbs / hbm, "peak_source": "MEASURED_PEAKS.json hbm_gbs"},
                     "context": "paper Table 12 (A100, Llama2-7B, 0.1 BPW, 128 new tokens): 203.20 "

@@ -328,11 +328,13 @@ size_t littlebit_decoder_workspace_size(const lb_linear *lin, const lb_decoder_s
  * workspace's error word and the step writes nothing (read it with
  * littlebit_decoder_poll_error).  Every linear's d_out and ranks must be
  * multiples of 8 (else LB_ERR_UNSUPPORTED).  ws: zero-filled before first
- * use, not shared with concurrent calls.  Enqueues 1 + (7 .. 10) * n_layers
- * launches on the stream: per layer the single-token LittleBit linears, with
- * q / k / v (or k / v) and gate / up each grouped into one launch when they
- * share a shape (as littlebit_linear_forward_multi) and down reading
- * silu(gate) * up itself, and the attention and norm kernels. */
+ * use, not shared with concurrent calls.  Enqueues 2 + 5 * n_layers launches
+ * on the stream when q / k / v share a shape (up to 1 + 10 * n_layers
+ * otherwise): per layer the single-token LittleBit linears, with q / k / v
+ * (or k / v) and gate / up each grouped into one launch when they share a
+ * shape (as littlebit_linear_forward_multi) -- a grouped launch also does the
+ * residual add and RMS norm ahead of it -- down reading silu(gate) * up
+ * itself, the attention kernel, and the norm kernels the grouping leaves. */
 lb_status littlebit_decoder_step(const lb_linear *lin, const lb_decoder_shape *S,
                                  const uint16_t *x, float *kcache, float *vcache, int32_t *pos,
                                  float *out, void *ws, size_t ws_bytes, lb_stream_t stream);

@@ -417,21 +417,28 @@ lb_status littlebit_decoder_step(const lb_linear *lin, const lb_decoder_shape *S
                                             sms, s);
         return e == cudaErrorCooperativeLaunchTooLarge ? LB_ERR_UNSUPPORTED : from_err(e);
     };
-    // linears j .. j + M - 1 of layer l in one launch (outputs back to back)
-    auto group = [&](int l, int j, int M, size_t ws_off, const float *xin, float *yout) {
+    // linears j .. j + M - 1 of layer l in one launch (outputs back to back);
+    // with fold, their input is a += y and they apply rho themselves
+    auto group = [&](int l, int j, int M, size_t ws_off, const float *xin, float *yout,
+                     bool fold = false) {
         char *gw = w + ws_off;
-        const cudaError_t e = launch_decode_multi(&lin[7 * (size_t)l + j], M, xin, 1, yout, 1,
+        const cudaError_t e = launch_decode_multi(&lin[7 * (size_t)l + j], M, fold ? nullptr : xin,
+                                                  fold ? 3 : 1, yout, 1,
                                                   reinterpret_cast<unsigned *>(gw),
-                                                  gw + kWsHeader, sms, s);
+                                                  gw + kWsHeader, sms, s, fold ? a : nullptr,
+                                                  fold ? y : nullptr);
         return e == cudaErrorCooperativeLaunchTooLarge ? LB_ERR_UNSUPPORTED : from_err(e);
     };
     const DecGroups G = groups_of(lin, sms);
     k_dec_start<<<1, kNormThreads, 0, s>>>(x, a, n, d, pos, S->max_pos, hdr);
     if ((st = from_err(cudaGetLastError())) != LB_OK) return st;
+    // The residual add and RMS norm ahead of a grouped launch run inside it
+    // (a += y, its outputs scaled by 1 / rms(a)): ahead of gate / up always,
+    // ahead of q / k / v when the three are grouped (from layer 1 on).
     for (int l = 0; l < S->n_layers; ++l) {
         const bool last = l + 1 == S->n_layers;
         if (G.qkv == 3) {
-            if ((st = group(l, 0, 3, o.qkv_ws, n, q)) != LB_OK) return st;
+            if ((st = group(l, 0, 3, o.qkv_ws, n, q, l > 0)) != LB_OK) return st;
         } else if (G.qkv == 2) {
             if ((st = linear(l, 0, n, q)) != LB_OK || (st = group(l, 1, 2, o.qkv_ws, n, k)) != LB_OK)
                 return st;
@@ -455,18 +462,22 @@ lb_status littlebit_decoder_step(const lb_linear *lin, const lb_decoder_shape *S
                                                               S->max_pos, freq, pos, hdr);
         if ((st = from_err(cudaGetLastError())) != LB_OK) return st;
         if ((st = linear(l, 3, attn, y)) != LB_OK) return st;
-        k_dec_residual<<<1, kNormThreads, 0, s>>>(a, y, n, d, nullptr, nullptr, hdr);
-        if ((st = from_err(cudaGetLastError())) != LB_OK) return st;
         if (G.gu) {
-            if ((st = group(l, 4, 2, o.gu_ws, n, g)) != LB_OK) return st;
-        } else if ((st = linear(l, 4, n, g)) != LB_OK || (st = linear(l, 5, n, u)) != LB_OK) {
-            return st;
+            if ((st = group(l, 4, 2, o.gu_ws, nullptr, g, true)) != LB_OK) return st;
+        } else {
+            k_dec_residual<<<1, kNormThreads, 0, s>>>(a, y, n, d, nullptr, nullptr, hdr);
+            if ((st = from_err(cudaGetLastError())) != LB_OK) return st;
+            if ((st = linear(l, 4, n, g)) != LB_OK || (st = linear(l, 5, n, u)) != LB_OK)
+                return st;
         }
         // down reads silu(gate) * up straight from the gate / up outputs
         if ((st = linear(l, 6, g, y, 2)) != LB_OK) return st;
-        k_dec_residual<<<1, kNormThreads, 0, s>>>(a, y, last ? nullptr : n, d, last ? out : nullptr,
-                                                  last ? pos : nullptr, hdr);
-        if ((st = from_err(cudaGetLastError())) != LB_OK) return st;
+        if (last || G.qkv != 3) {
+            k_dec_residual<<<1, kNormThreads, 0, s>>>(a, y, last ? nullptr : n, d,
+                                                      last ? out : nullptr, last ? pos : nullptr,
+                                                      hdr);
+            if ((st = from_err(cudaGetLastError())) != LB_OK) return st;
+        }
     }
     return LB_OK;
 }

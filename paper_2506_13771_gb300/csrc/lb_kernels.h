@@ -44,12 +44,15 @@ cudaError_t launch_decode(const lb_linear &L, const void *x, int x_fp32, void *y
                           unsigned *ws_words, void *xw, int num_sms, cudaStream_t s);
 
 // T = 1 through M linears of one shape that read the same x (lb_multi.cu).
+// x_fp32: 0 bf16 x, 1 fp32 x, 3 residual input: x = res_a + res_y (fp32,
+// written back to res_a) and every output scaled by 1 / rms(x).
 constexpr int kMaxMultiLinears = 24;
 bool multi_supported(const lb_linear *L, int M, int num_sms);
 size_t multi_ws_bytes(const lb_linear &L, int M);
 cudaError_t launch_decode_multi(const lb_linear *L, int M, const void *x, int x_fp32, void *y,
                                 int y_fp32, unsigned *ws_words, void *xw, int num_sms,
-                                cudaStream_t s);
+                                cudaStream_t s, float *res_a = nullptr,
+                                const float *res_y = nullptr);
 
 // Persistent decode of the seven-linear-per-layer stack (lb_stack.cu).
 struct StackShape {

@@ -15,7 +15,12 @@
 // slot being refilled once its linear's stage 2 is done (kSlots - kAhead
 // iterations ahead of its stage 1).  The exchange words of all M linears are
 // double-buffered by the workspace's launch epoch as in k_decode: every CTA
-// clears its stripe of the previous launch's buffer.  Every wait is bounded;
+// clears its stripe of the previous launch's buffer.  In the residual-input
+// mode (a decoder's a += y ahead of its q / k / v or gate / up) each CTA adds
+// its input slice into a, sends its share of sum(a^2) in one more exchange
+// word, and the outputs are scaled by 1 / rms(a) (the linears are homogeneous:
+// L(a / rms a) = L(a) / rms a), so no separate norm launch is needed.  Every
+// wait is bounded;
 // on a timeout the CTA records LB_ERR_TIMEOUT, lets its own copies land and
 // returns.
 #include <mutex>
@@ -48,8 +53,13 @@ struct MultiLayout {
 
 struct MultiParams {
     int d_in, d_out, np, r[2], M, N1, off1;
-    const void *x;  // bf16 [d_in], or fp32 when x_fp32
-    int x_fp32;
+    const void *x;  // bf16 [d_in] (x_fp32 = 0), or fp32 (x_fp32 = 1)
+    int x_fp32;     // 3: residual input, see res_a
+    // x_fp32 = 3: x = res_a + res_y (fp32 [d_in]), written back to res_a, and
+    // every output scaled by 1 / rms(x) (a decoder's residual add and RMS
+    // norm ahead of its linears: L(x / rms x) = L(x) / rms x)
+    float *res_a;
+    const float *res_y;
     void *y;        // [M][d_out], bf16 or fp32
     int y_fp32;
     unsigned *ws_words;
@@ -90,12 +100,17 @@ __device__ __forceinline__ int csync_and_m(int pred) {
 __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__ MultiParams P) {
     __shared__ __align__(8) unsigned long long vbar[kSlots], ubar[kSlots], fbar[kSlots];
     __shared__ int s_ok, s_issued;
+    __shared__ float s_ss, s_inv;  // residual input: sum of squares of the slice, 1 / rms
     unsigned *err = P.ws_words + kErrWord;
     if (ld_relaxed_gpu(err) != 0u) return;
     const unsigned epoch = ld_relaxed_gpu(P.ws_words + kEpochWord);
-    const size_t words = (size_t)P.M * P.N1;
-    unsigned long long *xw = P.xw + (size_t)(epoch & 1u) * words;
-    unsigned long long *xold = P.xw + (size_t)((epoch + 1u) & 1u) * words;
+    // a buffer holds M * N1 words of t, then the sum-of-squares word and one
+    // spare word (N1 is a sum of multiples of 8, so the stride keeps the
+    // second buffer 16-byte aligned for the paired 64-bit loads)
+    const size_t words = (size_t)P.M * P.N1, stride = words + 2;
+    unsigned long long *xw = P.xw + (size_t)(epoch & 1u) * stride;
+    unsigned long long *xold = P.xw + (size_t)((epoch + 1u) & 1u) * stride;
+    const bool res = P.x_fp32 == 3;
     const MultiLayout &o = P.o;
     const int N = gridDim.x, c = blockIdx.x, tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31, np = P.np;
@@ -120,6 +135,8 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
         fence_barrier_init();
         s_ok = 1;
         s_issued = 0;
+        s_ss = 0.f;
+        s_inv = 1.f;
     }
     __syncthreads();
     auto slot = [&](int m) { return g_smem + o.slots + (m % kSlots) * o.slot_bytes; };
@@ -161,16 +178,34 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
         // ---------------- compute warps (named barrier 1)
         // the x slice (fp32), and the previous launch's exchange words back to zero
         float *xs = reinterpret_cast<float *>(g_smem + o.xs);
-        for (int i = tid; i < 32 * nw; i += kCT)
-            xs[i] = P.x_fp32 ? static_cast<const float *>(P.x)[32 * iw0 + i]
-                             : bf16_bits_to_float(static_cast<const uint16_t *>(P.x)[32 * iw0 + i]);
+        float ss = 0.f;
+        for (int i = tid; i < 32 * nw; i += kCT) {
+            const int e = 32 * iw0 + i;
+            float v;
+            if (res) {
+                v = P.res_a[e] + P.res_y[e];
+                P.res_a[e] = v;  // this CTA's inputs only
+                ss += v * v;
+            } else {
+                v = P.x_fp32 ? static_cast<const float *>(P.x)[e]
+                             : bf16_bits_to_float(static_cast<const uint16_t *>(P.x)[e]);
+            }
+            xs[i] = v;
+        }
+        if (res) {
+#pragma unroll
+            for (int of = 16; of > 0; of >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, of);
+            if (lane == 0) atomicAdd(&s_ss, ss);
+        }
         {
-            const size_t a = (size_t)c * words / N, e = (size_t)(c + 1) * words / N;
+            const size_t a = (size_t)c * stride / N, e = (size_t)(c + 1) * stride / N;
             for (size_t i = a + tid; i < e; i += kCT) xold[i] = 0ull;
         }
         float *y = reinterpret_cast<float *>(g_smem + o.y);
         for (int i = tid; i < nrows; i += kCT) y[i] = 0.f;
         csync_m();
+        // every CTA's share of the sum of squares, counted like linear 0's words
+        if (res && tid == 0) red_add_u64(xw + words, enc_fix(s_ss, P.fix_limit, err));
         const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
         bool ok = true;
         // the exchange words a thread polls for stage 2 (its table tid; ntab <=
@@ -248,6 +283,28 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
             }
             if (tid != 0) mbar_try_wait(ubar + mm % kSlots, (unsigned)((mm / kSlots) & 1));
             int pok = 1;
+            if (res && mm == 0 && tid == 0) {
+                // the sum of squares of the whole input (all CTAs counted)
+                unsigned long long wv = 0, t0 = 0;
+                for (int spin = 0;; ++spin) {
+                    wv = ld_relaxed_u64(xw + words);
+                    if (counted(wv, n_first)) break;
+                    if ((spin & 15) == 15) {
+                        if (ld_relaxed_gpu(err) != 0u) {
+                            pok = 0;
+                            break;
+                        }
+                        const unsigned long long now = globaltimer_ns();
+                        if (t0 == 0) t0 = now;
+                        if (now - t0 > kWaitLimitNs) {
+                            atomicCAS(err, 0u, static_cast<unsigned>(LB_ERR_TIMEOUT));
+                            pok = 0;
+                            break;
+                        }
+                    }
+                }
+                if (pok) s_inv = rsqrtf(dec_fix(wv) / (float)P.d_in);
+            }
             for (int idx = tid; idx < ntab && pok; idx += kCT) {
                 const int p = idx >= nt0 ? 1 : 0, n = idx - (p ? nt0 : 0);
                 const int r = P.r[p];
@@ -322,12 +379,13 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
             csync_m();
             // the slot is free for the producer
             if (tid == 0) mbar_arrive(fbar + mm % kSlots);
+            const float sc = s_inv;  // 1 unless the input is a residual add
             for (int i = tid; i < nrows; i += kCT) {
                 const size_t at = (size_t)mm * P.d_out + o0 + i;
                 if (P.y_fp32)
-                    static_cast<float *>(P.y)[at] = y[i];
+                    static_cast<float *>(P.y)[at] = y[i] * sc;
                 else
-                    static_cast<uint16_t *>(P.y)[at] = float_to_bf16_bits(y[i]);
+                    static_cast<uint16_t *>(P.y)[at] = float_to_bf16_bits(y[i] * sc);
                 y[i] = 0.f;
             }
             csync_m();
@@ -428,12 +486,14 @@ bool multi_supported(const lb_linear *L, int M, int num_sms) {
 }
 
 size_t multi_ws_bytes(const lb_linear &L, int M) {
-    return ((size_t)2 * M * rsum(L) * sizeof(unsigned long long) + 255) & ~(size_t)255;
+    // two buffers of M * rsum words of t, a sum-of-squares word and a spare
+    return ((size_t)2 * ((size_t)M * rsum(L) + 2) * sizeof(unsigned long long) + 255) &
+           ~(size_t)255;
 }
 
 cudaError_t launch_decode_multi(const lb_linear *L, int M, const void *x, int x_fp32, void *y,
                                 int y_fp32, unsigned *ws_words, void *xw, int num_sms,
-                                cudaStream_t s) {
+                                cudaStream_t s, float *res_a, const float *res_y) {
     int max_smem = 0;
     cudaError_t e = multi_setup(&max_smem);
     if (e != cudaSuccess) return e;
@@ -449,6 +509,8 @@ cudaError_t launch_decode_multi(const lb_linear *L, int M, const void *x, int x_
     P.off1 = A.path[0].r;
     P.x = x;
     P.x_fp32 = x_fp32;
+    P.res_a = res_a;
+    P.res_y = res_y;
     P.y = y;
     P.y_fp32 = y_fp32;
     P.ws_words = ws_words;
