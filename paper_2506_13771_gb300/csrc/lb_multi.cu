@@ -17,7 +17,7 @@
 // double-buffered by the workspace's launch epoch as in k_decode: every CTA
 // clears its stripe of the previous launch's buffer.  In the residual-input
 // mode (a decoder's a += y ahead of its q / k / v or gate / up) each CTA adds
-// its input slice into a, sends its share of sum(a^2) in one more exchange
+// its input slice into a, sends its share of mean(a^2) in one more exchange
 // word, and the outputs are scaled by 1 / rms(a) (the linears are homogeneous:
 // L(a / rms a) = L(a) / rms a), so no separate norm launch is needed.  Every
 // wait is bounded;
@@ -204,8 +204,11 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
         float *y = reinterpret_cast<float *>(g_smem + o.y);
         for (int i = tid; i < nrows; i += kCT) y[i] = 0.f;
         csync_m();
-        // every CTA's share of the sum of squares, counted like linear 0's words
-        if (res && tid == 0) red_add_u64(xw + words, enc_fix(s_ss, P.fix_limit, err));
+        // every CTA's share of the mean square (sum / d_in: the fixed-point
+        // word then holds outlier-sized activations too), counted like linear
+        // 0's words
+        if (res && tid == 0)
+            red_add_u64(xw + words, enc_fix(s_ss / (float)P.d_in, P.fix_limit, err));
         const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
         bool ok = true;
         // the exchange words a thread polls for stage 2 (its table tid; ntab <=
@@ -303,7 +306,7 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
                         }
                     }
                 }
-                if (pok) s_inv = rsqrtf(dec_fix(wv) / (float)P.d_in);
+                if (pok) s_inv = rsqrtf(dec_fix(wv));
             }
             for (int idx = tid; idx < ntab && pok; idx += kCT) {
                 const int p = idx >= nt0 ? 1 : 0, n = idx - (p ? nt0 : 0);
