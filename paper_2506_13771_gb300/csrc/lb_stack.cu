@@ -389,15 +389,15 @@ __device__ __noinline__ bool run_poll_tables(int prog, int s, const unsigned lon
     for (int u = st.first + st.wo[warp]; u < u1 && ok; ++u) {
         int4 a, b;
         item_at(prog, u, a, b);
-        // lane 0 first waits, gently, for the unit's first word: the words
-        // of a region complete at about the same time, and one poller per
-        // warp keeps the L2 free for the contributions still arriving
+        // lane 0 first waits for the unit's last word (its stage-1 column
+        // block is sent after those of the unit's other words): one poller
+        // per warp keeps the L2 free for the contributions still arriving,
+        // and once it sees its word complete the whole unit usually is
         if (lane == 0 && a.z > 0) {
             const unsigned long long t0 = globaltimer_ns();
-            while (!counted(ld_relaxed_u64(xbase + b.x), n_ctas)) {
-                __nanosleep(64);
-                if (globaltimer_ns() - t0 > kWaitLimitNs) break;  // the full wait below decides
-            }
+            const unsigned long long *gw = xbase + b.x + (min(a.z, 4 * a.y) - 1);
+            for (int spin = 0; !counted(ld_relaxed_u64(gw), n_ctas); ++spin)
+                if ((spin & 15) == 15 && globaltimer_ns() - t0 > kWaitLimitNs) break;
         }
         __syncwarp();
         if (lane >= a.y) continue;
