@@ -401,7 +401,7 @@ lb_status littlebit_decoder_step(const lb_linear *lin, const lb_decoder_shape *S
     float *part = reinterpret_cast<float *>(w + o.part);
     unsigned *cnt = reinterpret_cast<unsigned *>(w + o.cnt);
     const int d = S->n_heads * S->head_dim, dkv = S->n_kv_heads * S->head_dim;
-    const int dff = lin[4].d_out, D = S->head_dim;
+    const int D = S->head_dim;
     const size_t layer_rows = (size_t)S->max_pos * dkv;
     const size_t attn_smem = (size_t)(2 * D + 32 + S->max_pos + D * D / 32) * sizeof(float);
     RopeFreq freq{};
