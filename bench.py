@@ -206,70 +206,119 @@ def recorded_traffic(kernel: str, sha: str):
 # ----------------------------------------------------------------- CPU oracle legs
 
 
-def oracle_sample_seconds(layers, x0, n_sample_layers: int, reps: int):
-    import oracle
-    o = oracle.default()
-    o.set_threads(os.cpu_count() or 1)
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu, else /proc/cpuinfo, else platform)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    import platform
+    return platform.machine()
+
+
+def host_weight_bytes(layers) -> int:
+    """Sign words and fp16 scales of every linear, as the device holds them."""
+    return int(sum(P[k].nbytes for L in layers for P in L["paths"]
+                   for k in ("v_words", "u_words", "g", "l", "h")))
+
+
+def stack_io_bytes(n_layers: int) -> int:
+    """x0 (bf16) in; the final hidden state, q and k / v of every layer (fp32) out."""
+    s = __import__("paper_2506_13771_gb300.inputs", fromlist=["STACK_70B"]).STACK_70B
+    return 2 * s["d_model"] + 4 * s["d_model"] + 4 * n_layers * (s["d_model"] + 2 * s["d_kv"])
+
+
+def line_config(n_layers: int, world: int, weight_bytes: int) -> dict:
+    """The bench line's config, the same for both arms."""
+    return dict(workload_config(n_layers), parallelism=f"replicas{world}",
+                bytes_per_token=weight_bytes + stack_io_bytes(n_layers),
+                l2=("no flush: weights %.2f GB > %d MB L2, streamed from DRAM every step"
+                    if weight_bytes > L2_BYTES else
+                    "no flush: weights %.2f GB fit the %d MB L2 (a shortened profiling stack)")
+                   % (weight_bytes / 1e9, L2_BYTES >> 20))
+
+
+def oracle_chain_seconds(o, layers, x0, n_chain: int, reps: int) -> list:
+    """Wall times of `reps` runs of the oracle's decode chain over the first
+    n_chain layers (7 linears, attention at position 0, norms; fp64)."""
     times = []
     for _ in range(reps):
         t0 = time.perf_counter()
-        o.stack_forward(layers[:7 * n_sample_layers], x0, head_dim=128, want_q=True,
-                        want_kv=True)
+        o.stack_forward(layers[:7 * n_chain], x0, head_dim=128, want_q=True, want_kv=True)
         times.append(time.perf_counter() - t0)
-    return statistics.median(times), o.get_threads()
+    return times
 
 
 def cpu_baseline(layers, x0, n_layers: int) -> dict:
-    """The fp64 oracle's decode chain over the whole stack, repeated until
-    about 10 s of CPU work (at most 1 s when a single pass is slower)."""
-    t1, cores = oracle_sample_seconds(layers, x0, n_layers, 1)
+    """The fp64 oracle's decode chain over the whole stack on all host cores,
+    repeated until about 10 s of work (median), and a one-thread figure from
+    the chain over the first layers (about 5 s), scaled to the whole stack."""
+    import oracle
+    o = oracle.default()
+    o.set_threads(os.cpu_count() or 1)
+    t1 = oracle_chain_seconds(o, layers, x0, n_layers, 1)[0]
     reps = max(1, min(50, int(10.0 / max(t1, 1e-3))))
-    t, cores = oracle_sample_seconds(layers, x0, n_layers, reps) if reps > 1 else (t1, cores)
+    t = statistics.median(oracle_chain_seconds(o, layers, x0, n_layers, reps)) if reps > 1 else t1
+    cores = o.get_threads()
+    # one thread: as many leading layers as take about 5 s (the per-layer work is uniform)
+    o.set_threads(1)
+    per_layer_guess = t / n_layers * max(1, cores)
+    n1 = max(1, min(n_layers, int(5.0 / max(per_layer_guess, 1e-4))))
+    s1 = oracle_chain_seconds(o, layers, x0, n1, 1)[0] * n_layers / n1
+    o.set_threads(cores)
     return {"value": 1.0 / t, "unit": "tokens/s", "cores": cores, "kind": "oracle",
-            "sample": f"fp64 oracle decode chain over all {n_layers} layers, median of {reps} "
-                      f"run(s) of {t:.3f} s"}
+            "cpu_model": cpu_model(),
+            "sample": f"fp64 oracle decode chain over all {n_layers} layers on {cores} threads, "
+                      f"median of {reps} run(s) of {t:.3f} s",
+            "threads_1": {"value": 1.0 / s1, "unit": "tokens/s",
+                          "sample": f"chain over the first {n1} of {n_layers} layers on one "
+                                    f"thread, scaled by {n_layers}/{n1}"}}
 
 
 def run_reference(args):
-    """The fp64 CPU oracle on the same metric; one step = one LittleBit linear
-    of layer 0 (cycling q, k, v, o, gate, up, down), tokens/s extrapolated from
-    the mean time of each linear type x n_layers."""
-    import numpy as np
-
+    """The fp64 CPU oracle on the same metric and workload: each step is the
+    oracle's decode chain (the full stack, or -- when K + W steps of it would
+    take more than about 150 s -- its first n layers, tokens/s scaled by
+    n / n_layers) on all host cores; the line's value is the median step."""
     import oracle
     from paper_2506_13771_gb300 import inputs
     world, rank, _ = dist_env()
     if rank != 0:
         return
-    layers, x0 = inputs.make_stack(n_layers=1)
+    kw = {k: v for k, v in inputs.STACK_70B.items() if k not in ("n_layers",)}
+    layers, x0 = inputs.make_stack(n_layers=args.layers, **kw)
     o = oracle.default()
     o.set_threads(os.cpu_count() or 1)
-    rng = np.random.default_rng(0)
-    xin = [rng.standard_normal((1, L["d_in"])) for L in layers]
-    per_type = [[] for _ in range(7)]
-    for i in range(args.warmup + args.steps):
-        k = i % 7
-        t0 = time.perf_counter()
-        o.apply_factored(layers[k], xin[k])
-        dt = time.perf_counter() - t0
-        if i >= args.warmup:
-            per_type[k].append(dt)
-    covered = [statistics.mean(v) for v in per_type if v]
-    if len(covered) < 7:
-        # fewer than 7 timed steps: fall back on the types that were timed
-        per_layer = statistics.mean(covered) * 7
-    else:
-        per_layer = sum(covered)
-    value = 1.0 / (per_layer * args.layers)
+    probe = oracle_chain_seconds(o, layers, x0, args.layers, 1)[0]
+    n_steps = max(1, args.steps + args.warmup)
+    n_chain = args.layers
+    if n_steps * probe > 150.0:
+        n_chain = max(1, int(150.0 / (n_steps * probe / args.layers)))
+    times = oracle_chain_seconds(o, layers, x0, n_chain, n_steps)[args.warmup:] or [probe]
+    per_token = statistics.median(times) * args.layers / n_chain
+    value = 1.0 / per_token
+    sample = (f"fp64 oracle decode chain over {'all' if n_chain == args.layers else 'the first'} "
+              f"{n_chain} of {args.layers} layers per step on {o.get_threads()} threads, median "
+              f"of {len(times)} step(s)" + ("" if n_chain == args.layers else
+                                            f", scaled by {args.layers}/{n_chain}"))
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
             "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
-            "ms_per_step": 1e3 * per_layer / 7, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": workload_config(args.layers),
+            "ms_per_step": 1e3 * per_token, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data":
+                "synthetic (seeded random sign bits and fp16 scales; no trained weights)",
+            "config": line_config(args.layers, world, host_weight_bytes(layers)),
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": o.get_threads(),
-                             "kind": "oracle",
-                             "sample": "one LittleBit linear of layer 0 per step, cycling "
-                                       "q,k,v,o,gate,up,down; x n_layers"},
+                             "kind": "oracle", "cpu_model": cpu_model(), "sample": sample},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -304,6 +353,7 @@ def run_ours(args):
     kv_out = torch.empty((S.n_layers, 2, S.d_kv), dtype=torch.float32, device=dev)
     io_bytes = x0.numel() * 2 + out.numel() * 4 + q_out.numel() * 4 + kv_out.numel() * 4
     step_bytes = weight_bytes + io_bytes
+    assert weight_bytes == host_weight_bytes(layers) and io_bytes == stack_io_bytes(args.layers)
     stream = torch.cuda.current_stream(dev)
 
     def step():
@@ -388,10 +438,7 @@ def run_ours(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic (seeded random sign bits and fp16 scales; no trained weights)",
-        "config": dict(workload_config(args.layers), parallelism=f"replicas{world}",
-                       bytes_per_token=step_bytes,
-                       l2="no flush: weights %.2f GB > %d MB L2, streamed from DRAM every step"
-                          % (weight_bytes / 1e9, L2_BYTES >> 20)),
+        "config": line_config(args.layers, world, host_weight_bytes(layers)),
         "hbm_gbs": achieved,
         "roofline": {"bound": "hbm", "kernel": "k_stack", "achieved": achieved,
                      "peak": peak, "peak_source": peak_src, "unit": "GB/s",
