@@ -375,9 +375,12 @@ lb_status littlebit_linear_forward_multi(const lb_linear *L, int32_t M, const ui
  * nothing and calls no allocating routine.
  *   - Limit: T * (sum of the paths' ranks) <= 65536 fp32 values; a larger
  *     request returns LB_ERR_WORKSPACE without launching anything.
- *   - The first call on each device looks up the array's device address
- *     (cudaGetSymbolAddress, with that device current); make that first call
- *     before any stream capture.  Later calls reuse the address.
+ *   - The first call in each CUDA context looks up the array's device
+ *     address (cudaGetSymbolAddress, with that context's device current);
+ *     make that first call before any stream capture.  Later calls in the
+ *     same context reuse the address; a new context on the device (after
+ *     cudaDeviceReset, or another context made current) gets a fresh
+ *     look-up on its first call, which again belongs before any capture.
  *   - Each call clears the part of the array it uses before adding into it,
  *     but the array keeps the last call's contents afterwards.  Calls whose
  *     kernels overlap on the GPU (different streams, or different host

@@ -5,8 +5,11 @@
 // Scratch: kNoAllocFloats fp32 words (256 KiB) in a file-scope __device__
 // array.  Every GPU that loads the library holds it until the process exits.
 // Host code cannot use the array's name as a device address, so the first
-// call on each device looks the address up with cudaGetSymbolAddress (with
-// that device current) and caches it; later calls reuse it.
+// call in each CUDA context looks the address up with cudaGetSymbolAddress
+// (with that context's device current) and caches it with the context
+// handle; later calls in the same context reuse it.  A new context on the
+// device (after cudaDeviceReset, or another context made current) reloads
+// the module, so the address is looked up again rather than reused.
 #include <mutex>
 
 #include "lb_common.cuh"
@@ -21,16 +24,39 @@ __device__ __align__(256) float g_noalloc_scratch[kNoAllocFloats];
 
 std::mutex g_mu;
 float *g_scratch_ptr[kMaxDevices];
+void *g_scratch_ctx[kMaxDevices];  // the context the cached address belongs to
 
-// Device address of g_noalloc_scratch on the current device (set up once).
+// cuCtxGetCurrent through the runtime's driver entry point (no link to libcuda).
+using CtxGetCurrentFn = int (*)(void **);
+CtxGetCurrentFn ctx_get_current() {
+    static CtxGetCurrentFn fn = [] {
+        void *f = nullptr;
+        cudaDriverEntryPointQueryResult q{};
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000, cudaEnableDefault,
+                                             &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            f = nullptr;
+        return reinterpret_cast<CtxGetCurrentFn>(f);
+    }();
+    return fn;
+}
+
+// Device address of g_noalloc_scratch in the current context (looked up on
+// the first call in each context).
 lb_status scratch_on_current_device(float **out) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return LB_ERR_CUDA;
+    const CtxGetCurrentFn get = ctx_get_current();
+    void *ctx = nullptr;
+    if (!get || get(&ctx) != 0) return LB_ERR_CUDA;
     std::lock_guard<std::mutex> lock(g_mu);
-    if (!g_scratch_ptr[dev]) {
+    if (!ctx || !g_scratch_ptr[dev] || g_scratch_ctx[dev] != ctx) {
+        // (also makes the device's primary context current when none was)
         void *p = nullptr;
         if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return LB_ERR_CUDA;
+        if (get(&ctx) != 0 || !ctx) return LB_ERR_CUDA;
         g_scratch_ptr[dev] = static_cast<float *>(p);
+        g_scratch_ctx[dev] = ctx;
     }
     *out = g_scratch_ptr[dev];
     return LB_OK;

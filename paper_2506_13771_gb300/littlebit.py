@@ -260,15 +260,29 @@ def new_workspace(nbytes: int, device="cuda") -> torch.Tensor:
     return torch.zeros(max(int(nbytes), 256), dtype=torch.uint8, device=device)
 
 
-def linear_forward(L: DeviceLinear, x: torch.Tensor, out_dtype=torch.bfloat16,
-                   y: torch.Tensor | None = None, ws: torch.Tensor | None = None,
-                   stream=None) -> torch.Tensor:
-    """Y = X W^T (Prop. 1 per path, Eq. 6 sum) for x bf16 [T][d_in] on device."""
+def _forward_args(L: DeviceLinear, x: torch.Tensor, out_dtype, y: torch.Tensor | None):
+    """Checks x (bf16 [T][d_in] on the current CUDA device) and the output y
+    ([T][d_out], bf16 or fp32, contiguous, on x's device), allocating y when
+    it is None; returns (contiguous x, y)."""
     assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.shape[1] == L.d_in
+    assert x.is_cuda and x.device.index == torch.cuda.current_device(), \
+        "x must be on the current CUDA device"
     x = x.contiguous()
     T = x.shape[0]
     if y is None:
         y = torch.empty((T, L.d_out), dtype=out_dtype, device=x.device)
+    assert tuple(y.shape) == (T, L.d_out), (tuple(y.shape), (T, L.d_out))
+    assert y.dtype in (torch.bfloat16, torch.float32) and y.is_contiguous()
+    assert y.device == x.device
+    return x, y
+
+
+def linear_forward(L: DeviceLinear, x: torch.Tensor, out_dtype=torch.bfloat16,
+                   y: torch.Tensor | None = None, ws: torch.Tensor | None = None,
+                   stream=None) -> torch.Tensor:
+    """Y = X W^T (Prop. 1 per path, Eq. 6 sum) for x bf16 [T][d_in] on device."""
+    x, y = _forward_args(L, x, out_dtype, y)
+    T = x.shape[0]
     y_dtype = LB_OUT_FP32 if y.dtype == torch.float32 else LB_OUT_BF16
     if ws is None:
         ws = new_workspace(workspace_size(L, T), x.device)
@@ -497,11 +511,8 @@ def linear_forward_noalloc(L: DeviceLinear, x: torch.Tensor, out_dtype=torch.bfl
                            y: torch.Tensor | None = None, stream=None) -> torch.Tensor:
     """Y = X W^T without a workspace: the library's built-in scratch is used
     (for callers that cannot allocate device memory; see littlebit.h)."""
-    assert x.dtype == torch.bfloat16 and x.dim() == 2 and x.shape[1] == L.d_in
-    x = x.contiguous()
+    x, y = _forward_args(L, x, out_dtype, y)
     T = x.shape[0]
-    if y is None:
-        y = torch.empty((T, L.d_out), dtype=out_dtype, device=x.device)
     y_dtype = LB_OUT_FP32 if y.dtype == torch.float32 else LB_OUT_BF16
     _check(lib().littlebit_linear_forward_noalloc(ctypes.byref(L.c), x.data_ptr(), T, y.data_ptr(),
                                                   y_dtype, _stream(stream)),
