@@ -1381,15 +1381,17 @@ static cudaError_t set_smem_attributes() {
     return e;
 }
 
-// SM count of the current device (cached per device).
+// SM count of the current device (cached per device); 0 when it cannot be
+// read, which the cooperative launch turns into an error (its grid must be
+// exactly one CTA per SM, never a guess).
 static int device_sms() {
     static int sms[64];
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
     if (sms[dev] == 0) {
         int n = 0;
         if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
-            return 148;
+            return 0;
         sms[dev] = n;
     }
     return sms[dev];
@@ -1480,8 +1482,10 @@ cudaError_t launch_fused(const CUtensorMap &xmap, const CUtensorMap &bvmap,
     void *args[] = {const_cast<CUtensorMap *>(&xmap), const_cast<CUtensorMap *>(&bvmap),
                     const_cast<CUtensorMap *>(&zmap), const_cast<CUtensorMap *>(&bumap),
                     const_cast<PrefillParams *>(&P), const_cast<FusedPlan *>(&F)};
-    return cudaLaunchCooperativeKernel((const void *)k_fused, dim3(device_sms()), dim3(kThreads),
-                                       args, kTilesSmem, s);
+    const int sms = device_sms();
+    if (sms <= 0) return cudaErrorInvalidDevice;
+    return cudaLaunchCooperativeKernel((const void *)k_fused, dim3(sms), dim3(kThreads), args,
+                                       kTilesSmem, s);
 }
 
 // Stage-1 and stage-2 tilings of the persistent phases.
