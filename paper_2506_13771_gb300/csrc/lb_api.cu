@@ -435,6 +435,7 @@ lb_status littlebit_stack_prepare(const lb_linear *lin, int32_t n_layers, int32_
         return LB_ERR_WORKSPACE;
     int sms = 0;
     if ((st = num_sms(&sms)) != LB_OK) return st;
+    if ((sms = lb::stack_grid_ctas(lin, shape, sms)) <= 0) return LB_ERR_UNSUPPORTED;
     const cudaError_t e = lb::launch_stack_prepare(
         lin, n_layers, shape, sms, stack_fingerprint(lin, n_layers, head_dim, sms),
         static_cast<unsigned *>(ws), static_cast<char *>(ws) + kWsHeader, (cudaStream_t)stream);
@@ -455,6 +456,7 @@ lb_status littlebit_stack_forward(const lb_linear *lin, int32_t n_layers, int32_
         return LB_ERR_WORKSPACE;
     int sms = 0;
     if ((st = num_sms(&sms)) != LB_OK) return st;
+    if ((sms = lb::stack_grid_ctas(lin, shape, sms)) <= 0) return LB_ERR_UNSUPPORTED;
     if (!lb::stack_supported(lin, shape, sms)) return LB_ERR_UNSUPPORTED;
     return from_cuda(lb::launch_stack(lin, n_layers, shape,
                                       stack_fingerprint(lin, n_layers, head_dim, sms), x0, out,

@@ -7,10 +7,11 @@
 //     slice of input words, all columns) and U rows (its slice of output
 //     rows, all words); U lands while stage 1 runs;
 //   * stage 1: nibble tables of the CTA's g . x, then 32 columns per warp
-//     over the slice, each partial t added to a 64-bit exchange word whose
-//     low 8 bits count contributions ((round(t 2^24) << 8) + 1);
-//   * stage 2: every thread waits for the four words of one l . t table and
-//     builds it; then 32 rows per warp over all words of a path;
+//     over the slice, each partial t added to the exchange pair of its
+//     element (an exact two-word fixed-point sum whose low bits count the
+//     contributions, see send_fix2);
+//   * stage 2: every thread waits for the four elements of one l . t table
+//     and builds it; then 32 rows per warp over all words of a path;
 //   * the exchange words are double-buffered by a launch epoch kept in the
 //     workspace header: while a launch uses one buffer, every CTA clears its
 //     stripe of the other (the previous launch's), so no launch needs a
@@ -42,7 +43,7 @@ struct DecodeParams {
     void *y;
     int y_fp32;
     unsigned *ws_words;
-    unsigned long long *xw;  // exchange words: two buffers of N1 (paths concatenated)
+    unsigned long long *xw;  // exchange pairs: two buffers of N1 (paths concatenated)
     int N1, off1;
     float fix_limit;         // |partial| bound that keeps the fixed-point sum in range
     DecodeLayout o;
@@ -69,8 +70,9 @@ __global__ void __launch_bounds__(kDT, 1) k_decode(const __grid_constant__ Decod
     // epoch moves on only after every CTA has read it (block 0 bumps it once
     // its exchange completed, which needs every CTA's contributions)
     const unsigned epoch = ld_relaxed_gpu(P.ws_words + kEpochWord);
-    unsigned long long *xw = P.xw + (size_t)(epoch & 1u) * P.N1;
-    unsigned long long *xold = P.xw + (size_t)((epoch + 1u) & 1u) * P.N1;
+    const int nwords = (int)fix2_words(P.N1);  // one buffer
+    unsigned long long *xw = P.xw + (size_t)(epoch & 1u) * nwords;
+    unsigned long long *xold = P.xw + (size_t)((epoch + 1u) & 1u) * nwords;
     const LinDesc &L = P.L;
     const DecodeLayout &o = P.o;
     const int N = gridDim.x, c = blockIdx.x, tid = threadIdx.x;
@@ -158,16 +160,16 @@ __global__ void __launch_bounds__(kDT, 1) k_decode(const __grid_constant__ Decod
             }
             if (w < nw) acc0 += lut_word(Vw[w * r], copy, tb + w * 1024);
             if (col < r)
-                red_add_u64(xw + (p ? P.off1 : 0) + col, enc_fix(acc0 + acc1, P.fix_limit, err));
+                send_fix2(fix2_at(xw, (p ? P.off1 : 0) + col), acc0 + acc1, P.fix_limit, err);
         }
     }
     // the previous launch's words: this CTA's stripe back to zero
     {
-        const int a = (int)((long long)c * P.N1 / N), b = (int)((long long)(c + 1) * P.N1 / N);
+        const int a = (int)((long long)c * nwords / N), b = (int)((long long)(c + 1) * nwords / N);
         for (int i = a + tid; i < b; i += kDT) xold[i] = 0ull;
     }
 
-    // ---- stage 2 tables: thread i waits for the words of table i (l . t)
+    // ---- stage 2 tables: thread i waits for the elements of table i (l . t)
     const int nt0 = 8 * ((L.r[0] + 31) >> 5), ntab = nt0 + (np > 1 ? 8 * ((L.r[1] + 31) >> 5) : 0);
     int pok = ok ? 1 : 0;
     for (int idx = tid; idx < ntab && pok; idx += kDT) {
@@ -176,14 +178,11 @@ __global__ void __launch_bounds__(kDT, 1) k_decode(const __grid_constant__ Decod
         float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
         if (4 * n < r) {
             const uint2 lw = __ldg(reinterpret_cast<const uint2 *>((p ? L.l[1] : L.l[0]) + 4 * n));
-            const unsigned long long *wd = xw + (p ? P.off1 : 0) + 4 * n;
-            unsigned long long a0 = 0, a1 = 0, a2 = 0, a3 = 0, t0 = 0;
+            const unsigned long long *wd = fix2_at(xw, (p ? P.off1 : 0) + 4 * n);
+            unsigned long long a[8], t0 = 0;
             for (int spin = 0;; ++spin) {
-                ld_relaxed_v2_u64(wd, a0, a1);
-                ld_relaxed_v2_u64(wd + 2, a2, a3);
-                if (counted(a0, n_ctas) && counted(a1, n_ctas) && counted(a2, n_ctas) &&
-                    counted(a3, n_ctas))
-                    break;
+                ld_fix2x4(wd, a);
+                if (counted2x4(a, n_ctas)) break;
                 if ((spin & 15) == 15) {
                     if (ld_relaxed_gpu(err) != 0u) {
                         pok = 0;
@@ -198,10 +197,10 @@ __global__ void __launch_bounds__(kDT, 1) k_decode(const __grid_constant__ Decod
                     }
                 }
             }
-            v = make_float4(dec_fix(a0) * half_bits_to_float((uint16_t)(lw.x & 0xffffu)),
-                            dec_fix(a1) * half_bits_to_float((uint16_t)(lw.x >> 16)),
-                            dec_fix(a2) * half_bits_to_float((uint16_t)(lw.y & 0xffffu)),
-                            dec_fix(a3) * half_bits_to_float((uint16_t)(lw.y >> 16)));
+            v = make_float4(dec_fix2(a[0], a[1]) * half_bits_to_float((uint16_t)(lw.x & 0xffffu)),
+                            dec_fix2(a[2], a[3]) * half_bits_to_float((uint16_t)(lw.x >> 16)),
+                            dec_fix2(a[4], a[5]) * half_bits_to_float((uint16_t)(lw.y & 0xffffu)),
+                            dec_fix2(a[6], a[7]) * half_bits_to_float((uint16_t)(lw.y >> 16)));
         }
         store_table(g_smem + o.t2 + idx * 128, v, lane);
     }
@@ -318,7 +317,8 @@ bool decode_supported(const lb_linear &L, int num_sms) {
 }
 
 size_t decode_ws_bytes(const lb_linear &L) {
-    return ((size_t)2 * rsum_of(L) * sizeof(unsigned long long) + 255) & ~(size_t)255;
+    // two buffers of rsum exchange elements
+    return (2 * fix2_words(rsum_of(L)) * sizeof(unsigned long long) + 255) & ~(size_t)255;
 }
 
 cudaError_t launch_decode(const lb_linear &L, const void *x, int x_fp32, void *y, int y_fp32,
@@ -336,7 +336,7 @@ cudaError_t launch_decode(const lb_linear &L, const void *x, int x_fp32, void *y
     P.xw = static_cast<unsigned long long *>(xw);
     P.N1 = rsum_of(L);
     P.off1 = L.path[0].r;
-    P.fix_limit = 2147483648.f / (float)num_sms;
+    P.fix_limit = fix2_limit(num_sms);
     P.o = layout_of(L, num_sms);
     if (P.o.bytes > max_smem) return cudaErrorCooperativeLaunchTooLarge;
     void *args[] = {&P};

@@ -69,6 +69,10 @@ cudaError_t launch_stack_prepare(const lb_linear *lin, int n_layers, const Stack
 // (ranks multiples of 8, head_dim multiple of 32, d_kv multiple of 8, the
 // shared-memory plan fits).
 bool stack_supported(const lb_linear *lin, const StackShape &shape, int num_sms);
+// The grid of the one-launch stack kernel on this GPU: a whole number of
+// co-resident thread-block clusters, at most num_sms CTAs (0: cannot launch).
+// Programs, fingerprints and launches all use this count.
+int stack_grid_ctas(const lb_linear *lin, const StackShape &shape, int num_sms);
 // One persistent launch; leaves counters and accumulators zeroed.
 cudaError_t launch_stack(const lb_linear *lin, int n_layers, const StackShape &shape,
                          unsigned long long plan, const uint16_t *x0, float *out, float *q_out,

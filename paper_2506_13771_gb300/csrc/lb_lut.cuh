@@ -4,8 +4,8 @@
 // A +-1 sum over 32 values is 8 lookups in 4-bit tables: table n of a
 // vector v holds, for e = 0..15, sum_{k<4} (bit k of e ? -v : +v)[4n + k],
 // stored twice (entries e and 16 + e) so the two half-warps read disjoint
-// banks.  An exchange word is a 64-bit fixed-point sum whose low 8 bits count
-// its contributions.
+// banks.  An exchanged element is a pair of 64-bit fixed-point words whose
+// low 8 bits count its contributions (see send_fix2).
 #pragma once
 
 #include "lb_common.cuh"
@@ -15,8 +15,6 @@ namespace {
 
 extern __shared__ __align__(1024) unsigned char g_smem[];
 
-constexpr float kFix = 16777216.f;            // 2^24
-constexpr float kFixInv = 1.f / 16777216.f;
 
 // ---------------------------------------------------------------- PTX helpers
 
@@ -50,6 +48,59 @@ __device__ __forceinline__ bool mbar_try_wait(unsigned long long *bar, unsigned 
         : "r"(saddr(bar)), "r"(parity)
         : "memory");
     return ok != 0;
+}
+
+// ---------------------------------------------------------------- clusters
+
+__device__ __forceinline__ unsigned cluster_rank() {
+    unsigned r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// The shared::cluster address of byte offset `local` (a shared::cta address)
+// in the CTA of rank `rank` of this cluster.
+__device__ __forceinline__ uint32_t mapa(uint32_t local, unsigned rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
+    return r;
+}
+
+// 4 bytes into another CTA's shared memory, completing 4 bytes of the
+// transaction count of that CTA's mbarrier (both shared::cluster addresses).
+__device__ __forceinline__ void st_async_f32(uint32_t raddr, float v, uint32_t rbar) {
+    asm volatile(
+        "st.async.shared::cluster.mbarrier::complete_tx::bytes.b32 [%0], %1, [%2];" ::"r"(raddr),
+        "r"(__float_as_uint(v)), "r"(rbar)
+        : "memory");
+}
+
+// Arrival of this thread on bar with `bytes` more transaction bytes expected.
+__device__ __forceinline__ void mbar_arrive_expect_tx(unsigned long long *bar, unsigned bytes) {
+    asm volatile(
+        "{\n\t.reg .b64 st;\n\tmbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1;\n\t}" ::"r"(
+            saddr(bar)),
+        "r"(bytes)
+        : "memory");
+}
+
+// try_wait with cluster-scope acquire: data written into this CTA's shared
+// memory by other CTAs of the cluster (st.async) is visible once it succeeds.
+__device__ __forceinline__ bool mbar_try_wait_cluster(unsigned long long *bar, unsigned parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], "
+        "%2;\n\tselp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(saddr(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Cluster-wide barrier of every thread (not .aligned: threads may arrive
+// from divergent paths).
+__device__ __forceinline__ void cluster_sync_all() {
+    asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
 }
 
 // 1D TMA bulk copy global -> this CTA's shared memory, completing on bar.
@@ -110,21 +161,100 @@ __device__ __forceinline__ float lut_word(uint32_t word, uint32_t copy, uint32_t
     return lut8(lo, hi, base);
 }
 
-// One contribution to an exchange word: (round(v * 2^24) << 8) + 1.
-__device__ __forceinline__ unsigned long long enc_fix(float v, float limit, unsigned *err) {
+// ---------------------------------------------------------------- exchange
+//
+// An element of an exchange (one value of the rank-r t all-reduced across
+// the CTAs) is a pair of 64-bit words (hi, lo) that holds the EXACT sum of
+// its fp32 contributions in fixed point with resolution 2^-64.  Elements are
+// laid out in blocks of 32: the hi words of elements 32b .. 32b + 31, then
+// their lo words (fix2_at), so a warp's 32 consecutive elements take two
+// cache lines of hi words and two of lo words.  A
+// contribution v is split as v * 2^64 = H * 2^47 + L with H = trunc(v 2^17)
+// and |L| < 2^47, and adds (H << 8) + 1 to hi and (L << 8) + 1 to lo with
+// one red.add each: the low 8 bits of both words count the contributions
+// (at most 255), the high 56 bits carry the integer sums.  Every fp32 v with
+// 2^-41 <= |v| < 2^34 / n (n contributions) is represented exactly, smaller
+// ones to within 2^-65, so the sum is exact whatever the order of arrival
+// and, decoded with one correct rounding, scales exactly with the inputs:
+// Prop. 1 is linear, and so is this exchange over 66 binades.  A
+// contribution outside the range records LB_ERR_RANGE and is sent as zero.
+
+// 2^34 / n: the largest |contribution| that keeps the sum of n of them
+// below 2^51 in H (the range dec_fix2 rounds correctly).
+__host__ __device__ constexpr float fix2_limit(int n) { return 17179869184.f / (float)n; }
+
+// The hi word of element e of an exchange buffer at x (its lo word is 32
+// words further).  Buffers hold a whole number of 32-element blocks.
+__host__ __device__ __forceinline__ size_t fix2_words(size_t elements) {
+    return 2 * ((elements + 31) & ~(size_t)31);
+}
+__device__ __forceinline__ unsigned long long *fix2_at(unsigned long long *x, int e) {
+    return x + 64 * (e >> 5) + (e & 31);
+}
+__device__ __forceinline__ const unsigned long long *fix2_at(const unsigned long long *x, int e) {
+    return x + 64 * (e >> 5) + (e & 31);
+}
+
+// One contribution v to the element whose hi word is w.
+__device__ __forceinline__ void send_fix2(unsigned long long *w, float v, float limit,
+                                          unsigned *err) {
     if (!(fabsf(v) < limit)) {
         atomicCAS(err, 0u, static_cast<unsigned>(LB_ERR_RANGE));
         v = 0.f;
     }
-    const long long f = __float2ll_rn(v * kFix);
-    return (static_cast<unsigned long long>(f) << 8) + 1ull;
+    const float a = v * 0x1p17f;  // exact
+    const float t = truncf(a);
+    const long long H = __float2ll_rz(t);
+    const long long L = __float2ll_rn((a - t) * 0x1p47f);  // a - t is exact, |.| < 1
+    red_add_u64(w, (static_cast<unsigned long long>(H) << 8) + 1ull);
+    red_add_u64(w + 32, (static_cast<unsigned long long>(L) << 8) + 1ull);
 }
 
-__device__ __forceinline__ float dec_fix(unsigned long long w) {
-    return __ll2float_rn((long long)w >> 8) * kFixInv;
+// A contribution of zero that only counts (a CTA with nothing to add).
+__device__ __forceinline__ void send_count2(unsigned long long *w) {
+    red_add_u64(w, 1ull);
+    red_add_u64(w + 32, 1ull);
 }
-__device__ __forceinline__ bool counted(unsigned long long w, unsigned n_ctas) {
-    return (unsigned)(w & 0xffull) == n_ctas;
+
+// The hi and lo words of one element (hi word at w), relaxed.
+__device__ __forceinline__ void ld_fix2(const unsigned long long *w, unsigned long long &hi,
+                                        unsigned long long &lo) {
+    hi = ld_relaxed_u64(w);
+    lo = ld_relaxed_u64(w + 32);
+}
+
+__device__ __forceinline__ bool counted2(unsigned long long hi, unsigned long long lo,
+                                         unsigned n) {
+    return (unsigned)(hi & 0xffull) == n && (unsigned)(lo & 0xffull) == n;
+}
+
+// Elements e .. e + 3 (e a multiple of 4; hi word of e at p), relaxed:
+// a[2k], a[2k + 1] = hi, lo of element e + k.
+__device__ __forceinline__ void ld_fix2x4(const unsigned long long *p, unsigned long long (&a)[8]) {
+    ld_relaxed_v2_u64(p, a[0], a[2]);
+    ld_relaxed_v2_u64(p + 2, a[4], a[6]);
+    ld_relaxed_v2_u64(p + 32, a[1], a[3]);
+    ld_relaxed_v2_u64(p + 34, a[5], a[7]);
+}
+
+__device__ __forceinline__ bool counted2x4(const unsigned long long (&a)[8], unsigned n) {
+    return counted2(a[0], a[1], n) && counted2(a[2], a[3], n) && counted2(a[4], a[5], n) &&
+           counted2(a[6], a[7], n);
+}
+
+// The sum held by a complete pair, (H 2^47 + L) 2^-64, rounded to nearest
+// fp32 (ties to even): exactly while it fits 64 bits (|H| < 2^15); beyond
+// that from floor(sum / 2^36) with a sticky bit for the dropped remainder
+// (the quotient then has more than 26 bits, so the sticky bit sits below the
+// rounding position and cannot move a tie).  |H| < 2^51 (fix2_limit) keeps
+// 2 floor(sum / 2^36) + 1 inside 64 bits.
+__device__ __forceinline__ float dec_fix2(unsigned long long hi, unsigned long long lo) {
+    const long long H = static_cast<long long>(hi) >> 8;
+    const long long L = static_cast<long long>(lo) >> 8;
+    if (H > -32768ll && H < 32768ll) return __ll2float_rn(H * 140737488355328ll + L) * 0x1p-64f;
+    const long long q = H * 2048ll + (L >> 36);
+    const long long sticky = (L & 68719476735ll) != 0 ? 1 : 0;
+    return __ll2float_rn(2 * q + sticky) * 0x1p-29f;
 }
 
 // Stores table n of a unit at T from its four values (see run_tables).

@@ -63,7 +63,7 @@ struct MultiParams {
     void *y;        // [M][d_out], bf16 or fp32
     int y_fp32;
     unsigned *ws_words;
-    unsigned long long *xw;  // exchange words: two buffers of M * N1
+    unsigned long long *xw;  // exchange pairs: two buffers of M * N1 + 1
     float fix_limit;
     MultiLayout o;
     MultiPtrs p[kMaxMultiLinears];
@@ -104,10 +104,9 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
     unsigned *err = P.ws_words + kErrWord;
     if (ld_relaxed_gpu(err) != 0u) return;
     const unsigned epoch = ld_relaxed_gpu(P.ws_words + kEpochWord);
-    // a buffer holds M * N1 words of t, then the sum-of-squares word and one
-    // spare word (N1 is a sum of multiples of 8, so the stride keeps the
-    // second buffer 16-byte aligned for the paired 64-bit loads)
-    const size_t words = (size_t)P.M * P.N1, stride = words + 2;
+    // a buffer holds M * N1 exchange elements of t, then the sum-of-squares
+    // element (element `words`)
+    const size_t words = (size_t)P.M * P.N1, stride = fix2_words(words + 1);
     unsigned long long *xw = P.xw + (size_t)(epoch & 1u) * stride;
     unsigned long long *xold = P.xw + (size_t)((epoch + 1u) & 1u) * stride;
     const bool res = P.x_fp32 == 3;
@@ -208,27 +207,25 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
         // word then holds outlier-sized activations too), counted like linear
         // 0's words
         if (res && tid == 0)
-            red_add_u64(xw + words, enc_fix(s_ss / (float)P.d_in, P.fix_limit, err));
+            send_fix2(fix2_at(xw, (int)words), s_ss / (float)P.d_in, P.fix_limit, err);
         const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
         bool ok = true;
         // the exchange words a thread polls for stage 2 (its table tid; ntab <=
         // kCT whenever the ranks sum to at most 1920), loaded while the row
         // sums of the linear before run, so that the L2 round trip overlaps them
-        unsigned long long pre[4] = {0ull, 0ull, 0ull, 0ull};
+        unsigned long long pre[8] = {0ull, 0ull, 0ull, 0ull, 0ull, 0ull, 0ull, 0ull};
         auto prefetch = [&](int mm) {
             if (mm < 0 || mm >= P.M || tid >= ntab) return;
             const int p = tid >= nt0 ? 1 : 0, n = tid - (p ? nt0 : 0);
             if (4 * n >= P.r[p]) return;
-            const unsigned long long *wd = xw + (size_t)mm * P.N1 + (p ? P.off1 : 0) + 4 * n;
-            ld_relaxed_v2_u64(wd, pre[0], pre[1]);
-            ld_relaxed_v2_u64(wd + 2, pre[2], pre[3]);
+            ld_fix2x4(fix2_at(xw, mm * P.N1 + (p ? P.off1 : 0) + 4 * n), pre);
         };
         for (int it = 0; it < P.M + kAhead && ok; ++it) {
             if (it == kAhead) prefetch(0);
             // ---------------- stage 1 of linear it
             if (it == 0 && nw == 0) {
                 // a CTA without input words still counts itself into linear 0's words
-                for (int i = tid; i < P.N1; i += kCT) red_add_u64(xw + i, 1ull);
+                for (int i = tid; i < P.N1; i += kCT) send_count2(fix2_at(xw, i));
             }
             if (it < P.M && nw > 0) {
                 const int m = it;
@@ -252,7 +249,7 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
                     store_table(g_smem + o.t1 + idx * 128, v, lane);
                 }
                 csync_m();
-                unsigned long long *xm = xw + (size_t)m * P.N1;
+                const int xm = m * P.N1;  // the linear's first element
                 for (int u = warp; u < cbs; u += kCW) {
                     const int p = u >= R0 ? 1 : 0, cb = u - (p ? R0 : 0);
                     const int r = P.r[p];
@@ -268,14 +265,15 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
                     }
                     if (w < nw) acc0 += lut_word(Vw[w * r], copy, tb + w * 1024);
                     if (col < r)
-                        red_add_u64(xm + (p ? P.off1 : 0) + col, enc_fix(acc0 + acc1, P.fix_limit, err));
+                        send_fix2(fix2_at(xw, xm + (p ? P.off1 : 0) + col), acc0 + acc1,
+                                  P.fix_limit, err);
                 }
                 csync_m();  // t1 is rebuilt by the next linear
             }
             // ---------------- stage 2 of linear it - kAhead
             const int mm = it - kAhead;
             if (mm < 0) continue;
-            const unsigned long long *xm = xw + (size_t)mm * P.N1;
+            const int xm = mm * P.N1;  // the linear's first element
             unsigned char *b = slot(mm);
             // the slot's U rows, h and l (thread 0 waits, the rest observe the phase)
             bool u_ok = true;
@@ -288,10 +286,10 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
             int pok = 1;
             if (res && mm == 0 && tid == 0) {
                 // the sum of squares of the whole input (all CTAs counted)
-                unsigned long long wv = 0, t0 = 0;
+                unsigned long long wh = 0, wl = 0, t0 = 0;
                 for (int spin = 0;; ++spin) {
-                    wv = ld_relaxed_u64(xw + words);
-                    if (counted(wv, n_first)) break;
+                    ld_fix2(fix2_at(xw, (int)words), wh, wl);
+                    if (counted2(wh, wl, n_first)) break;
                     if ((spin & 15) == 15) {
                         if (ld_relaxed_gpu(err) != 0u) {
                             pok = 0;
@@ -306,7 +304,7 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
                         }
                     }
                 }
-                if (pok) s_inv = rsqrtf(dec_fix(wv));
+                if (pok) s_inv = rsqrtf(dec_fix2(wh, wl));
             }
             for (int idx = tid; idx < ntab && pok; idx += kCT) {
                 const int p = idx >= nt0 ? 1 : 0, n = idx - (p ? nt0 : 0);
@@ -314,22 +312,17 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
                 float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
                 if (4 * n < r) {
                     const uint2 lw = *reinterpret_cast<const uint2 *>(b + o.l[p] + 8 * n);
-                    const unsigned long long *wd = xm + (p ? P.off1 : 0) + 4 * n;
-                    unsigned long long a0 = 0, a1 = 0, a2 = 0, a3 = 0, t0 = 0;
+                    const unsigned long long *wd = fix2_at(xw, xm + (p ? P.off1 : 0) + 4 * n);
+                    unsigned long long a[8], t0 = 0;
                     for (int spin = 0;; ++spin) {
                         if (spin == 0 && idx == tid) {
-                            a0 = pre[0];
-                            a1 = pre[1];
-                            a2 = pre[2];
-                            a3 = pre[3];
+#pragma unroll
+                            for (int k = 0; k < 8; ++k) a[k] = pre[k];
                         } else {
-                            ld_relaxed_v2_u64(wd, a0, a1);
-                            ld_relaxed_v2_u64(wd + 2, a2, a3);
+                            ld_fix2x4(wd, a);
                         }
                         const unsigned want = mm == 0 ? n_first : n_contrib;
-                        if (counted(a0, want) && counted(a1, want) && counted(a2, want) &&
-                            counted(a3, want))
-                            break;
+                        if (counted2x4(a, want)) break;
                         if ((spin & 15) == 15) {
                             if (ld_relaxed_gpu(err) != 0u) {
                                 pok = 0;
@@ -344,10 +337,10 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
                             }
                         }
                     }
-                    v = make_float4(dec_fix(a0) * half_bits_to_float((uint16_t)(lw.x & 0xffffu)),
-                                    dec_fix(a1) * half_bits_to_float((uint16_t)(lw.x >> 16)),
-                                    dec_fix(a2) * half_bits_to_float((uint16_t)(lw.y & 0xffffu)),
-                                    dec_fix(a3) * half_bits_to_float((uint16_t)(lw.y >> 16)));
+                    v = make_float4(dec_fix2(a[0], a[1]) * half_bits_to_float((uint16_t)(lw.x & 0xffffu)),
+                                    dec_fix2(a[2], a[3]) * half_bits_to_float((uint16_t)(lw.x >> 16)),
+                                    dec_fix2(a[4], a[5]) * half_bits_to_float((uint16_t)(lw.y & 0xffffu)),
+                                    dec_fix2(a[6], a[7]) * half_bits_to_float((uint16_t)(lw.y >> 16)));
                 }
                 store_table(g_smem + o.t2 + idx * 128, v, lane);
             }
@@ -489,8 +482,8 @@ bool multi_supported(const lb_linear *L, int M, int num_sms) {
 }
 
 size_t multi_ws_bytes(const lb_linear &L, int M) {
-    // two buffers of M * rsum words of t, a sum-of-squares word and a spare
-    return ((size_t)2 * ((size_t)M * rsum(L) + 2) * sizeof(unsigned long long) + 255) &
+    // two buffers of M * rsum exchange elements of t and a sum-of-squares element
+    return (2 * fix2_words((size_t)M * rsum(L) + 1) * sizeof(unsigned long long) + 255) &
            ~(size_t)255;
 }
 
@@ -518,7 +511,7 @@ cudaError_t launch_decode_multi(const lb_linear *L, int M, const void *x, int x_
     P.y_fp32 = y_fp32;
     P.ws_words = ws_words;
     P.xw = static_cast<unsigned long long *>(xw);
-    P.fix_limit = 2147483648.f / (float)num_sms;
+    P.fix_limit = fix2_limit(num_sms);
     P.o = layout_of(A, num_sms);
     if (P.o.bytes > max_smem) return cudaErrorCooperativeLaunchTooLarge;
     for (int m = 0; m < M; ++m)

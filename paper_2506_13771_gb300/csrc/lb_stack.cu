@@ -29,17 +29,20 @@
 //    the stage-1 tables of those rows), 32 columns x the slice for stage 1.
 //    The shapes are those of every layer, so the program is the same for all
 //    of them; the device code is a handful of generic loops;
-//  * the all-reduce of t accumulates fixed-point values in 64-bit words whose
-//    low 8 bits count contributions: each CTA adds (round(v * 2^24) << 8) + 1
-//    with one red.add per element and readers poll the words they need until
-//    the count reaches the CTA count -- no fence, no separate barrier, and an
-//    order-independent (bitwise reproducible) sum;
+//  * the all-reduce of t accumulates every element as an exact fixed-point
+//    sum in a pair of 64-bit words whose low 8 bits count contributions
+//    (send_fix2: two red.add per element and CTA) and readers poll the pairs
+//    they need until the count reaches the CTA count -- no fence, no
+//    separate barrier, an order-independent sum, exact for contributions
+//    from 2^-41 to 2^34 / n, so the exchange is equivariant under scaling of
+//    the inputs;
 //  * q and k (not read again at position 0) are computed after the CTA has
 //    sent its share of the next exchange, off the critical path.
 // Every wait is bounded (about one second); on a timeout the CTA records
 // LB_ERR_TIMEOUT, waits for its own bulk copies to land, and returns.
 #include <algorithm>
 #include <cstring>
+#include <mutex>
 #include <vector>
 
 #include "lb_common.cuh"
@@ -51,6 +54,14 @@ namespace lb {
 namespace {
 
 constexpr int kST = 512;        // threads per CTA
+#ifndef LB_STACK_CLUSTER
+#define LB_STACK_CLUSTER 2
+#endif
+// CTAs per thread-block cluster: the stage-1 partial sums of a cluster's
+// CTAs meet in distributed shared memory before one exchange contribution
+// per cluster goes out (1: no clusters, every CTA contributes)
+constexpr int kCluster = LB_STACK_CLUSTER;
+static_assert(kCluster >= 1 && kCluster <= 8, "portable cluster sizes");
 constexpr int kCW = 15;         // compute warps; warp 15 issues the bulk copies
 constexpr int kCT = kCW * 32;   // compute threads
 // ---------------------------------------------------------------- parameters
@@ -74,6 +85,10 @@ struct Offsets {
     // outputs (added into, zeroed once stored), the sum-of-squares
     // accumulator, the program
     int t2, t1, res0, res1, yq, yk, yv, ssacc, prog;
+    // cluster reduction of the stage-1 partials, per phase X = A..D: the
+    // receive slots of the units this CTA owns (kCluster x 32 floats each,
+    // one row per sending rank) and the index of their first mbarrier in ubar
+    int slot[4], ubar0[4], ubar, n_ubar;
 };
 
 // Steps of the per-CTA program (one per table build or unit loop).
@@ -92,7 +107,9 @@ enum StepId {
 //   poll-table  : tb, n_tab, n_vals, mode, e0, scale, ss_el, -  (e0, ss_el:
 //                 exchange word indices in the layer; ss_el < 0: none)
 //   stage-2 unit: U, R, nw, tb, h, out, nrows, -
-//   stage-1 unit: V, r, nw, tb, dst, ncols, -, -
+//   stage-1 unit: V, r, nw, tb, dst, ncols, own, slot  (own: the cluster rank
+//                 that sums the unit's partials and sends them; slot: the
+//                 unit's receive slot and mbarrier at that rank)
 //   row unit    : a header  n_pair, n_job, mode, nrows, res_in, res_out, -, -
 //                 then per pair two segments (first for lanes 0-15, second
 //                 for lanes 16-31)  U, R, nw, tb, h, -, -, -
@@ -127,7 +144,8 @@ struct Params {
     float *out, *q_out, *kv_out;
     unsigned *ws_words;
     unsigned long long plan;
-    unsigned long long *xacc;  // exchange words, n_layers * acc_layer
+    unsigned long long *xacc;  // exchange pairs, n_layers * acc_layer (2 words each)
+    unsigned n_t;              // contributions per t element: one per cluster
     int acc_layer, offA, offQ, offB, offC, offD, lenA, lenQ, lenB, lenC, lenD;
     float fix_limit;  // |contribution| bound that keeps the fixed-point sum in range
     Offsets o;
@@ -287,17 +305,81 @@ __device__ __noinline__ void run_s2(int prog, int s) {
     }
 }
 
-// Stage-1 units: t[col] partial over the CTA's input slice, added to the
-// exchange words (lane = column).  Every CTA has a unit for every column,
-// also when its slice is empty, so each element counts one contribution
-// per CTA.
-__device__ __noinline__ void run_s1(int prog, int s, unsigned long long *xbase, float limit,
-                                    unsigned *err) {
+__device__ __forceinline__ bool sticky(const unsigned *ws_words) {
+    return ld_relaxed_gpu(ws_words + kErrWord) != 0u;
+}
+
+__device__ __forceinline__ void record(unsigned *ws_words, lb_status st) {
+    atomicCAS(ws_words + kErrWord, 0u, static_cast<unsigned>(st));
+}
+
+// Stage-1 units: t[col] partial over the CTA's input slice (lane = column).
+// Every CTA has a unit for every column, also when its slice is empty (it
+// then contributes zeros).  Without clusters each partial goes straight into
+// the exchange pairs.  With clusters a unit belongs to one rank of the
+// cluster: the other ranks store their partials into its receive slot in
+// the owner's shared memory (st.async, completing on the slot's mbarrier),
+// and the owner adds them to its own in rank order and sends the sum -- one
+// contribution per cluster.  A warp runs the units it does not own first.
+// Returns false (this warp) when an owner's wait ran out.
+__device__ __noinline__ bool run_s1(int prog, int s, unsigned long long *xbase, float limit,
+                                    unsigned *err, int slot0, int ubar0, int ubar, unsigned par,
+                                    unsigned rank, unsigned *ws_words) {
     const Step &st = step_at(prog, s);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
-    const int u1 = st.first + st.wo[warp + 1];
-    int u = st.first + st.wo[warp];
+    const int u0 = st.first + st.wo[warp], u1 = st.first + st.wo[warp + 1];
+    auto bar_of = [&](int slot) {
+        return reinterpret_cast<unsigned long long *>(g_smem + ubar) + ubar0 + slot;
+    };
+    if (kCluster > 1 && lane == 0) {
+        // arm the mbarriers of this warp's own units for this use
+        for (int u = u0; u < u1; ++u) {
+            int4 a, b;
+            item_at(prog, u, a, b);
+            if ((unsigned)b.z == rank)
+                mbar_arrive_expect_tx(bar_of(b.w), (unsigned)((kCluster - 1) * 4 * b.y));
+        }
+    }
+    __syncwarp();
+    bool ok = true;
+    // one finished unit: its partial v of column `lane`
+    auto finish = [&](const int4 &b, float v) {
+        const int dst = b.x, ncols = b.y;
+        if (kCluster == 1) {
+            if (lane < ncols) send_fix2(fix2_at(xbase, dst + lane), v, limit, err);
+            return;
+        }
+        const unsigned own = (unsigned)b.z;
+        const int slot = b.w;
+        if (own != rank) {
+            if (lane < ncols) {
+                const uint32_t loc =
+                    saddr(g_smem + slot0 + (slot * kCluster + (int)rank) * 128 + 4 * lane);
+                st_async_f32(mapa(loc, own), v, mapa(saddr(bar_of(slot)), own));
+            }
+            return;
+        }
+        // owner: the other ranks' partials, then the sum in rank order
+        if (!ok) return;
+        unsigned long long *bar = bar_of(slot);
+        if (!mbar_try_wait_cluster(bar, par)) {
+            const unsigned long long t0 = globaltimer_ns();
+            while (!mbar_try_wait_cluster(bar, par)) {
+                if (sticky(ws_words) || globaltimer_ns() - t0 > kWaitLimitNs) {
+                    record(ws_words, LB_ERR_TIMEOUT);
+                    ok = false;
+                    return;
+                }
+            }
+        }
+        const float *rx = reinterpret_cast<const float *>(g_smem + slot0 + slot * kCluster * 128);
+        float sum = 0.f;
+#pragma unroll
+        for (int k = 0; k < kCluster; ++k) sum += (unsigned)k == rank ? v : rx[32 * k + lane];
+        if (lane < ncols) send_fix2(fix2_at(xbase, dst + lane), sum, limit, err);
+    };
+    int u = u0;
     // two units per pass; a unit whose input slice is empty (no words) reads
     // the first entries of its buffer and table, masked out, and sends zero
     for (; u + 2 <= u1; u += 2) {
@@ -315,8 +397,8 @@ __device__ __noinline__ void run_s1(int prog, int s, unsigned long long *xbase, 
             acc0 += w < a.z ? v0 : 0.f;
             acc1 += w < c.z ? v1 : 0.f;
         }
-        if (lane < b.y) red_add_u64(xbase + b.x + lane, enc_fix(acc0, limit, err));
-        if (lane < d.y) red_add_u64(xbase + d.x + lane, enc_fix(acc1, limit, err));
+        finish(b, acc0);
+        finish(d, acc1);
     }
     if (u < u1) {
         int4 a, b;
@@ -332,8 +414,9 @@ __device__ __noinline__ void run_s1(int prog, int s, unsigned long long *xbase, 
             acc1 += lut_word(w1, copy, tb + (w + 1) * 1024);
         }
         if (w < nw) acc0 += lut_word(Vw[w * r], copy, tb + w * 1024);
-        if (lane < ncols) red_add_u64(xbase + b.x + lane, enc_fix(acc0 + acc1, limit, err));
+        finish(b, acc0 + acc1);
     }
+    return ok;
 }
 
 // Barrier over the compute warps only (named barrier 1).
@@ -364,23 +447,15 @@ __device__ __forceinline__ void zero_stripe(unsigned long long *region, const in
     for (int i = z[0] + threadIdx.x; i < z[1]; i += kCT) region[i] = 0ull;
 }
 
-__device__ __forceinline__ bool sticky(const unsigned *ws_words) {
-    return ld_relaxed_gpu(ws_words + kErrWord) != 0u;
-}
-
-__device__ __forceinline__ void record(unsigned *ws_words, lb_status st) {
-    atomicCAS(ws_words + kErrWord, 0u, static_cast<unsigned>(st));
-}
-
 // Poll-table units: the stage-2 tables of a phase built straight from the
-// exchange words.  Lane n waits until the words e0 + 4n .. +3 (those below
-// n_vals) -- and the word ss_el, for a TAB_MUL unit that has one -- count
-// n_ctas contributions, decodes them and builds table n of v_i = t_i * l_i
-// (* inv with TAB_MUL, inv = rsqrt(ss * inv_d) of word ss_el, or the
+// exchange pairs.  Lane n waits until the elements e0 + 4n .. +3 (those below
+// n_vals) -- and the element ss_el, for a TAB_MUL unit that has one -- count
+// n_t contributions (n_ss for ss_el), decodes them and builds table n of v_i = t_i * l_i
+// (* inv with TAB_MUL, inv = rsqrt(mean square) of element ss_el, or the
 // argument when the unit has no ss_el).  Bounded; returns false (to every
 // compute thread) on failure.
 __device__ __noinline__ bool run_poll_tables(int prog, int s, const unsigned long long *xbase,
-                                             unsigned n_ctas, float inv, float inv_d,
+                                             unsigned n_t, unsigned n_ss, float inv,
                                              unsigned *ws_words) {
     const Step &st = step_at(prog, s);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -395,23 +470,24 @@ __device__ __noinline__ bool run_poll_tables(int prog, int s, const unsigned lon
         // and once it sees its word complete the whole unit usually is
         if (lane == 0 && a.z > 0) {
             const unsigned long long t0 = globaltimer_ns();
-            const unsigned long long *gw = xbase + b.x + (min(a.z, 4 * a.y) - 1);
-            for (int spin = 0; !counted(ld_relaxed_u64(gw), n_ctas); ++spin)
+            const unsigned long long *gw = fix2_at(xbase, b.x + (min(a.z, 4 * a.y) - 1));
+            unsigned long long gh, gl;
+            for (int spin = 0;; ++spin) {
+                ld_fix2(gw, gh, gl);
+                if (counted2(gh, gl, n_t)) break;
                 if ((spin & 15) == 15 && globaltimer_ns() - t0 > kWaitLimitNs) break;
+            }
         }
         __syncwarp();
         if (lane >= a.y) continue;
         const bool have = a.z - 4 * lane > 0;
         const bool need_ss = have && (a.w & TAB_MUL) && b.z >= 0;
-        const unsigned long long *w = xbase + b.x + 4 * lane;
-        unsigned long long v0 = 0, v1 = 0, v2 = 0, v3 = 0, vs = 0, t0 = 0;
+        const unsigned long long *w = fix2_at(xbase, b.x + 4 * lane);
+        unsigned long long v[8], sh = 0, sl = 0, t0 = 0;
         for (int spin = 0; have; ++spin) {
-            ld_relaxed_v2_u64(w, v0, v1);
-            ld_relaxed_v2_u64(w + 2, v2, v3);
-            if (need_ss) vs = ld_relaxed_u64(xbase + b.z);
-            if (counted(v0, n_ctas) && counted(v1, n_ctas) && counted(v2, n_ctas) &&
-                counted(v3, n_ctas) && (!need_ss || counted(vs, n_ctas)))
-                break;
+            ld_fix2x4(w, v);
+            if (need_ss) ld_fix2(fix2_at(xbase, b.z), sh, sl);
+            if (counted2x4(v, n_t) && (!need_ss || counted2(sh, sl, n_ss))) break;
             if ((spin & 15) == 15) {
                 if (sticky(ws_words)) {
                     ok = 0;
@@ -430,11 +506,11 @@ __device__ __noinline__ bool run_poll_tables(int prog, int s, const unsigned lon
         float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
         if (have) {
             const uint2 hb = *reinterpret_cast<const uint2 *>(g_smem + b.y + 8 * lane);
-            const float m = (a.w & TAB_MUL) ? (need_ss ? rsqrtf(dec_fix(vs) * inv_d) : inv) : 1.f;
-            x.x = dec_fix(v0) * half_bits_to_float((uint16_t)(hb.x & 0xffffu)) * m;
-            x.y = dec_fix(v1) * half_bits_to_float((uint16_t)(hb.x >> 16)) * m;
-            x.z = dec_fix(v2) * half_bits_to_float((uint16_t)(hb.y & 0xffffu)) * m;
-            x.w = dec_fix(v3) * half_bits_to_float((uint16_t)(hb.y >> 16)) * m;
+            const float m = (a.w & TAB_MUL) ? (need_ss ? rsqrtf(dec_fix2(sh, sl)) : inv) : 1.f;
+            x.x = dec_fix2(v[0], v[1]) * half_bits_to_float((uint16_t)(hb.x & 0xffffu)) * m;
+            x.y = dec_fix2(v[2], v[3]) * half_bits_to_float((uint16_t)(hb.x >> 16)) * m;
+            x.z = dec_fix2(v[4], v[5]) * half_bits_to_float((uint16_t)(hb.y & 0xffffu)) * m;
+            x.w = dec_fix2(v[6], v[7]) * half_bits_to_float((uint16_t)(hb.y >> 16)) * m;
         }
         store_table(g_smem + a.x + lane * 128, x, lane);
     }
@@ -638,7 +714,8 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         return;
     }
     const int N = gridDim.x, c = blockIdx.x;
-    const unsigned n_ctas = (unsigned)N;
+    const unsigned n_ctas = (unsigned)N, n_t = P.n_t;
+    const unsigned rank = kCluster > 1 ? cluster_rank() : 0u;
     Part s;
     {
         const int Wd = P.d >> 5, Wf = P.dff >> 5, Ukv = P.dkv >> 3;
@@ -655,20 +732,26 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
             mbar_init(full + b, 1);
             mbar_init(empty + b, 1);
         }
+        for (int b = 0; b < P.o.n_ubar; ++b)
+            mbar_init(reinterpret_cast<unsigned long long *>(g_smem + P.o.ubar) + b, 1);
         fence_barrier_init();
     }
     if (threadIdx.x < XR_N) {
         const int t = threadIdx.x;
         const int n = t == XR_A ? P.lenA : t == XR_Q ? P.lenQ : t == XR_B ? P.lenB
                     : t == XR_C ? P.lenC : P.lenD;
-        s_zs[threadIdx.x][0] = (int)((long long)c * n / N);
-        s_zs[threadIdx.x][1] = (int)((long long)(c + 1) * n / N);
+        // in words: the region's whole 32-element blocks
+        const long long w = (long long)fix2_words(n);
+        s_zs[threadIdx.x][0] = (int)(c * w / N);
+        s_zs[threadIdx.x][1] = (int)((c + 1) * w / N);
     }
     __syncthreads();
+    // every CTA of the cluster has initialised its mbarriers before any
+    // other may complete a transaction on them
+    if (kCluster > 1) cluster_sync_all();
     if (threadIdx.x >= kCT) {
         if (threadIdx.x == kCT) producer(Loader{&P, s, full}, empty, P.ws_words);
-        return;
-    }
+    } else {
 
     // ------------------------------------------------------------ compute warps
     const Offsets &o = P.o;
@@ -696,47 +779,57 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
     const int ssA = nr[LV], ssC = nr[LG] + nr[LU];
     const bool lead = threadIdx.x == 0;
     const float lim = P.fix_limit, inv_d = 1.f / (float)P.d;
+    // the first word of region off (a multiple of 32 elements) in the layer at x
+    auto at = [](unsigned long long *x, int off) { return x + 2 * off; };
     auto release = [&](int b) {
         csync();
         if (lead) mbar_arrive(empty + b);
     };
+    // this CTA's share of the mean square (sum / d), so that outlier-sized
+    // activations stay in range
     auto send_ss = [&](unsigned long long *p) {
         if (lead) {
-            red_add_u64(p, enc_fix(ssacc[0], lim, err));
+            send_fix2(p, ssacc[0] * inv_d, lim, err);
             ssacc[0] = 0.f;
         }
     };
-#define FAIL_EXIT() return
+    // a failed wait leaves the layer loop; the CTA still meets its cluster at
+    // the end, so no other CTA stores into its shared memory after it exits
+#define FAIL_EXIT() goto done
 
     for (int l = 0; l < P.n_layers; ++l) {
-        unsigned long long *xl = P.xacc + (size_t)l * P.acc_layer;
-        unsigned long long *xp = xl - P.acc_layer;  // the previous layer's words
+        unsigned long long *xl = P.xacc + (size_t)2 * l * P.acc_layer;
+        unsigned long long *xp = xl - 2 * P.acc_layer;  // the previous layer's pairs
         const unsigned par = (unsigned)(l & 1);
 
         // ================= phase A: a = h + Down_{l-1}(m) on R_c; stage 1 of q, k, v
         if (!wait_full(full + 0, par, P.ws_words)) FAIL_EXIT();
-        if (l > 0 && !run_poll_tables(pg, A_P2, xp, n_ctas, 1.f, inv_d, P.ws_words))
+        if (l > 0 && !run_poll_tables(pg, A_P2, xp, n_t, n_ctas, 1.f, P.ws_words))
             FAIL_EXIT();
         run_rows(pg, A_R, l > 0, true, o.ssacc);  // a = res0 + Down(m) -> res1; tables
         csync();
-        send_ss(xl + P.offA + ssA);
-        run_s1(pg, A_S1, xl, lim, err);
+        send_ss(fix2_at(xl, P.offA + ssA));
+        if (!csync_and(run_s1(pg, A_S1, xl, lim, err, o.slot[0], o.ubar0[0], o.ubar, par, rank,
+                              P.ws_words)))
+            FAIL_EXIT();
         // regions C and Q of the previous layer: every CTA has passed the
         // poll that read them (exchange D, polled above, counts all CTAs)
         if (l > 0) {
-            zero_stripe(xp + P.offC, s_zs[XR_C]);
-            zero_stripe(xp + P.offQ, s_zs[XR_Q]);
+            zero_stripe(at(xp, P.offC), s_zs[XR_C]);
+            zero_stripe(at(xp, P.offQ), s_zs[XR_Q]);
         }
         release(0);
 
         // ================= phase B: v rows for attention, stage 1 of o; then q, k, v out
         if (!wait_full(full + 1, par, P.ws_words)) FAIL_EXIT();
         // tables of v (critical) and of q, k (region Q, sent with region A)
-        if (!run_poll_tables(pg, B_P2, xl, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
+        if (!run_poll_tables(pg, B_P2, xl, n_t, n_ctas, 1.f, P.ws_words)) FAIL_EXIT();
         run_rows(pg, B_R, true, true, o.ssacc);  // v on the attention rows; tables of o
         csync();
-        run_s1(pg, B_S1, xl, lim, err);
-        if (l > 0) zero_stripe(xp + P.offD, s_zs[XR_D]);  // read by phase A's poll
+        if (!csync_and(run_s1(pg, B_S1, xl, lim, err, o.slot[1], o.ubar0[1], o.ubar, par, rank,
+                              P.ws_words)))
+            FAIL_EXIT();
+        if (l > 0) zero_stripe(at(xp, P.offD), s_zs[XR_D]);  // read by phase A's poll
         // ---- off the critical path, while exchange B is in flight: q on R_c,
         //      k and v on K_c (their tables were built with v's)
         run_s2(pg, B_S2QKV);  // -> yq, yk, yv
@@ -756,32 +849,36 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
 
         // ================= phase C: h = a + O(attn) on R_c; stage 1 of gate, up
         if (!wait_full(full + 2, par, P.ws_words)) FAIL_EXIT();
-        if (!run_poll_tables(pg, C_P2, xl, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
+        if (!run_poll_tables(pg, C_P2, xl, n_t, n_ctas, 1.f, P.ws_words)) FAIL_EXIT();
         run_rows(pg, C_R, true, true, o.ssacc);  // h = res1 + O(attn) -> res0; tables
         csync();
-        send_ss(xl + P.offC + ssC);
-        run_s1(pg, C_S1, xl, lim, err);
-        zero_stripe(xl + P.offA, s_zs[XR_A]);  // read by phase B's poll
+        send_ss(fix2_at(xl, P.offC + ssC));
+        if (!csync_and(run_s1(pg, C_S1, xl, lim, err, o.slot[2], o.ubar0[2], o.ubar, par, rank,
+                              P.ws_words)))
+            FAIL_EXIT();
+        zero_stripe(at(xl, P.offA), s_zs[XR_A]);  // read by phase B's poll
         release(2);
 
         // ================= phase D: m = silu(gate) * up on F_c; stage 1 of down
         if (!wait_full(full + 3, par, P.ws_words)) FAIL_EXIT();
-        if (!run_poll_tables(pg, D_P2, xl, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
+        if (!run_poll_tables(pg, D_P2, xl, n_t, n_ctas, 1.f, P.ws_words)) FAIL_EXIT();
         run_rows(pg, D_R, true, true, o.ssacc);  // m = silu(gate) * up; tables of down
         csync();
-        run_s1(pg, D_S1, xl, lim, err);
-        zero_stripe(xl + P.offB, s_zs[XR_B]);  // read by phase C's poll
+        if (!csync_and(run_s1(pg, D_S1, xl, lim, err, o.slot[3], o.ubar0[3], o.ubar, par, rank,
+                              P.ws_words)))
+            FAIL_EXIT();
+        zero_stripe(at(xl, P.offB), s_zs[XR_B]);  // read by phase C's poll
         release(3);
     }
 
     // ================= final: out = h + Down_{L-1}(m) on R_c
     {
         const int l = P.n_layers;
-        unsigned long long *xp = P.xacc + (size_t)(l - 1) * P.acc_layer;
+        unsigned long long *xp = P.xacc + (size_t)2 * (l - 1) * P.acc_layer;
         if (!wait_full(full + 0, (unsigned)(l & 1), P.ws_words)) FAIL_EXIT();
-        if (!run_poll_tables(pg, A_P2, xp, n_ctas, 1.f, inv_d, P.ws_words)) FAIL_EXIT();
-        zero_stripe(xp + P.offC, s_zs[XR_C]);
-        zero_stripe(xp + P.offQ, s_zs[XR_Q]);
+        if (!run_poll_tables(pg, A_P2, xp, n_t, n_ctas, 1.f, P.ws_words)) FAIL_EXIT();
+        zero_stripe(at(xp, P.offC), s_zs[XR_C]);
+        zero_stripe(at(xp, P.offQ), s_zs[XR_Q]);
         run_rows(pg, A_R, true, false, o.ssacc);  // a = res0 + Down(m) -> res1
         csync();
         for (int i = threadIdx.x; i < rows_d; i += kCT) P.out[32 * s.dw0 + i] = res1[i];
@@ -794,10 +891,16 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         csync();
         if (s_last) {
             __threadfence();
-            for (int i = threadIdx.x; i < P.lenD; i += kCT) xp[P.offD + i] = 0ull;
+            for (int i = threadIdx.x; i < (int)fix2_words(P.lenD); i += kCT)
+                at(xp, P.offD)[i] = 0ull;
             if (lead) P.ws_words[kDoneWord] = 0u;
         }
     }
+    }  // compute warps
+done:
+    // no CTA leaves while another CTA of its cluster may still store into its
+    // shared memory (every wait above is bounded, so every thread gets here)
+    if (kCluster > 1) cluster_sync_all();
 #undef FAIL_EXIT
 }
 
@@ -831,9 +934,9 @@ int rsum(const lb_linear &L) {
 
 int up(int n, int a) { return (n + a - 1) / a * a; }
 
-// Exchange words per layer: A = t of v + ss(a); Q = t of q, k (read off
-// the critical path); B = t of o; C = t of gate, up + ss(h); D = t of down;
-// each region padded to 32 words.
+// Exchange elements (pairs of words) per layer: A = t of v + ss(a); Q = t of
+// q, k (read off the critical path); B = t of o; C = t of gate, up + ss(h);
+// D = t of down; each region padded to 32 elements.
 struct XLayout {
     int acc_layer, offA, offQ, offB, offC, offD, lenA, lenQ, lenB, lenC, lenD;
 };
@@ -856,6 +959,14 @@ XLayout xlayout(const lb_linear *lin) {
 
 size_t desc_bytes_for(int n_layers) {
     return ((size_t)7 * n_layers * sizeof(LinDesc) + 255) & ~(size_t)255;
+}
+
+// Stage-1 units (32-column blocks over every path) of linears k0..k1.
+int s1_units(const lb_linear *lin, int k0, int k1) {
+    int n = 0;
+    for (int k = k0; k <= k1; ++k)
+        for (int p = 0; p < lin[k].n_paths; ++p) n += (lin[k].path[p].r + 31) / 32;
+    return n;
 }
 
 // Shared-memory plan from the largest slices any CTA gets.
@@ -956,6 +1067,19 @@ SmemPlan smem_plan(const lb_linear *lin, const StackShape &sh, int N) {
     o.yv = take(4 * nkv);
     o.ssacc = take(16);
     o.prog = take(kProgBytes);
+    // cluster reduction: per phase, the receive slots and mbarriers of the
+    // ceil(units / kCluster) stage-1 units a rank owns at most
+    const int units[4] = {s1_units(lin, LQ, LV), s1_units(lin, LO, LO), s1_units(lin, LG, LU),
+                          s1_units(lin, LD, LD)};
+    o.n_ubar = 0;
+    for (int ph = 0; ph < 4; ++ph) {
+        const int owned = kCluster > 1 ? (units[ph] + kCluster - 1) / kCluster : 0;
+        o.slot[ph] = take(owned * kCluster * 128);
+        o.ubar0[ph] = o.n_ubar;
+        o.n_ubar += owned;
+    }
+    at = up(at, 8);
+    o.ubar = take(8 * o.n_ubar);
     S.bytes = up(at, 128);
     return S;
 }
@@ -1146,18 +1270,25 @@ struct ProgBuild {
         }
         place(s, best, best_wo);
     }
-    // 32-column blocks over the whole input slice.
-    void s1(int s, const std::vector<S1Job> &jobs) {
+    // 32-column blocks over the whole input slice.  Unit g of the phase
+    // belongs to cluster rank g % kCluster (its receive slot there: g /
+    // kCluster); each warp runs the units its CTA (rank `rank`) does not own
+    // first, so their partials are on their way before it waits for its own.
+    void s1(int s, const std::vector<S1Job> &jobs, int rank) {
         std::vector<Costed> us;
+        int g = 0;
         for (const S1Job &J : jobs)
-            for (int c0 = 0; c0 < J.r; c0 += 32)
+            for (int c0 = 0; c0 < J.r; c0 += 32, ++g)
                 us.push_back({Item{{J.V + 4 * c0, J.r, J.nw, J.tb, J.dst + c0,
-                                    std::min(32, J.r - c0), 0, 0}},
+                                    std::min(32, J.r - c0), g % kCluster, g / kCluster}},
                               J.nw + 1.0});
-        std::vector<Item> g;
+        std::vector<Item> grouped;
         int wo[kCW + 1];
-        lpt(us, g, wo);
-        place(s, g, wo);
+        lpt(us, grouped, wo);
+        for (int w = 0; w < kCW; ++w)
+            std::stable_partition(grouped.begin() + wo[w], grouped.begin() + wo[w + 1],
+                                  [rank](const Item &it) { return it.f[6] != rank; });
+        place(s, grouped, wo);
     }
 };
 
@@ -1184,8 +1315,9 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
         B.s2(s, U);
         U.clear();
     };
+    const int rank = c % kCluster;  // cluster rank of CTA c (1-D clusters of kCluster)
     auto flush_v = [&](int s) {
-        B.s1(s, V);
+        B.s1(s, V, rank);
         V.clear();
     };
     auto pair_of = [](const std::vector<Seg> &g) {
@@ -1365,7 +1497,8 @@ static_assert(sizeof(LinDesc) % sizeof(uint32_t) == 0, "descriptor is copied as 
 
 size_t stack_ws_bytes_after_header(const lb_linear *lin, int n_layers) {
     const XLayout X = xlayout(lin);
-    return desc_bytes_for(n_layers) + (size_t)n_layers * X.acc_layer * sizeof(unsigned long long) +
+    return desc_bytes_for(n_layers) +
+           (size_t)2 * n_layers * X.acc_layer * sizeof(unsigned long long) +
            (size_t)kMaxCtas * kProgBytes;
 }
 
@@ -1373,14 +1506,15 @@ namespace {
 char *programs_at(const lb_linear *lin, int n_layers, char *ws_after_header) {
     const XLayout X = xlayout(lin);
     return ws_after_header + desc_bytes_for(n_layers) +
-           (size_t)n_layers * X.acc_layer * sizeof(unsigned long long);
+           (size_t)2 * n_layers * X.acc_layer * sizeof(unsigned long long);
 }
 }  // namespace
 
 cudaError_t launch_stack_prepare(const lb_linear *lin, int n_layers, const StackShape &sh,
                                  int num_sms, unsigned long long plan, unsigned *ws_words,
                                  char *ws_after_header, cudaStream_t s) {
-    if (!shapes_ok(lin, sh, num_sms) || !smem_fits(lin, sh, num_sms)) return cudaErrorNotSupported;
+    if (num_sms % kCluster != 0 || !shapes_ok(lin, sh, num_sms) || !smem_fits(lin, sh, num_sms))
+        return cudaErrorNotSupported;
     std::vector<int> progs;
     if (!build_programs(lin, sh, num_sms, progs)) return cudaErrorNotSupported;
     const XLayout X = xlayout(lin);
@@ -1388,8 +1522,8 @@ cudaError_t launch_stack_prepare(const lb_linear *lin, int n_layers, const Stack
     char *xacc = ws_after_header + desc_bytes_for(n_layers);
     cudaError_t e = cudaMemsetAsync(ws_words + kCounterWord, 0, 2 * sizeof(unsigned), s);
     if (e == cudaSuccess)
-        e = cudaMemsetAsync(xacc, 0, (size_t)n_layers * X.acc_layer * sizeof(unsigned long long),
-                            s);
+        e = cudaMemsetAsync(xacc, 0,
+                            (size_t)2 * n_layers * X.acc_layer * sizeof(unsigned long long), s);
     // pageable source: the call returns once the data is staged
     if (e == cudaSuccess)
         e = cudaMemcpyAsync(programs_at(lin, n_layers, ws_after_header), progs.data(),
@@ -1409,7 +1543,46 @@ cudaError_t launch_stack_prepare(const lb_linear *lin, int n_layers, const Stack
 }
 
 bool stack_supported(const lb_linear *lin, const StackShape &sh, int num_sms) {
-    return shapes_ok(lin, sh, num_sms) && smem_fits(lin, sh, num_sms);
+    return num_sms % kCluster == 0 && shapes_ok(lin, sh, num_sms) && smem_fits(lin, sh, num_sms);
+}
+
+int stack_grid_ctas(const lb_linear *lin, const StackShape &sh, int num_sms) {
+    if (kCluster == 1) return num_sms;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+    // the plan of the full grid bounds the shared memory from below (smaller
+    // grids give each CTA larger slices); clusters need not fill every SM
+    const int smem = smem_plan(lin, sh, num_sms).bytes;
+    static std::mutex mu;
+    static int cached_dev = -1, cached_smem = -1, cached_sms = -1, cached_n = 0;
+    std::lock_guard<std::mutex> lock(mu);
+    if (dev == cached_dev && smem == cached_smem && num_sms == cached_sms) return cached_n;
+    if (cudaFuncSetAttribute((const void *)k_stack, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             smem) != cudaSuccess)
+        return 0;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(kCluster, 1, 1);
+    cfg.blockDim = dim3(kST, 1, 1);
+    cfg.dynamicSmemBytes = (size_t)smem;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = kCluster;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 1;
+    int n_cl = 0;
+    if (cudaOccupancyMaxActiveClusters(&n_cl, (const void *)k_stack, &cfg) != cudaSuccess ||
+        n_cl <= 0)
+        return 0;
+    const int n = std::min(num_sms / kCluster, n_cl) * kCluster;
+    // the larger slices of the smaller grid must still fit
+    if (!smem_fits(lin, sh, n)) return 0;
+    cached_dev = dev;
+    cached_smem = smem;
+    cached_sms = num_sms;
+    cached_n = n;
+    return n;
 }
 
 cudaError_t launch_stack(const lb_linear *lin, int n_layers, const StackShape &sh,
@@ -1448,7 +1621,9 @@ cudaError_t launch_stack(const lb_linear *lin, int n_layers, const StackShape &s
     P.lenB = X.lenB;
     P.lenC = X.lenC;
     P.lenD = X.lenD;
-    P.fix_limit = 2147483648.f / (float)num_sms;
+    if (num_sms % kCluster != 0) return cudaErrorInvalidConfiguration;
+    P.n_t = (unsigned)(num_sms / kCluster);
+    P.fix_limit = fix2_limit(num_sms);
     P.o = S.o;
     const size_t smem = (size_t)S.bytes;
     cudaError_t e = cudaFuncSetAttribute((const void *)k_stack,
@@ -1458,9 +1633,23 @@ cudaError_t launch_stack(const lb_linear *lin, int n_layers, const StackShape &s
     e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, (const void *)k_stack, kST, smem);
     if (e != cudaSuccess) return e;
     if (per_sm < 1) return cudaErrorCooperativeLaunchTooLarge;
-    void *args[] = {&P};
-    return cudaLaunchCooperativeKernel((const void *)k_stack, dim3(num_sms), dim3(kST), args, smem,
-                                       s);
+    // cooperative: the grid is launched only if every CTA is co-resident (the
+    // kernel's waits need that); clusters of kCluster consecutive CTAs
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(num_sms, 1, 1);
+    cfg.blockDim = dim3(kST, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute at[2];
+    at[0].id = cudaLaunchAttributeCooperative;
+    at[0].val.cooperative = 1;
+    at[1].id = cudaLaunchAttributeClusterDimension;
+    at[1].val.clusterDim.x = kCluster;
+    at[1].val.clusterDim.y = 1;
+    at[1].val.clusterDim.z = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 2;
+    return cudaLaunchKernelEx(&cfg, k_stack, P);
 }
 
 }  // namespace lb

@@ -32,9 +32,9 @@ def f32_to_bf16_bits(a: np.ndarray) -> np.ndarray:
     return rounded.astype(np.uint16)
 
 
-def bf16_normal(rng: np.random.Generator, shape) -> np.ndarray:
-    """N(0,1) activations stored as bf16 bit patterns."""
-    return f32_to_bf16_bits(rng.standard_normal(shape).astype(np.float32))
+def bf16_normal(rng: np.random.Generator, shape, scale: float = 1.0) -> np.ndarray:
+    """N(0,1) * scale activations stored as bf16 bit patterns."""
+    return f32_to_bf16_bits((rng.standard_normal(shape) * scale).astype(np.float32))
 
 
 def fp16_abs_normal(rng: np.random.Generator, n: int, c: float) -> np.ndarray:
@@ -72,11 +72,13 @@ def random_v_words(rng: np.random.Generator, d_in: int, r: int) -> np.ndarray:
 
 
 def make_linear(rng: np.random.Generator, d_in: int, d_out: int, r, n_paths: int = 2,
-                scale: float = 0.02, explicit_signs: bool = False) -> dict:
+                scale: float = 0.02, explicit_signs: bool = False, g_mul: float = 1.0,
+                l_mul: float = 1.0, h_mul: float = 1.0) -> dict:
     """One LittleBit linear.  With explicit_signs=True each path carries
     'u_signs' [d_out][r] and 'v_signs' [d_in][r] (+-1 int8) and no words;
     otherwise it carries random 'u_words' / 'v_words' in the packed layout.
-    r may be an int or a per-path list."""
+    r may be an int or a per-path list.  g, l and h are drawn at scale times
+    g_mul, l_mul and h_mul."""
     rs = list(r) if isinstance(r, (list, tuple)) else [int(r)] * n_paths
     paths = []
     for p in range(n_paths):
@@ -88,9 +90,9 @@ def make_linear(rng: np.random.Generator, d_in: int, d_out: int, r, n_paths: int
         else:
             P["v_words"] = random_v_words(rng, d_in, rp)
             P["u_words"] = random_u_words(rng, d_out, rp)
-        P["g"] = fp16_abs_normal(rng, d_in, scale)
-        P["l"] = fp16_abs_normal(rng, rp, scale)
-        P["h"] = fp16_abs_normal(rng, d_out, scale)
+        P["g"] = fp16_abs_normal(rng, d_in, scale * g_mul)
+        P["l"] = fp16_abs_normal(rng, rp, scale * l_mul)
+        P["h"] = fp16_abs_normal(rng, d_out, scale * h_mul)
         paths.append(P)
     return {"d_in": int(d_in), "d_out": int(d_out), "paths": paths}
 
@@ -164,17 +166,21 @@ def unit_gain_scale(d_in: int, r: int, n_paths: int = 2) -> float:
 
 def make_stack(n_layers: int = 80, d_model: int = 8192, d_kv: int = 1024, d_ff: int = 28672,
                r_qo: int = 192, r_kv: int = 32, r_mlp: int = 320, head_dim: int = 128,
-               config_id: int = 5):
+               config_id: int = 5, x_scale: float = 1.0, g_mul: float = 1.0,
+               l_mul: float = 1.0, out_h_mul: float = 1.0):
     """Llama2-70B-shaped decode stack: n_layers x (q,k,v,o,gate,up,down), two
-    paths each, random sign words, unit-gain scales.
-    Returns (list of 7*n_layers linears, x0 bf16 bits [d_model])."""
+    paths each, random sign words, unit-gain scales (g and l times g_mul and
+    l_mul, the h of o and down -- the branches that write the residual
+    stream -- times out_h_mul).
+    Returns (list of 7*n_layers linears, x0 bf16 bits [d_model], N(0,1) * x_scale)."""
     rng = rng_for(config_id)
     shapes = stack_shapes(d_model, d_kv, d_ff, r_qo, r_kv, r_mlp)
     layers = []
     for _ in range(n_layers):
-        for (di, do, r) in shapes:
-            layers.append(make_linear(rng, di, do, r, 2, unit_gain_scale(di, r, 2)))
-    x0 = bf16_normal(rng, (d_model,))
+        for k, (di, do, r) in enumerate(shapes):
+            layers.append(make_linear(rng, di, do, r, 2, unit_gain_scale(di, r, 2), g_mul=g_mul,
+                                      l_mul=l_mul, h_mul=out_h_mul if k in (3, 6) else 1.0))
+    x0 = bf16_normal(rng, (d_model,), x_scale)
     return layers, x0
 
 
