@@ -24,7 +24,9 @@ latent-state halves (littlebit_linear_latent / _expand: the 70B key
 projection at T = 1 and a 4096-token cache, 4096x4096 r512 at T = 2048);
 7 = Dual-SVID initialisation of a dense weight into two paths (ms per layer);
 8 = one QAT step (forward + SmoothSign backward) at 2048 tokens (TFLOP/s
-against the TF32 tensor peak).
+against the TF32 tensor peak); 10 = the exchange floor of the 70B-shaped
+stack: one token's 320 dependent rank-r all-reduces (four per layer, of the
+stack's element counts) with nothing between them (littlebit_selftest_exchange).
 Cases 2, 3 and the CUDA-core cases of 6 report algorithmic GB/s with L2
 flushed before every call; 4 and the tensor-core cases of 6 report TFLOP/s
 (2 flops per +-1 MAC, both paths) against the dense bf16 peak.
@@ -61,7 +63,7 @@ def parse_args():
     ap.add_argument("--layers", type=int, default=80,
                     help="stack depth (80 = the Llama2-70B workload; smaller only for profiling)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--config", type=int, choices=[2, 3, 4, 6, 7, 8, 9], default=None,
+    ap.add_argument("--config", type=int, choices=[2, 3, 4, 6, 7, 8, 9, 10], default=None,
                     help="time a single-linear workload instead of the stack")
     ap.add_argument("--only", default=None,
                     help="with --config: only the cases whose 'name:T' contains this text")
@@ -798,6 +800,34 @@ def run_config(args):
                                "tokens/s; other hardware and a trained model"}
             print(json.dumps(line), flush=True)
             del dec, graph
+    elif args.config == 10:
+        # the exchange floor: per layer the four all-reduces on the stack's
+        # critical path (t of v + the mean square; o; gate, up + the mean
+        # square; down), 80 layers, nothing between them
+        s70 = inputs.STACK_70B
+        sizes = [2 * s70["r_kv"] + 1, 2 * s70["r_qo"], 4 * s70["r_mlp"] + 1, 2 * s70["r_mlp"]]
+        rounds = 4 * s70["n_layers"]
+        for cluster in (1, 2):
+            ws = lb.selftest_exchange(rounds, sizes, cluster, device=dev)
+            torch.cuda.synchronize(dev)
+            times = []
+            for _ in range(max(3, args.warmup) + steps):
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record()
+                lb.selftest_exchange(rounds, sizes, cluster, ws=ws, device=dev)
+                e1.record()
+                torch.cuda.synchronize(dev)
+                times.append(e0.elapsed_time(e1))
+            if lb.poll_error(ws) != lb.LB_OK:
+                raise RuntimeError("exchange diagnostic reported an error")
+            ms = statistics.median(times[max(3, args.warmup):])
+            print(json.dumps({"config": 10, "case": "exchange floor", "cluster": cluster,
+                              "sizes": sizes, "rounds": rounds, "ms_per_token": ms,
+                              "us_per_exchange": 1e3 * ms / rounds,
+                              "us_per_layer": 4e3 * ms / rounds,
+                              "note": "launch included; one cooperative launch per token"}),
+                  flush=True)
     elif args.config == 6:
         # latent states (KV cache compression): the 70B key projection's latent
         # for one new token and the expansion of a 4096-token latent cache

@@ -400,6 +400,25 @@ lb_status littlebit_poll_error(void *ws, lb_stream_t stream);
  * littlebit_poll_error.  ws: a zero-filled workspace of at least 256 bytes. */
 lb_status littlebit_selftest_wait_timeout(void *ws, lb_stream_t stream);
 
+/* Diagnostic: the latency floor of the exchange that the single-token
+ * kernels run between stage 1 and stage 2 of every linear (Prop. 1: the
+ * rank-r partial sums t = V_sign^T (g . x) of every CTA's input slice,
+ * all-reduced across the GPU before stage 2).  One persistent launch, one CTA
+ * per SM, runs n_rounds dependent exchanges of sizes[k % n_sizes] elements
+ * (1 <= n_sizes <= 8, 1 <= sizes[i] <= 2048) with the encoding, polling and
+ * (cluster = 2) two-CTA distributed-shared-memory pre-reduction that
+ * littlebit_stack_forward uses, and nothing else: elapsed time / n_rounds is
+ * the exchange's cost on the stack's critical path.  ws: 256-byte aligned,
+ * littlebit_selftest_exchange_workspace_size bytes, header zero-filled before
+ * the first use (the call clears the rest); an error (a wait that ran out)
+ * is recorded in the header like the other kernels', read with
+ * littlebit_poll_error.  The paper has no counterpart: it is a measurement. */
+size_t littlebit_selftest_exchange_workspace_size(int32_t n_rounds, const int32_t *sizes,
+                                                   int32_t n_sizes);
+lb_status littlebit_selftest_exchange(int32_t n_rounds, const int32_t *sizes, int32_t n_sizes,
+                                      int32_t cluster, void *ws, size_t ws_bytes,
+                                      lb_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

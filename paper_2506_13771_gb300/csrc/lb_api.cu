@@ -489,4 +489,29 @@ lb_status littlebit_selftest_wait_timeout(void *ws, lb_stream_t stream) {
     return from_cuda(lb::launch_wait_timeout(static_cast<unsigned *>(ws), (cudaStream_t)stream));
 }
 
+size_t littlebit_selftest_exchange_workspace_size(int32_t n_rounds, const int32_t *sizes,
+                                                   int32_t n_sizes) {
+    if (n_rounds < 1 || !sizes || n_sizes < 1 || n_sizes > 8) return 0;
+    return lb::xchain_ws_bytes(n_rounds, sizes, n_sizes);
+}
+
+lb_status littlebit_selftest_exchange(int32_t n_rounds, const int32_t *sizes, int32_t n_sizes,
+                                      int32_t cluster, void *ws, size_t ws_bytes,
+                                      lb_stream_t stream) {
+    if (n_rounds < 1 || !sizes || n_sizes < 1 || n_sizes > 8 || (cluster != 1 && cluster != 2))
+        return LB_ERR_INVALID_ARG;
+    for (int i = 0; i < n_sizes; ++i)
+        if (sizes[i] < 1 || sizes[i] > 2048) return LB_ERR_INVALID_ARG;
+    if (!ws || ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) ||
+        ws_bytes < lb::xchain_ws_bytes(n_rounds, sizes, n_sizes))
+        return LB_ERR_WORKSPACE;
+    int sms = 0;
+    lb_status st = num_sms(&sms);
+    if (st != LB_OK) return st;
+    return from_cuda(lb::launch_xchain(n_rounds, sizes, n_sizes, cluster,
+                                       static_cast<unsigned *>(ws),
+                                       static_cast<char *>(ws) + kWsHeader, sms,
+                                       (cudaStream_t)stream));
+}
+
 }  // extern "C"

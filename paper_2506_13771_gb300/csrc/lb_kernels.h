@@ -113,6 +113,13 @@ cudaError_t launch_train_backward(const lb_train_linear &L, const float *x, cons
 // Bounded-wait diagnostic (lb_persistent.cu).
 cudaError_t launch_wait_timeout(unsigned *ws_words, cudaStream_t s);
 
+// Exchange-chain diagnostic (lb_xchain.cu): n_rounds dependent all-reduces
+// of sizes[k % n_sizes] elements over the grid (cluster 1 or 2); buf holds
+// n_rounds buffers and is cleared by the launcher.
+size_t xchain_ws_bytes(int n_rounds, const int *sizes, int n_sizes);
+cudaError_t launch_xchain(int n_rounds, const int *sizes, int n_sizes, int cluster,
+                          unsigned *ws_words, void *buf, int num_sms, cudaStream_t s);
+
 // Sign packing (lb_pack.cu).
 cudaError_t launch_pack(const int8_t *signs, int64_t rows, int64_t cols, int layout,
                         uint32_t *out, int32_t *bad, cudaStream_t s);

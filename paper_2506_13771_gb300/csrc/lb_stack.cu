@@ -210,12 +210,25 @@ __device__ __noinline__ void run_rows(int prog, int s, bool do_s2, bool do_tab, 
                 const uint32_t *Uw = sm_u32(half ? a1.x : a0.x) + row * (half ? a1.y : a0.y);
                 const uint32_t tb = (uint32_t)(half ? a1.w : a0.w);
                 float s0 = 0.f, s1 = 0.f;
-                for (int w = 0; w < nwm; w += 2) {
-                    const int wa = max(min(w, nw - 1), 0), wb = max(min(w + 1, nw - 1), 0);
-                    const float va = lut_word(Uw[wa], copy, tb + wa * 1024);
-                    const float vb = lut_word(Uw[wb], copy, tb + wb * 1024);
-                    s0 += w < nw ? va : 0.f;
-                    s1 += w + 1 < nw ? vb : 0.f;
+                if (a0.z == a1.z) {
+                    // both halves sum the same number of words: no clamps, no masks
+                    int w = 0;
+#pragma unroll 1
+            #pragma unroll 1
+        for (; w + 2 <= nw; w += 2) {
+                        s0 += lut_word(Uw[w], copy, tb + w * 1024);
+                        s1 += lut_word(Uw[w + 1], copy, tb + (w + 1) * 1024);
+                    }
+                    if (w < nw) s0 += lut_word(Uw[w], copy, tb + w * 1024);
+                } else {
+#pragma unroll 1
+                    for (int w = 0; w < nwm; w += 2) {
+                        const int wa = max(min(w, nw - 1), 0), wb = max(min(w + 1, nw - 1), 0);
+                        const float va = lut_word(Uw[wa], copy, tb + wa * 1024);
+                        const float vb = lut_word(Uw[wb], copy, tb + wb * 1024);
+                        s0 += w < nw ? va : 0.f;
+                        s1 += w + 1 < nw ? vb : 0.f;
+                    }
                 }
                 const float h = half_bits_to_float(sm_u16(half ? b1.x : b0.x)[row]);
                 acc += nw > 0 ? (s0 + s1) * h : 0.f;
@@ -241,6 +254,7 @@ __device__ __noinline__ void run_rows(int prog, int s, bool do_s2, bool do_tab, 
                                          __shfl_sync(0xffffffffu, x, 4 * n + 1),
                                          __shfl_sync(0xffffffffu, x, 4 * n + 2),
                                          __shfl_sync(0xffffffffu, x, 4 * n + 3));
+#pragma unroll 1
             for (int L = lane; L < 4 * njob; L += 32) {
                 int4 ta, tz;
                 item_at(prog, u + 1 + 2 * npair + (L >> 2), ta, tz);
@@ -275,6 +289,7 @@ __device__ __noinline__ void run_s2(int prog, int s) {
         const uint32_t *U1 = sm_u32(c.x) + min(lane, d.z - 1) * c.y;
         const int nw = max(a.z, c.z);
         float acc0 = 0.f, acc1 = 0.f;
+#pragma unroll 1
         for (int w = 0; w < nw; ++w) {
             const int w0 = min(w, a.z - 1), w1 = min(w, c.z - 1);
             const float v0 = lut_word(U0[w0], copy, (uint32_t)a.w + w0 * 1024);
@@ -294,6 +309,7 @@ __device__ __noinline__ void run_s2(int prog, int s) {
         const uint32_t *Uw = sm_u32(a.x) + row * R;
         float acc0 = 0.f, acc1 = 0.f;
         int w = 0;
+#pragma unroll 1
         for (; w + 2 <= nw; w += 2) {
             const uint32_t w0 = Uw[w], w1 = Uw[w + 1];
             acc0 += lut_word(w0, copy, tb + w * 1024);
@@ -390,6 +406,7 @@ __device__ __noinline__ bool run_s1(int prog, int s, unsigned long long *xbase, 
         const uint32_t *V1 = sm_u32(c.x) + min(lane, d.y - 1);
         const int nw = max(a.z, c.z);
         float acc0 = 0.f, acc1 = 0.f;
+#pragma unroll 1
         for (int w = 0; w < nw; ++w) {
             const int w0 = max(min(w, a.z - 1), 0), w1 = max(min(w, c.z - 1), 0);
             const float v0 = lut_word(V0[w0 * a.y], copy, (uint32_t)a.w + w0 * 1024);
@@ -408,6 +425,7 @@ __device__ __noinline__ bool run_s1(int prog, int s, unsigned long long *xbase, 
         const uint32_t *Vw = sm_u32(a.x) + min(lane, ncols - 1);
         float acc0 = 0.f, acc1 = 0.f;
         int w = 0;
+#pragma unroll 1
         for (; w + 2 <= nw; w += 2) {
             const uint32_t w0 = Vw[w * r], w1 = Vw[(w + 1) * r];
             acc0 += lut_word(w0, copy, tb + w * 1024);
@@ -470,13 +488,10 @@ __device__ __noinline__ bool run_poll_tables(int prog, int s, const unsigned lon
         // and once it sees its word complete the whole unit usually is
         if (lane == 0 && a.z > 0) {
             const unsigned long long t0 = globaltimer_ns();
-            const unsigned long long *gw = fix2_at(xbase, b.x + (min(a.z, 4 * a.y) - 1));
-            unsigned long long gh, gl;
-            for (int spin = 0;; ++spin) {
-                ld_fix2(gw, gh, gl);
-                if (counted2(gh, gl, n_t)) break;
+            // the lo word of the last element (the lo words are sent after the hi words)
+            const unsigned long long *gw = fix2_at(xbase, b.x + (min(a.z, 4 * a.y) - 1)) + 32;
+            for (int spin = 0; (unsigned)(ld_relaxed_u64(gw) & 0xffull) != n_t; ++spin)
                 if ((spin & 15) == 15 && globaltimer_ns() - t0 > kWaitLimitNs) break;
-            }
         }
         __syncwarp();
         if (lane >= a.y) continue;

@@ -32,7 +32,8 @@ EXPORTED = ["littlebit_status_string", "littlebit_pack", "littlebit_workspace_si
             "littlebit_selftest_wait_timeout", "littlebit_linear_forward_noalloc",
             "littlebit_decoder_workspace_size", "littlebit_decoder_step",
             "littlebit_decoder_poll_error", "littlebit_multi_workspace_size",
-            "littlebit_linear_forward_multi"]
+            "littlebit_linear_forward_multi", "littlebit_selftest_exchange_workspace_size",
+            "littlebit_selftest_exchange"]
 
 
 class lb_decoder_shape(ctypes.Structure):
@@ -157,6 +158,10 @@ def lib(path: str | None = None):
         L.littlebit_linear_forward_noalloc.argtypes = [ctypes.POINTER(lb_linear), vp, i64, vp,
                                                        i32, vp]
         L.littlebit_linear_forward_noalloc.restype = ctypes.c_int
+        L.littlebit_selftest_exchange_workspace_size.argtypes = [i32, vp, i32]
+        L.littlebit_selftest_exchange_workspace_size.restype = sz
+        L.littlebit_selftest_exchange.argtypes = [i32, vp, i32, i32, vp, sz, vp]
+        L.littlebit_selftest_exchange.restype = ctypes.c_int
         if path is None:
             _lib = L
         return L
@@ -505,6 +510,22 @@ def selftest_wait_timeout(ws: torch.Tensor, stream=None) -> None:
     """Launch the bounded-wait diagnostic (records LB_ERR_TIMEOUT in ws)."""
     _check(lib().littlebit_selftest_wait_timeout(ws.data_ptr(), _stream(stream)),
            "littlebit_selftest_wait_timeout")
+
+
+def selftest_exchange(n_rounds: int, sizes, cluster: int = 2, ws: torch.Tensor | None = None,
+                      device="cuda", stream=None) -> torch.Tensor:
+    """Launch the exchange-chain diagnostic (n_rounds dependent all-reduces of
+    sizes[k % len(sizes)] elements); returns the workspace (poll it)."""
+    arr = (ctypes.c_int32 * len(sizes))(*[int(v) for v in sizes])
+    need = int(lib().littlebit_selftest_exchange_workspace_size(int(n_rounds), arr, len(sizes)))
+    if need == 0:
+        raise LittleBitError(LB_ERR_INVALID_ARG, "littlebit_selftest_exchange_workspace_size")
+    if ws is None:
+        ws = new_workspace(need, device)
+    _check(lib().littlebit_selftest_exchange(int(n_rounds), arr, len(sizes), int(cluster),
+                                             ws.data_ptr(), ws.numel(), _stream(stream)),
+           "littlebit_selftest_exchange")
+    return ws
 
 
 def linear_forward_noalloc(L: DeviceLinear, x: torch.Tensor, out_dtype=torch.bfloat16,

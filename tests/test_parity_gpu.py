@@ -7,6 +7,8 @@ unit-scale data carry a relative error of order 2^-24 * sqrt(n) (about 1e-5
 for the largest reduction here, n = 28672), so 1e-4 leaves a 10x margin;
 bf16 outputs carry the bf16 rounding itself (relative RMS about 1.2e-3).
 """
+import ctypes
+
 import numpy as np
 import pytest
 import torch
@@ -629,3 +631,15 @@ def test_grid_wait_times_out_and_is_sticky():
     lb.linear_forward(D, xin, y=y, ws=ws)
     torch.cuda.synchronize()
     check(y.cpu().numpy().astype(np.float64), oracle.forward_factored(L, x), torch.float32)
+
+
+def test_exchange_diagnostic_runs_clean():
+    """The exchange-chain diagnostic (the stack's all-reduce with nothing around
+    it) completes every round, with and without the two-CTA clusters, and
+    rejects sizes it cannot hold."""
+    for cluster in (1, 2):
+        ws = lb.selftest_exchange(40, [65, 384, 1281, 640], cluster, device=DEV)
+        assert lb.poll_error(ws) == lb.LB_OK
+    arr = (ctypes.c_int32 * 1)(4096)
+    assert lb.lib().littlebit_selftest_exchange(4, arr, 1, 2, ws.data_ptr(), ws.numel(),
+                                                None) == lb.LB_ERR_INVALID_ARG
