@@ -19,7 +19,7 @@ LIB = os.path.join(BUILD, "liblittlebit.so")
 
 SOURCES = ["lb_api.cu", "lb_generic.cu", "lb_persistent.cu", "lb_stack.cu", "lb_pack.cu",
            "lb_noalloc.cu", "lb_prefill.cu", "lb_decode.cu", "lb_svid.cu",
-           "lb_qat.cu", "lb_decoder.cu", "lb_multi.cu", "lb_xchain.cu"]
+           "lb_qat.cu", "lb_decoder.cu", "lb_multi.cu", "lb_xchain.cu", "lb_gemm.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2",
                      "--cudart", "shared", "-I", INCLUDE, "-I", CSRC]

@@ -101,8 +101,27 @@ cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, c
                              uint16_t *const *l, uint16_t *const *h, int iters, void *ws,
                              cudaStream_t s);
 
+// C[M][N] (+)= A[M][K] B[N][K]^T on the tensor cores, TF32 operands and fp32
+// accumulation (lb_gemm.cu).  An operand is fp32, row-major [rows][ld] with
+// its K = k columns first (ld >= k, ld a multiple of 4, 16-byte aligned base);
+// C is row-major at ldc.  A long K over few tiles is split into slices whose
+// partials go to part (gemm_part_floats floats; with less the split is
+// dropped) and are added in slice order.  A bounded wait that runs out
+// records LB_ERR_TIMEOUT in *err; launches return early while it is set.
+struct GemmOperand {
+    const float *p;
+    int rows, k;
+    long long ld;
+};
+bool gemm_operand_ok(const GemmOperand &A);
+size_t gemm_part_floats(int M, int N, int K);
+cudaError_t gemm_tf32(const GemmOperand &A, const GemmOperand &B, float *C, long long ldc,
+                      bool accumulate, float *part, size_t part_floats, unsigned *err,
+                      cudaStream_t s);
+
 // QAT forward / backward on latent factors (lb_qat.cu); ws: qat_ws_bytes for
-// the largest rank.
+// the largest rank (a 256-byte header whose first word is the error word,
+// then the buffers).
 size_t qat_ws_bytes(int d_in, int d_out, int rmax, long long T);
 cudaError_t launch_train_forward(const lb_train_linear &L, const float *x, long long T, float *y,
                                  void *ws, cudaStream_t s);
