@@ -372,16 +372,13 @@ lb_status check_train(const lb_train_linear *L) {
     }
     return LB_OK;
 }
-int train_rmax(const lb_train_linear &L) {
-    int r = 0;
-    for (int p = 0; p < L.n_paths; ++p) r = r > L.path[p].r ? r : L.path[p].r;
-    return r;
-}
 }  // namespace
 
 size_t littlebit_train_workspace_size(const lb_train_linear *L, int64_t T) {
     if (check_train(L) != LB_OK || T < 0 || T > INT32_MAX) return 0;
-    return lb::qat_ws_bytes(L->d_in, L->d_out, train_rmax(*L), T);
+    int rsum = 0;
+    for (int p = 0; p < L->n_paths; ++p) rsum += L->path[p].r;
+    return lb::qat_ws_bytes(L->d_in, L->d_out, rsum, T);
 }
 
 lb_status littlebit_train_forward(const lb_train_linear *L, const float *x, int64_t T, float *y,

@@ -51,6 +51,10 @@ struct GemmParams {
     int bn, tiles_n, split, n_tiles;
     float *part;     // split > 1: [split][M][N] partials
     unsigned *err;
+    // optional second output C2[m][n] = C[m][n] * scale2[n] at ldc2 (not with accumulate)
+    float *C2;
+    const float *scale2;
+    long long ldc2;
 };
 
 struct GemmBars {
@@ -308,6 +312,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
             float *dst = P.split > 1 ? P.part + (size_t)z * P.M * P.N : P.C;
             const long long ld = P.split > 1 ? P.N : P.ldc;
             const bool acc = P.split == 1 && P.accumulate;
+            const bool two = P.split == 1 && P.C2 != nullptr;
             for (int cb = c0; cb < c1; cb += 32) {
                 float v[32];
                 gtmem_ld32(lane_base + (uint32_t)(b * bn + cb), v);
@@ -317,12 +322,31 @@ __global__ void __launch_bounds__(kGThreads, 1)
                 for (int j = 0; j < 32; ++j) stg[lane * kGPitch + j] = v[j];
                 __syncwarp();
                 const int col = n0 + cb + lane;
-                for (int rr = 0; rr < 32; ++rr) {
-                    const int row = m0 + 32 * wq + rr;
-                    if (row >= P.M || col >= P.N) continue;
-                    float *c = dst + (size_t)row * ld + col;
-                    const float x = stg[rr * kGPitch + lane];
-                    *c = acc ? *c + x : x;
+                if (acc) {
+                    // every old value in flight before the first store
+                    float old[32];
+#pragma unroll
+                    for (int rr = 0; rr < 32; ++rr) {
+                        const int row = m0 + 32 * wq + rr;
+                        old[rr] = row < P.M && col < P.N ? dst[(size_t)row * ld + col] : 0.f;
+                    }
+#pragma unroll
+                    for (int rr = 0; rr < 32; ++rr) {
+                        const int row = m0 + 32 * wq + rr;
+                        if (row < P.M && col < P.N)
+                            dst[(size_t)row * ld + col] = old[rr] + stg[rr * kGPitch + lane];
+                    }
+                } else {
+                    const float s2 = two && col < P.N ? P.scale2[col] : 0.f;
+#pragma unroll 8
+                    for (int rr = 0; rr < 32; ++rr) {
+                        const int row = m0 + 32 * wq + rr;
+                        if (row < P.M && col < P.N) {
+                            const float x = stg[rr * kGPitch + lane];
+                            dst[(size_t)row * ld + col] = x;
+                            if (two) P.C2[(size_t)row * P.ldc2 + col] = x * s2;
+                        }
+                    }
                 }
                 __syncwarp();
             }
@@ -360,6 +384,7 @@ __global__ void k_gemm_reduce(const __grid_constant__ GemmParams P) {
         const int row = (int)(i / P.N), col = (int)(i - (long long)row * P.N);
         float *c = P.C + (size_t)row * P.ldc + col;
         *c = P.accumulate ? *c + s : s;
+        if (P.C2) P.C2[(size_t)row * P.ldc2 + col] = s * P.scale2[col];
     }
 }
 
@@ -447,9 +472,10 @@ size_t gemm_part_floats(int M, int N, int K) {
 
 cudaError_t gemm_tf32(const GemmOperand &A, const GemmOperand &B, float *C, long long ldc,
                       bool accumulate, float *part, size_t part_floats, unsigned *err,
-                      cudaStream_t s) {
+                      cudaStream_t s, float *C2, const float *scale2, long long ldc2) {
     if (!gemm_operand_ok(A) || !gemm_operand_ok(B) || A.k != B.k || !C || ldc < B.rows)
         return cudaErrorInvalidValue;
+    if (C2 && (accumulate || !scale2 || ldc2 < B.rows)) return cudaErrorInvalidValue;
     if (!genc()) return cudaErrorNotSupported;
     const int sms = gemm_sms();
     if (sms <= 0) return cudaErrorInvalidDevice;
@@ -469,6 +495,9 @@ cudaError_t gemm_tf32(const GemmOperand &A, const GemmOperand &B, float *C, long
     P.n_tiles = ((P.M + GM - 1) / GM) * P.tiles_n * P.split;
     P.part = part;
     P.err = err;
+    P.C2 = C2;
+    P.scale2 = scale2;
+    P.ldc2 = ldc2;
     CUtensorMap am, bm;
     if (!gmap(&am, A, GM) || !gmap(&bm, B, P.bn)) return cudaErrorInvalidValue;
     const int grid = std::min(P.n_tiles, sms);

@@ -115,14 +115,17 @@ struct GemmOperand {
 };
 bool gemm_operand_ok(const GemmOperand &A);
 size_t gemm_part_floats(int M, int N, int K);
+// C2 (optional, not with accumulate): C2[m][n] = C[m][n] * scale2[n] at ldc2,
+// written beside C (a column scaling that follows the product).
 cudaError_t gemm_tf32(const GemmOperand &A, const GemmOperand &B, float *C, long long ldc,
                       bool accumulate, float *part, size_t part_floats, unsigned *err,
-                      cudaStream_t s);
+                      cudaStream_t s, float *C2 = nullptr, const float *scale2 = nullptr,
+                      long long ldc2 = 0);
 
 // QAT forward / backward on latent factors (lb_qat.cu); ws: qat_ws_bytes for
-// the largest rank (a 256-byte header whose first word is the error word,
-// then the buffers).
-size_t qat_ws_bytes(int d_in, int d_out, int rmax, long long T);
+// the sum of the paths' ranks (a 256-byte header whose first word is the
+// error word, then the buffers).
+size_t qat_ws_bytes(int d_in, int d_out, int rsum, long long T);
 cudaError_t launch_train_forward(const lb_train_linear &L, const float *x, long long T, float *y,
                                  void *ws, cudaStream_t s);
 cudaError_t launch_train_backward(const lb_train_linear &L, const float *x, const float *dy,

@@ -35,117 +35,121 @@ namespace {
 
 __device__ __forceinline__ float sgn(float x) { return x < 0.f ? -1.f : 1.f; }
 
-// Uh[o][j] = h_o S(U_oj) at ld_r, UhT[j][o] = Uh[o][j] at ld_o, Vg[i][j] =
-// g_i S(V_ij) at ld_r and VgT[j][i] at ld_i.
-__global__ void k_fold_signs(const float *U, const float *V, const float *h, const float *g,
-                             int d_out, int d_in, int r, int ld_r, int ld_o, int ld_i, float *Uh,
-                             float *UhT, float *Vg, float *VgT) {
-    const long long nu = (long long)d_out * r, nv = (long long)d_in * r;
-    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < nu + nv;
-         idx += (long long)gridDim.x * blockDim.x) {
-        if (idx < nu) {
-            const int o = (int)(idx / r), j = (int)(idx - (long long)o * r);
-            const float w = h[o] * sgn(U[idx]);
-            Uh[(size_t)o * ld_r + j] = w;
-            UhT[(size_t)j * ld_o + o] = w;
-        } else {
-            const long long q = idx - nu;
-            const int i = (int)(q / r), j = (int)(q - (long long)i * r);
-            const float w = g[i] * sgn(V[q]);
-            Vg[(size_t)i * ld_r + j] = w;
-            VgT[(size_t)j * ld_i + i] = w;
+// Columns [c0, c0 + r) of one path-concatenated sign factor: F[i][c0 + j] =
+// s_i S(L_ij) at ld (L the latent [rows][r], s the row scale) and its
+// transpose FT[c0 + j][i] at ldt, in 64 x 64 tiles through shared memory so
+// that every read and both writes move whole rows.
+__global__ void __launch_bounds__(256) k_fold_signs(const float *Lat, const float *sc, int rows,
+                                                     int r, int c0, int ld, int ldt, float *F,
+                                                     float *FT) {
+    __shared__ float tile[64][65];
+    const int tx = threadIdx.x & 63, ty = threadIdx.x >> 6;  // 64 x 4
+    const int tr = (rows + 63) / 64, tc = (r + 63) / 64;
+    for (long long b = blockIdx.x; b < (long long)tr * tc; b += gridDim.x) {
+        const int i0 = (int)(b / tc) * 64, j0 = (int)(b % tc) * 64;
+#pragma unroll 4
+        for (int k = ty; k < 64; k += 4) {
+            const int i = i0 + k, j = j0 + tx;
+            if (i < rows && j < r) {
+                const float w = sc[i] * sgn(Lat[(size_t)i * r + j]);
+                F[(size_t)i * ld + c0 + j] = w;
+                tile[k][tx] = w;
+            }
         }
+        __syncthreads();
+#pragma unroll 4
+        for (int k = ty; k < 64; k += 4) {
+            const int j = j0 + k, i = i0 + tx;
+            if (i < rows && j < r) FT[(size_t)(c0 + j) * ldt + i] = tile[tx][k];
+        }
+        __syncthreads();
     }
 }
 
 // dst = src ([rows][cols] at lds) or its transpose ([cols][rows]), at ldd.
-// 32 x 32 tiles through shared memory, so both sides move whole rows.
-__global__ void k_copy_t(const float *src, int rows, int cols, long long lds, int transpose,
-                         float *dst, long long ldd) {
-    __shared__ float tile[32][33];
-    const int tr = (rows + 31) / 32, tc = (cols + 31) / 32;
+// 64 x 64 tiles through shared memory, so both sides move whole rows.
+__global__ void __launch_bounds__(256) k_copy_t(const float *src, int rows, int cols,
+                                                 long long lds, int transpose, float *dst,
+                                                 long long ldd) {
+    __shared__ float tile[64][65];
+    const int tx = threadIdx.x & 63, ty = threadIdx.x >> 6;  // 64 x 4
+    const int tr = (rows + 63) / 64, tc = (cols + 63) / 64;
     for (long long b = blockIdx.x; b < (long long)tr * tc; b += gridDim.x) {
-        const int r0 = (int)(b / tc) * 32, c0 = (int)(b % tc) * 32;
-        for (int k = threadIdx.y; k < 32; k += blockDim.y) {
-            const int r = r0 + k, c = c0 + threadIdx.x;
-            if (r < rows && c < cols) tile[k][threadIdx.x] = src[(size_t)r * lds + c];
+        const int r0 = (int)(b / tc) * 64, c0 = (int)(b % tc) * 64;
+#pragma unroll 4
+        for (int k = ty; k < 64; k += 4) {
+            const int rr = r0 + k, c = c0 + tx;
+            if (rr < rows && c < cols) tile[k][tx] = src[(size_t)rr * lds + c];
         }
         __syncthreads();
-        for (int k = threadIdx.y; k < 32; k += blockDim.y) {
+#pragma unroll 4
+        for (int k = ty; k < 64; k += 4) {
             if (transpose) {
-                const int c = c0 + k, r = r0 + threadIdx.x;
-                if (r < rows && c < cols) dst[(size_t)c * ldd + r] = tile[threadIdx.x][k];
+                const int c = c0 + k, rr = r0 + tx;
+                if (rr < rows && c < cols) dst[(size_t)c * ldd + rr] = tile[tx][k];
             } else {
-                const int r = r0 + k, c = c0 + threadIdx.x;
-                if (r < rows && c < cols) dst[(size_t)r * ldd + c] = tile[k][threadIdx.x];
+                const int rr = r0 + k, c = c0 + tx;
+                if (rr < rows && c < cols) dst[(size_t)rr * ldd + c] = tile[k][tx];
             }
         }
         __syncthreads();
     }
 }
 
-// z[t][j] (at ld_z) = t[t][j] l_j, t dense [T][r].
-__global__ void k_scale_cols(const float *t, const float *l, long long T, int r, float *z,
-                             int ld_z) {
-    const long long n = T * r;
-    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < n;
-         idx += (long long)gridDim.x * blockDim.x) {
-        const long long row = idx / r;
-        const int j = (int)(idx - row * r);
-        z[(size_t)row * ld_z + j] = t[idx] * l[j];
-    }
-}
-
-// One warp per row of M (rows x r): out_row[row] = sum_j S(lat_rj) M_rj and
-// grad[row][j] = scale_row M_rj k (1 - tanh^2(k lat_rj)).
-__global__ void k_grad_rows(const float *M, const float *lat, const float *scale, int rows, int r,
-                            float k, float *out_row, float *grad) {
+// One warp per row of M's columns [c0, c0 + r) (M: rows x R, dense): the
+// path's out_row[row] = sum_j S(lat_rj) M_r,c0+j and grad[row][j] = scale_row
+// M_r,c0+j k (1 - tanh^2(k lat_rj)) (lat, grad: rows x r).  Four columns per
+// lane in flight.
+__global__ void __launch_bounds__(256) k_grad_rows(const float *M, int R, int c0,
+                                                   const float *lat, const float *scale, int rows,
+                                                   int r, float k, float *out_row, float *grad) {
     const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5, lane = threadIdx.x & 31;
     const int nw = (gridDim.x * blockDim.x) >> 5;
     for (int row = warp; row < rows; row += nw) {
         const float sc = scale[row];
+        const float *Mr = M + (size_t)row * R + c0;
+        const float *Lr = lat + (size_t)row * r;
+        float *Gr = grad + (size_t)row * r;
         float acc = 0.f;
+#pragma unroll 4
         for (int j = lane; j < r; j += 32) {
-            const size_t e = (size_t)row * r + j;
-            const float m = M[e], x = lat[e];
+            const float m = Mr[j], x = Lr[j];
             acc += sgn(x) * m;
             const float th = tanhf(k * x);
-            grad[e] = sc * m * k * (1.f - th * th);
+            Gr[j] = sc * m * k * (1.f - th * th);
         }
         for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
         if (lane == 0) out_row[row] = acc;
     }
 }
 
-// dl_j = sum_t dz[t][j] t[t][j] (fp32 partials added with red.add into dl,
-// zeroed by the caller), then dz <- dz . l in place.  Threads walk the T x r
-// elements; each block adds its column partials once.
-__global__ void k_dl_dt(float *dz, const float *t, const float *l, int T, int r, float *dl) {
-    extern __shared__ float s_part[];  // [r]
-    for (int j = threadIdx.x; j < r; j += blockDim.x) s_part[j] = 0.f;
-    __syncthreads();
-    const long long n = (long long)T * r;
-    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < n;
-         idx += (long long)gridDim.x * blockDim.x) {
-        const int j = (int)(idx % r);
-        const float d = dz[idx];
-        atomicAdd(&s_part[j], d * t[idx]);
-        dz[idx] = d * l[j];
-    }
-    __syncthreads();
-    for (int j = threadIdx.x; j < r; j += blockDim.x) red_add_f32(dl + j, s_part[j]);
+// dl_j = sum_t dz[t][j] t[t][j] over the concatenated columns: thread j of a
+// block sums its column over the block's run of rows in a register and adds
+// it to dl (zeroed by the caller) once.
+__global__ void __launch_bounds__(256) k_dl(const float *dz, const float *t, int T, int R,
+                                            int rows_per, float *dl) {
+    const int j = blockIdx.x * 256 + threadIdx.x;
+    if (j >= R) return;
+    const int t0 = blockIdx.y * rows_per, t1 = min(T, t0 + rows_per);
+    float acc = 0.f;
+#pragma unroll 4
+    for (int q = t0; q < t1; ++q) acc += dz[(size_t)q * R + j] * t[(size_t)q * R + j];
+    red_add_f32(dl + j, acc);
 }
 
 int blocks_for(long long n) { return (int)std::min<long long>((n + 255) / 256, 152 * 8); }
 long long pad4(long long n) { return (n + 3) & ~3LL; }
 
-// Workspace carve-up (sizes in floats, each buffer 256-byte aligned).
+// Workspace carve-up (each buffer 256-byte aligned).  R = the paths' ranks
+// concatenated (Eq. 6 sums the paths, so both GEMMs of a product take the
+// paths side by side: the path sum is their K dimension, or their outputs
+// sit side by side).
 struct QatBuf {
     unsigned *err;
-    float *Uh, *UhT, *Vg, *VgT, *t, *z, *zT, *dz, *dtp, *dtT, *dYz, *XTdt, *XT, *dYT, *Xp, *dYp,
-        *part;
+    float *Uh, *UhT, *Vg, *VgT, *lc, *dlc, *t, *z, *zT, *dz, *dt, *dtT, *dYz, *XTdt, *XT, *dYT,
+        *Xp, *dYp, *part;
     size_t part_floats;
-    int ldr, ldo, ldi, ldT;
+    int R, ldr, ldo, ldi, ldT;
 };
 
 struct Carver {
@@ -158,56 +162,59 @@ struct Carver {
     }
 };
 
-QatBuf carve(void *ws, int d_in, int d_out, int rmax, long long T, size_t *bytes) {
+QatBuf carve(void *ws, int d_in, int d_out, int R, long long T, size_t *bytes) {
     QatBuf b{};
     Carver c{static_cast<char *>(ws)};
     c.total = kWsHeader;
     b.err = ws ? static_cast<unsigned *>(ws) + kErrWord : nullptr;
-    b.ldr = (int)pad4(rmax);
+    b.R = R;
+    b.ldr = (int)pad4(R);
     b.ldo = (int)pad4(d_out);
     b.ldi = (int)pad4(d_in);
     b.ldT = (int)pad4(T);
     b.Uh = c.take((size_t)d_out * b.ldr);
-    b.UhT = c.take((size_t)rmax * b.ldo);
+    b.UhT = c.take((size_t)R * b.ldo);
     b.Vg = c.take((size_t)d_in * b.ldr);
-    b.VgT = c.take((size_t)rmax * b.ldi);
-    b.t = c.take((size_t)T * rmax);
+    b.VgT = c.take((size_t)R * b.ldi);
+    b.lc = c.take((size_t)R);
+    b.dlc = c.take((size_t)R);
+    b.t = c.take((size_t)T * R);
     b.z = c.take((size_t)T * b.ldr);
-    b.zT = c.take((size_t)rmax * b.ldT);
-    b.dz = c.take((size_t)T * rmax);
-    b.dtp = c.take((size_t)T * b.ldr);
-    b.dtT = c.take((size_t)rmax * b.ldT);
-    b.dYz = c.take((size_t)d_out * rmax);
-    b.XTdt = c.take((size_t)d_in * rmax);
+    b.zT = c.take((size_t)R * b.ldT);
+    b.dz = c.take((size_t)T * R);
+    b.dt = c.take((size_t)T * b.ldr);
+    b.dtT = c.take((size_t)R * b.ldT);
+    b.dYz = c.take((size_t)d_out * R);
+    b.XTdt = c.take((size_t)d_in * R);
     b.XT = c.take((size_t)d_in * b.ldT);
     b.dYT = c.take((size_t)d_out * b.ldT);
     b.Xp = c.take(d_in % 4 ? (size_t)T * b.ldi : 0);
     b.dYp = c.take(d_out % 4 ? (size_t)T * b.ldo : 0);
-    // split-K partials of the largest product (ranks up to rmax)
-    const int Ti = (int)T, r = rmax;
+    // split-K partials of the largest product
+    const int Ti = (int)T;
     size_t pf = 0;
-    pf = std::max(pf, gemm_part_floats(Ti, r, d_in));   // t = X Vg
-    pf = std::max(pf, gemm_part_floats(Ti, d_out, r));  // Y = z Uh^T
-    pf = std::max(pf, gemm_part_floats(d_out, r, Ti));  // dY^T z
-    pf = std::max(pf, gemm_part_floats(Ti, r, d_out));  // dY Uh
-    pf = std::max(pf, gemm_part_floats(d_in, r, Ti));   // X^T dt
-    pf = std::max(pf, gemm_part_floats(Ti, d_in, r));   // dt Vg^T
+    pf = std::max(pf, gemm_part_floats(Ti, R, d_in));   // t = X Vg
+    pf = std::max(pf, gemm_part_floats(Ti, d_out, R));  // Y = z Uh^T
+    pf = std::max(pf, gemm_part_floats(d_out, R, Ti));  // dY^T z
+    pf = std::max(pf, gemm_part_floats(Ti, R, d_out));  // dY Uh
+    pf = std::max(pf, gemm_part_floats(d_in, R, Ti));   // X^T dt
+    pf = std::max(pf, gemm_part_floats(Ti, d_in, R));   // dt Vg^T
     b.part = c.take(pf);
     b.part_floats = pf;
     if (bytes) *bytes = c.total + 256;
     return b;
 }
 
-int rmax_of(const lb_train_linear &L) {
+int rsum_of(const lb_train_linear &L) {
     int r = 0;
-    for (int p = 0; p < L.n_paths; ++p) r = std::max(r, (int)L.path[p].r);
+    for (int p = 0; p < L.n_paths; ++p) r += (int)L.path[p].r;
     return r;
 }
 
 cudaError_t copy_t(const float *src, int rows, int cols, long long lds, bool transpose, float *dst,
                    long long ldd, cudaStream_t s) {
-    const long long tiles = (long long)((rows + 31) / 32) * ((cols + 31) / 32);
-    k_copy_t<<<(int)std::min<long long>(tiles, 152 * 16), dim3(32, 8), 0, s>>>(
+    const long long tiles = (long long)((rows + 63) / 64) * ((cols + 63) / 64);
+    k_copy_t<<<(int)std::min<long long>(tiles, 152 * 8), 256, 0, s>>>(
         src, rows, cols, lds, transpose ? 1 : 0, dst, ldd);
     return cudaGetLastError();
 }
@@ -224,93 +231,101 @@ cudaError_t k_major(const float *a, int rows, int cols, float *pad, int ldp, Gem
     return copy_t(a, rows, cols, cols, false, pad, ldp, s);
 }
 
-// The per-path forward products: t = X Vg, z = t . l, Y (+)= z Uh^T.
-cudaError_t path_forward(const lb_train_linear &L, const lb_train_path &P, const GemmOperand &Xk,
-                         long long T, float *y, bool accumulate, const QatBuf &b, cudaStream_t s) {
-    const int r = P.r;
-    k_fold_signs<<<blocks_for((long long)(L.d_out + L.d_in) * r), 256, 0, s>>>(
-        P.u, P.v, P.h, P.g, L.d_out, L.d_in, r, b.ldr, b.ldo, b.ldi, b.Uh, b.UhT, b.Vg, b.VgT);
-    cudaError_t e = gemm_tf32(Xk, GemmOperand{b.VgT, r, L.d_in, b.ldi}, b.t, r, false, b.part,
-                              b.part_floats, b.err, s);
-    if (e != cudaSuccess) return e;
-    k_scale_cols<<<blocks_for(T * r), 256, 0, s>>>(b.t, P.l, T, r, b.z, b.ldr);
-    if (!y) return cudaGetLastError();
-    return gemm_tf32(GemmOperand{b.z, (int)T, r, b.ldr}, GemmOperand{b.Uh, L.d_out, r, b.ldr}, y,
-                     L.d_out, accumulate, b.part, b.part_floats, b.err, s);
+// The sign folds of every path side by side (Uh and UhT, Vg and VgT) and the
+// concatenated l; then t = X Vg and z = t . l.
+cudaError_t forward_latent(const lb_train_linear &L, const GemmOperand &Xk, long long T,
+                           const QatBuf &b, cudaStream_t s) {
+    int c0 = 0;
+    cudaError_t e = cudaSuccess;
+    for (int p = 0; p < L.n_paths && e == cudaSuccess; ++p) {
+        const lb_train_path &P = L.path[p];
+        const int tu = ((L.d_out + 63) / 64) * ((P.r + 63) / 64);
+        const int tv = ((L.d_in + 63) / 64) * ((P.r + 63) / 64);
+        k_fold_signs<<<std::min(tu, 152 * 8), 256, 0, s>>>(P.u, P.h, L.d_out, P.r, c0, b.ldr,
+                                                           b.ldo, b.Uh, b.UhT);
+        k_fold_signs<<<std::min(tv, 152 * 8), 256, 0, s>>>(P.v, P.g, L.d_in, P.r, c0, b.ldr,
+                                                           b.ldi, b.Vg, b.VgT);
+        e = cudaMemcpyAsync(b.lc + c0, P.l, (size_t)P.r * sizeof(float), cudaMemcpyDeviceToDevice,
+                            s);
+        c0 += P.r;
+    }
+    // t = X Vg, and z = t . l beside it
+    if (e == cudaSuccess)
+        e = gemm_tf32(Xk, GemmOperand{b.VgT, b.R, L.d_in, b.ldi}, b.t, b.R, false, b.part,
+                      b.part_floats, b.err, s, b.z, b.lc, b.ldr);
+    return e;
 }
 
 }  // namespace
 
-size_t qat_ws_bytes(int d_in, int d_out, int rmax, long long T) {
+size_t qat_ws_bytes(int d_in, int d_out, int rsum, long long T) {
     size_t bytes = 0;
-    carve(nullptr, d_in, d_out, rmax, T, &bytes);
+    carve(nullptr, d_in, d_out, rsum, T, &bytes);
     return bytes;
 }
 
 cudaError_t launch_train_forward(const lb_train_linear &L, const float *x, long long T, float *y,
                                  void *ws, cudaStream_t s) {
-    QatBuf b = carve(ws, L.d_in, L.d_out, rmax_of(L), T, nullptr);
+    QatBuf b = carve(ws, L.d_in, L.d_out, rsum_of(L), T, nullptr);
     cudaError_t e = cudaMemsetAsync(b.err, 0, sizeof(unsigned), s);
     GemmOperand Xk;
     if (e == cudaSuccess) e = k_major(x, (int)T, L.d_in, b.Xp, b.ldi, &Xk, s);
-    for (int p = 0; p < L.n_paths && e == cudaSuccess; ++p)
-        e = path_forward(L, L.path[p], Xk, T, y, p > 0, b, s);
+    if (e == cudaSuccess) e = forward_latent(L, Xk, T, b, s);
+    // Y = z Uh^T: both paths in one product (Eq. 6's sum is its K dimension)
+    if (e == cudaSuccess)
+        e = gemm_tf32(GemmOperand{b.z, (int)T, b.R, b.ldr}, GemmOperand{b.Uh, L.d_out, b.R, b.ldr},
+                      y, L.d_out, false, b.part, b.part_floats, b.err, s);
     return e;
 }
 
 cudaError_t launch_train_backward(const lb_train_linear &L, const float *x, const float *dy,
                                   long long T, float k, const lb_train_grad *G, float *dx, void *ws,
                                   cudaStream_t s) {
-    QatBuf b = carve(ws, L.d_in, L.d_out, rmax_of(L), T, nullptr);
-    const int Ti = (int)T;
+    QatBuf b = carve(ws, L.d_in, L.d_out, rsum_of(L), T, nullptr);
+    const int Ti = (int)T, R = b.R;
     cudaError_t e = cudaMemsetAsync(b.err, 0, sizeof(unsigned), s);
-    // the forward's operand, and the token-major copies of X and dY
+    // the forward's operand, the token-major copies of X and dY, t and z
     GemmOperand Xk, dYk;
     if (e == cudaSuccess) e = k_major(x, Ti, L.d_in, b.Xp, b.ldi, &Xk, s);
     if (e == cudaSuccess) e = k_major(dy, Ti, L.d_out, b.dYp, b.ldo, &dYk, s);
     if (e == cudaSuccess) e = copy_t(x, Ti, L.d_in, L.d_in, true, b.XT, b.ldT, s);
     if (e == cudaSuccess) e = copy_t(dy, Ti, L.d_out, L.d_out, true, b.dYT, b.ldT, s);
-    for (int p = 0; p < L.n_paths && e == cudaSuccess; ++p) {
-        const lb_train_path &P = L.path[p];
-        const lb_train_grad &D = G[p];
-        const int r = P.r;
-        // forward intermediates t = X Vg, z = t . l (and the fold of this path)
-        e = path_forward(L, P, Xk, T, nullptr, false, b, s);
-        // dYz = dY^T z -> dh, dU
-        if (e == cudaSuccess) e = copy_t(b.z, Ti, r, b.ldr, true, b.zT, b.ldT, s);
-        if (e == cudaSuccess)
-            e = gemm_tf32(GemmOperand{b.dYT, L.d_out, Ti, b.ldT}, GemmOperand{b.zT, r, Ti, b.ldT},
-                          b.dYz, r, false, b.part, b.part_floats, b.err, s);
-        if (e != cudaSuccess) break;
-        k_grad_rows<<<blocks_for((long long)L.d_out * 32), 256, 0, s>>>(b.dYz, P.u, P.h, L.d_out,
-                                                                        r, k, D.dh, D.du);
-        // dz = dY Uh -> dl, dt (in dz)
-        e = gemm_tf32(dYk, GemmOperand{b.UhT, r, L.d_out, b.ldo}, b.dz, r, false, b.part,
-                      b.part_floats, b.err, s);
-        if (e == cudaSuccess) e = cudaMemsetAsync(D.dl, 0, (size_t)r * sizeof(float), s);
-        if (e != cudaSuccess) break;
-        k_dl_dt<<<blocks_for(T * r), 256, (size_t)r * sizeof(float), s>>>(b.dz, b.t, P.l, Ti, r,
-                                                                           D.dl);
-        // XTdt = X^T dt -> dg, dV
-        e = copy_t(b.dz, Ti, r, r, true, b.dtT, b.ldT, s);
-        if (e == cudaSuccess)
-            e = gemm_tf32(GemmOperand{b.XT, L.d_in, Ti, b.ldT}, GemmOperand{b.dtT, r, Ti, b.ldT},
-                          b.XTdt, r, false, b.part, b.part_floats, b.err, s);
-        if (e != cudaSuccess) break;
-        k_grad_rows<<<blocks_for((long long)L.d_in * 32), 256, 0, s>>>(b.XTdt, P.v, P.g, L.d_in,
-                                                                       r, k, D.dg, D.dv);
-        // dX (+)= dt Vg^T
-        if (dx) {
-            GemmOperand dtk{b.dz, Ti, r, r};
-            if (r % 4 != 0) {
-                e = copy_t(b.dz, Ti, r, r, false, b.dtp, b.ldr, s);
-                dtk = GemmOperand{b.dtp, Ti, r, b.ldr};
-            }
-            if (e == cudaSuccess)
-                e = gemm_tf32(dtk, GemmOperand{b.Vg, L.d_in, r, b.ldr}, dx, L.d_in, p > 0, b.part,
-                              b.part_floats, b.err, s);
-        }
+    if (e == cudaSuccess) e = forward_latent(L, Xk, T, b, s);
+    // dYz = dY^T z -> dh, dU per path
+    if (e == cudaSuccess) e = copy_t(b.z, Ti, R, b.ldr, true, b.zT, b.ldT, s);
+    if (e == cudaSuccess)
+        e = gemm_tf32(GemmOperand{b.dYT, L.d_out, Ti, b.ldT}, GemmOperand{b.zT, R, Ti, b.ldT},
+                      b.dYz, R, false, b.part, b.part_floats, b.err, s);
+    if (e != cudaSuccess) return e;
+    for (int p = 0, c0 = 0; p < L.n_paths; c0 += L.path[p].r, ++p)
+        k_grad_rows<<<blocks_for((long long)L.d_out * 32), 256, 0, s>>>(
+            b.dYz, R, c0, L.path[p].u, L.path[p].h, L.d_out, L.path[p].r, k, G[p].dh, G[p].du);
+    // dz = dY Uh and dt = dz . l beside it -> dl
+    e = gemm_tf32(dYk, GemmOperand{b.UhT, R, L.d_out, b.ldo}, b.dz, R, false, b.part,
+                  b.part_floats, b.err, s, b.dt, b.lc, b.ldr);
+    if (e == cudaSuccess) e = cudaMemsetAsync(b.dlc, 0, (size_t)R * sizeof(float), s);
+    if (e != cudaSuccess) return e;
+    {
+        const int rows_per = 64;
+        k_dl<<<dim3((R + 255) / 256, (Ti + rows_per - 1) / rows_per), 256, 0, s>>>(
+            b.dz, b.t, Ti, R, rows_per, b.dlc);
     }
+    for (int p = 0, c0 = 0; p < L.n_paths && e == cudaSuccess; c0 += L.path[p].r, ++p)
+        e = cudaMemcpyAsync(G[p].dl, b.dlc + c0, (size_t)L.path[p].r * sizeof(float),
+                            cudaMemcpyDeviceToDevice, s);
+    // XTdt = X^T dt -> dg, dV per path
+    if (e == cudaSuccess) e = copy_t(b.dt, Ti, R, b.ldr, true, b.dtT, b.ldT, s);
+    if (e == cudaSuccess)
+        e = gemm_tf32(GemmOperand{b.XT, L.d_in, Ti, b.ldT}, GemmOperand{b.dtT, R, Ti, b.ldT},
+                      b.XTdt, R, false, b.part, b.part_floats, b.err, s);
+    if (e != cudaSuccess) return e;
+    for (int p = 0, c0 = 0; p < L.n_paths; c0 += L.path[p].r, ++p)
+        k_grad_rows<<<blocks_for((long long)L.d_in * 32), 256, 0, s>>>(
+            b.XTdt, R, c0, L.path[p].v, L.path[p].g, L.d_in, L.path[p].r, k, G[p].dg, G[p].dv);
+    // dX = dt Vg^T: both paths in one product
+    if (dx)
+        e = gemm_tf32(GemmOperand{b.dt, Ti, R, b.ldr}, GemmOperand{b.Vg, L.d_in, R, b.ldr}, dx,
+                      L.d_in, false, b.part, b.part_floats, b.err, s);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
