@@ -183,7 +183,7 @@ class ClockSampler:
 
 def kernel_source_sha() -> str:
     h = hashlib.sha256()
-    for f in ("lb_stack.cu", "lb_common.cuh"):
+    for f in ("lb_stack.cu", "lb_common.cuh", "lb_lut.cuh"):
         with open(os.path.join(ROOT, "paper_2506_13771_gb300", "csrc", f), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]

@@ -58,6 +58,13 @@ __device__ __forceinline__ unsigned cluster_rank() {
     return r;
 }
 
+// CTAs in this CTA's cluster (1 when the launch formed no clusters).
+__device__ __forceinline__ unsigned cluster_size() {
+    unsigned n;
+    asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(n));
+    return n;
+}
+
 // The shared::cluster address of byte offset `local` (a shared::cta address)
 // in the CTA of rank `rank` of this cluster.
 __device__ __forceinline__ uint32_t mapa(uint32_t local, unsigned rank) {

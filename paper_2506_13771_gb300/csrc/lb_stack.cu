@@ -728,6 +728,13 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         if (blockIdx.x == 0 && threadIdx.x == 0) record(P.ws_words, LB_ERR_PLAN);
         return;
     }
+    // the partials of a cluster meet in its CTAs' shared memory: a launch
+    // that did not form clusters of kCluster CTAs (the per-CTA programs
+    // assume them) records an error and touches no other CTA's memory
+    if (kCluster > 1 && cluster_size() != (unsigned)kCluster) {
+        if (threadIdx.x == 0) record(P.ws_words, LB_ERR_UNSUPPORTED);
+        return;
+    }
     const int N = gridDim.x, c = blockIdx.x;
     const unsigned n_ctas = (unsigned)N, n_t = P.n_t;
     const unsigned rank = kCluster > 1 ? cluster_rank() : 0u;

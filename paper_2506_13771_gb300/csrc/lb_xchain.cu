@@ -45,6 +45,11 @@ __global__ void __launch_bounds__(kXT, 1) k_xchain(const __grid_constant__ Xchai
     __shared__ float slot[kXMaxUnits / 2][32];
     unsigned *ws = P.ws_words;
     if (xc_sticky(ws)) return;
+    if (C > 1 && cluster_size() != (unsigned)C) {
+        // not launched in clusters of C: no other CTA's memory is touched
+        if (threadIdx.x == 0) atomicCAS(ws + kErrWord, 0u, static_cast<unsigned>(LB_ERR_UNSUPPORTED));
+        return;
+    }
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const unsigned rank = C > 1 ? cluster_rank() : 0u;
     if (threadIdx.x == 0) {
