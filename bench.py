@@ -671,7 +671,7 @@ def run_config(args):
             sig = (1.0 + torch.arange(k0, device=dev, dtype=torch.float32)) ** -0.6
             W = (A * sig) @ B.t() + 1e-3 * torch.randn((m, n), generator=g, device=dev) / n ** 0.5
             del A, B
-            lb.dual_svid(W, [r, r], iters=8)  # warm-up (cuBLAS handle, workspace)
+            lb.dual_svid(W, [r, r], iters=8)  # warm-up (workspace, first launches)
             torch.cuda.synchronize(dev)
             ts = []
             for _ in range(max(1, min(steps, 3))):

@@ -194,8 +194,9 @@ size_t littlebit_dual_svid_workspace_size(int32_t d_out, int32_t d_in, int32_t n
  * truncated SVD when the r-th and (r + 9)-th singular values are apart.
  * W: DEVICE fp32 row-major [d_out][d_in]; paths: HOST array of n_paths
  * (1 or 2) output descriptors.  ws: littlebit_dual_svid_workspace_size
- * bytes, 256-byte aligned (no zero fill needed).  Uses cuBLAS for its GEMMs
- * on the given stream.  Errors: LB_ERR_INVALID_ARG (shapes, ranks,
+ * bytes, 256-byte aligned (no zero fill needed).  Its GEMMs are the
+ * library's own fp32 / fp64 CUDA-core GEMM (full-precision products) on the
+ * given stream; the library keeps no handle.  Errors: LB_ERR_INVALID_ARG (shapes, ranks,
  * pointers), LB_ERR_WORKSPACE, LB_ERR_CUDA. */
 lb_status littlebit_dual_svid(const float *W, int32_t d_out, int32_t d_in, int32_t n_paths,
                               const lb_path_init *paths, int32_t iters, void *ws, size_t ws_bytes,

@@ -19,7 +19,8 @@ LIB = os.path.join(BUILD, "liblittlebit.so")
 
 SOURCES = ["lb_api.cu", "lb_generic.cu", "lb_persistent.cu", "lb_stack.cu", "lb_pack.cu",
            "lb_noalloc.cu", "lb_prefill.cu", "lb_decode.cu", "lb_svid.cu",
-           "lb_qat.cu", "lb_decoder.cu", "lb_multi.cu", "lb_xchain.cu", "lb_gemm.cu"]
+           "lb_qat.cu", "lb_decoder.cu", "lb_multi.cu", "lb_xchain.cu", "lb_gemm.cu",
+           "lb_simt_gemm.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2",
                      "--cudart", "shared", "-I", INCLUDE, "-I", CSRC]
@@ -65,7 +66,7 @@ def build(force: bool = False, verbose: bool = False, extra_flags: list[str] | N
     with ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
         objs = list(ex.map(compile_one, SOURCES))
     tmp = LIB + f".tmp{os.getpid()}"
-    cmd = [nvcc] + ARCH + ["-shared", "--cudart", "shared", "-o", tmp] + objs + ["-lcublas"]
+    cmd = [nvcc] + ARCH + ["-shared", "--cudart", "shared", "-o", tmp] + objs
     res = subprocess.run(cmd, capture_output=True, text=True)
     if res.returncode != 0:
         raise RuntimeError(f"link failed:\n{res.stdout}\n{res.stderr}")

@@ -7,13 +7,7 @@
 
 #include "littlebit.h"
 
-struct cublasContext;
-
 namespace lb {
-
-// The library's cuBLAS handle for the current device (created on first use,
-// one per device, shared by the calls that run plain GEMMs).
-cublasContext *blas_handle();
 
 struct LinDesc;
 
@@ -91,6 +85,16 @@ cudaError_t launch_prefill_latent(const lb_linear &L, const uint16_t *x, int64_t
                                   float *z32, unsigned *ws_words, void *ws, cudaStream_t s);
 cudaError_t launch_prefill_expand(const lb_linear &L, const uint16_t *z16, int64_t T, void *y,
                                   int y_fp32, unsigned *ws_words, void *ws, cudaStream_t s);
+
+// Column-major C = alpha op(A) op(B) + beta C on the CUDA cores, fp32 or fp64
+// (lb_simt_gemm.cu): op(A) M x K is A[m + k lda] or, with ta, A[k + m lda];
+// op(B) K x N likewise; beta = 0 does not read C.
+cudaError_t gemm_simt(bool ta, bool tb, int M, int N, int K, float alpha, const float *A,
+                      long long lda, const float *B, long long ldb, float beta, float *C,
+                      long long ldc, cudaStream_t s);
+cudaError_t gemm_simt(bool ta, bool tb, int M, int N, int K, double alpha, const double *A,
+                      long long lda, const double *B, long long ldb, double beta, double *C,
+                      long long ldc, cudaStream_t s);
 
 // Dual-SVID initialisation (lb_svid.cu): W fp32 row-major [d_out][d_in],
 // per path the output sign words and fp16 scales; ws: svid_ws_bytes.

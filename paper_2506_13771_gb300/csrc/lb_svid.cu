@@ -17,13 +17,12 @@
 //   (3) |U'| ~ h l_u^T, |V'| ~ g l_v^T, the leading singular pair of each
 //       nonnegative matrix by power iteration (fp64, 50 steps), the singular value split
 //       evenly; l = l_u . l_v.  h, g, l are rounded to fp16 (nearest even).
-// The GEMMs are cuBLAS (plain fp32 / fp64 GEMMs); the Cholesky factor of
+// The GEMMs are the library's CUDA-core GEMM (lb_simt_gemm.cu: fp32 / fp64
+// FMA, column-major like the matrices here); the Cholesky factor of
 // a k x k Gram matrix and the triangular solve with it are blocked (64-wide
 // diagonal blocks in one CTA each, rows below by many CTAs, updates by GEMM);
 // the k x k Jacobi SVD runs in one CTA; the rest are elementwise / reduction
 // kernels below.
-#include <cublas_v2.h>
-
 #include <algorithm>
 #include <cmath>
 #include <mutex>
@@ -445,7 +444,7 @@ __global__ void k_what_factors(const float *U, const float *V, int d_out, int d_
     }
 }
 
-// ---------------------------------------------------------------- cuBLAS
+// ---------------------------------------------------------------- the driver
 
 int grid_for(long long n) { return (int)std::min<long long>((n + 255) / 256, 152 * 8); }
 
@@ -461,17 +460,6 @@ struct Buf {
 };
 
 }  // namespace
-
-static std::mutex g_blas_mu;
-static cublasHandle_t g_blas[64];
-
-cublasHandle_t blas_handle() {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-    std::lock_guard<std::mutex> lock(g_blas_mu);
-    if (!g_blas[dev] && cublasCreate(&g_blas[dev]) != CUBLAS_STATUS_SUCCESS) g_blas[dev] = nullptr;
-    return g_blas[dev];
-}
 
 int svid_k(int r, int d_out, int d_in) { return std::min(r + kOversample, std::min(d_out, d_in)); }
 
@@ -501,10 +489,6 @@ cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, c
                              uint32_t *const *v_bits, uint32_t *const *u_bits, uint16_t *const *g,
                              uint16_t *const *l, uint16_t *const *h, int iters, void *ws,
                              cudaStream_t s) {
-    cublasHandle_t H = blas_handle();
-    if (!H) return cudaErrorNotSupported;
-    if (cublasSetStream(H, s) != CUBLAS_STATUS_SUCCESS) return cudaErrorUnknown;
-    cublasSetPointerMode(H, CUBLAS_POINTER_MODE_HOST);
     const int m = d_out, n = d_in;
     int kmax = 0;
     for (int p = 0; p < n_paths; ++p) kmax = std::max(kmax, svid_k(ranks[p], d_out, d_in));
@@ -530,11 +514,13 @@ cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, c
     (void)G32;
     const double done = 1.0, dzero = 0.0;
     bool blas_ok = true;
-    auto gemm = [&](cublasOperation_t ta, cublasOperation_t tb, int mm, int nn, int kk,
-                    const float *A, int lda, const float *B, int ldb, const float *beta, float *C,
-                    int ldc, const float *alpha) {
-        blas_ok = blas_ok && cublasSgemm(H, ta, tb, mm, nn, kk, alpha, A, lda, B, ldb, beta, C, ldc) ==
-                                 CUBLAS_STATUS_SUCCESS;
+    constexpr bool N_ = false, T_ = true;  // op(X) = X, op(X) = X^T
+    auto gemm = [&](bool ta, bool tb, int mm, int nn, int kk, const float *A, int lda,
+                    const float *B, int ldb, const float *beta, float *C, int ldc,
+                    const float *alpha) {
+        blas_ok = blas_ok &&
+                  gemm_simt(ta, tb, mm, nn, kk, *alpha, A, lda, B, ldb, *beta, C, ldc, s) ==
+                      cudaSuccess;
     };
     // blocked Cholesky of the k x k Gram matrix Gm (lower, in place): per
     // 64-wide block, the diagonal block in one CTA, the rows below it by a
@@ -548,12 +534,10 @@ cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, c
             k_potrf_diag<double><<<1, kNB, 0, s>>>(Gm, k, jb, bw, dfloor);
             if (rest > 0) {
                 k_trsm_panel<double><<<(rest + 127) / 128, 128, 0, s>>>(Gm, k, jb, bw);
-                const double dminus = -1.0;
                 blas_ok = blas_ok &&
-                          cublasDgemm(H, CUBLAS_OP_N, CUBLAS_OP_T, rest, rest, bw, &dminus,
-                                      Gm + (size_t)jb * k + jb + bw, k, Gm + (size_t)jb * k + jb + bw,
-                                      k, &done, Gm + (size_t)(jb + bw) * k + jb + bw, k) ==
-                              CUBLAS_STATUS_SUCCESS;
+                          gemm_simt(N_, T_, rest, rest, bw, -1.0, Gm + (size_t)jb * k + jb + bw, k,
+                                    Gm + (size_t)jb * k + jb + bw, k, done,
+                                    Gm + (size_t)(jb + bw) * k + jb + bw, k, s) == cudaSuccess;
             }
         }
     };
@@ -564,7 +548,7 @@ cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, c
             k_potrf_diag<float><<<1, kNB, 0, s>>>(Gm, k, jb, bw, ffloor);
             if (rest > 0) {
                 k_trsm_panel<float><<<(rest + 127) / 128, 128, 0, s>>>(Gm, k, jb, bw);
-                gemm(CUBLAS_OP_N, CUBLAS_OP_T, rest, rest, bw, Gm + (size_t)jb * k + jb + bw, k,
+                gemm(N_, T_, rest, rest, bw, Gm + (size_t)jb * k + jb + bw, k,
                      Gm + (size_t)jb * k + jb + bw, k, &one, Gm + (size_t)(jb + bw) * k + jb + bw,
                      k, &minus);
             }
@@ -575,7 +559,7 @@ cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, c
         for (int jb = 0; jb < k; jb += kNB) {
             const int bw = std::min(kNB, k - jb);
             if (jb > 0)
-                gemm(CUBLAS_OP_N, CUBLAS_OP_T, rows, bw, jb, X, rows, L32 + jb, k, &one,
+                gemm(N_, T_, rows, bw, jb, X, rows, L32 + jb, k, &one,
                      X + (size_t)jb * rows, rows, &minus);
             k_trsm_cols<<<(rows + 127) / 128, 128, 0, s>>>(X, rows, L32, k, jb, bw);
         }
@@ -586,12 +570,13 @@ cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, c
     // result
     auto orth = [&](float *X, float *, int rows, int k) {
         k_to_f64<<<grid_for((long long)rows * k), 256, 0, s>>>(X, D, (long long)rows * k);
-        blas_ok = blas_ok && cublasDgemm(H, CUBLAS_OP_T, CUBLAS_OP_N, k, k, rows, &done, D, rows, D,
-                                         rows, &dzero, G, k) == CUBLAS_STATUS_SUCCESS;
+        blas_ok = blas_ok &&
+                  gemm_simt(T_, N_, k, k, rows, done, D, rows, D, rows, dzero, G, k, s) ==
+                      cudaSuccess;
         chol64(G, k);
         k_lower_f32<double><<<grid_for((long long)k * k), 256, 0, s>>>(G, k, Lt, 0);
         trsm_right(X, rows, Lt, k);
-        gemm(CUBLAS_OP_T, CUBLAS_OP_N, k, k, rows, X, rows, X, rows, &zero, G32, k, &one);
+        gemm(T_, N_, k, k, rows, X, rows, X, rows, &zero, G32, k, &one);
         chol32(G32, k);
         k_lower_f32<float><<<grid_for((long long)k * k), 256, 0, s>>>(G32, k, Lt, 0);
         trsm_right(X, rows, Lt, k);
@@ -603,24 +588,24 @@ cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, c
         orth(Q, Q2, n, k);
         for (int it = 0; it < iters; ++it) {
             // Y = R Q  (R is n x m column-major: op T gives m x n)
-            gemm(CUBLAS_OP_T, CUBLAS_OP_N, m, k, n, R, n, Q, n, &zero, Y, m, &one);
+            gemm(T_, N_, m, k, n, R, n, Q, n, &zero, Y, m, &one);
             orth(Y, Y2, m, k);
             // Q = R^T Y
-            gemm(CUBLAS_OP_N, CUBLAS_OP_N, n, k, m, R, n, Y, m, &zero, Q, n, &one);
+            gemm(N_, N_, n, k, m, R, n, Y, m, &zero, Q, n, &one);
             orth(Q, Q2, n, k);
         }
         // Rayleigh-Ritz: B = R Q (in Y); B = Y' L^T with L the Cholesky factor
         // of B^T B (fp64); the SVD of the k x k L^T (one-sided Jacobi) gives
         // B's singular values and right vectors E: V_r = Q E_r, U_r = B E_r / s
-        gemm(CUBLAS_OP_T, CUBLAS_OP_N, m, k, n, R, n, Q, n, &zero, Y, m, &one);
+        gemm(T_, N_, m, k, n, R, n, Q, n, &zero, Y, m, &one);
         k_to_f64<<<grid_for((long long)m * k), 256, 0, s>>>(Y, D, (long long)m * k);
-        blas_ok = blas_ok && cublasDgemm(H, CUBLAS_OP_T, CUBLAS_OP_N, k, k, m, &done, D, m, D, m,
-                                         &dzero, G, k) == CUBLAS_STATUS_SUCCESS;
+        blas_ok = blas_ok &&
+                  gemm_simt(T_, N_, k, k, m, done, D, m, D, m, dzero, G, k, s) == cudaSuccess;
         chol64(G, k);
         k_lower_f32<double><<<grid_for((long long)k * k), 256, 0, s>>>(G, k, G32, 1);
         k_svd_jacobi<<<1, kSmallThreads, 0, s>>>(G32, JV32, k, sv, Lt);
-        gemm(CUBLAS_OP_N, CUBLAS_OP_N, n, r, k, Q, n, Lt, k, &zero, Q2, n, &one);
-        gemm(CUBLAS_OP_N, CUBLAS_OP_N, m, r, k, Y, m, Lt, k, &zero, Y2, m, &one);
+        gemm(N_, N_, n, r, k, Q, n, Lt, k, &zero, Q2, n, &one);
+        gemm(N_, N_, m, r, k, Y, m, Lt, k, &zero, Y2, m, &one);
         k_ritz_scale<<<grid_for((long long)m * r), 256, 0, s>>>(sv, Y2, m, r);
         k_sign_split<<<r, 256, 0, s>>>(Y2, Q2, m, n, sv);
         k_pack_u_cm<<<grid_for((long long)m * ((r + 31) / 32)), 256, 0, s>>>(Y2, m, r, u_bits[p]);
@@ -653,7 +638,7 @@ cudaError_t launch_dual_svid(const float *W, int d_out, int d_in, int n_paths, c
             float *A1 = Y, *B1 = Q;
             k_what_factors<<<grid_for((long long)(m + n) * r), 256, 0, s>>>(Y2, Q2, m, n, r, h[p],
                                                                              g[p], l[p], A1, B1);
-            gemm(CUBLAS_OP_N, CUBLAS_OP_T, n, m, r, B1, n, A1, m, &one, R, n, &minus);
+            gemm(N_, T_, n, m, r, B1, n, A1, m, &one, R, n, &minus);
         }
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
