@@ -264,6 +264,49 @@ __device__ __forceinline__ float dec_fix2(unsigned long long hi, unsigned long l
     return __ll2float_rn(2 * q + sticky) * 0x1p-29f;
 }
 
+// ---------------------------------------------------------------- bounded one-word exchange
+//
+// The stack kernel's exchanges are one 64-bit word per element: the sum of
+// the contributions round(v 2^s) in the high 56 bits, their count in the low
+// 8.  The scale 2^s is chosen per exchange, by every CTA alike, from a bound
+// B on every contribution's magnitude (fix1_scale): n B 2^s < 2^54, so no sum
+// of n contributions can leave the word, and the resolution 2^-s is about
+// 2^-53 n B -- relative to a typical value t, n (B / t) 2^-53, far below fp32
+// rounding for any bound within 2^20 of the values, whatever their scale.
+
+// 2^s and 2^-s with n B 2^s < 2^54 (B >= 0; a zero or non-finite bound gives
+// the scale of B = 1).
+__device__ __forceinline__ float2 fix1_scale(float B, int n) {
+    float x = B * (float)n;
+    if (!(x > 0.f) || !(x < 3.0e38f)) x = (float)n;
+    int e = (int)((__float_as_uint(x) >> 23) & 0xffu) - 127;  // floor(log2 x), x normal
+    int sh = 53 - e;
+    sh = sh > 126 ? 126 : (sh < -126 ? -126 : sh);
+    return make_float2(__uint_as_float((unsigned)(sh + 127) << 23),
+                       __uint_as_float((unsigned)(127 - sh) << 23));
+}
+
+// One contribution v at scale sc (= 2^s); |v sc| must stay below lim = 2^54
+// / n (else LB_ERR_RANGE is recorded and zero sent: the bound was wrong).
+__device__ __forceinline__ void send_fix1(unsigned long long *w, float v, float sc, float lim,
+                                          unsigned *err) {
+    float a = v * sc;
+    if (!(fabsf(a) < lim)) {
+        atomicCAS(err, 0u, static_cast<unsigned>(LB_ERR_RANGE));
+        a = 0.f;
+    }
+    red_add_u64(w, (static_cast<unsigned long long>(__float2ll_rn(a)) << 8) + 1ull);
+}
+
+__device__ __forceinline__ bool counted1(unsigned long long w, unsigned n) {
+    return (unsigned)(w & 0xffull) == n;
+}
+
+// The sum held by a complete word, in fp32 (one rounding), at inverse scale inv.
+__device__ __forceinline__ float dec_fix1(unsigned long long w, float inv) {
+    return __ll2float_rn(static_cast<long long>(w) >> 8) * inv;
+}
+
 // Stores table n of a unit at T from its four values (see run_tables).
 __device__ __forceinline__ void store_table(unsigned char *T, float4 x, int lane) {
 #pragma unroll

@@ -29,18 +29,26 @@
 //    the stage-1 tables of those rows), 32 columns x the slice for stage 1.
 //    The shapes are those of every layer, so the program is the same for all
 //    of them; the device code is a handful of generic loops;
-//  * the all-reduce of t accumulates every element as an exact fixed-point
-//    sum in a pair of 64-bit words whose low 8 bits count contributions
-//    (send_fix2: two red.add per element and CTA) and readers poll the pairs
-//    they need until the count reaches the CTA count -- no fence, no
-//    separate barrier, an order-independent sum, exact for contributions
-//    from 2^-41 to 2^34 / n, so the exchange is equivariant under scaling of
-//    the inputs;
+//  * the all-reduce of t accumulates every element as a fixed-point sum in
+//    one 64-bit word whose low 8 bits count contributions (send_fix1: one
+//    red.add per element and contribution) and readers poll the words they
+//    need until the count is complete -- no fence, no separate barrier, an
+//    order-independent sum.  Its scale is set per exchange, identically in
+//    every CTA, from a rigorous bound on the contributions: |t_j| <= max|g|
+//    x the L1 norm of the stage-1 input, that norm bounded through the
+//    chain's residual adds, attention and SiLU product from per-linear
+//    constants (max|g|, the L1 norm and maximum of |h|, computed once by
+//    littlebit_stack_prepare) and the largest per-unit |z| sum of the tables
+//    each CTA built from the previous exchange (an order-independent max, so
+//    every CTA derives the same scale).  The resolution is then about 2^-53
+//    n B at any input scale, and a contribution beyond twice the bound (a
+//    broken bound) is recorded as LB_ERR_RANGE, never wrapped;
 //  * q and k (not read again at position 0) are computed after the CTA has
 //    sent its share of the next exchange, off the critical path.
 // Every wait is bounded (about one second); on a timeout the CTA records
 // LB_ERR_TIMEOUT, waits for its own bulk copies to land, and returns.
 #include <algorithm>
+#include <cmath>
 #include <cstring>
 #include <mutex>
 #include <vector>
@@ -80,6 +88,8 @@ struct Offsets {
     int c_Uo[2], c_ho[2], c_lo[2], c_Vg[2], c_Vu[2], c_gg[2], c_gu[2];
     // phase D: stage 2 of gate, up, stage 1 of down
     int d_Ug[2], d_Uu[2], d_hg[2], d_hu[2], d_lg[2], d_lu[2], d_Vd[2], d_gd[2];
+    // the phase's two float4 of exchange-bound constants (cst, per layer)
+    int cst[4];
     // work areas: stage-2 and stage-1 tables, residual stream (two buffers:
     // phase A reads 0 and writes 1, phase C the reverse), the off-path q, k, v
     // outputs (added into, zeroed once stored), the sum-of-squares
@@ -104,8 +114,9 @@ enum StepId {
 };
 
 // One program record (8 ints).  Meaning by step kind:
-//   poll-table  : tb, n_tab, n_vals, mode, e0, scale, ss_el, -  (e0, ss_el:
-//                 exchange word indices in the layer; ss_el < 0: none)
+//   poll-table  : tb, n_tab, n_vals, mode, e0, scale, ss_el, job  (e0, ss_el:
+//                 exchange word indices in the layer; ss_el < 0: none; job:
+//                 the bound entry 0-3 the unit's |z| sum goes to, -1: none)
 //   stage-2 unit: U, R, nw, tb, h, out, nrows, -
 //   stage-1 unit: V, r, nw, tb, dst, ncols, own, slot  (own: the cluster rank
 //                 that sums the unit's partials and sends them; slot: the
@@ -144,10 +155,16 @@ struct Params {
     float *out, *q_out, *kv_out;
     unsigned *ws_words;
     unsigned long long plan;
-    unsigned long long *xacc;  // exchange pairs, n_layers * acc_layer (2 words each)
+    unsigned long long *xacc;  // exchange words, n_layers * acc_layer
     unsigned n_t;              // contributions per t element: one per cluster
+    // per layer l (0..n_layers) and phase X, two float4 of constants for the
+    // exchange bounds (k_stack_consts): c[0..3], then max|g| of the
+    // linears whose stage 1 the phase sends
+    const float4 *cst;
     int acc_layer, offA, offQ, offB, offC, offD, lenA, lenQ, lenB, lenC, lenD;
-    float fix_limit;  // |contribution| bound that keeps the fixed-point sum in range
+    // largest |scaled contribution| of a t / mean-square element: below
+    // 2^55 / contributions, so no complete sum leaves the word
+    float lim_t, lim_ss;
     Offsets o;
 };
 
@@ -332,15 +349,15 @@ __device__ __forceinline__ void record(unsigned *ws_words, lb_status st) {
 // Stage-1 units: t[col] partial over the CTA's input slice (lane = column).
 // Every CTA has a unit for every column, also when its slice is empty (it
 // then contributes zeros).  Without clusters each partial goes straight into
-// the exchange pairs.  With clusters a unit belongs to one rank of the
+// the exchange words (at scale sc).  With clusters a unit belongs to one rank of the
 // cluster: the other ranks store their partials into its receive slot in
 // the owner's shared memory (st.async, completing on the slot's mbarrier),
 // and the owner adds them to its own in rank order and sends the sum -- one
 // contribution per cluster.  A warp runs the units it does not own first.
 // Returns false (this warp) when an owner's wait ran out.
-__device__ __noinline__ bool run_s1(int prog, int s, unsigned long long *xbase, float limit,
-                                    unsigned *err, int slot0, int ubar0, int ubar, unsigned par,
-                                    unsigned rank, unsigned *ws_words) {
+__device__ __noinline__ bool run_s1(int prog, int s, unsigned long long *xbase, float sc,
+                                    float limit, unsigned *err, int slot0, int ubar0, int ubar,
+                                    unsigned par, unsigned rank, unsigned *ws_words) {
     const Step &st = step_at(prog, s);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
@@ -363,7 +380,7 @@ __device__ __noinline__ bool run_s1(int prog, int s, unsigned long long *xbase, 
     auto finish = [&](const int4 &b, float v) {
         const int dst = b.x, ncols = b.y;
         if (kCluster == 1) {
-            if (lane < ncols) send_fix2(fix2_at(xbase, dst + lane), v, limit, err);
+            if (lane < ncols) send_fix1(xbase + dst + lane, v, sc, limit, err);
             return;
         }
         const unsigned own = (unsigned)b.z;
@@ -393,7 +410,7 @@ __device__ __noinline__ bool run_s1(int prog, int s, unsigned long long *xbase, 
         float sum = 0.f;
 #pragma unroll
         for (int k = 0; k < kCluster; ++k) sum += (unsigned)k == rank ? v : rx[32 * k + lane];
-        if (lane < ncols) send_fix2(fix2_at(xbase, dst + lane), sum, limit, err);
+        if (lane < ncols) send_fix1(xbase + dst + lane, sum, sc, limit, err);
     };
     int u = u0;
     // two units per pass; a unit whose input slice is empty (no words) reads
@@ -466,15 +483,18 @@ __device__ __forceinline__ void zero_stripe(unsigned long long *region, const in
 }
 
 // Poll-table units: the stage-2 tables of a phase built straight from the
-// exchange pairs.  Lane n waits until the elements e0 + 4n .. +3 (those below
+// exchange words.  Lane n waits until the elements e0 + 4n .. +3 (those below
 // n_vals) -- and the element ss_el, for a TAB_MUL unit that has one -- count
-// n_t contributions (n_ss for ss_el), decodes them and builds table n of v_i = t_i * l_i
-// (* inv with TAB_MUL, inv = rsqrt(mean square) of element ss_el, or the
-// argument when the unit has no ss_el).  Bounded; returns false (to every
-// compute thread) on failure.
+// n_t contributions (n_ss for ss_el), decodes them (inverse scales it, and
+// iss for ss_el) and builds table n of v_i = t_i * l_i (* inv with TAB_MUL,
+// inv = rsqrt(mean square) of element ss_el, or the argument when the unit
+// has no ss_el).  A unit with a job adds the sum of its |v_i| (a fixed-order
+// warp sum) to zmax[job] by max (fp32 bits of a non-negative value: an
+// order-independent result).  Bounded; returns false (to every compute
+// thread) on failure.
 __device__ __noinline__ bool run_poll_tables(int prog, int s, const unsigned long long *xbase,
-                                             unsigned n_t, unsigned n_ss, float inv,
-                                             unsigned *ws_words) {
+                                             unsigned n_t, unsigned n_ss, float inv, float it,
+                                             float iss, unsigned *zmax, unsigned *ws_words) {
     const Step &st = step_at(prog, s);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     int ok = 1;
@@ -488,21 +508,22 @@ __device__ __noinline__ bool run_poll_tables(int prog, int s, const unsigned lon
         // and once it sees its word complete the whole unit usually is
         if (lane == 0 && a.z > 0) {
             const unsigned long long t0 = globaltimer_ns();
-            // the lo word of the last element (the lo words are sent after the hi words)
-            const unsigned long long *gw = fix2_at(xbase, b.x + (min(a.z, 4 * a.y) - 1)) + 32;
-            for (int spin = 0; (unsigned)(ld_relaxed_u64(gw) & 0xffull) != n_t; ++spin)
+            const unsigned long long *gw = xbase + b.x + (min(a.z, 4 * a.y) - 1);
+            for (int spin = 0; !counted1(ld_relaxed_u64(gw), n_t); ++spin)
                 if ((spin & 15) == 15 && globaltimer_ns() - t0 > kWaitLimitNs) break;
         }
         __syncwarp();
-        if (lane >= a.y) continue;
-        const bool have = a.z - 4 * lane > 0;
+        const bool have = lane < a.y && a.z - 4 * lane > 0;
         const bool need_ss = have && (a.w & TAB_MUL) && b.z >= 0;
-        const unsigned long long *w = fix2_at(xbase, b.x + 4 * lane);
-        unsigned long long v[8], sh = 0, sl = 0, t0 = 0;
+        const unsigned long long *w = xbase + b.x + 4 * lane;
+        unsigned long long v0 = 0, v1 = 0, v2 = 0, v3 = 0, vs = 0, t0 = 0;
         for (int spin = 0; have; ++spin) {
-            ld_fix2x4(w, v);
-            if (need_ss) ld_fix2(fix2_at(xbase, b.z), sh, sl);
-            if (counted2x4(v, n_t) && (!need_ss || counted2(sh, sl, n_ss))) break;
+            ld_relaxed_v2_u64(w, v0, v1);
+            ld_relaxed_v2_u64(w + 2, v2, v3);
+            if (need_ss) vs = ld_relaxed_u64(xbase + b.z);
+            if (counted1(v0, n_t) && counted1(v1, n_t) && counted1(v2, n_t) &&
+                counted1(v3, n_t) && (!need_ss || counted1(vs, n_ss)))
+                break;
             if ((spin & 15) == 15) {
                 if (sticky(ws_words)) {
                     ok = 0;
@@ -517,17 +538,27 @@ __device__ __noinline__ bool run_poll_tables(int prog, int s, const unsigned lon
                 }
             }
         }
-        if (!ok) break;
+        // every lane of the warp leaves together (the sum below is warp-wide)
+        if (__any_sync(0xffffffffu, !ok)) {
+            ok = 0;
+            break;
+        }
         float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
         if (have) {
             const uint2 hb = *reinterpret_cast<const uint2 *>(g_smem + b.y + 8 * lane);
-            const float m = (a.w & TAB_MUL) ? (need_ss ? rsqrtf(dec_fix2(sh, sl)) : inv) : 1.f;
-            x.x = dec_fix2(v[0], v[1]) * half_bits_to_float((uint16_t)(hb.x & 0xffffu)) * m;
-            x.y = dec_fix2(v[2], v[3]) * half_bits_to_float((uint16_t)(hb.x >> 16)) * m;
-            x.z = dec_fix2(v[4], v[5]) * half_bits_to_float((uint16_t)(hb.y & 0xffffu)) * m;
-            x.w = dec_fix2(v[6], v[7]) * half_bits_to_float((uint16_t)(hb.y >> 16)) * m;
+            const float m = (a.w & TAB_MUL) ? (need_ss ? rsqrtf(dec_fix1(vs, iss)) : inv) : 1.f;
+            x.x = dec_fix1(v0, it) * half_bits_to_float((uint16_t)(hb.x & 0xffffu)) * m;
+            x.y = dec_fix1(v1, it) * half_bits_to_float((uint16_t)(hb.x >> 16)) * m;
+            x.z = dec_fix1(v2, it) * half_bits_to_float((uint16_t)(hb.y & 0xffffu)) * m;
+            x.w = dec_fix1(v3, it) * half_bits_to_float((uint16_t)(hb.y >> 16)) * m;
         }
-        store_table(g_smem + a.x + lane * 128, x, lane);
+        if (b.w >= 0) {
+            float zs = (fabsf(x.x) + fabsf(x.y)) + (fabsf(x.z) + fabsf(x.w));
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) zs += __shfl_xor_sync(0xffffffffu, zs, o);
+            if (lane == 0) atomicMax(zmax + b.w, __float_as_uint(zs));
+        }
+        if (lane < a.y) store_table(g_smem + a.x + lane * 128, x, lane);
     }
     return csync_and(ok) != 0;
 }
@@ -584,12 +615,17 @@ struct Loader {
     __device__ void lat(int dl, const LinDesc &L, int p, unsigned long long *b) const {
         copy(dl, L.l[p], (unsigned)(L.r[p] * 2), b);
     }
+    // the exchange-bound constants of phase X of layer l
+    __device__ void consts(int X, int l, unsigned long long *b) const {
+        copy(P->o.cst[X], P->cst + ((size_t)l * 4 + X) * 2, 32u, b);
+    }
 
     // phase A of layer l (0 <= l <= n_layers): down of layer l-1 on R_c rows,
     // stage 1 of q, k, v of layer l on R_c (absent for l = n_layers).
     __device__ void issue_A(int l) const {
         unsigned long long *b = full + 0;
         const Offsets &o = P->o;
+        consts(0, l, b);
         if (l > 0) {
             const LinDesc &D = P->lin[7 * (l - 1) + LD];
             for (int p = 0; p < D.n_paths; ++p) {
@@ -609,6 +645,7 @@ struct Loader {
     __device__ void issue_B(int l) const {
         unsigned long long *b = full + 1;
         const Offsets &o = P->o;
+        consts(1, l, b);
         const LinDesc &Q = P->lin[7 * l + LQ], &K = P->lin[7 * l + LK], &V = P->lin[7 * l + LV],
                       &O = P->lin[7 * l + LO];
         const int grp = P->d / P->dkv;
@@ -638,6 +675,7 @@ struct Loader {
     __device__ void issue_C(int l) const {
         unsigned long long *b = full + 2;
         const Offsets &o = P->o;
+        consts(2, l, b);
         const LinDesc &O = P->lin[7 * l + LO], &G = P->lin[7 * l + LG], &U = P->lin[7 * l + LU];
         for (int p = 0; p < O.n_paths; ++p) {
             rows(o.c_Uo[p], o.c_ho[p], O, p, 32 * s.dw0, 32 * s.nd, b);
@@ -650,6 +688,7 @@ struct Loader {
     __device__ void issue_D(int l) const {
         unsigned long long *b = full + 3;
         const Offsets &o = P->o;
+        consts(3, l, b);
         const LinDesc &G = P->lin[7 * l + LG], &U = P->lin[7 * l + LU], &D = P->lin[7 * l + LD];
         for (int p = 0; p < G.n_paths; ++p) {
             rows(o.d_Ug[p], o.d_hg[p], G, p, 32 * s.fw0, 32 * s.nf, b);
@@ -722,6 +761,9 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
     __shared__ __align__(8) unsigned long long full[4], empty[4];
     __shared__ int s_last;
     __shared__ int s_zs[XR_N][2];  // this CTA's stripe of each exchange region
+    // per phase, the largest |z| sum of a poll unit of each bound entry; and
+    // the largest per-thread share of the L1 norm of x0 (fp32 bits)
+    __shared__ unsigned s_zmax[4][4], s_x0max;
     unsigned *err = P.ws_words + kErrWord;
     if (sticky(P.ws_words)) return;
     if (*reinterpret_cast<const volatile unsigned long long *>(P.ws_words + kPlanWord) != P.plan) {
@@ -757,13 +799,14 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         for (int b = 0; b < P.o.n_ubar; ++b)
             mbar_init(reinterpret_cast<unsigned long long *>(g_smem + P.o.ubar) + b, 1);
         fence_barrier_init();
+        for (int k = 0; k < 16; ++k) s_zmax[k >> 2][k & 3] = 0u;
+        s_x0max = 0u;
     }
     if (threadIdx.x < XR_N) {
         const int t = threadIdx.x;
         const int n = t == XR_A ? P.lenA : t == XR_Q ? P.lenQ : t == XR_B ? P.lenB
                     : t == XR_C ? P.lenC : P.lenD;
-        // in words: the region's whole 32-element blocks
-        const long long w = (long long)fix2_words(n);
+        const long long w = (long long)n;
         s_zs[threadIdx.x][0] = (int)(c * w / N);
         s_zs[threadIdx.x][1] = (int)((c + 1) * w / N);
     }
@@ -794,45 +837,73 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
     zero_f(yk, nkv);
     zero_f(yv, nkv);
     if (threadIdx.x == 0) ssacc[0] = 0.f;
+    {
+        // ||x0||_1 <= kCT x the largest per-thread share (every CTA alike)
+        float a = 0.f;
+        for (int i = threadIdx.x; i < P.d; i += kCT) a += fabsf(bf16_bits_to_float(P.x0[i]));
+        atomicMax(&s_x0max, __float_as_uint(a));
+    }
     csync();
     int nr[7];
 #pragma unroll
     for (int k = 0; k < 7; ++k) nr[k] = P.r[k][0] + (P.np[k] > 1 ? P.r[k][1] : 0);
-    const int ssA = nr[LV], ssC = nr[LG] + nr[LU];
+    const int ssA_el = nr[LV], ssC_el = nr[LG] + nr[LU];
     const bool lead = threadIdx.x == 0;
-    const float lim = P.fix_limit, inv_d = 1.f / (float)P.d;
-    // the first word of region off (a multiple of 32 elements) in the layer at x
-    auto at = [](unsigned long long *x, int off) { return x + 2 * off; };
+    const float inv_d = 1.f / (float)P.d;
+    const int n_tc = (int)n_t, n_cc = (int)n_ctas;
+    // Exchange bounds (identical in every CTA).  Ba, Bh: L1 norms of a and
+    // h; per exchange the scale of its t (sc*) and mean square (ss*) and the
+    // inverses its readers decode with (i*).
+    float Ba = (float)kCT * __uint_as_float(s_x0max), Bh = 0.f;
+    float2 scA = make_float2(1.f, 1.f), ssA = scA, scB = scA, scC = scA, ssC = scA, scD = scA;
+    // phase X's constants and largest unit |z| sums
+    auto cst = [&](int X, int k) { return reinterpret_cast<const float4 *>(g_smem + o.cst[X])[k]; };
+    auto zm = [&](int X, int j) { return __uint_as_float(s_zmax[X][j]); };
+    // the first word of region off in the layer at x
+    auto at = [](unsigned long long *x, int off) { return x + off; };
     auto release = [&](int b) {
         csync();
         if (lead) mbar_arrive(empty + b);
     };
-    // this CTA's share of the mean square (sum / d), so that outlier-sized
-    // activations stay in range
-    auto send_ss = [&](unsigned long long *p) {
+    // this CTA's share of the mean square (sum / d); its bound is B^2 / d
+    // for B the L1 norm of the vector.  The lead also clears the phase's
+    // |z| maxima: every compute thread read them before the barrier that
+    // precedes this call.
+    auto send_ss = [&](unsigned long long *p, float2 sc, int X) {
         if (lead) {
-            send_fix2(p, ssacc[0] * inv_d, lim, err);
+            send_fix1(p, ssacc[0] * inv_d, sc.x, P.lim_ss, err);
             ssacc[0] = 0.f;
         }
+        if (threadIdx.x < 4) s_zmax[X][threadIdx.x] = 0u;
+    };
+    auto clear_z = [&](int X) {
+        if (threadIdx.x < 4) s_zmax[X][threadIdx.x] = 0u;
     };
     // a failed wait leaves the layer loop; the CTA still meets its cluster at
     // the end, so no other CTA stores into its shared memory after it exits
 #define FAIL_EXIT() goto done
 
     for (int l = 0; l < P.n_layers; ++l) {
-        unsigned long long *xl = P.xacc + (size_t)2 * l * P.acc_layer;
-        unsigned long long *xp = xl - 2 * P.acc_layer;  // the previous layer's pairs
+        unsigned long long *xl = P.xacc + (size_t)l * P.acc_layer;
+        unsigned long long *xp = xl - P.acc_layer;  // the previous layer's words
         const unsigned par = (unsigned)(l & 1);
 
         // ================= phase A: a = h + Down_{l-1}(m) on R_c; stage 1 of q, k, v
         if (!wait_full(full + 0, par, P.ws_words)) FAIL_EXIT();
-        if (l > 0 && !run_poll_tables(pg, A_P2, xp, n_t, n_ctas, 1.f, P.ws_words))
-            FAIL_EXIT();
+        if (l > 0) {
+            if (!run_poll_tables(pg, A_P2, xp, n_t, n_ctas, 1.f, scD.y, 1.f, s_zmax[0],
+                                 P.ws_words))
+                FAIL_EXIT();
+            const float4 c = cst(0, 0);
+            Ba = Bh + (c.x * zm(0, 0) + c.y * zm(0, 1));  // ||a|| <= ||h|| + ||Down(m)||
+        }
+        scA = fix1_scale(cst(0, 1).x * Ba, n_tc);  // |t| <= max|g| ||a||
+        ssA = fix1_scale(Ba * Ba * inv_d, n_cc);
         run_rows(pg, A_R, l > 0, true, o.ssacc);  // a = res0 + Down(m) -> res1; tables
         csync();
-        send_ss(fix2_at(xl, P.offA + ssA));
-        if (!csync_and(run_s1(pg, A_S1, xl, lim, err, o.slot[0], o.ubar0[0], o.ubar, par, rank,
-                              P.ws_words)))
+        send_ss(xl + P.offA + ssA_el, ssA, 0);
+        if (!csync_and(run_s1(pg, A_S1, xl, scA.x, P.lim_t, err, o.slot[0], o.ubar0[0], o.ubar,
+                              par, rank, P.ws_words)))
             FAIL_EXIT();
         // regions C and Q of the previous layer: every CTA has passed the
         // poll that read them (exchange D, polled above, counts all CTAs)
@@ -845,11 +916,19 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         // ================= phase B: v rows for attention, stage 1 of o; then q, k, v out
         if (!wait_full(full + 1, par, P.ws_words)) FAIL_EXIT();
         // tables of v (critical) and of q, k (region Q, sent with region A)
-        if (!run_poll_tables(pg, B_P2, xl, n_t, n_ctas, 1.f, P.ws_words)) FAIL_EXIT();
+        if (!run_poll_tables(pg, B_P2, xl, n_t, n_ctas, 1.f, scA.y, ssA.y, s_zmax[1],
+                             P.ws_words))
+            FAIL_EXIT();
+        {
+            // the attention rows repeat v: ||attn|| <= grp ||v|| (grp in c)
+            const float4 c = cst(1, 0);
+            scB = fix1_scale(cst(1, 1).x * (c.x * zm(1, 0) + c.y * zm(1, 1)), n_tc);
+        }
         run_rows(pg, B_R, true, true, o.ssacc);  // v on the attention rows; tables of o
         csync();
-        if (!csync_and(run_s1(pg, B_S1, xl, lim, err, o.slot[1], o.ubar0[1], o.ubar, par, rank,
-                              P.ws_words)))
+        clear_z(1);
+        if (!csync_and(run_s1(pg, B_S1, xl, scB.x, P.lim_t, err, o.slot[1], o.ubar0[1], o.ubar,
+                              par, rank, P.ws_words)))
             FAIL_EXIT();
         if (l > 0) zero_stripe(at(xp, P.offD), s_zs[XR_D]);  // read by phase A's poll
         // ---- off the critical path, while exchange B is in flight: q on R_c,
@@ -871,23 +950,40 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
 
         // ================= phase C: h = a + O(attn) on R_c; stage 1 of gate, up
         if (!wait_full(full + 2, par, P.ws_words)) FAIL_EXIT();
-        if (!run_poll_tables(pg, C_P2, xl, n_t, n_ctas, 1.f, P.ws_words)) FAIL_EXIT();
+        if (!run_poll_tables(pg, C_P2, xl, n_t, n_ctas, 1.f, scB.y, 1.f, s_zmax[2],
+                             P.ws_words))
+            FAIL_EXIT();
+        {
+            const float4 c = cst(2, 0);
+            Bh = Ba + (c.x * zm(2, 0) + c.y * zm(2, 1));  // ||h|| <= ||a|| + ||O(attn)||
+            scC = fix1_scale(cst(2, 1).x * Bh, n_tc);
+            ssC = fix1_scale(Bh * Bh * inv_d, n_cc);
+        }
         run_rows(pg, C_R, true, true, o.ssacc);  // h = res1 + O(attn) -> res0; tables
         csync();
-        send_ss(fix2_at(xl, P.offC + ssC));
-        if (!csync_and(run_s1(pg, C_S1, xl, lim, err, o.slot[2], o.ubar0[2], o.ubar, par, rank,
-                              P.ws_words)))
+        send_ss(xl + P.offC + ssC_el, ssC, 2);
+        if (!csync_and(run_s1(pg, C_S1, xl, scC.x, P.lim_t, err, o.slot[2], o.ubar0[2], o.ubar,
+                              par, rank, P.ws_words)))
             FAIL_EXIT();
         zero_stripe(at(xl, P.offA), s_zs[XR_A]);  // read by phase B's poll
         release(2);
 
         // ================= phase D: m = silu(gate) * up on F_c; stage 1 of down
         if (!wait_full(full + 3, par, P.ws_words)) FAIL_EXIT();
-        if (!run_poll_tables(pg, D_P2, xl, n_t, n_ctas, 1.f, P.ws_words)) FAIL_EXIT();
+        if (!run_poll_tables(pg, D_P2, xl, n_t, n_ctas, 1.f, scC.y, ssC.y, s_zmax[3],
+                             P.ws_words))
+            FAIL_EXIT();
+        {
+            // ||silu(G) * U|| <= max|G| ||U||
+            const float4 c = cst(3, 0);
+            const float Bm = (c.x * zm(3, 0) + c.y * zm(3, 1)) * (c.z * zm(3, 2) + c.w * zm(3, 3));
+            scD = fix1_scale(cst(3, 1).x * Bm, n_tc);
+        }
         run_rows(pg, D_R, true, true, o.ssacc);  // m = silu(gate) * up; tables of down
         csync();
-        if (!csync_and(run_s1(pg, D_S1, xl, lim, err, o.slot[3], o.ubar0[3], o.ubar, par, rank,
-                              P.ws_words)))
+        clear_z(3);
+        if (!csync_and(run_s1(pg, D_S1, xl, scD.x, P.lim_t, err, o.slot[3], o.ubar0[3], o.ubar,
+                              par, rank, P.ws_words)))
             FAIL_EXIT();
         zero_stripe(at(xl, P.offB), s_zs[XR_B]);  // read by phase C's poll
         release(3);
@@ -896,9 +992,10 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
     // ================= final: out = h + Down_{L-1}(m) on R_c
     {
         const int l = P.n_layers;
-        unsigned long long *xp = P.xacc + (size_t)2 * (l - 1) * P.acc_layer;
+        unsigned long long *xp = P.xacc + (size_t)(l - 1) * P.acc_layer;
         if (!wait_full(full + 0, (unsigned)(l & 1), P.ws_words)) FAIL_EXIT();
-        if (!run_poll_tables(pg, A_P2, xp, n_t, n_ctas, 1.f, P.ws_words)) FAIL_EXIT();
+        if (!run_poll_tables(pg, A_P2, xp, n_t, n_ctas, 1.f, scD.y, 1.f, s_zmax[0], P.ws_words))
+            FAIL_EXIT();
         zero_stripe(at(xp, P.offC), s_zs[XR_C]);
         zero_stripe(at(xp, P.offQ), s_zs[XR_Q]);
         run_rows(pg, A_R, true, false, o.ssacc);  // a = res0 + Down(m) -> res1
@@ -913,7 +1010,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         csync();
         if (s_last) {
             __threadfence();
-            for (int i = threadIdx.x; i < (int)fix2_words(P.lenD); i += kCT)
+            for (int i = threadIdx.x; i < P.lenD; i += kCT)
                 at(xp, P.offD)[i] = 0ull;
             if (lead) P.ws_words[kDoneWord] = 0u;
         }
@@ -956,7 +1053,7 @@ int rsum(const lb_linear &L) {
 
 int up(int n, int a) { return (n + a - 1) / a * a; }
 
-// Exchange elements (pairs of words) per layer: A = t of v + ss(a); Q = t of
+// Exchange elements (one word each) per layer: A = t of v + ss(a); Q = t of
 // q, k (read off the critical path); B = t of o; C = t of gate, up + ss(h);
 // D = t of down; each region padded to 32 elements.
 struct XLayout {
@@ -981,6 +1078,113 @@ XLayout xlayout(const lb_linear *lin) {
 
 size_t desc_bytes_for(int n_layers) {
     return ((size_t)7 * n_layers * sizeof(LinDesc) + 255) & ~(size_t)255;
+}
+
+// One exchange word per element.
+size_t xacc_bytes(const XLayout &X, int n_layers) {
+    return ((size_t)n_layers * X.acc_layer * sizeof(unsigned long long) + 255) & ~(size_t)255;
+}
+
+// Two float4 per phase and layer, layers 0..n_layers.
+size_t cst_bytes(int n_layers) { return ((size_t)(n_layers + 1) * 4 * 32 + 255) & ~(size_t)255; }
+
+// 2^55 / n rounded down: n contributions below it sum to less than 2^55.
+float fix1_limit(int n) {
+    float l = (float)(std::ldexp(1.0, 55) / n);
+    while ((double)l * n >= std::ldexp(1.0, 55)) l = std::nextafter(l, 0.f);
+    return l;
+}
+
+// ---------------------------------------------------------------- bound constants
+
+constexpr int kConstThreads = 256;
+
+// Block-wide sum (fp64) and max of |v| over n fp16 values.
+__device__ void abs_stats(const uint16_t *v, int n, double &sum, float &mx) {
+    __shared__ double s_sum[kConstThreads / 32];
+    __shared__ float s_max[kConstThreads / 32];
+    double a = 0.0;
+    float m = 0.f;
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+        const float x = fabsf(half_bits_to_float(v[i]));
+        a += (double)x;
+        m = fmaxf(m, x);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        a += __shfl_xor_sync(0xffffffffu, a, o);
+        m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+    }
+    __syncthreads();  // the previous call's readers are done
+    if ((threadIdx.x & 31) == 0) {
+        s_sum[threadIdx.x >> 5] = a;
+        s_max[threadIdx.x >> 5] = m;
+    }
+    __syncthreads();
+    sum = 0.0;
+    mx = 0.f;
+    for (int w = 0; w < kConstThreads / 32; ++w) {
+        sum += s_sum[w];
+        mx = fmaxf(mx, s_max[w]);
+    }
+}
+
+// Constants of the exchange bounds, block l for layer l (0..n_layers).  A
+// poll unit covers 128 values of t, so a path of rank r has nu = ceil(r /
+// 128) units and sum |z| <= nu x the largest unit sum zmax.  Per phase
+// (c[0..3]; then max|g| of the linears whose stage 1 the phase sends):
+//   A: ||h_down(l-1),p||_1 nu (p = 0, 1)                  ; q, k, v of layer l
+//   B: grp ||h_v,p||_1 nu (attention repeats v grp times) ; o
+//   C: ||h_o,p||_1 nu                                     ; gate, up
+//   D: max|h_gate,p| nu, ||h_up,p||_1 nu                  ; down
+// (sums in fp64, rounded up to fp32).
+__global__ void __launch_bounds__(kConstThreads) k_stack_consts(const LinDesc *lin, int n_layers,
+                                                                int grp, float4 *cst) {
+    const int l = blockIdx.x;
+    float c[4][4] = {}, gmax[4] = {};
+    auto nu = [](int r) { return (double)((r + 127) / 128); };
+    auto hsum = [&](const LinDesc &L, int p, double mul) {
+        double s;
+        float m;
+        abs_stats(L.h[p], L.d_out, s, m);
+        return __double2float_ru(s * mul * nu(L.r[p]));
+    };
+    auto hmax = [&](const LinDesc &L, int p) {
+        double s;
+        float m;
+        abs_stats(L.h[p], L.d_out, s, m);
+        return __double2float_ru((double)m * nu(L.r[p]));
+    };
+    auto gm = [&](const LinDesc &L) {
+        float r = 0.f;
+        for (int p = 0; p < L.n_paths; ++p) {
+            double s;
+            float m;
+            abs_stats(L.g[p], L.d_in, s, m);
+            r = fmaxf(r, m);
+        }
+        return r;
+    };
+    if (l > 0) {
+        const LinDesc &D = lin[7 * (l - 1) + LD];
+        for (int p = 0; p < D.n_paths; ++p) c[0][p] = hsum(D, p, 1.0);
+    }
+    if (l < n_layers) {
+        const LinDesc *L = lin + 7 * l;
+        gmax[0] = fmaxf(gm(L[LQ]), fmaxf(gm(L[LK]), gm(L[LV])));
+        for (int p = 0; p < L[LV].n_paths; ++p) c[1][p] = hsum(L[LV], p, (double)grp);
+        gmax[1] = gm(L[LO]);
+        for (int p = 0; p < L[LO].n_paths; ++p) c[2][p] = hsum(L[LO], p, 1.0);
+        gmax[2] = fmaxf(gm(L[LG]), gm(L[LU]));
+        for (int p = 0; p < L[LG].n_paths; ++p) c[3][p] = hmax(L[LG], p);
+        for (int p = 0; p < L[LU].n_paths; ++p) c[3][2 + p] = hsum(L[LU], p, 1.0);
+        gmax[3] = gm(L[LD]);
+    }
+    if (threadIdx.x < 4) {
+        const int X = threadIdx.x;
+        cst[((size_t)l * 4 + X) * 2 + 0] = make_float4(c[X][0], c[X][1], c[X][2], c[X][3]);
+        cst[((size_t)l * 4 + X) * 2 + 1] = make_float4(gmax[X], 0.f, 0.f, 0.f);
+    }
 }
 
 // Stage-1 units (32-column blocks over every path) of linears k0..k1.
@@ -1021,6 +1225,7 @@ SmemPlan smem_plan(const lb_linear *lin, const StackShape &sh, int N) {
             o.a_g[k][p] = take(ok ? 64 * nd : 0);
         }
     }
+    o.cst[0] = take(32);
     at = up(at, 128);
     for (int p = 0; p < 2; ++p) {
         const bool v = p < lin[LV].n_paths, oo = p < lin[LO].n_paths, q = p < lin[LQ].n_paths,
@@ -1039,6 +1244,7 @@ SmemPlan smem_plan(const lb_linear *lin, const StackShape &sh, int N) {
         o.b_hk[p] = take(k ? 2 * nkv : 0);
         o.b_lk[p] = take(k ? 2 * r(LK, p) : 0);
     }
+    o.cst[1] = take(32);
     at = up(at, 128);
     for (int p = 0; p < 2; ++p) {
         const bool oo = p < lin[LO].n_paths, g = p < lin[LG].n_paths, u = p < lin[LU].n_paths;
@@ -1050,6 +1256,7 @@ SmemPlan smem_plan(const lb_linear *lin, const StackShape &sh, int N) {
         o.c_Vu[p] = take(u ? nd * r(LU, p) * 4 : 0);
         o.c_gu[p] = take(u ? 64 * nd : 0);
     }
+    o.cst[2] = take(32);
     at = up(at, 128);
     for (int p = 0; p < 2; ++p) {
         const bool g = p < lin[LG].n_paths, u = p < lin[LU].n_paths, dd = p < lin[LD].n_paths;
@@ -1062,6 +1269,7 @@ SmemPlan smem_plan(const lb_linear *lin, const StackShape &sh, int N) {
         o.d_Vd[p] = take(dd ? nf * r(LD, p) * 4 : 0);
         o.d_gd[p] = take(dd ? 64 * nf : 0);
     }
+    o.cst[3] = take(32);
     // nibble tables (1 KB per 32 values): the largest set a phase holds at once
     auto utab = [&](int k, int p0, int p1) {
         int b = 0;
@@ -1108,9 +1316,10 @@ SmemPlan smem_plan(const lb_linear *lin, const StackShape &sh, int N) {
 
 // ---------------------------------------------------------------- the program
 
-// e0, ss_el: exchange word indices within a layer (ss_el < 0: none)
-Item ptab(int tb, int n_tab, int n_vals, int mode, int e0, int scale, int ss_el) {
-    return Item{{tb, n_tab, n_vals, mode, e0, scale, ss_el, 0}};
+// e0, ss_el: exchange word indices within a layer (ss_el < 0: none); job:
+// the bound entry of the unit's |z| sums (-1: none)
+Item ptab(int tb, int n_tab, int n_vals, int mode, int e0, int scale, int ss_el, int job) {
+    return Item{{tb, n_tab, n_vals, mode, e0, scale, ss_el, job}};
 }
 
 struct Costed {
@@ -1253,7 +1462,7 @@ struct ProgBuild {
             const int nt = J.f[1];
             for (int t0 = 0; t0 < nt; t0 += 32)
                 us.push_back({Item{{J.f[0] + 128 * t0, std::min(32, nt - t0), J.f[2] - 4 * t0,
-                                    J.f[3], J.f[4] + 4 * t0, J.f[5] + 8 * t0, J.f[6], 0}},
+                                    J.f[3], J.f[4] + 4 * t0, J.f[5] + 8 * t0, J.f[6], J.f[7]}},
                               1.0 + std::min(32, nt - t0) / 32.0});
         }
         std::vector<Item> g;
@@ -1351,7 +1560,7 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
         int tb = o.t2, off = X.offD;  // words of the previous layer
         std::vector<Seg> g;
         for (int p = 0; p < np(LD); ++p) {
-            T.push_back(ptab(tb, 8 * Rk(LD, p), rk(LD, p), TAB_PLAIN, off, o.a_ld[p], -1));
+            T.push_back(ptab(tb, 8 * Rk(LD, p), rk(LD, p), TAB_PLAIN, off, o.a_ld[p], -1, p));
             g.push_back({o.a_Ud[p], Rk(LD, p), Rk(LD, p), tb, o.a_hd[p]});
             tb += Rk(LD, p) * 1024;
             off += rk(LD, p);
@@ -1380,7 +1589,7 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
         std::vector<Seg> g;
         for (int p = 0; p < np(LV); ++p) {
             T.push_back(ptab(tb, 8 * Rk(LV, p), rk(LV, p), TAB_PLAIN | TAB_MUL, off, o.b_lv[p],
-                             ssA));
+                             ssA, p));
             g.push_back({o.b_Uat[p], Rk(LV, p), Rk(LV, p), tb, o.b_hat[p]});
             tbv[p] = tb;
             tb += Rk(LV, p) * 1024;
@@ -1390,14 +1599,14 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
         off = X.offQ;
         for (int p = 0; p < np(LQ); ++p) {
             T.push_back(ptab(tb, 8 * Rk(LQ, p), rk(LQ, p), TAB_PLAIN | TAB_MUL, off, o.b_lq[p],
-                             ssA));
+                             ssA, -1));
             Uqkv.push_back({o.b_Uq[p], o.b_hq[p], Rk(LQ, p), rows_d, tb, o.yq});
             tb += Rk(LQ, p) * 1024;
             off += rk(LQ, p);
         }
         for (int p = 0; p < np(LK); ++p) {
             T.push_back(ptab(tb, 8 * Rk(LK, p), rk(LK, p), TAB_PLAIN | TAB_MUL, off, o.b_lk[p],
-                             ssA));
+                             ssA, -1));
             Uqkv.push_back({o.b_Uk[p], o.b_hk[p], Rk(LK, p), nkv, tb, o.yk});
             tb += Rk(LK, p) * 1024;
             off += rk(LK, p);
@@ -1424,7 +1633,7 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
         int tb = o.t2, off = X.offB;
         std::vector<Seg> g;
         for (int p = 0; p < np(LO); ++p) {
-            T.push_back(ptab(tb, 8 * Rk(LO, p), rk(LO, p), TAB_PLAIN, off, o.c_lo[p], -1));
+            T.push_back(ptab(tb, 8 * Rk(LO, p), rk(LO, p), TAB_PLAIN, off, o.c_lo[p], -1, p));
             g.push_back({o.c_Uo[p], Rk(LO, p), Rk(LO, p), tb, o.c_ho[p]});
             tb += Rk(LO, p) * 1024;
             off += rk(LO, p);
@@ -1451,7 +1660,7 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
         for (int k = LG; k <= LU; ++k)
             for (int p = 0; p < np(k); ++p) {
                 T.push_back(ptab(tb, 8 * Rk(k, p), rk(k, p), TAB_PLAIN | TAB_MUL, off,
-                                 k == LG ? o.d_lg[p] : o.d_lu[p], ssC));
+                                 k == LG ? o.d_lg[p] : o.d_lu[p], ssC, 2 * (k - LG) + p));
                 gs[k - LG].push_back({k == LG ? o.d_Ug[p] : o.d_Uu[p], Rk(k, p), Rk(k, p), tb,
                                       k == LG ? o.d_hg[p] : o.d_hu[p]});
                 tb += Rk(k, p) * 1024;
@@ -1517,18 +1726,24 @@ bool shapes_ok(const lb_linear *lin, const StackShape &sh, int num_sms) {
 
 static_assert(sizeof(LinDesc) % sizeof(uint32_t) == 0, "descriptor is copied as words");
 
+// Workspace after the header: descriptors, exchange words, bound constants,
+// programs.
 size_t stack_ws_bytes_after_header(const lb_linear *lin, int n_layers) {
     const XLayout X = xlayout(lin);
-    return desc_bytes_for(n_layers) +
-           (size_t)2 * n_layers * X.acc_layer * sizeof(unsigned long long) +
+    return desc_bytes_for(n_layers) + xacc_bytes(X, n_layers) + cst_bytes(n_layers) +
            (size_t)kMaxCtas * kProgBytes;
 }
 
 namespace {
+char *xacc_at(int n_layers, char *ws_after_header) {
+    return ws_after_header + desc_bytes_for(n_layers);
+}
+float4 *cst_at(const lb_linear *lin, int n_layers, char *ws_after_header) {
+    return reinterpret_cast<float4 *>(xacc_at(n_layers, ws_after_header) +
+                                      xacc_bytes(xlayout(lin), n_layers));
+}
 char *programs_at(const lb_linear *lin, int n_layers, char *ws_after_header) {
-    const XLayout X = xlayout(lin);
-    return ws_after_header + desc_bytes_for(n_layers) +
-           (size_t)2 * n_layers * X.acc_layer * sizeof(unsigned long long);
+    return reinterpret_cast<char *>(cst_at(lin, n_layers, ws_after_header)) + cst_bytes(n_layers);
 }
 }  // namespace
 
@@ -1541,11 +1756,9 @@ cudaError_t launch_stack_prepare(const lb_linear *lin, int n_layers, const Stack
     if (!build_programs(lin, sh, num_sms, progs)) return cudaErrorNotSupported;
     const XLayout X = xlayout(lin);
     LinDesc *desc = reinterpret_cast<LinDesc *>(ws_after_header);
-    char *xacc = ws_after_header + desc_bytes_for(n_layers);
+    char *xacc = xacc_at(n_layers, ws_after_header);
     cudaError_t e = cudaMemsetAsync(ws_words + kCounterWord, 0, 2 * sizeof(unsigned), s);
-    if (e == cudaSuccess)
-        e = cudaMemsetAsync(xacc, 0,
-                            (size_t)2 * n_layers * X.acc_layer * sizeof(unsigned long long), s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(xacc, 0, xacc_bytes(X, n_layers), s);
     // pageable source: the call returns once the data is staged
     if (e == cudaSuccess)
         e = cudaMemcpyAsync(programs_at(lin, n_layers, ws_after_header), progs.data(),
@@ -1560,6 +1773,10 @@ cudaError_t launch_stack_prepare(const lb_linear *lin, int n_layers, const Stack
         e = cudaGetLastError();
         if (e != cudaSuccess) return e;
     }
+    k_stack_consts<<<n_layers + 1, kConstThreads, 0, s>>>(desc, n_layers, sh.d / sh.dkv,
+                                                         cst_at(lin, n_layers, ws_after_header));
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
     k_set_plan<<<1, 1, 0, s>>>(ws_words, plan);
     return cudaGetLastError();
 }
@@ -1631,7 +1848,8 @@ cudaError_t launch_stack(const lb_linear *lin, int n_layers, const StackShape &s
     P.kv_out = kv_out;
     P.ws_words = ws_words;
     P.plan = plan;
-    P.xacc = reinterpret_cast<unsigned long long *>(ws_after_header + desc_bytes_for(n_layers));
+    P.xacc = reinterpret_cast<unsigned long long *>(xacc_at(n_layers, ws_after_header));
+    P.cst = cst_at(lin, n_layers, ws_after_header);
     P.acc_layer = X.acc_layer;
     P.offA = X.offA;
     P.offQ = X.offQ;
@@ -1645,7 +1863,8 @@ cudaError_t launch_stack(const lb_linear *lin, int n_layers, const StackShape &s
     P.lenD = X.lenD;
     if (num_sms % kCluster != 0) return cudaErrorInvalidConfiguration;
     P.n_t = (unsigned)(num_sms / kCluster);
-    P.fix_limit = fix2_limit(num_sms);
+    P.lim_t = fix1_limit((int)P.n_t);
+    P.lim_ss = fix1_limit(num_sms);
     P.o = S.o;
     const size_t smem = (size_t)S.bytes;
     cudaError_t e = cudaFuncSetAttribute((const void *)k_stack,
