@@ -63,7 +63,7 @@ namespace {
 
 constexpr int kST = 512;        // threads per CTA
 #ifndef LB_STACK_CLUSTER
-#define LB_STACK_CLUSTER 2
+#define LB_STACK_CLUSTER 1
 #endif
 // CTAs per thread-block cluster: the stage-1 partial sums of a cluster's
 // CTAs meet in distributed shared memory before one exchange contribution
@@ -92,9 +92,10 @@ struct Offsets {
     int cst[4];
     // work areas: stage-2 and stage-1 tables, residual stream (two buffers:
     // phase A reads 0 and writes 1, phase C the reverse), the off-path q, k, v
-    // outputs (added into, zeroed once stored), the sum-of-squares
-    // accumulator, the program
-    int t2, t1, res0, res1, yq, yk, yv, ssacc, prog;
+    // outputs (added into, zeroed once stored), the program
+    int t2, t1, res0, res1, yq, yk, yv, prog;
+    // per-unit sums of squares of the residual row steps (kMaxSlots floats)
+    int ssslot;
     // cluster reduction of the stage-1 partials, per phase X = A..D: the
     // receive slots of the units this CTA owns (kCluster x 32 floats each,
     // one row per sending rank) and the index of their first mbarrier in ubar
@@ -121,11 +122,13 @@ enum StepId {
 //   stage-1 unit: V, r, nw, tb, dst, ncols, own, slot  (own: the cluster rank
 //                 that sums the unit's partials and sends them; slot: the
 //                 unit's receive slot and mbarrier at that rank)
-//   row unit    : a header  n_pair, n_job, mode, nrows, res_in, res_out, -, -
-//                 then per pair two segments (first for lanes 0-15, second
-//                 for lanes 16-31)  U, R, nw, tb, h, -, -, -
+//   row unit    : a header  nseg, n_job, mode | log2(nr) << 8, nrows, res_in,
+//                 res_out, slot, -
+//                 then per lane group (32 / nr of them) nseg segments
+//                 U, R, nw, tb, h, -, -, -
 //                 then per table job  tb, g, -, -, -, -, -, -
-//                 (offsets of the unit's first row)
+//                 (offsets of the unit's first row; slot: the unit's
+//                 sum-of-squares slot, ROW_RES)
 struct Item {
     int f[8];
 };
@@ -140,11 +143,17 @@ enum { ROW_SUM = 0, ROW_RES = 1, ROW_SILU = 2 };
 struct Step {
     int first;
     int wo[kCW + 1];
+    int nslot;  // sum-of-squares slots written by the step (ROW_RES)
 };
 constexpr int kStepBytes = (int)((N_STEPS * sizeof(Step) + 15) / 16 * 16);
 constexpr int kProgBytes = 16384;  // per CTA, in the workspace and in shared memory
 constexpr int kMaxItems = (kProgBytes - kStepBytes) / (int)sizeof(Item);
 constexpr int kMaxCtas = 255;      // the 8-bit contribution count of the exchange
+constexpr int kMaxSlots = 64;      // row units of a residual step
+#ifndef LB_ROW_MIN_LNR
+#define LB_ROW_MIN_LNR 3
+#endif
+constexpr int kRowMinLnr = LB_ROW_MIN_LNR;  // smallest row unit: 1 << kRowMinLnr rows
 
 struct Params {
     const LinDesc *lin;  // 7 * n_layers descriptors in the workspace
@@ -195,86 +204,85 @@ __device__ __forceinline__ void item_at(int prog, int u, int4 &a, int4 &b) {
     b = *reinterpret_cast<const int4 *>(p + 16);
 }
 
-// Row units: 16 output rows of a stage-2 step summed whole inside one warp,
-// then the stage-1 tables of those rows, with no shared accumulator and no
-// barrier in between.  Lanes 0-15 take the rows with the first segment of
-// every pair, lanes 16-31 the same rows with the second (the two halves read
-// the two copies of every table, so their lookups never share a bank); one
-// shuffle joins the halves into x (by the unit's mode).  Table job j then
-// gets the unit's four tables, table n of v_i = x_i * g_j[i], i = 4n + k,
-// built by lane 4j + n.  do_s2 = false takes A = B = 0 (the first layer has
-// no previous down); do_tab = false builds no tables (the last phase).
-__device__ __noinline__ void run_rows(int prog, int s, bool do_s2, bool do_tab, int ss_off) {
+// Row units: nr = 16, 8 or 4 output rows of a stage-2 step summed whole
+// inside one warp, then the stage-1 tables of those rows, with no shared
+// accumulator and no barrier in between.  Lane l takes row l mod nr and lane
+// group l / nr: the groups of lanes 0-15 split the words of the first half
+// of the work (path 0, or gate in phase D) and those of lanes 16-31 the
+// second (path 1, or up), each group a run of words of one or more segments.
+// The two half-warps read the two copies of every table.  Shuffles join the
+// groups into x (by the unit's mode; a butterfly, so every lane of a row gets
+// the same value).  Table job j then gets the unit's nr / 4 tables, table n
+// of v_i = x_i * g_j[i], i = 4n + k.  do_s2 = false takes A = B = 0 (the
+// first layer has no previous down); do_tab = false builds no tables (the
+// last phase).  ROW_RES units leave the sum of squares of their rows in
+// ss[slot] (added in slot order later, so the total does not depend on
+// which warp finishes first).
+__device__ __noinline__ void run_rows(int prog, int s, bool do_s2, bool do_tab, float *ss) {
     const Step &st = step_at(prog, s);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int half = lane >> 4, r = lane & 15;
-    const uint32_t copy = half ? 0x40404040u : 0u;
+    const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
     const int u1 = st.first + st.wo[warp + 1];
     for (int u = st.first + st.wo[warp]; u < u1;) {
         int4 hd, he;
         item_at(prog, u, hd, he);
-        const int npair = hd.x, njob = hd.y, mode = hd.z, nrows = hd.w;
-        const int row = min(r, nrows - 1);
+        const int nseg = hd.x, njob = hd.y, mode = hd.z & 0xff, lnr = hd.z >> 8, nrows = hd.w;
+        const int nr = 1 << lnr, G = 32 >> lnr;
+        const int row = min(lane & (nr - 1), nrows - 1);
+        const int seg0 = u + 1 + (lane >> lnr) * nseg;
+        // the residual input does not depend on the sums: load it first
+        const float res = mode == ROW_RES && lane < nrows ? sm_f(he.x)[lane] : 0.f;
         float acc = 0.f;
         if (do_s2) {
-            for (int k = 0; k < npair; ++k) {
-                int4 a0, b0, a1, b1;
-                item_at(prog, u + 1 + 2 * k, a0, b0);
-                item_at(prog, u + 2 + 2 * k, a1, b1);
-                // a segment without words points at its partner's rows and
-                // tables: its clamped reads stay in place and are masked out
-                const int nw = half ? a1.z : a0.z, nwm = max(a0.z, a1.z);
-                const uint32_t *Uw = sm_u32(half ? a1.x : a0.x) + row * (half ? a1.y : a0.y);
-                const uint32_t tb = (uint32_t)(half ? a1.w : a0.w);
+#pragma unroll 1
+            for (int k = 0; k < nseg; ++k) {
+                int4 a, b;
+                item_at(prog, seg0 + k, a, b);
+                const int nw = a.z;
+                const uint32_t *Uw = sm_u32(a.x) + row * a.y;
+                const uint32_t tb = (uint32_t)a.w;
                 float s0 = 0.f, s1 = 0.f;
-                if (a0.z == a1.z) {
-                    // both halves sum the same number of words: no clamps, no masks
-                    int w = 0;
+                int w = 0;
 #pragma unroll 1
-            #pragma unroll 1
-        for (; w + 2 <= nw; w += 2) {
-                        s0 += lut_word(Uw[w], copy, tb + w * 1024);
-                        s1 += lut_word(Uw[w + 1], copy, tb + (w + 1) * 1024);
-                    }
-                    if (w < nw) s0 += lut_word(Uw[w], copy, tb + w * 1024);
-                } else {
-#pragma unroll 1
-                    for (int w = 0; w < nwm; w += 2) {
-                        const int wa = max(min(w, nw - 1), 0), wb = max(min(w + 1, nw - 1), 0);
-                        const float va = lut_word(Uw[wa], copy, tb + wa * 1024);
-                        const float vb = lut_word(Uw[wb], copy, tb + wb * 1024);
-                        s0 += w < nw ? va : 0.f;
-                        s1 += w + 1 < nw ? vb : 0.f;
-                    }
+                for (; w + 2 <= nw; w += 2) {
+                    s0 += lut_word(Uw[w], copy, tb + w * 1024);
+                    s1 += lut_word(Uw[w + 1], copy, tb + (w + 1) * 1024);
                 }
-                const float h = half_bits_to_float(sm_u16(half ? b1.x : b0.x)[row]);
-                acc += nw > 0 ? (s0 + s1) * h : 0.f;
+                if (w < nw) s0 += lut_word(Uw[w], copy, tb + w * 1024);
+                if (nw > 0) acc += (s0 + s1) * half_bits_to_float(sm_u16(b.x)[row]);
             }
         }
-        const float other = __shfl_xor_sync(0xffffffffu, acc, 16);
-        float x = mode == ROW_SILU ? silu(acc) * other : acc + other;
-        if (lane >= nrows) x = 0.f;  // also every lane of the second half
+        float x = acc;
+        if (mode == ROW_SILU) {
+            // gate in lanes 0-15, up in lanes 16-31
+            for (int o = nr; o < 16; o <<= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+            const float other = __shfl_xor_sync(0xffffffffu, x, 16);
+            x = silu(x) * other;
+        } else {
+            for (int o = nr; o < 32; o <<= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+        }
+        if (lane >= nrows) x = 0.f;  // also every lane beyond the unit's rows
         if (mode == ROW_RES) {
-            float ss = 0.f;
+            float q = 0.f;
             if (lane < nrows) {
-                x += sm_f(he.x)[lane];
+                x += res;
                 sm_f(he.y)[lane] = x;
-                ss = x * x;
+                q = x * x;
             }
-#pragma unroll
-            for (int o = 8; o > 0; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
-            if (lane == 0) atomicAdd(sm_f(ss_off), ss);
+            for (int o = nr >> 1; o > 0; o >>= 1) q += __shfl_xor_sync(0xffffffffu, q, o);
+            if (lane == 0) ss[he.z] = q;
         }
         if (do_tab) {
-            const int n = lane & 3;
+            const int ltj = lnr - 2;  // log2 of the tables per job
+            const int n = lane & ((1 << ltj) - 1);
             const float4 v = make_float4(__shfl_sync(0xffffffffu, x, 4 * n),
                                          __shfl_sync(0xffffffffu, x, 4 * n + 1),
                                          __shfl_sync(0xffffffffu, x, 4 * n + 2),
                                          __shfl_sync(0xffffffffu, x, 4 * n + 3));
 #pragma unroll 1
-            for (int L = lane; L < 4 * njob; L += 32) {
+            for (int L = lane; L < (njob << ltj); L += 32) {
                 int4 ta, tz;
-                item_at(prog, u + 1 + 2 * npair + (L >> 2), ta, tz);
+                item_at(prog, u + 1 + G * nseg + (L >> ltj), ta, tz);
                 const uint2 hb = *reinterpret_cast<const uint2 *>(g_smem + ta.y + 8 * n);
                 const float4 t =
                     make_float4(v.x * half_bits_to_float((uint16_t)(hb.x & 0xffffu)),
@@ -284,7 +292,7 @@ __device__ __noinline__ void run_rows(int prog, int s, bool do_s2, bool do_tab, 
                 store_table(g_smem + ta.x + 128 * n, t, lane);
             }
         }
-        u += 1 + 2 * npair + njob;
+        u += 1 + G * nseg + njob;
     }
 }
 
@@ -829,14 +837,14 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
     const int rows_d = 32 * s.nd, nkv = s.nkv;
     float *res0 = sm_f(o.res0), *res1 = sm_f(o.res1), *yq = sm_f(o.yq);
     float *yk = sm_f(o.yk), *yv = sm_f(o.yv);
-    float *ssacc = sm_f(o.ssacc);  // sum of squares of this CTA's slice
+    float *ssslot = sm_f(o.ssslot);  // per-unit sums of squares (residual row steps)
     for (int i = threadIdx.x; i < rows_d; i += kCT) {
         res0[i] = bf16_bits_to_float(P.x0[32 * s.dw0 + i]);
         yq[i] = 0.f;
     }
     zero_f(yk, nkv);
     zero_f(yv, nkv);
-    if (threadIdx.x == 0) ssacc[0] = 0.f;
+    for (int i = threadIdx.x; i < kMaxSlots; i += kCT) ssslot[i] = 0.f;
     {
         // ||x0||_1 <= kCT x the largest per-thread share (every CTA alike)
         float a = 0.f;
@@ -865,17 +873,20 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         csync();
         if (lead) mbar_arrive(empty + b);
     };
-    // this CTA's share of the mean square (sum / d); its bound is B^2 / d
-    // for B the L1 norm of the vector.  The lead also clears the phase's
-    // |z| maxima: every compute thread read them before the barrier that
-    // precedes this call.
-    auto send_ss = [&](unsigned long long *p, float2 sc, int X) {
+    // The lead sends this CTA's share of the mean square (sum / d: the row
+    // step's slots added in slot order, zero for a CTA without rows) once
+    // its own stage-1 units are out, so the sum is off the critical path;
+    // the share's bound is B^2 / d for B the L1 norm of the vector.
+    auto send_ss = [&](unsigned long long *p, float2 sc, int step) {
         if (lead) {
-            send_fix1(p, ssacc[0] * inv_d, sc.x, P.lim_ss, err);
-            ssacc[0] = 0.f;
+            const int n = step_at(pg, step).nslot;
+            float q = 0.f;
+            for (int i = 0; i < n; ++i) q += ssslot[i];
+            send_fix1(p, q * inv_d, sc.x, P.lim_ss, err);
         }
-        if (threadIdx.x < 4) s_zmax[X][threadIdx.x] = 0u;
     };
+    // Threads 0-3 clear a phase's |z| maxima once every compute thread has
+    // read them (after the barrier that follows the row step).
     auto clear_z = [&](int X) {
         if (threadIdx.x < 4) s_zmax[X][threadIdx.x] = 0u;
     };
@@ -899,12 +910,15 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         }
         scA = fix1_scale(cst(0, 1).x * Ba, n_tc);  // |t| <= max|g| ||a||
         ssA = fix1_scale(Ba * Ba * inv_d, n_cc);
-        run_rows(pg, A_R, l > 0, true, o.ssacc);  // a = res0 + Down(m) -> res1; tables
+        run_rows(pg, A_R, l > 0, true, ssslot);  // a = res0 + Down(m) -> res1; tables
         csync();
-        send_ss(xl + P.offA + ssA_el, ssA, 0);
-        if (!csync_and(run_s1(pg, A_S1, xl, scA.x, P.lim_t, err, o.slot[0], o.ubar0[0], o.ubar,
-                              par, rank, P.ws_words)))
-            FAIL_EXIT();
+        clear_z(0);
+        {
+            const bool ok1 = run_s1(pg, A_S1, xl, scA.x, P.lim_t, err, o.slot[0], o.ubar0[0],
+                                    o.ubar, par, rank, P.ws_words);
+            send_ss(xl + P.offA + ssA_el, ssA, A_R);
+            if (!csync_and(ok1)) FAIL_EXIT();
+        }
         // regions C and Q of the previous layer: every CTA has passed the
         // poll that read them (exchange D, polled above, counts all CTAs)
         if (l > 0) {
@@ -924,7 +938,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
             const float4 c = cst(1, 0);
             scB = fix1_scale(cst(1, 1).x * (c.x * zm(1, 0) + c.y * zm(1, 1)), n_tc);
         }
-        run_rows(pg, B_R, true, true, o.ssacc);  // v on the attention rows; tables of o
+        run_rows(pg, B_R, true, true, ssslot);  // v on the attention rows; tables of o
         csync();
         clear_z(1);
         if (!csync_and(run_s1(pg, B_S1, xl, scB.x, P.lim_t, err, o.slot[1], o.ubar0[1], o.ubar,
@@ -959,12 +973,15 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
             scC = fix1_scale(cst(2, 1).x * Bh, n_tc);
             ssC = fix1_scale(Bh * Bh * inv_d, n_cc);
         }
-        run_rows(pg, C_R, true, true, o.ssacc);  // h = res1 + O(attn) -> res0; tables
+        run_rows(pg, C_R, true, true, ssslot);  // h = res1 + O(attn) -> res0; tables
         csync();
-        send_ss(xl + P.offC + ssC_el, ssC, 2);
-        if (!csync_and(run_s1(pg, C_S1, xl, scC.x, P.lim_t, err, o.slot[2], o.ubar0[2], o.ubar,
-                              par, rank, P.ws_words)))
-            FAIL_EXIT();
+        clear_z(2);
+        {
+            const bool ok1 = run_s1(pg, C_S1, xl, scC.x, P.lim_t, err, o.slot[2], o.ubar0[2],
+                                    o.ubar, par, rank, P.ws_words);
+            send_ss(xl + P.offC + ssC_el, ssC, C_R);
+            if (!csync_and(ok1)) FAIL_EXIT();
+        }
         zero_stripe(at(xl, P.offA), s_zs[XR_A]);  // read by phase B's poll
         release(2);
 
@@ -979,7 +996,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
             const float Bm = (c.x * zm(3, 0) + c.y * zm(3, 1)) * (c.z * zm(3, 2) + c.w * zm(3, 3));
             scD = fix1_scale(cst(3, 1).x * Bm, n_tc);
         }
-        run_rows(pg, D_R, true, true, o.ssacc);  // m = silu(gate) * up; tables of down
+        run_rows(pg, D_R, true, true, ssslot);  // m = silu(gate) * up; tables of down
         csync();
         clear_z(3);
         if (!csync_and(run_s1(pg, D_S1, xl, scD.x, P.lim_t, err, o.slot[3], o.ubar0[3], o.ubar,
@@ -998,7 +1015,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
             FAIL_EXIT();
         zero_stripe(at(xp, P.offC), s_zs[XR_C]);
         zero_stripe(at(xp, P.offQ), s_zs[XR_Q]);
-        run_rows(pg, A_R, true, false, o.ssacc);  // a = res0 + Down(m) -> res1
+        run_rows(pg, A_R, true, false, ssslot);  // a = res0 + Down(m) -> res1
         csync();
         for (int i = threadIdx.x; i < rows_d; i += kCT) P.out[32 * s.dw0 + i] = res1[i];
         // The last CTA to finish has seen every other CTA's reads of the final
@@ -1295,7 +1312,7 @@ SmemPlan smem_plan(const lb_linear *lin, const StackShape &sh, int N) {
     o.yq = take(4 * 32 * nd);
     o.yk = take(4 * nkv);
     o.yv = take(4 * nkv);
-    o.ssacc = take(16);
+    o.ssslot = take(4 * kMaxSlots);
     o.prog = take(kProgBytes);
     // cluster reduction: per phase, the receive slots and mbarriers of the
     // ceil(units / kCluster) stage-1 units a rank owns at most
@@ -1384,6 +1401,7 @@ struct S1Job {
 struct ProgBuild {
     Step step[N_STEPS] = {};
     std::vector<Item> items;
+    int min_lnr = kRowMinLnr;  // smallest log2 rows per row unit (4: only the two halves)
 
     void place(int s, const std::vector<Item> &grouped, const int (&wo)[kCW + 1]) {
         step[s].first = (int)items.size();
@@ -1398,62 +1416,108 @@ struct ProgBuild {
             step[s].wo[w + 1] = (int)items.size() - step[s].first;
         }
     }
-    // Row units of a stage-2 step (16 rows each, see run_rows): pairs of
-    // segments given at row 0, the table jobs of the rows, the mode and the
-    // residual buffers.  Units go to the warps longest first (cost: the words
-    // of the longer segment of each pair plus a fixed overhead).
-    void rows(int s, const std::vector<std::pair<Seg, Seg>> &pairs,
-              const std::vector<TabJob> &jobs, int mode, int res_in, int res_out, int nrows) {
+    // Row units of a stage-2 step (see run_rows): the work of lanes 0-15 and
+    // of lanes 16-31 as segments given at row 0 (half[0], half[1]), the table
+    // jobs of the rows, the mode and the residual buffers.  The rows per unit
+    // (16, 8 or 4: 2, 4 or 8 lane groups, each half's words split evenly
+    // over its groups) minimise the estimated makespan over the warps (in
+    // sign words per lane: a fixed cost per unit, the longest group's words,
+    // the mode and the table jobs); units go to the warps longest first.
+    // Returns false when a residual step needs more than kMaxSlots units.
+    bool rows(int s, const std::vector<Seg> (&half)[2], const std::vector<TabJob> &jobs,
+              int mode, int res_in, int res_out, int nrows) {
         struct Unit {
             std::vector<Item> it;
             double cost;
         };
-        std::vector<Unit> us;
-        for (int r0 = 0; r0 < nrows; r0 += 16) {
-            Unit U{{}, 2.0 + jobs.size() / 8.0};
-            U.it.push_back(Item{{(int)pairs.size(), (int)jobs.size(), mode,
-                                 std::min(16, nrows - r0), res_in + 4 * r0, res_out + 4 * r0, 0,
-                                 0}});
-            for (const auto &pr : pairs) {
-                for (const Seg *g : {&pr.first, &pr.second})
-                    U.it.push_back(Item{{g->U + 4 * r0 * g->R, g->R, g->nw, g->tb, g->h + 2 * r0,
-                                         0, 0, 0}});
-                U.cost += std::max(pr.first.nw, pr.second.nw);
+        std::vector<Unit> best;
+        double best_mk = 1e300;
+        for (int lnr = 4; lnr >= min_lnr; --lnr) {
+            const int nr = 1 << lnr, G = 32 >> lnr, gh = G / 2;
+            // each half's words in gh runs: group g of half h covers words
+            // [g W / gh, (g + 1) W / gh) of the half's segments laid end to end
+            std::vector<std::vector<Seg>> grp(G);
+            int maxw = 0;
+            for (int h = 0; h < 2; ++h) {
+                int W = 0;
+                for (const Seg &g : half[h]) W += g.nw;
+                for (int g = 0; g < gh; ++g) {
+                    const int w0 = (int)((long long)g * W / gh), w1 = (int)((long long)(g + 1) * W / gh);
+                    maxw = std::max(maxw, w1 - w0);
+                    int base = 0;
+                    for (const Seg &sg : half[h]) {
+                        const int a = std::max(w0, base), b = std::min(w1, base + sg.nw);
+                        if (a < b)
+                            grp[h * gh + g].push_back({sg.U + 4 * (a - base), sg.R, b - a,
+                                                       sg.tb + 1024 * (a - base), sg.h});
+                        base += sg.nw;
+                    }
+                }
             }
-            for (const TabJob &J : jobs)
-                U.it.push_back(Item{{J.tb + 128 * (r0 / 4), J.g + 2 * r0, 0, 0, 0, 0, 0, 0}});
-            us.push_back(U);
+            size_t nseg = 1;
+            for (const auto &g : grp) nseg = std::max(nseg, g.size());
+            // pad with segments without words (their reads are never made)
+            for (int g = 0; g < G; ++g) {
+                const Seg pad = grp[g].empty() ? half[g / gh].front() : grp[g].front();
+                while (grp[g].size() < nseg) grp[g].push_back({pad.U, pad.R, 0, pad.tb, pad.h});
+            }
+            const int ntab = (int)jobs.size() * (nr / 4);
+            const double cost = 3.0 + maxw + 0.5 * (double)(nseg - 1) +
+                                (mode == ROW_RES ? 1.0 : 0.5) + (ntab > 0 ? 2.0 : 0.0) +
+                                (ntab > 32 ? 2.0 : 0.0);
+            std::vector<Unit> us;
+            int slot = 0;
+            for (int r0 = 0; r0 < nrows; r0 += nr, ++slot) {
+                Unit U{{}, cost};
+                U.it.push_back(Item{{(int)nseg, (int)jobs.size(), mode | (lnr << 8),
+                                     std::min(nr, nrows - r0), res_in + 4 * r0, res_out + 4 * r0,
+                                     slot, 0}});
+                for (int g = 0; g < G; ++g)
+                    for (const Seg &sg : grp[g])
+                        U.it.push_back(Item{{sg.U + 4 * r0 * sg.R, sg.R, sg.nw, sg.tb,
+                                             sg.h + 2 * r0, 0, 0, 0}});
+                for (const TabJob &J : jobs)
+                    U.it.push_back(Item{{J.tb + 128 * (r0 / 4), J.g + 2 * r0, 0, 0, 0, 0, 0, 0}});
+                us.push_back(U);
+            }
+            const double mk = std::ceil((double)us.size() / kCW) * cost;
+            if (mk < best_mk - 1e-9) {
+                best_mk = mk;
+                best = us;
+            }
         }
-        std::vector<int> idx(us.size());
-        for (size_t i = 0; i < us.size(); ++i) idx[i] = (int)i;
-        std::stable_sort(idx.begin(), idx.end(),
-                         [&](int a, int b) { return us[a].cost > us[b].cost; });
+        if (mode == ROW_RES && (int)best.size() > kMaxSlots) return false;
         PerWarp per;
         double load[kCW] = {};
-        for (int i : idx) {
+        for (const Unit &U : best) {
             int w = 0;
             for (int k = 1; k < kCW; ++k)
                 if (load[k] < load[w]) w = k;
-            load[w] += us[i].cost;
-            per[w].insert(per[w].end(), us[i].it.begin(), us[i].it.end());
+            load[w] += U.cost;
+            per[w].insert(per[w].end(), U.it.begin(), U.it.end());
         }
         place(s, per);
+        step[s].nslot = mode == ROW_RES ? (int)best.size() : 0;
+        return true;
     }
-    // The segment pair of one linear summed over its paths: path 0 beside
-    // path 1, or one path split into two runs of words.
-    static std::pair<Seg, Seg> sum_pair(const Seg &p0, const Seg *p1) {
-        if (p1) return {p0, *p1};
-        Seg a = p0, b = p0;
-        a.nw = (p0.nw + 1) / 2;
-        b.nw = p0.nw - a.nw;
-        if (b.nw > 0) {
-            b.U += 4 * a.nw;
-            b.tb += 1024 * a.nw;
-        } else {
-            b = a;
-            b.nw = 0;
+    // The two halves of one linear summed over its paths: path 0 beside
+    // path 1, or one path's words split between the halves.
+    static void halves_of(const std::vector<Seg> &g, std::vector<Seg> (&half)[2]) {
+        half[0].clear();
+        half[1].clear();
+        if (g.size() > 1) {
+            half[0].push_back(g[0]);
+            half[1].push_back(g[1]);
+            return;
         }
-        return {a, b};
+        Seg a = g[0], b = g[0];
+        a.nw = (g[0].nw + 1) / 2;
+        b.nw = g[0].nw - a.nw;
+        b.U += 4 * a.nw;
+        b.tb += 1024 * a.nw;
+        half[0].push_back(a);
+        if (b.nw > 0) half[1].push_back(b);
+        else half[1].push_back({a.U, a.R, 0, a.tb, a.h});
     }
     // Poll-table units: the same split, word indices instead of offsets.
     void ptables(int s, const std::vector<Item> &jobs) {
@@ -1524,8 +1588,11 @@ struct ProgBuild {
 };
 
 // The program of CTA c (kProgBytes, zero-padded); false when it does not fit.
-bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, const Offsets &o,
-                   const XLayout &X, std::vector<int> &prog_out) {
+// Row units of 8 or 4 rows take more records: a program that does not fit
+// with them is built again with 16-row units only.
+bool build_program_at(const lb_linear *lin, const StackShape &sh, int N, int c,
+                      const Offsets &o, const XLayout &X, int min_lnr,
+                      std::vector<int> &prog_out) {
     const int Wd = sh.d / 32, Wf = sh.dff / 32, Ukv = sh.dkv / 8;
     const int dw0 = (int)((long long)c * Wd / N), nd = (int)((long long)(c + 1) * Wd / N) - dw0;
     const int fw0 = (int)((long long)c * Wf / N), nf = (int)((long long)(c + 1) * Wf / N) - fw0;
@@ -1535,6 +1602,7 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
     auto rk = [&](int k, int p) { return lin[k].path[p].r; };
     auto Rk = [&](int k, int p) { return (lin[k].path[p].r + 31) / 32; };
     ProgBuild B;
+    B.min_lnr = min_lnr;
     std::vector<Item> T;
     std::vector<S2Job> U;
     std::vector<S1Job> V;
@@ -1551,9 +1619,7 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
         B.s1(s, V, rank);
         V.clear();
     };
-    auto pair_of = [](const std::vector<Seg> &g) {
-        return ProgBuild::sum_pair(g[0], g.size() > 1 ? &g[1] : nullptr);
-    };
+    std::vector<Seg> hv[2];
     // phase A: stage 2 of down (previous layer) in row units, a = res0 +
     // Down(m) written to res1, the stage-1 tables of q, k, v; stage 1 of q, k, v
     {
@@ -1577,7 +1643,8 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
                 tb1 += nd * 1024;
                 dst += rk(k, p);
             }
-        B.rows(A_R, {pair_of(g)}, tj, ROW_RES, o.res0, o.res1, rows_d);
+        ProgBuild::halves_of(g, hv);
+        if (!B.rows(A_R, hv, tj, ROW_RES, o.res0, o.res1, rows_d)) return false;
         flush_v(A_S1);
     }
     // phase B: tables of v, q, k (scaled by the rms factor of a); v on the
@@ -1622,7 +1689,8 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
             tb1 += nd * 1024;
             dst += rk(LO, p);
         }
-        B.rows(B_R, {pair_of(g)}, tj, ROW_SUM, 0, 0, rows_d);
+        ProgBuild::halves_of(g, hv);
+        B.rows(B_R, hv, tj, ROW_SUM, 0, 0, rows_d);
         flush_v(B_S1);
         U = Uqkv;
         flush_u(B_S2QKV);
@@ -1648,7 +1716,8 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
                 tb1 += nd * 1024;
                 dst += rk(k, p);
             }
-        B.rows(C_R, {pair_of(g)}, tj, ROW_RES, o.res1, o.res0, rows_d);
+        ProgBuild::halves_of(g, hv);
+        if (!B.rows(C_R, hv, tj, ROW_RES, o.res1, o.res0, rows_d)) return false;
         flush_v(C_S1);
     }
     // phase D: stage 2 of gate (lanes 0-15) and up (lanes 16-31) in row
@@ -1667,14 +1736,6 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
                 off += rk(k, p);
             }
         flush_p(D_P2);
-        std::vector<std::pair<Seg, Seg>> pairs;
-        for (size_t p = 0; p < std::max(gs[0].size(), gs[1].size()); ++p) {
-            Seg a = p < gs[0].size() ? gs[0][p] : gs[1][p];
-            Seg b = p < gs[1].size() ? gs[1][p] : gs[0][p];
-            if (p >= gs[0].size()) a.nw = 0;
-            if (p >= gs[1].size()) b.nw = 0;
-            pairs.push_back({a, b});
-        }
         std::vector<TabJob> tj;
         int tb1 = o.t1, dst = X.offD;
         for (int p = 0; p < np(LD); ++p) {
@@ -1683,7 +1744,7 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
             tb1 += nf * 1024;
             dst += rk(LD, p);
         }
-        B.rows(D_R, pairs, tj, ROW_SILU, 0, 0, rows_f);
+        B.rows(D_R, gs, tj, ROW_SILU, 0, 0, rows_f);
         flush_v(D_S1);
     }
     if ((int)B.items.size() > kMaxItems) return false;
@@ -1691,6 +1752,12 @@ bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, con
     std::memcpy(prog_out.data(), B.step, sizeof(B.step));
     std::memcpy(prog_out.data() + kStepBytes / 4, B.items.data(), B.items.size() * sizeof(Item));
     return true;
+}
+
+bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, const Offsets &o,
+                   const XLayout &X, std::vector<int> &prog_out) {
+    return build_program_at(lin, sh, N, c, o, X, kRowMinLnr, prog_out) ||
+           build_program_at(lin, sh, N, c, o, X, 4, prog_out);
 }
 
 bool build_programs(const lb_linear *lin, const StackShape &sh, int N, std::vector<int> &all) {
