@@ -502,7 +502,8 @@ __device__ __forceinline__ void zero_stripe(unsigned long long *region, const in
 // thread) on failure.
 __device__ __noinline__ bool run_poll_tables(int prog, int s, const unsigned long long *xbase,
                                              unsigned n_t, unsigned n_ss, float inv, float it,
-                                             float iss, unsigned *zmax, unsigned *ws_words) {
+                                             float iss, unsigned *zmax, bool late,
+                                             unsigned *ws_words) {
     const Step &st = step_at(prog, s);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     int ok = 1;
@@ -510,46 +511,59 @@ __device__ __noinline__ bool run_poll_tables(int prog, int s, const unsigned lon
     for (int u = st.first + st.wo[warp]; u < u1 && ok; ++u) {
         int4 a, b;
         item_at(prog, u, a, b);
-        // lane 0 first waits for the unit's last word (its stage-1 column
-        // block is sent after those of the unit's other words): one poller
-        // per warp keeps the L2 free for the contributions still arriving,
-        // and once it sees its word complete the whole unit usually is
-        if (lane == 0 && a.z > 0) {
-            const unsigned long long t0 = globaltimer_ns();
-            const unsigned long long *gw = xbase + b.x + (min(a.z, 4 * a.y) - 1);
-            for (int spin = 0; !counted1(ld_relaxed_u64(gw), n_t); ++spin)
-                if ((spin & 15) == 15 && globaltimer_ns() - t0 > kWaitLimitNs) break;
-        }
-        __syncwarp();
         const bool have = lane < a.y && a.z - 4 * lane > 0;
         const bool need_ss = have && (a.w & TAB_MUL) && b.z >= 0;
         const unsigned long long *w = xbase + b.x + 4 * lane;
         unsigned long long v0 = 0, v1 = 0, v2 = 0, v3 = 0, vs = 0, t0 = 0;
-        for (int spin = 0; have; ++spin) {
+        auto complete = [&]() {
+            return counted1(v0, n_t) && counted1(v1, n_t) && counted1(v2, n_t) &&
+                   counted1(v3, n_t) && (!need_ss || counted1(vs, n_ss));
+        };
+        // late: the step starts when its exchange has usually completed
+        // (phase C, behind the off-path q, k, v work), so every lane reads
+        // once first -- one round trip to the L2.  (Early, such reads only
+        // load the L2 while the contributions arrive.)
+        if (late && have) {
             ld_relaxed_v2_u64(w, v0, v1);
             ld_relaxed_v2_u64(w + 2, v2, v3);
             if (need_ss) vs = ld_relaxed_u64(xbase + b.z);
-            if (counted1(v0, n_t) && counted1(v1, n_t) && counted1(v2, n_t) &&
-                counted1(v3, n_t) && (!need_ss || counted1(vs, n_ss)))
-                break;
-            if ((spin & 15) == 15) {
-                if (sticky(ws_words)) {
-                    ok = 0;
-                    break;
-                }
-                const unsigned long long now = globaltimer_ns();
-                if (t0 == 0) t0 = now;
-                if (now - t0 > kWaitLimitNs) {
-                    record(ws_words, LB_ERR_TIMEOUT);
-                    ok = 0;
-                    break;
+        }
+        if (!late || !__all_sync(0xffffffffu, !have || complete())) {
+            // lane 0 waits for the unit's last word (its stage-1 column block
+            // is sent after those of the unit's other words): one poller per
+            // warp keeps the L2 free for the contributions still arriving,
+            // and once it sees its word complete the whole unit usually is
+            if (lane == 0 && a.z > 0) {
+                const unsigned long long s0 = globaltimer_ns();
+                const unsigned long long *gw = xbase + b.x + (min(a.z, 4 * a.y) - 1);
+                for (int spin = 0; !counted1(ld_relaxed_u64(gw), n_t); ++spin)
+                    if ((spin & 15) == 15 && globaltimer_ns() - s0 > kWaitLimitNs) break;
+            }
+            __syncwarp();
+            for (int spin = 0; have; ++spin) {
+                ld_relaxed_v2_u64(w, v0, v1);
+                ld_relaxed_v2_u64(w + 2, v2, v3);
+                if (need_ss) vs = ld_relaxed_u64(xbase + b.z);
+                if (complete()) break;
+                if ((spin & 15) == 15) {
+                    if (sticky(ws_words)) {
+                        ok = 0;
+                        break;
+                    }
+                    const unsigned long long now = globaltimer_ns();
+                    if (t0 == 0) t0 = now;
+                    if (now - t0 > kWaitLimitNs) {
+                        record(ws_words, LB_ERR_TIMEOUT);
+                        ok = 0;
+                        break;
+                    }
                 }
             }
-        }
-        // every lane of the warp leaves together (the sum below is warp-wide)
-        if (__any_sync(0xffffffffu, !ok)) {
-            ok = 0;
-            break;
+            // every lane of the warp leaves together (the sum below is warp-wide)
+            if (__any_sync(0xffffffffu, !ok)) {
+                ok = 0;
+                break;
+            }
         }
         float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
         if (have) {
@@ -902,7 +916,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         // ================= phase A: a = h + Down_{l-1}(m) on R_c; stage 1 of q, k, v
         if (!wait_full(full + 0, par, P.ws_words)) FAIL_EXIT();
         if (l > 0) {
-            if (!run_poll_tables(pg, A_P2, xp, n_t, n_ctas, 1.f, scD.y, 1.f, s_zmax[0],
+            if (!run_poll_tables(pg, A_P2, xp, n_t, n_ctas, 1.f, scD.y, 1.f, s_zmax[0], false,
                                  P.ws_words))
                 FAIL_EXIT();
             const float4 c = cst(0, 0);
@@ -930,7 +944,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         // ================= phase B: v rows for attention, stage 1 of o; then q, k, v out
         if (!wait_full(full + 1, par, P.ws_words)) FAIL_EXIT();
         // tables of v (critical) and of q, k (region Q, sent with region A)
-        if (!run_poll_tables(pg, B_P2, xl, n_t, n_ctas, 1.f, scA.y, ssA.y, s_zmax[1],
+        if (!run_poll_tables(pg, B_P2, xl, n_t, n_ctas, 1.f, scA.y, ssA.y, s_zmax[1], false,
                              P.ws_words))
             FAIL_EXIT();
         {
@@ -964,7 +978,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
 
         // ================= phase C: h = a + O(attn) on R_c; stage 1 of gate, up
         if (!wait_full(full + 2, par, P.ws_words)) FAIL_EXIT();
-        if (!run_poll_tables(pg, C_P2, xl, n_t, n_ctas, 1.f, scB.y, 1.f, s_zmax[2],
+        if (!run_poll_tables(pg, C_P2, xl, n_t, n_ctas, 1.f, scB.y, 1.f, s_zmax[2], true,
                              P.ws_words))
             FAIL_EXIT();
         {
@@ -987,7 +1001,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
 
         // ================= phase D: m = silu(gate) * up on F_c; stage 1 of down
         if (!wait_full(full + 3, par, P.ws_words)) FAIL_EXIT();
-        if (!run_poll_tables(pg, D_P2, xl, n_t, n_ctas, 1.f, scC.y, ssC.y, s_zmax[3],
+        if (!run_poll_tables(pg, D_P2, xl, n_t, n_ctas, 1.f, scC.y, ssC.y, s_zmax[3], false,
                              P.ws_words))
             FAIL_EXIT();
         {
@@ -1011,7 +1025,8 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         const int l = P.n_layers;
         unsigned long long *xp = P.xacc + (size_t)(l - 1) * P.acc_layer;
         if (!wait_full(full + 0, (unsigned)(l & 1), P.ws_words)) FAIL_EXIT();
-        if (!run_poll_tables(pg, A_P2, xp, n_t, n_ctas, 1.f, scD.y, 1.f, s_zmax[0], P.ws_words))
+        if (!run_poll_tables(pg, A_P2, xp, n_t, n_ctas, 1.f, scD.y, 1.f, s_zmax[0], false,
+                             P.ws_words))
             FAIL_EXIT();
         zero_stripe(at(xp, P.offC), s_zs[XR_C]);
         zero_stripe(at(xp, P.offQ), s_zs[XR_Q]);
