@@ -30,6 +30,32 @@ constexpr int kDoneWord = 2;
 constexpr int kEpochWord = 3;  // launches of the single-token kernel on this workspace
 constexpr int kPlanWord = 4;
 
+#ifndef LB_S1_WORDS
+#define LB_S1_WORDS 1
+#endif
+// Stage 1 of the single-token kernels (k_decode, k_decode_multi) runs on the
+// first s1_ctas(W, N) CTAs of the grid, at least kS1Words of the W input
+// words each, the others holding none; an exchange element takes one
+// contribution per stage-1 CTA.  (Concentrating stage 1 on fewer CTAs cuts
+// the exchange's atomics but lengthens those CTAs' share of the ±1 sums:
+// 2 words per CTA measured slower than 1 on the 4096 x 11008 r512 shape.)
+constexpr int kS1Words = LB_S1_WORDS;
+__host__ __device__ inline int s1_ctas(int W, int N) {
+    const int n = (W + kS1Words - 1) / kS1Words;
+    return n < 1 ? 1 : (n > N ? N : n);
+}
+// Input words [w0, w0 + nw) of CTA c.
+__host__ __device__ inline void s1_slice(int W, int N, int c, int &w0, int &nw) {
+    const int n = s1_ctas(W, N);
+    if (c >= n) {
+        w0 = 0;
+        nw = 0;
+        return;
+    }
+    w0 = (int)((long long)c * W / n);
+    nw = (int)((long long)(c + 1) * W / n) - w0;
+}
+
 // Device copy of one linear (paths 0..n_paths-1).
 struct LinDesc {
     int d_in, d_out, n_paths, r[2];

@@ -77,10 +77,16 @@ __global__ void __launch_bounds__(kDT, 1) k_decode(const __grid_constant__ Decod
     const DecodeLayout &o = P.o;
     const int N = gridDim.x, c = blockIdx.x, tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
-    const unsigned n_ctas = (unsigned)N;
-    // input words [iw0, iw0 + nw), output rows [o0, o0 + nrows) (whole octets)
+    // input words [iw0, iw0 + nw) (stage-1 CTAs only), output rows [o0, o0 +
+    // nrows) (whole octets)
     const int W = L.d_in >> 5, Q = L.d_out >> 3;
-    const int iw0 = (int)((long long)c * W / N), nw = (int)((long long)(c + 1) * W / N) - iw0;
+    int iw0, nw;
+    s1_slice(W, N, c, iw0, nw);
+    // contributions per exchange element: the stage-1 CTAs; element 0 also
+    // counts every other CTA once, so that block 0's exchange completes only
+    // after every CTA has read the epoch
+    const int n_s1 = s1_ctas(W, N);
+    const unsigned n_all = (unsigned)N, n_part = (unsigned)n_s1;
     const int q0 = (int)((long long)c * Q / N), nq = (int)((long long)(c + 1) * Q / N) - q0;
     const int o0 = 8 * q0, nrows = 8 * nq;
     const int np = L.n_paths;
@@ -142,7 +148,8 @@ __global__ void __launch_bounds__(kDT, 1) k_decode(const __grid_constant__ Decod
     }
     bool ok = wait_bar(bar + 0, P.ws_words);
     ok = __syncthreads_and(ok) != 0;
-    if (ok) {
+    if (ok && c >= n_s1 && tid == 0) send_count2(fix2_at(xw, 0));
+    if (ok && c < n_s1) {
         const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
         const int cb0 = (L.r[0] + 31) >> 5, cbs = cb0 + (np > 1 ? (L.r[1] + 31) >> 5 : 0);
         for (int u = warp; u < cbs; u += kDW) {
@@ -182,7 +189,7 @@ __global__ void __launch_bounds__(kDT, 1) k_decode(const __grid_constant__ Decod
             unsigned long long a[8], t0 = 0;
             for (int spin = 0;; ++spin) {
                 ld_fix2x4(wd, a);
-                if (counted2x4(a, n_ctas)) break;
+                if (counted2x4(a, idx == 0 ? n_all : n_part, n_part)) break;
                 if ((spin & 15) == 15) {
                     if (ld_relaxed_gpu(err) != 0u) {
                         pok = 0;
@@ -248,7 +255,8 @@ __global__ void __launch_bounds__(kDT, 1) k_decode(const __grid_constant__ Decod
 int up16(int n) { return (n + 15) & ~15; }
 
 DecodeLayout layout_of(const lb_linear &L, int N) {
-    const int nw = (L.d_in / 32 + N - 1) / N, nrows = 8 * ((L.d_out / 8 + N - 1) / N);
+    const int W = L.d_in / 32, n_s1 = s1_ctas(W, N);
+    const int nw = (W + n_s1 - 1) / n_s1, nrows = 8 * ((L.d_out / 8 + N - 1) / N);
     DecodeLayout o{};
     int at = 0;
     auto take = [&at](int bytes) {

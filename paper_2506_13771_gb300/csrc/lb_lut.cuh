@@ -249,6 +249,14 @@ __device__ __forceinline__ bool counted2x4(const unsigned long long (&a)[8], uns
            counted2(a[6], a[7], n);
 }
 
+// The same with n0 contributions expected for the first element (element 0
+// of an exchange, which every CTA counts into) and n for the others.
+__device__ __forceinline__ bool counted2x4(const unsigned long long (&a)[8], unsigned n0,
+                                           unsigned n) {
+    return counted2(a[0], a[1], n0) && counted2(a[2], a[3], n) && counted2(a[4], a[5], n) &&
+           counted2(a[6], a[7], n);
+}
+
 // The sum held by a complete pair, (H 2^47 + L) 2^-64, rounded to nearest
 // fp32 (ties to even): exactly while it fits 64 bits (|H| < 2^15); beyond
 // that from floor(sum / 2^36) with a sticky bit for the dropped remainder

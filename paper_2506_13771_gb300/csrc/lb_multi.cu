@@ -115,13 +115,15 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
     const int warp = tid >> 5, lane = tid & 31, np = P.np;
     // input words [iw0, iw0 + nw), output rows [o0, o0 + nrows) (whole octets)
     const int W = P.d_in >> 5, Q = P.d_out >> 3;
-    const int iw0 = (int)((long long)c * W / N), nw = (int)((long long)(c + 1) * W / N) - iw0;
+    int iw0, nw;
+    s1_slice(W, N, c, iw0, nw);
     const int q0 = (int)((long long)c * Q / N), nq = (int)((long long)(c + 1) * Q / N) - q0;
     const int o0 = 8 * q0, nrows = 8 * nq;
-    // Contributions per exchange word: every CTA for linear 0 (so that no CTA
-    // can still be about to read the epoch when block 0 moves it on), only
-    // the CTAs holding input words for the others.
-    const unsigned n_contrib = (unsigned)(W < N ? W : N), n_first = (unsigned)N;
+    // Contributions per exchange word: the stage-1 CTAs; element 0 of linear
+    // 0 also counts every other CTA once (so that no CTA can still be about
+    // to read the epoch when block 0 moves it on), as does the sum-of-squares
+    // element.
+    const unsigned n_contrib = (unsigned)s1_ctas(W, N), n_first = (unsigned)N;
     const int R0 = (P.r[0] + 31) >> 5, R1 = np > 1 ? (P.r[1] + 31) >> 5 : 0;
     const int cbs = R0 + R1, nt0 = 8 * R0, ntab = 8 * (R0 + R1);
 
@@ -223,9 +225,10 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
         for (int it = 0; it < P.M + kAhead && ok; ++it) {
             if (it == kAhead) prefetch(0);
             // ---------------- stage 1 of linear it
-            if (it == 0 && nw == 0) {
-                // a CTA without input words still counts itself into linear 0's words
-                for (int i = tid; i < P.N1; i += kCT) send_count2(fix2_at(xw, i));
+            if (it == 0 && nw == 0 && tid == 0) {
+                // a CTA without input words still counts itself into linear 0's
+                // element 0
+                send_count2(fix2_at(xw, 0));
             }
             if (it < P.M && nw > 0) {
                 const int m = it;
@@ -321,8 +324,8 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
                         } else {
                             ld_fix2x4(wd, a);
                         }
-                        const unsigned want = mm == 0 ? n_first : n_contrib;
-                        if (counted2x4(a, want)) break;
+                        const unsigned want0 = mm == 0 && idx == 0 ? n_first : n_contrib;
+                        if (counted2x4(a, want0, n_contrib)) break;
                         if ((spin & 15) == 15) {
                             if (ld_relaxed_gpu(err) != 0u) {
                                 pok = 0;
@@ -403,7 +406,8 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
 int up16(int n) { return (n + 15) & ~15; }
 
 MultiLayout layout_of(const lb_linear &L, int N) {
-    const int nw = (L.d_in / 32 + N - 1) / N, nrows = 8 * ((L.d_out / 8 + N - 1) / N);
+    const int W = L.d_in / 32, n_s1 = s1_ctas(W, N);
+    const int nw = (W + n_s1 - 1) / n_s1, nrows = 8 * ((L.d_out / 8 + N - 1) / N);
     MultiLayout o{};
     int at = 0;
     auto take = [&at](int bytes) {
