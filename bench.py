@@ -807,15 +807,15 @@ def run_config(args):
         s70 = inputs.STACK_70B
         sizes = [2 * s70["r_kv"] + 1, 2 * s70["r_qo"], 4 * s70["r_mlp"] + 1, 2 * s70["r_mlp"]]
         rounds = 4 * s70["n_layers"]
-        for cluster in (1, 2):
-            ws = lb.selftest_exchange(rounds, sizes, cluster, device=dev)
+        for words, cluster in ((1, 1), (1, 2), (2, 1), (2, 2)):
+            ws = lb.selftest_exchange(rounds, sizes, cluster, words, device=dev)
             torch.cuda.synchronize(dev)
             times = []
             for _ in range(max(3, args.warmup) + steps):
                 e0 = torch.cuda.Event(enable_timing=True)
                 e1 = torch.cuda.Event(enable_timing=True)
                 e0.record()
-                lb.selftest_exchange(rounds, sizes, cluster, ws=ws, device=dev)
+                lb.selftest_exchange(rounds, sizes, cluster, words, ws=ws, device=dev)
                 e1.record()
                 torch.cuda.synchronize(dev)
                 times.append(e0.elapsed_time(e1))
@@ -823,6 +823,7 @@ def run_config(args):
                 raise RuntimeError("exchange diagnostic reported an error")
             ms = statistics.median(times[max(3, args.warmup):])
             print(json.dumps({"config": 10, "case": "exchange floor", "cluster": cluster,
+                              "words_per_element": words,
                               "sizes": sizes, "rounds": rounds, "ms_per_token": ms,
                               "us_per_exchange": 1e3 * ms / rounds,
                               "us_per_layer": 4e3 * ms / rounds,

@@ -406,10 +406,12 @@ lb_status littlebit_selftest_wait_timeout(void *ws, lb_stream_t stream);
  * rank-r partial sums t = V_sign^T (g . x) of every CTA's input slice,
  * all-reduced across the GPU before stage 2).  One persistent launch, one CTA
  * per SM, runs n_rounds dependent exchanges of sizes[k % n_sizes] elements
- * (1 <= n_sizes <= 8, 1 <= sizes[i] <= 2048) with the encoding, polling and
- * (cluster = 2) two-CTA distributed-shared-memory pre-reduction that
- * littlebit_stack_forward uses, and nothing else: elapsed time / n_rounds is
- * the exchange's cost on the stack's critical path.  ws: 256-byte aligned,
+ * (1 <= n_sizes <= 8, 1 <= sizes[i] <= 2048) with the polling of
+ * littlebit_stack_forward, optionally (cluster = 2) its two-CTA
+ * distributed-shared-memory pre-reduction, and the encoding of the stack
+ * (words = 1: one 64-bit word per element at a bounded scale) or of the
+ * single-linear kernels (words = 2: the exact hi / lo pair), and nothing
+ * else: elapsed time / n_rounds is the exchange's cost on the critical path.  ws: 256-byte aligned,
  * littlebit_selftest_exchange_workspace_size bytes, header zero-filled before
  * the first use (the call clears the rest); an error (a wait that ran out)
  * is recorded in the header like the other kernels', read with
@@ -417,7 +419,7 @@ lb_status littlebit_selftest_wait_timeout(void *ws, lb_stream_t stream);
 size_t littlebit_selftest_exchange_workspace_size(int32_t n_rounds, const int32_t *sizes,
                                                    int32_t n_sizes);
 lb_status littlebit_selftest_exchange(int32_t n_rounds, const int32_t *sizes, int32_t n_sizes,
-                                      int32_t cluster, void *ws, size_t ws_bytes,
+                                      int32_t cluster, int32_t words, void *ws, size_t ws_bytes,
                                       lb_stream_t stream);
 
 #ifdef __cplusplus

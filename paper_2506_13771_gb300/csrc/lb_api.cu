@@ -2,6 +2,7 @@
 // validation, workspace layout and dispatch to the kernels.  See
 // include/littlebit.h for the contract of every function.
 #include <cstdint>
+#include <cstdlib>
 #include <cstring>
 
 #include "lb_common.cuh"
@@ -96,10 +97,19 @@ lb_status check_stack(const lb_linear *lin, int32_t n_layers, int32_t head_dim,
     return LB_OK;
 }
 
-// FNV-1a over the host description of a stack (shapes, ranks and pointers)
-// and the SM count the per-CTA programs were built for.
+// CTAs per thread-block cluster of the stack kernel: 2 when the environment
+// variable LB_STACK_CLUSTER is "2", else 1 (read at every prepare and
+// forward; the fingerprint holds it, so a workspace prepared with the other
+// value is refused with LB_ERR_PLAN).
+int stack_cluster() {
+    const char *v = std::getenv("LB_STACK_CLUSTER");
+    return v && v[0] == '2' && v[1] == '\0' ? 2 : 1;
+}
+
+// FNV-1a over the host description of a stack (shapes, ranks and pointers),
+// the SM count the per-CTA programs were built for and the cluster size.
 unsigned long long stack_fingerprint(const lb_linear *lin, int32_t n_layers, int32_t head_dim,
-                                     int sms) {
+                                     int sms, int cluster) {
     unsigned long long h = 1469598103934665603ull;
     auto mix = [&h](unsigned long long v) {
         for (int b = 0; b < 8; ++b) {
@@ -110,6 +120,7 @@ unsigned long long stack_fingerprint(const lb_linear *lin, int32_t n_layers, int
     mix((unsigned long long)n_layers);
     mix((unsigned long long)head_dim);
     mix((unsigned long long)sms);
+    mix((unsigned long long)cluster);
     for (int i = 0; i < 7 * n_layers; ++i) {
         const lb_linear &L = lin[i];
         mix((unsigned long long)L.d_in);
@@ -432,9 +443,10 @@ lb_status littlebit_stack_prepare(const lb_linear *lin, int32_t n_layers, int32_
         return LB_ERR_WORKSPACE;
     int sms = 0;
     if ((st = num_sms(&sms)) != LB_OK) return st;
-    if ((sms = lb::stack_grid_ctas(lin, shape, sms)) <= 0) return LB_ERR_UNSUPPORTED;
+    const int cl = stack_cluster();
+    if ((sms = lb::stack_grid_ctas(lin, shape, sms, cl)) <= 0) return LB_ERR_UNSUPPORTED;
     const cudaError_t e = lb::launch_stack_prepare(
-        lin, n_layers, shape, sms, stack_fingerprint(lin, n_layers, head_dim, sms),
+        lin, n_layers, shape, sms, cl, stack_fingerprint(lin, n_layers, head_dim, sms, cl),
         static_cast<unsigned *>(ws), static_cast<char *>(ws) + kWsHeader, (cudaStream_t)stream);
     return e == cudaErrorNotSupported ? LB_ERR_UNSUPPORTED : from_cuda(e);
 }
@@ -453,13 +465,13 @@ lb_status littlebit_stack_forward(const lb_linear *lin, int32_t n_layers, int32_
         return LB_ERR_WORKSPACE;
     int sms = 0;
     if ((st = num_sms(&sms)) != LB_OK) return st;
-    if ((sms = lb::stack_grid_ctas(lin, shape, sms)) <= 0) return LB_ERR_UNSUPPORTED;
-    if (!lb::stack_supported(lin, shape, sms)) return LB_ERR_UNSUPPORTED;
+    const int cl = stack_cluster();
+    if ((sms = lb::stack_grid_ctas(lin, shape, sms, cl)) <= 0) return LB_ERR_UNSUPPORTED;
+    if (!lb::stack_supported(lin, shape, sms, cl)) return LB_ERR_UNSUPPORTED;
     return from_cuda(lb::launch_stack(lin, n_layers, shape,
-                                      stack_fingerprint(lin, n_layers, head_dim, sms), x0, out,
-                                      q_out,
-                                      kv_out, static_cast<unsigned *>(ws),
-                                      static_cast<char *>(ws) + kWsHeader, sms,
+                                      stack_fingerprint(lin, n_layers, head_dim, sms, cl), x0,
+                                      out, q_out, kv_out, static_cast<unsigned *>(ws),
+                                      static_cast<char *>(ws) + kWsHeader, sms, cl,
                                       (cudaStream_t)stream));
 }
 
@@ -493,9 +505,10 @@ size_t littlebit_selftest_exchange_workspace_size(int32_t n_rounds, const int32_
 }
 
 lb_status littlebit_selftest_exchange(int32_t n_rounds, const int32_t *sizes, int32_t n_sizes,
-                                      int32_t cluster, void *ws, size_t ws_bytes,
+                                      int32_t cluster, int32_t words, void *ws, size_t ws_bytes,
                                       lb_stream_t stream) {
-    if (n_rounds < 1 || !sizes || n_sizes < 1 || n_sizes > 8 || (cluster != 1 && cluster != 2))
+    if (n_rounds < 1 || !sizes || n_sizes < 1 || n_sizes > 8 || (cluster != 1 && cluster != 2) ||
+        (words != 1 && words != 2))
         return LB_ERR_INVALID_ARG;
     for (int i = 0; i < n_sizes; ++i)
         if (sizes[i] < 1 || sizes[i] > 2048) return LB_ERR_INVALID_ARG;
@@ -505,7 +518,7 @@ lb_status littlebit_selftest_exchange(int32_t n_rounds, const int32_t *sizes, in
     int sms = 0;
     lb_status st = num_sms(&sms);
     if (st != LB_OK) return st;
-    return from_cuda(lb::launch_xchain(n_rounds, sizes, n_sizes, cluster,
+    return from_cuda(lb::launch_xchain(n_rounds, sizes, n_sizes, cluster, words,
                                        static_cast<unsigned *>(ws),
                                        static_cast<char *>(ws) + kWsHeader, sms,
                                        (cudaStream_t)stream));

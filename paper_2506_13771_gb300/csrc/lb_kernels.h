@@ -53,25 +53,27 @@ struct StackShape {
     int n_layers, d, dkv, dff, head_dim;
 };
 size_t stack_ws_bytes_after_header(const lb_linear *lin, int n_layers);
+// `cluster`: CTAs per thread-block cluster, 1 or 2 (with 2 the stage-1
+// partials of a pair meet in distributed shared memory before the exchange).
 // Writes the device descriptor table and the per-CTA programs for num_sms
 // CTAs, zeroes counters and accumulators, and stores the plan fingerprint.
 // cudaErrorNotSupported when the shapes or the programs do not fit.
 cudaError_t launch_stack_prepare(const lb_linear *lin, int n_layers, const StackShape &shape,
-                                 int num_sms, unsigned long long plan, unsigned *ws_words,
-                                 char *ws_after_header, cudaStream_t s);
+                                 int num_sms, int cluster, unsigned long long plan,
+                                 unsigned *ws_words, char *ws_after_header, cudaStream_t s);
 // Whether the one-launch stack kernel handles these shapes on this GPU
 // (ranks multiples of 8, head_dim multiple of 32, d_kv multiple of 8, the
-// shared-memory plan fits).
-bool stack_supported(const lb_linear *lin, const StackShape &shape, int num_sms);
+// shared-memory plan fits, num_sms a multiple of the cluster size).
+bool stack_supported(const lb_linear *lin, const StackShape &shape, int num_sms, int cluster);
 // The grid of the one-launch stack kernel on this GPU: a whole number of
 // co-resident thread-block clusters, at most num_sms CTAs (0: cannot launch).
 // Programs, fingerprints and launches all use this count.
-int stack_grid_ctas(const lb_linear *lin, const StackShape &shape, int num_sms);
+int stack_grid_ctas(const lb_linear *lin, const StackShape &shape, int num_sms, int cluster);
 // One persistent launch; leaves counters and accumulators zeroed.
 cudaError_t launch_stack(const lb_linear *lin, int n_layers, const StackShape &shape,
                          unsigned long long plan, const uint16_t *x0, float *out, float *q_out,
                          float *kv_out, unsigned *ws_words, char *ws_after_header, int num_sms,
-                         cudaStream_t s);
+                         int cluster, cudaStream_t s);
 
 // Many-token path on the tensor cores (lb_prefill.cu).  The latent half
 // writes z = l . ((X . g) V_sign) as fp16 into z16, or as fp32 into z32 when
@@ -143,7 +145,7 @@ cudaError_t launch_wait_timeout(unsigned *ws_words, cudaStream_t s);
 // of sizes[k % n_sizes] elements over the grid (cluster 1 or 2); buf holds
 // n_rounds buffers and is cleared by the launcher.
 size_t xchain_ws_bytes(int n_rounds, const int *sizes, int n_sizes);
-cudaError_t launch_xchain(int n_rounds, const int *sizes, int n_sizes, int cluster,
+cudaError_t launch_xchain(int n_rounds, const int *sizes, int n_sizes, int cluster, int words,
                           unsigned *ws_words, void *buf, int num_sms, cudaStream_t s);
 
 // Sign packing (lb_pack.cu).

@@ -62,14 +62,11 @@ namespace lb {
 namespace {
 
 constexpr int kST = 512;        // threads per CTA
-#ifndef LB_STACK_CLUSTER
-#define LB_STACK_CLUSTER 1
-#endif
-// CTAs per thread-block cluster: the stage-1 partial sums of a cluster's
+// CTAs per thread-block cluster, C (the kernel is built for C = 1 and 2 and
+// chosen at run time): with C = 2 the stage-1 partial sums of a cluster's
 // CTAs meet in distributed shared memory before one exchange contribution
-// per cluster goes out (1: no clusters, every CTA contributes)
-constexpr int kCluster = LB_STACK_CLUSTER;
-static_assert(kCluster >= 1 && kCluster <= 8, "portable cluster sizes");
+// per cluster goes out; with C = 1 every CTA contributes.
+constexpr int kMaxCluster = 2;
 constexpr int kCW = 15;         // compute warps; warp 15 issues the bulk copies
 constexpr int kCT = kCW * 32;   // compute threads
 // ---------------------------------------------------------------- parameters
@@ -97,7 +94,7 @@ struct Offsets {
     // per-unit sums of squares of the residual row steps (kMaxSlots floats)
     int ssslot;
     // cluster reduction of the stage-1 partials, per phase X = A..D: the
-    // receive slots of the units this CTA owns (kCluster x 32 floats each,
+    // receive slots of the units this CTA owns (C x 32 floats each,
     // one row per sending rank) and the index of their first mbarrier in ubar
     int slot[4], ubar0[4], ubar, n_ubar;
 };
@@ -178,6 +175,23 @@ struct Params {
 };
 
 // ---------------------------------------------------------------- small pieces
+
+// Units [w0, w0 + n) of W (32-row words or 8-row octets) owned by CTA c of N.
+// In clusters the clusters split the units evenly in whole multiples of the
+// cluster size and each member takes an equal share: the members' stage-1
+// partials meet in the owner, which would wait for a member with more work.
+// (Units not divisible that way are split per CTA.)
+__host__ __device__ inline void slice_of(int W, int N, int c, int C, int &w0, int &n) {
+    if (C > 1 && W % C == 0 && N % C == 0) {
+        const int Wc = W / C, Nc = N / C, k = c / C;
+        const int u0 = (int)((long long)k * Wc / Nc), u1 = (int)((long long)(k + 1) * Wc / Nc);
+        n = u1 - u0;
+        w0 = C * u0 + (c % C) * n;
+        return;
+    }
+    w0 = (int)((long long)c * W / N);
+    n = (int)((long long)(c + 1) * W / N) - w0;
+}
 
 __device__ __forceinline__ int wordsR(int r) { return (r + 31) >> 5; }
 
@@ -363,6 +377,7 @@ __device__ __forceinline__ void record(unsigned *ws_words, lb_status st) {
 // and the owner adds them to its own in rank order and sends the sum -- one
 // contribution per cluster.  A warp runs the units it does not own first.
 // Returns false (this warp) when an owner's wait ran out.
+template <int C>
 __device__ __noinline__ bool run_s1(int prog, int s, unsigned long long *xbase, float sc,
                                     float limit, unsigned *err, int slot0, int ubar0, int ubar,
                                     unsigned par, unsigned rank, unsigned *ws_words) {
@@ -373,13 +388,13 @@ __device__ __noinline__ bool run_s1(int prog, int s, unsigned long long *xbase, 
     auto bar_of = [&](int slot) {
         return reinterpret_cast<unsigned long long *>(g_smem + ubar) + ubar0 + slot;
     };
-    if (kCluster > 1 && lane == 0) {
+    if (C > 1 && lane == 0) {
         // arm the mbarriers of this warp's own units for this use
         for (int u = u0; u < u1; ++u) {
             int4 a, b;
             item_at(prog, u, a, b);
             if ((unsigned)b.z == rank)
-                mbar_arrive_expect_tx(bar_of(b.w), (unsigned)((kCluster - 1) * 4 * b.y));
+                mbar_arrive_expect_tx(bar_of(b.w), (unsigned)((C - 1) * 4 * b.y));
         }
     }
     __syncwarp();
@@ -387,7 +402,7 @@ __device__ __noinline__ bool run_s1(int prog, int s, unsigned long long *xbase, 
     // one finished unit: its partial v of column `lane`
     auto finish = [&](const int4 &b, float v) {
         const int dst = b.x, ncols = b.y;
-        if (kCluster == 1) {
+        if (C == 1) {
             if (lane < ncols) send_fix1(xbase + dst + lane, v, sc, limit, err);
             return;
         }
@@ -396,7 +411,7 @@ __device__ __noinline__ bool run_s1(int prog, int s, unsigned long long *xbase, 
         if (own != rank) {
             if (lane < ncols) {
                 const uint32_t loc =
-                    saddr(g_smem + slot0 + (slot * kCluster + (int)rank) * 128 + 4 * lane);
+                    saddr(g_smem + slot0 + (slot * C + (int)rank) * 128 + 4 * lane);
                 st_async_f32(mapa(loc, own), v, mapa(saddr(bar_of(slot)), own));
             }
             return;
@@ -414,10 +429,10 @@ __device__ __noinline__ bool run_s1(int prog, int s, unsigned long long *xbase, 
                 }
             }
         }
-        const float *rx = reinterpret_cast<const float *>(g_smem + slot0 + slot * kCluster * 128);
+        const float *rx = reinterpret_cast<const float *>(g_smem + slot0 + slot * C * 128);
         float sum = 0.f;
 #pragma unroll
-        for (int k = 0; k < kCluster; ++k) sum += (unsigned)k == rank ? v : rx[32 * k + lane];
+        for (int k = 0; k < C; ++k) sum += (unsigned)k == rank ? v : rx[32 * k + lane];
         if (lane < ncols) send_fix1(xbase + dst + lane, sum, sc, limit, err);
     };
     int u = u0;
@@ -779,6 +794,7 @@ __device__ void producer(const Loader &ld, unsigned long long *empty, unsigned *
     }
 }
 
+template <int C>
 __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params P) {
     __shared__ __align__(8) unsigned long long full[4], empty[4];
     __shared__ int s_last;
@@ -793,25 +809,23 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         return;
     }
     // the partials of a cluster meet in its CTAs' shared memory: a launch
-    // that did not form clusters of kCluster CTAs (the per-CTA programs
+    // that did not form clusters of C CTAs (the per-CTA programs
     // assume them) records an error and touches no other CTA's memory
-    if (kCluster > 1 && cluster_size() != (unsigned)kCluster) {
+    if (C > 1 && cluster_size() != (unsigned)C) {
         if (threadIdx.x == 0) record(P.ws_words, LB_ERR_UNSUPPORTED);
         return;
     }
     const int N = gridDim.x, c = blockIdx.x;
     const unsigned n_ctas = (unsigned)N, n_t = P.n_t;
-    const unsigned rank = kCluster > 1 ? cluster_rank() : 0u;
+    const unsigned rank = C > 1 ? cluster_rank() : 0u;
     Part s;
     {
-        const int Wd = P.d >> 5, Wf = P.dff >> 5, Ukv = P.dkv >> 3;
-        s.dw0 = (int)((long long)c * Wd / N);
-        s.nd = (int)((long long)(c + 1) * Wd / N) - s.dw0;
-        s.fw0 = (int)((long long)c * Wf / N);
-        s.nf = (int)((long long)(c + 1) * Wf / N) - s.fw0;
-        const int u0 = (int)((long long)c * Ukv / N), u1 = (int)((long long)(c + 1) * Ukv / N);
+        int u0, nu;
+        slice_of(P.d >> 5, N, c, C, s.dw0, s.nd);
+        slice_of(P.dff >> 5, N, c, C, s.fw0, s.nf);
+        slice_of(P.dkv >> 3, N, c, C, u0, nu);
         s.k0 = 8 * u0;
-        s.nkv = 8 * (u1 - u0);
+        s.nkv = 8 * nu;
     }
     if (threadIdx.x == 0) {
         for (int b = 0; b < 4; ++b) {
@@ -835,7 +849,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
     __syncthreads();
     // every CTA of the cluster has initialised its mbarriers before any
     // other may complete a transaction on them
-    if (kCluster > 1) cluster_sync_all();
+    if (C > 1) cluster_sync_all();
     if (threadIdx.x >= kCT) {
         if (threadIdx.x == kCT) producer(Loader{&P, s, full}, empty, P.ws_words);
     } else {
@@ -928,7 +942,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         csync();
         clear_z(0);
         {
-            const bool ok1 = run_s1(pg, A_S1, xl, scA.x, P.lim_t, err, o.slot[0], o.ubar0[0],
+            const bool ok1 = run_s1<C>(pg, A_S1, xl, scA.x, P.lim_t, err, o.slot[0], o.ubar0[0],
                                     o.ubar, par, rank, P.ws_words);
             send_ss(xl + P.offA + ssA_el, ssA, A_R);
             if (!csync_and(ok1)) FAIL_EXIT();
@@ -955,7 +969,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         run_rows(pg, B_R, true, true, ssslot);  // v on the attention rows; tables of o
         csync();
         clear_z(1);
-        if (!csync_and(run_s1(pg, B_S1, xl, scB.x, P.lim_t, err, o.slot[1], o.ubar0[1], o.ubar,
+        if (!csync_and(run_s1<C>(pg, B_S1, xl, scB.x, P.lim_t, err, o.slot[1], o.ubar0[1], o.ubar,
                               par, rank, P.ws_words)))
             FAIL_EXIT();
         if (l > 0) zero_stripe(at(xp, P.offD), s_zs[XR_D]);  // read by phase A's poll
@@ -991,7 +1005,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         csync();
         clear_z(2);
         {
-            const bool ok1 = run_s1(pg, C_S1, xl, scC.x, P.lim_t, err, o.slot[2], o.ubar0[2],
+            const bool ok1 = run_s1<C>(pg, C_S1, xl, scC.x, P.lim_t, err, o.slot[2], o.ubar0[2],
                                     o.ubar, par, rank, P.ws_words);
             send_ss(xl + P.offC + ssC_el, ssC, C_R);
             if (!csync_and(ok1)) FAIL_EXIT();
@@ -1013,7 +1027,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
         run_rows(pg, D_R, true, true, ssslot);  // m = silu(gate) * up; tables of down
         csync();
         clear_z(3);
-        if (!csync_and(run_s1(pg, D_S1, xl, scD.x, P.lim_t, err, o.slot[3], o.ubar0[3], o.ubar,
+        if (!csync_and(run_s1<C>(pg, D_S1, xl, scD.x, P.lim_t, err, o.slot[3], o.ubar0[3], o.ubar,
                               par, rank, P.ws_words)))
             FAIL_EXIT();
         zero_stripe(at(xl, P.offB), s_zs[XR_B]);  // read by phase C's poll
@@ -1051,7 +1065,7 @@ __global__ void __launch_bounds__(kST, 1) k_stack(const __grid_constant__ Params
 done:
     // no CTA leaves while another CTA of its cluster may still store into its
     // shared memory (every wait above is bounded, so every thread gets here)
-    if (kCluster > 1) cluster_sync_all();
+    if (C > 1) cluster_sync_all();
 #undef FAIL_EXIT
 }
 
@@ -1233,7 +1247,7 @@ struct SmemPlan {
     int bytes;
 };
 
-SmemPlan smem_plan(const lb_linear *lin, const StackShape &sh, int N) {
+SmemPlan smem_plan(const lb_linear *lin, const StackShape &sh, int N, int C) {
     const int nd = (sh.d / 32 + N - 1) / N, nf = (sh.dff / 32 + N - 1) / N;
     const int nkv = 8 * ((sh.dkv / 8 + N - 1) / N);
     SmemPlan S{};
@@ -1330,13 +1344,13 @@ SmemPlan smem_plan(const lb_linear *lin, const StackShape &sh, int N) {
     o.ssslot = take(4 * kMaxSlots);
     o.prog = take(kProgBytes);
     // cluster reduction: per phase, the receive slots and mbarriers of the
-    // ceil(units / kCluster) stage-1 units a rank owns at most
+    // ceil(units / C) stage-1 units a rank owns at most
     const int units[4] = {s1_units(lin, LQ, LV), s1_units(lin, LO, LO), s1_units(lin, LG, LU),
                           s1_units(lin, LD, LD)};
     o.n_ubar = 0;
     for (int ph = 0; ph < 4; ++ph) {
-        const int owned = kCluster > 1 ? (units[ph] + kCluster - 1) / kCluster : 0;
-        o.slot[ph] = take(owned * kCluster * 128);
+        const int owned = C > 1 ? (units[ph] + C - 1) / C : 0;
+        o.slot[ph] = take(owned * C * 128);
         o.ubar0[ph] = o.n_ubar;
         o.n_ubar += owned;
     }
@@ -1581,16 +1595,17 @@ struct ProgBuild {
         place(s, best, best_wo);
     }
     // 32-column blocks over the whole input slice.  Unit g of the phase
-    // belongs to cluster rank g % kCluster (its receive slot there: g /
-    // kCluster); each warp runs the units its CTA (rank `rank`) does not own
+    // belongs to cluster rank g % C (its receive slot there: g / C); each
+    // warp runs the units its CTA (rank `rank`) does not own
     // first, so their partials are on their way before it waits for its own.
+    int C = 1;  // CTAs per cluster
     void s1(int s, const std::vector<S1Job> &jobs, int rank) {
         std::vector<Costed> us;
         int g = 0;
         for (const S1Job &J : jobs)
             for (int c0 = 0; c0 < J.r; c0 += 32, ++g)
                 us.push_back({Item{{J.V + 4 * c0, J.r, J.nw, J.tb, J.dst + c0,
-                                    std::min(32, J.r - c0), g % kCluster, g / kCluster}},
+                                    std::min(32, J.r - c0), g % C, g / C}},
                               J.nw + 1.0});
         std::vector<Item> grouped;
         int wo[kCW + 1];
@@ -1605,19 +1620,21 @@ struct ProgBuild {
 // The program of CTA c (kProgBytes, zero-padded); false when it does not fit.
 // Row units of 8 or 4 rows take more records: a program that does not fit
 // with them is built again with 16-row units only.
-bool build_program_at(const lb_linear *lin, const StackShape &sh, int N, int c,
+bool build_program_at(const lb_linear *lin, const StackShape &sh, int N, int C, int c,
                       const Offsets &o, const XLayout &X, int min_lnr,
                       std::vector<int> &prog_out) {
-    const int Wd = sh.d / 32, Wf = sh.dff / 32, Ukv = sh.dkv / 8;
-    const int dw0 = (int)((long long)c * Wd / N), nd = (int)((long long)(c + 1) * Wd / N) - dw0;
-    const int fw0 = (int)((long long)c * Wf / N), nf = (int)((long long)(c + 1) * Wf / N) - fw0;
-    const int nkv = 8 * ((int)((long long)(c + 1) * Ukv / N) - (int)((long long)c * Ukv / N));
+    int dw0, nd, fw0, nf, k0u, nku;
+    slice_of(sh.d / 32, N, c, C, dw0, nd);
+    slice_of(sh.dff / 32, N, c, C, fw0, nf);
+    slice_of(sh.dkv / 8, N, c, C, k0u, nku);
+    const int nkv = 8 * nku;
     const int rows_d = 32 * nd, rows_f = 32 * nf;
     auto np = [&](int k) { return lin[k].n_paths; };
     auto rk = [&](int k, int p) { return lin[k].path[p].r; };
     auto Rk = [&](int k, int p) { return (lin[k].path[p].r + 31) / 32; };
     ProgBuild B;
     B.min_lnr = min_lnr;
+    B.C = C;
     std::vector<Item> T;
     std::vector<S2Job> U;
     std::vector<S1Job> V;
@@ -1629,7 +1646,7 @@ bool build_program_at(const lb_linear *lin, const StackShape &sh, int N, int c,
         B.s2(s, U);
         U.clear();
     };
-    const int rank = c % kCluster;  // cluster rank of CTA c (1-D clusters of kCluster)
+    const int rank = c % C;  // cluster rank of CTA c (1-D clusters of C)
     auto flush_v = [&](int s) {
         B.s1(s, V, rank);
         V.clear();
@@ -1769,26 +1786,27 @@ bool build_program_at(const lb_linear *lin, const StackShape &sh, int N, int c,
     return true;
 }
 
-bool build_program(const lb_linear *lin, const StackShape &sh, int N, int c, const Offsets &o,
-                   const XLayout &X, std::vector<int> &prog_out) {
-    return build_program_at(lin, sh, N, c, o, X, kRowMinLnr, prog_out) ||
-           build_program_at(lin, sh, N, c, o, X, 4, prog_out);
+bool build_program(const lb_linear *lin, const StackShape &sh, int N, int C, int c,
+                   const Offsets &o, const XLayout &X, std::vector<int> &prog_out) {
+    return build_program_at(lin, sh, N, C, c, o, X, kRowMinLnr, prog_out) ||
+           build_program_at(lin, sh, N, C, c, o, X, 4, prog_out);
 }
 
-bool build_programs(const lb_linear *lin, const StackShape &sh, int N, std::vector<int> &all) {
-    const SmemPlan S = smem_plan(lin, sh, N);
+bool build_programs(const lb_linear *lin, const StackShape &sh, int N, int C,
+                    std::vector<int> &all) {
+    const SmemPlan S = smem_plan(lin, sh, N, C);
     const XLayout X = xlayout(lin);
     all.assign((size_t)N * (kProgBytes / 4), 0);
     std::vector<int> one;
     for (int c = 0; c < N; ++c) {
-        if (!build_program(lin, sh, N, c, S.o, X, one)) return false;
+        if (!build_program(lin, sh, N, C, c, S.o, X, one)) return false;
         std::copy(one.begin(), one.end(), all.begin() + (size_t)c * (kProgBytes / 4));
     }
     return true;
 }
 
-bool smem_fits(const lb_linear *lin, const StackShape &sh, int num_sms) {
-    const SmemPlan S = smem_plan(lin, sh, num_sms);
+bool smem_fits(const lb_linear *lin, const StackShape &sh, int num_sms, int C) {
+    const SmemPlan S = smem_plan(lin, sh, num_sms, C);
     int max_optin = 0, dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess ||
         cudaDeviceGetAttribute(&max_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
@@ -1797,7 +1815,8 @@ bool smem_fits(const lb_linear *lin, const StackShape &sh, int num_sms) {
     return S.bytes + 1024 <= max_optin;
 }
 
-bool shapes_ok(const lb_linear *lin, const StackShape &sh, int num_sms) {
+bool shapes_ok(const lb_linear *lin, const StackShape &sh, int num_sms, int C) {
+    if (C < 1 || C > kMaxCluster || num_sms % C != 0) return false;
     for (int k = 0; k < 7; ++k)
         for (int p = 0; p < lin[k].n_paths; ++p)
             if (lin[k].path[p].r % 8 != 0) return false;
@@ -1830,12 +1849,12 @@ char *programs_at(const lb_linear *lin, int n_layers, char *ws_after_header) {
 }  // namespace
 
 cudaError_t launch_stack_prepare(const lb_linear *lin, int n_layers, const StackShape &sh,
-                                 int num_sms, unsigned long long plan, unsigned *ws_words,
-                                 char *ws_after_header, cudaStream_t s) {
-    if (num_sms % kCluster != 0 || !shapes_ok(lin, sh, num_sms) || !smem_fits(lin, sh, num_sms))
+                                 int num_sms, int cluster, unsigned long long plan,
+                                 unsigned *ws_words, char *ws_after_header, cudaStream_t s) {
+    if (!shapes_ok(lin, sh, num_sms, cluster) || !smem_fits(lin, sh, num_sms, cluster))
         return cudaErrorNotSupported;
     std::vector<int> progs;
-    if (!build_programs(lin, sh, num_sms, progs)) return cudaErrorNotSupported;
+    if (!build_programs(lin, sh, num_sms, cluster, progs)) return cudaErrorNotSupported;
     const XLayout X = xlayout(lin);
     LinDesc *desc = reinterpret_cast<LinDesc *>(ws_after_header);
     char *xacc = xacc_at(n_layers, ws_after_header);
@@ -1863,42 +1882,42 @@ cudaError_t launch_stack_prepare(const lb_linear *lin, int n_layers, const Stack
     return cudaGetLastError();
 }
 
-bool stack_supported(const lb_linear *lin, const StackShape &sh, int num_sms) {
-    return num_sms % kCluster == 0 && shapes_ok(lin, sh, num_sms) && smem_fits(lin, sh, num_sms);
+bool stack_supported(const lb_linear *lin, const StackShape &sh, int num_sms, int cluster) {
+    return shapes_ok(lin, sh, num_sms, cluster) && smem_fits(lin, sh, num_sms, cluster);
 }
 
-int stack_grid_ctas(const lb_linear *lin, const StackShape &sh, int num_sms) {
-    if (kCluster == 1) return num_sms;
+int stack_grid_ctas(const lb_linear *lin, const StackShape &sh, int num_sms, int cluster) {
+    if (cluster == 1) return num_sms;
+    if (cluster != 2) return 0;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return 0;
     // the plan of the full grid bounds the shared memory from below (smaller
     // grids give each CTA larger slices); clusters need not fill every SM
-    const int smem = smem_plan(lin, sh, num_sms).bytes;
+    const int smem = smem_plan(lin, sh, num_sms, cluster).bytes;
     static std::mutex mu;
     static int cached_dev = -1, cached_smem = -1, cached_sms = -1, cached_n = 0;
     std::lock_guard<std::mutex> lock(mu);
     if (dev == cached_dev && smem == cached_smem && num_sms == cached_sms) return cached_n;
-    if (cudaFuncSetAttribute((const void *)k_stack, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             smem) != cudaSuccess)
+    const void *fn = (const void *)k_stack<2>;
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+        cudaSuccess)
         return 0;
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(kCluster, 1, 1);
+    cfg.gridDim = dim3(cluster, 1, 1);
     cfg.blockDim = dim3(kST, 1, 1);
     cfg.dynamicSmemBytes = (size_t)smem;
     cudaLaunchAttribute at[1];
     at[0].id = cudaLaunchAttributeClusterDimension;
-    at[0].val.clusterDim.x = kCluster;
+    at[0].val.clusterDim.x = cluster;
     at[0].val.clusterDim.y = 1;
     at[0].val.clusterDim.z = 1;
     cfg.attrs = at;
     cfg.numAttrs = 1;
     int n_cl = 0;
-    if (cudaOccupancyMaxActiveClusters(&n_cl, (const void *)k_stack, &cfg) != cudaSuccess ||
-        n_cl <= 0)
-        return 0;
-    const int n = std::min(num_sms / kCluster, n_cl) * kCluster;
+    if (cudaOccupancyMaxActiveClusters(&n_cl, fn, &cfg) != cudaSuccess || n_cl <= 0) return 0;
+    const int n = std::min(num_sms / cluster, n_cl) * cluster;
     // the larger slices of the smaller grid must still fit
-    if (!smem_fits(lin, sh, n)) return 0;
+    if (!smem_fits(lin, sh, n, cluster)) return 0;
     cached_dev = dev;
     cached_smem = smem;
     cached_sms = num_sms;
@@ -1909,9 +1928,11 @@ int stack_grid_ctas(const lb_linear *lin, const StackShape &sh, int num_sms) {
 cudaError_t launch_stack(const lb_linear *lin, int n_layers, const StackShape &sh,
                          unsigned long long plan, const uint16_t *x0, float *out, float *q_out,
                          float *kv_out, unsigned *ws_words, char *ws_after_header, int num_sms,
-                         cudaStream_t s) {
+                         int cluster, cudaStream_t s) {
+    if (cluster < 1 || cluster > kMaxCluster || num_sms % cluster != 0)
+        return cudaErrorInvalidConfiguration;
     const XLayout X = xlayout(lin);
-    const SmemPlan S = smem_plan(lin, sh, num_sms);
+    const SmemPlan S = smem_plan(lin, sh, num_sms, cluster);
     Params P{};
     P.lin = reinterpret_cast<const LinDesc *>(ws_after_header);
     P.prog = reinterpret_cast<const int *>(programs_at(lin, n_layers, ws_after_header));
@@ -1943,21 +1964,21 @@ cudaError_t launch_stack(const lb_linear *lin, int n_layers, const StackShape &s
     P.lenB = X.lenB;
     P.lenC = X.lenC;
     P.lenD = X.lenD;
-    if (num_sms % kCluster != 0) return cudaErrorInvalidConfiguration;
-    P.n_t = (unsigned)(num_sms / kCluster);
+    P.n_t = (unsigned)(num_sms / cluster);
     P.lim_t = fix1_limit((int)P.n_t);
     P.lim_ss = fix1_limit(num_sms);
     P.o = S.o;
     const size_t smem = (size_t)S.bytes;
-    cudaError_t e = cudaFuncSetAttribute((const void *)k_stack,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    const void *fn = cluster == 2 ? (const void *)k_stack<2> : (const void *)k_stack<1>;
+    cudaError_t e =
+        cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     int per_sm = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, (const void *)k_stack, kST, smem);
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fn, kST, smem);
     if (e != cudaSuccess) return e;
     if (per_sm < 1) return cudaErrorCooperativeLaunchTooLarge;
     // cooperative: the grid is launched only if every CTA is co-resident (the
-    // kernel's waits need that); clusters of kCluster consecutive CTAs
+    // kernel's waits need that); clusters of `cluster` consecutive CTAs
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(num_sms, 1, 1);
     cfg.blockDim = dim3(kST, 1, 1);
@@ -1967,12 +1988,13 @@ cudaError_t launch_stack(const lb_linear *lin, int n_layers, const StackShape &s
     at[0].id = cudaLaunchAttributeCooperative;
     at[0].val.cooperative = 1;
     at[1].id = cudaLaunchAttributeClusterDimension;
-    at[1].val.clusterDim.x = kCluster;
+    at[1].val.clusterDim.x = cluster;
     at[1].val.clusterDim.y = 1;
     at[1].val.clusterDim.z = 1;
     cfg.attrs = at;
     cfg.numAttrs = 2;
-    return cudaLaunchKernelEx(&cfg, k_stack, P);
+    return cluster == 2 ? cudaLaunchKernelEx(&cfg, k_stack<2>, P)
+                        : cudaLaunchKernelEx(&cfg, k_stack<1>, P);
 }
 
 }  // namespace lb

@@ -12,8 +12,11 @@
 // contribution per cluster), then polls every element exactly as the stack
 // kernel's stage-2 tables do (one gating lane per 128-element unit, then four
 // elements per lane) until all are complete, and only then starts round k+1.
-// The time per round is the exchange's floor on the critical path: the
-// stack kernel adds its +-1 sums to it.  Every wait is bounded.
+// W = 1 encodes every element as the stack does (one word at a scale set
+// from a bound, send_fix1), W = 2 as the single-token kernels do (the exact
+// hi / lo pair, send_fix2).  The time per round is the exchange's floor on
+// the critical path: the kernels add their +-1 sums to it.  Every wait is
+// bounded.
 #include "lb_common.cuh"
 #include "lb_kernels.h"
 #include "lb_lut.cuh"
@@ -39,7 +42,7 @@ __device__ __forceinline__ bool xc_sticky(const unsigned *w) {
     return ld_relaxed_gpu(w + kErrWord) != 0u;
 }
 
-template <int C>
+template <int C, int W>
 __global__ void __launch_bounds__(kXT, 1) k_xchain(const __grid_constant__ XchainParams P) {
     __shared__ __align__(8) unsigned long long ubar[kXMaxUnits / 2];
     __shared__ float slot[kXMaxUnits / 2][32];
@@ -58,10 +61,21 @@ __global__ void __launch_bounds__(kXT, 1) k_xchain(const __grid_constant__ Xchai
     }
     __syncthreads();
     if (C > 1) cluster_sync_all();
-    // this CTA's contribution: 2^-10 * (blockIdx + 1), exactly representable
+    // this CTA's contribution: 2^-10 * (blockIdx + 1), exactly representable;
+    // a cluster's sum is below 2 gridDim 2^-10 (the one-word scale's bound)
     const float v = (float)(blockIdx.x + 1) * 0x1p-10f;
+    const float sc = fix1_scale(2.f * (float)gridDim.x * 0x1p-10f, (int)P.n_contrib).x;
+
+    unsigned long long *xk = P.buf;
+    auto x_at = [&](int e) { return xk + e; };
+    auto send = [&](int e, float a) {
+        if (W == 1)
+            send_fix1(x_at(e), a, sc, P.limit, ws + kErrWord);
+        else
+            send_fix2(fix2_at(xk, e), a, P.limit, ws + kErrWord);
+    };
     for (int k = 0; k < P.n_rounds; ++k) {
-        unsigned long long *x = P.buf + (size_t)k * P.stride;
+        xk = P.buf + (size_t)k * P.stride;
         const int n = P.sizes[k % P.n_sizes];
         const int units = (n + 31) >> 5;
         const unsigned par = (unsigned)(k & 1);
@@ -78,7 +92,7 @@ __global__ void __launch_bounds__(kXT, 1) k_xchain(const __grid_constant__ Xchai
         for (int u = warp; u < units; u += kXW) {
             const int e = 32 * u + lane;
             if (C == 1) {
-                if (e < n) send_fix2(fix2_at(x, e), v, P.limit, ws + kErrWord);
+                if (e < n) send(e, v);
                 continue;
             }
             const unsigned own = (unsigned)(u % C);
@@ -102,13 +116,14 @@ __global__ void __launch_bounds__(kXT, 1) k_xchain(const __grid_constant__ Xchai
             }
             // the peer's partial beside this CTA's own, in rank order
             const float sum = rank == 0 ? v + slot[u / C][lane] : slot[u / C][lane] + v;
-            if (e < n) send_fix2(fix2_at(x, e), sum, P.limit, ws + kErrWord);
+            if (e < n) send(e, sum);
         }
         // ---- polls: 128-element unit q on warp q % 16
         for (int q = warp; q < (n + 127) / 128 && ok; q += kXW) {
             const int e0 = 128 * q, m = min(128, n - e0);
             if (lane == 0) {
-                const unsigned long long *gw = fix2_at(x, e0 + m - 1) + 32;
+                // the last element's (lo) word
+                const unsigned long long *gw = W == 1 ? x_at(e0 + m - 1) : fix2_at(xk, e0 + m - 1) + 32;
                 const unsigned long long t0 = globaltimer_ns();
                 for (int spin = 0; (unsigned)(ld_relaxed_u64(gw) & 0xffull) != P.n_contrib; ++spin)
                     if ((spin & 15) == 15 && globaltimer_ns() - t0 > kWaitLimitNs) break;
@@ -117,14 +132,21 @@ __global__ void __launch_bounds__(kXT, 1) k_xchain(const __grid_constant__ Xchai
             if (4 * lane >= m) continue;
             // element groups of 4 stay inside one 32-element block (n is padded
             // to whole blocks in the buffer, and the padding stays zero)
-            const unsigned long long *w = fix2_at(x, e0 + 4 * lane);
+            const unsigned long long *w = W == 1 ? x_at(e0 + 4 * lane) : fix2_at(xk, e0 + 4 * lane);
             const int have = min(4, m - 4 * lane);
             unsigned long long a[8];
             const unsigned long long t0 = globaltimer_ns();
             for (int spin = 0;; ++spin) {
-                ld_fix2x4(w, a);
                 bool done = true;
-                for (int j = 0; j < have; ++j) done = done && counted2(a[2 * j], a[2 * j + 1], P.n_contrib);
+                if (W == 1) {
+                    ld_relaxed_v2_u64(w, a[0], a[1]);
+                    ld_relaxed_v2_u64(w + 2, a[2], a[3]);
+                    for (int j = 0; j < have; ++j) done = done && counted1(a[j], P.n_contrib);
+                } else {
+                    ld_fix2x4(w, a);
+                    for (int j = 0; j < have; ++j)
+                        done = done && counted2(a[2 * j], a[2 * j + 1], P.n_contrib);
+                }
                 if (done) break;
                 if ((spin & 15) == 15 &&
                     (xc_sticky(ws) || globaltimer_ns() - t0 > kWaitLimitNs)) {
@@ -148,9 +170,10 @@ size_t xchain_ws_bytes(int n_rounds, const int *sizes, int n_sizes) {
     return kWsHeader + (size_t)n_rounds * fix2_words((size_t)mx) * sizeof(unsigned long long);
 }
 
-cudaError_t launch_xchain(int n_rounds, const int *sizes, int n_sizes, int cluster,
+cudaError_t launch_xchain(int n_rounds, const int *sizes, int n_sizes, int cluster, int words,
                           unsigned *ws_words, void *buf, int num_sms, cudaStream_t s) {
-    if (n_rounds < 1 || n_sizes < 1 || n_sizes > 8 || (cluster != 1 && cluster != 2))
+    if (n_rounds < 1 || n_sizes < 1 || n_sizes > 8 || (cluster != 1 && cluster != 2) ||
+        (words != 1 && words != 2))
         return cudaErrorInvalidValue;
     XchainParams P{};
     int mx = 0;
@@ -167,7 +190,8 @@ cudaError_t launch_xchain(int n_rounds, const int *sizes, int n_sizes, int clust
     P.n_sizes = n_sizes;
     P.stride = (int)fix2_words((size_t)mx);
     P.n_contrib = (unsigned)(N / cluster);
-    P.limit = fix2_limit(N);
+    // one word: below 2^55 / n (n contributions then sum to less than 2^55)
+    P.limit = words == 1 ? 0x1p54f / (float)P.n_contrib : fix2_limit(N);
     cudaError_t e = cudaMemsetAsync(buf, 0, (size_t)n_rounds * P.stride * sizeof(unsigned long long),
                                     s);
     if (e != cudaSuccess) return e;
@@ -184,8 +208,11 @@ cudaError_t launch_xchain(int n_rounds, const int *sizes, int n_sizes, int clust
     at[1].val.clusterDim.z = 1;
     cfg.attrs = at;
     cfg.numAttrs = 2;
-    return cluster == 2 ? cudaLaunchKernelEx(&cfg, k_xchain<2>, P)
-                        : cudaLaunchKernelEx(&cfg, k_xchain<1>, P);
+    if (words == 1)
+        return cluster == 2 ? cudaLaunchKernelEx(&cfg, k_xchain<2, 1>, P)
+                            : cudaLaunchKernelEx(&cfg, k_xchain<1, 1>, P);
+    return cluster == 2 ? cudaLaunchKernelEx(&cfg, k_xchain<2, 2>, P)
+                        : cudaLaunchKernelEx(&cfg, k_xchain<1, 2>, P);
 }
 
 }  // namespace lb

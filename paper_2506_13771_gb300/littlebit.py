@@ -160,7 +160,7 @@ def lib(path: str | None = None):
         L.littlebit_linear_forward_noalloc.restype = ctypes.c_int
         L.littlebit_selftest_exchange_workspace_size.argtypes = [i32, vp, i32]
         L.littlebit_selftest_exchange_workspace_size.restype = sz
-        L.littlebit_selftest_exchange.argtypes = [i32, vp, i32, i32, vp, sz, vp]
+        L.littlebit_selftest_exchange.argtypes = [i32, vp, i32, i32, i32, vp, sz, vp]
         L.littlebit_selftest_exchange.restype = ctypes.c_int
         if path is None:
             _lib = L
@@ -512,10 +512,11 @@ def selftest_wait_timeout(ws: torch.Tensor, stream=None) -> None:
            "littlebit_selftest_wait_timeout")
 
 
-def selftest_exchange(n_rounds: int, sizes, cluster: int = 2, ws: torch.Tensor | None = None,
-                      device="cuda", stream=None) -> torch.Tensor:
+def selftest_exchange(n_rounds: int, sizes, cluster: int = 1, words: int = 1,
+                      ws: torch.Tensor | None = None, device="cuda", stream=None) -> torch.Tensor:
     """Launch the exchange-chain diagnostic (n_rounds dependent all-reduces of
-    sizes[k % len(sizes)] elements); returns the workspace (poll it)."""
+    sizes[k % len(sizes)] elements; words = 1: the stack's encoding, 2: the
+    single-linear kernels'); returns the workspace (poll it)."""
     arr = (ctypes.c_int32 * len(sizes))(*[int(v) for v in sizes])
     need = int(lib().littlebit_selftest_exchange_workspace_size(int(n_rounds), arr, len(sizes)))
     if need == 0:
@@ -523,7 +524,8 @@ def selftest_exchange(n_rounds: int, sizes, cluster: int = 2, ws: torch.Tensor |
     if ws is None:
         ws = new_workspace(need, device)
     _check(lib().littlebit_selftest_exchange(int(n_rounds), arr, len(sizes), int(cluster),
-                                             ws.data_ptr(), ws.numel(), _stream(stream)),
+                                             int(words), ws.data_ptr(), ws.numel(),
+                                             _stream(stream)),
            "littlebit_selftest_exchange")
     return ws
 

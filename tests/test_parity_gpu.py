@@ -8,6 +8,7 @@ for the largest reduction here, n = 28672), so 1e-4 leaves a 10x margin;
 bf16 outputs carry the bf16 rounding itself (relative RMS about 1.2e-3).
 """
 import ctypes
+import os
 
 import numpy as np
 import pytest
@@ -561,6 +562,34 @@ def test_stack_70b_full():
     check_stack(run_stack(layers, x0, 128), oracle.stack_forward(layers, x0, head_dim=128))
 
 
+def test_stack_cluster_pairs():
+    """The two-CTA cluster variant (LB_STACK_CLUSTER=2: the stage-1 partials of
+    each CTA pair meet in distributed shared memory and one contribution per
+    pair goes to the exchange) against the oracle, on the 80-layer 70B shape
+    and on a small stack with ragged slices; a workspace prepared for one
+    cluster size is refused by the other with LB_ERR_PLAN."""
+    old = os.environ.get("LB_STACK_CLUSTER")
+    try:
+        os.environ["LB_STACK_CLUSTER"] = "2"
+        layers, x0 = inputs.config5()
+        check_stack(run_stack(layers, x0, 128), oracle.stack_forward(layers, x0, head_dim=128))
+        layers, x0 = inputs.make_stack(n_layers=2, d_model=640, d_kv=160, d_ff=1696, r_qo=40,
+                                       r_kv=8, r_mlp=56, head_dim=32, config_id=103)
+        check_stack(run_stack(layers, x0, 32), oracle.stack_forward(layers, x0, head_dim=32))
+        S = lb.DeviceStack(layers, 32, DEV)
+        ws = S.prepare()
+        os.environ["LB_STACK_CLUSTER"] = "1"
+        out = torch.full((S.d_model,), float("nan"), device=DEV)
+        lb.stack_forward(S, lb.bf16_tensor(x0, DEV), out=out, want_q=False, want_kv=False, ws=ws)
+        assert lb.poll_error(ws) == lb.LB_ERR_PLAN
+        assert torch.isnan(out).all()
+    finally:
+        if old is None:
+            os.environ.pop("LB_STACK_CLUSTER", None)
+        else:
+            os.environ["LB_STACK_CLUSTER"] = old
+
+
 def test_fused_launch_reuses_workspace():
     """From four token tiles on, the forward (and each of latent / expand) is
     one cooperative launch whose grid barriers count on workspace words 1 and
@@ -635,11 +664,16 @@ def test_grid_wait_times_out_and_is_sticky():
 
 def test_exchange_diagnostic_runs_clean():
     """The exchange-chain diagnostic (the stack's all-reduce with nothing around
-    it) completes every round, with and without the two-CTA clusters, and
+    it) completes every round in both encodings, with and without the two-CTA
+    clusters, and
     rejects sizes it cannot hold."""
-    for cluster in (1, 2):
-        ws = lb.selftest_exchange(40, [65, 384, 1281, 640], cluster, device=DEV)
-        assert lb.poll_error(ws) == lb.LB_OK
+    for words in (1, 2):
+        for cluster in (1, 2):
+            ws = lb.selftest_exchange(40, [65, 384, 1281, 640], cluster, words, device=DEV)
+            assert lb.poll_error(ws) == lb.LB_OK
     arr = (ctypes.c_int32 * 1)(4096)
-    assert lb.lib().littlebit_selftest_exchange(4, arr, 1, 2, ws.data_ptr(), ws.numel(),
+    assert lb.lib().littlebit_selftest_exchange(4, arr, 1, 2, 1, ws.data_ptr(), ws.numel(),
+                                                None) == lb.LB_ERR_INVALID_ARG
+    arr = (ctypes.c_int32 * 1)(64)
+    assert lb.lib().littlebit_selftest_exchange(4, arr, 1, 1, 3, ws.data_ptr(), ws.numel(),
                                                 None) == lb.LB_ERR_INVALID_ARG
