@@ -366,6 +366,19 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
                 const uint32_t tb = (uint32_t)(o.t2 + (p ? nt0 : 0) * 128);
                 float acc0 = 0.f, acc1 = 0.f;
                 int w = 0;
+                if ((R & 3) == 0) {
+                    // rows of R = 4k words are 16-byte aligned: one 128-bit load takes four
+                    // words (a warp's 32 rows at a stride of R words fall in few banks, so
+                    // a 32-bit load per word would replay up to 16 times); even words still
+                    // go to acc0 and odd ones to acc1, in order
+                    for (; w < R; w += 4) {
+                        const uint4 q = *reinterpret_cast<const uint4 *>(Uw + w);
+                        acc0 += lut_word(q.x, copy, tb + w * 1024);
+                        acc1 += lut_word(q.y, copy, tb + (w + 1) * 1024);
+                        acc0 += lut_word(q.z, copy, tb + (w + 2) * 1024);
+                        acc1 += lut_word(q.w, copy, tb + (w + 3) * 1024);
+                    }
+                }
                 for (; w + 2 <= R; w += 2) {
                     const uint32_t w0 = Uw[w], w1 = Uw[w + 1];
                     acc0 += lut_word(w0, copy, tb + w * 1024);
