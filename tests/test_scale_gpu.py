@@ -167,6 +167,36 @@ def test_stack_two_layers_small_scales():
     check_stack(run_stack(layers, x0, 64), oracle.stack_forward(layers, x0, head_dim=64))
 
 
+@pytest.mark.parametrize("bad", [0x7F80, 0xFFC0])  # bf16 +inf, NaN
+def test_nonfinite_input_reports_range(bad):
+    """An infinite or NaN input entry leaves every exchange's range: the stack
+    and the single-token kernel record LB_ERR_RANGE (the exchanges still
+    complete -- out-of-range contributions are sent as zero, so nothing
+    waits), and a workspace prepared again afterwards computes the finite
+    input correctly."""
+    layers, x0 = inputs.make_stack(n_layers=2, config_id=207, **SMALL)
+    xb = x0.copy()
+    xb[17] = bad
+    S = lb.DeviceStack(layers, 64, DEV)
+    ws = S.prepare()
+    lb.stack_forward(S, lb.bf16_tensor(xb, DEV), ws=ws)
+    assert lb.poll_error(ws) == lb.LB_ERR_RANGE
+    S.prepare(ws)
+    out, q, kv = lb.stack_forward(S, lb.bf16_tensor(x0, DEV), ws=ws)
+    assert lb.poll_error(ws) == lb.LB_OK
+    got = tuple(t.cpu().numpy().astype(np.float64) for t in (out, q, kv))
+    check_stack(got, oracle.stack_forward(layers, x0, head_dim=64))
+
+    L, _ = inputs.config2(1)
+    D = lb.DeviceLinear(L, DEV)
+    x = inputs.bf16_normal(inputs.rng_for(208), (1, L["d_in"]))
+    x[0, 5] = bad
+    ws1 = lb.new_workspace(lb.workspace_size(D, 1), DEV)
+    y = torch.empty((1, D.d_out), dtype=torch.float32, device=DEV)
+    lb.linear_forward(D, lb.bf16_tensor(x, DEV), y=y, ws=ws1)
+    assert lb.poll_error(ws1) == lb.LB_ERR_RANGE
+
+
 @pytest.fixture(scope="module")
 def stack70b():
     layers, x0 = inputs.config5()
