@@ -136,8 +136,8 @@ __global__ void __launch_bounds__(kDT, 1) k_decode(const __grid_constant__ Decod
             xg[i] = xe * half_bits_to_float(g[e]);
         }
     }
+    // stage-2 part slots: path 0's s2_parts(R0) slots, then path 1's, nrows each
     float *y = reinterpret_cast<float *>(g_smem + o.y);
-    for (int i = tid; i < nrows; i += kDT) y[i] = 0.f;
     __syncthreads();
 
     // ---- stage 1: tables of g . x (8 per input word and path), then columns
@@ -217,46 +217,27 @@ __global__ void __launch_bounds__(kDT, 1) k_decode(const __grid_constant__ Decod
     // of them have read the epoch: the next launch may use the other buffer
     if (ok && c == 0 && tid == 0) P.ws_words[kEpochWord] = epoch + 1u;
     if (ok) {
-        // ---- stage 2: 32 rows x all words of one path per warp task
+        // ---- stage 2: parts of 32 rows x up to four words of one path
         const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
         const int rb = (nrows + 31) >> 5;
-        for (int u = warp; u < np * rb; u += kDW) {
-            const int p = u / rb, b = u - p * rb;
-            const int R = ((p ? L.r[1] : L.r[0]) + 31) >> 5;
-            const int row = 32 * b + lane, rr = min(row, nrows - 1);
-            const float hs =
-                half_bits_to_float(reinterpret_cast<const uint16_t *>(g_smem + o.h[p])[rr]);
-            const uint32_t *Uw = reinterpret_cast<const uint32_t *>(g_smem + o.U[p]) + rr * R;
-            const uint32_t tb = (uint32_t)(o.t2 + (p ? nt0 : 0) * 128);
-            float acc0 = 0.f, acc1 = 0.f;
-            int w = 0;
-            if ((R & 3) == 0) {
-                // rows of R = 4k words are 16-byte aligned: one 128-bit load takes four
-                // words (a warp's 32 rows at a stride of R words fall in few banks, so
-                // a 32-bit load per word would replay up to 16 times); even words still
-                // go to acc0 and odd ones to acc1, in order
-                for (; w < R; w += 4) {
-                    const uint4 q = *reinterpret_cast<const uint4 *>(Uw + w);
-                    acc0 += lut_word(q.x, copy, tb + w * 1024);
-                    acc1 += lut_word(q.y, copy, tb + (w + 1) * 1024);
-                    acc0 += lut_word(q.z, copy, tb + (w + 2) * 1024);
-                    acc1 += lut_word(q.w, copy, tb + (w + 3) * 1024);
-                }
-            }
-            for (; w + 2 <= R; w += 2) {
-                const uint32_t w0 = Uw[w], w1 = Uw[w + 1];
-                acc0 += lut_word(w0, copy, tb + w * 1024);
-                acc1 += lut_word(w1, copy, tb + (w + 1) * 1024);
-            }
-            if (w < R) acc0 += lut_word(Uw[w], copy, tb + w * 1024);
-            if (row < nrows) atomicAdd(y + row, (acc0 + acc1) * hs);
+        const int R0 = (L.r[0] + 31) >> 5, R1 = np > 1 ? (L.r[1] + 31) >> 5 : 0;
+        const int S0 = s2_parts(R0), S1 = np > 1 ? s2_parts(R1) : 0;
+        const int n0 = rb * S0, nu = n0 + rb * S1;
+        for (int u = warp; u < nu; u += kDW) {
+            const int p = u >= n0 ? 1 : 0, v = u - (p ? n0 : 0), S = p ? S1 : S0;
+            const int b = v / S, sp = v - b * S;
+            s2_part(reinterpret_cast<const uint32_t *>(g_smem + o.U[p]), p ? R1 : R0,
+                    reinterpret_cast<const uint16_t *>(g_smem + o.h[p]),
+                    (uint32_t)(o.t2 + (p ? nt0 : 0) * 128), nrows, b, sp,
+                    y + (size_t)((p ? S0 : 0) + sp) * nrows, copy, lane);
         }
         __syncthreads();
         for (int i = tid; i < nrows; i += kDT) {
+            const float v = s2_combine(y, nrows, S0 + S1, i);
             if (P.y_fp32)
-                static_cast<float *>(P.y)[o0 + i] = y[i];
+                static_cast<float *>(P.y)[o0 + i] = v;
             else
-                static_cast<uint16_t *>(P.y)[o0 + i] = float_to_bf16_bits(y[i]);
+                static_cast<uint16_t *>(P.y)[o0 + i] = float_to_bf16_bits(v);
         }
     } else if (tid == 0) {
         // the copies of this CTA must land before it goes away
@@ -277,7 +258,7 @@ DecodeLayout layout_of(const lb_linear &L, int N) {
         at += up16(bytes);
         return off;
     };
-    int ntab2 = 0;
+    int ntab2 = 0, nslot = 0;
     for (int p = 0; p < 2; ++p) {
         const bool on = p < L.n_paths;
         const int r = on ? L.path[p].r : 0, R = (r + 31) / 32;
@@ -286,13 +267,14 @@ DecodeLayout layout_of(const lb_linear &L, int N) {
         o.h[p] = take(2 * nrows);
         o.xg[p] = take(on ? 128 * nw : 0);
         ntab2 += 8 * R;
+        nslot += on ? s2_parts(R) : 0;
     }
     // table bases are 1024-aligned: lut8 splices the entry byte into them
     at = (at + 1023) & ~1023;
     o.t1 = take(L.n_paths * 8 * nw * 128);
     at = (at + 1023) & ~1023;
     o.t2 = take(ntab2 * 128);
-    o.y = take(4 * nrows);
+    o.y = take(4 * nrows * nslot);
     o.bytes = at;
     return o;
 }

@@ -315,6 +315,54 @@ __device__ __forceinline__ float dec_fix1(unsigned long long w, float inv) {
     return __ll2float_rn(static_cast<long long>(w) >> 8) * inv;
 }
 
+// ---------------------------------------------------------------- single-linear stage 2
+//
+// Stage 2 of the single-linear kernels (k_decode, k_decode_multi) runs in
+// parts: rows [32 b, 32 b + 32) of path p (lane = row) over words [4 s,
+// 4 s + 4) of the row (the last part may be shorter), so a CTA's rows spread
+// over many warps however few rows it has.  Each part leaves (the sum of its
+// +-1 lookups, even words then odd words) * h[row] in a slot of its own;
+// s2_combine adds a row's slots in slot order (path 0's parts, then path
+// 1's), so both kernels give the same bits whichever warp ran which part.
+constexpr int kPartWords = 4;
+__host__ __device__ inline int s2_parts(int R) { return (R + kPartWords - 1) / kPartWords; }
+
+// One part: U (the path's rows, R words each, row 0 at U), h (fp16 of row 0),
+// tables tb (word 0's), into dst[row] for rows below nrows.
+__device__ __forceinline__ void s2_part(const uint32_t *U, int R, const uint16_t *h,
+                                        uint32_t tb, int nrows, int b, int s, float *dst,
+                                        uint32_t copy, int lane) {
+    const int row = 32 * b + lane, rr = min(row, nrows - 1);
+    const uint32_t *Uw = U + rr * R;
+    const int w0 = kPartWords * s, w1 = min(R, w0 + kPartWords);
+    float acc0 = 0.f, acc1 = 0.f;
+    if (w1 - w0 == 4 && (R & 3) == 0) {
+        // rows of R = 4k words are 16-byte aligned: one 128-bit load takes the
+        // part (a warp's 32 rows at a stride of R words fall in few banks, so
+        // a 32-bit load per word would replay up to 16 times)
+        const uint4 q = *reinterpret_cast<const uint4 *>(Uw + w0);
+        acc0 += lut_word(q.x, copy, tb + w0 * 1024);
+        acc1 += lut_word(q.y, copy, tb + (w0 + 1) * 1024);
+        acc0 += lut_word(q.z, copy, tb + (w0 + 2) * 1024);
+        acc1 += lut_word(q.w, copy, tb + (w0 + 3) * 1024);
+    } else {
+        int w = w0;
+        for (; w + 2 <= w1; w += 2) {
+            acc0 += lut_word(Uw[w], copy, tb + w * 1024);
+            acc1 += lut_word(Uw[w + 1], copy, tb + (w + 1) * 1024);
+        }
+        if (w < w1) acc0 += lut_word(Uw[w], copy, tb + w * 1024);
+    }
+    if (row < nrows) dst[row] = (acc0 + acc1) * half_bits_to_float(h[rr]);
+}
+
+// Output row `row`: its nslot slots (stride `stride` floats) added in order.
+__device__ __forceinline__ float s2_combine(const float *slots, int stride, int nslot, int row) {
+    float y = slots[row];
+    for (int k = 1; k < nslot; ++k) y += slots[k * stride + row];
+    return y;
+}
+
 // Stores table n of a unit at T from its four values (see run_tables).
 __device__ __forceinline__ void store_table(unsigned char *T, float4 x, int lane) {
 #pragma unroll

@@ -7,13 +7,14 @@
 // summed through self-counting exchange words; stage 2 y = h . (U_sign (l . t))
 // over each CTA's output rows; Eq. 6 sums the paths.  The single-linear
 // kernel (k_decode) runs the two stages back to back and waits for its
-// exchange in between.  Here the linears are software-pipelined: iteration i
-// runs stage 1 of linear i and stage 2 of linear i - kAhead, so each
-// exchange has kAhead - 1 whole iterations of other linears' work to
-// complete behind.  Thread 0 bulk-copies (cp.async.bulk) each linear's V
-// slice, g slice, U rows and h into a ring of kSlots shared-memory slots, a
-// slot being refilled once its linear's stage 2 is done (kSlots - kAhead
-// iterations ahead of its stage 1).  The exchange words of all M linears are
+// exchange in between.  Here the compute warps form two groups that run the
+// two stages of different linears at once: the stage-1 group sends linear
+// m's partial t while the stage-2 group builds the outputs of an earlier
+// linear, so each exchange completes behind other linears' work and neither
+// stage waits for the other's barriers.  A producer warp bulk-copies
+// (cp.async.bulk) each linear's V slice, g slice, U rows and h into a ring of
+// kSlots shared-memory slots, a slot being refilled once its linear's stage 2
+// is done (so stage 1 runs at most kSlots linears ahead of stage 2).  The exchange words of all M linears are
 // double-buffered by the workspace's launch epoch as in k_decode: every CTA
 // clears its stripe of the previous launch's buffer.  In the residual-input
 // mode (a decoder's a += y ahead of its q / k / v or gate / up) each CTA adds
@@ -23,6 +24,7 @@
 // wait is bounded;
 // on a timeout the CTA records LB_ERR_TIMEOUT, lets its own copies land and
 // returns.
+#include <algorithm>
 #include <mutex>
 
 #include "lb_common.cuh"
@@ -36,8 +38,6 @@ namespace {
 constexpr int kMT = 512;  // threads per CTA
 constexpr int kMW = kMT / 32;
 constexpr int kSlots = 7;
-constexpr int kAhead = 4;
-static_assert(kSlots > kAhead + 1, "a slot must be refilled ahead of its next stage 1");
 constexpr int kCW = kMW - 1;       // compute warps; the last warp issues the copies
 constexpr int kCT = kCW * 32;
 
@@ -53,6 +53,7 @@ struct MultiLayout {
 
 struct MultiParams {
     int d_in, d_out, np, r[2], M, N1, off1;
+    int k1;  // compute warps of the stage-1 group (the rest run stage 2)
     const void *x;  // bf16 [d_in] (x_fp32 = 0), or fp32 (x_fp32 = 1)
     int x_fp32;     // 3: residual input, see res_a
     // x_fp32 = 3: x = res_a + res_y (fp32 [d_in]), written back to res_a, and
@@ -85,14 +86,18 @@ __device__ bool wait_bar_m(unsigned long long *bar, unsigned parity, unsigned *w
 __device__ __forceinline__ void csync_m() {
     asm volatile("bar.sync 1, %0;" ::"n"(kCT) : "memory");
 }
-// AND of pred over the compute threads (named barrier 1), returned to each.
-__device__ __forceinline__ int csync_and_m(int pred) {
+// Barrier over a warp group (named barrier id of n threads, n a multiple of 32).
+__device__ __forceinline__ void gsync(int id, int n) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+// AND of pred over a warp group, returned to each of its threads.
+__device__ __forceinline__ int gsync_and(int id, int n, int pred) {
     int r;
     asm volatile(
-        "{\n\t.reg .pred p, q;\n\tsetp.ne.s32 p, %1, 0;\n\tbar.red.and.pred q, 1, %2, p;\n\t"
+        "{\n\t.reg .pred p, q;\n\tsetp.ne.s32 p, %1, 0;\n\tbar.red.and.pred q, %2, %3, p;\n\t"
         "selp.s32 %0, 1, 0, q;\n\t}"
         : "=r"(r)
-        : "r"(pred), "n"(kCT)
+        : "r"(pred), "r"(id), "r"(n)
         : "memory");
     return r;
 }
@@ -176,7 +181,7 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
         }
         __syncwarp();
     } else {
-        // ---------------- compute warps (named barrier 1)
+        // ---------------- compute warps (named barrier 1; then two groups)
         // the x slice (fp32), and the previous launch's exchange words back to zero
         float *xs = reinterpret_cast<float *>(g_smem + o.xs);
         float ss = 0.f;
@@ -202,8 +207,6 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
             const size_t a = (size_t)c * stride / N, e = (size_t)(c + 1) * stride / N;
             for (size_t i = a + tid; i < e; i += kCT) xold[i] = 0ull;
         }
-        float *y = reinterpret_cast<float *>(g_smem + o.y);
-        for (int i = tid; i < nrows; i += kCT) y[i] = 0.f;
         csync_m();
         // every CTA's share of the mean square (sum / d_in: the fixed-point
         // word then holds outlier-sized activations too), counted like linear
@@ -212,120 +215,103 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
             send_fix2(fix2_at(xw, (int)words), s_ss / (float)P.d_in, P.fix_limit, err);
         const uint32_t copy = (lane >> 4) ? 0x40404040u : 0u;
         bool ok = true;
-        // the exchange words a thread polls for stage 2 (its table tid; ntab <=
-        // kCT whenever the ranks sum to at most 1920), loaded while the row
-        // sums of the linear before run, so that the L2 round trip overlaps them
-        unsigned long long pre[8] = {0ull, 0ull, 0ull, 0ull, 0ull, 0ull, 0ull, 0ull};
-        auto prefetch = [&](int mm) {
-            if (mm < 0 || mm >= P.M || tid >= ntab) return;
-            const int p = tid >= nt0 ? 1 : 0, n = tid - (p ? nt0 : 0);
-            if (4 * n >= P.r[p]) return;
-            ld_fix2x4(fix2_at(xw, mm * P.N1 + (p ? P.off1 : 0) + 4 * n), pre);
-        };
-        for (int it = 0; it < P.M + kAhead && ok; ++it) {
-            if (it == kAhead) prefetch(0);
-            // ---------------- stage 1 of linear it
-            if (it == 0 && nw == 0 && tid == 0) {
+        // Two warp groups run the two stages of different linears at once:
+        // warps [0, k1) stage 1 of linear m, warps [k1, kCW) stage 2 of linear
+        // m - (how far stage 1 has got); each group synchronises on a named
+        // barrier of its own.  Stage 1 can run ahead of stage 2 as far as the
+        // slot ring allows (the producer refills a slot once stage 2 freed it).
+        const int k1 = P.k1, n1t = 32 * k1, n2t = kCT - n1t;
+        if (warp < k1) {
+            // ---------------- stage 1 group (named barrier 2)
+            if (nw == 0) {
                 // a CTA without input words still counts itself into linear 0's
                 // element 0
-                send_count2(fix2_at(xw, 0));
+                if (tid == 0) send_count2(fix2_at(xw, 0));
+            } else {
+                for (int m = 0; m < P.M && ok; ++m) {
+                    unsigned char *b = slot(m);
+                    // tables of g . x (8 per input word and path), once the slice landed
+                    bool got = true;
+                    if (tid == 0)
+                        got = wait_bar_m(vbar + m % kSlots, (unsigned)((m / kSlots) & 1),
+                                         P.ws_words);
+                    if (!gsync_and(2, n1t, got)) {
+                        ok = false;
+                        break;
+                    }
+                    if (tid != 0) mbar_try_wait(vbar + m % kSlots, (unsigned)((m / kSlots) & 1));
+                    for (int idx = tid; idx < np * 8 * nw; idx += n1t) {
+                        const int p = idx / (8 * nw), n = idx - p * 8 * nw;
+                        const float4 xv = *reinterpret_cast<const float4 *>(xs + 4 * n);
+                        const uint2 gw = *reinterpret_cast<const uint2 *>(b + o.g[p] + 8 * n);
+                        const float4 v =
+                            make_float4(xv.x * half_bits_to_float((uint16_t)(gw.x & 0xffffu)),
+                                        xv.y * half_bits_to_float((uint16_t)(gw.x >> 16)),
+                                        xv.z * half_bits_to_float((uint16_t)(gw.y & 0xffffu)),
+                                        xv.w * half_bits_to_float((uint16_t)(gw.y >> 16)));
+                        store_table(g_smem + o.t1 + idx * 128, v, lane);
+                    }
+                    gsync(2, n1t);
+                    const int xm = m * P.N1;  // the linear's first element
+                    for (int u = warp; u < cbs; u += k1) {
+                        const int p = u >= R0 ? 1 : 0, cb = u - (p ? R0 : 0);
+                        const int r = P.r[p];
+                        const int col = 32 * cb + lane, cc = min(col, r - 1);
+                        const uint32_t *Vw = reinterpret_cast<const uint32_t *>(b + o.V[p]) + cc;
+                        const uint32_t tb = (uint32_t)(o.t1 + p * 8 * nw * 128);
+                        float acc0 = 0.f, acc1 = 0.f;
+                        int w = 0;
+                        for (; w + 2 <= nw; w += 2) {
+                            const uint32_t w0 = Vw[w * r], w1 = Vw[(w + 1) * r];
+                            acc0 += lut_word(w0, copy, tb + w * 1024);
+                            acc1 += lut_word(w1, copy, tb + (w + 1) * 1024);
+                        }
+                        if (w < nw) acc0 += lut_word(Vw[w * r], copy, tb + w * 1024);
+                        if (col < r)
+                            send_fix2(fix2_at(xw, xm + (p ? P.off1 : 0) + col), acc0 + acc1,
+                                      P.fix_limit, err);
+                    }
+                    gsync(2, n1t);  // t1 is rebuilt by the next linear
+                }
             }
-            if (it < P.M && nw > 0) {
-                const int m = it;
-                unsigned char *b = slot(m);
-                // tables of g . x (8 per input word and path), once the slice landed
-                bool got = true;
-                if (tid == 0) got = wait_bar_m(vbar + m % kSlots, (unsigned)((m / kSlots) & 1), P.ws_words);
-                if (!csync_and_m(got)) {
+        } else {
+            // ---------------- stage 2 group (named barrier 3)
+            const int t2 = tid - n1t, w2 = warp - k1, nw2 = kCW - k1;
+            const bool lead2 = t2 == 0;
+            const int S0 = s2_parts(R0), S1 = np > 1 ? s2_parts(R1) : 0;
+            const int rb = (nrows + 31) >> 5, nu0 = rb * S0, nu = nu0 + rb * S1;
+            float *y = reinterpret_cast<float *>(g_smem + o.y);  // part slots
+            // the exchange words a thread polls for stage 2 (its table t2 when
+            // t2 < ntab), loaded while the row sums of the linear before run,
+            // so that the L2 round trip overlaps them
+            unsigned long long pre[8] = {0ull, 0ull, 0ull, 0ull, 0ull, 0ull, 0ull, 0ull};
+            auto prefetch = [&](int mm) {
+                if (mm < 0 || mm >= P.M || t2 >= ntab) return;
+                const int p = t2 >= nt0 ? 1 : 0, n = t2 - (p ? nt0 : 0);
+                if (4 * n >= P.r[p]) return;
+                ld_fix2x4(fix2_at(xw, mm * P.N1 + (p ? P.off1 : 0) + 4 * n), pre);
+            };
+            prefetch(0);
+            for (int mm = 0; mm < P.M && ok; ++mm) {
+                const int xm = mm * P.N1;  // the linear's first element
+                unsigned char *b = slot(mm);
+                // the slot's U rows, h and l (the lead waits, the rest observe the phase)
+                bool u_ok = true;
+                if (lead2)
+                    u_ok = wait_bar_m(ubar + mm % kSlots, (unsigned)((mm / kSlots) & 1),
+                                      P.ws_words);
+                if (!gsync_and(3, n2t, u_ok)) {
                     ok = false;
                     break;
                 }
-                if (tid != 0) mbar_try_wait(vbar + m % kSlots, (unsigned)((m / kSlots) & 1));
-                for (int idx = tid; idx < np * 8 * nw; idx += kCT) {
-                    const int p = idx / (8 * nw), n = idx - p * 8 * nw;
-                    const float4 xv = *reinterpret_cast<const float4 *>(xs + 4 * n);
-                    const uint2 gw = *reinterpret_cast<const uint2 *>(b + o.g[p] + 8 * n);
-                    const float4 v = make_float4(xv.x * half_bits_to_float((uint16_t)(gw.x & 0xffffu)),
-                                                 xv.y * half_bits_to_float((uint16_t)(gw.x >> 16)),
-                                                 xv.z * half_bits_to_float((uint16_t)(gw.y & 0xffffu)),
-                                                 xv.w * half_bits_to_float((uint16_t)(gw.y >> 16)));
-                    store_table(g_smem + o.t1 + idx * 128, v, lane);
-                }
-                csync_m();
-                const int xm = m * P.N1;  // the linear's first element
-                for (int u = warp; u < cbs; u += kCW) {
-                    const int p = u >= R0 ? 1 : 0, cb = u - (p ? R0 : 0);
-                    const int r = P.r[p];
-                    const int col = 32 * cb + lane, cc = min(col, r - 1);
-                    const uint32_t *Vw = reinterpret_cast<const uint32_t *>(b + o.V[p]) + cc;
-                    const uint32_t tb = (uint32_t)(o.t1 + p * 8 * nw * 128);
-                    float acc0 = 0.f, acc1 = 0.f;
-                    int w = 0;
-                    for (; w + 2 <= nw; w += 2) {
-                        const uint32_t w0 = Vw[w * r], w1 = Vw[(w + 1) * r];
-                        acc0 += lut_word(w0, copy, tb + w * 1024);
-                        acc1 += lut_word(w1, copy, tb + (w + 1) * 1024);
-                    }
-                    if (w < nw) acc0 += lut_word(Vw[w * r], copy, tb + w * 1024);
-                    if (col < r)
-                        send_fix2(fix2_at(xw, xm + (p ? P.off1 : 0) + col), acc0 + acc1,
-                                  P.fix_limit, err);
-                }
-                csync_m();  // t1 is rebuilt by the next linear
-            }
-            // ---------------- stage 2 of linear it - kAhead
-            const int mm = it - kAhead;
-            if (mm < 0) continue;
-            const int xm = mm * P.N1;  // the linear's first element
-            unsigned char *b = slot(mm);
-            // the slot's U rows, h and l (thread 0 waits, the rest observe the phase)
-            bool u_ok = true;
-            if (tid == 0) u_ok = wait_bar_m(ubar + mm % kSlots, (unsigned)((mm / kSlots) & 1), P.ws_words);
-            if (!csync_and_m(u_ok)) {
-                ok = false;
-                break;
-            }
-            if (tid != 0) mbar_try_wait(ubar + mm % kSlots, (unsigned)((mm / kSlots) & 1));
-            int pok = 1;
-            if (res && mm == 0 && tid == 0) {
-                // the sum of squares of the whole input (all CTAs counted)
-                unsigned long long wh = 0, wl = 0, t0 = 0;
-                for (int spin = 0;; ++spin) {
-                    ld_fix2(fix2_at(xw, (int)words), wh, wl);
-                    if (counted2(wh, wl, n_first)) break;
-                    if ((spin & 15) == 15) {
-                        if (ld_relaxed_gpu(err) != 0u) {
-                            pok = 0;
-                            break;
-                        }
-                        const unsigned long long now = globaltimer_ns();
-                        if (t0 == 0) t0 = now;
-                        if (now - t0 > kWaitLimitNs) {
-                            atomicCAS(err, 0u, static_cast<unsigned>(LB_ERR_TIMEOUT));
-                            pok = 0;
-                            break;
-                        }
-                    }
-                }
-                if (pok) s_inv = rsqrtf(dec_fix2(wh, wl));
-            }
-            for (int idx = tid; idx < ntab && pok; idx += kCT) {
-                const int p = idx >= nt0 ? 1 : 0, n = idx - (p ? nt0 : 0);
-                const int r = P.r[p];
-                float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-                if (4 * n < r) {
-                    const uint2 lw = *reinterpret_cast<const uint2 *>(b + o.l[p] + 8 * n);
-                    const unsigned long long *wd = fix2_at(xw, xm + (p ? P.off1 : 0) + 4 * n);
-                    unsigned long long a[8], t0 = 0;
+                if (!lead2) mbar_try_wait(ubar + mm % kSlots, (unsigned)((mm / kSlots) & 1));
+                int pok = 1;
+                if (res && mm == 0 && lead2) {
+                    // the sum of squares of the whole input (all CTAs counted)
+                    unsigned long long wh = 0, wl = 0, t0 = 0;
                     for (int spin = 0;; ++spin) {
-                        if (spin == 0 && idx == tid) {
-#pragma unroll
-                            for (int k = 0; k < 8; ++k) a[k] = pre[k];
-                        } else {
-                            ld_fix2x4(wd, a);
-                        }
-                        const unsigned want0 = mm == 0 && idx == 0 ? n_first : n_contrib;
-                        if (counted2x4(a, want0, n_contrib)) break;
+                        ld_fix2(fix2_at(xw, (int)words), wh, wl);
+                        if (counted2(wh, wl, n_first)) break;
                         if ((spin & 15) == 15) {
                             if (ld_relaxed_gpu(err) != 0u) {
                                 pok = 0;
@@ -340,69 +326,82 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
                             }
                         }
                     }
-                    v = make_float4(dec_fix2(a[0], a[1]) * half_bits_to_float((uint16_t)(lw.x & 0xffffu)),
-                                    dec_fix2(a[2], a[3]) * half_bits_to_float((uint16_t)(lw.x >> 16)),
-                                    dec_fix2(a[4], a[5]) * half_bits_to_float((uint16_t)(lw.y & 0xffffu)),
-                                    dec_fix2(a[6], a[7]) * half_bits_to_float((uint16_t)(lw.y >> 16)));
+                    if (pok) s_inv = rsqrtf(dec_fix2(wh, wl));
                 }
-                store_table(g_smem + o.t2 + idx * 128, v, lane);
-            }
-            if (!csync_and_m(pok)) {
-                ok = false;
-                break;
-            }
-            prefetch(mm + 1);
-            // every CTA contributed to linear 0's words before any could
-            // complete, so all have read the epoch: the next launch may use
-            // the other buffer
-            if (mm == 0 && c == 0 && tid == 0) P.ws_words[kEpochWord] = epoch + 1u;
-            const int rb = (nrows + 31) >> 5;
-            for (int u = warp; u < np * rb; u += kCW) {
-                const int p = u / rb, blk = u - p * rb;
-                const int R = (P.r[p] + 31) >> 5;
-                const int row = 32 * blk + lane, rr = min(row, nrows - 1);
-                const float hs = half_bits_to_float(reinterpret_cast<const uint16_t *>(b + o.h[p])[rr]);
-                const uint32_t *Uw = reinterpret_cast<const uint32_t *>(b + o.U[p]) + rr * R;
-                const uint32_t tb = (uint32_t)(o.t2 + (p ? nt0 : 0) * 128);
-                float acc0 = 0.f, acc1 = 0.f;
-                int w = 0;
-                if ((R & 3) == 0) {
-                    // rows of R = 4k words are 16-byte aligned: one 128-bit load takes four
-                    // words (a warp's 32 rows at a stride of R words fall in few banks, so
-                    // a 32-bit load per word would replay up to 16 times); even words still
-                    // go to acc0 and odd ones to acc1, in order
-                    for (; w < R; w += 4) {
-                        const uint4 q = *reinterpret_cast<const uint4 *>(Uw + w);
-                        acc0 += lut_word(q.x, copy, tb + w * 1024);
-                        acc1 += lut_word(q.y, copy, tb + (w + 1) * 1024);
-                        acc0 += lut_word(q.z, copy, tb + (w + 2) * 1024);
-                        acc1 += lut_word(q.w, copy, tb + (w + 3) * 1024);
+                for (int idx = t2; idx < ntab && pok; idx += n2t) {
+                    const int p = idx >= nt0 ? 1 : 0, n = idx - (p ? nt0 : 0);
+                    const int r = P.r[p];
+                    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+                    if (4 * n < r) {
+                        const uint2 lw = *reinterpret_cast<const uint2 *>(b + o.l[p] + 8 * n);
+                        const unsigned long long *wd = fix2_at(xw, xm + (p ? P.off1 : 0) + 4 * n);
+                        unsigned long long a[8], t0 = 0;
+                        for (int spin = 0;; ++spin) {
+                            if (spin == 0 && idx == t2) {
+#pragma unroll
+                                for (int k = 0; k < 8; ++k) a[k] = pre[k];
+                            } else {
+                                ld_fix2x4(wd, a);
+                            }
+                            const unsigned want0 = mm == 0 && idx == 0 ? n_first : n_contrib;
+                            if (counted2x4(a, want0, n_contrib)) break;
+                            if ((spin & 15) == 15) {
+                                if (ld_relaxed_gpu(err) != 0u) {
+                                    pok = 0;
+                                    break;
+                                }
+                                const unsigned long long now = globaltimer_ns();
+                                if (t0 == 0) t0 = now;
+                                if (now - t0 > kWaitLimitNs) {
+                                    atomicCAS(err, 0u, static_cast<unsigned>(LB_ERR_TIMEOUT));
+                                    pok = 0;
+                                    break;
+                                }
+                            }
+                        }
+                        v = make_float4(
+                            dec_fix2(a[0], a[1]) * half_bits_to_float((uint16_t)(lw.x & 0xffffu)),
+                            dec_fix2(a[2], a[3]) * half_bits_to_float((uint16_t)(lw.x >> 16)),
+                            dec_fix2(a[4], a[5]) * half_bits_to_float((uint16_t)(lw.y & 0xffffu)),
+                            dec_fix2(a[6], a[7]) * half_bits_to_float((uint16_t)(lw.y >> 16)));
                     }
+                    store_table(g_smem + o.t2 + idx * 128, v, lane);
                 }
-                for (; w + 2 <= R; w += 2) {
-                    const uint32_t w0 = Uw[w], w1 = Uw[w + 1];
-                    acc0 += lut_word(w0, copy, tb + w * 1024);
-                    acc1 += lut_word(w1, copy, tb + (w + 1) * 1024);
+                if (!gsync_and(3, n2t, pok)) {
+                    ok = false;
+                    break;
                 }
-                if (w < R) acc0 += lut_word(Uw[w], copy, tb + w * 1024);
-                // at most two paths meet in a row: 0 + a + b is exact in either order
-                if (row < nrows) atomicAdd(y + row, (acc0 + acc1) * hs);
+                prefetch(mm + 1);
+                // every CTA contributed to linear 0's element 0 before it could
+                // complete, so all have read the epoch: the next launch may use
+                // the other buffer
+                if (mm == 0 && c == 0 && lead2) P.ws_words[kEpochWord] = epoch + 1u;
+                // parts of 32 rows x up to four words of one path
+                for (int u = w2; u < nu; u += nw2) {
+                    const int p = u >= nu0 ? 1 : 0, v = u - (p ? nu0 : 0), S = p ? S1 : S0;
+                    const int bb = v / S, sp = v - bb * S;
+                    s2_part(reinterpret_cast<const uint32_t *>(b + o.U[p]), p ? R1 : R0,
+                            reinterpret_cast<const uint16_t *>(b + o.h[p]),
+                            (uint32_t)(o.t2 + (p ? nt0 : 0) * 128), nrows, bb, sp,
+                            y + (size_t)((p ? S0 : 0) + sp) * nrows, copy, lane);
+                }
+                gsync(3, n2t);
+                // the slot is free for the producer
+                if (lead2) mbar_arrive(fbar + mm % kSlots);
+                const float sc = s_inv;  // 1 unless the input is a residual add
+                for (int i = t2; i < nrows; i += n2t) {
+                    const size_t at = (size_t)mm * P.d_out + o0 + i;
+                    const float v = s2_combine(y, nrows, S0 + S1, i) * sc;
+                    if (P.y_fp32)
+                        static_cast<float *>(P.y)[at] = v;
+                    else
+                        static_cast<uint16_t *>(P.y)[at] = float_to_bf16_bits(v);
+                }
+                // the next linear's parts overwrite the slots: its first group
+                // barrier (after its slot wait) orders them after these reads
             }
-            csync_m();
-            // the slot is free for the producer
-            if (tid == 0) mbar_arrive(fbar + mm % kSlots);
-            const float sc = s_inv;  // 1 unless the input is a residual add
-            for (int i = tid; i < nrows; i += kCT) {
-                const size_t at = (size_t)mm * P.d_out + o0 + i;
-                if (P.y_fp32)
-                    static_cast<float *>(P.y)[at] = y[i] * sc;
-                else
-                    static_cast<uint16_t *>(P.y)[at] = float_to_bf16_bits(y[i] * sc);
-                y[i] = 0.f;
-            }
-            csync_m();
         }
-        if (!ok && tid == 0) s_ok = 0;
+        if (!ok) s_ok = 0;
     }
     __syncthreads();
     if (!s_ok && tid == 0) {
@@ -429,7 +428,7 @@ MultiLayout layout_of(const lb_linear &L, int N) {
         return off;
     };
     // one slot: V and g slices, U rows and h of each path
-    int ntab2 = 0;
+    int ntab2 = 0, nslot = 0;
     for (int p = 0; p < 2; ++p) {
         const bool on = p < L.n_paths;
         const int r = on ? L.path[p].r : 0, R = (r + 31) / 32;
@@ -439,6 +438,7 @@ MultiLayout layout_of(const lb_linear &L, int N) {
         o.h[p] = take(2 * nrows);
         o.l[p] = take(2 * r);
         ntab2 += 8 * R;
+        nslot += on ? s2_parts(R) : 0;
     }
     o.slot_bytes = up16(at);
     at = 0;
@@ -449,9 +449,41 @@ MultiLayout layout_of(const lb_linear &L, int N) {
     o.t1 = take(L.n_paths * 8 * nw * 128);
     at = (at + 1023) & ~1023;
     o.t2 = take(ntab2 * 128);
-    o.y = take(4 * nrows);
+    o.y = take(4 * nrows * nslot);
     o.bytes = at;
     return o;
+}
+
+// Warps of the stage-1 group: the split of the 15 compute warps whose
+// slower group is fastest, counting per warp its units (stage 1: 32 columns
+// x the input slice; stage 2: 32 rows x up to four words of one path, plus
+// the tables it polls) in sign words with one word of fixed cost per unit.
+int stage1_warps(const lb_linear &L, int N) {
+    const int W = L.d_in / 32, n_s1 = s1_ctas(W, N);
+    const int nw = (W + n_s1 - 1) / n_s1, nrows = 8 * ((L.d_out / 8 + N - 1) / N);
+    const int rb = (nrows + 31) / 32;
+    int cbs = 0, nu = 0, ntab = 0, part = 0;
+    for (int p = 0; p < L.n_paths; ++p) {
+        const int R = (L.path[p].r + 31) / 32;
+        cbs += R;
+        nu += rb * s2_parts(R);
+        ntab += 8 * R;
+        part = std::max(part, std::min(R, kPartWords));
+    }
+    int best = 1;
+    double best_t = 1e300;
+    for (int k1 = 1; k1 < kCW; ++k1) {
+        const int k2 = kCW - k1;
+        const double t1 = (double)((cbs + k1 - 1) / k1) * (nw + 1);
+        const double t2 = (double)((nu + k2 - 1) / k2) * (part + 1) +
+                          2.0 * ((ntab + 32 * k2 - 1) / (32 * k2));
+        const double t = std::max(t1, t2);
+        if (t < best_t - 1e-9) {
+            best_t = t;
+            best = k1;
+        }
+    }
+    return best;
 }
 
 int rsum(const lb_linear &L) {
@@ -530,6 +562,7 @@ cudaError_t launch_decode_multi(const lb_linear *L, int M, const void *x, int x_
     P.xw = static_cast<unsigned long long *>(xw);
     P.fix_limit = fix2_limit(num_sms);
     P.o = layout_of(A, num_sms);
+    P.k1 = stage1_warps(A, num_sms);
     if (P.o.bytes > max_smem) return cudaErrorCooperativeLaunchTooLarge;
     for (int m = 0; m < M; ++m)
         for (int p = 0; p < A.n_paths; ++p) {
