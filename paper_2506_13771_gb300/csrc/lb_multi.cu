@@ -53,7 +53,7 @@ struct MultiLayout {
 
 struct MultiParams {
     int d_in, d_out, np, r[2], M, N1, off1;
-    int k1;  // compute warps of the stage-1 group (the rest run stage 2)
+    int k1;  // compute warps of the stage-1 group (the rest run stage 2); 0: phased
     const void *x;  // bf16 [d_in] (x_fp32 = 0), or fp32 (x_fp32 = 1)
     int x_fp32;     // 3: residual input, see res_a
     // x_fp32 = 3: x = res_a + res_y (fp32 [d_in]), written back to res_a, and
@@ -220,7 +220,11 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
         // m - (how far stage 1 has got); each group synchronises on a named
         // barrier of its own.  Stage 1 can run ahead of stage 2 as far as the
         // slot ring allows (the producer refills a slot once stage 2 freed it).
-        const int k1 = P.k1, n1t = 32 * k1, n2t = kCT - n1t;
+        // Phased (k1 = 0, for few linears): every compute warp runs stage 1 of
+        // all the linears, then stage 2 of all of them.
+        const bool phased = P.k1 == 0;
+        const int k1 = phased ? kCW : P.k1, n1t = 32 * k1;
+        const int g2 = phased ? 0 : k1, n2t = kCT - 32 * g2;
         if (warp < k1) {
             // ---------------- stage 1 group (named barrier 2)
             if (nw == 0) {
@@ -274,9 +278,11 @@ __global__ void __launch_bounds__(kMT, 1) k_decode_multi(const __grid_constant__
                     gsync(2, n1t);  // t1 is rebuilt by the next linear
                 }
             }
-        } else {
+        }
+        if (phased) csync_m();
+        if (warp >= g2 && ok) {
             // ---------------- stage 2 group (named barrier 3)
-            const int t2 = tid - n1t, w2 = warp - k1, nw2 = kCW - k1;
+            const int t2 = tid - 32 * g2, w2 = warp - g2, nw2 = kCW - g2;
             const bool lead2 = t2 == 0;
             const int S0 = s2_parts(R0), S1 = np > 1 ? s2_parts(R1) : 0;
             const int rb = (nrows + 31) >> 5, nu0 = rb * S0, nu = nu0 + rb * S1;
@@ -454,11 +460,16 @@ MultiLayout layout_of(const lb_linear &L, int N) {
     return o;
 }
 
-// Warps of the stage-1 group: the split of the 15 compute warps whose
-// slower group is fastest, counting per warp its units (stage 1: 32 columns
-// x the input slice; stage 2: 32 rows x up to four words of one path, plus
-// the tables it polls) in sign words with one word of fixed cost per unit.
-int stage1_warps(const lb_linear &L, int N) {
+// Warps of the stage-1 group, or 0 for the phased schedule: the choice with
+// the shortest estimated launch for M linears.  Per warp, units cost their
+// sign words plus a fixed cost measured per unit: a stage-1 unit (32 columns
+// x the input slice) its words + 3 (mostly its exchange sends), a stage-2
+// part (32 rows x up to four words) its words + 1, a round of polled tables
+// 3; an exchange takes about 20 such units to complete.  Split: max(M t1, t1
+// + exchange + M t2); phased: M t1 + what is left of the first exchange
+// after the other linears' stage 1, + M t2, both stages on all 15 warps
+// (phased needs M <= kSlots).
+int stage1_warps(const lb_linear &L, int N, int M) {
     const int W = L.d_in / 32, n_s1 = s1_ctas(W, N);
     const int nw = (W + n_s1 - 1) / n_s1, nrows = 8 * ((L.d_out / 8 + N - 1) / N);
     const int rb = (nrows + 31) / 32;
@@ -470,14 +481,21 @@ int stage1_warps(const lb_linear &L, int N) {
         ntab += 8 * R;
         part = std::max(part, std::min(R, kPartWords));
     }
-    int best = 1;
-    double best_t = 1e300;
+    const double xchg = 20.0;
+    auto t1_of = [&](int k) { return (double)((cbs + k - 1) / k) * (nw + 3); };
+    auto t2_of = [&](int k) {
+        return (double)((nu + k - 1) / k) * (part + 1) + 3.0 * ((ntab + 32 * k - 1) / (32 * k)) +
+               1.0;
+    };
+    // phased only while every linear has a slot of its own (stage 1 of linear
+    // kSlots would wait for a slot that only stage 2 frees)
+    int best = 0;
+    double best_t = M <= kSlots ? M * t1_of(kCW) + std::max(0.0, xchg - (M - 1) * t1_of(kCW)) +
+                                      M * t2_of(kCW)
+                                : 1e300;
     for (int k1 = 1; k1 < kCW; ++k1) {
-        const int k2 = kCW - k1;
-        const double t1 = (double)((cbs + k1 - 1) / k1) * (nw + 1);
-        const double t2 = (double)((nu + k2 - 1) / k2) * (part + 1) +
-                          2.0 * ((ntab + 32 * k2 - 1) / (32 * k2));
-        const double t = std::max(t1, t2);
+        const double t1 = t1_of(k1), t2 = t2_of(kCW - k1);
+        const double t = std::max(M * t1, t1 + xchg + M * t2);
         if (t < best_t - 1e-9) {
             best_t = t;
             best = k1;
@@ -562,7 +580,7 @@ cudaError_t launch_decode_multi(const lb_linear *L, int M, const void *x, int x_
     P.xw = static_cast<unsigned long long *>(xw);
     P.fix_limit = fix2_limit(num_sms);
     P.o = layout_of(A, num_sms);
-    P.k1 = stage1_warps(A, num_sms);
+    P.k1 = stage1_warps(A, num_sms, M);
     if (P.o.bytes > max_smem) return cudaErrorCooperativeLaunchTooLarge;
     for (int m = 0; m < M; ++m)
         for (int p = 0; p < A.n_paths; ++p) {
