@@ -250,6 +250,24 @@ lb_status littlebit_train_backward(const lb_train_linear *L, const float *x, con
                                    int64_t T, float k_smooth, const lb_train_grad *grads,
                                    float *dx, void *ws, size_t ws_bytes, lb_stream_t stream);
 
+/* The same backward reusing its forward, as a training framework keeps a
+ * forward's activations for the backward: littlebit_train_forward leaves in
+ * its workspace the signs of U and V folded with h and g, l, the latent t
+ * and z = l . t, and a fingerprint of (L's shapes and pointers, x, T); this
+ * call uses them instead of recomputing them (the sign folds and the t
+ * product are the part of a backward the forward already did).  Its
+ * arguments and results are those of littlebit_train_backward.  Contract:
+ * the workspace's most recent forward was littlebit_train_forward with the
+ * same L, x and T, and neither the factors, the scales nor x have changed
+ * since (a backward may come in between).  A fingerprint that differs is
+ * refused on the device: LB_ERR_PLAN is recorded in the workspace's error
+ * word (read it with littlebit_poll_error) and the gradients are
+ * meaningless. */
+lb_status littlebit_train_backward_saved(const lb_train_linear *L, const float *x,
+                                         const float *dy, int64_t T, float k_smooth,
+                                         const lb_train_grad *grads, float *dx, void *ws,
+                                         size_t ws_bytes, lb_stream_t stream);
+
 /* Workspace bytes littlebit_stack_prepare / littlebit_stack_forward need
  * (0 if the arguments are invalid). */
 size_t littlebit_stack_workspace_size(const lb_linear *lin, int32_t n_layers, int32_t head_dim);

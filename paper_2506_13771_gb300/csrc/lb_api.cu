@@ -371,6 +371,33 @@ lb_status littlebit_dual_svid(const float *W, int32_t d_out, int32_t d_in, int32
 }
 
 namespace {
+// FNV-1a over a QAT linear's shapes and pointers, the input pointer and T:
+// what a forward leaves in its workspace is keyed by it.
+unsigned long long train_tag(const lb_train_linear *L, const float *x, int64_t T) {
+    unsigned long long h = 1469598103934665603ull;
+    auto mix = [&h](unsigned long long v) {
+        for (int b = 0; b < 8; ++b) {
+            h ^= (v >> (8 * b)) & 0xffu;
+            h *= 1099511628211ull;
+        }
+    };
+    mix((unsigned long long)L->d_in);
+    mix((unsigned long long)L->d_out);
+    mix((unsigned long long)L->n_paths);
+    for (int p = 0; p < L->n_paths; ++p) {
+        const lb_train_path &P = L->path[p];
+        mix((unsigned long long)P.r);
+        mix(reinterpret_cast<uintptr_t>(P.u));
+        mix(reinterpret_cast<uintptr_t>(P.v));
+        mix(reinterpret_cast<uintptr_t>(P.g));
+        mix(reinterpret_cast<uintptr_t>(P.l));
+        mix(reinterpret_cast<uintptr_t>(P.h));
+    }
+    mix(reinterpret_cast<uintptr_t>(x));
+    mix((unsigned long long)T);
+    return h;
+}
+
 lb_status check_train(const lb_train_linear *L) {
     if (!L || L->d_in <= 0 || L->d_out <= 0 || (L->n_paths != 1 && L->n_paths != 2))
         return LB_ERR_INVALID_ARG;
@@ -402,12 +429,14 @@ lb_status littlebit_train_forward(const lb_train_linear *L, const float *x, int6
     if (!ws || ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) ||
         ws_bytes < littlebit_train_workspace_size(L, T))
         return LB_ERR_WORKSPACE;
-    return from_cuda(lb::launch_train_forward(*L, x, T, y, ws, (cudaStream_t)stream));
+    return from_cuda(lb::launch_train_forward(*L, x, T, y, ws, train_tag(L, x, T),
+                                              (cudaStream_t)stream));
 }
 
-lb_status littlebit_train_backward(const lb_train_linear *L, const float *x, const float *dy,
-                                   int64_t T, float k_smooth, const lb_train_grad *grads,
-                                   float *dx, void *ws, size_t ws_bytes, lb_stream_t stream) {
+namespace {
+lb_status train_backward(const lb_train_linear *L, const float *x, const float *dy, int64_t T,
+                         float k_smooth, const lb_train_grad *grads, float *dx, void *ws,
+                         size_t ws_bytes, bool saved, lb_stream_t stream) {
     lb_status st = check_train(L);
     if (st != LB_OK) return st;
     if (T < 0 || T > INT32_MAX || !grads || !(k_smooth > 0.f)) return LB_ERR_INVALID_ARG;
@@ -423,8 +452,22 @@ lb_status littlebit_train_backward(const lb_train_linear *L, const float *x, con
     if (!ws || ((reinterpret_cast<uintptr_t>(ws) & 255u) != 0) ||
         ws_bytes < littlebit_train_workspace_size(L, T))
         return LB_ERR_WORKSPACE;
-    return from_cuda(lb::launch_train_backward(*L, x, dy, T, k_smooth, grads, dx, ws,
-                                               (cudaStream_t)stream));
+    return from_cuda(lb::launch_train_backward(*L, x, dy, T, k_smooth, grads, dx, ws, saved,
+                                               train_tag(L, x, T), (cudaStream_t)stream));
+}
+}  // namespace
+
+lb_status littlebit_train_backward(const lb_train_linear *L, const float *x, const float *dy,
+                                   int64_t T, float k_smooth, const lb_train_grad *grads,
+                                   float *dx, void *ws, size_t ws_bytes, lb_stream_t stream) {
+    return train_backward(L, x, dy, T, k_smooth, grads, dx, ws, ws_bytes, false, stream);
+}
+
+lb_status littlebit_train_backward_saved(const lb_train_linear *L, const float *x,
+                                         const float *dy, int64_t T, float k_smooth,
+                                         const lb_train_grad *grads, float *dx, void *ws,
+                                         size_t ws_bytes, lb_stream_t stream) {
+    return train_backward(L, x, dy, T, k_smooth, grads, dx, ws, ws_bytes, true, stream);
 }
 
 size_t littlebit_stack_workspace_size(const lb_linear *lin, int32_t n_layers, int32_t head_dim) {

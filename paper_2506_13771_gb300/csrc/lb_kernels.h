@@ -132,11 +132,14 @@ cudaError_t gemm_tf32(const GemmOperand &A, const GemmOperand &B, float *C, long
 // the sum of the paths' ranks (a 256-byte header whose first word is the
 // error word, then the buffers).
 size_t qat_ws_bytes(int d_in, int d_out, int rsum, long long T);
+// tag: a fingerprint of (L, x, T); the forward records it in the workspace,
+// a backward with saved = true reuses the forward's folded factors, l, t and
+// z instead of recomputing them and records LB_ERR_PLAN if the tags differ.
 cudaError_t launch_train_forward(const lb_train_linear &L, const float *x, long long T, float *y,
-                                 void *ws, cudaStream_t s);
+                                 void *ws, unsigned long long tag, cudaStream_t s);
 cudaError_t launch_train_backward(const lb_train_linear &L, const float *x, const float *dy,
                                   long long T, float k, const lb_train_grad *G, float *dx, void *ws,
-                                  cudaStream_t s);
+                                  bool saved, unsigned long long tag, cudaStream_t s);
 
 // Bounded-wait diagnostic (lb_persistent.cu).
 cudaError_t launch_wait_timeout(unsigned *ws_words, cudaStream_t s);

@@ -256,6 +256,17 @@ cudaError_t forward_latent(const lb_train_linear &L, const GemmOperand &Xk, long
     return e;
 }
 
+// The workspace's record of the forward it holds (header words kPlanWord ..
+// + 1): written by a forward, compared by a backward that reuses its state
+// (a mismatch records LB_ERR_PLAN).
+__global__ void k_qat_tag(unsigned *ws_words, unsigned long long tag, int check) {
+    unsigned long long *w = reinterpret_cast<unsigned long long *>(ws_words + kPlanWord);
+    if (!check)
+        *w = tag;
+    else if (*w != tag)
+        atomicCAS(ws_words + kErrWord, 0u, static_cast<unsigned>(LB_ERR_PLAN));
+}
+
 }  // namespace
 
 size_t qat_ws_bytes(int d_in, int d_out, int rsum, long long T) {
@@ -265,7 +276,7 @@ size_t qat_ws_bytes(int d_in, int d_out, int rsum, long long T) {
 }
 
 cudaError_t launch_train_forward(const lb_train_linear &L, const float *x, long long T, float *y,
-                                 void *ws, cudaStream_t s) {
+                                 void *ws, unsigned long long tag, cudaStream_t s) {
     QatBuf b = carve(ws, L.d_in, L.d_out, rsum_of(L), T, nullptr);
     cudaError_t e = cudaMemsetAsync(b.err, 0, sizeof(unsigned), s);
     GemmOperand Xk;
@@ -275,12 +286,17 @@ cudaError_t launch_train_forward(const lb_train_linear &L, const float *x, long 
     if (e == cudaSuccess)
         e = gemm_tf32(GemmOperand{b.z, (int)T, b.R, b.ldr}, GemmOperand{b.Uh, L.d_out, b.R, b.ldr},
                       y, L.d_out, false, b.part, b.part_floats, b.err, s);
+    // the folds, l, t and z stay in the workspace for a backward that reuses them
+    if (e == cudaSuccess) {
+        k_qat_tag<<<1, 1, 0, s>>>(static_cast<unsigned *>(ws), tag, 0);
+        e = cudaGetLastError();
+    }
     return e;
 }
 
 cudaError_t launch_train_backward(const lb_train_linear &L, const float *x, const float *dy,
                                   long long T, float k, const lb_train_grad *G, float *dx, void *ws,
-                                  cudaStream_t s) {
+                                  bool saved, unsigned long long tag, cudaStream_t s) {
     QatBuf b = carve(ws, L.d_in, L.d_out, rsum_of(L), T, nullptr);
     const int Ti = (int)T, R = b.R;
     cudaError_t e = cudaMemsetAsync(b.err, 0, sizeof(unsigned), s);
@@ -290,7 +306,15 @@ cudaError_t launch_train_backward(const lb_train_linear &L, const float *x, cons
     if (e == cudaSuccess) e = k_major(dy, Ti, L.d_out, b.dYp, b.ldo, &dYk, s);
     if (e == cudaSuccess) e = copy_t(x, Ti, L.d_in, L.d_in, true, b.XT, b.ldT, s);
     if (e == cudaSuccess) e = copy_t(dy, Ti, L.d_out, L.d_out, true, b.dYT, b.ldT, s);
-    if (e == cudaSuccess) e = forward_latent(L, Xk, T, b, s);
+    if (e == cudaSuccess) {
+        if (saved) {
+            // the forward's folds, l, t and z, if the workspace holds this forward
+            k_qat_tag<<<1, 1, 0, s>>>(static_cast<unsigned *>(ws), tag, 1);
+            e = cudaGetLastError();
+        } else {
+            e = forward_latent(L, Xk, T, b, s);
+        }
+    }
     // dYz = dY^T z -> dh, dU per path
     if (e == cudaSuccess) e = copy_t(b.z, Ti, R, b.ldr, true, b.zT, b.ldT, s);
     if (e == cudaSuccess)

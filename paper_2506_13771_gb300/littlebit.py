@@ -26,7 +26,7 @@ EXPORTED = ["littlebit_status_string", "littlebit_pack", "littlebit_workspace_si
             "littlebit_linear_forward", "littlebit_linear_latent", "littlebit_linear_expand",
             "littlebit_dual_svid_workspace_size", "littlebit_dual_svid",
             "littlebit_train_workspace_size", "littlebit_train_forward",
-            "littlebit_train_backward",
+            "littlebit_train_backward", "littlebit_train_backward_saved",
             "littlebit_stack_workspace_size",
             "littlebit_stack_prepare", "littlebit_stack_forward", "littlebit_poll_error",
             "littlebit_selftest_wait_timeout", "littlebit_linear_forward_noalloc",
@@ -129,6 +129,8 @@ def lib(path: str | None = None):
                                                ctypes.c_float, ctypes.POINTER(lb_train_grad), vp,
                                                vp, sz, vp]
         L.littlebit_train_backward.restype = ctypes.c_int
+        L.littlebit_train_backward_saved.argtypes = L.littlebit_train_backward.argtypes
+        L.littlebit_train_backward_saved.restype = ctypes.c_int
         L.littlebit_stack_workspace_size.argtypes = [ctypes.POINTER(lb_linear), i32, i32]
         L.littlebit_stack_workspace_size.restype = sz
         L.littlebit_stack_prepare.argtypes = [ctypes.POINTER(lb_linear), i32, i32, vp, sz, vp]
@@ -424,8 +426,10 @@ def train_forward(L: TrainLinear, x: torch.Tensor, ws: torch.Tensor | None = Non
 
 
 def train_backward(L: TrainLinear, x: torch.Tensor, dy: torch.Tensor, k: float = 100.0,
-                   want_dx: bool = True, ws: torch.Tensor | None = None, stream=None):
-    """QAT backward with SmoothSign: (per-path dicts du, dv, dg, dl, dh; dX or None)."""
+                   want_dx: bool = True, ws: torch.Tensor | None = None, stream=None,
+                   saved: bool = False):
+    """QAT backward with SmoothSign: (per-path dicts du, dv, dg, dl, dh; dX or None).
+    saved: reuse what train_forward(L, x) left in ws (littlebit_train_backward_saved)."""
     x, dy = x.contiguous(), dy.contiguous()
     T = x.shape[0]
     grads = (lb_train_grad * len(L.paths))()
@@ -439,9 +443,9 @@ def train_backward(L: TrainLinear, x: torch.Tensor, dy: torch.Tensor, k: float =
             setattr(grads[p], key, ten.data_ptr())
     dx = torch.empty_like(x) if want_dx else None
     ws = ws if ws is not None else L.workspace(T, x.device)
-    _check(lib().littlebit_train_backward(ctypes.byref(L.c), x.data_ptr(), dy.data_ptr(), T,
-                                          float(k), grads, dx.data_ptr() if want_dx else None,
-                                          ws.data_ptr(), ws.numel(), _stream(stream)),
+    fn = lib().littlebit_train_backward_saved if saved else lib().littlebit_train_backward
+    _check(fn(ctypes.byref(L.c), x.data_ptr(), dy.data_ptr(), T, float(k), grads,
+              dx.data_ptr() if want_dx else None, ws.data_ptr(), ws.numel(), _stream(stream)),
            "littlebit_train_backward")
     return out, dx
 

@@ -159,8 +159,12 @@ def test_train_argument_validation(L):
     assert fwd(ref, FAKE, 16, FAKE, FAKE, 64, None) == lb.LB_ERR_WORKSPACE
     assert bwd(ref, FAKE, FAKE, 16, 0.0, g, None, FAKE, n, None) == lb.LB_ERR_INVALID_ARG  # k
     assert bwd(ref, FAKE, FAKE, 16, 100.0, None, None, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    sav = L.littlebit_train_backward_saved
+    assert sav(ref, FAKE, FAKE, 16, 0.0, g, None, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    assert sav(ref, FAKE, FAKE, 16, 100.0, g, None, FAKE, 64, None) == lb.LB_ERR_WORKSPACE
     g[0].dl = 0
     assert bwd(ref, FAKE, FAKE, 16, 100.0, g, None, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
+    assert sav(ref, FAKE, FAKE, 16, 100.0, g, None, FAKE, n, None) == lb.LB_ERR_INVALID_ARG
     c.n_paths = 3
     assert L.littlebit_train_workspace_size(ref, 16) == 0
 

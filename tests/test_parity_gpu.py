@@ -466,6 +466,33 @@ def test_train_forward_backward_vs_oracle(d_in, d_out, rs, T):
             assert e <= TOL_TF32, (p, key, e)
 
 
+def test_train_backward_saved_matches_and_checks_its_forward():
+    """The backward that reuses its forward's workspace state gives the same
+    bits as the one that recomputes it, also after another backward in
+    between; on a workspace whose last forward had another input it records
+    LB_ERR_PLAN."""
+    rng = inputs.rng_for(110)
+    d_in, d_out, rs, T = 512, 384, (32, 24), 96
+    layer = _train_case(rng, d_in, d_out, rs)
+    TL = lb.TrainLinear(layer, DEV)
+    x = torch.from_numpy(rng.standard_normal((T, d_in)).astype(np.float32)).to(DEV)
+    x2 = torch.from_numpy(rng.standard_normal((T, d_in)).astype(np.float32)).to(DEV)
+    dy = torch.from_numpy(rng.standard_normal((T, d_out)).astype(np.float32)).to(DEV)
+    ws = TL.workspace(T, DEV)
+    lb.train_forward(TL, x, ws=ws)
+    g_ref, dx_ref = lb.train_backward(TL, x, dy, ws=ws)
+    g_sav, dx_sav = lb.train_backward(TL, x, dy, ws=ws, saved=True)
+    torch.cuda.synchronize()
+    assert lb.poll_error(ws) == lb.LB_OK
+    assert torch.equal(dx_sav, dx_ref)
+    for p in range(len(rs)):
+        for key in ("du", "dv", "dg", "dl", "dh"):
+            assert torch.equal(g_sav[p][key], g_ref[p][key]), (p, key)
+    lb.train_forward(TL, x2, ws=ws)
+    lb.train_backward(TL, x, dy, ws=ws, saved=True)
+    assert lb.poll_error(ws) == lb.LB_ERR_PLAN
+
+
 # ------------------------------------------------------------------ stack
 
 
