@@ -147,6 +147,7 @@ constexpr int kProgBytes = 16384;  // per CTA, in the workspace and in shared me
 constexpr int kMaxItems = (kProgBytes - kStepBytes) / (int)sizeof(Item);
 constexpr int kMaxCtas = 255;      // the 8-bit contribution count of the exchange
 constexpr int kMaxSlots = 64;      // row units of a residual step
+constexpr unsigned kEarlyRead = 30;  // a poll's lanes read this many contributions early
 #ifndef LB_ROW_MIN_LNR
 #define LB_ROW_MIN_LNR 3
 #endif
@@ -544,14 +545,18 @@ __device__ __noinline__ bool run_poll_tables(int prog, int s, const unsigned lon
             if (need_ss) vs = ld_relaxed_u64(xbase + b.z);
         }
         if (!late || !__all_sync(0xffffffffu, !have || complete())) {
-            // lane 0 waits for the unit's last word (its stage-1 column block
+            // lane 0 waits on the unit's last word (its stage-1 column block
             // is sent after those of the unit's other words): one poller per
-            // warp keeps the L2 free for the contributions still arriving,
-            // and once it sees its word complete the whole unit usually is
+            // warp keeps the L2 free for the contributions still arriving.
+            // It lets the lanes read once all but kEarlyRead contributions
+            // are in, so their round trip overlaps the last ones' arrival
+            // (against waiting for all of them: 1.513 -> 1.501 ms per token
+            // with 152 contributions; 30 to 48 early measured alike).
             if (lane == 0 && a.z > 0) {
                 const unsigned long long s0 = globaltimer_ns();
                 const unsigned long long *gw = xbase + b.x + (min(a.z, 4 * a.y) - 1);
-                for (int spin = 0; !counted1(ld_relaxed_u64(gw), n_t); ++spin)
+                for (int spin = 0; (unsigned)(ld_relaxed_u64(gw) & 0xffull) + kEarlyRead < n_t;
+                     ++spin)
                     if ((spin & 15) == 15 && globaltimer_ns() - s0 > kWaitLimitNs) break;
             }
             __syncwarp();
