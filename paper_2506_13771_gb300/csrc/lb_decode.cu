@@ -11,7 +11,9 @@
 //     element (an exact two-word fixed-point sum whose low bits count the
 //     contributions, see send_fix2);
 //   * stage 2: every thread waits for the four elements of one l . t table
-//     and builds it; then 32 rows per warp over all words of a path;
+//     and builds it; then each warp sums one part (32 rows x up to 4 words
+//     of a path), times h, into its own shared slot, and the slots of a row
+//     are added in a fixed order into y;
 //   * the exchange words are double-buffered by a launch epoch kept in the
 //     workspace header: while a launch uses one buffer, every CTA clears its
 //     stripe of the other (the previous launch's), so no launch needs a

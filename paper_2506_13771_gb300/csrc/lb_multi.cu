@@ -11,7 +11,9 @@
 // two stages of different linears at once: the stage-1 group sends linear
 // m's partial t while the stage-2 group builds the outputs of an earlier
 // linear, so each exchange completes behind other linears' work and neither
-// stage waits for the other's barriers.  A producer warp bulk-copies
+// stage waits for the other's barriers (for a few linears, a phased schedule
+// instead runs every compute warp over stage 1 of all of them, then stage 2,
+// when its cost model says that is cheaper).  A producer warp bulk-copies
 // (cp.async.bulk) each linear's V slice, g slice, U rows and h into a ring of
 // kSlots shared-memory slots, a slot being refilled once its linear's stage 2
 // is done (so stage 1 runs at most kSlots linears ahead of stage 2).  The exchange words of all M linears are
