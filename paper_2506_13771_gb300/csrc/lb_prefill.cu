@@ -1206,6 +1206,366 @@ __device__ bool run_tiles_pair(const CUtensorMap *amap, const CUtensorMap *bmap,
 }
 
 
+// ------------------------------------------------ 2-SM tiles (cta_group::2)
+//
+// For long token runs the expanded path can also run on SM pairs: a cluster
+// of two CTAs computes a 256-token tile with tcgen05.mma.cta_group::2
+// (M = 256, N = 256).  Each CTA holds 128 rows of A and 128 of the 256 B
+// rows of each MMA in its own shared memory; the MMA, issued by one thread
+// of the even CTA (the leader), reads both CTAs' halves and leaves rows
+// 128 c .. 128 c + 127 of D in the TMEM of CTA c.  Per SM, the B operand's
+// shared-memory traffic (its TMA write and the MMA's read) halves against
+// the 1-SM tile of the same work.
+//   stage 1: 256 x 512 tiles (two N = 256 MMAs over each converted A stage,
+//            all 512 TMEM columns), 64-wide K-stages of 48 KB, four deep;
+//   stage 2: 256 x 256 tiles, two accumulators, 32 KB stages, six deep.
+// Every CTA's copy warp loads its own halves.  In stage 1 they complete on
+// its own `full` barrier, its conversion warps then arrive on the leader's
+// `ready` barrier, and the leader's MMA thread waits for that; in stage 2
+// both CTAs' copies complete on the leader's `full` barrier (the 2-SM form
+// of the TMA copy) and the MMA thread waits for it.  The leader's
+// tcgen05.commit arrives on the `empty` (or `acc_full`) barrier of both CTAs
+// at once (multicast).  The epilogue warps of both CTAs read their own TMEM
+// and arrive on the leader's `acc_empty`.  These kernels are cluster
+// launches of their own (expansion, stage 1, stage 2: three launches), not
+// cooperative, as they need no grid barrier.
+constexpr int kPairRows = 128;                  // rows of A and of each B half per CTA
+constexpr int PM = 2 * kPairRows;               // tokens per pair tile (MMA M)
+constexpr int PA_BYTES = kPairRows * BK * 2;    // 16 KB
+constexpr int PB_BYTES = kPairRows * BK * 2;    // 16 KB
+constexpr int PSB1 = PA_BYTES + 2 * PB_BYTES;   // stage 1: A, two B halves
+constexpr int PSB2 = PA_BYTES + PB_BYTES;       // stage 2: A, one B half
+constexpr int PNST1 = RING_BYTES / PSB1;        // 4
+constexpr int PNST2 = RING_BYTES / PSB2;        // 6
+static_assert(PNST1 >= 2 && PNST2 <= kMaxStages, "pair rings");
+
+__device__ __forceinline__ unsigned pair_rank() {
+    unsigned r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ unsigned pair_ctas() {
+    unsigned n;
+    asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(n));
+    return n;
+}
+// shared::cluster address of a barrier of this CTA in the CTA of rank `rank`
+__device__ __forceinline__ uint32_t bar_in(const uint64_t *b, unsigned rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(su32(b)), "r"(rank));
+    return r;
+}
+// Arrive on a barrier of the other CTA (or this one) of the pair.  Default
+// semantics (release at CTA scope): a release at cluster scope serialised
+// the arriving thread (about 1 us per arrival) and halved the pipeline's
+// rate.  What it orders is either TMA-written data, complete before the
+// arriving thread saw its own barrier, or the conversion warps' stores,
+// published to the tensor cores' async proxy by fence.proxy.async before
+// the arrival.
+__device__ __forceinline__ void mb_arrive_remote(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+// A wait with its own limit (the teardown's short waits).
+__device__ bool mb_wait_ns(uint64_t *b, unsigned parity, unsigned long long limit) {
+    if (mb_try(b, parity)) return true;
+    const unsigned long long t0 = globaltimer_ns();
+    while (!mb_try(b, parity))
+        if (globaltimer_ns() - t0 > limit) return false;
+    return true;
+}
+// TMA load into this CTA's shared memory that completes on a barrier of
+// the pair's leader (a shared::cluster address): the 2-SM form of the copy.
+__device__ __forceinline__ void tma_load_2d_lead(void *dst, const CUtensorMap *map, int x, int y,
+                                                 uint32_t lead_bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.cta_group::2.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];" ::"r"(su32(dst)),
+        "l"(map), "r"(x), "r"(y), "r"(lead_bar)
+        : "memory");
+}
+__device__ __forceinline__ void pair_sync() {
+    asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
+}
+__device__ __forceinline__ void mma_f16_pair(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                             uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(tmem_d),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+// arrive once on barrier b of both CTAs of the pair when the MMAs issued so
+// far have completed
+__device__ __forceinline__ void mma_commit_pair(uint64_t *bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
+        " [%0], %1;" ::"r"(su32(bar)),
+        "h"((uint16_t)3)
+        : "memory");
+}
+
+// One 2-SM tile phase; launched with clusters of two CTAs, grid even.
+// amap: x (stage 1, bf16) or z (stage 2), boxes of 64 x 128; bmap: the
+// expanded B operand (bv or bu), boxes of 64 x 128.  Stage 1's epilogue
+// warps expand the +-h operand of stage 2 first when expand_u is set.
+template <bool STAGE1>
+__global__ void __launch_bounds__(kThreads, 1)
+    k_pair(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
+           const __grid_constant__ PrefillParams P, int tiles_n, int n_tiles, int expand_u) {
+    __shared__ PhaseBars B;
+    __shared__ uint32_t s_tmem;
+    __shared__ int s_fail;
+    unsigned char *smem = reinterpret_cast<unsigned char *>(
+        (reinterpret_cast<uintptr_t>(p_smem) + 1023) & ~(uintptr_t)1023);
+    // A launch that formed no pairs (a profiler may replay it without
+    // clusters) must not touch another CTA or issue a 2-SM instruction.
+    if (pair_ctas() != 2) {
+        if (threadIdx.x == 0)
+            atomicCAS(P.ws_words + kErrWord, 0u, static_cast<unsigned>(LB_ERR_UNSUPPORTED));
+        return;
+    }
+    constexpr int SB = STAGE1 ? PSB1 : PSB2, NST = STAGE1 ? PNST1 : PNST2;
+    constexpr int kEpiWarps = STAGE1 ? 4 : kWorkWarps;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const unsigned rank = pair_rank();
+    const bool leader = rank == 0;
+    const int pair = blockIdx.x >> 1, n_pairs = gridDim.x >> 1;
+    const int KT = (STAGE1 ? P.L.d_in : P.N1) / BK;
+    volatile int *fail = &s_fail;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kMaxStages; ++s) {
+            mb_init(B.full + s, 1);
+            mb_init(B.ready + s, 2 * 4);  // stage 1: the conversion warps of both CTAs
+            mb_init(B.empty + s, 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            mb_init(B.acc_full + b, 1);
+            mb_init(B.acc_empty + b, 2 * kEpiWarps);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        s_fail = 0;
+    }
+    if (warp == 1) {
+        // one warp of each CTA of the pair, together
+        asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         su32(&s_tmem)),
+                     "r"(2 * BN)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    pair_sync();  // both CTAs' barriers exist before any arrival from the other
+    tc_fence_after();
+    const uint32_t tmem = s_tmem;
+    // Launched as a programmatic dependent of the previous kernel: the set-up
+    // above overlapped its tail; its results (the expanded operands, z) are
+    // read only after it has completed.  The next launch may start its own
+    // set-up on the SMs this one leaves free.
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
+    auto give_up = [&]() {
+        *fail = 1;
+        atomicCAS(P.ws_words + kErrWord, 0u, static_cast<unsigned>(LB_ERR_TIMEOUT));
+    };
+    // tile t -> token origin m0 of the pair tile, column origin n0
+    auto tile = [&](int t, int &m0, int &n0) {
+        m0 = (t / tiles_n) * PM;
+        n0 = (t % tiles_n) * (STAGE1 ? 2 * BN : BN);
+    };
+    auto advance = [&](int &s, unsigned &ph) {
+        if (++s == NST) {
+            s = 0;
+            ph ^= 1u;
+        }
+    };
+    int loads_issued = 0, mmas_issued = 0;
+
+    if (warp == 0) {
+        // ---------------- copy warp: this CTA's rows of A and of each B half
+        if (lane == 0) {
+            const uint32_t lead_full = bar_in(B.full, 0);
+            bool ok = true;
+            int s = 0;
+            unsigned ph = 0;
+            for (int t = pair; t < n_tiles && ok; t += n_pairs) {
+                int m0, n0;
+                tile(t, m0, n0);
+                const int ra = m0 + kPairRows * (int)rank, rb = n0 + kPairRows * (int)rank;
+                for (int i = 0; i < KT; ++i) {
+                    if (loads_issued >= NST && !mb_spin_role(B.empty + s, ph ^ 1u, fail)) {
+                        give_up();
+                        ok = false;
+                        break;
+                    }
+                    uint64_t *b = B.full + s;
+                    unsigned char *st = smem + s * SB;
+                    if (STAGE1) {
+                        // own barrier: the conversion warps wait for it
+                        mb_expect_tx(b, (unsigned)SB);
+                        tma_load_2d(st, &amap, i * BK, ra, b);
+                        tma_load_2d(st + PA_BYTES, &bmap, i * BK, rb, b);
+                        tma_load_2d(st + PA_BYTES + PB_BYTES, &bmap, i * BK, rb + BN, b);
+                    } else {
+                        // both CTAs' halves complete on the leader's barrier
+                        if (leader) mb_expect_tx(b, 2u * SB);
+                        const uint32_t lb = lead_full + 8u * (uint32_t)s;
+                        tma_load_2d_lead(st, &amap, i * BK, ra, lb);
+                        tma_load_2d_lead(st + PA_BYTES, &bmap, i * BK, rb, lb);
+                    }
+                    ++loads_issued;
+                    advance(s, ph);
+                }
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        if (leader && lane == 0) {
+            // ---------------- MMA thread (leader only)
+            const uint32_t idesc = instr_desc(PM, BN);
+            bool ok = true;
+            int ti = 0, s = 0;
+            unsigned ph = 0;
+            for (int t = pair; t < n_tiles && ok; t += n_pairs, ++ti) {
+                const int b = STAGE1 ? 0 : (ti & 1), uses = STAGE1 ? ti : (ti >> 1);
+                if (uses >= 1 &&
+                    !mb_spin_role(B.acc_empty + b, (unsigned)((uses - 1) & 1), fail)) {
+                    give_up();
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t d = tmem + (uint32_t)(b * BN);
+                for (int i = 0; i < KT; ++i) {
+                    if (!mb_spin_role(STAGE1 ? B.ready + s : B.full + s, ph, fail)) {
+                        give_up();
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t a0 = su32(smem + s * SB), b0 = a0 + PA_BYTES;
+#pragma unroll
+                    for (int k = 0; k < BK / 16; ++k) {
+                        const uint64_t ad = smem_desc(a0 + 32 * k);
+                        const uint32_t acc = (i > 0 || k > 0) ? 1u : 0u;
+                        mma_f16_pair(d, ad, smem_desc(b0 + 32 * k), idesc, acc);
+                        if (STAGE1)
+                            mma_f16_pair(d + BN, ad, smem_desc(b0 + PB_BYTES + 32 * k), idesc,
+                                         acc);
+                    }
+                    mma_commit_pair(B.empty + s);
+                    ++mmas_issued;
+                    advance(s, ph);
+                }
+                if (ok) mma_commit_pair(B.acc_full + b);
+            }
+        }
+        __syncwarp();
+    } else if (STAGE1 && warp < 6) {
+        // ---------------- conversion warps: bf16 -> fp16 of this CTA's A rows
+        const int tid = threadIdx.x - 64;
+        const uint32_t rdy = bar_in(B.ready, 0);
+        int s = 0;
+        unsigned ph = 0;
+        bool ok = true;
+        for (int t = pair; t < n_tiles && ok; t += n_pairs) {
+            for (int i = 0; i < KT; ++i, advance(s, ph)) {
+                const bool got = mb_wait_role(B.full + s, ph, fail);
+                if (!__all_sync(0xffffffffu, got)) {
+                    if (lane == 0) give_up();
+                    ok = false;
+                    break;
+                }
+                convert_a<128>(smem + s * SB, tid);
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) mb_arrive_remote(rdy + 8u * (uint32_t)s);
+            }
+        }
+    } else {
+        // ---------------- epilogue warps: TMEM lanes 32(w%4) .. +31 of this
+        //                  CTA (tile rows 128 rank + ...), stage 1 all 512
+        //                  columns, stage 2 one half of 256
+        const int wq = warp & 3;
+        const int half = STAGE1 ? 0 : (warp - 2) >> 2;
+        const int cb0 = STAGE1 ? 0 : half * (BN / 2), cb1 = STAGE1 ? 2 * BN : cb0 + BN / 2;
+        const uint32_t lane_base = tmem + ((uint32_t)(32 * wq) << 16);
+        const uint32_t aempty = bar_in(B.acc_empty, 0);
+        if (STAGE1 && expand_u)
+            expand_u_items(P, blockIdx.x * 128LL + (threadIdx.x - 192), gridDim.x * 128LL);
+        int ti = 0;
+        for (int t = pair; t < n_tiles; t += n_pairs, ++ti) {
+            int m0, n0;
+            tile(t, m0, n0);
+            const int b = STAGE1 ? 0 : (ti & 1), uses = STAGE1 ? ti : (ti >> 1);
+            const bool got = mb_wait_role(B.acc_full + b, (unsigned)(uses & 1), fail);
+            if (!__all_sync(0xffffffffu, got)) {
+                if (lane == 0) give_up();
+                break;
+            }
+            tc_fence_after();
+            const int row0 = m0 + kPairRows * (int)rank + 32 * wq;
+            for (int cb = cb0; cb < cb1; cb += 32) {
+                float v[32];
+                tmem_ld32(lane_base + (uint32_t)(b * BN + cb), v);
+                if (STAGE1) {
+                    if (row0 + lane < P.T) store_chunk<true>(P, v, row0 + lane, n0 + cb, 0, 1);
+                } else {
+                    float *stg =
+                        reinterpret_cast<float *>(smem + RING_BYTES + (warp - 2) * kStageBytes);
+                    store_y_coalesced(P, v, stg, row0, n0 + cb, lane);
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mb_arrive_remote(aempty + 8u * (uint32_t)b);
+        }
+    }
+
+    // Teardown.  After a failure, let this CTA's copies (and, in the leader,
+    // its MMAs) land.  Every CTA then waits for the arrivals of the MMAs
+    // that read its last stages (they come from the leader's commits; on a
+    // failure some never come, hence the short limit), so that nothing
+    // lands in a CTA that has left; both CTAs meet before the TMEM is freed.
+    if (__syncthreads_or(*fail)) {
+        if (threadIdx.x == 0) {
+            if (STAGE1 || leader) {
+                for (int i = loads_issued - NST; i < loads_issued; ++i)
+                    if (i >= 0) mb_wait(B.full + i % NST, (unsigned)((i / NST) & 1));
+            } else {
+                // stage 2's odd CTA: its copies complete on the leader's
+                // barriers, which it cannot wait on; a copy lands within
+                // microseconds of its issue
+                const unsigned long long t0 = globaltimer_ns();
+                while (globaltimer_ns() - t0 < 100000ull) __nanosleep(1000);
+            }
+        }
+        if (threadIdx.x == 32)
+            for (int i = mmas_issued - NST; i < mmas_issued; ++i)
+                if (i >= 0) mb_wait(B.empty + i % NST, (unsigned)((i / NST) & 1));
+    }
+    if (threadIdx.x == 0)
+        for (int i = loads_issued - NST; i < loads_issued; ++i)
+            if (i >= 0) mb_wait_ns(B.empty + i % NST, (unsigned)((i / NST) & 1), 200000ull);
+    tc_fence_before();
+    pair_sync();
+    tc_fence_after();
+    if (warp == 1)
+        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                     "r"(2 * BN)
+                     : "memory");
+}
+
+// The +-g V_sign (and +-h U_sign) expansion of the 2-SM path, a plain launch.
+__global__ void __launch_bounds__(kThreads) k_expand(const __grid_constant__ PrefillParams P,
+                                                     int flags) {
+    const long long gi = blockIdx.x * (long long)blockDim.x + threadIdx.x;
+    const long long gn = (long long)gridDim.x * blockDim.x;
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    if (flags & 1) expand_v_items(P, gi, gn);
+    if (flags & 2) expand_u_items(P, gi, gn);
+}
+
 // What one launch of k_fused does, in this order: expand V and / or U, stage
 // 1 (and the reduction of its K slices), stage 2.
 enum : int { kDoExpandV = 1, kDoExpandU = 2, kDoStage1 = 4, kDoStage2 = 8 };
@@ -1503,6 +1863,82 @@ void plan_stage2(const PrefillParams &P, FusedPlan &F) {
 }
 }  // namespace
 
+namespace {
+// The 2-SM path is the default for the column-pair shapes; LB_PREFILL_2SM=0
+// selects the 1-SM form (k_fused) instead, for comparison.
+bool pair2_enabled() {
+    const char *e = getenv("LB_PREFILL_2SM");
+    return !(e && e[0] == '0');
+}
+
+cudaError_t launch_pair_kernel(bool stage1, const CUtensorMap &amap, const CUtensorMap &bmap,
+                               const PrefillParams &P, int tiles_n, int n_tiles, int expand_u,
+                               int grid, cudaStream_t s) {
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kTilesSmem;
+    cfg.stream = s;
+    cudaLaunchAttribute at[2];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 2;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = 1;
+    at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 2;
+    return stage1 ? cudaLaunchKernelEx(&cfg, k_pair<true>, amap, bmap, P, tiles_n, n_tiles, expand_u)
+                  : cudaLaunchKernelEx(&cfg, k_pair<false>, amap, bmap, P, tiles_n, n_tiles,
+                                       expand_u);
+}
+
+// The expanded path on SM pairs, in stream order: the +-g V_sign expansion
+// (and +-h U_sign when stage 1 does not run), stage 1 in 256 x 512 tiles
+// (its epilogue warps expand +-h U_sign meanwhile when stage 2 follows),
+// stage 2 in 256 x 256 tiles.  x is read by stage 1, P.z is stage 1's output
+// and stage 2's input.
+cudaError_t launch_pair(const lb_linear &L, const uint16_t *x, int64_t T, const PrefillParams &P,
+                        bool stage1, bool stage2, cudaStream_t s) {
+    CUtensorMap xmap{}, bvmap{}, zmap{}, bumap{};
+    if (stage1 &&
+        (!make_map(&xmap, x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, T, L.d_in, kPairRows) ||
+         !make_map(&bvmap, P.bv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, P.N1, L.d_in, kPairRows)))
+        return cudaErrorInvalidValue;
+    if (stage2 &&
+        (!make_map(&zmap, P.z, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, T, P.N1, kPairRows) ||
+         !make_map(&bumap, P.bu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, L.d_out, P.N1, kPairRows)))
+        return cudaErrorInvalidValue;
+    static std::once_flag once;
+    static cudaError_t attr = cudaSuccess;
+    std::call_once(once, [] {
+        attr = cudaFuncSetAttribute(k_pair<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    kTilesSmem);
+        if (attr == cudaSuccess)
+            attr = cudaFuncSetAttribute(k_pair<false>,
+                                        cudaFuncAttributeMaxDynamicSharedMemorySize, kTilesSmem);
+    });
+    if (attr != cudaSuccess) return attr;
+    const int sms = device_sms() & ~1;
+    if (sms <= 0) return cudaErrorInvalidDevice;
+    k_expand<<<sms, kThreads, 0, s>>>(P, (stage1 ? 1 : 0) | (stage1 ? 0 : 2));
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const int tm = (int)((T + PM - 1) / PM);
+    if (stage1) {
+        const int tn1 = P.N1 / (2 * BN), n1 = tm * tn1;
+        e = launch_pair_kernel(true, xmap, bvmap, P, tn1, n1, stage2 ? 1 : 0,
+                               std::min(sms, 2 * n1), s);
+        if (e != cudaSuccess) return e;
+    }
+    if (stage2) {
+        const int tn2 = (P.d_out + BN - 1) / BN, n2 = tm * tn2;
+        e = launch_pair_kernel(false, zmap, bumap, P, tn2, n2, 0, std::min(sms, 2 * n2), s);
+    }
+    return e;
+}
+}  // namespace
+
 cudaError_t launch_prefill_latent(const lb_linear &L, const uint16_t *x, int64_t T, uint16_t *z16,
                                   float *z32, unsigned *ws_words, void *ws, cudaStream_t s) {
     if (!encoder()) return cudaErrorNotSupported;
@@ -1515,6 +1951,7 @@ cudaError_t launch_prefill_latent(const lb_linear &L, const uint16_t *x, int64_t
     if (P.expanded &&
         !make_map(&bvmap, P.bv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, P.N1, L.d_in, P.bn1, P.pair))
         return cudaErrorInvalidValue;
+    if (P.expanded && P.pair && pair2_enabled()) return launch_pair(L, x, T, P, true, false, s);
     cudaError_t e = set_smem_attributes();
     if (e != cudaSuccess) return e;
     if (P.expanded) {
@@ -1545,6 +1982,8 @@ cudaError_t launch_prefill_expand(const lb_linear &L, const uint16_t *z16, int64
     if (!make_map(&zmap, z16, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, T, P.N1)) return cudaErrorInvalidValue;
     if (P.expanded && !make_map(&bumap, P.bu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, L.d_out, P.N1, BN))
         return cudaErrorInvalidValue;
+    if (P.expanded && P.pair && pair2_enabled())
+        return launch_pair(L, nullptr, T, P, false, true, s);
     cudaError_t e = set_smem_attributes();
     if (e != cudaSuccess) return e;
     if (P.expanded) {
@@ -1558,6 +1997,7 @@ cudaError_t launch_prefill_expand(const lb_linear &L, const uint16_t *z16, int64
     k_prefill<false><<<g2, kThreads, smem_bytes<false>(), s>>>(zmap, P);
     return cudaGetLastError();
 }
+
 
 cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, void *y, int y_fp32,
                            unsigned *ws_words, void *ws, cudaStream_t s) {
@@ -1573,6 +2013,7 @@ cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, voi
     P.z = z16;
     P.y = y;
     P.y_fp32 = y_fp32;
+    if (P.pair && pair2_enabled()) return launch_pair(L, x, T, P, true, true, s);
     CUtensorMap xmap, bvmap, zmap, bumap;
     if (!make_map(&xmap, x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, T, L.d_in, BM, P.pair) ||
         !make_map(&bvmap, P.bv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, P.N1, L.d_in, P.bn1, P.pair) ||

@@ -198,10 +198,26 @@ PAIR = [
 
 
 @pytest.mark.parametrize("d_in,d_out,rs,T", PAIR)
-def test_prefill_column_pair_tiles(d_in, d_out, rs, T):
-    """Long token runs with N1 a multiple of 512 take stage 1 in 128 x 512
-    tiles (two 256-wide MMAs per converted x stage, 64-byte swizzle): sampled
-    rows of the forward and of both latent types against the oracle."""
+@pytest.mark.parametrize("two_sm", [True, False])
+def test_prefill_column_pair_tiles(d_in, d_out, rs, T, two_sm):
+    """Long token runs with N1 a multiple of 512 take stage 1 in column-pair
+    tiles: by default on SM pairs (tcgen05 cta_group::2, 256 x 512 tiles,
+    then stage 2 in 256 x 256 pair tiles, three launches), with
+    LB_PREFILL_2SM=0 in the one-launch 1-SM form (128 x 512 tiles, 64-byte
+    swizzle).  Sampled rows of the forward and of both latent types against
+    the oracle."""
+    old = os.environ.get("LB_PREFILL_2SM")
+    os.environ["LB_PREFILL_2SM"] = "1" if two_sm else "0"
+    try:
+        _column_pair_case(d_in, d_out, rs, T)
+    finally:
+        if old is None:
+            os.environ.pop("LB_PREFILL_2SM", None)
+        else:
+            os.environ["LB_PREFILL_2SM"] = old
+
+
+def _column_pair_case(d_in, d_out, rs, T):
     rng = inputs.rng_for(109, salt=d_in + T)
     L = inputs.make_linear(rng, d_in, d_out, list(rs), len(rs), 0.05)
     x = inputs.bf16_normal(rng, (T, d_in))
@@ -226,6 +242,15 @@ def test_prefill_column_pair_tiles(d_in, d_out, rs, T):
         assert np.all(np.isfinite(zg))
         e = rel(zg[rows], z_ref)
         assert e <= tol, e
+    # the expansion alone (stage 2 on its own) from seeded fp16 latents
+    z16 = rng.standard_normal((T, sum(rs))).astype(np.float16)
+    ye = torch.full((T, d_out), float("nan"), dtype=torch.float32, device=DEV)
+    lb.linear_expand(D, torch.from_numpy(z16).to(DEV), y=ye, ws=ws)
+    torch.cuda.synchronize()
+    yeg = ye.cpu().numpy().astype(np.float64)
+    assert np.all(np.isfinite(yeg))
+    e = rel(yeg[rows], oracle.expand(L, z16[rows].astype(np.float64)))
+    assert e <= 1e-4, e
     assert lb.poll_error(ws) == lb.LB_OK
 
 
