@@ -1556,8 +1556,11 @@ __global__ void __launch_bounds__(kThreads, 1)
                      : "memory");
 }
 
-// The +-g V_sign (and +-h U_sign) expansion of the 2-SM path, a plain launch.
-__global__ void __launch_bounds__(kThreads) k_expand(const __grid_constant__ PrefillParams P,
+// The +-g V_sign (and +-h U_sign) expansion of the 2-SM path, a plain launch
+// of kExpandPerSm CTAs per SM (its loads are latency-bound: more warps in
+// flight).
+constexpr int kExpandPerSm = 2;
+__global__ void __launch_bounds__(kThreads, kExpandPerSm) k_expand(const __grid_constant__ PrefillParams P,
                                                      int flags) {
     const long long gi = blockIdx.x * (long long)blockDim.x + threadIdx.x;
     const long long gn = (long long)gridDim.x * blockDim.x;
@@ -1921,7 +1924,7 @@ cudaError_t launch_pair(const lb_linear &L, const uint16_t *x, int64_t T, const 
     if (attr != cudaSuccess) return attr;
     const int sms = device_sms() & ~1;
     if (sms <= 0) return cudaErrorInvalidDevice;
-    k_expand<<<sms, kThreads, 0, s>>>(P, (stage1 ? 1 : 0) | (stage1 ? 0 : 2));
+    k_expand<<<kExpandPerSm * sms, kThreads, 0, s>>>(P, (stage1 ? 1 : 0) | (stage1 ? 0 : 2));
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const int tm = (int)((T + PM - 1) / PM);
