@@ -1436,13 +1436,8 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 tc_fence_after();
                 const uint32_t d = tmem + (uint32_t)(b * BN);
-                for (int i = 0; i < KT; ++i) {
-                    if (!mb_spin_role(STAGE1 ? B.ready + s : B.full + s, ph, fail)) {
-                        give_up();
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
+                // the MMAs of one K-stage into the accumulator
+                auto issue = [&](int i) {
                     const uint32_t a0 = su32(smem + s * SB), b0 = a0 + PA_BYTES;
 #pragma unroll
                     for (int k = 0; k < BK / 16; ++k) {
@@ -1456,6 +1451,45 @@ __global__ void __launch_bounds__(kThreads, 1)
                     mma_commit_pair(B.empty + s);
                     ++mmas_issued;
                     advance(s, ph);
+                };
+                // Stage 2 waits for two stages at once and issues them back to
+                // back: each wait of this thread costs the tensor pipe a gap
+                // whether or not the stage has landed (4096 x 4096 r512,
+                // T = 8192: 112.3 -> 109.5 us; groups of 4: 114.3).  Stage 1
+                // waits on its conversion warps, and grouping there delays
+                // the MMAs (groups of 2: 119.5 us); so does grouping the 1-SM
+                // kernel's stage 2 (133.8 -> 137.9 us).
+                constexpr int G = STAGE1 ? 1 : 2;
+                if (G > 1 && KT % G == 0) {
+                    for (int i = 0; i < KT; i += G) {
+                        int s2 = s;
+                        unsigned ph2 = ph;
+                        bool got = true;
+#pragma unroll
+                        for (int j = 0; j < G; ++j) {
+                            got = got && mb_spin_role(STAGE1 ? B.ready + s2 : B.full + s2, ph2,
+                                                      fail);
+                            advance(s2, ph2);
+                        }
+                        if (!got) {
+                            give_up();
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+#pragma unroll
+                        for (int j = 0; j < G; ++j) issue(i + j);
+                    }
+                } else {
+                    for (int i = 0; i < KT; ++i) {
+                        if (!mb_spin_role(STAGE1 ? B.ready + s : B.full + s, ph, fail)) {
+                            give_up();
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        issue(i);
+                    }
                 }
                 if (ok) mma_commit_pair(B.acc_full + b);
             }
