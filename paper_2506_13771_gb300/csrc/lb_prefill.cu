@@ -73,12 +73,11 @@ __host__ __device__ constexpr int smem_bytes() {
     return RING_BYTES + (STAGE1 ? STAGES * SRC_BYTES : SLAB_BYTES) + 1024;
 }
 static_assert(smem_bytes<true>() <= 232448 && smem_bytes<false>() <= 232448, "shared memory");
-// The persistent form: the A|B ring, then (stage 2) one 32 x 16 fp32 staging
-// tile per epilogue warp, rows padded to 20 floats so that each quarter-warp
-// float4 access hits distinct banks.
-constexpr int kStagePitch = 20;
+// The persistent form: the A|B ring, then (stage 2) one output staging tile
+// per epilogue warp: 32 rows x 128 bytes (64 bf16 or 32 fp32 columns) in the
+// 128-byte-swizzled layout of the y tensor map, which a TMA store writes out.
 constexpr int kMaxStages = 8;
-constexpr int kStageBytes = 32 * kStagePitch * 4;
+constexpr int kStageBytes = 32 * 128;
 constexpr int kTilesSmem = RING_BYTES + kWorkWarps * kStageBytes + 1024;
 static_assert(kTilesSmem <= 232448, "shared memory");
 
@@ -627,43 +626,71 @@ __global__ void __launch_bounds__(kThreads, 1)
                      : "memory");
 }
 
-// Stage 2 output of one warp's 32 x 32 accumulator chunk (thread = row, v =
-// its 32 columns starting at c0) written through shared memory so that each
-// store instruction covers whole row segments: per 16-column half, every
-// thread parks its row in stg (32 rows x kStagePitch floats), then in four
-// passes reads back four columns of row 8i + lane/4 and writes them (8 bytes
-// bf16 / 16 bytes fp32), four lanes per row, eight rows per pass.
-__device__ __forceinline__ void store_y_coalesced(const PrefillParams &P, const float (&v)[32],
-                                                  float *stg, int row0, int c0, int lane) {
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-        float4 *mine = reinterpret_cast<float4 *>(stg + lane * kStagePitch);
-#pragma unroll
-        for (int q = 0; q < 4; ++q)
-            mine[q] = make_float4(v[16 * h + 4 * q], v[16 * h + 4 * q + 1], v[16 * h + 4 * q + 2],
-                                  v[16 * h + 4 * q + 3]);
+// TMA store of a shared-memory tile (this CTA's) into the tensor map at
+// (x, y); out-of-range rows and columns are not written.
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, int x, int y, const void *src) {
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
+                     map),
+                 "r"(x), "r"(y), "r"(su32(src))
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() {
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+// until this thread's bulk stores have read their shared-memory sources
+__device__ __forceinline__ void bulk_wait_read0() {
+    asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+// until this thread's bulk stores are complete
+__device__ __forceinline__ void bulk_wait0() {
+    asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+
+// Stage 2 output of one warp: its 32 accumulator rows (thread = row) and
+// columns [c0, c1) of the tile at TMEM address taddr, written through the
+// warp's 4 KB staging tile by TMA stores of 32 rows x 128 bytes (64 bf16 or
+// 32 fp32 columns) at (col0 + c, row0).  The staging tile is 128-byte
+// swizzled (16-byte chunk q of row n at n * 128 + ((q ^ n % 8) << 4)), so
+// each warp-wide 16-byte store hits every bank four times, the minimum.
+// Lane 0 issues the stores and waits for the previous one to have read the
+// tile before the warp refills it; it must call bulk_wait0() before the CTA
+// ends.
+__device__ __forceinline__ void store_y_tma(const CUtensorMap *ymap, int y_fp32, uint32_t taddr,
+                                            int c0, int c1, int row0, int col0,
+                                            unsigned char *stg, int lane) {
+    const int G = y_fp32 ? 32 : 64;
+    for (int c = c0; c < c1; c += G) {
+        float v[32], w[32];
+        tmem_ld32(taddr + (uint32_t)c, v);
+        if (!y_fp32) tmem_ld32(taddr + (uint32_t)(c + 32), w);
+        if (lane == 0) bulk_wait_read0();
         __syncwarp();
-        const int j = lane & 3;
-        const int col = c0 + 16 * h + 4 * j;
+        unsigned char *rowp = stg + (lane >> 3) * 1024 + (lane & 7) * 128;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const int r = 8 * i + (lane >> 2);
-            const float4 f = *reinterpret_cast<const float4 *>(stg + r * kStagePitch + 4 * j);
-            const int row = row0 + r;
-            if (row >= P.T || col >= P.d_out) continue;  // d_out % 8 == 0: whole groups of 4
-            if (P.y_fp32) {
-                *reinterpret_cast<float4 *>(static_cast<float *>(P.y) + (size_t)row * P.d_out +
-                                            col) = f;
+        for (int q = 0; q < 8; ++q) {
+            uint4 u;
+            if (y_fp32) {
+                u = make_uint4(__float_as_uint(v[4 * q]), __float_as_uint(v[4 * q + 1]),
+                               __float_as_uint(v[4 * q + 2]), __float_as_uint(v[4 * q + 3]));
             } else {
-                const uint32_t w0 = (uint32_t)float_to_bf16_bits(f.x) |
-                                    ((uint32_t)float_to_bf16_bits(f.y) << 16);
-                const uint32_t w1 = (uint32_t)float_to_bf16_bits(f.z) |
-                                    ((uint32_t)float_to_bf16_bits(f.w) << 16);
-                *reinterpret_cast<uint2 *>(static_cast<uint16_t *>(P.y) + (size_t)row * P.d_out +
-                                           col) = make_uint2(w0, w1);
+                const float *f = q < 4 ? v + 8 * q : w + 8 * (q - 4);
+                u = make_uint4((uint32_t)float_to_bf16_bits(f[0]) |
+                                   ((uint32_t)float_to_bf16_bits(f[1]) << 16),
+                               (uint32_t)float_to_bf16_bits(f[2]) |
+                                   ((uint32_t)float_to_bf16_bits(f[3]) << 16),
+                               (uint32_t)float_to_bf16_bits(f[4]) |
+                                   ((uint32_t)float_to_bf16_bits(f[5]) << 16),
+                               (uint32_t)float_to_bf16_bits(f[6]) |
+                                   ((uint32_t)float_to_bf16_bits(f[7]) << 16));
             }
+            *reinterpret_cast<uint4 *>(rowp + ((q ^ (lane & 7)) << 4)) = u;
         }
+        fence_proxy_async_smem();
         __syncwarp();
+        if (lane == 0) {
+            tma_store_2d(ymap, col0 + c, row0, stg);
+            bulk_commit();
+        }
     }
 }
 
@@ -823,8 +850,9 @@ __device__ __forceinline__ void fence_proxy_async_global() {
 // (every copy and MMA it issued has landed by then).
 template <bool STAGE1>
 __device__ bool run_tiles(const CUtensorMap *amap, const CUtensorMap *bmap,
-                          const PrefillParams &P, int tiles_n, int nsplit, int n_tiles,
-                          PhaseBars &B, uint32_t tmem, unsigned char *smem, volatile int *fail,
+                          const CUtensorMap *ymap, const PrefillParams &P, int tiles_n,
+                          int nsplit, int n_tiles, PhaseBars &B, uint32_t tmem,
+                          unsigned char *smem, volatile int *fail,
                           bool expand_u_meanwhile = false) {
     // stage 1 streams x as bf16: warps 2..5 convert each A stage to fp16 in
     // place and warps 6..9 run the epilogue; stage 2 uses all eight for it
@@ -976,16 +1004,15 @@ __device__ bool run_tiles(const CUtensorMap *amap, const CUtensorMap *bmap,
             }
             tc_fence_after();
             const int row = m0 + 32 * wq + lane;
-            for (int cb = cb0; cb < cb1; cb += 32) {
-                float v[32];
-                tmem_ld32(lane_base + (uint32_t)(b * BN + cb), v);
-                if (STAGE1) {
+            if (STAGE1) {
+                for (int cb = cb0; cb < cb1; cb += 32) {
+                    float v[32];
+                    tmem_ld32(lane_base + (uint32_t)(b * BN + cb), v);
                     if (row < P.T) store_chunk<STAGE1>(P, v, row, n0 + cb, z, nsplit);
-                } else {
-                    float *stg = reinterpret_cast<float *>(smem + RING_BYTES +
-                                                           (warp - 2) * kStageBytes);
-                    store_y_coalesced(P, v, stg, m0 + 32 * wq, n0 + cb, lane);
                 }
+            } else {
+                store_y_tma(ymap, P.y_fp32, lane_base + (uint32_t)(b * BN), cb0, cb1, m0 + 32 * wq,
+                            n0, smem + RING_BYTES + (warp - 2) * kStageBytes, lane);
             }
             tc_fence_before();
             __syncwarp();
@@ -993,6 +1020,8 @@ __device__ bool run_tiles(const CUtensorMap *amap, const CUtensorMap *bmap,
                 asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(B.acc_empty + b))
                              : "memory");
         }
+        if (!STAGE1 && lane == 0) bulk_wait0();  // this warp's output stores
+        __syncwarp();
     }
     if (__syncthreads_or(*fail)) {
         // let every issued copy and MMA land before the CTA goes away
@@ -1311,7 +1340,8 @@ __device__ __forceinline__ void mma_commit_pair(uint64_t *bar) {
 template <bool STAGE1>
 __global__ void __launch_bounds__(kThreads, 1)
     k_pair(const __grid_constant__ CUtensorMap amap, const __grid_constant__ CUtensorMap bmap,
-           const __grid_constant__ PrefillParams P, int tiles_n, int n_tiles, int expand_u) {
+           const __grid_constant__ CUtensorMap ymap, const __grid_constant__ PrefillParams P,
+           int tiles_n, int n_tiles, int expand_u) {
     __shared__ PhaseBars B;
     __shared__ uint32_t s_tmem;
     __shared__ int s_fail;
@@ -1539,21 +1569,22 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tc_fence_after();
             const int row0 = m0 + kPairRows * (int)rank + 32 * wq;
-            for (int cb = cb0; cb < cb1; cb += 32) {
-                float v[32];
-                tmem_ld32(lane_base + (uint32_t)(b * BN + cb), v);
-                if (STAGE1) {
+            if (STAGE1) {
+                for (int cb = cb0; cb < cb1; cb += 32) {
+                    float v[32];
+                    tmem_ld32(lane_base + (uint32_t)(b * BN + cb), v);
                     if (row0 + lane < P.T) store_chunk<true>(P, v, row0 + lane, n0 + cb, 0, 1);
-                } else {
-                    float *stg =
-                        reinterpret_cast<float *>(smem + RING_BYTES + (warp - 2) * kStageBytes);
-                    store_y_coalesced(P, v, stg, row0, n0 + cb, lane);
                 }
+            } else {
+                store_y_tma(&ymap, P.y_fp32, lane_base + (uint32_t)(b * BN), cb0, cb1, row0, n0,
+                            smem + RING_BYTES + (warp - 2) * kStageBytes, lane);
             }
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mb_arrive_remote(aempty + 8u * (uint32_t)b);
         }
+        if (!STAGE1 && lane == 0) bulk_wait0();  // this warp's output stores
+        __syncwarp();
     }
 
     // Teardown.  After a failure, let this CTA's copies (and, in the leader,
@@ -1623,7 +1654,8 @@ struct FusedPlan {
 __global__ void __launch_bounds__(kThreads, 1)
     k_fused(const __grid_constant__ CUtensorMap xmap, const __grid_constant__ CUtensorMap bvmap,
             const __grid_constant__ CUtensorMap zmap, const __grid_constant__ CUtensorMap bumap,
-            const __grid_constant__ PrefillParams P, const __grid_constant__ FusedPlan F) {
+            const __grid_constant__ CUtensorMap ymap, const __grid_constant__ PrefillParams P,
+            const __grid_constant__ FusedPlan F) {
     __shared__ PhaseBars bars[2];
     __shared__ uint32_t s_tmem;
     __shared__ int s_fail;
@@ -1692,7 +1724,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (ok && (F.flags & kDoStage1)) {
         ok = P.pair ? run_tiles_pair(&xmap, &bvmap, P, F.tiles_n1, F.n_tiles1, bars[0], tmem,
                                      smem, fail, u_in_stage1)
-                    : run_tiles<true>(&xmap, &bvmap, P, F.tiles_n1, F.split, F.n_tiles1, bars[0],
+                    : run_tiles<true>(&xmap, &bvmap, nullptr, P, F.tiles_n1, F.split, F.n_tiles1, bars[0],
                                       tmem, smem, fail, u_in_stage1);
         if (ok && F.split > 1) {
             ok = grid_barrier(P.ws_words, n_ctas * ++nbar);
@@ -1704,7 +1736,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     }
     if (ok && (F.flags & kDoStage2))
-        ok = run_tiles<false>(&zmap, &bumap, P, F.tiles_n2, 1, F.n_tiles2, bars[1], tmem, smem,
+        ok = run_tiles<false>(&zmap, &bumap, &ymap, P, F.tiles_n2, 1, F.n_tiles2, bars[1], tmem, smem,
                               fail);
     if (ok && threadIdx.x == 0) {
         // every CTA counted here has passed its last barrier
@@ -1752,6 +1784,20 @@ bool make_map(CUtensorMap *m, const void *base, CUtensorMapDataType dt, int64_t 
                     CU_TENSOR_MAP_INTERLEAVE_NONE,
                     narrow ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_128B,
                     CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// The output map of stage 2's TMA stores: [T][d_out] bf16 or fp32, boxes of
+// 32 rows x 128 bytes (64 or 32 columns), 128-byte swizzle.
+bool make_ymap(CUtensorMap *m, void *y, int y_fp32, int64_t T, int64_t d_out) {
+    const int es = y_fp32 ? 4 : 2;
+    const cuuint64_t dims[2] = {(cuuint64_t)d_out, (cuuint64_t)T};
+    const cuuint64_t strides[1] = {(cuuint64_t)d_out * es};
+    const cuuint32_t box[2] = {(cuuint32_t)(128 / es), 32};
+    const cuuint32_t estr[2] = {1, 1};
+    return g_encode(m, y_fp32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16,
+                    2, y, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                    CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -1875,10 +1921,12 @@ namespace {
 // every CTA resident).  Maps of phases the plan skips are never read.
 cudaError_t launch_fused(const CUtensorMap &xmap, const CUtensorMap &bvmap,
                          const CUtensorMap &zmap, const CUtensorMap &bumap,
-                         const PrefillParams &P, const FusedPlan &F, cudaStream_t s) {
+                         const CUtensorMap &ymap, const PrefillParams &P, const FusedPlan &F,
+                         cudaStream_t s) {
     void *args[] = {const_cast<CUtensorMap *>(&xmap), const_cast<CUtensorMap *>(&bvmap),
                     const_cast<CUtensorMap *>(&zmap), const_cast<CUtensorMap *>(&bumap),
-                    const_cast<PrefillParams *>(&P), const_cast<FusedPlan *>(&F)};
+                    const_cast<CUtensorMap *>(&ymap), const_cast<PrefillParams *>(&P),
+                    const_cast<FusedPlan *>(&F)};
     const int sms = device_sms();
     if (sms <= 0) return cudaErrorInvalidDevice;
     return cudaLaunchCooperativeKernel((const void *)k_fused, dim3(sms), dim3(kThreads), args,
@@ -1909,8 +1957,8 @@ bool pair2_enabled() {
 }
 
 cudaError_t launch_pair_kernel(bool stage1, const CUtensorMap &amap, const CUtensorMap &bmap,
-                               const PrefillParams &P, int tiles_n, int n_tiles, int expand_u,
-                               int grid, cudaStream_t s) {
+                               const CUtensorMap &ymap, const PrefillParams &P, int tiles_n,
+                               int n_tiles, int expand_u, int grid, cudaStream_t s) {
     cudaLaunchConfig_t cfg{};
     cfg.gridDim = dim3((unsigned)grid);
     cfg.blockDim = dim3(kThreads);
@@ -1925,8 +1973,9 @@ cudaError_t launch_pair_kernel(bool stage1, const CUtensorMap &amap, const CUten
     at[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = at;
     cfg.numAttrs = 2;
-    return stage1 ? cudaLaunchKernelEx(&cfg, k_pair<true>, amap, bmap, P, tiles_n, n_tiles, expand_u)
-                  : cudaLaunchKernelEx(&cfg, k_pair<false>, amap, bmap, P, tiles_n, n_tiles,
+    return stage1 ? cudaLaunchKernelEx(&cfg, k_pair<true>, amap, bmap, ymap, P, tiles_n, n_tiles,
+                                       expand_u)
+                  : cudaLaunchKernelEx(&cfg, k_pair<false>, amap, bmap, ymap, P, tiles_n, n_tiles,
                                        expand_u);
 }
 
@@ -1937,14 +1986,15 @@ cudaError_t launch_pair_kernel(bool stage1, const CUtensorMap &amap, const CUten
 // and stage 2's input.
 cudaError_t launch_pair(const lb_linear &L, const uint16_t *x, int64_t T, const PrefillParams &P,
                         bool stage1, bool stage2, cudaStream_t s) {
-    CUtensorMap xmap{}, bvmap{}, zmap{}, bumap{};
+    CUtensorMap xmap{}, bvmap{}, zmap{}, bumap{}, ymap{};
     if (stage1 &&
         (!make_map(&xmap, x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, T, L.d_in, kPairRows) ||
          !make_map(&bvmap, P.bv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, P.N1, L.d_in, kPairRows)))
         return cudaErrorInvalidValue;
     if (stage2 &&
         (!make_map(&zmap, P.z, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, T, P.N1, kPairRows) ||
-         !make_map(&bumap, P.bu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, L.d_out, P.N1, kPairRows)))
+         !make_map(&bumap, P.bu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, L.d_out, P.N1, kPairRows) ||
+         !make_ymap(&ymap, P.y, P.y_fp32, T, L.d_out)))
         return cudaErrorInvalidValue;
     static std::once_flag once;
     static cudaError_t attr = cudaSuccess;
@@ -1964,13 +2014,13 @@ cudaError_t launch_pair(const lb_linear &L, const uint16_t *x, int64_t T, const 
     const int tm = (int)((T + PM - 1) / PM);
     if (stage1) {
         const int tn1 = P.N1 / (2 * BN), n1 = tm * tn1;
-        e = launch_pair_kernel(true, xmap, bvmap, P, tn1, n1, stage2 ? 1 : 0,
+        e = launch_pair_kernel(true, xmap, bvmap, ymap, P, tn1, n1, stage2 ? 1 : 0,
                                std::min(sms, 2 * n1), s);
         if (e != cudaSuccess) return e;
     }
     if (stage2) {
         const int tn2 = (P.d_out + BN - 1) / BN, n2 = tm * tn2;
-        e = launch_pair_kernel(false, zmap, bumap, P, tn2, n2, 0, std::min(sms, 2 * n2), s);
+        e = launch_pair_kernel(false, zmap, bumap, ymap, P, tn2, n2, 0, std::min(sms, 2 * n2), s);
     }
     return e;
 }
@@ -1995,7 +2045,7 @@ cudaError_t launch_prefill_latent(const lb_linear &L, const uint16_t *x, int64_t
         FusedPlan F{};
         F.flags = kDoExpandV | kDoStage1;
         plan_stage1(P, F);
-        return launch_fused(xmap, bvmap, none, none, P, F, s);
+        return launch_fused(xmap, bvmap, none, none, none, P, F, s);
     }
     const int tm = (int)((T + BM - 1) / BM), tn = (P.N1 + P.bn1 - 1) / P.bn1;
     const dim3 g1((unsigned)tm, (unsigned)tn, (unsigned)P.split);
@@ -2015,8 +2065,9 @@ cudaError_t launch_prefill_expand(const lb_linear &L, const uint16_t *z16, int64
     P.z = const_cast<uint16_t *>(z16);
     P.y = y;
     P.y_fp32 = y_fp32;
-    CUtensorMap zmap, bumap{}, none{};
+    CUtensorMap zmap, bumap{}, ymap{}, none{};
     if (!make_map(&zmap, z16, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, T, P.N1)) return cudaErrorInvalidValue;
+    if (P.expanded && !make_ymap(&ymap, y, y_fp32, T, L.d_out)) return cudaErrorInvalidValue;
     if (P.expanded && !make_map(&bumap, P.bu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, L.d_out, P.N1, BN))
         return cudaErrorInvalidValue;
     if (P.expanded && P.pair && pair2_enabled())
@@ -2027,7 +2078,7 @@ cudaError_t launch_prefill_expand(const lb_linear &L, const uint16_t *z16, int64
         FusedPlan F{};
         F.flags = kDoExpandU | kDoStage2;
         plan_stage2(P, F);
-        return launch_fused(none, none, zmap, bumap, P, F, s);
+        return launch_fused(none, none, zmap, bumap, ymap, P, F, s);
     }
     const int tm = (int)((T + BM - 1) / BM), tn = (L.d_out + BN - 1) / BN;
     const dim3 g2((unsigned)tm, (unsigned)tn);
@@ -2051,11 +2102,12 @@ cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, voi
     P.y = y;
     P.y_fp32 = y_fp32;
     if (P.pair && pair2_enabled()) return launch_pair(L, x, T, P, true, true, s);
-    CUtensorMap xmap, bvmap, zmap, bumap;
+    CUtensorMap xmap, bvmap, zmap, bumap, ymap;
     if (!make_map(&xmap, x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, T, L.d_in, BM, P.pair) ||
         !make_map(&bvmap, P.bv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, P.N1, L.d_in, P.bn1, P.pair) ||
         !make_map(&zmap, z16, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, T, P.N1) ||
-        !make_map(&bumap, P.bu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, L.d_out, P.N1, BN))
+        !make_map(&bumap, P.bu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, L.d_out, P.N1, BN) ||
+        !make_ymap(&ymap, y, y_fp32, T, L.d_out))
         return cudaErrorInvalidValue;
     cudaError_t e = set_smem_attributes();
     if (e != cudaSuccess) return e;
@@ -2063,7 +2115,7 @@ cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, voi
     F.flags = kDoExpandV | kDoExpandU | kDoStage1 | kDoStage2;
     plan_stage1(P, F);
     plan_stage2(P, F);
-    return launch_fused(xmap, bvmap, zmap, bumap, P, F, s);
+    return launch_fused(xmap, bvmap, zmap, bumap, ymap, P, F, s);
 }
 
 }  // namespace lb
