@@ -198,6 +198,17 @@ __device__ __forceinline__ void mma_f16(uint32_t tmem_d, uint64_t adesc, uint64_
         : "memory");
 }
 
+// The same with A (M rows x 16 K, two fp16 per 32-bit column, row m in lane
+// m) read from TMEM at a_taddr.
+__device__ __forceinline__ void mma_f16_ta(uint32_t tmem_d, uint32_t a_taddr, uint64_t bdesc,
+                                           uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tsetp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(tmem_d),
+        "r"(a_taddr), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
 __device__ __forceinline__ void mma_commit(uint64_t *bar) {
     asm volatile(
         "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
@@ -231,6 +242,21 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
         : "memory");
 #pragma unroll
     for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// 32 consecutive 32-bit columns of this thread's TMEM lane from r; the store
+// and its wait are one asm statement.
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,"
+        "%13,%14,%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};\n\t"
+        "tcgen05.wait::st.sync.aligned;" ::"r"(taddr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]),
+        "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]),
+        "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]),
+        "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]),
+        "r"(r[29]), "r"(r[30]), "r"(r[31])
+        : "memory");
 }
 
 // Byte offset of the 16-byte chunk c (0..7) of row n in a K-major tile with
@@ -864,6 +890,14 @@ __device__ bool run_tiles(const CUtensorMap *amap, const CUtensorMap *bmap,
     const int SB = A_BYTES + bn * BK * 2;
     const int nst = min(kMaxStages, RING_BYTES / SB);
     const uint32_t idesc = instr_desc(BM, bn);
+    // Stage 1 with tiles at most 128 wide: the two accumulators take TMEM
+    // columns [0, 256) and the conversion warps put each stage's fp16 A into
+    // a TMEM ring at columns 256 + 32 s (at most six stages of 32 columns),
+    // from which the MMAs read it: no fp16 A in shared memory, 64 instead of
+    // 96 KB of shared-memory traffic per K-stage at bn = 128.
+    const bool a_tm = STAGE1 && bn <= 128;
+    const int acc_stride = a_tm ? 128 : BN;
+    constexpr int kATmCol = 2 * 128;
     auto give_up = [&]() {
         *fail = 1;
         atomicCAS(P.ws_words + kErrWord, 0u, static_cast<unsigned>(LB_ERR_TIMEOUT));
@@ -931,7 +965,7 @@ __device__ bool run_tiles(const CUtensorMap *amap, const CUtensorMap *bmap,
                     break;
                 }
                 tc_fence_after();
-                const uint32_t d = tmem + (uint32_t)(b * BN);
+                const uint32_t d = tmem + (uint32_t)(b * acc_stride);
                 for (int i = 0; i < kc; ++i) {
                     // stage 1: the stage is ready once its A half is fp16
                     if (!mb_spin_role(STAGE1 ? B.ready + s : B.full + s, ph, fail)) {
@@ -941,10 +975,18 @@ __device__ bool run_tiles(const CUtensorMap *amap, const CUtensorMap *bmap,
                     }
                     tc_fence_after();
                     const uint32_t a0 = su32(smem + s * SB), b0 = su32(smem + s * SB + A_BYTES);
+                    if (a_tm) {
+                        const uint32_t at = tmem + (uint32_t)(kATmCol + 32 * s);
 #pragma unroll
-                    for (int k = 0; k < BK / 16; ++k)
-                        mma_f16(d, smem_desc(a0 + 32 * k), smem_desc(b0 + 32 * k), idesc,
-                                (i > 0 || k > 0) ? 1u : 0u);
+                        for (int k = 0; k < BK / 16; ++k)
+                            mma_f16_ta(d, at + 8 * k, smem_desc(b0 + 32 * k), idesc,
+                                       (i > 0 || k > 0) ? 1u : 0u);
+                    } else {
+#pragma unroll
+                        for (int k = 0; k < BK / 16; ++k)
+                            mma_f16(d, smem_desc(a0 + 32 * k), smem_desc(b0 + 32 * k), idesc,
+                                    (i > 0 || k > 0) ? 1u : 0u);
+                    }
                     mma_commit(B.empty + s);
                     ++mmas_issued;
                     advance(s, ph);
@@ -969,8 +1011,32 @@ __device__ bool run_tiles(const CUtensorMap *amap, const CUtensorMap *bmap,
                     ok = false;
                     break;
                 }
-                convert_a<128>(smem + s * SB, tid);
-                fence_proxy_async_smem();
+                if (a_tm) {
+                    // this lane's row n = 32 (w % 4) + lane of the 128-byte-
+                    // swizzled bf16 stage into its TMEM lane as fp16
+                    const int n = 32 * (warp & 3) + lane;
+                    const unsigned char *rowp = smem + s * SB + (n >> 3) * 1024 + (n & 7) * 128;
+                    uint32_t r[32];
+#pragma unroll
+                    for (int c = 0; c < 8; ++c) {
+                        const uint4 u =
+                            *reinterpret_cast<const uint4 *>(rowp + ((c ^ (n & 7)) << 4));
+                        const uint32_t w4[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const __half2 h = __floats2half2_rn(
+                                __uint_as_float(w4[e] << 16), __uint_as_float(w4[e] & 0xffff0000u));
+                            r[4 * c + e] = *reinterpret_cast<const uint32_t *>(&h);
+                        }
+                    }
+                    tmem_st32(tmem + ((uint32_t)(32 * (warp & 3)) << 16) +
+                                  (uint32_t)(kATmCol + 32 * s),
+                              r);
+                    tc_fence_before();
+                } else {
+                    convert_a<128>(smem + s * SB, tid);
+                    fence_proxy_async_smem();
+                }
                 __syncwarp();
                 if (lane == 0)
                     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(B.ready + s))
@@ -1007,7 +1073,7 @@ __device__ bool run_tiles(const CUtensorMap *amap, const CUtensorMap *bmap,
             if (STAGE1) {
                 for (int cb = cb0; cb < cb1; cb += 32) {
                     float v[32];
-                    tmem_ld32(lane_base + (uint32_t)(b * BN + cb), v);
+                    tmem_ld32(lane_base + (uint32_t)(b * acc_stride + cb), v);
                     if (row < P.T) store_chunk<STAGE1>(P, v, row, n0 + cb, z, nsplit);
                 }
             } else {

@@ -173,6 +173,9 @@ PREFILL = [
     (4096, 11008, (128, 128), 64), (64, 8, (64, 64), 65), (512, 1000, (512,), 17),
     # stage 1 split along d_in into K slices (long d_in, few token tiles)
     (11008, 4096, (128, 128), 48), (4096, 2048, (512, 512), 300), (2048, 64, (64, 64), 72),
+    # four token tiles or more with stage-1 tiles at most 128 wide: fp16 x in
+    # a TMEM ring (N1 = 128: six stages, N1 = 64: eight)
+    (1024, 520, (64, 64), 700), (2048, 1000, (64,), 900),
 ]
 
 
