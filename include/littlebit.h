@@ -123,7 +123,12 @@ size_t littlebit_workspace_size(const lb_linear *L, int64_t T);
  * and T * (r_0 + r_1) > 8192, with d_in and every r multiples of 64,
  * r <= 512 and d_out % 8 == 0 -> the tensor-core path (fp16 operands, see
  * its tolerance in the design notes); otherwise the two-launch CUDA-core
- * path. */
+ * path.  On the tensor-core path with T >= 385, r_0 + r_1 a multiple of 512
+ * and at least 96 stage-1 tiles of 128 x 512 (T >= 6144 at r_0 + r_1 =
+ * 1024), the forward runs on SM pairs (tcgen05 cta_group::2) as three
+ * launches in stream order; the environment variable LB_PREFILL_2SM=0, read
+ * at each call, selects the one-launch form on single SMs instead.  Results
+ * of the two forms agree to the path's tolerance, not bit for bit. */
 lb_status littlebit_linear_forward(const lb_linear *L, const uint16_t *x, int64_t T, void *y,
                                    int32_t y_dtype, void *ws, size_t ws_bytes,
                                    lb_stream_t stream);
