@@ -280,6 +280,7 @@ struct PrefillParams {
     LinDesc L;
     int T, N1, d_out;
     int bn1;           // stage-1 tile width: N1 if N1 <= 256, else 256
+    int bn2;           // k_prefill's stage-2 tile width: 256, 128 or 64 (enough tiles for the SMs)
     int off1;          // column offset of path 1 in the N1 concatenation (= r_0)
     uint16_t *z;       // stage 1 output / stage 2 input, fp16 [T][N1]
     float *z32;        // stage 1 output in fp32 instead of z (latent entry point), or null
@@ -468,14 +469,14 @@ __global__ void __launch_bounds__(kThreads, 1)
         (reinterpret_cast<uintptr_t>(p_smem) + 1023) & ~(uintptr_t)1023);
     constexpr int SB = A_BYTES + B_BYTES;
     unsigned char *slab = smem + RING_BYTES;
-    const int m0 = blockIdx.x * BM, n0 = blockIdx.y * BN;
+    const int bn = STAGE1 ? P.bn1 : P.bn2;
+    const int m0 = blockIdx.x * BM, n0 = blockIdx.y * (STAGE1 ? BN : bn);
     const int K = STAGE1 ? P.L.d_in : P.N1;
     // stage 1 may be split along K: slice z of split takes chunks [kbeg, kbeg + KC)
     const int KT = K / BK, nsplit = STAGE1 ? P.split : 1;
     const int kbeg = (int)((long long)blockIdx.z * KT / nsplit);
     const int KC = (int)((long long)(blockIdx.z + 1) * KT / nsplit) - kbeg;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int bn = STAGE1 ? P.bn1 : BN;
     volatile int *fail = &s_fail;
     if (ld_relaxed_gpu(P.ws_words + kErrWord) != 0u) return;
 
@@ -545,7 +546,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) {
             if (!STAGE1) {
                 // the tile's U rows and h of every path, once
-                const int nrows = min(BN, P.d_out - n0);
+                const int nrows = min(bn, P.d_out - n0);
                 for (int p = 0; p < P.L.n_paths; ++p) {
                     const int R = ((p ? P.L.r[1] : P.L.r[0]) + 31) >> 5;
                     mb_expect_only(&slab_bar, (unsigned)(nrows * R * 4 + nrows * 2));
@@ -742,7 +743,11 @@ struct ItemWalk {
 };
 
 // z = l . (sum over the K slices of the partial t), as fp16 (or fp32 into z32),
-// four columns per item; items i0, i0 + di, ... of [T][N1 / 4].
+// four columns per item; items i0, i0 + di, ... of [T][N1 / 4].  MANY: the
+// stand-alone reduction of k_prefill's up to 32 slices, which batches the
+// loads of several slices of one item; else (k_fused's few slices) the loads
+// of several items of one slice.
+template <bool MANY = false>
 __device__ __forceinline__ void reduce_z_items(const PrefillParams &P, long long i0, long long di) {
     constexpr int kB = kBatch / 2;
     ItemWalk w(i0, di, P.N1 / 4);
@@ -757,16 +762,43 @@ __device__ __forceinline__ void reduce_z_items(const PrefillParams &P, long long
             a[k] = make_float4(0.f, 0.f, 0.f, 0.f);
             w.step();
         }
-        for (int z = 0; z < P.split; ++z) {
+        if (MANY) {
+            // up to kZ slices' loads in flight at a time; the sums run in slice
+            // order (with up to 32 slices and few tokens the slices, not the
+            // items, are what a thread has many of)
+            constexpr int kZ = 8;
+            for (int z0 = 0; z0 < P.split; z0 += kZ) {
 #pragma unroll
-            for (int k = 0; k < kB; ++k) {
-                if (row[k] < P.T) {
-                    const float4 b = *reinterpret_cast<const float4 *>(
-                        P.zpart + z * slice + (size_t)row[k] * P.N1 + c[k]);
-                    a[k].x += b.x;
-                    a[k].y += b.y;
-                    a[k].z += b.z;
-                    a[k].w += b.w;
+                for (int k = 0; k < kB; ++k) {
+                    if (row[k] >= P.T) continue;
+                    const float *src = P.zpart + z0 * slice + (size_t)row[k] * P.N1 + c[k];
+                    float4 b[kZ];
+#pragma unroll
+                    for (int q = 0; q < kZ; ++q)
+                        if (z0 + q < P.split)
+                            b[q] = *reinterpret_cast<const float4 *>(src + q * slice);
+#pragma unroll
+                    for (int q = 0; q < kZ; ++q)
+                        if (z0 + q < P.split) {
+                            a[k].x += b[q].x;
+                            a[k].y += b[q].y;
+                            a[k].z += b[q].z;
+                            a[k].w += b[q].w;
+                        }
+                }
+            }
+        } else {
+            for (int z = 0; z < P.split; ++z) {
+#pragma unroll
+                for (int k = 0; k < kB; ++k) {
+                    if (row[k] < P.T) {
+                        const float4 b = *reinterpret_cast<const float4 *>(
+                            P.zpart + z * slice + (size_t)row[k] * P.N1 + c[k]);
+                        a[k].x += b.x;
+                        a[k].y += b.y;
+                        a[k].z += b.z;
+                        a[k].w += b.w;
+                    }
                 }
             }
         }
@@ -1106,8 +1138,8 @@ __device__ bool run_tiles(const CUtensorMap *amap, const CUtensorMap *bmap,
 // The split stage 1 of the non-persistent path (k_prefill) reduces its K
 // slices in a launch of its own.
 __global__ void k_reduce_z(const __grid_constant__ PrefillParams P) {
-    reduce_z_items(P, blockIdx.x * (long long)blockDim.x + threadIdx.x,
-                   (long long)gridDim.x * blockDim.x);
+    reduce_z_items<true>(P, blockIdx.x * (long long)blockDim.x + threadIdx.x,
+                         (long long)gridDim.x * blockDim.x);
 }
 
 // Column-pair form of stage 1 for long token runs (N1 a multiple of 512):
@@ -1968,6 +2000,14 @@ PrefillParams params_of(const lb_linear &L, int64_t T, unsigned *ws_words, void 
     P.N1 = (int)n1_of(L);
     P.off1 = L.path[0].r;
     P.bn1 = P.N1 <= BN ? P.N1 : BN;
+    // k_prefill's stage 2 (fewer than four token tiles): narrower tiles
+    // until there are enough for the SMs (the CTA unpacks its U rows for
+    // every K-stage, so with few tokens the row count per CTA sets the time)
+    {
+        const int64_t tm = (T + BM - 1) / BM;
+        P.bn2 = BN;
+        while (P.bn2 > 64 && tm * ((L.d_out + P.bn2 - 1) / P.bn2) < 148) P.bn2 /= 2;
+    }
     P.d_out = L.d_out;
     char *wsb = static_cast<char *>(ws);
     P.z = reinterpret_cast<uint16_t *>(wsb);
@@ -2146,7 +2186,7 @@ cudaError_t launch_prefill_expand(const lb_linear &L, const uint16_t *z16, int64
         plan_stage2(P, F);
         return launch_fused(none, none, zmap, bumap, ymap, P, F, s);
     }
-    const int tm = (int)((T + BM - 1) / BM), tn = (L.d_out + BN - 1) / BN;
+    const int tm = (int)((T + BM - 1) / BM), tn = (L.d_out + P.bn2 - 1) / P.bn2;
     const dim3 g2((unsigned)tm, (unsigned)tn);
     k_prefill<false><<<g2, kThreads, smem_bytes<false>(), s>>>(zmap, P);
     return cudaGetLastError();
