@@ -2000,13 +2000,14 @@ PrefillParams params_of(const lb_linear &L, int64_t T, unsigned *ws_words, void 
     P.N1 = (int)n1_of(L);
     P.off1 = L.path[0].r;
     P.bn1 = P.N1 <= BN ? P.N1 : BN;
-    // k_prefill's stage 2 (fewer than four token tiles): narrower tiles
-    // until there are enough for the SMs (the CTA unpacks its U rows for
-    // every K-stage, so with few tokens the row count per CTA sets the time)
+    // k_prefill's stage 2 (fewer than four token tiles): the narrowest of
+    // 256 / 128 / 64 columns whose tiles still fit one wave of 148 CTAs (one
+    // per SM: the CTA unpacks its U rows for every K-stage, so with few
+    // tokens the rows per CTA set the time, and a second wave doubles it)
     {
         const int64_t tm = (T + BM - 1) / BM;
         P.bn2 = BN;
-        while (P.bn2 > 64 && tm * ((L.d_out + P.bn2 - 1) / P.bn2) < 148) P.bn2 /= 2;
+        while (P.bn2 > 64 && tm * ((L.d_out + P.bn2 / 2 - 1) / (P.bn2 / 2)) <= 148) P.bn2 /= 2;
     }
     P.d_out = L.d_out;
     char *wsb = static_cast<char *>(ws);
