@@ -304,37 +304,47 @@ __device__ __forceinline__ void unpack_b(const PrefillParams &P, unsigned char *
                                          int kc, int n0, int bn, int tid) {
     const uint32_t *words = reinterpret_cast<const uint32_t *>(src);
     const uint16_t *gs = reinterpret_cast<const uint16_t *>(src + 2 * BN * 4);
-    // each item = one 16-byte chunk (8 K values) of one B row
-    for (int item = tid; item < bn * 8; item += kWork) {
-        const int n = item >> 3, c = item & 7;
-        uint4 v = make_uint4(0, 0, 0, 0);
+    // each item = four 16-byte chunks (32 K values, one sign word) of one B
+    // row: half hf of row n
+    for (int item = tid; item < bn * 2; item += kWork) {
+        const int n = item >> 1, hf = item & 1;
+        uint32_t word = 0u;
+        bool live = false;
+        uint4 mag[4];
         if (STAGE1) {
             const int col = n0 + n;
-            if (col < P.N1) {
+            live = col < P.N1;
+            if (live) {
                 const int p = col >= P.off1 ? 1 : 0;
-                // inputs 64kc + 8c .. +7: word row (c >> 2), bits 8(c&3) ..
-                const uint32_t word = words[(c >> 2) * BN + n];
-                const uint32_t bits = (word >> (8 * (c & 3))) & 0xffu;
-                const uint4 mag = *reinterpret_cast<const uint4 *>(gs + p * 64 + 8 * c);
-                v = signed8(bits, mag);
+                // inputs 64kc + 32hf .. +31: word row hf
+                word = words[hf * BN + n];
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                    mag[q] = *reinterpret_cast<const uint4 *>(gs + p * 64 + 8 * (4 * hf + q));
             }
         } else {
             const int o = n0 + n;
-            if (o < P.d_out) {
+            live = o < P.d_out;
+            if (live) {
                 const int k0 = 64 * kc;
                 const int p = k0 >= P.off1 ? 1 : 0, j0 = k0 - (p ? P.off1 : 0);
                 const int R = ((p ? P.L.r[1] : P.L.r[0]) + 31) >> 5;
                 const uint32_t *U = reinterpret_cast<const uint32_t *>(slab + p * SLAB_U_BYTES);
                 const uint16_t *h =
                     reinterpret_cast<const uint16_t *>(slab + 2 * SLAB_U_BYTES) + p * BN;
-                const uint32_t word = U[n * R + (j0 >> 5) + (c >> 2)];
-                const uint32_t bits = (word >> (8 * (c & 3))) & 0xffu;
+                word = U[n * R + (j0 >> 5) + hf];
                 const uint32_t hb = h[n];
                 const uint32_t hh = hb | (hb << 16);
-                v = signed8(bits, make_uint4(hh, hh, hh, hh));
+#pragma unroll
+                for (int q = 0; q < 4; ++q) mag[q] = make_uint4(hh, hh, hh, hh);
             }
         }
-        *reinterpret_cast<uint4 *>(Bs + sw128(n, c)) = v;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const uint4 v =
+                live ? signed8((word >> (8 * q)) & 0xffu, mag[q]) : make_uint4(0, 0, 0, 0);
+            *reinterpret_cast<uint4 *>(Bs + sw128(n, 4 * hf + q)) = v;
+        }
     }
 }
 
