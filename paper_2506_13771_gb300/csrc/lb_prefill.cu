@@ -20,7 +20,11 @@
 // stage 2 run as phases separated by grid barriers, and each tile phase is
 // persistent, with two TMEM accumulators so the epilogue of one tile overlaps
 // the K loop of the next.  z goes to the workspace as fp16 and comes back by
-// TMA.
+// TMA.  For long runs whose N1 is a multiple of 512 the expanded path runs
+// instead on SM pairs (k_pair, tcgen05 cta_group::2, three launches chained
+// by programmatic dependent launch; see the 2-SM section below).  Stage 2 of
+// both forms writes y by TMA tensor stores from a swizzled staging tile per
+// epilogue warp.
 //
 // One CTA computes a 128 x BN tile (BN <= 256 fp32 TMEM columns) with
 // specialised warps: warp 0 issues the TMA / bulk copies of each 64-element
@@ -2068,7 +2072,7 @@ void plan_stage2(const PrefillParams &P, FusedPlan &F) {
 namespace {
 // The 2-SM path is the default for the column-pair shapes; LB_PREFILL_2SM=0
 // selects the 1-SM form (k_fused) instead, for comparison.
-bool pair2_enabled() {
+bool two_sm_enabled() {
     const char *e = getenv("LB_PREFILL_2SM");
     return !(e && e[0] == '0');
 }
@@ -2155,7 +2159,7 @@ cudaError_t launch_prefill_latent(const lb_linear &L, const uint16_t *x, int64_t
     if (P.expanded &&
         !make_map(&bvmap, P.bv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, P.N1, L.d_in, P.bn1, P.pair))
         return cudaErrorInvalidValue;
-    if (P.expanded && P.pair && pair2_enabled()) return launch_pair(L, x, T, P, true, false, s);
+    if (P.expanded && P.pair && two_sm_enabled()) return launch_pair(L, x, T, P, true, false, s);
     cudaError_t e = set_smem_attributes();
     if (e != cudaSuccess) return e;
     if (P.expanded) {
@@ -2187,7 +2191,7 @@ cudaError_t launch_prefill_expand(const lb_linear &L, const uint16_t *z16, int64
     if (P.expanded && !make_ymap(&ymap, y, y_fp32, T, L.d_out)) return cudaErrorInvalidValue;
     if (P.expanded && !make_map(&bumap, P.bu, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, L.d_out, P.N1, BN))
         return cudaErrorInvalidValue;
-    if (P.expanded && P.pair && pair2_enabled())
+    if (P.expanded && P.pair && two_sm_enabled())
         return launch_pair(L, nullptr, T, P, false, true, s);
     cudaError_t e = set_smem_attributes();
     if (e != cudaSuccess) return e;
@@ -2218,7 +2222,7 @@ cudaError_t launch_prefill(const lb_linear &L, const uint16_t *x, int64_t T, voi
     P.z = z16;
     P.y = y;
     P.y_fp32 = y_fp32;
-    if (P.pair && pair2_enabled()) return launch_pair(L, x, T, P, true, true, s);
+    if (P.pair && two_sm_enabled()) return launch_pair(L, x, T, P, true, true, s);
     CUtensorMap xmap, bvmap, zmap, bumap, ymap;
     if (!make_map(&xmap, x, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, T, L.d_in, BM, P.pair) ||
         !make_map(&bvmap, P.bv, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, P.N1, L.d_in, P.bn1, P.pair) ||
