@@ -936,12 +936,14 @@ __device__ bool run_tiles(const CUtensorMap *amap, const CUtensorMap *bmap,
     const int SB = A_BYTES + bn * BK * 2;
     const int nst = min(kMaxStages, RING_BYTES / SB);
     const uint32_t idesc = instr_desc(BM, bn);
-    // Stage 1 with tiles at most 128 wide: the two accumulators take TMEM
+    // Stage 1 with tiles at most 128 wide, or with at most one tile per CTA
+    // (which then uses accumulator 0 only): the accumulators take TMEM
     // columns [0, 256) and the conversion warps put each stage's fp16 A into
-    // a TMEM ring at columns 256 + 32 s (at most six stages of 32 columns),
-    // from which the MMAs read it: no fp16 A in shared memory, 64 instead of
-    // 96 KB of shared-memory traffic per K-stage at bn = 128.
-    const bool a_tm = STAGE1 && bn <= 128;
+    // a TMEM ring at columns 256 + 32 s (at most eight stages of 32 columns),
+    // from which the MMAs read it: no fp16 A in shared memory (per K-stage 64
+    // instead of 96 KB of shared-memory traffic at bn = 128, 96 instead of
+    // 128 KB at bn = 256).
+    const bool a_tm = STAGE1 && (bn <= 128 || n_tiles <= (int)gridDim.x);
     const int acc_stride = a_tm ? 128 : BN;
     constexpr int kATmCol = 2 * 128;
     auto give_up = [&]() {
