@@ -910,8 +910,9 @@ __device__ __forceinline__ void fence_proxy_async_global() {
 }
 
 // One persistent tile phase over pre-expanded B operands (A and B both
-// stream by TMA; in stage 1 four warps convert each bf16 x stage to fp16 in
-// place): the CTAs walk the tiles t = blockIdx.x, blockIdx.x + gridDim.x, ...
+// stream by TMA; in stage 1 four warps convert each bf16 x stage to fp16, in
+// place or, where the accumulators leave room, into a TMEM ring that the
+// MMAs read A from): the CTAs walk the tiles t = blockIdx.x, blockIdx.x + gridDim.x, ...
 // (column tile fastest, then K slice, then token tile) and keep two fp32
 // accumulators in TMEM (2 x BN columns), so the epilogue warps read out tile
 // t while the MMA warp already accumulates tile t + gridDim.x and the copy
@@ -926,8 +927,9 @@ __device__ bool run_tiles(const CUtensorMap *amap, const CUtensorMap *bmap,
                           int nsplit, int n_tiles, PhaseBars &B, uint32_t tmem,
                           unsigned char *smem, volatile int *fail,
                           bool expand_u_meanwhile = false) {
-    // stage 1 streams x as bf16: warps 2..5 convert each A stage to fp16 in
-    // place and warps 6..9 run the epilogue; stage 2 uses all eight for it
+    // stage 1 streams x as bf16: warps 2..5 convert each A stage to fp16 (in
+    // place or into TMEM, below) and warps 6..9 run the epilogue; stage 2
+    // uses all eight for it
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int bn = STAGE1 ? P.bn1 : BN;
     const int KT = (STAGE1 ? P.L.d_in : P.N1) / BK;
