@@ -176,6 +176,9 @@ PREFILL = [
     # four token tiles or more with stage-1 tiles at most 128 wide: fp16 x in
     # a TMEM ring (N1 = 128: six stages, N1 = 64: eight)
     (1024, 520, (64, 64), 700), (2048, 1000, (64,), 900),
+    # outputs narrower than one TMA store box (64 bf16 / 32 fp32 columns): the
+    # stores clip the columns beyond d_out
+    (1024, 8, (64, 64), 400), (512, 24, (64,), 512), (256, 40, (128, 128), 700),
 ]
 
 
